@@ -1,0 +1,381 @@
+#!/usr/bin/env python
+"""Throughput of the split-VFL training step on GB300, through the C ABI.
+
+One "step" is one training mini-batch through the whole path: passive bottom
+forward, publish, active bottom forward, top forward, loss, backward, publish
+the cut-layer gradient, both bottoms' backward and the SGD updates (Algorithm 1
+with the delayed update of App. D).  Default workload: the credit-shaped
+preset (30000 rows, 12/11 features, 12/11-128-64 bottoms, top 128-64-1, BCE,
+batch 1024, staleness 2 on the seeded schedule, fp32).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config C]
+
+--impl reference times the CPU oracle (the only other implementation of the
+method) on the same workload.  With N > 1 (torchrun) every rank runs an
+independent replica of the workload on its own GPU (the path has no exchange
+between GPUs); value = all ranks' samples / the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "split-VFL training samples/sec at 1 GB300; % of roofline per kernel"
+FP32_ALU_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12   # SMs x FP32 lanes x FMA x max clock
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=150)
+    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2, help="workload preset 1..5 (default 2, credit-shaped)")
+    ap.add_argument("--rows", type=int, default=0, help="override the preset's row count")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    return ap.parse_args()
+
+
+def workload(args):
+    import synth
+    p = synth.preset(args.config)
+    if args.rows:
+        p = p.with_(n_rows=args.rows)
+    desc = (f"{p.name}: N={p.n_rows}, d_p/d_a={p.d_passive}/{p.d_active}, "
+            f"passive {'-'.join(map(str, (p.d_passive,) + p.passive))}, "
+            f"active {'-'.join(map(str, (p.d_active,) + p.active))}, "
+            f"top {'-'.join(map(str, (p.e_active + p.e_passive,) + p.top))} {p.loss.upper()}, "
+            f"B={p.batch}, S={p.staleness} ({p.schedule} schedule), {p.dtype}, "
+            f"{p.workers} worker stream(s) per party" + (f", DP C={p.dp_clip} sigma={p.dp_sigma}" if p.dp_clip else ""))
+    return p, desc
+
+
+def dtype_tag(p):
+    return "f32" if p.dtype == "fp32" else "bf16"
+
+
+def rows_of(p, k):
+    j = k % p.steps_per_epoch
+    r0 = j * p.batch
+    return r0, min(p.n_rows, r0 + p.batch)
+
+
+def samples(p, k0, n):
+    return sum(rows_of(p, k)[1] - rows_of(p, k)[0] for k in range(k0, k0 + n))
+
+
+def sched_kind(p):
+    return 0 if p.schedule == "sync" else 2
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.dev = device_index
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(device_index), f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.p.terminate()
+        self.p.wait()
+        self.f.flush()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.f.name) as fh:
+            for line in fh:
+                parts = [t.strip() for t in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(name)
+        os.unlink(self.f.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle timing (subprocess: its own threads, no CUDA)
+# --------------------------------------------------------------------------
+CPU_SNIPPET = r"""
+import sys, time, json, os
+sys.path.insert(0, {root!r})
+import numpy as np, synth, oracle
+p = synth.preset({cid})
+if {rows}: p = p.with_(n_rows={rows})
+n_steps = {n_steps}
+nb = p.steps_per_epoch
+last = min(n_steps, nb) * p.batch
+rows = min(p.n_rows, last)
+if n_steps > nb: rows = p.n_rows
+xp, xa, y = synth.make_dataset(p, rows=(0, rows))
+q = p.with_(n_rows=rows)
+params = synth.init_params(q)
+tp, ta = oracle.make_schedule(q.seed, q.staleness, {kind}, n_steps)
+o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
+t0 = time.perf_counter(); done = 0; nsamp = 0
+while done < n_steps:
+    r = o.step(int(tp[done]), int(ta[done]))
+    nsamp += r.rows[1] - r.rows[0]
+    done += 1
+    if time.perf_counter() - t0 > {budget}: break
+dt = time.perf_counter() - t0
+print(json.dumps(dict(steps=done, samples=nsamp, seconds=dt)))
+"""
+
+
+def run_oracle(p, args, n_steps, budget):
+    cores = os.cpu_count() or 1
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    code = CPU_SNIPPET.format(root=ROOT, cid=p.cid, rows=args.rows, n_steps=n_steps, kind=sched_kind(p),
+                              budget=budget)
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle timing failed: {r.stderr[-2000:]}")
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    res["cores"] = cores
+    return res
+
+
+def cpu_baseline(p, args):
+    res = run_oracle(p, args, args.warmup + args.steps, args.cpu_seconds)
+    return {"value": res["samples"] / res["seconds"], "unit": "samples/s", "cores": res["cores"], "kind": "oracle",
+            "sample": f"first {res['steps']} training steps ({res['samples']} samples) of the same workload, "
+                      f"float64 numpy oracle, {res['seconds']:.2f} s, BLAS threads={res['cores']}"}
+
+
+# --------------------------------------------------------------------------
+# the GPU arm
+# --------------------------------------------------------------------------
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "src": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
+
+
+def roofline(prof, pk):
+    """Dominant kernel class (largest summed time) against its bound."""
+    if not prof:
+        return None
+    name, (n, ms, flops, nbytes) = max(prof.items(), key=lambda kv: kv[1][1])
+    sec = ms / 1e3
+    tensor = name.startswith("gemm_tc")
+    if tensor:
+        peak = pk["bf16_tflops_sustained"]
+        ach = flops / sec / 1e12
+        compute_bound = True
+        bound, unit = "tensor", "TFLOP/s"
+    else:
+        alu_peak = FP32_ALU_PEAK_TFLOPS
+        balance = alu_peak * 1e12 / (pk["hbm_gbs"] * 1e9)
+        compute_bound = flops > 0 and flops / max(nbytes, 1.0) > balance
+        if compute_bound:
+            peak, ach, bound, unit = alu_peak, flops / sec / 1e12, "alu", "TFLOP/s"
+        else:
+            peak, ach, bound, unit = pk["hbm_gbs"], nbytes / sec / 1e9, "hbm", "GB/s"
+    return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
+            "traffic": None, "launches": n, "avg_us": ms / n * 1e3,
+            "peak_src": ("measured (sustained bf16)" if tensor else
+                         ("FP32 lanes x clock" if bound == "alu" else "measured HBM copy")) + f" [{pk['src']}]",
+            "all_classes_ms": {k: round(v[1], 4) for k, v in sorted(prof.items(), key=lambda kv: -kv[1][1])}}
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import paper_2510_12494_gb300 as vfl
+    from paper_2510_12494_gb300 import build
+    import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    build.build()
+
+    p, desc = workload(args)
+    cpu = None
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        cpu = cpu_baseline(p, args)          # before the GPU work: the oracle runs on idle host cores
+
+    xp, xa, y = synth.make_dataset(p)
+    params = synth.init_params(p)
+    W, K = args.warmup, args.steps
+    total = W + 3 * K
+    tp, ta = vfl.make_schedule(p.seed, p.staleness, sched_kind(p), total)
+    ctx = vfl.Context(p, p.n_rows)
+    ctx.load_data(xp, xa, y)
+    ctx.set_params(params)
+    main = torch.cuda.Stream()
+    flush = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")   # > 129 MB L2
+    nb = p.steps_per_epoch
+
+    def timed_block(k0, n, profile=False):
+        """Time steps [k0, k0+n) in iterations of one epoch each; L2 flushed before each."""
+        total_ms = 0.0
+        k = k0
+        if profile:
+            ctx.profile(True)
+        while k < k0 + n:
+            m = min(nb, k0 + n - k)
+            with torch.cuda.stream(main):
+                flush.zero_()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(main)
+            for s in ctx.streams:
+                s.wait_event(e0)
+            ctx.train_steps(k, m, tp, ta)
+            for s in ctx.streams:
+                ev = torch.cuda.Event()
+                ev.record(s)
+                main.wait_event(ev)
+            e1.record(main)
+            main.synchronize()
+            total_ms += e0.elapsed_time(e1)
+            k += m
+        prof = None
+        if profile:
+            ctx.profile(False)
+            prof = ctx.profile_summary()
+        return total_ms, prof
+
+    # warm-up
+    ctx.train_steps(0, W, tp, ta)
+    ctx.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks = Clocks(local)
+    l0 = ctx.launches
+    ms, _ = timed_block(W, K)
+    launches = ctx.launches - l0
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    n_samp = samples(p, W, K) * world
+    value = n_samp / (ms / 1e3)
+
+    # per-kernel timing: the same workload again, every launch bracketed by CUDA events
+    _, prof = timed_block(W + K, K, profile=True)
+    roof = roofline(prof, peaks())
+
+    # end to end through the public API with host buffers: every step stages
+    # its rows from pinned host memory and reads its loss back
+    e2e = None
+    if not args.skip_e2e:
+        pin_xp = torch.from_numpy(xp).pin_memory()
+        pin_xa = torch.from_numpy(xa).pin_memory()
+        pin_y = torch.from_numpy(y).pin_memory()
+        loss_host = torch.zeros(K, dtype=torch.float32).pin_memory()
+        k0 = W + 2 * K
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        k = k0
+        while k < k0 + K:
+            m = min(nb, k0 + K - k)
+            for kk in range(k, k + m):
+                r0, r1 = rows_of(p, kk)
+                ctx.stage_rows(kk % p.workers, r0, pin_xp[r0:r1], pin_xa[r0:r1], pin_y[r0:r1])
+            ctx.train_steps(k, m, tp, ta)
+            for kk in range(k, k + m):
+                ctx.fetch_loss(kk, loss_host.data_ptr() + 4 * (kk - k0))
+            k += m
+        ctx.synchronize()
+        dt = time.perf_counter() - t0
+        assert np.isfinite(loss_host.numpy()).all()
+        h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
+        e2e = {"value": samples(p, k0, K) * world / dt, "unit": "samples/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": 4}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "samples/s", "n_gpus": world, "steps": K, "warmup": W,
+            "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": dtype_tag(p), "data": "synthetic (seeded stand-in for the paper's tabular data)",
+            "config": {"workload": desc, "l2": "flushed (256 MiB write) before each timed iteration of one epoch",
+                       "parallelism": f"replicas x{world}" if world > 1 else "1 GPU, 2 parties on separate streams"},
+            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roof, "cpu_baseline": cpu,
+        }
+        print(json.dumps(line))
+    ctx.close()
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    p, desc = workload(args)
+    budget = 60.0
+    t0 = time.perf_counter()
+    # warm-up steps, then the timed steps, each a bounded sample of the workload
+    run_oracle(p, args, max(args.warmup, 1), 20.0)
+    res = run_oracle(p, args, args.steps, budget)
+    value = res["samples"] / res["seconds"]
+    cpu = {"value": value, "unit": "samples/s", "cores": res["cores"], "kind": "oracle",
+           "sample": f"first {res['steps']} of {args.steps} training steps ({res['samples']} samples), "
+                     f"float64 numpy oracle, {res['seconds']:.2f} s"}
+    line = {"metric": METRIC, "value": value, "unit": "samples/s", "n_gpus": world, "steps": res["steps"],
+            "warmup": args.warmup, "ms_per_step": res["seconds"] / max(res["steps"], 1) * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded stand-in for the paper's tabular data)", "impl": "reference",
+            "config": {"workload": desc, "parallelism": "CPU oracle, host cores"},
+            "cpu_baseline": cpu, "e2e": {"value": value, "unit": "samples/s", "h2d_bytes_per_step": 0,
+                                         "d2h_bytes_per_step": 0},
+            "wall_s": time.perf_counter() - t0}
+    print(json.dumps(line))
+
+
+if __name__ == "__main__":
+    a = parse()
+    if a.impl == "reference":
+        run_reference(a)
+    else:
+        run_ours(a)

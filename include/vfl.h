@@ -1,0 +1,251 @@
+/*
+ * vfl.h -- C ABI of the GB300 split-VFL training step (PubSub-VFL, arxiv 2510.12494).
+ *
+ * The library runs the two-party split-learning training step of the paper on
+ * one GPU: the passive party's bottom MLP forward publishes its embedding into a
+ * device-side channel, the active party runs its bottom MLP, the top MLP on
+ * [z^a | z^p], the loss and the backward pass, publishes the embedding gradient
+ * back, and both parties apply SGD (paper Sec. 3, Eq. 1-2; Algorithm 1).  The
+ * weight versions each step consumes come from a staleness schedule (the
+ * delayed update of App. D, Assumption 4).
+ *
+ * Conventions shared by every entry point:
+ *  - Every function returns a vfl_status and never throws.  On failure the
+ *    context keeps a message readable through vfl_last_error().
+ *  - Matrices are row-major.  A Linear layer with `in` inputs and `out`
+ *    outputs has W [out, in] and b [out], and computes Y = X W^T + b.
+ *  - Party ids: 0 = passive bottom f_p (theta_2), 1 = active bottom f_a,
+ *    2 = top model g (1 and 2 together are theta_1).
+ *  - "Host pointer" arguments are read or written before the call returns
+ *    (except vfl_stage_rows, which is asynchronous); the caller keeps ownership.
+ *  - Device memory comes from the caller: vfl_workspace_bytes() says how much,
+ *    vfl_create() carves every device buffer out of that one allocation.
+ *  - Work is enqueued on caller-provided CUDA streams (vfl_set_streams);
+ *    without them the library uses the legacy default stream for every worker.
+ *  - After VFL_E_CUDA the context is unusable except for vfl_destroy().
+ */
+#ifndef VFL_H
+#define VFL_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t vfl_status;
+
+#define VFL_OK 0
+#define VFL_E_INVAL 1     /* bad argument (shape, range, null pointer)                  */
+#define VFL_E_OOM 2       /* workspace smaller than vfl_workspace_bytes()               */
+#define VFL_E_CUDA 3      /* a CUDA call failed; the context is now unusable            */
+#define VFL_E_STATE 4     /* call out of order (step ordering / staleness contract)    */
+#define VFL_E_VERSION 5   /* a subscriber found a channel header for another step      */
+#define VFL_E_TIMEOUT 6   /* a bounded device-side wait gave up                         */
+
+#define VFL_MAX_LAYERS 8
+
+#define VFL_LOSS_BCE 0    /* binary cross-entropy on one logit (Eq. 1)                  */
+#define VFL_LOSS_CE 1     /* softmax cross-entropy on n_out >= 2 logits                */
+
+#define VFL_FP32 0        /* fp32 storage and arithmetic                               */
+#define VFL_BF16 1        /* bf16 weights copies / activations, fp32 accumulate+master */
+
+#define VFL_SCHED_SYNC 0  /* tau = 0                                                    */
+#define VFL_SCHED_MAX 1   /* tau(k) = min(k, S)                                         */
+#define VFL_SCHED_SEEDED 2
+
+/* what vfl_tap() reads */
+#define VFL_TAP_EMB 0     /* published embedding z^p of step k, [B_k, e_p]              */
+#define VFL_TAP_GRAD 1    /* published gradient dLoss/dz^p of step k, [B_k, e_p]        */
+#define VFL_TAP_LOGITS 2  /* logits of the last active step run on k's worker, [B_k, n_out] */
+#define VFL_TAP_ZA 3      /* active embedding z^a of that step, [B_k, e_a]              */
+#define VFL_TAP_DZA 4     /* dLoss/dz^a of that step, [B_k, e_a]                        */
+
+typedef struct vfl_config {
+    int32_t d_passive;                      /* passive feature count d_p                 */
+    int32_t d_active;                       /* active feature count d_a                  */
+    int32_t n_passive, n_active, n_top;     /* Linear layers in f_p, f_a, g (1..8)       */
+    int32_t passive_out[VFL_MAX_LAYERS];    /* output width of each f_p layer            */
+    int32_t active_out[VFL_MAX_LAYERS];     /* output width of each f_a layer            */
+    int32_t top_out[VFL_MAX_LAYERS];        /* output width of each g layer; last = n_out */
+    int32_t loss;                           /* VFL_LOSS_BCE (n_out == 1) | VFL_LOSS_CE   */
+    int32_t dtype;                          /* VFL_FP32 | VFL_BF16                       */
+    int32_t batch;                          /* rows per step B (the last batch may be shorter) */
+    float lr;                               /* SGD step size eta (Eq. 2)                 */
+    int32_t staleness;                      /* bound S on tau; channels hold S+1 slots   */
+    int32_t workers;                        /* worker streams per party (1..16)          */
+    float dp_clip;                          /* > 0 enables DP on the published gradient  */
+    float dp_sigma;                         /* noise multiplier; noise std = sigma * clip */
+    uint64_t dp_seed;                       /* Philox key of the DP noise                */
+} vfl_config;
+
+typedef struct vfl_ctx vfl_ctx;
+
+/* Bytes of device workspace vfl_create() needs for `cfg` and a dataset of n_rows rows. */
+vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* bytes);
+
+/*
+ * Create a context on the current CUDA device.  `workspace` is a device pointer
+ * (256-byte aligned) of at least vfl_workspace_bytes() bytes; it stays owned by
+ * the caller and must outlive the context.  Parameters start at zero: set them
+ * with vfl_set_params() before training.
+ */
+vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, uint64_t workspace_bytes,
+                      vfl_ctx** out);
+vfl_status vfl_destroy(vfl_ctx* ctx);
+
+/*
+ * Borrow 2*workers CUDA streams (cudaStream_t passed as void*): entries
+ * [0, workers) run the passive party's work, [workers, 2*workers) the active
+ * party's.  Steps go to worker k mod workers.  The streams must outlive the context.
+ */
+vfl_status vfl_set_streams(vfl_ctx* ctx, int32_t n, void* const* streams);
+
+/*
+ * Copy the whole dataset from host memory: x_passive [n_rows, d_p] and
+ * x_active [n_rows, d_a] fp32, y [n_rows] int32 (BCE: 0/1, CE: class id in
+ * [0, n_out)).  Synchronous.  bf16 contexts round the features to bf16 here.
+ */
+vfl_status vfl_load_data(vfl_ctx* ctx, const float* x_passive, const float* x_active, const int32_t* y);
+
+/*
+ * Asynchronously copy rows [row0, row0+n) of the dataset from host memory
+ * (pinned for true asynchrony) into the device copy: the passive rows on the
+ * passive stream of worker `worker`, the active rows and labels on the active
+ * one.  The host buffers hold only those n rows and must stay valid until the
+ * streams pass this point.  Work enqueued afterwards on the same workers sees
+ * the new rows.
+ */
+vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n, const float* x_passive,
+                          const float* x_active, const int32_t* y);
+
+/*
+ * Set / read the fp32 master parameters of one layer: W [out, in], b [out]
+ * (host pointers).  vfl_set_params resets every stored weight version of the
+ * layer to the new values and is only valid before the first step.
+ * vfl_get_params synchronizes the context first.
+ */
+vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const float* W, const float* b);
+vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, float* b);
+
+/*
+ * Gradient dLoss/dW [out, in] and dLoss/db [out] of one layer from the most
+ * recent step of that party on worker `worker` (before the SGD update used
+ * it).  Synchronizes the context.
+ */
+vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t worker, float* dW, float* db);
+
+/*
+ * Checkpoint / restore.  Valid only while no step is in flight (every enqueued
+ * step has run all three phases).
+ *  - vfl_step_cursor: number of finished steps k = the current weight version.
+ *  - vfl_get_version: the stored compute copy of weight version v
+ *    (max(0, k-S) <= v <= k) as fp32 (exact: bf16 copies widen losslessly).
+ *  - vfl_set_cursor: make k the next step (for resuming a checkpoint); the
+ *    caller then stores versions max(0, k-S) .. k with vfl_set_version.
+ *  - vfl_set_version: store version v of one layer (rounded to the compute
+ *    dtype); for v == k it also sets the fp32 master that SGD updates.
+ * The fp32 master of version k is read with vfl_get_params.  A context
+ * restored this way continues bit-identically to the one checkpointed.
+ */
+vfl_status vfl_step_cursor(vfl_ctx* ctx, int64_t* k);
+vfl_status vfl_get_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, float* W, float* b);
+vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k);
+vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, const float* W, const float* b);
+
+/*
+ * Staleness schedule (host only, pure).  tau_p[k], tau_a[k] for k < n_steps:
+ * SYNC 0; MAX min(k, S); SEEDED tau(0) = 0, tau(k) = min(k, S, tau(k-1)+1,
+ * u_k mod (S+1)) with u_k word 0 of Philox4x32-10(key = (seed lo, seed hi),
+ * counter = (k lo, k hi, party, 0x5343)).  Paper: App. D Assumption 4 bounds the
+ * delay; the seeded draw is this library's schedule.
+ */
+vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_steps, int32_t* tau_p,
+                             int32_t* tau_a);
+
+/*
+ * Publisher phase of step k (Algorithm 1, passive): z^p = f_p(x^p) with the
+ * passive weights of version k - tau_p, then publish z^p to the embedding
+ * channel slot k mod (S+1) with header {k, batch, version}.  Steps must be
+ * published in order (k = number of earlier calls); the version must still be
+ * stored: 0 <= tau_p <= min(k, S) and k - tau_p >= (passive updates so far) - S.
+ */
+vfl_status vfl_passive_forward(vfl_ctx* ctx, int64_t k, int32_t tau_p);
+
+/*
+ * Subscriber phase of step k (Algorithm 1, active): fetch z^p (header check,
+ * VFL_E_VERSION on mismatch), z^a = f_a(x^a) and y_hat = g(z^a, z^p) with the
+ * active+top weights of version k - tau_a, loss, backward, optional DP on the
+ * gradient, publish dLoss/dz^p to the gradient channel, then the SGD update of
+ * f_a and g (Eq. 2, applied in step order).  Requires the embedding of step k
+ * to have been enqueued.
+ */
+vfl_status vfl_active_step(vfl_ctx* ctx, int64_t k, int32_t tau_a);
+
+/*
+ * Backward phase of step k (Algorithm 1, passive): fetch dLoss/dz^p (header
+ * check), backward through the passive version used by the forward of step k
+ * with its saved activations, SGD update of f_p in step order.
+ */
+vfl_status vfl_passive_backward(vfl_ctx* ctx, int64_t k);
+
+/*
+ * Enqueue steps [k0, k0 + n_steps) as one dependency graph across the worker
+ * streams: each publisher phase runs as soon as its weight version exists, so
+ * the parties overlap as far as tau allows.  tau_p / tau_a are host arrays
+ * indexed by absolute step (length >= k0 + n_steps).  Same contract as the three
+ * per-phase calls.
+ */
+vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
+                           const int32_t* tau_a);
+
+/* Wait for all enqueued work; returns VFL_E_VERSION / VFL_E_TIMEOUT recorded by kernels. */
+vfl_status vfl_synchronize(vfl_ctx* ctx);
+
+/* Mean loss of steps [k0, k0+n) (float per step) into host memory; synchronizes.
+ * Only the last 4096 steps are kept. */
+vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out);
+
+/*
+ * Enqueue an asynchronous copy of the mean loss of step k (already enqueued)
+ * into host memory `host_out` (pinned for asynchrony) on the stream of the
+ * step's active worker; valid once that stream passes this point.
+ */
+vfl_status vfl_fetch_loss(vfl_ctx* ctx, int64_t k, float* host_out);
+
+/* Copy a channel slot or a per-worker buffer of step k to host fp32 (see VFL_TAP_*); synchronizes. */
+vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out);
+
+/*
+ * Fault probe: a bounded device-side wait (at most max_iters polls) for the
+ * embedding (which = 0) or gradient (which = 1) channel slot of step k to carry
+ * header k.  Returns VFL_OK or VFL_E_TIMEOUT; never blocks indefinitely.
+ */
+vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_iters);
+
+/* Number of kernels this context has launched so far (for launch accounting). */
+int64_t vfl_kernel_launches(const vfl_ctx* ctx);
+
+/*
+ * Per-launch timing.  vfl_profile(ctx, 1) starts recording a CUDA event pair
+ * around every kernel launch, on the launch's stream; vfl_profile(ctx, 0)
+ * synchronizes and folds the records into per-class totals.  vfl_profile_get
+ * then returns, for kernel class `cls` (0 .. VFL_KERNEL_CLASSES-1, named by
+ * vfl_kernel_class_name), the number of launches, their summed duration in ms
+ * and their summed algorithmic flops and bytes.
+ */
+#define VFL_KERNEL_CLASSES 12
+vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);
+vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
+                           double* bytes);
+const char* vfl_kernel_class_name(int32_t cls);
+
+/* Last error message of the context (or of the last failed vfl_create / vfl_make_schedule when ctx is NULL). */
+const char* vfl_last_error(const vfl_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VFL_H */

@@ -1,0 +1,347 @@
+"""Python binding of libvfl, the GB300 split-VFL training step (PubSub-VFL,
+arxiv 2510.12494).  Argument marshalling only: every step of the training
+path runs in the library's CUDA kernels.  PyTorch provides the device
+workspace and the CUDA streams.
+
+There is no CPU fallback: if libvfl.so is missing, importing the library
+raises; build it with ``paper_2510_12494_gb300.build.build()``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libvfl.so")
+
+VFL_OK, VFL_E_INVAL, VFL_E_OOM, VFL_E_CUDA, VFL_E_STATE, VFL_E_VERSION, VFL_E_TIMEOUT = range(7)
+MAX_LAYERS = 8
+LOSS_BCE, LOSS_CE = 0, 1
+FP32, BF16 = 0, 1
+SCHED_SYNC, SCHED_MAX, SCHED_SEEDED = 0, 1, 2
+TAP_EMB, TAP_GRAD, TAP_LOGITS, TAP_ZA, TAP_DZA = range(5)
+PASSIVE, ACTIVE, TOP = 0, 1, 2
+KERNEL_CLASSES = 12
+
+STATUS_NAMES = {0: "VFL_OK", 1: "VFL_E_INVAL", 2: "VFL_E_OOM", 3: "VFL_E_CUDA", 4: "VFL_E_STATE",
+                5: "VFL_E_VERSION", 6: "VFL_E_TIMEOUT"}
+
+
+class VflError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class VflConfig(ctypes.Structure):
+    _fields_ = [
+        ("d_passive", ctypes.c_int32), ("d_active", ctypes.c_int32),
+        ("n_passive", ctypes.c_int32), ("n_active", ctypes.c_int32), ("n_top", ctypes.c_int32),
+        ("passive_out", ctypes.c_int32 * MAX_LAYERS), ("active_out", ctypes.c_int32 * MAX_LAYERS),
+        ("top_out", ctypes.c_int32 * MAX_LAYERS),
+        ("loss", ctypes.c_int32), ("dtype", ctypes.c_int32), ("batch", ctypes.c_int32),
+        ("lr", ctypes.c_float), ("staleness", ctypes.c_int32), ("workers", ctypes.c_int32),
+        ("dp_clip", ctypes.c_float), ("dp_sigma", ctypes.c_float), ("dp_seed", ctypes.c_uint64),
+    ]
+
+
+EXPORTS = {
+    # name: (restype, argtypes)
+    "vfl_workspace_bytes": (ctypes.c_int32, [ctypes.POINTER(VflConfig), ctypes.c_int64, ctypes.POINTER(ctypes.c_uint64)]),
+    "vfl_create": (ctypes.c_int32, [ctypes.POINTER(VflConfig), ctypes.c_int64, ctypes.c_void_p, ctypes.c_uint64,
+                                    ctypes.POINTER(ctypes.c_void_p)]),
+    "vfl_destroy": (ctypes.c_int32, [ctypes.c_void_p]),
+    "vfl_set_streams": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]),
+    "vfl_load_data": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_stage_rows": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64,
+                                        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_set_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+                                        ctypes.c_void_p]),
+    "vfl_get_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+                                        ctypes.c_void_p]),
+    "vfl_get_grads": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                       ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_step_cursor": (ctypes.c_int32, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)]),
+    "vfl_get_version": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                                         ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_set_cursor": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_set_version": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                                         ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_make_schedule": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                                           ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_passive_forward": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32]),
+    "vfl_active_step": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32]),
+    "vfl_passive_backward": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_train_steps": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+                                         ctypes.c_void_p]),
+    "vfl_synchronize": (ctypes.c_int32, [ctypes.c_void_p]),
+    "vfl_read_losses": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]),
+    "vfl_tap": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p]),
+    "vfl_fetch_loss": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
+    "vfl_wait_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64]),
+    "vfl_kernel_launches": (ctypes.c_int64, [ctypes.c_void_p]),
+    "vfl_profile": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32]),
+    "vfl_profile_get": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64),
+                                         ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                                         ctypes.POINTER(ctypes.c_double)]),
+    "vfl_kernel_class_name": (ctypes.c_char_p, [ctypes.c_int32]),
+    "vfl_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
+}
+
+_lib = None
+
+
+def lib():
+    """The loaded libvfl.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} is missing: build it with paper_2510_12494_gb300.build.build() "
+                              "(there is no CPU fallback)")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in EXPORTS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _check(st: int, ctx=None):
+    if st != VFL_OK:
+        msg = lib().vfl_last_error(ctx)
+        raise VflError(st, msg.decode() if msg else "")
+
+
+def make_config(p) -> VflConfig:
+    """VflConfig from an object with the preset fields (d_passive, d_active,
+    passive, active, top, loss, dtype, batch, lr, staleness, workers, dp_clip,
+    dp_sigma, seed)."""
+    c = VflConfig()
+    c.d_passive, c.d_active = p.d_passive, p.d_active
+    c.n_passive, c.n_active, c.n_top = len(p.passive), len(p.active), len(p.top)
+    for arr, vals in ((c.passive_out, p.passive), (c.active_out, p.active), (c.top_out, p.top)):
+        for i, v in enumerate(vals):
+            arr[i] = v
+    c.loss = LOSS_BCE if p.loss == "bce" else LOSS_CE
+    c.dtype = FP32 if p.dtype == "fp32" else BF16
+    c.batch = p.batch
+    c.lr = p.lr
+    c.staleness = p.staleness
+    c.workers = p.workers
+    c.dp_clip = p.dp_clip
+    c.dp_sigma = p.dp_sigma
+    c.dp_seed = getattr(p, "dp_seed", getattr(p, "seed", 0))
+    return c
+
+
+def make_schedule(seed: int, S: int, kind: int, n_steps: int):
+    """(tau_p, tau_a) int32 arrays from the library's host-side schedule."""
+    tp = np.zeros(max(n_steps, 1), np.int32)
+    ta = np.zeros(max(n_steps, 1), np.int32)
+    _check(lib().vfl_make_schedule(seed, S, kind, n_steps, _ptr(tp), _ptr(ta)))
+    return tp[:n_steps], ta[:n_steps]
+
+
+def workspace_bytes(p, n_rows: int) -> int:
+    cfg = make_config(p)
+    out = ctypes.c_uint64()
+    _check(lib().vfl_workspace_bytes(ctypes.byref(cfg), n_rows, ctypes.byref(out)))
+    return out.value
+
+
+class Context:
+    """One training context on the current CUDA device."""
+
+    def __init__(self, p, n_rows: int, streams=None):
+        import torch
+        self.p = p
+        self.cfg = make_config(p)
+        self.n_rows = n_rows
+        L = lib()
+        nbytes = workspace_bytes(p, n_rows)
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+        handle = ctypes.c_void_p()
+        _check(L.vfl_create(ctypes.byref(self.cfg), n_rows, ctypes.c_void_p(self.workspace.data_ptr()),
+                            nbytes, ctypes.byref(handle)))
+        self.h = handle
+        self.streams = streams if streams is not None else [torch.cuda.Stream() for _ in range(2 * p.workers)]
+        arr = (ctypes.c_void_p * len(self.streams))(*[s.cuda_stream for s in self.streams])
+        self._call(L.vfl_set_streams, len(self.streams), arr)
+        self.nb = -(-n_rows // p.batch)
+
+    def _call(self, f, *args):
+        st = f(self.h, *args)
+        if st != VFL_OK:
+            msg = lib().vfl_last_error(self.h)
+            raise VflError(st, msg.decode() if msg else "")
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().vfl_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # data / parameters -----------------------------------------------------
+    def load_data(self, xp, xa, y):
+        xp = np.ascontiguousarray(xp, np.float32)
+        xa = np.ascontiguousarray(xa, np.float32)
+        y = np.ascontiguousarray(y, np.int32)
+        assert xp.shape == (self.n_rows, self.p.d_passive) and xa.shape == (self.n_rows, self.p.d_active)
+        self._call(lib().vfl_load_data, _ptr(xp), _ptr(xa), _ptr(y))
+
+    def stage_rows(self, worker, row0, xp, xa, y):
+        """Asynchronous host->device copy of rows [row0, row0+len(y)); the arrays
+        (ideally pinned) must stay alive until the worker streams pass this point."""
+        def addr(a):
+            return a.data_ptr() if hasattr(a, "data_ptr") else a.ctypes.data
+        self._call(lib().vfl_stage_rows, worker, row0, len(y), ctypes.c_void_p(addr(xp)), ctypes.c_void_p(addr(xa)),
+                   ctypes.c_void_p(addr(y)))
+
+    def set_params(self, params: dict):
+        for (party, l), (W, b) in params.items():
+            W = np.ascontiguousarray(W, np.float32)
+            b = np.ascontiguousarray(b, np.float32)
+            self._call(lib().vfl_set_params, party, l, _ptr(W), _ptr(b))
+
+    def _shape(self, party, l):
+        widths = (self.p.passive, self.p.active, self.p.top)[party]
+        fin = (self.p.d_passive, self.p.d_active, self.p.e_active + self.p.e_passive)[party] if l == 0 else widths[l - 1]
+        return widths[l], fin
+
+    def get_params(self):
+        out = {}
+        for party, widths in ((0, self.p.passive), (1, self.p.active), (2, self.p.top)):
+            for l in range(len(widths)):
+                o, i = self._shape(party, l)
+                W = np.zeros((o, i), np.float32)
+                b = np.zeros(o, np.float32)
+                self._call(lib().vfl_get_params, party, l, _ptr(W), _ptr(b))
+                out[(party, l)] = (W, b)
+        return out
+
+    def get_grads(self, worker: int = 0, parties=(0, 1, 2)):
+        out = {}
+        for party in parties:
+            widths = (self.p.passive, self.p.active, self.p.top)[party]
+            for l in range(len(widths)):
+                o, i = self._shape(party, l)
+                dW = np.zeros((o, i), np.float32)
+                db = np.zeros(o, np.float32)
+                self._call(lib().vfl_get_grads, party, l, worker, _ptr(dW), _ptr(db))
+                out[(party, l)] = (dW, db)
+        return out
+
+    # checkpoint / restore --------------------------------------------------
+    def cursor(self) -> int:
+        k = ctypes.c_int64()
+        self._call(lib().vfl_step_cursor, ctypes.byref(k))
+        return k.value
+
+    def get_version(self, v: int):
+        """{(party, layer): (W, b)} of stored weight version v (compute copy, as fp32)."""
+        out = {}
+        for party, widths in ((0, self.p.passive), (1, self.p.active), (2, self.p.top)):
+            for l in range(len(widths)):
+                o, i = self._shape(party, l)
+                W = np.zeros((o, i), np.float32)
+                b = np.zeros(o, np.float32)
+                self._call(lib().vfl_get_version, party, l, v, _ptr(W), _ptr(b))
+                out[(party, l)] = (W, b)
+        return out
+
+    def set_cursor(self, k: int):
+        self._call(lib().vfl_set_cursor, k)
+
+    def set_version(self, v: int, params: dict, parties=(0, 1, 2)):
+        for (party, l), (W, b) in params.items():
+            if party not in parties:
+                continue
+            W = np.ascontiguousarray(W, np.float32)
+            b = np.ascontiguousarray(b, np.float32)
+            self._call(lib().vfl_set_version, party, l, v, _ptr(W), _ptr(b))
+
+    def checkpoint(self):
+        """(k, {version: params}, fp32 masters of version k)."""
+        k = self.cursor()
+        vers = {v: self.get_version(v) for v in range(max(0, k - self.p.staleness), k + 1)}
+        return k, vers, self.get_params()
+
+    def restore(self, ckpt):
+        k, vers, master = ckpt
+        self.set_cursor(k)
+        for v, params in vers.items():
+            self.set_version(v, master if v == k else params)
+
+    # the three phases and the whole DAG ------------------------------------
+    def passive_forward(self, k, tau_p):
+        self._call(lib().vfl_passive_forward, k, tau_p)
+
+    def active_step(self, k, tau_a):
+        self._call(lib().vfl_active_step, k, tau_a)
+
+    def passive_backward(self, k):
+        self._call(lib().vfl_passive_backward, k)
+
+    def train_steps(self, k0, n, tau_p, tau_a):
+        tau_p = np.ascontiguousarray(tau_p, np.int32)
+        tau_a = np.ascontiguousarray(tau_a, np.int32)
+        assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
+        self._call(lib().vfl_train_steps, k0, n, _ptr(tau_p), _ptr(tau_a))
+
+    def synchronize(self):
+        self._call(lib().vfl_synchronize)
+
+    def read_losses(self, k0, n):
+        out = np.zeros(max(n, 1), np.float32)
+        self._call(lib().vfl_read_losses, k0, n, _ptr(out))
+        return out[:n]
+
+    def fetch_loss(self, k, host_ptr: int):
+        """Asynchronous device->host copy of step k's mean loss to host address host_ptr."""
+        self._call(lib().vfl_fetch_loss, k, ctypes.c_void_p(host_ptr))
+
+    def batch_rows(self, k):
+        j = k % self.nb
+        r0 = j * self.p.batch
+        return r0, min(self.n_rows, r0 + self.p.batch)
+
+    def tap(self, k, what):
+        r0, r1 = self.batch_rows(k)
+        cols = {TAP_EMB: self.p.e_passive, TAP_GRAD: self.p.e_passive, TAP_LOGITS: self.p.n_out,
+                TAP_ZA: self.p.e_active, TAP_DZA: self.p.e_active}[what]
+        out = np.zeros((r1 - r0, cols), np.float32)
+        self._call(lib().vfl_tap, k, what, _ptr(out))
+        return out
+
+    def wait_channel(self, which, k, max_iters):
+        self._call(lib().vfl_wait_channel, which, k, max_iters)
+
+    @property
+    def launches(self) -> int:
+        return lib().vfl_kernel_launches(self.h)
+
+    def profile(self, enable: bool):
+        self._call(lib().vfl_profile, 1 if enable else 0)
+
+    def profile_summary(self):
+        """{class name: (launches, ms, flops, bytes)} of the last profiled region."""
+        out = {}
+        for c in range(KERNEL_CLASSES):
+            n, ms, fl, by = ctypes.c_int64(), ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+            _check(lib().vfl_profile_get(self.h, c, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(fl),
+                                         ctypes.byref(by)), self.h)
+            if n.value:
+                out[lib().vfl_kernel_class_name(c).decode()] = (n.value, ms.value, fl.value, by.value)
+        return out

@@ -1,0 +1,400 @@
+// SIMT kernels of the split-VFL step: the fp32 GEMM used for fp32 contexts and
+// for narrow layers, the fused loss, DP clip+noise, ReLU mask, fused SGD,
+// channel headers and data casts.
+#include "vfl_kernels.cuh"
+
+namespace vfl {
+
+namespace {
+
+__device__ __forceinline__ float ldf(const float* p) { return *p; }
+__device__ __forceinline__ float ldf(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+
+__device__ __forceinline__ void stf(void* base, long long idx, int bf16, float v) {
+    if (bf16)
+        static_cast<__nv_bfloat16*>(base)[idx] = __float2bfloat16_rn(v);
+    else
+        static_cast<float*>(base)[idx] = v;
+}
+
+__device__ __forceinline__ float ldany(const void* base, long long idx, int bf16) {
+    return bf16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(base)[idx])
+                : static_cast<const float*>(base)[idx];
+}
+
+// Philox4x32-10 (Salmon et al., SC'11): ten rounds of two 32x32->64 products,
+// key bumped by the Weyl increments between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 key) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const unsigned lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+        const unsigned lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+        c = make_uint4(hi1 ^ c.y ^ key.x, lo1, hi0 ^ c.w ^ key.y, lo0);
+        key.x += 0x9E3779B9u;
+        key.y += 0xBB67AE85u;
+    }
+    return c;
+}
+
+constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
+
+template <typename TA, typename TB, typename TM>
+__global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
+    __shared__ float As[BK][BM + 1];
+    __shared__ float Bs[BK][BN + 1];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+    const int kb = blockIdx.z * g.kchunk;
+    const int ke = min(g.K, kb + g.kchunk);
+    const TA* A = static_cast<const TA*>(g.A);
+    const TA* A2 = static_cast<const TA*>(g.A2);
+    const TB* B = static_cast<const TB*>(g.B);
+    float acc[4][4] = {};
+    float bsum[4] = {};
+    const bool want_bsum = g.mode == GEMM_DW && blockIdx.y == 0 && tx == 0 && g.Pb != nullptr;
+
+    for (int k0 = kb; k0 < ke; k0 += BK) {
+        for (int e = threadIdx.x; e < BM * BK; e += NT) {
+            int mm, kk;
+            if (g.a_cs == 1) { mm = e / BK; kk = e % BK; } else { kk = e / BM; mm = e % BM; }
+            const int m = m0 + mm, k = k0 + kk;
+            float v = 0.f;
+            if (m < g.M && k < ke) {
+                if (A2 != nullptr && k >= g.ka)
+                    v = ldf(A2 + (long long)m * g.a2_rs + (long long)(k - g.ka) * g.a_cs);
+                else
+                    v = ldf(A + (long long)m * g.a_rs + (long long)k * g.a_cs);
+            }
+            As[kk][mm] = v;
+        }
+        for (int e = threadIdx.x; e < BN * BK; e += NT) {
+            int nn, kk;
+            if (g.b_cs == 1) { nn = e / BK; kk = e % BK; } else { kk = e / BN; nn = e % BN; }
+            const int n = n0 + nn, k = k0 + kk;
+            float v = 0.f;
+            if (n < g.N && k < ke) v = ldf(B + (long long)n * g.b_rs + (long long)k * g.b_cs);
+            Bs[kk][nn] = v;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < BK; ++kk) {
+            float av[4], bv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) av[i] = As[kk][ty * 4 + i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                if (want_bsum) bsum[i] += av[i];
+            }
+        }
+        __syncthreads();
+    }
+
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int m = m0 + ty * 4 + i;
+        if (m >= g.M) continue;
+        if (want_bsum) g.Pb[(long long)blockIdx.z * g.pb_stride + m] = bsum[i];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int n = n0 + tx * 4 + j;
+            if (n >= g.N) continue;
+            float v = acc[i][j];
+            if (g.mode == GEMM_FWD) {
+                if (g.bias) v += g.bias[n];
+                if (g.relu) v = fmaxf(v, 0.f);
+                stf(g.C, (long long)m * g.ldc + n, g.c_bf16, v);
+            } else if (g.mode == GEMM_DX) {
+                if (n < g.n_split) {
+                    if (g.mask1 && !(ldf(static_cast<const TM*>(g.mask1) + (long long)m * g.mask1_ld + n) > 0.f))
+                        v = 0.f;
+                    stf(g.C, (long long)m * g.ldc + n, g.c_bf16, v);
+                } else {
+                    const int n2 = n - g.n_split;
+                    if (g.mask2 && !(ldf(static_cast<const TM*>(g.mask2) + (long long)m * g.mask2_ld + n2) > 0.f))
+                        v = 0.f;
+                    stf(g.C2, (long long)m * g.ldc2 + n2, g.c2_bf16, v);
+                }
+            } else {
+                g.P[(long long)blockIdx.z * g.p_stride + (long long)m * g.ldc + n] = v;
+            }
+        }
+    }
+}
+
+template <typename TA, typename TB>
+cudaError_t gemm_dispatch_mask(const GemmArgs& g, int mask_bf16, dim3 grid, cudaStream_t s) {
+    if (mask_bf16)
+        gemm_simt_kernel<TA, TB, __nv_bfloat16><<<grid, NT, 0, s>>>(g);
+    else
+        gemm_simt_kernel<TA, TB, float><<<grid, NT, 0, s>>>(g);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Loss (BCE in logit form / softmax CE), one block, fixed-order reduction.
+// ---------------------------------------------------------------------------
+constexpr int LOSS_NT = 1024;
+
+__global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__ logits, const int* __restrict__ y,
+                                                        int rows, int n_out, int kind, float* __restrict__ ds,
+                                                        float* __restrict__ loss_out) {
+    __shared__ float red[LOSS_NT / 32];
+    const float inv_b = 1.0f / (float)rows;
+    float part = 0.f;
+    for (int r = threadIdx.x; r < rows; r += LOSS_NT) {
+        const float* s = logits + (long long)r * n_out;
+        float* d = ds + (long long)r * n_out;
+        const int label = y[r];
+        if (kind == VFL_LOSS_BCE) {
+            const float x = s[0];
+            const float yf = (float)label;
+            part += fmaxf(x, 0.f) - x * yf + log1pf(expf(-fabsf(x)));
+            const float sig = 1.0f / (1.0f + expf(-x));
+            d[0] = (sig - yf) * inv_b;
+        } else {
+            float m = s[0];
+            for (int j = 1; j < n_out; ++j) m = fmaxf(m, s[j]);
+            float z = 0.f;
+            for (int j = 0; j < n_out; ++j) z += expf(s[j] - m);
+            part += logf(z) + m - s[label];
+            const float iz = 1.0f / z;
+            for (int j = 0; j < n_out; ++j) {
+                const float p = expf(s[j] - m) * iz - (j == label ? 1.f : 0.f);
+                d[j] = p * inv_b;
+            }
+        }
+    }
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = part;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float v = red[threadIdx.x];
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+        if (threadIdx.x == 0) *loss_out = v * inv_b;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// DP: per-row clip of the per-sample gradient B*dz to norm C, plus sigma*C*N(0,1).
+// ---------------------------------------------------------------------------
+constexpr int DP_NT = 256;
+
+__global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in, long long ld_in, void* out,
+                                                    long long ld_out, int out_bf16, int e, float clip, float sigma,
+                                                    unsigned long long seed, long long k, float bk) {
+    __shared__ float red[DP_NT / 32];
+    __shared__ float s_factor;
+    const int r = blockIdx.x;
+    const float* row = in + (long long)r * ld_in;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < e; c += DP_NT) {
+        const float gv = row[c] * bk;
+        ss = fmaf(gv, gv, ss);
+    }
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_down_sync(0xffffffffu, ss, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float v = threadIdx.x < DP_NT / 32 ? red[threadIdx.x] : 0.f;
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+        if (threadIdx.x == 0) {
+            const float norm = sqrtf(v);
+            s_factor = norm > clip ? clip / norm : 1.0f;
+        }
+    }
+    __syncthreads();
+    const float factor = s_factor;
+    const uint2 key = make_uint2((unsigned)(seed & 0xFFFFFFFFull), (unsigned)(seed >> 32));
+    const float scale = sigma * clip;
+    for (int q = threadIdx.x; q * 4 < e; q += DP_NT) {
+        const uint4 w = philox4x32_10(make_uint4((unsigned)q, (unsigned)r, (unsigned)(k & 0xFFFFFFFFll), 0x4450u), key);
+        const unsigned xs[4] = {w.x, w.y, w.z, w.w};
+        float z[4];
+#pragma unroll
+        for (int p = 0; p < 2; ++p) {
+            const float u1 = (float)((xs[2 * p] >> 8) + 1u) * 0x1p-24f;
+            const float u2 = (float)(xs[2 * p + 1] >> 8) * 0x1p-24f;
+            const float rad = sqrtf(-2.0f * logf(u1));
+            float sn, cs;
+            sincospif(2.0f * u2, &sn, &cs);
+            z[2 * p] = rad * cs;
+            z[2 * p + 1] = rad * sn;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int c = 4 * q + j;
+            if (c < e) {
+                const float gv = row[c] * bk;
+                const float v = (gv * factor + scale * z[j]) / bk;
+                stf(out, (long long)r * ld_out + c, out_bf16, v);
+            }
+        }
+    }
+}
+
+template <typename T>
+__global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ z, T* __restrict__ out,
+                                 long long ld, int rows, int e) {
+    const long long n = (long long)rows * e;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const long long r = i / e, c = i % e;
+        const long long idx = r * ld + c;
+        out[idx] = ldf(z + idx) > 0.f ? g[idx] : T(0.f);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// SGD (Eq. 2): master -= lr * sum_z partial[z]; write the new version's copy.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < a.total;
+         i += (long long)gridDim.x * blockDim.x) {
+        int l = 0;
+        while (l + 1 < a.n_layers && i >= a.L[l + 1].begin) ++l;
+        const SgdLayer& L = a.L[l];
+        const long long idx = i - L.begin;
+        const long long nw = (long long)L.out * L.in;
+        if (idx < nw) {
+            float gsum = 0.f;
+            for (int z = 0; z < L.nsplit; ++z) gsum += L.pW[z * L.pW_stride + idx];
+            const float w = L.W[idx] - a.lr * gsum;
+            L.W[idx] = w;
+            const long long r = idx / L.in, c = idx % L.in;
+            stf(L.cW, r * L.in_ld + c, a.c_bf16, w);
+        } else {
+            const long long j = idx - nw;
+            float gsum = 0.f;
+            for (int z = 0; z < L.nsplit; ++z) gsum += L.pb[z * L.pb_stride + j];
+            const float b = L.b[j] - a.lr * gsum;
+            L.b[j] = b;
+            L.cb[j] = b;
+        }
+    }
+}
+
+__global__ void write_header_kernel(ChannelHeader* h, long long k, int batch, int version) {
+    h->k = k;
+    h->batch = batch;
+    h->version = version;
+    __threadfence();
+}
+
+__global__ void check_header_kernel(const ChannelHeader* h, long long k, int* status) {
+    if (h->k != k) atomicOr(status, ST_VERSION);
+}
+
+// Bounded poll: gives up after max_iters reads and records ST_TIMEOUT.
+__global__ void wait_header_kernel(const ChannelHeader* h, long long k, long long max_iters, int* status) {
+    const volatile long long* pk = &h->k;
+    for (long long it = 0; it < max_iters; ++it) {
+        if (*pk == k) return;
+        __nanosleep(256);
+    }
+    atomicOr(status, ST_TIMEOUT);
+}
+
+__global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d, void* dst, long long ld, int bf16) {
+    const long long n = (long long)rows * ld;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const long long r = i / ld, c = i % ld;
+        const float v = c < d ? src[r * d + c] : 0.f;
+        stf(dst, i, bf16, v);
+    }
+}
+
+__global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
+    const long long n = (long long)rows * cols;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const long long r = i / cols, c = i % cols;
+        dst[i] = ldany(src, r * ld + c, bf16);
+    }
+}
+
+inline int grid_for(long long n, int nt) {
+    long long b = (n + nt - 1) / nt;
+    if (b < 1) b = 1;
+    if (b > 152 * 16) b = 152 * 16;
+    return (int)b;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask_bf16, int nsplit, cudaStream_t s) {
+    if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+    GemmArgs a = g;
+    if (a.mode != GEMM_DW) {
+        nsplit = 1;
+        a.kchunk = a.K;
+    }
+    // DW: every one of the nsplit partials is written (zeros where its chunk is empty)
+    if (nsplit < 1 || a.kchunk < 1) return cudaErrorInvalidValue;
+    dim3 grid((a.M + BM - 1) / BM, (a.N + BN - 1) / BN, nsplit);
+    if (a_bf16 && b_bf16) return gemm_dispatch_mask<__nv_bfloat16, __nv_bfloat16>(a, mask_bf16, grid, s);
+    if (a_bf16) return gemm_dispatch_mask<__nv_bfloat16, float>(a, mask_bf16, grid, s);
+    if (b_bf16) return gemm_dispatch_mask<float, __nv_bfloat16>(a, mask_bf16, grid, s);
+    return gemm_dispatch_mask<float, float>(a, mask_bf16, grid, s);
+}
+
+cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
+                        float* loss_out, cudaStream_t s) {
+    loss_kernel<<<1, LOSS_NT, 0, s>>>(logits, y, rows, n_out, loss_kind, ds, loss_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_out, int out_bf16, int rows, int e,
+                      float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    dp_kernel<<<rows, DP_NT, 0, s>>>(in, ld_in, out, ld_out, out_bf16, e, clip, sigma, seed, k, (float)rows);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
+                             cudaStream_t s) {
+    const int nb = grid_for((long long)rows * e, 256);
+    if (bf16)
+        relu_mask_kernel<__nv_bfloat16><<<nb, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(g),
+                                                           static_cast<const __nv_bfloat16*>(z),
+                                                           static_cast<__nv_bfloat16*>(out), ld, rows, e);
+    else
+        relu_mask_kernel<float><<<nb, 256, 0, s>>>(static_cast<const float*>(g), static_cast<const float*>(z),
+                                                   static_cast<float*>(out), ld, rows, e);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
+    sgd_kernel<<<grid_for(a.total, 256), 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_write_header(ChannelHeader* h, long long k, int batch, int version, cudaStream_t s) {
+    write_header_kernel<<<1, 1, 0, s>>>(h, k, batch, version);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status, cudaStream_t s) {
+    check_header_kernel<<<1, 1, 0, s>>>(h, k, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status, cudaStream_t s) {
+    wait_header_kernel<<<1, 1, 0, s>>>(h, k, max_iters, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    cast_rows_kernel<<<grid_for((long long)rows * ld, 256), 256, 0, s>>>(src, rows, d, dst, ld, bf16);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_to_f32(const void* src, long long ld, int rows, int cols, int bf16, float* dst, cudaStream_t s) {
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    to_f32_kernel<<<grid_for((long long)rows * cols, 256), 256, 0, s>>>(src, ld, rows, cols, bf16, dst);
+    return cudaGetLastError();
+}
+
+}  // namespace vfl

@@ -1,0 +1,95 @@
+// Internal declarations shared by the kernels and the host runtime of libvfl.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "vfl.h"
+
+namespace vfl {
+
+// Header written after a channel payload (embedding or gradient) is complete.
+struct ChannelHeader {
+    long long k;      // step that published the slot
+    int batch;        // batch id j of that step
+    int version;      // weight version that produced the payload
+};
+
+// Bits of the device status word.
+enum : int { ST_VERSION = 1, ST_TIMEOUT = 2 };
+
+enum GemmMode : int { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
+
+// C[m, n] = sum_k A(m, k) * B(n, k) with strided operands.
+//   A(m, k) = A[m * a_rs + k * a_cs]   (k >= ka reads A2[m * a2_rs + (k - ka) * a_cs])
+//   B(n, k) = B[n * b_rs + k * b_cs]
+// Epilogues:
+//   FWD: C = act(acc + bias[n]); act = ReLU when relu != 0.
+//   DX : columns n < n_split go to C (masked by mask1[m, n] > 0 when mask1 != 0),
+//        columns n >= n_split to C2 at column n - n_split (masked by mask2 when set).
+//   DW : split-K partial: P[z * p_stride + m * ldc + n] = sum over k in chunk z;
+//        Pb[z * pb_stride + m] = sum_k A(m, k) over the chunk (bias gradient).
+struct GemmArgs {
+    int mode;
+    int M, N, K;
+    const void* A; long long a_rs, a_cs;
+    const void* A2; long long a2_rs; int ka;
+    const void* B; long long b_rs, b_cs;
+    const float* bias; int relu;
+    void* C; long long ldc; int c_bf16;
+    void* C2; long long ldc2; int c2_bf16; int n_split;
+    const void* mask1; long long mask1_ld;
+    const void* mask2; long long mask2_ld;
+    float* P; long long p_stride;
+    float* Pb; long long pb_stride;
+    int kchunk;
+};
+
+// Launch the SIMT GEMM (fp32 FFMA).  a_bf16 / b_bf16 select operand element
+// types; masks share the element type of the compute dtype (mask_bf16).
+cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask_bf16, int nsplit,
+                             cudaStream_t s);
+
+// Loss + d(logits) over one batch (single block, deterministic reduction):
+//   rows: B_k; logits fp32 [B_k, n_out]; y int32 labels of the batch rows.
+//   ds [B_k, n_out] = dLoss/dlogits of the batch-mean loss; loss_out = mean loss.
+cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
+                        float* loss_out, cudaStream_t s);
+
+// DP on the published gradient (one block per row):
+//   in fp32 [rows, e] (ld_in), out compute dtype [rows, e] (ld_out).
+cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_out, int out_bf16, int rows,
+                      int e, float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s);
+
+// out[r, c] = g[r, c] * (z[r, c] > 0), compute dtype, [rows, e] with leading dim ld.
+cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
+                             cudaStream_t s);
+
+struct SgdLayer {
+    float* W; float* b;           // fp32 master
+    const float* pW; const float* pb;  // split-K partial gradients
+    long long pW_stride, pb_stride;
+    int nsplit;
+    int out, in, in_ld;
+    void* cW; float* cb;          // compute copy to write (ring slot of the new version)
+    long long begin;              // first flat element index of this layer
+};
+constexpr int kMaxSgdLayers = 16;
+struct SgdArgs {
+    SgdLayer L[kMaxSgdLayers];
+    int n_layers;
+    long long total;
+    float lr;
+    int c_bf16;
+};
+cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s);
+
+cudaError_t launch_write_header(ChannelHeader* h, long long k, int batch, int version, cudaStream_t s);
+cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status, cudaStream_t s);
+cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,
+                               cudaStream_t s);
+cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s);
+cudaError_t launch_to_f32(const void* src, long long ld, int rows, int cols, int bf16, float* dst, cudaStream_t s);
+
+}  // namespace vfl

@@ -1,0 +1,1204 @@
+// Host runtime of libvfl: context, workspace layout, channel rings, the
+// per-phase enqueue logic and the exported C ABI (include/vfl.h).
+//
+// Mapping to the paper (arxiv 2510.12494):
+//  - Sec. 3 / Eq. 1-2: split forward, loss, cut-layer gradient exchange, SGD.
+//  - Algorithm 1: vfl_passive_forward = publisher phase, vfl_active_step =
+//    subscriber phase, vfl_passive_backward = backward phase.
+//  - Sec. 4.1 channels keyed by batch id with bounded buffers: here HBM rings of
+//    S+1 slots with a header {k, batch, version}; a CUDA event per publish
+//    orders the subscriber's stream after the publisher's.
+//  - App. D (Assumption 4, theorem): the gradient applied at step k was
+//    computed with weights of version k - tau(k); updates apply in step order.
+//    Each party keeps its S+1 most recent weight versions in a ring.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "vfl_kernels.cuh"
+#include "vfl_tc.cuh"
+
+using namespace vfl;
+
+namespace {
+
+constexpr int kMaxWorkers = 16;
+constexpr int kMaxSlots = 16;
+constexpr int kEvPool = 64;
+constexpr int kLossCap = 4096;
+
+thread_local std::string g_global_err;
+
+// Kernel classes for launch accounting and per-class CUDA-event timing.
+enum KClass : int {
+    K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
+    K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST, K_NCLASS
+};
+const char* const kClassNames[K_NCLASS] = {
+    "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
+    "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast"};
+
+struct ProfRec {
+    int cls;
+    double flops, bytes;
+    cudaEvent_t e0, e1;
+};
+struct ProfAgg {
+    long long n = 0;
+    double ms = 0, flops = 0, bytes = 0;
+};
+
+inline long long ld8(long long x) { return (x + 7) / 8 * 8; }
+
+struct Layer {
+    int party = 0, idx = 0, in = 0, out = 0;
+    long long in_ld = 0;                  // leading dim of the compute copy of W
+    float* W = nullptr;                   // fp32 master [out, in]
+    float* b = nullptr;                   // fp32 master [out]
+    void* cW[kMaxSlots] = {};             // version copies [out, in_ld], compute dtype
+    float* cb[kMaxSlots] = {};            // version copies of b, fp32
+    float* pW[kMaxWorkers] = {};          // split-K partial dW [nsplit][out*in]
+    float* pb[kMaxWorkers] = {};          // partial db [nsplit][out]
+    int nsplit = 1;
+    int kchunk = 0;
+};
+
+// Bump allocator over the caller's workspace (dry run when base == nullptr).
+struct Carver {
+    char* base;
+    unsigned long long off = 0;
+    explicit Carver(void* b) : base(static_cast<char*>(b)) {}
+    void* take(unsigned long long bytes) {
+        off = (off + 255) / 256 * 256;
+        void* p = base ? base + off : nullptr;
+        off += bytes;
+        return p;
+    }
+};
+
+}  // namespace
+
+struct vfl_ctx {
+    vfl_config cfg{};
+    long long n_rows = 0;
+    int S1 = 1;                 // slots = staleness + 1
+    int W = 1;                  // workers per party
+    int esz = 4;                // bytes per compute element
+    int bf16 = 0;
+    int nb = 1;                 // steps per epoch
+    std::string err;
+    long long launches = 0;
+    bool broken = false;
+
+    std::vector<Layer> P, A, T;   // passive bottom, active bottom, top
+
+    // device buffers
+    void* Xp = nullptr; void* Xa = nullptr; int* Y = nullptr;
+    long long ldxp = 0, ldxa = 0;
+    float* stage_p[kMaxWorkers] = {};
+    float* stage_a[kMaxWorkers] = {};
+    std::vector<void*> act_p[kMaxSlots];          // per slot, per passive layer [B, ld8(out)]
+    std::vector<void*> dpre_p[kMaxWorkers];       // per worker, per passive layer
+    std::vector<void*> act_a[kMaxWorkers], dpre_a[kMaxWorkers];
+    std::vector<void*> act_t[kMaxWorkers], dpre_t[kMaxWorkers];  // top hidden layers
+    float* logits[kMaxWorkers] = {};
+    float* ds[kMaxWorkers] = {};
+    float* dzp32[kMaxWorkers] = {};
+    void* grad[kMaxSlots] = {};
+    ChannelHeader* emb_hdr = nullptr;   // [S1]
+    ChannelHeader* grad_hdr = nullptr;  // [S1]
+    float* losses = nullptr;            // [kLossCap]
+    int* status = nullptr;
+    float* scratch_f32 = nullptr;       // for taps [B * max width]
+    unsigned long long ws_bytes = 0;
+
+    // streams / events
+    cudaStream_t ps[kMaxWorkers] = {};
+    cudaStream_t as[kMaxWorkers] = {};
+    cudaEvent_t ev_pver[kEvPool] = {}, ev_aver[kEvPool] = {}, ev_emb[kEvPool] = {}, ev_grad[kEvPool] = {};
+
+    // per-launch timing (vfl_profile)
+    bool prof_on = false;
+    std::vector<ProfRec> prof;
+    std::vector<cudaEvent_t> ev_spare;
+    ProfAgg agg[K_NCLASS];
+
+    // host-side ordering state
+    long long n_fwd = 0, n_act = 0, n_bwd = 0;
+    int fwd_version[kMaxSlots] = {};
+    long long slot_step_p[kMaxSlots];
+    long long grad_step[kMaxSlots];
+    long long last_act_step[kMaxWorkers];
+    bool started = false;
+
+    vfl_status fail(vfl_status st, const char* fmt, ...) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(buf, sizeof buf, fmt, ap);
+        va_end(ap);
+        err = buf;
+        if (st == VFL_E_CUDA) broken = true;
+        return st;
+    }
+    vfl_status cuda(cudaError_t e, const char* what, int line) {
+        return fail(VFL_E_CUDA, "%s failed (line %d): %s", what, line, cudaGetErrorString(e));
+    }
+    int batch_rows(long long k, long long* r0) const {
+        const long long j = k % nb;
+        *r0 = j * cfg.batch;
+        return (int)std::min<long long>(cfg.batch, n_rows - *r0);
+    }
+};
+
+#define CK(call)                                                     \
+    do {                                                             \
+        cudaError_t e_ = (call);                                     \
+        if (e_ != cudaSuccess) return ctx->cuda(e_, #call, __LINE__); \
+    } while (0)
+
+namespace {
+
+cudaEvent_t spare_event(vfl_ctx* ctx) {
+    if (!ctx->ev_spare.empty()) {
+        cudaEvent_t e = ctx->ev_spare.back();
+        ctx->ev_spare.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+// Opens a profiled launch: records the start event when profiling is on.
+bool prof_begin(vfl_ctx* ctx, ProfRec* r, int cls, double flops, double bytes, cudaStream_t s) {
+    ++ctx->launches;
+    if (!ctx->prof_on) return false;
+    r->cls = cls;
+    r->flops = flops;
+    r->bytes = bytes;
+    r->e0 = spare_event(ctx);
+    r->e1 = spare_event(ctx);
+    if (!r->e0 || !r->e1) return false;
+    cudaEventRecord(r->e0, s);
+    return true;
+}
+
+void prof_end(vfl_ctx* ctx, ProfRec* r, bool on, cudaStream_t s) {
+    if (!on) return;
+    cudaEventRecord(r->e1, s);
+    ctx->prof.push_back(*r);
+}
+
+}  // namespace
+
+// Launch `call` (returning cudaError_t) on stream s as kernel class cls with
+// the given algorithmic flops / bytes.
+#define PLAUNCH(cls, flops, bytes, s, call)                              \
+    do {                                                                 \
+        ProfRec pr_;                                                     \
+        const bool on_ = prof_begin(ctx, &pr_, (cls), (flops), (bytes), (s)); \
+        cudaError_t e_ = (call);                                         \
+        if (e_ != cudaSuccess) return ctx->cuda(e_, #call, __LINE__);    \
+        prof_end(ctx, &pr_, on_, (s));                                   \
+    } while (0)
+
+namespace {
+
+vfl_status check_config(const vfl_config* c, long long n_rows, std::string* why) {
+    char buf[256];
+    auto bad = [&](const char* m) { *why = m; return VFL_E_INVAL; };
+    if (!c) return bad("null config");
+    if (n_rows < 1) return bad("n_rows must be >= 1");
+    if (c->d_passive < 1 || c->d_active < 1) return bad("feature dims must be >= 1");
+    if (c->n_passive < 1 || c->n_passive > VFL_MAX_LAYERS || c->n_active < 1 || c->n_active > VFL_MAX_LAYERS ||
+        c->n_top < 1 || c->n_top > VFL_MAX_LAYERS)
+        return bad("layer counts must be in [1, 8]");
+    for (int i = 0; i < c->n_passive; ++i) if (c->passive_out[i] < 1) return bad("passive width < 1");
+    for (int i = 0; i < c->n_active; ++i) if (c->active_out[i] < 1) return bad("active width < 1");
+    for (int i = 0; i < c->n_top; ++i) if (c->top_out[i] < 1) return bad("top width < 1");
+    const int n_out = c->top_out[c->n_top - 1];
+    if (c->loss == VFL_LOSS_BCE) {
+        if (n_out != 1) return bad("BCE needs n_out == 1");
+    } else if (c->loss == VFL_LOSS_CE) {
+        if (n_out < 2) return bad("CE needs n_out >= 2");
+    } else {
+        return bad("unknown loss");
+    }
+    if (c->dtype != VFL_FP32 && c->dtype != VFL_BF16) return bad("unknown dtype");
+    if (c->batch < 1) return bad("batch must be >= 1");
+    if (c->staleness < 0 || c->staleness + 1 > kMaxSlots) return bad("staleness must be in [0, 15]");
+    if (c->workers < 1 || c->workers > kMaxWorkers) return bad("workers must be in [1, 16]");
+    if (c->staleness + 1 + c->workers + 2 > kEvPool) return bad("staleness + workers too large");
+    if (!(c->lr >= 0.f)) return bad("lr must be >= 0");
+    if (c->dp_clip < 0.f || c->dp_sigma < 0.f) return bad("dp_clip / dp_sigma must be >= 0");
+    if (c->n_active + c->n_top > kMaxSgdLayers || c->n_passive > kMaxSgdLayers) return bad("too many layers");
+    (void)buf;
+    return VFL_OK;
+}
+
+// Split-K factor of a weight-gradient GEMM reducing over B rows.
+void choose_split(Layer& L, int B) {
+    const long long tiles = (long long)((L.out + 63) / 64) * ((L.in + 63) / 64);
+    long long ns = std::max<long long>(1, 2 * 152 / std::max<long long>(1, tiles));
+    ns = std::min<long long>(ns, std::max(1, B / 64));
+    ns = std::min<long long>(ns, 32);
+    L.kchunk = (int)(((B + ns - 1) / ns + 15) / 16 * 16);
+    L.nsplit = (B + L.kchunk - 1) / L.kchunk;
+}
+
+void build_layers(vfl_ctx* ctx) {
+    const vfl_config& c = ctx->cfg;
+    auto mk = [&](std::vector<Layer>& v, int party, int n, const int32_t* outs, int d_in) {
+        v.clear();
+        for (int l = 0; l < n; ++l) {
+            Layer L;
+            L.party = party;
+            L.idx = l;
+            L.in = d_in;
+            L.out = outs[l];
+            L.in_ld = ld8(d_in);
+            choose_split(L, c.batch);
+            v.push_back(L);
+            d_in = outs[l];
+        }
+    };
+    mk(ctx->P, 0, c.n_passive, c.passive_out, c.d_passive);
+    mk(ctx->A, 1, c.n_active, c.active_out, c.d_active);
+    mk(ctx->T, 2, c.n_top, c.top_out, c.active_out[c.n_active - 1] + c.passive_out[c.n_passive - 1]);
+}
+
+// Lay out every device buffer; with base == nullptr only measures.
+unsigned long long carve_all(vfl_ctx* ctx, void* base) {
+    Carver cv(base);
+    const vfl_config& c = ctx->cfg;
+    const int es = ctx->esz;
+    const long long B = c.batch;
+    ctx->ldxp = ld8(c.d_passive);
+    ctx->ldxa = ld8(c.d_active);
+    ctx->Xp = cv.take((unsigned long long)ctx->n_rows * ctx->ldxp * es);
+    ctx->Xa = cv.take((unsigned long long)ctx->n_rows * ctx->ldxa * es);
+    ctx->Y = static_cast<int*>(cv.take((unsigned long long)ctx->n_rows * 4));
+    for (int w = 0; w < ctx->W; ++w) {
+        ctx->stage_p[w] = static_cast<float*>(cv.take(B * c.d_passive * 4ull));
+        ctx->stage_a[w] = static_cast<float*>(cv.take(B * c.d_active * 4ull));
+    }
+    for (std::vector<Layer>* v : {&ctx->P, &ctx->A, &ctx->T}) {
+        for (Layer& L : *v) {
+            L.W = static_cast<float*>(cv.take((unsigned long long)L.out * L.in * 4));
+            L.b = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
+            for (int s = 0; s < ctx->S1; ++s) {
+                L.cW[s] = cv.take((unsigned long long)L.out * L.in_ld * es);
+                L.cb[s] = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
+            }
+            for (int w = 0; w < ctx->W; ++w) {
+                L.pW[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * L.in * 4));
+                L.pb[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * 4));
+            }
+        }
+    }
+    for (int s = 0; s < ctx->S1; ++s) {
+        ctx->act_p[s].clear();
+        for (const Layer& L : ctx->P) ctx->act_p[s].push_back(cv.take(B * ld8(L.out) * es));
+        ctx->grad[s] = cv.take(B * ld8(ctx->P.back().out) * es);
+    }
+    const int n_out = ctx->T.back().out;
+    for (int w = 0; w < ctx->W; ++w) {
+        ctx->dpre_p[w].clear();
+        for (const Layer& L : ctx->P) ctx->dpre_p[w].push_back(cv.take(B * ld8(L.out) * es));
+        ctx->act_a[w].clear();
+        ctx->dpre_a[w].clear();
+        for (const Layer& L : ctx->A) {
+            ctx->act_a[w].push_back(cv.take(B * ld8(L.out) * es));
+            ctx->dpre_a[w].push_back(cv.take(B * ld8(L.out) * es));
+        }
+        ctx->act_t[w].clear();
+        ctx->dpre_t[w].clear();
+        for (size_t l = 0; l + 1 < ctx->T.size(); ++l) {
+            ctx->act_t[w].push_back(cv.take(B * ld8(ctx->T[l].out) * es));
+            ctx->dpre_t[w].push_back(cv.take(B * ld8(ctx->T[l].out) * es));
+        }
+        ctx->logits[w] = static_cast<float*>(cv.take(B * n_out * 4ull));
+        ctx->ds[w] = static_cast<float*>(cv.take(B * n_out * 4ull));
+        ctx->dzp32[w] = static_cast<float*>(cv.take(B * ld8(ctx->P.back().out) * 4ull));
+    }
+    ctx->emb_hdr = static_cast<ChannelHeader*>(cv.take(sizeof(ChannelHeader) * ctx->S1));
+    ctx->grad_hdr = static_cast<ChannelHeader*>(cv.take(sizeof(ChannelHeader) * ctx->S1));
+    ctx->losses = static_cast<float*>(cv.take(kLossCap * 4ull));
+    ctx->status = static_cast<int*>(cv.take(256));
+    // scratch for taps and version reads/writes: a [B, widest] activation or a whole weight matrix
+    long long maxw = std::max<long long>(c.d_passive, c.d_active);
+    long long maxwt = 0;
+    for (auto* v : {&ctx->P, &ctx->A, &ctx->T})
+        for (const Layer& L : *v) {
+            maxw = std::max<long long>(maxw, std::max(L.out, L.in));
+            maxwt = std::max<long long>(maxwt, (long long)L.out * L.in_ld);
+        }
+    ctx->scratch_f32 = static_cast<float*>(cv.take(std::max(B * ld8(maxw), maxwt) * 4ull));
+    return cv.off + 256;
+}
+
+inline cudaStream_t pstream(vfl_ctx* ctx, long long k) { return ctx->ps[k % ctx->W]; }
+inline cudaStream_t astream(vfl_ctx* ctx, long long k) { return ctx->as[k % ctx->W]; }
+
+// ---- GEMM helpers ---------------------------------------------------------
+GemmArgs gemm_base(int mode, int M, int N, int K) {
+    GemmArgs g;
+    std::memset(&g, 0, sizeof g);
+    g.mode = mode;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.n_split = N;
+    return g;
+}
+
+// Y[rows, out] = act(X W^T + b); X may be [X1 | X2] split at column ka.
+vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, long long ldx, const void* X2,
+                      long long ldx2, int ka, int rows, void* Y, long long ldy, bool relu, bool y_f32,
+                      cudaStream_t s) {
+    const int in_bf = ctx->bf16;
+    const double flops = 2.0 * rows * L.out * L.in;
+    const double bytes = ((double)rows * L.in + (double)L.out * L.in) * ctx->esz +
+                         (double)rows * L.out * (y_f32 ? 4 : ctx->esz) + L.out * 4.0;
+    if (in_bf && tc_supported_fwd(L.in, L.out, X2 != nullptr, ka, y_f32)) {
+        TcGemm t = {};
+        t.mode = GEMM_FWD;
+        t.M = rows; t.N = L.out; t.K = L.in;
+        t.A = X; t.lda = ldx; t.A2 = X2; t.lda2 = ldx2; t.ka = X2 ? ka : L.in;
+        t.B = L.cW[slot]; t.ldb = L.in_ld;
+        t.bias = L.cb[slot]; t.relu = relu;
+        t.C = Y; t.ldc = ldy;
+        PLAUNCH(K_TC_FWD, flops, bytes, s, launch_tc_gemm(t, s));
+        return VFL_OK;
+    }
+    GemmArgs g = gemm_base(GEMM_FWD, rows, L.out, L.in);
+    g.A = X; g.a_rs = ldx; g.a_cs = 1;
+    if (X2) { g.A2 = X2; g.a2_rs = ldx2; g.ka = ka; }
+    g.B = L.cW[slot]; g.b_rs = L.in_ld; g.b_cs = 1;
+    g.bias = L.cb[slot];
+    g.relu = relu ? 1 : 0;
+    g.C = Y; g.ldc = ldy; g.c_bf16 = y_f32 ? 0 : in_bf;
+    PLAUNCH(K_SIMT_FWD, flops, bytes, s, launch_gemm_simt(g, in_bf, in_bf, in_bf, 1, s));
+    return VFL_OK;
+}
+
+// Partial dW, db of layer L for the step on worker w:
+//   dW[out, in] = dpre^T X, dpre [rows, out] (leading dim ldd, fp32 when dpre_f32).
+//   X may be [X1 | X2] split at column ka (then two GEMMs write the two column blocks).
+vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long long ldd, bool dpre_f32,
+                     const void* X, long long ldx, const void* X2, long long ldx2, int ka, int rows, cudaStream_t s) {
+    const int bf = ctx->bf16;
+    const int a_bf = dpre_f32 ? 0 : bf;
+    const double flops = 2.0 * rows * L.out * L.in;
+    const double bytes = (double)rows * L.out * (dpre_f32 ? 4 : ctx->esz) + (double)rows * L.in * ctx->esz +
+                         (double)L.nsplit * ((double)L.out * L.in + L.out) * 4;
+    if (bf && !dpre_f32 && tc_supported_dw(L.out, L.in, X2 != nullptr, ka)) {
+        TcGemm t = {};
+        t.mode = GEMM_DW;
+        t.M = L.out; t.N = L.in; t.K = rows;
+        t.A = dpre; t.lda = ldd;
+        t.B = X; t.ldb = ldx; t.B2 = X2; t.ldb2 = ldx2; t.kb = X2 ? ka : L.in;
+        t.P = L.pW[w]; t.p_stride = (long long)L.out * L.in; t.ldc = L.in;
+        t.Pb = L.pb[w]; t.pb_stride = L.out;
+        t.nsplit = L.nsplit; t.kchunk = L.kchunk;
+        PLAUNCH(K_TC_DW, flops, bytes, s, launch_tc_gemm(t, s));
+        return VFL_OK;
+    }
+    const int n1 = X2 ? ka : L.in;
+    GemmArgs g = gemm_base(GEMM_DW, L.out, n1, rows);
+    g.A = dpre; g.a_rs = 1; g.a_cs = ldd;
+    g.B = X; g.b_rs = 1; g.b_cs = ldx;
+    g.P = L.pW[w]; g.p_stride = (long long)L.out * L.in; g.ldc = L.in;
+    g.Pb = L.pb[w]; g.pb_stride = L.out;
+    g.kchunk = L.kchunk;
+    const double f1 = X2 ? flops * n1 / L.in : flops, b1 = X2 ? bytes * n1 / L.in : bytes;
+    PLAUNCH(K_SIMT_DW, f1, b1, s, launch_gemm_simt(g, a_bf, bf, bf, L.nsplit, s));
+    if (X2) {
+        GemmArgs g2 = gemm_base(GEMM_DW, L.out, L.in - ka, rows);
+        g2.A = dpre; g2.a_rs = 1; g2.a_cs = ldd;
+        g2.B = X2; g2.b_rs = 1; g2.b_cs = ldx2;
+        g2.P = L.pW[w] + ka; g2.p_stride = (long long)L.out * L.in; g2.ldc = L.in;
+        g2.Pb = nullptr;
+        g2.kchunk = L.kchunk;
+        PLAUNCH(K_SIMT_DW, flops - f1, bytes - b1, s, launch_gemm_simt(g2, a_bf, bf, bf, L.nsplit, s));
+    }
+    return VFL_OK;
+}
+
+// dX[rows, in] = dpre W (W of version slot), columns < n_split -> C (masked by
+// mask1 > 0), the rest -> C2 (masked by mask2 when given).
+vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, long long ldd, bool dpre_f32,
+                     int rows, void* C, long long ldc, const void* mask1, int n_split, void* C2, long long ldc2,
+                     bool c2_f32, const void* mask2, cudaStream_t s) {
+    const int bf = ctx->bf16;
+    const double flops = 2.0 * rows * L.out * L.in;
+    const double bytes = (double)rows * L.out * (dpre_f32 ? 4 : ctx->esz) + (double)L.out * L.in * ctx->esz +
+                         (double)rows * L.in * ctx->esz * 2;
+    if (bf && !dpre_f32 && tc_supported_dx(L.in, L.out, n_split, c2_f32)) {
+        TcGemm t = {};
+        t.mode = GEMM_DX;
+        t.M = rows; t.N = L.in; t.K = L.out;
+        t.A = dpre; t.lda = ldd;
+        t.B = L.cW[slot]; t.ldb = L.in_ld;
+        t.C = C; t.ldc = ldc; t.mask1 = mask1;
+        t.n_split = n_split; t.C2 = C2; t.ldc2 = ldc2; t.mask2 = mask2;
+        PLAUNCH(K_TC_DX, flops, bytes, s, launch_tc_gemm(t, s));
+        return VFL_OK;
+    }
+    GemmArgs g = gemm_base(GEMM_DX, rows, L.in, L.out);
+    g.A = dpre; g.a_rs = ldd; g.a_cs = 1;
+    g.B = L.cW[slot]; g.b_rs = 1; g.b_cs = L.in_ld;
+    g.C = C; g.ldc = ldc; g.c_bf16 = bf;
+    g.mask1 = mask1; g.mask1_ld = ldc;
+    g.n_split = n_split;
+    g.C2 = C2; g.ldc2 = ldc2; g.c2_bf16 = c2_f32 ? 0 : bf;
+    g.mask2 = mask2; g.mask2_ld = ldc2;
+    PLAUNCH(K_SIMT_DX, flops, bytes, s, launch_gemm_simt(g, dpre_f32 ? 0 : bf, bf, bf, 1, s));
+    return VFL_OK;
+}
+
+vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w, int new_slot, cudaStream_t s) {
+    SgdArgs args;
+    std::memset(&args, 0, sizeof args);
+    long long off = 0;
+    int n = 0;
+    for (std::vector<Layer>* v : {a, b}) {
+        if (!v) continue;
+        for (Layer& L : *v) {
+            SgdLayer& d = args.L[n++];
+            d.W = L.W; d.b = L.b;
+            d.pW = L.pW[w]; d.pb = L.pb[w];
+            d.pW_stride = (long long)L.out * L.in;
+            d.pb_stride = L.out;
+            d.nsplit = L.nsplit;
+            d.out = L.out; d.in = L.in; d.in_ld = L.in_ld;
+            d.cW = L.cW[new_slot]; d.cb = L.cb[new_slot];
+            d.begin = off;
+            off += (long long)L.out * L.in + L.out;
+        }
+    }
+    args.n_layers = n;
+    args.total = off;
+    args.lr = ctx->cfg.lr;
+    args.c_bf16 = ctx->bf16;
+    double bytes = 0;
+    for (int i = 0; i < n; ++i) {
+        const SgdLayer& d = args.L[i];
+        const double np_ = (double)d.out * d.in + d.out;
+        bytes += np_ * (8.0 + 4.0 * d.nsplit) + (double)d.out * d.in * ctx->esz + d.out * 4.0;
+    }
+    PLAUNCH(K_SGD, 2.0 * off, bytes, s, launch_sgd(args, s));
+    return VFL_OK;
+}
+
+vfl_status wait_ev(vfl_ctx* ctx, cudaStream_t s, cudaEvent_t e) {
+    CK(cudaStreamWaitEvent(s, e, 0));
+    return VFL_OK;
+}
+
+#define TRY(x)                          \
+    do {                                \
+        vfl_status st_ = (x);           \
+        if (st_ != VFL_OK) return st_;  \
+    } while (0)
+
+// ---- the three phases ------------------------------------------------------
+vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
+    const vfl_config& c = ctx->cfg;
+    if (k != ctx->n_fwd) return ctx->fail(VFL_E_STATE, "passive_forward(%lld): next publish is step %lld", k, ctx->n_fwd);
+    if (tau_p < 0 || tau_p > c.staleness || tau_p > k)
+        return ctx->fail(VFL_E_STATE, "passive_forward(%lld): tau_p=%d outside [0, min(k, S=%d)]", k, tau_p, c.staleness);
+    const long long v = k - tau_p;
+    const long long u = ctx->n_bwd;  // passive updates enqueued
+    if (v > u)
+        return ctx->fail(VFL_E_STATE, "passive_forward(%lld): passive version %lld not produced yet (%lld updates)", k, v, u);
+    if (v < u - c.staleness)
+        return ctx->fail(VFL_E_STATE, "passive_forward(%lld): passive version %lld no longer stored", k, v);
+    cudaStream_t s = pstream(ctx, k);
+    const int slot = (int)(k % ctx->S1);
+    const int vslot = (int)(v % ctx->S1);
+    long long r0;
+    const int rows = ctx->batch_rows(k, &r0);
+    if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
+    const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+    long long ldx = ctx->ldxp;
+    for (size_t l = 0; l < ctx->P.size(); ++l) {
+        const Layer& L = ctx->P[l];
+        void* Y = ctx->act_p[slot][l];
+        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, Y, ld8(L.out), true, false, s));
+        X = Y;
+        ldx = ld8(L.out);
+    }
+    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)(k % ctx->nb), (int)v, s));
+    CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
+    ctx->fwd_version[slot] = (int)v;
+    ctx->slot_step_p[slot] = k;
+    ctx->n_fwd = k + 1;
+    ctx->started = true;
+    return VFL_OK;
+}
+
+vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
+    const vfl_config& c = ctx->cfg;
+    if (k != ctx->n_act) return ctx->fail(VFL_E_STATE, "active_step(%lld): next active step is %lld", k, ctx->n_act);
+    if (k >= ctx->n_fwd) return ctx->fail(VFL_E_STATE, "active_step(%lld): embedding not published yet", k);
+    if (tau_a < 0 || tau_a > c.staleness || tau_a > k)
+        return ctx->fail(VFL_E_STATE, "active_step(%lld): tau_a=%d outside [0, min(k, S=%d)]", k, tau_a, c.staleness);
+    const long long v = k - tau_a;
+    const int w = (int)(k % ctx->W);
+    cudaStream_t s = astream(ctx, k);
+    const int slot = (int)(k % ctx->S1);
+    const int vslot = (int)(v % ctx->S1);
+    const int es = ctx->esz;
+    long long r0;
+    const int rows = ctx->batch_rows(k, &r0);
+    const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size(), Lp = (int)ctx->P.size();
+    const int ea = ctx->A.back().out, ep = ctx->P.back().out;
+    const int n_out = ctx->T.back().out;
+
+    if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
+    // active bottom forward: z^a = f_a(x^a)
+    const void* Xa0 = static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * es;
+    const void* X = Xa0;
+    long long ldx = ctx->ldxa;
+    for (int l = 0; l < La; ++l) {
+        const Layer& L = ctx->A[l];
+        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, ctx->act_a[w][l], ld8(L.out), true, false, s));
+        X = ctx->act_a[w][l];
+        ldx = ld8(L.out);
+    }
+    // subscribe: wait for the embedding of step k, check its header
+    TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
+    PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->emb_hdr + slot, k, ctx->status, s));
+    const void* Za = ctx->act_a[w][La - 1];
+    const void* Zp = ctx->act_p[slot][Lp - 1];
+    // top forward on [z^a | z^p]
+    for (int l = 0; l < Lt; ++l) {
+        const Layer& L = ctx->T[l];
+        const bool last = l == Lt - 1;
+        void* Y = last ? (void*)ctx->logits[w] : ctx->act_t[w][l];
+        const long long ldy = last ? n_out : ld8(L.out);
+        if (l == 0)
+            TRY(linear_fwd(ctx, L, vslot, Za, ld8(ea), Zp, ld8(ep), ea, rows, Y, ldy, !last, last, s));
+        else
+            TRY(linear_fwd(ctx, L, vslot, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0, rows, Y, ldy,
+                           !last, last, s));
+    }
+    // loss and d(logits)
+    PLAUNCH(K_LOSS, 0, (double)rows * n_out * 8 + rows * 4.0, s,
+            launch_loss(ctx->logits[w], ctx->Y + r0, rows, n_out, c.loss, ctx->ds[w], ctx->losses + (k % kLossCap), s));
+    // top backward
+    const bool dp = c.dp_clip > 0.f;
+    for (int l = Lt - 1; l >= 0; --l) {
+        const Layer& L = ctx->T[l];
+        const bool last = l == Lt - 1;
+        const void* dpre = last ? (const void*)ctx->ds[w] : ctx->dpre_t[w][l];
+        const long long ldd = last ? n_out : ld8(L.out);
+        if (l == 0)
+            TRY(linear_dw(ctx, L, w, dpre, ldd, last, Za, ld8(ea), Zp, ld8(ep), ea, rows, s));
+        else
+            TRY(linear_dw(ctx, L, w, dpre, ldd, last, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0,
+                          rows, s));
+        if (l > 0) {
+            const long long ldo = ld8(ctx->T[l - 1].out);
+            TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_t[w][l - 1], ldo, ctx->act_t[w][l - 1],
+                          L.in, nullptr, 0, false, nullptr, s));
+        } else {
+            // split: dz^a (masked -> dpre of the active cut layer), dz^p -> gradient channel (or fp32 for DP)
+            void* C2 = dp ? (void*)ctx->dzp32[w] : ctx->grad[slot];
+            TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_a[w][La - 1], ld8(ea), Za, ea, C2,
+                          ld8(ep), dp, nullptr, s));
+        }
+    }
+    if (dp)
+        PLAUNCH(K_DP, 0, (double)rows * ep * (4 + ctx->esz), s,
+                launch_dp(ctx->dzp32[w], ld8(ep), ctx->grad[slot], ld8(ep), ctx->bf16, rows, ep, c.dp_clip,
+                          c.dp_sigma, c.dp_seed, k, s));
+    // publish the gradient
+    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)(k % ctx->nb), (int)v, s));
+    CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
+    ctx->grad_step[slot] = k;
+    // active bottom backward
+    for (int l = La - 1; l >= 0; --l) {
+        const Layer& L = ctx->A[l];
+        const void* Xin = l == 0 ? Xa0 : ctx->act_a[w][l - 1];
+        const long long ldin = l == 0 ? ctx->ldxa : ld8(ctx->A[l - 1].out);
+        TRY(linear_dw(ctx, L, w, ctx->dpre_a[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s));
+        if (l > 0) {
+            const long long ldo = ld8(ctx->A[l - 1].out);
+            TRY(linear_dx(ctx, L, vslot, ctx->dpre_a[w][l], ld8(L.out), false, rows, ctx->dpre_a[w][l - 1], ldo,
+                          ctx->act_a[w][l - 1], L.in, nullptr, 0, false, nullptr, s));
+        }
+    }
+    // SGD on theta_1 in step order: version k+1 from version k
+    if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+    TRY(sgd(ctx, &ctx->A, &ctx->T, w, (int)((k + 1) % ctx->S1), s));
+    CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
+    ctx->last_act_step[w] = k;
+    ctx->n_act = k + 1;
+    return VFL_OK;
+}
+
+vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
+    if (k != ctx->n_bwd) return ctx->fail(VFL_E_STATE, "passive_backward(%lld): next backward is %lld", k, ctx->n_bwd);
+    if (k >= ctx->n_act) return ctx->fail(VFL_E_STATE, "passive_backward(%lld): gradient not published yet", k);
+    const int w = (int)(k % ctx->W);
+    cudaStream_t s = pstream(ctx, k);
+    const int slot = (int)(k % ctx->S1);
+    const int vslot = ctx->fwd_version[slot] % ctx->S1;
+    long long r0;
+    const int rows = ctx->batch_rows(k, &r0);
+    const int Lp = (int)ctx->P.size();
+    const int ep = ctx->P.back().out;
+    TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
+    PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->grad_hdr + slot, k, ctx->status, s));
+    // dpre of the cut layer = dLoss/dz^p * [z^p > 0]
+    PLAUNCH(K_MASK, 0, 3.0 * rows * ep * ctx->esz, s,
+            launch_relu_mask(ctx->grad[slot], ctx->act_p[slot][Lp - 1], ctx->dpre_p[w][Lp - 1], ld8(ep), rows, ep,
+                             ctx->bf16, s));
+    const void* Xp0 = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+    for (int l = Lp - 1; l >= 0; --l) {
+        const Layer& L = ctx->P[l];
+        const void* Xin = l == 0 ? Xp0 : ctx->act_p[slot][l - 1];
+        const long long ldin = l == 0 ? ctx->ldxp : ld8(ctx->P[l - 1].out);
+        TRY(linear_dw(ctx, L, w, ctx->dpre_p[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s));
+        if (l > 0) {
+            const long long ldo = ld8(ctx->P[l - 1].out);
+            TRY(linear_dx(ctx, L, vslot, ctx->dpre_p[w][l], ld8(L.out), false, rows, ctx->dpre_p[w][l - 1], ldo,
+                          ctx->act_p[slot][l - 1], L.in, nullptr, 0, false, nullptr, s));
+        }
+    }
+    if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+    TRY(sgd(ctx, &ctx->P, nullptr, w, (int)((k + 1) % ctx->S1), s));
+    CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
+    ctx->n_bwd = k + 1;
+    return VFL_OK;
+}
+
+vfl_status read_status(vfl_ctx* ctx) {
+    int st = 0;
+    CK(cudaMemcpy(&st, ctx->status, sizeof(int), cudaMemcpyDeviceToHost));
+    if (st) {
+        CK(cudaMemset(ctx->status, 0, sizeof(int)));
+        if (st & ST_VERSION) return ctx->fail(VFL_E_VERSION, "a subscriber found a channel header of another step");
+        if (st & ST_TIMEOUT) return ctx->fail(VFL_E_TIMEOUT, "a bounded channel wait gave up");
+    }
+    return VFL_OK;
+}
+
+vfl_status sync_all(vfl_ctx* ctx) {
+    for (int w = 0; w < ctx->W; ++w) {
+        CK(cudaStreamSynchronize(ctx->ps[w]));
+        CK(cudaStreamSynchronize(ctx->as[w]));
+    }
+    return read_status(ctx);
+}
+
+Layer* find_layer(vfl_ctx* ctx, int party, int layer) {
+    std::vector<Layer>* v = party == 0 ? &ctx->P : party == 1 ? &ctx->A : party == 2 ? &ctx->T : nullptr;
+    if (!v || layer < 0 || layer >= (int)v->size()) return nullptr;
+    return &(*v)[layer];
+}
+
+}  // namespace
+
+// ============================================================================
+// C ABI
+// ============================================================================
+extern "C" {
+
+vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* bytes) {
+    std::string why;
+    if (!bytes) return VFL_E_INVAL;
+    vfl_status st = check_config(cfg, n_rows, &why);
+    if (st != VFL_OK) {
+        g_global_err = why;
+        return st;
+    }
+    vfl_ctx tmp;
+    tmp.cfg = *cfg;
+    tmp.n_rows = n_rows;
+    tmp.S1 = cfg->staleness + 1;
+    tmp.W = cfg->workers;
+    tmp.bf16 = cfg->dtype == VFL_BF16;
+    tmp.esz = tmp.bf16 ? 2 : 4;
+    build_layers(&tmp);
+    *bytes = carve_all(&tmp, nullptr);
+    return VFL_OK;
+}
+
+vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, uint64_t workspace_bytes,
+                      vfl_ctx** out) {
+    if (!out) return VFL_E_INVAL;
+    *out = nullptr;
+    std::string why;
+    vfl_status st = check_config(cfg, n_rows, &why);
+    if (st != VFL_OK) {
+        g_global_err = why;
+        return st;
+    }
+    if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255)) {
+        g_global_err = "workspace must be a non-null, 256-byte aligned device pointer";
+        return VFL_E_INVAL;
+    }
+    vfl_ctx* ctx = new vfl_ctx();
+    ctx->cfg = *cfg;
+    ctx->n_rows = n_rows;
+    ctx->S1 = cfg->staleness + 1;
+    ctx->W = cfg->workers;
+    ctx->bf16 = cfg->dtype == VFL_BF16;
+    ctx->esz = ctx->bf16 ? 2 : 4;
+    ctx->nb = (int)((n_rows + cfg->batch - 1) / cfg->batch);
+    for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
+    for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
+    build_layers(ctx);
+    const unsigned long long need = carve_all(ctx, nullptr);
+    if (workspace_bytes < need) {
+        g_global_err = "workspace too small: need " + std::to_string(need) + " bytes";
+        delete ctx;
+        return VFL_E_OOM;
+    }
+    carve_all(ctx, workspace);
+    ctx->ws_bytes = need;
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < kEvPool && e == cudaSuccess; ++i) {
+        e = cudaEventCreateWithFlags(&ctx->ev_pver[i], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_aver[i], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_emb[i], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_grad[i], cudaEventDisableTiming);
+    }
+    if (e == cudaSuccess) e = cudaMemset(workspace, 0, need);
+    if (e == cudaSuccess) e = cudaMemset(ctx->emb_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
+    if (e == cudaSuccess) e = cudaMemset(ctx->grad_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        g_global_err = std::string("vfl_create: ") + cudaGetErrorString(e);
+        vfl_destroy(ctx);
+        return VFL_E_CUDA;
+    }
+    *out = ctx;
+    return VFL_OK;
+}
+
+vfl_status vfl_destroy(vfl_ctx* ctx) {
+    if (!ctx) return VFL_OK;
+    if (!ctx->broken) {
+        for (int w = 0; w < ctx->W; ++w) {
+            cudaStreamSynchronize(ctx->ps[w]);
+            cudaStreamSynchronize(ctx->as[w]);
+        }
+    }
+    for (ProfRec& r : ctx->prof) {
+        ctx->ev_spare.push_back(r.e0);
+        ctx->ev_spare.push_back(r.e1);
+    }
+    for (cudaEvent_t e : ctx->ev_spare)
+        if (e) cudaEventDestroy(e);
+    for (int i = 0; i < kEvPool; ++i) {
+        if (ctx->ev_pver[i]) cudaEventDestroy(ctx->ev_pver[i]);
+        if (ctx->ev_aver[i]) cudaEventDestroy(ctx->ev_aver[i]);
+        if (ctx->ev_emb[i]) cudaEventDestroy(ctx->ev_emb[i]);
+        if (ctx->ev_grad[i]) cudaEventDestroy(ctx->ev_grad[i]);
+    }
+    delete ctx;
+    return VFL_OK;
+}
+
+vfl_status vfl_set_streams(vfl_ctx* ctx, int32_t n, void* const* streams) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (n != 2 * ctx->W || !streams) return ctx->fail(VFL_E_INVAL, "expected %d streams", 2 * ctx->W);
+    TRY(sync_all(ctx));
+    for (int w = 0; w < ctx->W; ++w) {
+        ctx->ps[w] = static_cast<cudaStream_t>(streams[w]);
+        ctx->as[w] = static_cast<cudaStream_t>(streams[ctx->W + w]);
+    }
+    return VFL_OK;
+}
+
+vfl_status vfl_load_data(vfl_ctx* ctx, const float* xp, const float* xa, const int32_t* y) {
+    if (!ctx || !xp || !xa || !y) return ctx ? ctx->fail(VFL_E_INVAL, "null data pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    TRY(sync_all(ctx));
+    const vfl_config& c = ctx->cfg;
+    const int n_out = ctx->T.back().out;
+    for (long long i = 0; i < ctx->n_rows; ++i) {
+        const int v = y[i];
+        if (v < 0 || v >= (c.loss == VFL_LOSS_BCE ? 2 : n_out))
+            return ctx->fail(VFL_E_INVAL, "label %d at row %lld outside the label range", v, i);
+    }
+    cudaStream_t s = ctx->ps[0];
+    for (long long r = 0; r < ctx->n_rows; r += c.batch) {
+        const int n = (int)std::min<long long>(c.batch, ctx->n_rows - r);
+        CK(cudaMemcpyAsync(ctx->stage_p[0], xp + r * c.d_passive, (size_t)n * c.d_passive * 4, cudaMemcpyHostToDevice, s));
+        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_p[0], n, c.d_passive,
+                                static_cast<char*>(ctx->Xp) + r * ctx->ldxp * ctx->esz, ctx->ldxp, ctx->bf16, s));
+        CK(cudaMemcpyAsync(ctx->stage_a[0], xa + r * c.d_active, (size_t)n * c.d_active * 4, cudaMemcpyHostToDevice, s));
+        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_a[0], n, c.d_active,
+                                static_cast<char*>(ctx->Xa) + r * ctx->ldxa * ctx->esz, ctx->ldxa, ctx->bf16, s));
+        CK(cudaStreamSynchronize(s));
+    }
+    CK(cudaMemcpy(ctx->Y, y, (size_t)ctx->n_rows * 4, cudaMemcpyHostToDevice));
+    return VFL_OK;
+}
+
+vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n, const float* xp, const float* xa,
+                          const int32_t* y) {
+    if (!ctx || !xp || !xa || !y) return ctx ? ctx->fail(VFL_E_INVAL, "null data pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    const vfl_config& c = ctx->cfg;
+    if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
+    if (row0 < 0 || n < 1 || n > c.batch || row0 + n > ctx->n_rows)
+        return ctx->fail(VFL_E_INVAL, "rows [%lld, %lld) invalid (at most one batch)", (long long)row0, (long long)(row0 + n));
+    cudaStream_t sp = ctx->ps[worker], sa = ctx->as[worker];
+    CK(cudaMemcpyAsync(ctx->stage_p[worker], xp, (size_t)n * c.d_passive * 4, cudaMemcpyHostToDevice, sp));
+    PLAUNCH(K_CAST, 0, n * c.d_passive * (4.0 + ctx->esz), sp, launch_cast_rows(ctx->stage_p[worker], (int)n, c.d_passive,
+                            static_cast<char*>(ctx->Xp) + row0 * ctx->ldxp * ctx->esz, ctx->ldxp, ctx->bf16, sp));
+    CK(cudaMemcpyAsync(ctx->stage_a[worker], xa, (size_t)n * c.d_active * 4, cudaMemcpyHostToDevice, sa));
+    PLAUNCH(K_CAST, 0, n * c.d_active * (4.0 + ctx->esz), sa, launch_cast_rows(ctx->stage_a[worker], (int)n, c.d_active,
+                            static_cast<char*>(ctx->Xa) + row0 * ctx->ldxa * ctx->esz, ctx->ldxa, ctx->bf16, sa));
+    CK(cudaMemcpyAsync(ctx->Y + row0, y, (size_t)n * 4, cudaMemcpyHostToDevice, sa));
+    return VFL_OK;
+}
+
+vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const float* W, const float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null parameter pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->started) return ctx->fail(VFL_E_STATE, "vfl_set_params after the first step");
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    TRY(sync_all(ctx));
+    const size_t nw = (size_t)L->out * L->in;
+    CK(cudaMemcpy(L->W, W, nw * 4, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(L->b, b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    // every version slot gets the same compute copy (padding columns stay zero)
+    for (int s = 0; s < ctx->S1; ++s) {
+        CK(cudaMemset(L->cW[s], 0, (size_t)L->out * L->in_ld * ctx->esz));
+        PLAUNCH(K_CAST, 0, 0, 0, launch_cast_rows(L->W, L->out, L->in, L->cW[s], L->in_ld, ctx->bf16, 0));
+        CK(cudaMemcpy(L->cb[s], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    }
+    CK(cudaDeviceSynchronize());
+    return VFL_OK;
+}
+
+vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null output pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    TRY(sync_all(ctx));
+    CK(cudaMemcpy(W, L->W, (size_t)L->out * L->in * 4, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(b, L->b, (size_t)L->out * 4, cudaMemcpyDeviceToHost));
+    return VFL_OK;
+}
+
+vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t worker, float* dW, float* db) {
+    if (!ctx || !dW || !db) return ctx ? ctx->fail(VFL_E_INVAL, "null output pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
+    TRY(sync_all(ctx));
+    const size_t nw = (size_t)L->out * L->in;
+    std::vector<float> pw((size_t)L->nsplit * nw), pb((size_t)L->nsplit * L->out);
+    CK(cudaMemcpy(pw.data(), L->pW[worker], pw.size() * 4, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(pb.data(), L->pb[worker], pb.size() * 4, cudaMemcpyDeviceToHost));
+    for (size_t i = 0; i < nw; ++i) {
+        float a = 0.f;
+        for (int z = 0; z < L->nsplit; ++z) a += pw[z * nw + i];
+        dW[i] = a;
+    }
+    for (int i = 0; i < L->out; ++i) {
+        float a = 0.f;
+        for (int z = 0; z < L->nsplit; ++z) a += pb[(size_t)z * L->out + i];
+        db[i] = a;
+    }
+    return VFL_OK;
+}
+
+vfl_status vfl_step_cursor(vfl_ctx* ctx, int64_t* k) {
+    if (!ctx || !k) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "steps in flight: %lld published, %lld active, %lld finished", ctx->n_fwd,
+                         ctx->n_act, ctx->n_bwd);
+    *k = ctx->n_bwd;
+    return VFL_OK;
+}
+
+vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (k < 0) return ctx->fail(VFL_E_INVAL, "cursor %lld < 0", (long long)k);
+    if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_set_cursor with steps in flight");
+    TRY(sync_all(ctx));
+    ctx->n_fwd = ctx->n_act = ctx->n_bwd = k;
+    for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
+    for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
+    ctx->started = true;
+    return VFL_OK;
+}
+
+vfl_status vfl_get_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, float* W, float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null output pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    int64_t k = 0;
+    TRY(vfl_step_cursor(ctx, &k));
+    if (v < std::max<int64_t>(0, k - ctx->cfg.staleness) || v > k)
+        return ctx->fail(VFL_E_INVAL, "version %lld is not stored (cursor %lld, S=%d)", (long long)v, (long long)k,
+                         ctx->cfg.staleness);
+    TRY(sync_all(ctx));
+    const int slot = (int)(v % ctx->S1);
+    ++ctx->launches;
+    CK(launch_to_f32(L->cW[slot], L->in_ld, L->out, L->in, ctx->bf16, ctx->scratch_f32, 0));
+    CK(cudaMemcpy(W, ctx->scratch_f32, (size_t)L->out * L->in * 4, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(b, L->cb[slot], (size_t)L->out * 4, cudaMemcpyDeviceToHost));
+    return VFL_OK;
+}
+
+vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, const float* W, const float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null parameter pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    int64_t k = 0;
+    TRY(vfl_step_cursor(ctx, &k));
+    if (v < std::max<int64_t>(0, k - ctx->cfg.staleness) || v > k)
+        return ctx->fail(VFL_E_INVAL, "version %lld cannot be stored (cursor %lld, S=%d)", (long long)v, (long long)k,
+                         ctx->cfg.staleness);
+    TRY(sync_all(ctx));
+    const int slot = (int)(v % ctx->S1);
+    const size_t nw = (size_t)L->out * L->in;
+    // stage through the master's storage when v is not the current version
+    float* tmp = ctx->scratch_f32;
+    CK(cudaMemcpy(tmp, W, nw * 4, cudaMemcpyHostToDevice));
+    CK(cudaMemset(L->cW[slot], 0, (size_t)L->out * L->in_ld * ctx->esz));
+    ++ctx->launches;
+    CK(launch_cast_rows(tmp, L->out, L->in, L->cW[slot], L->in_ld, ctx->bf16, 0));
+    CK(cudaMemcpy(L->cb[slot], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    if (v == k) {
+        CK(cudaMemcpy(L->W, W, nw * 4, cudaMemcpyHostToDevice));
+        CK(cudaMemcpy(L->b, b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    }
+    CK(cudaDeviceSynchronize());
+    return VFL_OK;
+}
+
+vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_steps, int32_t* tau_p,
+                             int32_t* tau_a) {
+    if (S < 0 || n_steps < 0 || (n_steps > 0 && (!tau_p || !tau_a))) {
+        g_global_err = "vfl_make_schedule: invalid argument";
+        return VFL_E_INVAL;
+    }
+    if (kind != VFL_SCHED_SYNC && kind != VFL_SCHED_MAX && kind != VFL_SCHED_SEEDED) {
+        g_global_err = "vfl_make_schedule: unknown kind";
+        return VFL_E_INVAL;
+    }
+    const uint32_t k0 = (uint32_t)(seed & 0xFFFFFFFFu), k1 = (uint32_t)(seed >> 32);
+    for (int party = 0; party < 2; ++party) {
+        int32_t* tau = party == 0 ? tau_p : tau_a;
+        int32_t prev = 0;
+        for (int64_t k = 0; k < n_steps; ++k) {
+            int32_t t = 0;
+            if (kind == VFL_SCHED_MAX) {
+                t = (int32_t)std::min<int64_t>(k, S);
+            } else if (kind == VFL_SCHED_SEEDED && k > 0) {
+                // Philox4x32-10, counter (k lo, k hi, party, 0x5343), key (seed lo, seed hi); word 0
+                uint32_t c[4] = {(uint32_t)(k & 0xFFFFFFFFu), (uint32_t)((uint64_t)k >> 32), (uint32_t)party, 0x5343u};
+                uint32_t key[2] = {k0, k1};
+                for (int r = 0; r < 10; ++r) {
+                    const uint64_t p0 = (uint64_t)0xD2511F53u * c[0];
+                    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c[2];
+                    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ key[0];
+                    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ key[1];
+                    c[0] = n0;
+                    c[1] = (uint32_t)p1;
+                    c[2] = n2;
+                    c[3] = (uint32_t)p0;
+                    key[0] += 0x9E3779B9u;
+                    key[1] += 0xBB67AE85u;
+                }
+                const int64_t u = (int64_t)(c[0] % (uint32_t)(S + 1));
+                t = (int32_t)std::min<int64_t>(std::min<int64_t>(k, S), std::min<int64_t>(prev + 1, u));
+            }
+            tau[k] = t;
+            prev = t;
+        }
+    }
+    return VFL_OK;
+}
+
+vfl_status vfl_passive_forward(vfl_ctx* ctx, int64_t k, int32_t tau_p) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    return do_passive_forward(ctx, k, tau_p);
+}
+
+vfl_status vfl_active_step(vfl_ctx* ctx, int64_t k, int32_t tau_a) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    return do_active_step(ctx, k, tau_a);
+}
+
+vfl_status vfl_passive_backward(vfl_ctx* ctx, int64_t k) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    return do_passive_backward(ctx, k);
+}
+
+vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (n_steps < 0 || (n_steps > 0 && (!tau_p || !tau_a))) return ctx->fail(VFL_E_INVAL, "invalid schedule arguments");
+    if (k0 != ctx->n_fwd || k0 != ctx->n_act || k0 != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_train_steps(%lld): steps before k0 are not all complete", (long long)k0);
+    const long long end = k0 + n_steps;
+    // Emit each phase as early as its inputs allow, so the publisher of step k+1
+    // is queued ahead of the backward of step k whenever tau_p permits.
+    while (ctx->n_bwd < end) {
+        bool progressed = false;
+        while (ctx->n_fwd < end && ctx->n_fwd - tau_p[ctx->n_fwd] <= ctx->n_bwd) {
+            TRY(do_passive_forward(ctx, ctx->n_fwd, tau_p[ctx->n_fwd]));
+            progressed = true;
+        }
+        while (ctx->n_act < ctx->n_fwd) {
+            TRY(do_active_step(ctx, ctx->n_act, tau_a[ctx->n_act]));
+            progressed = true;
+        }
+        if (ctx->n_bwd < ctx->n_act) {
+            TRY(do_passive_backward(ctx, ctx->n_bwd));
+            progressed = true;
+        }
+        if (!progressed) return ctx->fail(VFL_E_STATE, "schedule cannot make progress at step %lld", ctx->n_bwd);
+    }
+    return VFL_OK;
+}
+
+vfl_status vfl_synchronize(vfl_ctx* ctx) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    return sync_all(ctx);
+}
+
+vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out) {
+    if (!ctx || (n > 0 && !out)) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (k0 < 0 || n < 0 || k0 + n > ctx->n_act || k0 < ctx->n_act - kLossCap)
+        return ctx->fail(VFL_E_INVAL, "losses of steps [%lld, %lld) are not stored", (long long)k0, (long long)(k0 + n));
+    TRY(sync_all(ctx));
+    for (int64_t i = 0; i < n; ++i) {
+        CK(cudaMemcpy(out + i, ctx->losses + ((k0 + i) % kLossCap), 4, cudaMemcpyDeviceToHost));
+    }
+    return VFL_OK;
+}
+
+vfl_status vfl_fetch_loss(vfl_ctx* ctx, int64_t k, float* host_out) {
+    if (!ctx || !host_out) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (k < 0 || k >= ctx->n_act || k < ctx->n_act - kLossCap)
+        return ctx->fail(VFL_E_INVAL, "loss of step %lld is not stored", (long long)k);
+    CK(cudaMemcpyAsync(host_out, ctx->losses + (k % kLossCap), 4, cudaMemcpyDeviceToHost, astream(ctx, k)));
+    return VFL_OK;
+}
+
+vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out) {
+    if (!ctx || !out) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    TRY(sync_all(ctx));
+    long long r0;
+    const int rows = ctx->batch_rows(k, &r0);
+    const int slot = (int)(k % ctx->S1);
+    const int w = (int)(k % ctx->W);
+    const void* src = nullptr;
+    long long ld = 0;
+    int cols = 0, bf = ctx->bf16;
+    const int ep = ctx->P.back().out, ea = ctx->A.back().out;
+    switch (what) {
+        case VFL_TAP_EMB:
+            if (ctx->slot_step_p[slot] != k) return ctx->fail(VFL_E_STATE, "embedding of step %lld is not stored", (long long)k);
+            src = ctx->act_p[slot].back(); ld = ld8(ep); cols = ep;
+            break;
+        case VFL_TAP_GRAD:
+            if (ctx->grad_step[slot] != k) return ctx->fail(VFL_E_STATE, "gradient of step %lld is not stored", (long long)k);
+            src = ctx->grad[slot]; ld = ld8(ep); cols = ep;
+            break;
+        case VFL_TAP_LOGITS:
+        case VFL_TAP_ZA:
+        case VFL_TAP_DZA:
+            if (ctx->last_act_step[w] != k) return ctx->fail(VFL_E_STATE, "active buffers of step %lld are not stored", (long long)k);
+            if (what == VFL_TAP_LOGITS) { src = ctx->logits[w]; ld = ctx->T.back().out; cols = (int)ld; bf = 0; }
+            else if (what == VFL_TAP_ZA) { src = ctx->act_a[w].back(); ld = ld8(ea); cols = ea; }
+            else { src = ctx->dpre_a[w].back(); ld = ld8(ea); cols = ea; }
+            break;
+        default:
+            return ctx->fail(VFL_E_INVAL, "unknown tap %d", what);
+    }
+    ++ctx->launches;
+    CK(launch_to_f32(src, ld, rows, cols, bf, ctx->scratch_f32, 0));
+    CK(cudaMemcpy(out, ctx->scratch_f32, (size_t)rows * cols * 4, cudaMemcpyDeviceToHost));
+    return VFL_OK;
+}
+
+vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_iters) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if ((which != 0 && which != 1) || k < 0 || max_iters < 1 || max_iters > (1ll << 24))
+        return ctx->fail(VFL_E_INVAL, "invalid wait arguments");
+    TRY(sync_all(ctx));
+    const ChannelHeader* h = (which == 0 ? ctx->emb_hdr : ctx->grad_hdr) + (k % ctx->S1);
+    PLAUNCH(K_HEADER, 0, 0, ctx->ps[0], launch_wait_header(h, k, max_iters, ctx->status, ctx->ps[0]));
+    return sync_all(ctx);
+}
+
+int64_t vfl_kernel_launches(const vfl_ctx* ctx) { return ctx ? ctx->launches : 0; }
+
+vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (enable) {
+        for (ProfAgg& a : ctx->agg) a = ProfAgg();
+        ctx->prof.clear();
+        ctx->prof_on = true;
+        return VFL_OK;
+    }
+    if (!ctx->prof_on) return VFL_OK;
+    ctx->prof_on = false;
+    TRY(sync_all(ctx));
+    for (ProfRec& r : ctx->prof) {
+        float ms = 0.f;
+        CK(cudaEventElapsedTime(&ms, r.e0, r.e1));
+        ProfAgg& a = ctx->agg[r.cls];
+        a.n += 1;
+        a.ms += ms;
+        a.flops += r.flops;
+        a.bytes += r.bytes;
+        ctx->ev_spare.push_back(r.e0);
+        ctx->ev_spare.push_back(r.e1);
+    }
+    ctx->prof.clear();
+    return VFL_OK;
+}
+
+vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
+                           double* bytes) {
+    if (!ctx || cls < 0 || cls >= K_NCLASS || !launches || !ms || !flops || !bytes) return VFL_E_INVAL;
+    const ProfAgg& a = ctx->agg[cls];
+    *launches = a.n;
+    *ms = a.ms;
+    *flops = a.flops;
+    *bytes = a.bytes;
+    return VFL_OK;
+}
+
+const char* vfl_kernel_class_name(int32_t cls) { return cls >= 0 && cls < K_NCLASS ? kClassNames[cls] : nullptr; }
+
+const char* vfl_last_error(const vfl_ctx* ctx) { return ctx ? ctx->err.c_str() : g_global_err.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+"""Shared helpers of the GPU parity tests: run the same seeded inputs through
+the C ABI and through the oracle and compare."""
+import numpy as np
+
+import oracle
+import synth
+
+# Tolerances (relative, infinity norm): fp32 path 1e-5 per step and 1e-3 on
+# the epoch loss; bf16 path 2e-2 per step.
+TOL = {"fp32": 1e-5, "bf16": 2e-2}
+EPOCH_LOSS_TOL = 1e-3
+
+
+def rel_err(got, ref):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    if ref.size == 0:
+        return 0.0
+    return float(np.abs(got - ref).max() / max(np.abs(ref).max(), 1e-30))
+
+
+def schedule(p, n_steps):
+    kind = oracle.SCHED_SYNC if p.schedule == "sync" else oracle.SCHED_SEEDED
+    return oracle.make_schedule(p.seed, p.staleness, kind, n_steps)
+
+
+def setup(p, n_rows=None, rows=None):
+    """(preset with n_rows, xp, xa, y, params) for the first n_rows rows of the workload."""
+    n_rows = n_rows or p.n_rows
+    xp, xa, y = synth.make_dataset(p, rows=(0, n_rows)) if rows is None else rows
+    q = p.with_(n_rows=n_rows)
+    return q, xp, xa, y, synth.init_params(q)
+
+
+def new_context(vfl, q, xp, xa, y, params):
+    ctx = vfl.Context(q, q.n_rows)
+    ctx.load_data(xp, xa, y)
+    ctx.set_params(params)
+    return ctx
+
+
+def tensor_err(got, ref, dtype):
+    """Error of one tensor against the oracle, in the metric of its dtype.
+
+    fp32: relative infinity norm.  bf16: relative Frobenius norm, reported as
+    failing outright (1.0) when more than 1 % of the rows hold an element off by
+    more than 2e-2 of the tensor's largest magnitude.  Rows that differ are the
+    ones where a pre-activation within rounding distance of zero takes the other
+    ReLU branch; bf16 rounding upstream makes that happen in a few rows per
+    step, and a whole row's downstream gradient then moves."""
+    if dtype == "fp32":
+        return rel_err(got, ref)
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    if ref.size == 0:
+        return 0.0
+    fro = float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30))
+    d = np.abs(got - ref) > TOL["bf16"] * max(np.abs(ref).max(), 1e-30)
+    rows_off = d.reshape(d.shape[0], -1).any(axis=1).mean() if d.ndim > 1 else d.mean()
+    return fro if rows_off <= 0.01 else 1.0
+
+
+def compare_step(vfl, ctx, rec, tol, check_grads=True):
+    """Per-step taps, gradients and updated parameters against an oracle record."""
+    k = rec.k
+    dt = ctx.p.dtype
+    errs = {
+        "zp": tensor_err(ctx.tap(k, vfl.TAP_EMB), rec.zp, dt),
+        "dzp": tensor_err(ctx.tap(k, vfl.TAP_GRAD), rec.dzp, dt),
+        "logits": tensor_err(ctx.tap(k, vfl.TAP_LOGITS), rec.logits, dt),
+        "za": tensor_err(ctx.tap(k, vfl.TAP_ZA), rec.za, dt),
+        "dza": tensor_err(ctx.tap(k, vfl.TAP_DZA), rec.dza * (rec.za > 0), dt),
+    }
+    loss = ctx.read_losses(k, 1)[0]
+    errs["loss"] = abs(loss - rec.loss) / max(abs(rec.loss), 1e-30)
+    if check_grads:
+        g = ctx.get_grads(worker=k % ctx.p.workers)
+        for key, (dW, db) in g.items():
+            errs[f"dW{key}"] = tensor_err(dW, rec.grads[key][0], dt)
+            errs[f"db{key}"] = tensor_err(db, rec.grads[key][1], dt)
+    params = ctx.get_params()
+    for key, (W, b) in params.items():
+        errs[f"W{key}"] = tensor_err(W, rec.params[key][0], dt)
+        errs[f"b{key}"] = tensor_err(b, rec.params[key][1], dt)
+    bad = {name: e for name, e in errs.items() if not e <= tol}
+    return errs, bad

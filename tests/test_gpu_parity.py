@@ -1,0 +1,173 @@
+"""GPU parity: the CUDA path through the C ABI against the oracle, on the same
+seeded inputs, step by step (taps, gradients, updated weights) and over whole
+epochs.  fp32 presets within 1e-5 per step and 1e-3 on the epoch loss; bf16
+presets within 2e-2 per step."""
+import numpy as np
+import pytest
+
+import oracle
+from _parity import EPOCH_LOSS_TOL, TOL, compare_step, new_context, rel_err, schedule, setup
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def vfl():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2510_12494_gb300 import build
+    build.build()
+    import paper_2510_12494_gb300 as v
+    return v
+
+
+# Rows per preset: at least two full batches plus a ragged last batch, with the
+# full per-step shapes (batch, layer widths) of each workload.
+CASES = {
+    1: 4096 - 100,            # 16 steps, last batch 156 rows
+    2: 2 * 1024 + 304,        # full batch 1024 and the 304-row tail of the 30000-row set
+    3: 2 * 4096 + 288,
+    4: 8192 + 576,
+    5: 2 * 2048 + 1344,
+}
+
+
+def oracle_version(o, v):
+    """{(party, layer): (W, b)} of the oracle's stored weight version v."""
+    out = {}
+    for l, (W, b) in enumerate(o.versions_p[v]):
+        out[(0, l)] = (W, b)
+    A, T = o.versions_a[v]
+    for l, (W, b) in enumerate(A):
+        out[(1, l)] = (W, b)
+    for l, (W, b) in enumerate(T):
+        out[(2, l)] = (W, b)
+    return out
+
+
+def force_gpu_state(ctx, o, S):
+    """Put the GPU context into the oracle's state before step o.k: cursor and
+    every stored weight version (oracle -> GPU only)."""
+    k = o.k
+    ctx.set_cursor(k)
+    for v in range(max(0, k - S), k + 1):
+        ctx.set_version(v, oracle_version(o, v))
+
+
+def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None):
+    """Step-by-step comparison.  bf16 presets are teacher-forced: before each
+    step the GPU takes the oracle's weight versions, so one step's error is
+    measured without the drift of earlier roundings (a bf16 weight copy that
+    rounds the other way moves later ReLU masks)."""
+    import synth
+    p = synth.preset(cid)
+    q, xp, xa, y, params = setup(p, n_rows)
+    nb = -(-n_rows // q.batch)
+    steps = steps or nb + 2                      # one epoch and two steps of the next
+    if teacher_forced is None:
+        teacher_forced = q.dtype == "bf16"
+    tp, ta = schedule(q, steps)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
+    worst = {}
+    failures = []
+    for k in range(steps):
+        if teacher_forced and k > 0:
+            force_gpu_state(ctx, o, q.staleness)
+        rec = o.step(int(tp[k]), int(ta[k]), record=True)
+        ctx.passive_forward(k, int(tp[k]))
+        ctx.active_step(k, int(ta[k]))
+        ctx.passive_backward(k)
+        errs, bad = compare_step(vfl, ctx, rec, TOL[q.dtype])
+        for name, e in errs.items():
+            worst[name] = max(worst.get(name, 0.0), e)
+        if bad:
+            failures.append((k, bad))
+    return worst, failures
+
+
+@pytest.mark.parametrize("cid", [1, 2, 3, 4, 5])
+def test_step_parity(vfl, cid):
+    worst, failures = run_sequential(vfl, cid, CASES[cid])
+    assert not failures, f"preset {cid}: {failures[:3]}; worst {sorted(worst.items(), key=lambda t: -t[1])[:6]}"
+
+
+@pytest.mark.parametrize("cid", [1, 2])
+def test_fp32_epoch_loss_and_dag_equals_sequential(vfl, cid):
+    """The whole-DAG enqueue (vfl_train_steps, parties overlapping on their
+    streams) gives exactly the result of phase-by-phase execution, and the
+    full-size fp32 workloads match the oracle's epoch losses within 1e-3."""
+    import synth
+    p = synth.preset(cid)
+    q, xp, xa, y, params = setup(p)
+    n_steps = q.steps_per_epoch * q.epochs
+    tp, ta = schedule(q, n_steps)
+    dag = new_context(vfl, q, xp, xa, y, params)
+    dag.train_steps(0, n_steps, tp, ta)
+    losses = dag.read_losses(0, n_steps)
+    o = oracle.Oracle(q, xp, xa, y, params)
+    ref, _ = o.run(tp, ta, n_steps)
+    nb = q.steps_per_epoch
+    for e in range(q.epochs):
+        got = o.epoch_loss(losses[e * nb:(e + 1) * nb], e * nb)
+        want = o.epoch_loss(ref[e * nb:(e + 1) * nb], e * nb)
+        assert abs(got - want) <= EPOCH_LOSS_TOL * abs(want), (e, got, want)
+    gp = dag.get_params()
+    for key, (W, b) in gp.items():
+        assert rel_err(W, o.current_params()[key][0]) < 1e-3
+    # sequential phase-by-phase run of the first epoch: identical bits
+    seq = new_context(vfl, q, xp, xa, y, params)
+    for k in range(nb):
+        seq.passive_forward(k, int(tp[k]))
+        seq.active_step(k, int(ta[k]))
+        seq.passive_backward(k)
+    dag2 = new_context(vfl, q, xp, xa, y, params)
+    dag2.train_steps(0, nb, tp, ta)
+    np.testing.assert_array_equal(seq.read_losses(0, nb), dag2.read_losses(0, nb))
+    for key, (W, b) in seq.get_params().items():
+        W2, b2 = dag2.get_params()[key]
+        np.testing.assert_array_equal(W, W2)
+        np.testing.assert_array_equal(b, b2)
+
+
+@pytest.mark.parametrize("cid", [3, 5])
+def test_bf16_free_running_epoch_loss(vfl, cid):
+    """Without teacher forcing, a whole bf16 epoch stays within 2e-2 of the
+    oracle's per-step losses and weights."""
+    import synth
+    p = synth.preset(cid)
+    q, xp, xa, y, params = setup(p, CASES[cid])
+    n = q.steps_per_epoch + 1
+    tp, ta = schedule(q, n)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    ctx.train_steps(0, n, tp, ta)
+    o = oracle.Oracle(q, xp, xa, y, params)
+    ref, _ = o.run(tp, ta, n)
+    got = ctx.read_losses(0, n)
+    assert np.abs(got - ref).max() <= TOL["bf16"] * np.abs(ref).max()
+    for key, (W, b) in ctx.get_params().items():
+        assert rel_err(W, o.current_params()[key][0]) < TOL["bf16"]
+
+
+@pytest.mark.parametrize("cid", [2, 5])
+def test_checkpoint_restore_is_bit_exact(vfl, cid):
+    """Train k1 steps, checkpoint, restore into a fresh context, continue: the
+    result equals an uninterrupted run bit for bit."""
+    import synth
+    p = synth.preset(cid)
+    q, xp, xa, y, params = setup(p, CASES[cid] if cid != 2 else 4 * 1024 + 304)
+    n1, n2 = 3, 4
+    tp, ta = schedule(q, n1 + n2)
+    a = new_context(vfl, q, xp, xa, y, params)
+    a.train_steps(0, n1, tp, ta)
+    ck = a.checkpoint()
+    a.train_steps(n1, n2, tp, ta)
+    b = new_context(vfl, q, xp, xa, y, params)
+    b.restore(ck)
+    b.train_steps(n1, n2, tp, ta)
+    np.testing.assert_array_equal(a.read_losses(n1, n2), b.read_losses(n1, n2))
+    pa, pb = a.get_params(), b.get_params()
+    for key in pa:
+        np.testing.assert_array_equal(pa[key][0], pb[key][0])
+        np.testing.assert_array_equal(pa[key][1], pb[key][1])
