@@ -241,6 +241,36 @@ vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, d
                            double* bytes);
 const char* vfl_kernel_class_name(int32_t cls);
 
+/*
+ * Weight gradient of one Linear layer without any allocation (the paper has no
+ * counterpart; this is a convenience for restricted callers).
+ *
+ * Some callers cannot allocate device memory when they need a gradient: code
+ * running inside an allocator or memory-pool callback, a host that has fixed
+ * the process's device footprint in advance, or a process whose pools already
+ * hold all of HBM.  This call needs no workspace: its split-K partial sums live
+ * in a fixed 16 MiB array inside the library (every GPU that loads the library
+ * holds it until the process exits), and it calls no cudaMalloc, cudaFree or
+ * other allocating routine.
+ *
+ *   dpre  device [rows, out] row-major: gradient of the layer's pre-activation
+ *   x     device [rows, in]  row-major: the layer's input
+ *         (both float for dtype VFL_FP32, bf16 for VFL_BF16)
+ *   dW    device [out, in] fp32 output: dpre^T x
+ *   db    device [out] fp32 output: column sums of dpre
+ *   stream  cudaStream_t to enqueue on (NULL: legacy default stream); the call
+ *         returns before the work finishes.
+ *
+ * Limit: out*in + out <= 4,194,304; larger layers get VFL_E_INVAL with the
+ * reason in vfl_last_error(NULL).  The first call on a device looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture.  All calls share the array and it keeps the last call's
+ * partial sums (each call overwrites everything it reads, so nothing needs
+ * clearing); calls that can overlap on the GPU race on it, so serialize them.
+ */
+vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, int32_t rows, int32_t out, int32_t in,
+                                   int32_t dtype, float* dW, float* db, void* stream);
+
 /* Last error message of the context (or of the last failed vfl_create / vfl_make_schedule when ctx is NULL). */
 const char* vfl_last_error(const vfl_ctx* ctx);
 

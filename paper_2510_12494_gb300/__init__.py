@@ -87,6 +87,9 @@ EXPORTS = {
                                          ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
                                          ctypes.POINTER(ctypes.c_double)]),
     "vfl_kernel_class_name": (ctypes.c_char_p, [ctypes.c_int32]),
+    "vfl_weight_grad_noalloc": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                                 ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
+                                                 ctypes.c_void_p]),
     "vfl_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
 }
 
@@ -147,6 +150,20 @@ def make_schedule(seed: int, S: int, kind: int, n_steps: int):
     ta = np.zeros(max(n_steps, 1), np.int32)
     _check(lib().vfl_make_schedule(seed, S, kind, n_steps, _ptr(tp), _ptr(ta)))
     return tp[:n_steps], ta[:n_steps]
+
+
+def weight_grad_noalloc(dpre, x, dW, db, dtype: int, stream=None):
+    """dW = dpre^T x and db = column sums of dpre on device tensors (dpre [rows,
+    out], x [rows, in], dW [out, in] fp32, db [out] fp32), using the library's
+    fixed scratch instead of any allocation.  Enqueued on ``stream`` (a
+    torch.cuda.Stream; default: the current stream)."""
+    import torch
+    rows, out = dpre.shape
+    assert x.shape[0] == rows and dW.shape == (out, x.shape[1]) and db.shape == (out,)
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _check(lib().vfl_weight_grad_noalloc(ctypes.c_void_p(dpre.data_ptr()), ctypes.c_void_p(x.data_ptr()), rows, out,
+                                         x.shape[1], dtype, ctypes.c_void_p(dW.data_ptr()),
+                                         ctypes.c_void_p(db.data_ptr()), ctypes.c_void_p(s.cuda_stream)))
 
 
 def workspace_bytes(p, n_rows: int) -> int:

@@ -706,6 +706,10 @@ Layer* find_layer(vfl_ctx* ctx, int party, int layer) {
 
 }  // namespace
 
+namespace vfl {
+void set_global_error(const char* msg) { g_global_err = msg; }
+}  // namespace vfl
+
 // ============================================================================
 // C ABI
 // ============================================================================
