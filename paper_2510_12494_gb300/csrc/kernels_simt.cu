@@ -306,6 +306,15 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
     }
 }
 
+__global__ void transpose_f32_kernel(const float* __restrict__ src, int out, int in, float* __restrict__ dst,
+                                     long long ldt) {
+    const long long n = (long long)out * in;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const long long o = i / in, k = i % in;
+        dst[k * ldt + o] = src[i];
+    }
+}
+
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
     const long long n = (long long)rows * cols;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
@@ -388,6 +397,11 @@ cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long ma
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     cast_rows_kernel<<<grid_for((long long)rows * ld, 256), 256, 0, s>>>(src, rows, d, dst, ld, bf16);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s) {
+    transpose_f32_kernel<<<grid_for((long long)out * in, 256), 256, 0, s>>>(src, out, in, dst, ldt);
     return cudaGetLastError();
 }
 

@@ -90,6 +90,9 @@ cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,
                                cudaStream_t s);
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s);
+// dst[k * ldt + o] = src[o * in + k] for src [out, in] fp32.
+cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s);
+
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);
 

@@ -14,10 +14,12 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
 
+#include "vfl_fused.cuh"
 #include "vfl_kernels.cuh"
 #include "vfl_tc.cuh"
 
@@ -35,11 +37,13 @@ thread_local std::string g_global_err;
 // Kernel classes for launch accounting and per-class CUDA-event timing.
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
-    K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST, K_NCLASS
+    K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
-    "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast"};
+    "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd"};
 
 struct ProfRec {
     int cls;
@@ -60,6 +64,7 @@ struct Layer {
     float* b = nullptr;                   // fp32 master [out]
     void* cW[kMaxSlots] = {};             // version copies [out, in_ld], compute dtype
     float* cb[kMaxSlots] = {};            // version copies of b, fp32
+    float* cWt[kMaxSlots] = {};           // fused path: transposed version copies [in, ld8(out)], fp32
     float* pW[kMaxWorkers] = {};          // split-K partial dW [nsplit][out*in]
     float* pb[kMaxWorkers] = {};          // partial db [nsplit][out]
     int nsplit = 1;
@@ -114,6 +119,16 @@ struct vfl_ctx {
     int* status = nullptr;
     float* scratch_f32 = nullptr;       // for taps [B * max width]
     unsigned long long ws_bytes = 0;
+
+    // fused one-launch-per-phase path (narrow fp32 models)
+    bool fused = false;
+    int f_act_ld = 0, f_wp = 0, f_wa = 0;       // smem row stride, weight-stage floats per party
+    long long f_ptotal_p = 0, f_ptotal_a = 0;   // flat parameter counts
+    float* f_part_p = nullptr;                  // [tiles][ptotal_p]
+    float* f_part_a = nullptr;                  // [tiles][ptotal_a]
+    float* f_rowloss = nullptr;                 // [B]
+    int* f_counter = nullptr;
+    int f_grid_a = 1, f_grid_p = 1;
 
     // streams / events
     cudaStream_t ps[kMaxWorkers] = {};
@@ -250,6 +265,40 @@ void choose_split(Layer& L, int B) {
     L.nsplit = (B + L.kchunk - 1) / L.kchunk;
 }
 
+// The fused path serves fp32 models whose every width fits one shared-memory
+// row tile, with one worker stream per party and no DP.
+bool fused_eligible(const vfl_config& c) {
+    if (c.dtype != VFL_FP32 || c.workers != 1 || c.dp_clip > 0.f) return false;
+    if (c.d_passive > kFusedMaxWidth || c.d_active > kFusedMaxWidth) return false;
+    for (int i = 0; i < c.n_passive; ++i) if (c.passive_out[i] > kFusedMaxWidth) return false;
+    for (int i = 0; i < c.n_active; ++i) if (c.active_out[i] > kFusedMaxWidth) return false;
+    for (int i = 0; i < c.n_top; ++i) if (c.top_out[i] > kFusedMaxWidth) return false;
+    if (c.active_out[c.n_active - 1] + c.passive_out[c.n_passive - 1] > kFusedMaxWidth) return false;
+    if (c.n_active + c.n_top > kFusedMaxLayers) return false;
+    // the embeddings are copied into the top's input tile with 16-byte copies
+    if (c.active_out[c.n_active - 1] % 4 != 0 || c.passive_out[c.n_passive - 1] % 4 != 0) return false;
+    return true;
+}
+
+// Shared-memory layout of one fused launch: which layers stage W (for input
+// gradients) and W^T (for the forward).  Returns the floats used.
+int fused_weight_layout(FusedLayerArgs* L, int n, bool want_wt, int w_from, int w_layer0) {
+    int off = 0;
+    for (int l = 0; l < n; ++l) {
+        L[l].wts_off = -1;
+        L[l].ws_off = -1;
+        if (want_wt) {
+            L[l].wts_off = off;
+            off += (int)(L[l].in * L[l].out_ld);
+        }
+        if (l >= w_from && (l > 0 || w_layer0)) {
+            L[l].ws_off = off;
+            off += (int)(L[l].out * L[l].in_ld);
+        }
+    }
+    return off;
+}
+
 void build_layers(vfl_ctx* ctx) {
     const vfl_config& c = ctx->cfg;
     auto mk = [&](std::vector<Layer>& v, int party, int n, const int32_t* outs, int d_in) {
@@ -262,6 +311,10 @@ void build_layers(vfl_ctx* ctx) {
             L.out = outs[l];
             L.in_ld = ld8(d_in);
             choose_split(L, c.batch);
+            if (ctx->fused) {
+                L.nsplit = 1;
+                L.kchunk = c.batch;
+            }
             v.push_back(L);
             d_in = outs[l];
         }
@@ -269,6 +322,42 @@ void build_layers(vfl_ctx* ctx) {
     mk(ctx->P, 0, c.n_passive, c.passive_out, c.d_passive);
     mk(ctx->A, 1, c.n_active, c.active_out, c.d_active);
     mk(ctx->T, 2, c.n_top, c.top_out, c.active_out[c.n_active - 1] + c.passive_out[c.n_passive - 1]);
+    if (ctx->fused) {
+        int maxw = std::max(c.d_passive, c.d_active);
+        ctx->f_wp = ctx->f_wa = 0;
+        ctx->f_ptotal_p = ctx->f_ptotal_a = 0;
+        for (const Layer& L : ctx->P) {
+            maxw = std::max(maxw, std::max(L.in, L.out));
+            ctx->f_ptotal_p += (long long)L.out * L.in + L.out;
+        }
+        for (auto* v : {&ctx->A, &ctx->T})
+            for (const Layer& L : *v) {
+                maxw = std::max(maxw, std::max(L.in, L.out));
+                ctx->f_ptotal_a += (long long)L.out * L.in + L.out;
+            }
+        ctx->f_act_ld = (int)ld8(maxw);
+        // staged weights per launch: forward W^T of every layer; input-gradient W of every top layer and
+        // of every bottom layer but the first
+        long long wt_p = 0, w_p = 0, wt_a = 0, w_a = 0;
+        for (size_t l = 0; l < ctx->P.size(); ++l) {
+            wt_p += (long long)ctx->P[l].in * ld8(ctx->P[l].out);
+            if (l > 0) w_p += (long long)ctx->P[l].out * ctx->P[l].in_ld;
+        }
+        for (size_t l = 0; l < ctx->A.size(); ++l) {
+            wt_a += (long long)ctx->A[l].in * ld8(ctx->A[l].out);
+            if (l > 0) w_a += (long long)ctx->A[l].out * ctx->A[l].in_ld;
+        }
+        for (const Layer& L : ctx->T) {
+            wt_a += (long long)L.in * ld8(L.out);
+            w_a += (long long)L.out * L.in_ld;
+        }
+        ctx->f_wp = (int)std::max(wt_p, w_p);
+        ctx->f_wa = (int)(wt_a + w_a);
+        const size_t sa = fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size());
+        const size_t sp = fused_smem_pbwd((int)w_p, ctx->f_act_ld, (int)ctx->P.size());
+        const size_t sf = fused_smem_fwd((int)wt_p, ctx->f_act_ld);
+        if (std::max(sa, std::max(sp, sf)) > kFusedMaxSmem) ctx->fused = false;
+    }
 }
 
 // Lay out every device buffer; with base == nullptr only measures.
@@ -293,6 +382,7 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             for (int s = 0; s < ctx->S1; ++s) {
                 L.cW[s] = cv.take((unsigned long long)L.out * L.in_ld * es);
                 L.cb[s] = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
+                if (ctx->fused) L.cWt[s] = static_cast<float*>(cv.take((unsigned long long)L.in * ld8(L.out) * 4));
             }
             for (int w = 0; w < ctx->W; ++w) {
                 L.pW[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * L.in * 4));
@@ -338,6 +428,13 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             maxwt = std::max<long long>(maxwt, (long long)L.out * L.in_ld);
         }
     ctx->scratch_f32 = static_cast<float*>(cv.take(std::max(B * ld8(maxw), maxwt) * 4ull));
+    if (ctx->fused) {
+        const long long tiles = (B + kFusedRows - 1) / kFusedRows;
+        ctx->f_part_p = static_cast<float*>(cv.take((unsigned long long)tiles * ctx->f_ptotal_p * 4));
+        ctx->f_part_a = static_cast<float*>(cv.take((unsigned long long)tiles * ctx->f_ptotal_a * 4));
+        ctx->f_rowloss = static_cast<float*>(cv.take(B * 4ull));
+        ctx->f_counter = static_cast<int*>(cv.take(256));
+    }
     return cv.off + 256;
 }
 
@@ -506,6 +603,181 @@ vfl_status wait_ev(vfl_ctx* ctx, cudaStream_t s, cudaEvent_t e) {
         if (st_ != VFL_OK) return st_;  \
     } while (0)
 
+// ---- fused path -------------------------------------------------------------
+FusedLayerArgs fused_layer(const Layer& L, int vslot, int new_slot, int w, void* Y, long long ldy, void* D,
+                           long long ldd, long long poff) {
+    FusedLayerArgs f;
+    std::memset(&f, 0, sizeof f);
+    f.in = L.in;
+    f.out = L.out;
+    f.in_ld = L.in_ld;
+    f.out_ld = ld8(L.out);
+    f.W = static_cast<const float*>(L.cW[vslot]);
+    f.Wt = L.cWt[vslot];
+    f.b = L.cb[vslot];
+    f.Y = static_cast<float*>(Y);
+    f.ldy = ldy;
+    f.D = static_cast<float*>(D);
+    f.ldd = ldd;
+    f.poff = poff;
+    f.Wm = L.W;
+    f.bm = L.b;
+    f.Wc = static_cast<float*>(L.cW[new_slot]);
+    f.Wtc = L.cWt[new_slot];
+    f.bc = L.cb[new_slot];
+    f.gW = L.pW[w];
+    f.gb = L.pb[w];
+    return f;
+}
+
+double fused_flops(const std::vector<Layer>& v, int rows, bool fwd, bool dx_first, bool dw) {
+    double f = 0;
+    for (size_t l = 0; l < v.size(); ++l) {
+        const double mn = 2.0 * rows * v[l].in * v[l].out;
+        if (fwd) f += mn;
+        if (dw) f += mn;
+        if (dx_first || l > 0) f += dw ? mn : 0;
+    }
+    return f;
+}
+
+vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slot, int vslot, int rows,
+                                 const float* X, cudaStream_t s) {
+    FusedChainArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.nl = (int)ctx->P.size();
+    for (int l = 0; l < a.nl; ++l)
+        a.L[l] = fused_layer(ctx->P[l], vslot, vslot, 0, ctx->act_p[slot][l], ld8(ctx->P[l].out), nullptr, 0, 0);
+    a.x = X;
+    a.ldx = ctx->ldxp;
+    a.rows = rows;
+    a.act_ld = ctx->f_act_ld;
+    a.w_floats = fused_weight_layout(a.L, a.nl, true, 1 << 30, 0);
+    a.counter = ctx->f_counter;
+    a.hdr = ctx->emb_hdr + slot;
+    a.k = k;
+    a.batch = (int)(k % ctx->nb);
+    a.version = (int)v;
+    double bytes = (double)rows * ctx->cfg.d_passive * 4;
+    for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 4;
+    PLAUNCH(K_FUSED_PFWD, fused_flops(ctx->P, rows, true, false, false), bytes, s, launch_fused_passive_fwd(a, s));
+    return VFL_OK;
+}
+
+vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, int vslot, int rows,
+                             const float* Xa, cudaStream_t s) {
+    FusedStepArgs a;
+    std::memset(&a, 0, sizeof a);
+    const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size();
+    const int new_slot = (int)((k + 1) % ctx->S1);
+    const int n_out = ctx->T.back().out;
+    long long off = 0;
+    for (int l = 0; l < La; ++l) {
+        const Layer& L = ctx->A[l];
+        a.L[l] = fused_layer(L, vslot, new_slot, 0, ctx->act_a[0][l], ld8(L.out), ctx->dpre_a[0][l], ld8(L.out), off);
+        off += (long long)L.out * L.in + L.out;
+    }
+    for (int l = 0; l < Lt; ++l) {
+        const Layer& L = ctx->T[l];
+        const bool last = l == Lt - 1;
+        a.L[La + l] = fused_layer(L, vslot, new_slot, 0, last ? (void*)ctx->logits[0] : ctx->act_t[0][l],
+                                  last ? n_out : ld8(L.out), last ? (void*)ctx->ds[0] : ctx->dpre_t[0][l],
+                                  last ? n_out : ld8(L.out), off);
+        off += (long long)L.out * L.in + L.out;
+    }
+    a.na = La;
+    a.nt = Lt;
+    a.rows = rows;
+    a.act_ld = ctx->f_act_ld;
+    {
+        // W^T of every layer, then W of f_a's layers after the first and of every layer of g
+        int off = 0;
+        for (int l = 0; l < La + Lt; ++l) {
+            a.L[l].wts_off = off;
+            off += (int)(a.L[l].in * a.L[l].out_ld);
+        }
+        for (int l = 0; l < La + Lt; ++l) {
+            a.L[l].ws_off = -1;
+            if (l >= La || l > 0) {
+                a.L[l].ws_off = off;
+                off += (int)(a.L[l].out * a.L[l].in_ld);
+            }
+        }
+        a.w_floats = off;
+    }
+    a.x = Xa;
+    a.ldx = ctx->ldxa;
+    long long r0;
+    ctx->batch_rows(k, &r0);
+    a.y = ctx->Y + r0;
+    a.loss = ctx->cfg.loss;
+    a.zp = static_cast<const float*>(ctx->act_p[slot].back());
+    a.ldzp = ld8(ctx->P.back().out);
+    a.gradp = static_cast<float*>(ctx->grad[slot]);
+    a.ldgp = ld8(ctx->P.back().out);
+    a.ds = ctx->ds[0];
+    a.rowloss = ctx->f_rowloss;
+    a.loss_out = ctx->losses + (k % kLossCap);
+    a.part = ctx->f_part_a;
+    a.ptotal = ctx->f_ptotal_a;
+    a.lr = ctx->cfg.lr;
+    a.chk_hdr = ctx->emb_hdr + slot;
+    a.pub_hdr = ctx->grad_hdr + slot;
+    a.k = k;
+    a.batch = (int)(k % ctx->nb);
+    a.version = (int)v;
+    a.status = ctx->status;
+    const int tiles = (rows + kFusedRows - 1) / kFusedRows;
+    const int want = std::max<long long>(tiles, (ctx->f_ptotal_a + kFusedThreads - 1) / kFusedThreads);
+    const int grid = std::max(1, std::min(want, ctx->f_grid_a));
+    const double flops = fused_flops(ctx->A, rows, true, false, true) + fused_flops(ctx->T, rows, true, true, true);
+    double bytes = (double)rows * (ctx->cfg.d_active + 2.0 * ctx->P.back().out) * 4;
+    for (auto* vv : {&ctx->A, &ctx->T})
+        for (const Layer& L : *vv) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 16;
+    bytes += 2.0 * tiles * ctx->f_ptotal_a * 4;
+    PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, grid, s));
+    return VFL_OK;
+}
+
+vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot, int rows, const float* Xp,
+                                  cudaStream_t s) {
+    FusedStepArgs a;
+    std::memset(&a, 0, sizeof a);
+    const int Lp = (int)ctx->P.size();
+    const int new_slot = (int)((k + 1) % ctx->S1);
+    long long off = 0;
+    for (int l = 0; l < Lp; ++l) {
+        const Layer& L = ctx->P[l];
+        a.L[l] = fused_layer(L, vslot, new_slot, 0, ctx->act_p[slot][l], ld8(L.out), ctx->dpre_p[0][l], ld8(L.out),
+                             off);
+        off += (long long)L.out * L.in + L.out;
+    }
+    a.na = Lp;
+    a.nt = 0;
+    a.rows = rows;
+    a.act_ld = ctx->f_act_ld;
+    a.w_floats = fused_weight_layout(a.L, Lp, false, 1, 0);
+    a.x = Xp;
+    a.ldx = ctx->ldxp;
+    a.gradp = static_cast<float*>(ctx->grad[slot]);
+    a.ldgp = ld8(ctx->P.back().out);
+    a.part = ctx->f_part_p;
+    a.ptotal = ctx->f_ptotal_p;
+    a.lr = ctx->cfg.lr;
+    a.chk_hdr = ctx->grad_hdr + slot;
+    a.k = k;
+    a.status = ctx->status;
+    const int tiles = (rows + kFusedRows - 1) / kFusedRows;
+    const int want = std::max<long long>(tiles, (ctx->f_ptotal_p + kFusedThreads - 1) / kFusedThreads);
+    const int grid = std::max(1, std::min(want, ctx->f_grid_p));
+    double bytes = (double)rows * (ctx->cfg.d_passive + ctx->P.back().out) * 4;
+    for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 16;
+    bytes += 2.0 * tiles * ctx->f_ptotal_p * 4;
+    PLAUNCH(K_FUSED_PBWD, fused_flops(ctx->P, rows, false, false, true), bytes, s,
+            launch_fused_passive_bwd(a, grid, s));
+    return VFL_OK;
+}
+
 // ---- the three phases ------------------------------------------------------
 vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const vfl_config& c = ctx->cfg;
@@ -525,6 +797,15 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const int rows = ctx->batch_rows(k, &r0);
     if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
     const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+    if (ctx->fused) {
+        TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), s));
+        CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
+        ctx->fwd_version[slot] = (int)v;
+        ctx->slot_step_p[slot] = k;
+        ctx->n_fwd = k + 1;
+        ctx->started = true;
+        return VFL_OK;
+    }
     long long ldx = ctx->ldxp;
     for (size_t l = 0; l < ctx->P.size(); ++l) {
         const Layer& L = ctx->P[l];
@@ -561,8 +842,19 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const int n_out = ctx->T.back().out;
 
     if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
-    // active bottom forward: z^a = f_a(x^a)
     const void* Xa0 = static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * es;
+    if (ctx->fused) {
+        TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
+        if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+        TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), s));
+        CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
+        CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
+        ctx->grad_step[slot] = k;
+        ctx->last_act_step[w] = k;
+        ctx->n_act = k + 1;
+        return VFL_OK;
+    }
+    // active bottom forward: z^a = f_a(x^a)
     const void* X = Xa0;
     long long ldx = ctx->ldxa;
     for (int l = 0; l < La; ++l) {
@@ -655,6 +947,14 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int Lp = (int)ctx->P.size();
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
+    if (ctx->fused) {
+        if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+        const float* Xp = reinterpret_cast<const float*>(static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz);
+        TRY(fused_passive_backward(ctx, k, slot, vslot, rows, Xp, s));
+        CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
+        ctx->n_bwd = k + 1;
+        return VFL_OK;
+    }
     PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->grad_hdr + slot, k, ctx->status, s));
     // dpre of the cut layer = dLoss/dz^p * [z^p > 0]
     PLAUNCH(K_MASK, 0, 3.0 * rows * ep * ctx->esz, s,
@@ -730,6 +1030,7 @@ vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* 
     tmp.W = cfg->workers;
     tmp.bf16 = cfg->dtype == VFL_BF16;
     tmp.esz = tmp.bf16 ? 2 : 4;
+    tmp.fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
     build_layers(&tmp);
     *bytes = carve_all(&tmp, nullptr);
     return VFL_OK;
@@ -759,6 +1060,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     ctx->nb = (int)((n_rows + cfg->batch - 1) / cfg->batch);
     for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
     for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
+    ctx->fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
     build_layers(ctx);
     const unsigned long long need = carve_all(ctx, nullptr);
     if (workspace_bytes < need) {
@@ -778,6 +1080,15 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     if (e == cudaSuccess) e = cudaMemset(workspace, 0, need);
     if (e == cudaSuccess) e = cudaMemset(ctx->emb_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
     if (e == cudaSuccess) e = cudaMemset(ctx->grad_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
+    if (e == cudaSuccess && ctx->fused) {
+        long long w_p = 0;
+        for (size_t l = 1; l < ctx->P.size(); ++l) w_p += (long long)ctx->P[l].out * ctx->P[l].in_ld;
+        e = fused_max_grid(0, fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size()),
+                           &ctx->f_grid_a);
+        if (e == cudaSuccess)
+            e = fused_max_grid(1, fused_smem_pbwd((int)w_p, ctx->f_act_ld, (int)ctx->P.size()), &ctx->f_grid_p);
+        if (e == cudaSuccess && (ctx->f_grid_a < 1 || ctx->f_grid_p < 1)) e = cudaErrorInvalidConfiguration;
+    }
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         g_global_err = std::string("vfl_create: ") + cudaGetErrorString(e);
@@ -883,6 +1194,10 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
     for (int s = 0; s < ctx->S1; ++s) {
         CK(cudaMemset(L->cW[s], 0, (size_t)L->out * L->in_ld * ctx->esz));
         PLAUNCH(K_CAST, 0, 0, 0, launch_cast_rows(L->W, L->out, L->in, L->cW[s], L->in_ld, ctx->bf16, 0));
+        if (L->cWt[s]) {
+            CK(cudaMemset(L->cWt[s], 0, (size_t)L->in * ld8(L->out) * 4));
+            PLAUNCH(K_CAST, 0, 0, 0, launch_transpose_f32(L->W, L->out, L->in, L->cWt[s], ld8(L->out), 0));
+        }
         CK(cudaMemcpy(L->cb[s], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
     }
     CK(cudaDeviceSynchronize());
@@ -986,6 +1301,11 @@ vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
     CK(cudaMemset(L->cW[slot], 0, (size_t)L->out * L->in_ld * ctx->esz));
     ++ctx->launches;
     CK(launch_cast_rows(tmp, L->out, L->in, L->cW[slot], L->in_ld, ctx->bf16, 0));
+    if (L->cWt[slot]) {
+        CK(cudaMemset(L->cWt[slot], 0, (size_t)L->in * ld8(L->out) * 4));
+        ++ctx->launches;
+        CK(launch_transpose_f32(tmp, L->out, L->in, L->cWt[slot], ld8(L->out), 0));
+    }
     CK(cudaMemcpy(L->cb[slot], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
     if (v == k) {
         CK(cudaMemcpy(L->W, W, nw * 4, cudaMemcpyHostToDevice));

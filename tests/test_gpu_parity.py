@@ -171,3 +171,12 @@ def test_checkpoint_restore_is_bit_exact(vfl, cid):
     for key in pa:
         np.testing.assert_array_equal(pa[key][0], pb[key][0])
         np.testing.assert_array_equal(pa[key][1], pb[key][1])
+
+
+@pytest.mark.parametrize("cid", [1, 2])
+def test_step_parity_generic_kernels(vfl, cid, monkeypatch):
+    """The fp32 presets run the fused one-launch-per-phase kernels by default;
+    the per-layer kernels they would otherwise use must match the oracle too."""
+    monkeypatch.setenv("VFL_DISABLE_FUSED", "1")
+    worst, failures = run_sequential(vfl, cid, CASES[cid])
+    assert not failures, f"preset {cid}: {failures[:3]}"
