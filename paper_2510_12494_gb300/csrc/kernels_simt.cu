@@ -306,6 +306,17 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
     }
 }
 
+__global__ void colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16, float* __restrict__ Pb,
+                              long long pb_stride, int kchunk) {
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (o >= out) return;
+    const int r0 = blockIdx.y * kchunk;
+    const int r1 = min(rows, r0 + kchunk);
+    float acc = 0.f;
+    for (int r = r0; r < r1; ++r) acc += ldany(D, (long long)r * ldd + o, bf16);
+    Pb[(long long)blockIdx.y * pb_stride + o] = acc;
+}
+
 __global__ void transpose_f32_kernel(const float* __restrict__ src, int out, int in, float* __restrict__ dst,
                                      long long ldt) {
     const long long n = (long long)out * in;
@@ -397,6 +408,13 @@ cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long ma
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     cast_rows_kernel<<<grid_for((long long)rows * ld, 256), 256, 0, s>>>(src, rows, d, dst, ld, bf16);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
+                          int nsplit, int kchunk, cudaStream_t s) {
+    dim3 grid((out + 127) / 128, nsplit);
+    colsum_kernel<<<grid, 128, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride, kchunk);
     return cudaGetLastError();
 }
 

@@ -17,7 +17,7 @@ struct ChannelHeader {
 };
 
 // Bits of the device status word.
-enum : int { ST_VERSION = 1, ST_TIMEOUT = 2 };
+enum : int { ST_VERSION = 1, ST_TIMEOUT = 2, ST_KERNEL_TIMEOUT = 4 };
 
 enum GemmMode : int { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
 
@@ -90,6 +90,10 @@ cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,
                                cudaStream_t s);
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s);
+// Split-K column sums: Pb[z * pb_stride + o] = sum over rows r in chunk z of D[r * ldd + o].
+cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
+                          int nsplit, int kchunk, cudaStream_t s);
+
 // dst[k * ldt + o] = src[o * in + k] for src [out, in] fp32.
 cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s);
 

@@ -38,12 +38,12 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
-    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd"};
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum"};
 
 struct ProfRec {
     int cls;
@@ -311,6 +311,7 @@ void build_layers(vfl_ctx* ctx) {
             L.out = outs[l];
             L.in_ld = ld8(d_in);
             choose_split(L, c.batch);
+            if (c.dtype == VFL_BF16) tc_choose_split(L.out, L.in, c.batch, &L.nsplit, &L.kchunk);
             if (ctx->fused) {
                 L.nsplit = 1;
                 L.kchunk = c.batch;
@@ -469,6 +470,7 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
         t.B = L.cW[slot]; t.ldb = L.in_ld;
         t.bias = L.cb[slot]; t.relu = relu;
         t.C = Y; t.ldc = ldy;
+        t.err = ctx->status;
         PLAUNCH(K_TC_FWD, flops, bytes, s, launch_tc_gemm(t, s));
         return VFL_OK;
     }
@@ -502,7 +504,10 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
         t.P = L.pW[w]; t.p_stride = (long long)L.out * L.in; t.ldc = L.in;
         t.Pb = L.pb[w]; t.pb_stride = L.out;
         t.nsplit = L.nsplit; t.kchunk = L.kchunk;
+        t.err = ctx->status;
         PLAUNCH(K_TC_DW, flops, bytes, s, launch_tc_gemm(t, s));
+        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz + (double)L.nsplit * L.out * 4, s,
+                launch_colsum(dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit, L.kchunk, s));
         return VFL_OK;
     }
     const int n1 = X2 ? ka : L.in;
@@ -543,6 +548,8 @@ vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, l
         t.B = L.cW[slot]; t.ldb = L.in_ld;
         t.C = C; t.ldc = ldc; t.mask1 = mask1;
         t.n_split = n_split; t.C2 = C2; t.ldc2 = ldc2; t.mask2 = mask2;
+        t.c2_f32 = c2_f32 ? 1 : 0;
+        t.err = ctx->status;
         PLAUNCH(K_TC_DX, flops, bytes, s, launch_tc_gemm(t, s));
         return VFL_OK;
     }
@@ -986,6 +993,8 @@ vfl_status read_status(vfl_ctx* ctx) {
         CK(cudaMemset(ctx->status, 0, sizeof(int)));
         if (st & ST_VERSION) return ctx->fail(VFL_E_VERSION, "a subscriber found a channel header of another step");
         if (st & ST_TIMEOUT) return ctx->fail(VFL_E_TIMEOUT, "a bounded channel wait gave up");
+        if (st & ST_KERNEL_TIMEOUT)
+            return ctx->fail(VFL_E_TIMEOUT, "a tensor-core GEMM gave up waiting on its pipeline");
     }
     return VFL_OK;
 }

@@ -29,11 +29,17 @@ struct TcGemm {
     int n_split;
     void* C2; long long ldc2;
     const void* mask2;
+    int c2_f32;                 // DX: C2 is fp32 (the DP path perturbs it before publishing)
     float* P; long long p_stride;
     float* Pb; long long pb_stride;
     int nsplit, kchunk;
+    int* err;                   // status word: ST_KERNEL_TIMEOUT when a bounded wait gave up
 };
 
+// The driver's tensor-map encoder is reachable (false on machines without a driver).
+bool tc_available();
+// Split-K factor and chunk (a multiple of 64 rows) of a tensor-core weight gradient over `rows`.
+void tc_choose_split(int out, int in, int rows, int* nsplit, int* kchunk);
 bool tc_supported_fwd(int in, int out, bool concat, int ka, bool out_f32);
 bool tc_supported_dx(int in, int out, int n_split, bool c2_f32);
 bool tc_supported_dw(int out, int in, bool concat, int kb);
