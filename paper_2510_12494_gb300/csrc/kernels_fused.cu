@@ -24,7 +24,6 @@ namespace {
 
 constexpr int NT = kFusedThreads;     // 8 warps
 constexpr int R = kFusedRows;
-constexpr int RPW = R / 8;            // rows per warp
 
 __device__ __forceinline__ void cp16(float* s, const float* g) {
     const unsigned sa = (unsigned)__cvta_generic_to_shared(s);
@@ -59,108 +58,123 @@ __device__ void stage_layer_weights(float* ws, const FusedLayerArgs& L) {
     if (L.ws_off >= 0) async_copy(ws + L.ws_off, L.W, (long long)L.out * L.in_ld);
 }
 
-// Y[r][c] = act(sum_k X[r][k] Wt[k][c] + b[c]); warps own rows, lanes own
-// c = lane + 32 j.  To smem (ldy) and to global rows < nrows when yg != nullptr.
+// Y[r][c] = act(sum_k X[r][k] Wt[k][c] + b[c]) for the R = 16 rows of a tile.
+// Each thread owns a 2-row x 4-column block (16-byte weight loads, 8 independent
+// accumulators); Wt rows are zero beyond N.  To smem (ldy) and to global rows
+// < nrows when yg != nullptr.
 __device__ void tile_fwd(const float* xs, int ldx, int K, const float* wts, long long ldw,
                          const float* __restrict__ bias, int N, bool relu, float* ys, int ldy, float* yg,
                          long long ldyg, int nrows) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nj = (N + 31) / 32;
-    float acc[RPW][8];
-#pragma unroll
-    for (int i = 0; i < RPW; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-    for (int k = 0; k < K; ++k) {
-        float xv[RPW];
-#pragma unroll
-        for (int i = 0; i < RPW; ++i) xv[i] = xs[(warp + 8 * i) * ldx + k];
-        const float* wrow = wts + k * ldw;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (j < nj) {
-                const int c = lane + 32 * j;
-                const float w = c < N ? wrow[c] : 0.f;
-#pragma unroll
-                for (int i = 0; i < RPW; ++i) acc[i][j] = fmaf(xv[i], w, acc[i][j]);
-            }
+    const int n4 = (N + 3) / 4;
+    for (int u = threadIdx.x; u < (R / 2) * n4; u += NT) {
+        const int cg = u % n4, r0 = 2 * (u / n4);
+        const float* x0 = xs + r0 * ldx;
+        const float* x1 = x0 + ldx;
+        float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+        for (int k = 0; k < K; ++k) {
+            const float4 w = *reinterpret_cast<const float4*>(wts + k * ldw + 4 * cg);
+            const float v0 = x0[k], v1 = x1[k];
+            a0[0] = fmaf(v0, w.x, a0[0]); a0[1] = fmaf(v0, w.y, a0[1]);
+            a0[2] = fmaf(v0, w.z, a0[2]); a0[3] = fmaf(v0, w.w, a0[3]);
+            a1[0] = fmaf(v1, w.x, a1[0]); a1[1] = fmaf(v1, w.y, a1[1]);
+            a1[2] = fmaf(v1, w.z, a1[2]); a1[3] = fmaf(v1, w.w, a1[3]);
         }
-    }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int c = lane + 32 * j;
-        if (j >= nj || c >= N) continue;
-        const float bv = bias[c];
-#pragma unroll
-        for (int i = 0; i < RPW; ++i) {
-            const int r = warp + 8 * i;
-            float v = acc[i][j] + bv;
-            if (relu) v = fmaxf(v, 0.f);
-            ys[r * ldy + c] = v;
-            if (yg && r < nrows) yg[(long long)r * ldyg + c] = v;
+        for (int j = 0; j < 4; ++j) {
+            const int c = 4 * cg + j;
+            if (c >= N) break;
+            const float bv = bias[c];
+            float y0 = a0[j] + bv, y1 = a1[j] + bv;
+            if (relu) {
+                y0 = fmaxf(y0, 0.f);
+                y1 = fmaxf(y1, 0.f);
+            }
+            ys[r0 * ldy + c] = y0;
+            ys[(r0 + 1) * ldy + c] = y1;
+            if (yg) {
+                if (r0 < nrows) yg[(long long)r0 * ldyg + c] = y0;
+                if (r0 + 1 < nrows) yg[(long long)(r0 + 1) * ldyg + c] = y1;
+            }
         }
     }
 }
 
 // dX[r][k] = sum_c dY[r][c] W[c][k], zeroed where prev[r][k] <= 0 (when prev is
-// given); warps own rows, lanes own k = lane + 32 j.  To smem and global rows < nrows.
+// given); 2-row x 4-column blocks with 16-byte weight loads (W rows zero beyond
+// K).  To smem and to global rows < nrows.
 __device__ void tile_dx(const float* dys, int ldd, int N, const float* ws, long long ldw, int K, const float* prev,
                         int ldp, float* os, int ldo, float* og, long long ldog, int nrows) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nj = (K + 31) / 32;
-    float acc[RPW][8];
-#pragma unroll
-    for (int i = 0; i < RPW; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-    for (int c = 0; c < N; ++c) {
-        float dv[RPW];
-#pragma unroll
-        for (int i = 0; i < RPW; ++i) dv[i] = dys[(warp + 8 * i) * ldd + c];
-        const float* wrow = ws + c * ldw;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (j < nj) {
-                const int k = lane + 32 * j;
-                const float w = k < K ? wrow[k] : 0.f;
-#pragma unroll
-                for (int i = 0; i < RPW; ++i) acc[i][j] = fmaf(dv[i], w, acc[i][j]);
-            }
+    const int k4 = (K + 3) / 4;
+    for (int u = threadIdx.x; u < (R / 2) * k4; u += NT) {
+        const int kg = u % k4, r0 = 2 * (u / k4);
+        const float* d0 = dys + r0 * ldd;
+        const float* d1 = d0 + ldd;
+        float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+        for (int c = 0; c < N; ++c) {
+            const float4 w = *reinterpret_cast<const float4*>(ws + c * ldw + 4 * kg);
+            const float v0 = d0[c], v1 = d1[c];
+            a0[0] = fmaf(v0, w.x, a0[0]); a0[1] = fmaf(v0, w.y, a0[1]);
+            a0[2] = fmaf(v0, w.z, a0[2]); a0[3] = fmaf(v0, w.w, a0[3]);
+            a1[0] = fmaf(v1, w.x, a1[0]); a1[1] = fmaf(v1, w.y, a1[1]);
+            a1[2] = fmaf(v1, w.z, a1[2]); a1[3] = fmaf(v1, w.w, a1[3]);
         }
-    }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int k = lane + 32 * j;
-        if (j >= nj || k >= K) continue;
-#pragma unroll
-        for (int i = 0; i < RPW; ++i) {
-            const int r = warp + 8 * i;
-            float v = acc[i][j];
-            if (prev && !(prev[r * ldp + k] > 0.f)) v = 0.f;
-            os[r * ldo + k] = v;
-            if (og && r < nrows) og[(long long)r * ldog + k] = v;
+        for (int j = 0; j < 4; ++j) {
+            const int k = 4 * kg + j;
+            if (k >= K) break;
+            float y0 = a0[j], y1 = a1[j];
+            if (prev) {
+                if (!(prev[r0 * ldp + k] > 0.f)) y0 = 0.f;
+                if (!(prev[(r0 + 1) * ldp + k] > 0.f)) y1 = 0.f;
+            }
+            os[r0 * ldo + k] = y0;
+            os[(r0 + 1) * ldo + k] = y1;
+            if (og) {
+                if (r0 < nrows) og[(long long)r0 * ldog + k] = y0;
+                if (r0 + 1 < nrows) og[(long long)(r0 + 1) * ldog + k] = y1;
+            }
         }
     }
 }
 
 // Partial gradient of one layer over the tile's rows, [W | b] flat:
-// part[o*in + k] = sum_r D[r][o] X[r][k], part[out*in + o] = sum_r D[r][o].
-// Rows beyond the batch hold D = 0.
+// part[o*in + k] = sum_r D[r][o] X[r][k] and part[out*in + o] = sum_r D[r][o],
+// in 4 x 4 register blocks fed by 16-byte loads.  Rows beyond the batch hold
+// D = 0; columns past out / in in the tiles are never stored.
 __device__ void tile_partial(const float* Ds, int ldd, const float* Xs, int ldx, int out, int in,
                              float* __restrict__ part) {
-    const int n = out * (in + 1);
-    for (int i = threadIdx.x; i < n; i += NT) {
-        const int o = i / (in + 1), k = i - o * (in + 1);
-        float acc = 0.f;
-        if (k < in) {
+    const int o4 = (out + 3) / 4, i4 = (in + 3) / 4;
+    for (int u = threadIdx.x; u < o4 * i4; u += NT) {
+        const int ob = u / i4, ib = u - ob * i4;
+        float acc[4][4] = {};
 #pragma unroll
-            for (int r = 0; r < R; ++r) acc = fmaf(Ds[r * ldd + o], Xs[r * ldx + k], acc);
-            part[(long long)o * in + k] = acc;
-        } else {
+        for (int r = 0; r < R; ++r) {
+            const float4 d = *reinterpret_cast<const float4*>(Ds + r * ldd + 4 * ob);
+            const float4 x = *reinterpret_cast<const float4*>(Xs + r * ldx + 4 * ib);
+            const float dv[4] = {d.x, d.y, d.z, d.w}, xv[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-            for (int r = 0; r < R; ++r) acc += Ds[r * ldd + o];
-            part[(long long)out * in + o] = acc;
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(dv[i], xv[j], acc[i][j]);
         }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int o = 4 * ob + i;
+            if (o >= out) break;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int k = 4 * ib + j;
+                if (k < in) part[(long long)o * in + k] = acc[i][j];
+            }
+        }
+    }
+    for (int o = threadIdx.x; o < out; o += NT) {
+        float acc = 0.f;
+#pragma unroll
+        for (int r = 0; r < R; ++r) acc += Ds[r * ldd + o];
+        part[(long long)out * in + o] = acc;
     }
 }
 

@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
         } else {
             const long long j = idx - nw;
             float gsum = 0.f;
-            for (int z = 0; z < L.nsplit; ++z) gsum += L.pb[z * L.pb_stride + j];
+            for (int z = 0; z < L.nsplit_b; ++z) gsum += L.pb[z * L.pb_stride + j];
             const float b = L.b[j] - a.lr * gsum;
             L.b[j] = b;
             L.cb[j] = b;
@@ -306,15 +306,50 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
     }
 }
 
-__global__ void colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16, float* __restrict__ Pb,
-                              long long pb_stride, int kchunk) {
-    const int o = blockIdx.x * blockDim.x + threadIdx.x;
-    if (o >= out) return;
-    const int r0 = blockIdx.y * kchunk;
-    const int r1 = min(rows, r0 + kchunk);
-    float acc = 0.f;
-    for (int r = r0; r < r1; ++r) acc += ldany(D, (long long)r * ldd + o, bf16);
-    Pb[(long long)blockIdx.y * pb_stride + o] = acc;
+// Column sums over blocks of 64 rows: block (x, y) covers columns
+// [256 x, 256 x + 256) of rows [64 y, 64 y + 64); tx owns 8 adjacent columns,
+// ty every 8th row; the 8 row lanes are combined in a fixed order.
+// Reads 8 columns at a time, so D's row stride must cover ceil(out/8)*8 columns.
+__global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16,
+                                                     float* __restrict__ Pb, long long pb_stride) {
+    __shared__ float red[8][257];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int c0 = blockIdx.x * 256 + tx * 8;
+    const int rb = blockIdx.y * 64;
+    float acc[8] = {};
+    if (c0 < out) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int r = rb + ty + 8 * i;
+            if (r < rows) {
+                if (bf16) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(D) +
+                                                                    (long long)r * ldd + c0);
+                    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float2 f = __bfloat1622float2(h[q]);
+                        acc[2 * q] += f.x;
+                        acc[2 * q + 1] += f.y;
+                    }
+                } else {
+                    const float* row = static_cast<const float*>(D) + (long long)r * ldd + c0;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) acc[q] += row[q];
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) red[ty][tx * 8 + q] = acc[q];
+    __syncthreads();
+    const int c = blockIdx.x * 256 + threadIdx.x;
+    if (c < out) {
+        float t = 0.f;
+#pragma unroll
+        for (int y = 0; y < 8; ++y) t += red[y][threadIdx.x];
+        Pb[(long long)blockIdx.y * pb_stride + c] = t;
+    }
 }
 
 __global__ void transpose_f32_kernel(const float* __restrict__ src, int out, int in, float* __restrict__ dst,
@@ -412,9 +447,10 @@ cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long 
 }
 
 cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
-                          int nsplit, int kchunk, cudaStream_t s) {
-    dim3 grid((out + 127) / 128, nsplit);
-    colsum_kernel<<<grid, 128, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride, kchunk);
+                          int nblocks, cudaStream_t s) {
+    if (nblocks < 1) return cudaErrorInvalidValue;
+    dim3 grid((out + 255) / 256, nblocks);
+    colsum_kernel<<<grid, 256, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride);
     return cudaGetLastError();
 }
 

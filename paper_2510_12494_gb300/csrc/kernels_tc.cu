@@ -142,6 +142,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// bf16 bit pattern h (low 16 bits) is > 0: positive, non-zero, not NaN
+__device__ __forceinline__ bool bf16_positive(uint32_t h) {
+    return !(h & 0x8000u) && (h & 0x7FFFu) != 0 && (h & 0x7FFFu) <= 0x7F80u;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 __device__ __forceinline__ float bf16_at(const void* base, long long idx) {
     return __bfloat162float(static_cast<const __nv_bfloat16*>(base)[idx]);
 }
@@ -276,41 +286,89 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (*abort_flag || m >= p.M) continue;
             const int nbase = n0 + c0;
             if (p.mode == GEMM_FWD) {
-                __nv_bfloat16* C = static_cast<__nv_bfloat16*>(p.C) + (long long)m * p.ldc;
+                __nv_bfloat16* C = static_cast<__nv_bfloat16*>(p.C) + (long long)m * p.ldc + nbase;
+                if (nbase + 32 <= p.N) {
+                    const float4* b4 = reinterpret_cast<const float4*>(p.bias + nbase);
+                    uint32_t packed[16];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int n = nbase + i;
-                    if (n < p.N) {
-                        float x = v[i] + p.bias[n];
+                    for (int q = 0; q < 8; ++q) {
+                        const float4 bq = b4[q];
+                        float x0 = v[4 * q] + bq.x, x1 = v[4 * q + 1] + bq.y, x2 = v[4 * q + 2] + bq.z,
+                              x3 = v[4 * q + 3] + bq.w;
+                        if (p.relu) {
+                            x0 = fmaxf(x0, 0.f); x1 = fmaxf(x1, 0.f); x2 = fmaxf(x2, 0.f); x3 = fmaxf(x3, 0.f);
+                        }
+                        packed[2 * q] = pack_bf16(x0, x1);
+                        packed[2 * q + 1] = pack_bf16(x2, x3);
+                    }
+                    uint4* dst = reinterpret_cast<uint4*>(C);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+                } else {
+                    for (int i = 0; i < 32 && nbase + i < p.N; ++i) {
+                        float x = v[i] + p.bias[nbase + i];
                         if (p.relu) x = fmaxf(x, 0.f);
-                        C[n] = __float2bfloat16_rn(x);
+                        C[i] = __float2bfloat16_rn(x);
                     }
                 }
             } else if (p.mode == GEMM_DX) {
+                const bool to_c = nbase + 32 <= min(p.N, p.n_split);
+                const bool to_c2 = nbase >= p.n_split && nbase + 32 <= p.N && ((nbase - p.n_split) & 7) == 0;
+                if (to_c || to_c2) {
+                    const long long idx = to_c ? (long long)m * p.ldc + nbase : (long long)m * p.ldc2 + (nbase - p.n_split);
+                    const void* mask = to_c ? p.mask1 : p.mask2;
+                    if (mask) {
+                        const uint4* mk = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mask) + idx);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int n = nbase + i;
-                    if (n >= p.N) continue;
-                    float x = v[i];
-                    if (n < p.n_split) {
-                        const long long idx = (long long)m * p.ldc + n;
-                        if (p.mask1 && !(bf16_at(p.mask1, idx) > 0.f)) x = 0.f;
-                        static_cast<__nv_bfloat16*>(p.C)[idx] = __float2bfloat16_rn(x);
+                        for (int q = 0; q < 4; ++q) {
+                            const uint4 w = mk[q];
+                            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                            for (int h = 0; h < 4; ++h) {
+                                if (!bf16_positive(ws[h] & 0xFFFFu)) v[8 * q + 2 * h] = 0.f;
+                                if (!bf16_positive(ws[h] >> 16)) v[8 * q + 2 * h + 1] = 0.f;
+                            }
+                        }
+                    }
+                    if (to_c2 && p.c2_f32) {
+                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C2) + idx);
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                     } else {
-                        const long long idx = (long long)m * p.ldc2 + (n - p.n_split);
-                        if (p.mask2 && !(bf16_at(p.mask2, idx) > 0.f)) x = 0.f;
-                        if (p.c2_f32)
-                            static_cast<float*>(p.C2)[idx] = x;
-                        else
-                            static_cast<__nv_bfloat16*>(p.C2)[idx] = __float2bfloat16_rn(x);
+                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2) + idx);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            dst[q] = make_uint4(pack_bf16(v[8 * q], v[8 * q + 1]), pack_bf16(v[8 * q + 2], v[8 * q + 3]),
+                                                pack_bf16(v[8 * q + 4], v[8 * q + 5]), pack_bf16(v[8 * q + 6], v[8 * q + 7]));
+                    }
+                } else {
+                    for (int i = 0; i < 32; ++i) {
+                        const int n = nbase + i;
+                        if (n >= p.N) break;
+                        float x = v[i];
+                        if (n < p.n_split) {
+                            const long long idx = (long long)m * p.ldc + n;
+                            if (p.mask1 && !(bf16_at(p.mask1, idx) > 0.f)) x = 0.f;
+                            static_cast<__nv_bfloat16*>(p.C)[idx] = __float2bfloat16_rn(x);
+                        } else {
+                            const long long idx = (long long)m * p.ldc2 + (n - p.n_split);
+                            if (p.mask2 && !(bf16_at(p.mask2, idx) > 0.f)) x = 0.f;
+                            if (p.c2_f32)
+                                static_cast<float*>(p.C2)[idx] = x;
+                            else
+                                static_cast<__nv_bfloat16*>(p.C2)[idx] = __float2bfloat16_rn(x);
+                        }
                     }
                 }
             } else {
-                float* P = p.P + (long long)blockIdx.z * p.p_stride + (long long)m * p.ldc;
+                float* P = p.P + (long long)blockIdx.z * p.p_stride + (long long)m * p.ldc + nbase;
+                if (nbase + 32 <= p.N && (p.ldc & 3) == 0) {
+                    float4* dst = reinterpret_cast<float4*>(P);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int n = nbase + i;
-                    if (n < p.N) P[n] = v[i];
+                    for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                } else {
+                    for (int i = 0; i < 32 && nbase + i < p.N; ++i) P[i] = v[i];
                 }
             }
         }
@@ -376,11 +434,12 @@ bool tc_supported_dx(int in, int out, int n_split, bool c2_f32) {
     return tc_available();
 }
 
-bool tc_supported_dw(int out, int in, bool concat, int kb) {
+bool tc_shape_dw(int out, int in, bool concat, int kb) {
     if (out < 16 || in < 1) return false;
-    if (concat && kb % BN != 0) return false;
-    return tc_available();
+    return !(concat && kb % BN != 0);
 }
+
+bool tc_supported_dw(int out, int in, bool concat, int kb) { return tc_shape_dw(out, in, concat, kb) && tc_available(); }
 
 void tc_choose_split(int out, int in, int rows, int* nsplit, int* kchunk) {
     const long long tiles = (long long)((out + BM - 1) / BM) * ((in + BN - 1) / BN);

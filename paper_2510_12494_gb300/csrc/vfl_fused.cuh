@@ -6,7 +6,7 @@
 namespace vfl {
 
 constexpr int kFusedThreads = 256;
-constexpr int kFusedRows = 8;                  // rows per row tile (one per warp)
+constexpr int kFusedRows = 16;                 // rows per row tile
 constexpr int kFusedMaxWidth = 256;            // widest layer input or output
 constexpr int kFusedMaxLayers = 16;
 constexpr size_t kFusedMaxSmem = 227 * 1024;

@@ -70,7 +70,8 @@ struct SgdLayer {
     float* W; float* b;           // fp32 master
     const float* pW; const float* pb;  // split-K partial gradients
     long long pW_stride, pb_stride;
-    int nsplit;
+    int nsplit;                   // partials of dW
+    int nsplit_b;                 // partials of db
     int out, in, in_ld;
     void* cW; float* cb;          // compute copy to write (ring slot of the new version)
     long long begin;              // first flat element index of this layer
@@ -90,9 +91,11 @@ cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,
                                cudaStream_t s);
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s);
-// Split-K column sums: Pb[z * pb_stride + o] = sum over rows r in chunk z of D[r * ldd + o].
+// Column sums in blocks of 64 rows: Pb[z * pb_stride + o] = sum of D[r * ldd + o] over
+// rows r in [64 z, 64 z + 64) (zero for blocks past `rows`); z < nblocks.  D's row
+// stride must cover ceil(out / 8) * 8 columns.
 cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
-                          int nsplit, int kchunk, cudaStream_t s);
+                          int nblocks, cudaStream_t s);
 
 // dst[k * ldt + o] = src[o * in + k] for src [out, in] fp32.
 cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s);

@@ -67,7 +67,9 @@ struct Layer {
     float* cWt[kMaxSlots] = {};           // fused path: transposed version copies [in, ld8(out)], fp32
     float* pW[kMaxWorkers] = {};          // split-K partial dW [nsplit][out*in]
     float* pb[kMaxWorkers] = {};          // partial db [nsplit][out]
-    int nsplit = 1;
+    int nsplit = 1;                       // weight-gradient partials
+    int nsplit_b = 1;                     // bias-gradient partials
+    bool colsum_bias = false;             // db from 64-row column-sum blocks (tensor-core dW layers)
     int kchunk = 0;
 };
 
@@ -312,6 +314,7 @@ void build_layers(vfl_ctx* ctx) {
             L.in_ld = ld8(d_in);
             choose_split(L, c.batch);
             if (c.dtype == VFL_BF16) tc_choose_split(L.out, L.in, c.batch, &L.nsplit, &L.kchunk);
+            L.nsplit_b = L.nsplit;
             if (ctx->fused) {
                 L.nsplit = 1;
                 L.kchunk = c.batch;
@@ -323,6 +326,19 @@ void build_layers(vfl_ctx* ctx) {
     mk(ctx->P, 0, c.n_passive, c.passive_out, c.d_passive);
     mk(ctx->A, 1, c.n_active, c.active_out, c.d_active);
     mk(ctx->T, 2, c.n_top, c.top_out, c.active_out[c.n_active - 1] + c.passive_out[c.n_passive - 1]);
+    if (c.dtype == VFL_BF16) {
+        const int ea = ctx->A.back().out;
+        for (auto* v : {&ctx->P, &ctx->A, &ctx->T})
+            for (size_t l = 0; l < v->size(); ++l) {
+                Layer& L = (*v)[l];
+                const bool last_top = v == &ctx->T && l + 1 == v->size();
+                const bool concat = v == &ctx->T && l == 0;
+                if (!last_top && tc_shape_dw(L.out, L.in, concat, ea)) {
+                    L.colsum_bias = true;
+                    L.nsplit_b = (c.batch + 63) / 64;
+                }
+            }
+    }
     if (ctx->fused) {
         int maxw = std::max(c.d_passive, c.d_active);
         ctx->f_wp = ctx->f_wa = 0;
@@ -387,7 +403,7 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             }
             for (int w = 0; w < ctx->W; ++w) {
                 L.pW[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * L.in * 4));
-                L.pb[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * 4));
+                L.pb[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit_b * L.out * 4));
             }
         }
     }
@@ -506,8 +522,8 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
         t.nsplit = L.nsplit; t.kchunk = L.kchunk;
         t.err = ctx->status;
         PLAUNCH(K_TC_DW, flops, bytes, s, launch_tc_gemm(t, s));
-        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz + (double)L.nsplit * L.out * 4, s,
-                launch_colsum(dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit, L.kchunk, s));
+        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz + (double)L.nsplit_b * L.out * 4, s,
+                launch_colsum(dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit_b, s));
         return VFL_OK;
     }
     const int n1 = X2 ? ka : L.in;
@@ -515,10 +531,13 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
     g.A = dpre; g.a_rs = 1; g.a_cs = ldd;
     g.B = X; g.b_rs = 1; g.b_cs = ldx;
     g.P = L.pW[w]; g.p_stride = (long long)L.out * L.in; g.ldc = L.in;
-    g.Pb = L.pb[w]; g.pb_stride = L.out;
+    g.Pb = L.colsum_bias ? nullptr : L.pb[w]; g.pb_stride = L.out;
     g.kchunk = L.kchunk;
     const double f1 = X2 ? flops * n1 / L.in : flops, b1 = X2 ? bytes * n1 / L.in : bytes;
     PLAUNCH(K_SIMT_DW, f1, b1, s, launch_gemm_simt(g, a_bf, bf, bf, L.nsplit, s));
+    if (L.colsum_bias)
+        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz, s,
+                launch_colsum(dpre, ldd, rows, L.out, a_bf, L.pb[w], L.out, L.nsplit_b, s));
     if (X2) {
         GemmArgs g2 = gemm_base(GEMM_DW, L.out, L.in - ka, rows);
         g2.A = dpre; g2.a_rs = 1; g2.a_cs = ldd;
@@ -579,6 +598,7 @@ vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w
             d.pW_stride = (long long)L.out * L.in;
             d.pb_stride = L.out;
             d.nsplit = L.nsplit;
+            d.nsplit_b = L.nsplit_b;
             d.out = L.out; d.in = L.in; d.in_ld = L.in_ld;
             d.cW = L.cW[new_slot]; d.cb = L.cb[new_slot];
             d.begin = off;
@@ -593,7 +613,8 @@ vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w
     for (int i = 0; i < n; ++i) {
         const SgdLayer& d = args.L[i];
         const double np_ = (double)d.out * d.in + d.out;
-        bytes += np_ * (8.0 + 4.0 * d.nsplit) + (double)d.out * d.in * ctx->esz + d.out * 4.0;
+        bytes += np_ * 8.0 + 4.0 * ((double)d.out * d.in * d.nsplit + (double)d.out * d.nsplit_b) +
+                 (double)d.out * d.in * ctx->esz + d.out * 4.0;
     }
     PLAUNCH(K_SGD, 2.0 * off, bytes, s, launch_sgd(args, s));
     return VFL_OK;
@@ -1232,7 +1253,7 @@ vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t wor
     if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
     TRY(sync_all(ctx));
     const size_t nw = (size_t)L->out * L->in;
-    std::vector<float> pw((size_t)L->nsplit * nw), pb((size_t)L->nsplit * L->out);
+    std::vector<float> pw((size_t)L->nsplit * nw), pb((size_t)L->nsplit_b * L->out);
     CK(cudaMemcpy(pw.data(), L->pW[worker], pw.size() * 4, cudaMemcpyDeviceToHost));
     CK(cudaMemcpy(pb.data(), L->pb[worker], pb.size() * 4, cudaMemcpyDeviceToHost));
     for (size_t i = 0; i < nw; ++i) {
@@ -1242,7 +1263,7 @@ vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t wor
     }
     for (int i = 0; i < L->out; ++i) {
         float a = 0.f;
-        for (int z = 0; z < L->nsplit; ++z) a += pb[(size_t)z * L->out + i];
+        for (int z = 0; z < L->nsplit_b; ++z) a += pb[(size_t)z * L->out + i];
         db[i] = a;
     }
     return VFL_OK;

@@ -40,6 +40,8 @@ struct TcGemm {
 bool tc_available();
 // Split-K factor and chunk (a multiple of 64 rows) of a tensor-core weight gradient over `rows`.
 void tc_choose_split(int out, int in, int rows, int* nsplit, int* kchunk);
+// Shape rule for the tensor-core weight gradient (independent of the driver).
+bool tc_shape_dw(int out, int in, bool concat, int kb);
 bool tc_supported_fwd(int in, int out, bool concat, int ka, bool out_f32);
 bool tc_supported_dx(int in, int out, int n_split, bool c2_f32);
 bool tc_supported_dw(int out, int in, bool concat, int kb);
