@@ -224,6 +224,14 @@ vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out);
  */
 vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_iters);
 
+/*
+ * Non-blocking subscriber check: does the embedding (which = 0) or gradient
+ * (which = 1) channel slot of step k carry the header of step k?  VFL_OK or
+ * VFL_E_VERSION (the same device-side check the subscriber phases run).
+ * Synchronizes the context.
+ */
+vfl_status vfl_check_channel(vfl_ctx* ctx, int32_t which, int64_t k);
+
 /* Number of kernels this context has launched so far (for launch accounting). */
 int64_t vfl_kernel_launches(const vfl_ctx* ctx);
 

@@ -81,6 +81,7 @@ EXPORTS = {
     "vfl_tap": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p]),
     "vfl_fetch_loss": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_wait_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64]),
+    "vfl_check_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64]),
     "vfl_kernel_launches": (ctypes.c_int64, [ctypes.c_void_p]),
     "vfl_profile": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32]),
     "vfl_profile_get": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64),
@@ -344,6 +345,9 @@ class Context:
 
     def wait_channel(self, which, k, max_iters):
         self._call(lib().vfl_wait_channel, which, k, max_iters)
+
+    def check_channel(self, which, k):
+        self._call(lib().vfl_check_channel, which, k)
 
     @property
     def launches(self) -> int:

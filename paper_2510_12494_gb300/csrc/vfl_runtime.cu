@@ -686,6 +686,7 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     a.k = k;
     a.batch = (int)(k % ctx->nb);
     a.version = (int)v;
+    // algorithmic bytes: the batch's features in, the saved activations out, one read of the weights
     double bytes = (double)rows * ctx->cfg.d_passive * 4;
     for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 4;
     PLAUNCH(K_FUSED_PFWD, fused_flops(ctx->P, rows, true, false, false), bytes, s, launch_fused_passive_fwd(a, s));
@@ -759,10 +760,11 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     const int want = std::max<long long>(tiles, (ctx->f_ptotal_a + kFusedThreads - 1) / kFusedThreads);
     const int grid = std::max(1, std::min(want, ctx->f_grid_a));
     const double flops = fused_flops(ctx->A, rows, true, false, true) + fused_flops(ctx->T, rows, true, true, true);
-    double bytes = (double)rows * (ctx->cfg.d_active + 2.0 * ctx->P.back().out) * 4;
+    // algorithmic bytes: x^a, labels and z^p in, dz^p out; every weight read once,
+    // its master read and written, and the new version's copy written
+    double bytes = (double)rows * (ctx->cfg.d_active + 2.0 * ctx->P.back().out + 1) * 4;
     for (auto* vv : {&ctx->A, &ctx->T})
-        for (const Layer& L : *vv) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 16;
-    bytes += 2.0 * tiles * ctx->f_ptotal_a * 4;
+        for (const Layer& L : *vv) bytes += ((double)L.out * L.in + L.out) * 16;
     PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, grid, s));
     return VFL_OK;
 }
@@ -798,9 +800,9 @@ vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot
     const int tiles = (rows + kFusedRows - 1) / kFusedRows;
     const int want = std::max<long long>(tiles, (ctx->f_ptotal_p + kFusedThreads - 1) / kFusedThreads);
     const int grid = std::max(1, std::min(want, ctx->f_grid_p));
+    // algorithmic bytes: x^p, dz^p and the saved activations in; weights as in the active step
     double bytes = (double)rows * (ctx->cfg.d_passive + ctx->P.back().out) * 4;
-    for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 16;
-    bytes += 2.0 * tiles * ctx->f_ptotal_p * 4;
+    for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 16;
     PLAUNCH(K_FUSED_PBWD, fused_flops(ctx->P, rows, false, false, true), bytes, s,
             launch_fused_passive_bwd(a, grid, s));
     return VFL_OK;
@@ -1508,6 +1510,16 @@ vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_
     TRY(sync_all(ctx));
     const ChannelHeader* h = (which == 0 ? ctx->emb_hdr : ctx->grad_hdr) + (k % ctx->S1);
     PLAUNCH(K_HEADER, 0, 0, ctx->ps[0], launch_wait_header(h, k, max_iters, ctx->status, ctx->ps[0]));
+    return sync_all(ctx);
+}
+
+vfl_status vfl_check_channel(vfl_ctx* ctx, int32_t which, int64_t k) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if ((which != 0 && which != 1) || k < 0) return ctx->fail(VFL_E_INVAL, "invalid check arguments");
+    TRY(sync_all(ctx));
+    const ChannelHeader* h = (which == 0 ? ctx->emb_hdr : ctx->grad_hdr) + (k % ctx->S1);
+    PLAUNCH(K_HEADER, 0, 16, ctx->ps[0], launch_check_header(h, k, ctx->status, ctx->ps[0]));
     return sync_all(ctx);
 }
 
