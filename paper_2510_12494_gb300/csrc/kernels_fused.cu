@@ -24,20 +24,29 @@ namespace {
 
 constexpr int NT = kFusedThreads;     // 8 warps
 constexpr int R = kFusedRows;
+static_assert(R == 16, "the MMA tiles cover exactly 16 rows");
 
 __device__ __forceinline__ void cp16(float* s, const float* g) {
     const unsigned sa = (unsigned)__cvta_generic_to_shared(s);
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sa), "l"(g) : "memory");
 }
 
-__device__ __forceinline__ void cp_wait_all() {
-    asm volatile("cp.async.commit_group;\n" ::: "memory");
-    asm volatile("cp.async.wait_group 0;\n" ::: "memory");
-}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 
-// n floats (n % 4 == 0; both ends 16-byte aligned), asynchronously
-__device__ void async_copy(float* s, const float* g, long long n) {
-    for (long long i = threadIdx.x; i < n / 4; i += NT) cp16(s + 4 * i, g + 4 * i);
+// wait until at most n committed groups are still in flight (n <= 8), then make them visible block-wide
+__device__ __forceinline__ void cp_wait_pending(int n) {
+    switch (n) {
+        case 0: asm volatile("cp.async.wait_group 0;\n" ::: "memory"); break;
+        case 1: asm volatile("cp.async.wait_group 1;\n" ::: "memory"); break;
+        case 2: asm volatile("cp.async.wait_group 2;\n" ::: "memory"); break;
+        case 3: asm volatile("cp.async.wait_group 3;\n" ::: "memory"); break;
+        case 4: asm volatile("cp.async.wait_group 4;\n" ::: "memory"); break;
+        case 5: asm volatile("cp.async.wait_group 5;\n" ::: "memory"); break;
+        case 6: asm volatile("cp.async.wait_group 6;\n" ::: "memory"); break;
+        case 7: asm volatile("cp.async.wait_group 7;\n" ::: "memory"); break;
+        default: asm volatile("cp.async.wait_group 8;\n" ::: "memory"); break;
+    }
+    __syncthreads();
 }
 
 // R rows of `cols` floats (cols % 4 == 0): rows < nrows copied asynchronously
@@ -53,121 +62,177 @@ __device__ void async_rows(float* s, int lds, const float* g, long long ldg, int
     }
 }
 
-__device__ void stage_layer_weights(float* ws, const FusedLayerArgs& L) {
-    if (L.wts_off >= 0) async_copy(ws + L.wts_off, L.Wt, (long long)L.in * L.out_ld);
-    if (L.ws_off >= 0) async_copy(ws + L.ws_off, L.W, (long long)L.out * L.in_ld);
+// rows x cols floats (cols % 4 == 0, 16-byte aligned rows) into smem rows of stride lds, asynchronously
+__device__ void async_matrix(float* s, int lds, const float* g, long long ldg, int rows, int cols) {
+    const int q = cols / 4;
+    for (int i = threadIdx.x; i < rows * q; i += NT) {
+        const int r = i / q, c = (i - r * q) * 4;
+        cp16(s + r * lds + c, g + (long long)r * ldg + c);
+    }
 }
 
-// Y[r][c] = act(sum_k X[r][k] Wt[k][c] + b[c]) for the R = 16 rows of a tile.
-// Each thread owns a 2-row x 4-column block (16-byte weight loads, 8 independent
-// accumulators); Wt rows are zero beyond N.  To smem (ldy) and to global rows
-// < nrows when yg != nullptr.
-__device__ void tile_fwd(const float* xs, int ldx, int K, const float* wts, long long ldw,
-                         const float* __restrict__ bias, int N, bool relu, float* ys, int ldy, float* yg,
-                         long long ldyg, int nrows) {
-    const int n4 = (N + 3) / 4;
-    for (int u = threadIdx.x; u < (R / 2) * n4; u += NT) {
-        const int cg = u % n4, r0 = 2 * (u / n4);
-        const float* x0 = xs + r0 * ldx;
-        const float* x1 = x0 + ldx;
-        float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-        for (int k = 0; k < K; ++k) {
-            const float4 w = *reinterpret_cast<const float4*>(wts + k * ldw + 4 * cg);
-            const float v0 = x0[k], v1 = x1[k];
-            a0[0] = fmaf(v0, w.x, a0[0]); a0[1] = fmaf(v0, w.y, a0[1]);
-            a0[2] = fmaf(v0, w.z, a0[2]); a0[3] = fmaf(v0, w.w, a0[3]);
-            a1[0] = fmaf(v1, w.x, a1[0]); a1[1] = fmaf(v1, w.y, a1[1]);
-            a1[2] = fmaf(v1, w.z, a1[2]); a1[3] = fmaf(v1, w.w, a1[3]);
-        }
+__device__ void stage_layer_weights(float* ws, const FusedLayerArgs& L) {
+    if (L.ws_off >= 0) async_matrix(ws + L.ws_off, L.ws_ld, L.W, L.in_ld, L.out, (int)L.in_ld);
+}
+
+// ---- warp-level tensor-core tiles: mma.sync m16n8k8 TF32 in 3xTF32 form ----
+// Each fp32 operand x is split into hi = tf32(x) and lo = tf32(x - hi); the
+// product is accumulated as lo*hi + hi*lo + hi*hi in fp32 (the lo*lo term,
+// ~2^-22 relative, is dropped), which keeps fp32-level accuracy.
+__device__ __forceinline__ uint32_t to_tf32(float x) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return r;
+}
+
+__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
+    hi = to_tf32(x);
+    lo = to_tf32(x - __uint_as_float(hi));
+}
+
+__device__ __forceinline__ void mma_tf32(float* d, const uint32_t* a, const uint32_t* b) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// d += a_hi*b_hi and e += a_lo*b_hi + a_hi*b_lo for a 16x8 (A) by 8x8 (B)
+// fragment pair given as fp32 values; the caller adds e into d at the end
+// (two accumulators keep the dependent MMA chain short).
+__device__ __forceinline__ void mma_3xtf32(float* d, float* e, const float* a, const float* b) {
+    uint32_t ah[4], al[4], bh[2], bl[2];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) split_tf32(a[i], ah[i], al[i]);
+    split_tf32(b[0], bh[0], bl[0]);
+    split_tf32(b[1], bh[1], bl[1]);
+    mma_tf32(e, al, bh);
+    mma_tf32(d, ah, bh);
+    mma_tf32(e, ah, bl);
+}
+
+// Y[r][c] = act(sum_k X[r][k] W[c][k] + b[c]) for the 16 rows of a tile, W
+// row-major in smem.  Warp w owns the 8-column output tiles w, w+8, w+16, w+24
+// (N <= 256).  Values past K (stale smem) and rows past N are masked.
+// Fragment layout (g = lane/4, t = lane%4): A[g|g+8][t|t+4], B[t|t+4][g],
+// D[g|g+8][2t|2t+1].
+__device__ void tile_fwd(const float* xs, int ldx, int K, const float* ws, int ldw, const float* __restrict__ bias,
+                         int N, bool relu, float* ys, int ldy, float* yg, long long ldyg, int nrows) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
+    const int ntiles = (N + 7) / 8;
+    if (warp >= ntiles) return;
+    float d[4][4] = {}, e[4][4] = {};
+#pragma unroll 2
+    for (int k0 = 0; k0 < K; k0 += 8) {
+        const int ka = k0 + t, kb = k0 + t + 4;
+        float a[4];
+        a[0] = ka < K ? xs[g * ldx + ka] : 0.f;
+        a[1] = ka < K ? xs[(g + 8) * ldx + ka] : 0.f;
+        a[2] = kb < K ? xs[g * ldx + kb] : 0.f;
+        a[3] = kb < K ? xs[(g + 8) * ldx + kb] : 0.f;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const int c = 4 * cg + j;
-            if (c >= N) break;
-            const float bv = bias[c];
-            float y0 = a0[j] + bv, y1 = a1[j] + bv;
-            if (relu) {
-                y0 = fmaxf(y0, 0.f);
-                y1 = fmaxf(y1, 0.f);
+            const int nt = warp + 8 * j;
+            if (nt < ntiles) {
+                const int n = nt * 8 + g;
+                const float* wr = ws + n * ldw;
+                float b[2];
+                b[0] = (ka < K && n < N) ? wr[ka] : 0.f;
+                b[1] = (kb < K && n < N) ? wr[kb] : 0.f;
+                mma_3xtf32(d[j], e[j], a, b);
             }
-            ys[r0 * ldy + c] = y0;
-            ys[(r0 + 1) * ldy + c] = y1;
-            if (yg) {
-                if (r0 < nrows) yg[(long long)r0 * ldyg + c] = y0;
-                if (r0 + 1 < nrows) yg[(long long)(r0 + 1) * ldyg + c] = y1;
-            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int nt = warp + 8 * j;
+        if (nt >= ntiles) break;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int r = g + 8 * (q >> 1), c = nt * 8 + 2 * t + (q & 1);
+            if (c >= N) continue;
+            float y = d[j][q] + e[j][q] + bias[c];
+            if (relu) y = fmaxf(y, 0.f);
+            ys[r * ldy + c] = y;
+            if (yg && r < nrows) yg[(long long)r * ldyg + c] = y;
         }
     }
 }
 
 // dX[r][k] = sum_c dY[r][c] W[c][k], zeroed where prev[r][k] <= 0 (when prev is
-// given); 2-row x 4-column blocks with 16-byte weight loads (W rows zero beyond
-// K).  To smem and to global rows < nrows.
-__device__ void tile_dx(const float* dys, int ldd, int N, const float* ws, long long ldw, int K, const float* prev,
-                        int ldp, float* os, int ldo, float* og, long long ldog, int nrows) {
-    const int k4 = (K + 3) / 4;
-    for (int u = threadIdx.x; u < (R / 2) * k4; u += NT) {
-        const int kg = u % k4, r0 = 2 * (u / k4);
-        const float* d0 = dys + r0 * ldd;
-        const float* d1 = d0 + ldd;
-        float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-        for (int c = 0; c < N; ++c) {
-            const float4 w = *reinterpret_cast<const float4*>(ws + c * ldw + 4 * kg);
-            const float v0 = d0[c], v1 = d1[c];
-            a0[0] = fmaf(v0, w.x, a0[0]); a0[1] = fmaf(v0, w.y, a0[1]);
-            a0[2] = fmaf(v0, w.z, a0[2]); a0[3] = fmaf(v0, w.w, a0[3]);
-            a1[0] = fmaf(v1, w.x, a1[0]); a1[1] = fmaf(v1, w.y, a1[1]);
-            a1[2] = fmaf(v1, w.z, a1[2]); a1[3] = fmaf(v1, w.w, a1[3]);
-        }
+// given).  Warp w owns the 8-column output tiles w + 8 j (K <= 256); the
+// reduction over c < N runs in steps of 8 (values past N masked).
+__device__ void tile_dx(const float* dys, int ldd, int N, const float* ws, int ldw, int K, const float* prev, int ldp,
+                        float* os, int ldo, float* og, long long ldog, int nrows) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
+    const int ktiles = (K + 7) / 8;
+    if (warp >= ktiles) return;
+    float d[4][4] = {}, e[4][4] = {};
+#pragma unroll 2
+    for (int c0 = 0; c0 < N; c0 += 8) {
+        const int ca = c0 + t, cb = c0 + t + 4;
+        float a[4];
+        a[0] = ca < N ? dys[g * ldd + ca] : 0.f;
+        a[1] = ca < N ? dys[(g + 8) * ldd + ca] : 0.f;
+        a[2] = cb < N ? dys[g * ldd + cb] : 0.f;
+        a[3] = cb < N ? dys[(g + 8) * ldd + cb] : 0.f;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const int k = 4 * kg + j;
-            if (k >= K) break;
-            float y0 = a0[j], y1 = a1[j];
-            if (prev) {
-                if (!(prev[r0 * ldp + k] > 0.f)) y0 = 0.f;
-                if (!(prev[(r0 + 1) * ldp + k] > 0.f)) y1 = 0.f;
+            const int kt = warp + 8 * j;
+            if (kt < ktiles) {
+                const int k = kt * 8 + g;
+                float b[2];
+                b[0] = ca < N ? ws[ca * ldw + k] : 0.f;
+                b[1] = cb < N ? ws[cb * ldw + k] : 0.f;
+                mma_3xtf32(d[j], e[j], a, b);
             }
-            os[r0 * ldo + k] = y0;
-            os[(r0 + 1) * ldo + k] = y1;
-            if (og) {
-                if (r0 < nrows) og[(long long)r0 * ldog + k] = y0;
-                if (r0 + 1 < nrows) og[(long long)(r0 + 1) * ldog + k] = y1;
-            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int kt = warp + 8 * j;
+        if (kt >= ktiles) break;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int r = g + 8 * (q >> 1), k = kt * 8 + 2 * t + (q & 1);
+            if (k >= K) continue;
+            float v = d[j][q] + e[j][q];
+            if (prev && !(prev[r * ldp + k] > 0.f)) v = 0.f;
+            os[r * ldo + k] = v;
+            if (og && r < nrows) og[(long long)r * ldog + k] = v;
         }
     }
 }
 
-// Partial gradient of one layer over the tile's rows, [W | b] flat:
-// part[o*in + k] = sum_r D[r][o] X[r][k] and part[out*in + o] = sum_r D[r][o],
-// in 4 x 4 register blocks fed by 16-byte loads.  Rows beyond the batch hold
-// D = 0; columns past out / in in the tiles are never stored.
+// Partial gradient of one layer over the tile's 16 rows, [W | b] flat:
+// part[o*in + k] = sum_r D[r][o] X[r][k] (16-output x 8-input MMA tiles, K = 16
+// rows in two steps) and part[out*in + o] = sum_r D[r][o].  Rows beyond the
+// batch hold D = 0; smem columns past out / in are masked.
 __device__ void tile_partial(const float* Ds, int ldd, const float* Xs, int ldx, int out, int in,
                              float* __restrict__ part) {
-    const int o4 = (out + 3) / 4, i4 = (in + 3) / 4;
-    for (int u = threadIdx.x; u < o4 * i4; u += NT) {
-        const int ob = u / i4, ib = u - ob * i4;
-        float acc[4][4] = {};
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
+    const int mt = (out + 15) / 16, nt = (in + 7) / 8;
+    for (int it = warp; it < mt * nt; it += NT / 32) {
+        const int o0 = (it / nt) * 16, i0 = (it % nt) * 8;
+        const int oa = o0 + g, ob = o0 + g + 8, i = i0 + g;
+        float d[4] = {0.f, 0.f, 0.f, 0.f}, e[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const float4 d = *reinterpret_cast<const float4*>(Ds + r * ldd + 4 * ob);
-            const float4 x = *reinterpret_cast<const float4*>(Xs + r * ldx + 4 * ib);
-            const float dv[4] = {d.x, d.y, d.z, d.w}, xv[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(dv[i], xv[j], acc[i][j]);
+        for (int r0 = 0; r0 < R; r0 += 8) {
+            const float* d0 = Ds + (r0 + t) * ldd;
+            const float* d1 = Ds + (r0 + t + 4) * ldd;
+            float a[4], b[2];
+            a[0] = oa < out ? d0[oa] : 0.f;
+            a[1] = ob < out ? d0[ob] : 0.f;
+            a[2] = oa < out ? d1[oa] : 0.f;
+            a[3] = ob < out ? d1[ob] : 0.f;
+            b[0] = i < in ? Xs[(r0 + t) * ldx + i] : 0.f;
+            b[1] = i < in ? Xs[(r0 + t + 4) * ldx + i] : 0.f;
+            mma_3xtf32(d, e, a, b);
         }
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int o = 4 * ob + i;
-            if (o >= out) break;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int k = 4 * ib + j;
-                if (k < in) part[(long long)o * in + k] = acc[i][j];
-            }
+        for (int q = 0; q < 4; ++q) {
+            const int o = o0 + g + 8 * (q >> 1), k = i0 + 2 * t + (q & 1);
+            if (o < out && k < in) part[(long long)o * in + k] = d[q] + e[q];
         }
     }
     for (int o = threadIdx.x; o < out; o += NT) {
@@ -196,7 +261,6 @@ __device__ void reduce_and_sgd(const FusedStepArgs& a, int nl, int ntiles) {
             L.Wm[idx] = w;
             const long long o = idx / L.in, k = idx - o * L.in;
             L.Wc[o * L.in_ld + k] = w;
-            L.Wtc[k * L.out_ld + o] = w;
         } else {
             const long long o = idx - nw;
             L.gb[o] = g;
@@ -213,26 +277,40 @@ __global__ void __launch_bounds__(NT) fused_passive_fwd_kernel(const FusedChainA
     float* ws = smem;
     float* buf0 = smem + a.w_floats;
     float* buf1 = buf0 + R * a.act_ld;
-    for (int l = 0; l < a.nl; ++l) stage_layer_weights(ws, a.L[l]);
     const int ntiles = (a.rows + R - 1) / R;
+    bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
         __syncthreads();
         async_rows(buf0, a.act_ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)a.L[0].in_ld, nr);
-        cp_wait_all();
-        __syncthreads();
+        if (first) {
+            // group l holds layer l's weights (group 0 also the first tile), so layer l only
+            // waits for its own weights while the later ones are still arriving
+            for (int l = 0; l < a.nl; ++l) {
+                stage_layer_weights(ws, a.L[l]);
+                cp_commit();
+            }
+        } else {
+            cp_commit();
+        }
         float* cur = buf0;
         float* nxt = buf1;
         for (int l = 0; l < a.nl; ++l) {
             const FusedLayerArgs& L = a.L[l];
-            if (l) __syncthreads();
-            tile_fwd(cur, a.act_ld, L.in, ws + L.wts_off, L.out_ld, L.b, L.out, true, nxt, a.act_ld,
+            if (first)
+                cp_wait_pending(a.nl - 1 - l);
+            else if (l == 0)
+                cp_wait_pending(0);
+            else
+                __syncthreads();
+            tile_fwd(cur, a.act_ld, L.in, ws + L.ws_off, L.ws_ld, L.b, L.out, true, nxt, a.act_ld,
                      L.Y + (long long)r0 * L.ldy, L.ldy, nr);
             float* t = cur;
             cur = nxt;
             nxt = t;
         }
+        first = false;
     }
     // the last CTA to finish publishes the header after every payload write
     __syncthreads();
@@ -265,12 +343,12 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* A = a.L;
     const FusedLayerArgs* T = a.L + La;
-    for (int l = 0; l < La + Lt; ++l) stage_layer_weights(ws, a.L[l]);
     const int ea = A[La - 1].out;
     const int ep = T[0].in - ea;
     const int nout = T[Lt - 1].out;
     const int ntiles = (a.rows + R - 1) / R;
     const float inv_b = 1.0f / (float)a.rows;
+    bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
@@ -278,11 +356,23 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
         __syncthreads();
         async_rows(act(0), ldA, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
         async_rows(act(La + 1) + ea, ldA, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep, nr);
-        cp_wait_all();
-        __syncthreads();
+        if (first) {
+            // one commit group per layer, in the order the forward uses them
+            for (int l = 0; l < La + Lt; ++l) {
+                stage_layer_weights(ws, a.L[l]);
+                cp_commit();
+            }
+        } else {
+            cp_commit();
+        }
         for (int l = 0; l < La; ++l) {                                   // z^a = f_a(x^a)
-            if (l) __syncthreads();
-            tile_fwd(act(l), ldA, A[l].in, ws + A[l].wts_off, A[l].out_ld, A[l].b, A[l].out, true, act(l + 1), ldA,
+            if (first)
+                cp_wait_pending(La + Lt - 1 - l);
+            else if (l == 0)
+                cp_wait_pending(0);
+            else
+                __syncthreads();
+            tile_fwd(act(l), ldA, A[l].in, ws + A[l].ws_off, A[l].ws_ld, A[l].b, A[l].out, true, act(l + 1), ldA,
                      A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr);
         }
         __syncthreads();
@@ -291,8 +381,11 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             act(La + 1)[r * ldA + c] = act(La)[r * ldA + c];
         }
         for (int l = 0; l < Lt; ++l) {                                   // y_hat = g(z^a, z^p)
-            __syncthreads();
-            tile_fwd(act(La + 1 + l), ldA, T[l].in, ws + T[l].wts_off, T[l].out_ld, T[l].b, T[l].out, l < Lt - 1,
+            if (first)
+                cp_wait_pending(Lt - 1 - l);
+            else
+                __syncthreads();
+            tile_fwd(act(La + 1 + l), ldA, T[l].in, ws + T[l].ws_off, T[l].ws_ld, T[l].b, T[l].out, l < Lt - 1,
                      act(La + 2 + l), ldA, T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr);
         }
         __syncthreads();
@@ -329,10 +422,10 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             __syncthreads();
             tile_partial(gin, ldA, act(La + 1 + l), ldA, T[l].out, T[l].in, part + T[l].poff);
             if (l > 0)
-                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].in_ld, T[l].in, act(La + 1 + l), ldA, gout, ldA,
+                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, act(La + 1 + l), ldA, gout, ldA,
                         T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr);
             else
-                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].in_ld, T[l].in, nullptr, 0, gout, ldA, nullptr, 0,
+                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, nullptr, 0, gout, ldA, nullptr, 0,
                         nr);
             float* t = gin;
             gin = gout;
@@ -357,14 +450,16 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             __syncthreads();
             tile_partial(gin, ldA, act(l), ldA, A[l].out, A[l].in, part + A[l].poff);
             if (l > 0) {
-                tile_dx(gin, ldA, A[l].out, ws + A[l].ws_off, A[l].in_ld, A[l].in, act(l), ldA, gout, ldA,
+                tile_dx(gin, ldA, A[l].out, ws + A[l].ws_off, A[l].ws_ld, A[l].in, act(l), ldA, gout, ldA,
                         A[l - 1].D + (long long)r0 * A[l - 1].ldd, A[l - 1].ldd, nr);
                 float* t = gin;
                 gin = gout;
                 gout = t;
             }
         }
+        first = false;
     }
+    if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
     grid.sync();
     reduce_and_sgd(a, La + Lt, ntiles);
     if (blockIdx.x == 0) {
@@ -401,9 +496,9 @@ __global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepAr
     float* g1 = act(Lp + 2);
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* P = a.L;
-    for (int l = 1; l < Lp; ++l) stage_layer_weights(ws, P[l]);
     const int ep = P[Lp - 1].out;
     const int ntiles = (a.rows + R - 1) / R;
+    bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
@@ -413,8 +508,15 @@ __global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepAr
         for (int l = 0; l < Lp; ++l)
             async_rows(act(l + 1), ldA, P[l].Y + (long long)r0 * P[l].ldy, P[l].ldy, (int)P[l].out_ld, nr);
         async_rows(g1, ldA, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
-        cp_wait_all();
-        __syncthreads();
+        cp_commit();
+        if (first) {
+            // weights in the order the backward uses them: layer Lp-1 first
+            for (int l = Lp - 1; l >= 1; --l) {
+                stage_layer_weights(ws, P[l]);
+                cp_commit();
+            }
+        }
+        cp_wait_pending(first ? Lp - 1 : 0);
         for (int i = threadIdx.x; i < R * ep; i += NT) {                 // dz^p * [z^p > 0]
             const int r = i / ep, c = i - r * ep;
             const float v = act(Lp)[r * ldA + c] > 0.f ? g1[r * ldA + c] : 0.f;
@@ -427,14 +529,17 @@ __global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepAr
             __syncthreads();
             tile_partial(gin, ldA, act(l), ldA, P[l].out, P[l].in, part + P[l].poff);
             if (l > 0) {
-                tile_dx(gin, ldA, P[l].out, ws + P[l].ws_off, P[l].in_ld, P[l].in, act(l), ldA, gout, ldA,
+                if (first) cp_wait_pending(l - 1);   // this layer's weights
+                tile_dx(gin, ldA, P[l].out, ws + P[l].ws_off, P[l].ws_ld, P[l].in, act(l), ldA, gout, ldA,
                         P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr);
                 float* t = gin;
                 gin = gout;
                 gout = t;
             }
         }
+        first = false;
     }
+    if (first) cp_wait_pending(0);
     grid.sync();
     reduce_and_sgd(a, Lp, ntiles);
 }

@@ -352,15 +352,6 @@ __global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ld
     }
 }
 
-__global__ void transpose_f32_kernel(const float* __restrict__ src, int out, int in, float* __restrict__ dst,
-                                     long long ldt) {
-    const long long n = (long long)out * in;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
-        const long long o = i / in, k = i % in;
-        dst[k * ldt + o] = src[i];
-    }
-}
-
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
     const long long n = (long long)rows * cols;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
@@ -451,11 +442,6 @@ cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int b
     if (nblocks < 1) return cudaErrorInvalidValue;
     dim3 grid((out + 255) / 256, nblocks);
     colsum_kernel<<<grid, 256, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s) {
-    transpose_f32_kernel<<<grid_for((long long)out * in, 256), 256, 0, s>>>(src, out, in, dst, ldt);
     return cudaGetLastError();
 }
 

@@ -11,20 +11,24 @@ constexpr int kFusedMaxWidth = 256;            // widest layer input or output
 constexpr int kFusedMaxLayers = 16;
 constexpr size_t kFusedMaxSmem = 227 * 1024;
 
+// shared-memory row stride >= width, = 4 mod 32 (the MMA A fragments and the
+// forward's B fragments read 8 rows x 4 columns conflict-free), a 16-byte multiple
+inline int fused_act_stride(long long width) { return (int)(((width + 27) / 32) * 32 + 4); }
+inline int fused_w_stride(long long ld) { return fused_act_stride(ld); }
+
 struct FusedLayerArgs {
     int in, out;
     long long in_ld;         // row stride of W copies
-    long long out_ld;        // row stride of W^T copies
+    long long out_ld;        // row stride of activations this layer writes
     const float* W;          // weight version read by this step, [out, in_ld]
-    const float* Wt;         // the same version transposed, [in, out_ld]
     const float* b;
-    int ws_off, wts_off;     // shared-memory offsets (floats) of W and W^T, -1 when not staged
+    int ws_off;              // shared-memory offset (floats) of W, -1 when not staged
+    int ws_ld;               // its shared-memory row stride (= 4 mod 32)
     float* Y; long long ldy; // forward output rows of this step (global)
     float* D; long long ldd; // d(pre-activation) rows of this step (global), written in phase 1
     long long poff;          // offset of this layer's [W | b] gradient in the flat parameter vector
     float* Wm; float* bm;    // fp32 master (SGD)
     float* Wc; float* bc;    // copy of the new version
-    float* Wtc;              // transposed copy of the new version
     float* gW; float* gb;    // reduced gradient (read back by vfl_get_grads)
 };
 

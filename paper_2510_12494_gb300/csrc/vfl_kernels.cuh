@@ -97,9 +97,6 @@ cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long 
 cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
                           int nblocks, cudaStream_t s);
 
-// dst[k * ldt + o] = src[o * in + k] for src [out, in] fp32.
-cudaError_t launch_transpose_f32(const float* src, int out, int in, float* dst, long long ldt, cudaStream_t s);
-
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);
 

@@ -64,7 +64,6 @@ struct Layer {
     float* b = nullptr;                   // fp32 master [out]
     void* cW[kMaxSlots] = {};             // version copies [out, in_ld], compute dtype
     float* cb[kMaxSlots] = {};            // version copies of b, fp32
-    float* cWt[kMaxSlots] = {};           // fused path: transposed version copies [in, ld8(out)], fp32
     float* pW[kMaxWorkers] = {};          // split-K partial dW [nsplit][out*in]
     float* pb[kMaxWorkers] = {};          // partial db [nsplit][out]
     int nsplit = 1;                       // weight-gradient partials
@@ -284,18 +283,16 @@ bool fused_eligible(const vfl_config& c) {
 
 // Shared-memory layout of one fused launch: which layers stage W (for input
 // gradients) and W^T (for the forward).  Returns the floats used.
-int fused_weight_layout(FusedLayerArgs* L, int n, bool want_wt, int w_from, int w_layer0) {
+// Shared-memory layout of the weights one fused launch stages: layers
+// [w_from, n) get W.  Returns the floats used.
+int fused_weight_layout(FusedLayerArgs* L, int n, int w_from) {
     int off = 0;
     for (int l = 0; l < n; ++l) {
-        L[l].wts_off = -1;
+        L[l].ws_ld = fused_w_stride(L[l].in_ld);
         L[l].ws_off = -1;
-        if (want_wt) {
-            L[l].wts_off = off;
-            off += (int)(L[l].in * L[l].out_ld);
-        }
-        if (l >= w_from && (l > 0 || w_layer0)) {
+        if (l >= w_from) {
             L[l].ws_off = off;
-            off += (int)(L[l].out * L[l].in_ld);
+            off += L[l].out * L[l].ws_ld;
         }
     }
     return off;
@@ -352,27 +349,22 @@ void build_layers(vfl_ctx* ctx) {
                 maxw = std::max(maxw, std::max(L.in, L.out));
                 ctx->f_ptotal_a += (long long)L.out * L.in + L.out;
             }
-        ctx->f_act_ld = (int)ld8(maxw);
-        // staged weights per launch: forward W^T of every layer; input-gradient W of every top layer and
-        // of every bottom layer but the first
-        long long wt_p = 0, w_p = 0, wt_a = 0, w_a = 0;
+        ctx->f_act_ld = fused_act_stride(ld8(maxw));
+        // staged weights per launch (row-major W): every layer of f_p for the forward, every layer of
+        // f_a and g for the active step, f_p's layers after the first for the backward
+        long long w_pf = 0, w_pb = 0, w_a = 0;
         for (size_t l = 0; l < ctx->P.size(); ++l) {
-            wt_p += (long long)ctx->P[l].in * ld8(ctx->P[l].out);
-            if (l > 0) w_p += (long long)ctx->P[l].out * ctx->P[l].in_ld;
+            const long long w = (long long)ctx->P[l].out * fused_w_stride(ctx->P[l].in_ld);
+            w_pf += w;
+            if (l > 0) w_pb += w;
         }
-        for (size_t l = 0; l < ctx->A.size(); ++l) {
-            wt_a += (long long)ctx->A[l].in * ld8(ctx->A[l].out);
-            if (l > 0) w_a += (long long)ctx->A[l].out * ctx->A[l].in_ld;
-        }
-        for (const Layer& L : ctx->T) {
-            wt_a += (long long)L.in * ld8(L.out);
-            w_a += (long long)L.out * L.in_ld;
-        }
-        ctx->f_wp = (int)std::max(wt_p, w_p);
-        ctx->f_wa = (int)(wt_a + w_a);
+        for (auto* v : {&ctx->A, &ctx->T})
+            for (const Layer& L : *v) w_a += (long long)L.out * fused_w_stride(L.in_ld);
+        ctx->f_wp = (int)std::max(w_pf, w_pb);
+        ctx->f_wa = (int)w_a;
         const size_t sa = fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size());
-        const size_t sp = fused_smem_pbwd((int)w_p, ctx->f_act_ld, (int)ctx->P.size());
-        const size_t sf = fused_smem_fwd((int)wt_p, ctx->f_act_ld);
+        const size_t sp = fused_smem_pbwd((int)w_pb, ctx->f_act_ld, (int)ctx->P.size());
+        const size_t sf = fused_smem_fwd((int)w_pf, ctx->f_act_ld);
         if (std::max(sa, std::max(sp, sf)) > kFusedMaxSmem) ctx->fused = false;
     }
 }
@@ -399,7 +391,6 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             for (int s = 0; s < ctx->S1; ++s) {
                 L.cW[s] = cv.take((unsigned long long)L.out * L.in_ld * es);
                 L.cb[s] = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
-                if (ctx->fused) L.cWt[s] = static_cast<float*>(cv.take((unsigned long long)L.in * ld8(L.out) * 4));
             }
             for (int w = 0; w < ctx->W; ++w) {
                 L.pW[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * L.in * 4));
@@ -641,7 +632,6 @@ FusedLayerArgs fused_layer(const Layer& L, int vslot, int new_slot, int w, void*
     f.in_ld = L.in_ld;
     f.out_ld = ld8(L.out);
     f.W = static_cast<const float*>(L.cW[vslot]);
-    f.Wt = L.cWt[vslot];
     f.b = L.cb[vslot];
     f.Y = static_cast<float*>(Y);
     f.ldy = ldy;
@@ -651,7 +641,6 @@ FusedLayerArgs fused_layer(const Layer& L, int vslot, int new_slot, int w, void*
     f.Wm = L.W;
     f.bm = L.b;
     f.Wc = static_cast<float*>(L.cW[new_slot]);
-    f.Wtc = L.cWt[new_slot];
     f.bc = L.cb[new_slot];
     f.gW = L.pW[w];
     f.gb = L.pb[w];
@@ -680,7 +669,7 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     a.ldx = ctx->ldxp;
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
-    a.w_floats = fused_weight_layout(a.L, a.nl, true, 1 << 30, 0);
+    a.w_floats = fused_weight_layout(a.L, a.nl, 0);
     a.counter = ctx->f_counter;
     a.hdr = ctx->emb_hdr + slot;
     a.k = k;
@@ -718,22 +707,7 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     a.nt = Lt;
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
-    {
-        // W^T of every layer, then W of f_a's layers after the first and of every layer of g
-        int off = 0;
-        for (int l = 0; l < La + Lt; ++l) {
-            a.L[l].wts_off = off;
-            off += (int)(a.L[l].in * a.L[l].out_ld);
-        }
-        for (int l = 0; l < La + Lt; ++l) {
-            a.L[l].ws_off = -1;
-            if (l >= La || l > 0) {
-                a.L[l].ws_off = off;
-                off += (int)(a.L[l].out * a.L[l].in_ld);
-            }
-        }
-        a.w_floats = off;
-    }
+    a.w_floats = fused_weight_layout(a.L, La + Lt, 0);
     a.x = Xa;
     a.ldx = ctx->ldxa;
     long long r0;
@@ -786,7 +760,7 @@ vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot
     a.nt = 0;
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
-    a.w_floats = fused_weight_layout(a.L, Lp, false, 1, 0);
+    a.w_floats = fused_weight_layout(a.L, Lp, 1);
     a.x = Xp;
     a.ldx = ctx->ldxp;
     a.gradp = static_cast<float*>(ctx->grad[slot]);
@@ -1114,7 +1088,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     if (e == cudaSuccess) e = cudaMemset(ctx->grad_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
     if (e == cudaSuccess && ctx->fused) {
         long long w_p = 0;
-        for (size_t l = 1; l < ctx->P.size(); ++l) w_p += (long long)ctx->P[l].out * ctx->P[l].in_ld;
+        for (size_t l = 1; l < ctx->P.size(); ++l) w_p += (long long)ctx->P[l].out * fused_w_stride(ctx->P[l].in_ld);
         e = fused_max_grid(0, fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size()),
                            &ctx->f_grid_a);
         if (e == cudaSuccess)
@@ -1226,10 +1200,6 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
     for (int s = 0; s < ctx->S1; ++s) {
         CK(cudaMemset(L->cW[s], 0, (size_t)L->out * L->in_ld * ctx->esz));
         PLAUNCH(K_CAST, 0, 0, 0, launch_cast_rows(L->W, L->out, L->in, L->cW[s], L->in_ld, ctx->bf16, 0));
-        if (L->cWt[s]) {
-            CK(cudaMemset(L->cWt[s], 0, (size_t)L->in * ld8(L->out) * 4));
-            PLAUNCH(K_CAST, 0, 0, 0, launch_transpose_f32(L->W, L->out, L->in, L->cWt[s], ld8(L->out), 0));
-        }
         CK(cudaMemcpy(L->cb[s], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
     }
     CK(cudaDeviceSynchronize());
@@ -1333,11 +1303,6 @@ vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
     CK(cudaMemset(L->cW[slot], 0, (size_t)L->out * L->in_ld * ctx->esz));
     ++ctx->launches;
     CK(launch_cast_rows(tmp, L->out, L->in, L->cW[slot], L->in_ld, ctx->bf16, 0));
-    if (L->cWt[slot]) {
-        CK(cudaMemset(L->cWt[slot], 0, (size_t)L->in * ld8(L->out) * 4));
-        ++ctx->launches;
-        CK(launch_transpose_f32(tmp, L->out, L->in, L->cWt[slot], ld8(L->out), 0));
-    }
     CK(cudaMemcpy(L->cb[slot], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
     if (v == k) {
         CK(cudaMemcpy(L->W, W, nw * 4, cudaMemcpyHostToDevice));
