@@ -200,6 +200,22 @@ vfl_status vfl_passive_backward(vfl_ctx* ctx, int64_t k);
 vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
                            const int32_t* tau_a);
 
+/*
+ * CUDA-graph replay of a window of steps.  vfl_graph_capture records steps
+ * [k0, k0 + n_steps) -- the same kernels and cross-stream events
+ * vfl_train_steps would enqueue -- into an executable graph without running
+ * them; the context must be idle at cursor k0 and stays there.
+ * vfl_graph_launch replays it once (the context must be at cursor k0), ordered
+ * after all work already on the context's streams, and advances the cursor to
+ * k0 + n_steps.  Capture needs caller streams (vfl_set_streams) and per-launch
+ * timing off.  A graph belongs to one context; destroy it before the context.
+ */
+typedef struct vfl_graph vfl_graph;
+vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
+                             const int32_t* tau_a, vfl_graph** out);
+vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* graph);
+vfl_status vfl_graph_destroy(vfl_graph* graph);
+
 /* Wait for all enqueued work; returns VFL_E_VERSION / VFL_E_TIMEOUT recorded by kernels. */
 vfl_status vfl_synchronize(vfl_ctx* ctx);
 

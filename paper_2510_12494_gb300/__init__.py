@@ -76,6 +76,10 @@ EXPORTS = {
     "vfl_passive_backward": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
     "vfl_train_steps": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
                                          ctypes.c_void_p]),
+    "vfl_graph_capture": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+                                           ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
+    "vfl_graph_launch": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_graph_destroy": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_synchronize": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_read_losses": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_tap": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p]),
@@ -202,6 +206,9 @@ class Context:
 
     def close(self):
         if getattr(self, "h", None):
+            for g in getattr(self, "_graphs", []):
+                lib().vfl_graph_destroy(g)
+            self._graphs = []
             lib().vfl_destroy(self.h)
             self.h = None
 
@@ -317,6 +324,19 @@ class Context:
         tau_a = np.ascontiguousarray(tau_a, np.int32)
         assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
         self._call(lib().vfl_train_steps, k0, n, _ptr(tau_p), _ptr(tau_a))
+
+    def capture(self, k0, n, tau_p, tau_a):
+        """A CUDA graph of steps [k0, k0+n) (see vfl_graph_capture); replay with launch_graph."""
+        tau_p = np.ascontiguousarray(tau_p, np.int32)
+        tau_a = np.ascontiguousarray(tau_a, np.int32)
+        assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
+        g = ctypes.c_void_p()
+        self._call(lib().vfl_graph_capture, k0, n, _ptr(tau_p), _ptr(tau_a), ctypes.byref(g))
+        self._graphs = getattr(self, "_graphs", []) + [g]
+        return g
+
+    def launch_graph(self, g):
+        self._call(lib().vfl_graph_launch, g)
 
     def synchronize(self):
         self._call(lib().vfl_synchronize)

@@ -149,6 +149,11 @@ struct vfl_ctx {
     long long grad_step[kMaxSlots];
     long long last_act_step[kMaxWorkers];
     bool started = false;
+    // every weight version <= ordered_floor is already ordered before all further work on the
+    // context's streams (the context was idle, or a graph replay ended with every stream waiting on
+    // it), so waits on the events that produced those versions are skipped -- those events may have
+    // been recorded inside a graph capture, where they cannot be waited on from outside
+    long long ordered_floor = -1;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
         char buf[512];
@@ -168,6 +173,50 @@ struct vfl_ctx {
         *r0 = j * cfg.batch;
         return (int)std::min<long long>(cfg.batch, n_rows - *r0);
     }
+};
+
+// Host-side ordering state of a context (saved around graph capture).
+struct HostState {
+    long long n_fwd, n_act, n_bwd;
+    int fwd_version[kMaxSlots];
+    long long slot_step_p[kMaxSlots], grad_step[kMaxSlots], last_act_step[kMaxWorkers];
+    bool started;
+    long long launches;
+};
+
+static HostState save_state(const vfl_ctx* c) {
+    HostState h;
+    h.n_fwd = c->n_fwd;
+    h.n_act = c->n_act;
+    h.n_bwd = c->n_bwd;
+    std::memcpy(h.fwd_version, c->fwd_version, sizeof h.fwd_version);
+    std::memcpy(h.slot_step_p, c->slot_step_p, sizeof h.slot_step_p);
+    std::memcpy(h.grad_step, c->grad_step, sizeof h.grad_step);
+    std::memcpy(h.last_act_step, c->last_act_step, sizeof h.last_act_step);
+    h.started = c->started;
+    h.launches = c->launches;
+    return h;
+}
+
+static void load_state(vfl_ctx* c, const HostState& h) {
+    c->n_fwd = h.n_fwd;
+    c->n_act = h.n_act;
+    c->n_bwd = h.n_bwd;
+    std::memcpy(c->fwd_version, h.fwd_version, sizeof h.fwd_version);
+    std::memcpy(c->slot_step_p, h.slot_step_p, sizeof h.slot_step_p);
+    std::memcpy(c->grad_step, h.grad_step, sizeof h.grad_step);
+    std::memcpy(c->last_act_step, h.last_act_step, sizeof h.last_act_step);
+    c->started = h.started;
+    c->launches = h.launches;
+}
+
+struct vfl_graph {
+    vfl_ctx* ctx;
+    cudaGraphExec_t exec;
+    long long k0, n;
+    HostState after;           // host state once the captured steps have run
+    long long launches;        // kernels per replay
+    cudaEvent_t fork, join[2 * kMaxWorkers];
 };
 
 #define CK(call)                                                     \
@@ -799,7 +848,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const int vslot = (int)(v % ctx->S1);
     long long r0;
     const int rows = ctx->batch_rows(k, &r0);
-    if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
+    if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
     const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
     if (ctx->fused) {
         TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), s));
@@ -845,11 +894,11 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const int ea = ctx->A.back().out, ep = ctx->P.back().out;
     const int n_out = ctx->T.back().out;
 
-    if (v > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
+    if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
     const void* Xa0 = static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * es;
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
-        if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
         TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), s));
         CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
         CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
@@ -931,7 +980,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         }
     }
     // SGD on theta_1 in step order: version k+1 from version k
-    if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+    if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
     TRY(sgd(ctx, &ctx->A, &ctx->T, w, (int)((k + 1) % ctx->S1), s));
     CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
     ctx->last_act_step[w] = k;
@@ -952,7 +1001,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
     if (ctx->fused) {
-        if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
         const float* Xp = reinterpret_cast<const float*>(static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz);
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, Xp, s));
         CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
@@ -976,7 +1025,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
                           ctx->act_p[slot][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
     }
-    if (k > 0) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+    if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
     TRY(sgd(ctx, &ctx->P, nullptr, w, (int)((k + 1) % ctx->S1), s));
     CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
     ctx->n_bwd = k + 1;
@@ -1259,6 +1308,7 @@ vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k) {
         return ctx->fail(VFL_E_STATE, "vfl_set_cursor with steps in flight");
     TRY(sync_all(ctx));
     ctx->n_fwd = ctx->n_act = ctx->n_bwd = k;
+    ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k);
     for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
     for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
     ctx->started = true;
@@ -1399,6 +1449,109 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
         }
         if (!progressed) return ctx->fail(VFL_E_STATE, "schedule cannot make progress at step %lld", ctx->n_bwd);
     }
+    return VFL_OK;
+}
+
+vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
+                             vfl_graph** out) {
+    if (!ctx || !out) return VFL_E_INVAL;
+    *out = nullptr;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->prof_on) return ctx->fail(VFL_E_STATE, "vfl_graph_capture while per-launch timing is on");
+    for (int w = 0; w < ctx->W; ++w)
+        if (!ctx->ps[w] || !ctx->as[w])
+            return ctx->fail(VFL_E_STATE, "graph capture needs the caller's streams (vfl_set_streams)");
+    if (k0 != ctx->n_fwd || k0 != ctx->n_act || k0 != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_graph_capture(%lld): steps before k0 are not all enqueued", (long long)k0);
+    TRY(sync_all(ctx));
+    vfl_graph* g = new vfl_graph();
+    g->ctx = ctx;
+    g->k0 = k0;
+    g->n = n_steps;
+    cudaError_t e = cudaEventCreateWithFlags(&g->fork, cudaEventDisableTiming);
+    for (int i = 0; i < 2 * ctx->W && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        delete g;
+        return ctx->cuda(e, "cudaEventCreate", __LINE__);
+    }
+    const HostState before = save_state(ctx);
+    cudaStream_t origin = ctx->ps[0];
+    cudaGraph_t graph = nullptr;
+    vfl_status st = VFL_OK;
+    e = cudaStreamBeginCapture(origin, cudaStreamCaptureModeThreadLocal);
+    if (e == cudaSuccess) e = cudaEventRecord(g->fork, origin);
+    for (int w = 0; w < ctx->W && e == cudaSuccess; ++w) {
+        if (w > 0) e = cudaStreamWaitEvent(ctx->ps[w], g->fork, 0);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->as[w], g->fork, 0);
+    }
+    const long long floor_before = ctx->ordered_floor;
+    ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k0);
+    if (e == cudaSuccess) st = vfl_train_steps(ctx, k0, n_steps, tau_p, tau_a);
+    ctx->ordered_floor = floor_before;
+    // join every stream back into the origin, even after a failure, so that capture can end
+    int j = 0;
+    for (int w = 0; w < ctx->W; ++w) {
+        cudaStream_t ss[2] = {ctx->ps[w], ctx->as[w]};
+        for (cudaStream_t x : ss) {
+            if (x == origin) continue;
+            if (cudaEventRecord(g->join[j], x) == cudaSuccess) cudaStreamWaitEvent(origin, g->join[j], 0);
+            ++j;
+        }
+    }
+    cudaError_t e2 = cudaStreamEndCapture(origin, &graph);
+    if (e == cudaSuccess) e = e2;
+    const HostState after = save_state(ctx);
+    load_state(ctx, before);
+    if (st == VFL_OK && e == cudaSuccess) e = cudaGraphInstantiate(&g->exec, graph, 0);
+    if (graph) cudaGraphDestroy(graph);
+    if (st != VFL_OK || e != cudaSuccess) {
+        vfl_graph_destroy(g);
+        if (st != VFL_OK) return st;
+        return ctx->cuda(e, "graph capture", __LINE__);
+    }
+    g->after = after;
+    g->launches = after.launches - before.launches;
+    *out = g;
+    return VFL_OK;
+}
+
+vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* g) {
+    if (!ctx || !g || g->ctx != ctx) return ctx ? ctx->fail(VFL_E_INVAL, "graph of another context") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->n_fwd != g->k0 || ctx->n_act != g->k0 || ctx->n_bwd != g->k0)
+        return ctx->fail(VFL_E_STATE, "graph starts at step %lld but the context is at step %lld", g->k0, ctx->n_fwd);
+    cudaStream_t origin = ctx->ps[0];
+    // order the replay after everything already enqueued on the context's streams, and theirs after it
+    int j = 0;
+    for (int w = 0; w < ctx->W; ++w) {
+        cudaStream_t ss[2] = {ctx->ps[w], ctx->as[w]};
+        for (cudaStream_t x : ss) {
+            if (x == origin) continue;
+            CK(cudaEventRecord(g->join[j], x));
+            CK(cudaStreamWaitEvent(origin, g->join[j], 0));
+            ++j;
+        }
+    }
+    CK(cudaGraphLaunch(g->exec, origin));
+    CK(cudaEventRecord(g->fork, origin));
+    for (int w = 0; w < ctx->W; ++w) {
+        if (w > 0) CK(cudaStreamWaitEvent(ctx->ps[w], g->fork, 0));
+        CK(cudaStreamWaitEvent(ctx->as[w], g->fork, 0));
+    }
+    const long long launched = ctx->launches + g->launches;
+    load_state(ctx, g->after);
+    ctx->launches = launched;
+    ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, g->k0 + g->n);
+    return VFL_OK;
+}
+
+vfl_status vfl_graph_destroy(vfl_graph* g) {
+    if (!g) return VFL_OK;
+    if (g->exec) cudaGraphExecDestroy(g->exec);
+    if (g->fork) cudaEventDestroy(g->fork);
+    for (cudaEvent_t e : g->join)
+        if (e) cudaEventDestroy(e);
+    delete g;
     return VFL_OK;
 }
 

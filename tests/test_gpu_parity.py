@@ -180,3 +180,46 @@ def test_step_parity_generic_kernels(vfl, cid, monkeypatch):
     monkeypatch.setenv("VFL_DISABLE_FUSED", "1")
     worst, failures = run_sequential(vfl, cid, CASES[cid])
     assert not failures, f"preset {cid}: {failures[:3]}"
+
+
+@pytest.mark.parametrize("cid", [2, 3])
+def test_graph_replay_equals_direct_enqueue(vfl, cid):
+    """A captured CUDA graph of a window of steps replays exactly what the
+    direct enqueue computes, advances the cursor, and refuses the wrong cursor."""
+    import synth
+    p = synth.preset(cid)
+    q, xp, xa, y, params = setup(p, CASES[cid])
+    n = q.steps_per_epoch + 2
+    tp, ta = schedule(q, 2 * n)
+    direct = new_context(vfl, q, xp, xa, y, params)
+    direct.train_steps(0, 2 * n, tp, ta)
+    g_ctx = new_context(vfl, q, xp, xa, y, params)
+    g0 = g_ctx.capture(0, n, tp, ta)
+    assert g_ctx.cursor() == 0                      # capture does not run anything
+    g_ctx.launch_graph(g0)
+    with pytest.raises(vfl.VflError) as ei:
+        g_ctx.launch_graph(g0)                      # cursor is now n, the graph starts at 0
+    assert ei.value.status == vfl.VFL_E_STATE
+    g1 = g_ctx.capture(n, n, tp, ta)
+    g_ctx.launch_graph(g1)
+    assert g_ctx.cursor() == 2 * n
+    np.testing.assert_array_equal(g_ctx.read_losses(0, 2 * n), direct.read_losses(0, 2 * n))
+    for key, (W, b) in direct.get_params().items():
+        Wg, bg = g_ctx.get_params()[key]
+        np.testing.assert_array_equal(W, Wg)
+        np.testing.assert_array_equal(b, bg)
+
+
+def test_direct_enqueue_after_graph_replay(vfl):
+    """Direct phase calls continue exactly after a graph replay."""
+    import synth
+    q, xp, xa, y, params = setup(synth.preset(2), CASES[2])
+    n = q.steps_per_epoch
+    tp, ta = schedule(q, 3 * n)
+    direct = new_context(vfl, q, xp, xa, y, params)
+    direct.train_steps(0, 3 * n, tp, ta)
+    mixed = new_context(vfl, q, xp, xa, y, params)
+    mixed.launch_graph(mixed.capture(0, n, tp, ta))
+    mixed.train_steps(n, n, tp, ta)
+    mixed.launch_graph(mixed.capture(2 * n, n, tp, ta))
+    np.testing.assert_array_equal(mixed.read_losses(0, 3 * n), direct.read_losses(0, 3 * n))
