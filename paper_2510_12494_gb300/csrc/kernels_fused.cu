@@ -22,7 +22,7 @@ namespace vfl {
 
 namespace {
 
-constexpr int NT = kFusedThreads;     // 8 warps
+constexpr int NT = kFusedThreads;     // 16 warps
 constexpr int R = kFusedRows;
 static_assert(R == 16, "the MMA tiles cover exactly 16 rows");
 
@@ -111,97 +111,105 @@ __device__ __forceinline__ void mma_3xtf32(float* d, float* e, const float* a, c
     mma_tf32(e, ah, bl);
 }
 
-// Y[r][c] = act(sum_k X[r][k] W[c][k] + b[c]) for the 16 rows of a tile, W
-// row-major in smem.  Warp w owns the 8-column output tiles w, w+8, w+16, w+24
-// (N <= 256).  Values past K (stale smem) and rows past N are masked.
-// Fragment layout (g = lane/4, t = lane%4): A[g|g+8][t|t+4], B[t|t+4][g],
-// D[g|g+8][2t|2t+1].
-__device__ void tile_fwd(const float* xs, int ldx, int K, const float* ws, int ldw, const float* __restrict__ bias,
-                         int N, bool relu, float* ys, int ldy, float* yg, long long ldyg, int nrows) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
-    const int ntiles = (N + 7) / 8;
-    if (warp >= ntiles) return;
-    float d[4][4] = {}, e[4][4] = {};
-#pragma unroll 2
-    for (int k0 = 0; k0 < K; k0 += 8) {
+// One 16x8 output tile of  sum_k A[r][k] B[k][n]  for k in [kbeg, kend), 3xTF32.
+// A is the 16-row tile (row stride lda, columns past K masked); B[k][n] is read
+// as  bm[n * ldb_n + k * ldb_k]  (rows past N / K masked).  Accumulates into d, e.
+__device__ __forceinline__ void mma_tile_range(float* d, float* e, const float* as, int lda, int K, const float* bm,
+                                               int ldb_n, int ldb_k, int n, bool n_ok, int kbeg, int kend) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    for (int k0 = kbeg; k0 < kend; k0 += 8) {
         const int ka = k0 + t, kb = k0 + t + 4;
-        float a[4];
-        a[0] = ka < K ? xs[g * ldx + ka] : 0.f;
-        a[1] = ka < K ? xs[(g + 8) * ldx + ka] : 0.f;
-        a[2] = kb < K ? xs[g * ldx + kb] : 0.f;
-        a[3] = kb < K ? xs[(g + 8) * ldx + kb] : 0.f;
+        float a[4], b[2];
+        a[0] = ka < K ? as[g * lda + ka] : 0.f;
+        a[1] = ka < K ? as[(g + 8) * lda + ka] : 0.f;
+        a[2] = kb < K ? as[g * lda + kb] : 0.f;
+        a[3] = kb < K ? as[(g + 8) * lda + kb] : 0.f;
+        b[0] = (ka < K && n_ok) ? bm[n * ldb_n + ka * ldb_k] : 0.f;
+        b[1] = (kb < K && n_ok) ? bm[n * ldb_n + kb * ldb_k] : 0.f;
+        mma_3xtf32(d, e, a, b);
+    }
+}
+
+// C[16 x N] = A[16 x K] . B over the 16 warps of the block: output tile j (8
+// columns) goes to warp j mod 16; with at most 8 tiles the K range is split
+// between warps w and w + 8 and the second half is added through `red`
+// (fixed order).  The epilogue callback receives (row, col, value) for
+// every in-range output.
+template <typename Epi>
+__device__ void tile_gemm(const float* as, int lda, int K, const float* bm, int ldb_n, int ldb_k, int N, float* red,
+                          Epi epi) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
+    constexpr int NW = NT / 32;
+    const int ntiles = (N + 7) / 8;
+    const bool split = ntiles <= NW / 2;
+    const int ksteps = (K + 7) / 8;
+    const int khalf = ((ksteps + 1) / 2) * 8;
+    float d[2][4] = {}, e[2][4] = {};
+    int mine = 0;
+    if (split) {
+        const int j = warp % (NW / 2), half = warp / (NW / 2);
+        if (j < ntiles) {
+            const int n = j * 8 + g;
+            mma_tile_range(d[0], e[0], as, lda, K, bm, ldb_n, ldb_k, n, n < N, half ? khalf : 0, half ? K : min(K, khalf));
+            mine = 1;
+        }
+        if (mine && half) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int nt = warp + 8 * j;
-            if (nt < ntiles) {
-                const int n = nt * 8 + g;
-                const float* wr = ws + n * ldw;
-                float b[2];
-                b[0] = (ka < K && n < N) ? wr[ka] : 0.f;
-                b[1] = (kb < K && n < N) ? wr[kb] : 0.f;
-                mma_3xtf32(d[j], e[j], a, b);
-            }
+            for (int q = 0; q < 4; ++q) red[(j * 32 + lane) * 4 + q] = d[0][q] + e[0][q];
+        }
+        __syncthreads();
+        if (!mine || half) return;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) d[0][q] += e[0][q] + red[(j * 32 + lane) * 4 + q];
+        const int c0 = j * 8 + 2 * t;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int c = c0 + (q & 1);
+            if (c < N) epi(g + 8 * (q >> 1), c, d[0][q]);
+        }
+        return;
+    }
+#pragma unroll
+    for (int jj = 0; jj < 2; ++jj) {
+        const int j = warp + NW * jj;
+        if (j < ntiles) {
+            const int n = j * 8 + g;
+            mma_tile_range(d[jj], e[jj], as, lda, K, bm, ldb_n, ldb_k, n, n < N, 0, K);
         }
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int nt = warp + 8 * j;
-        if (nt >= ntiles) break;
+    for (int jj = 0; jj < 2; ++jj) {
+        const int j = warp + NW * jj;
+        if (j >= ntiles) break;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            const int r = g + 8 * (q >> 1), c = nt * 8 + 2 * t + (q & 1);
-            if (c >= N) continue;
-            float y = d[j][q] + e[j][q] + bias[c];
-            if (relu) y = fmaxf(y, 0.f);
-            ys[r * ldy + c] = y;
-            if (yg && r < nrows) yg[(long long)r * ldyg + c] = y;
+            const int c = j * 8 + 2 * t + (q & 1);
+            if (c < N) epi(g + 8 * (q >> 1), c, d[jj][q] + e[jj][q]);
         }
     }
 }
 
+// Y[r][c] = act(sum_k X[r][k] W[c][k] + b[c]) for the 16 rows of a tile (W
+// row-major in smem).  To smem (ldy) and to global rows < nrows when yg is set.
+__device__ void tile_fwd(const float* xs, int ldx, int K, const float* ws, int ldw, const float* __restrict__ bias,
+                         int N, bool relu, float* ys, int ldy, float* yg, long long ldyg, int nrows, float* red) {
+    tile_gemm(xs, ldx, K, ws, ldw, 1, N, red, [&](int r, int c, float v) {
+        float y = v + bias[c];
+        if (relu) y = fmaxf(y, 0.f);
+        ys[r * ldy + c] = y;
+        if (yg && r < nrows) yg[(long long)r * ldyg + c] = y;
+    });
+}
+
 // dX[r][k] = sum_c dY[r][c] W[c][k], zeroed where prev[r][k] <= 0 (when prev is
-// given).  Warp w owns the 8-column output tiles w + 8 j (K <= 256); the
-// reduction over c < N runs in steps of 8 (values past N masked).
+// given).  To smem and to global rows < nrows.
 __device__ void tile_dx(const float* dys, int ldd, int N, const float* ws, int ldw, int K, const float* prev, int ldp,
-                        float* os, int ldo, float* og, long long ldog, int nrows) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
-    const int ktiles = (K + 7) / 8;
-    if (warp >= ktiles) return;
-    float d[4][4] = {}, e[4][4] = {};
-#pragma unroll 2
-    for (int c0 = 0; c0 < N; c0 += 8) {
-        const int ca = c0 + t, cb = c0 + t + 4;
-        float a[4];
-        a[0] = ca < N ? dys[g * ldd + ca] : 0.f;
-        a[1] = ca < N ? dys[(g + 8) * ldd + ca] : 0.f;
-        a[2] = cb < N ? dys[g * ldd + cb] : 0.f;
-        a[3] = cb < N ? dys[(g + 8) * ldd + cb] : 0.f;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int kt = warp + 8 * j;
-            if (kt < ktiles) {
-                const int k = kt * 8 + g;
-                float b[2];
-                b[0] = ca < N ? ws[ca * ldw + k] : 0.f;
-                b[1] = cb < N ? ws[cb * ldw + k] : 0.f;
-                mma_3xtf32(d[j], e[j], a, b);
-            }
-        }
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int kt = warp + 8 * j;
-        if (kt >= ktiles) break;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int r = g + 8 * (q >> 1), k = kt * 8 + 2 * t + (q & 1);
-            if (k >= K) continue;
-            float v = d[j][q] + e[j][q];
-            if (prev && !(prev[r * ldp + k] > 0.f)) v = 0.f;
-            os[r * ldo + k] = v;
-            if (og && r < nrows) og[(long long)r * ldog + k] = v;
-        }
-    }
+                        float* os, int ldo, float* og, long long ldog, int nrows, float* red) {
+    tile_gemm(dys, ldd, N, ws, 1, ldw, K, red, [&](int r, int k, float v) {
+        if (prev && !(prev[r * ldp + k] > 0.f)) v = 0.f;
+        os[r * ldo + k] = v;
+        if (og && r < nrows) og[(long long)r * ldog + k] = v;
+    });
 }
 
 // Partial gradient of one layer over the tile's 16 rows, [W | b] flat:
@@ -272,11 +280,12 @@ __device__ void reduce_and_sgd(const FusedStepArgs& a, int nl, int ntiles) {
 }
 
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT) fused_passive_fwd_kernel(const FusedChainArgs a) {
+__global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedChainArgs a) {
     extern __shared__ __align__(16) float smem[];
     float* ws = smem;
     float* buf0 = smem + a.w_floats;
     float* buf1 = buf0 + R * a.act_ld;
+    float* red = buf1 + R * a.act_ld;           // K-split partial sums of tile_gemm
     const int ntiles = (a.rows + R - 1) / R;
     bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
@@ -305,7 +314,7 @@ __global__ void __launch_bounds__(NT) fused_passive_fwd_kernel(const FusedChainA
             else
                 __syncthreads();
             tile_fwd(cur, a.act_ld, L.in, ws + L.ws_off, L.ws_ld, L.b, L.out, true, nxt, a.act_ld,
-                     L.Y + (long long)r0 * L.ldy, L.ldy, nr);
+                     L.Y + (long long)r0 * L.ldy, L.ldy, nr, red);
             float* t = cur;
             cur = nxt;
             nxt = t;
@@ -328,7 +337,7 @@ __global__ void __launch_bounds__(NT) fused_passive_fwd_kernel(const FusedChainA
     }
 }
 
-__global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a) {
+__global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
     cg::grid_group grid = cg::this_grid();
     const int La = a.na, Lt = a.nt;
@@ -340,6 +349,7 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
     auto act = [&](int i) { return acts + i * R * ldA; };
     float* g0 = act(La + Lt + 2);
     float* g1 = act(La + Lt + 3);
+    float* red = act(La + Lt + 4);              // K-split partial sums of tile_gemm
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* A = a.L;
     const FusedLayerArgs* T = a.L + La;
@@ -373,7 +383,7 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             else
                 __syncthreads();
             tile_fwd(act(l), ldA, A[l].in, ws + A[l].ws_off, A[l].ws_ld, A[l].b, A[l].out, true, act(l + 1), ldA,
-                     A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr);
+                     A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
         }
         __syncthreads();
         for (int i = threadIdx.x; i < R * ea; i += NT) {                 // [z^a | z^p]
@@ -386,7 +396,7 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             else
                 __syncthreads();
             tile_fwd(act(La + 1 + l), ldA, T[l].in, ws + T[l].ws_off, T[l].ws_ld, T[l].b, T[l].out, l < Lt - 1,
-                     act(La + 2 + l), ldA, T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr);
+                     act(La + 2 + l), ldA, T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
         }
         __syncthreads();
         if (threadIdx.x < R) {                                           // loss, d(logits)
@@ -423,10 +433,10 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             tile_partial(gin, ldA, act(La + 1 + l), ldA, T[l].out, T[l].in, part + T[l].poff);
             if (l > 0)
                 tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, act(La + 1 + l), ldA, gout, ldA,
-                        T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr);
+                        T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr, red);
             else
                 tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, nullptr, 0, gout, ldA, nullptr, 0,
-                        nr);
+                        nr, red);
             float* t = gin;
             gin = gout;
             gout = t;
@@ -451,7 +461,7 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
             tile_partial(gin, ldA, act(l), ldA, A[l].out, A[l].in, part + A[l].poff);
             if (l > 0) {
                 tile_dx(gin, ldA, A[l].out, ws + A[l].ws_off, A[l].ws_ld, A[l].in, act(l), ldA, gout, ldA,
-                        A[l - 1].D + (long long)r0 * A[l - 1].ldd, A[l - 1].ldd, nr);
+                        A[l - 1].D + (long long)r0 * A[l - 1].ldd, A[l - 1].ldd, nr, red);
                 float* t = gin;
                 gin = gout;
                 gout = t;
@@ -483,7 +493,7 @@ __global__ void __launch_bounds__(NT) fused_active_kernel(const FusedStepArgs a)
     }
 }
 
-__global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepArgs a) {
+__global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
     cg::grid_group grid = cg::this_grid();
     const int Lp = a.na;
@@ -494,6 +504,7 @@ __global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepAr
     auto act = [&](int i) { return acts + i * R * ldA; };
     float* g0 = act(Lp + 1);
     float* g1 = act(Lp + 2);
+    float* red = act(Lp + 3);                   // K-split partial sums of tile_gemm
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* P = a.L;
     const int ep = P[Lp - 1].out;
@@ -531,7 +542,7 @@ __global__ void __launch_bounds__(NT) fused_passive_bwd_kernel(const FusedStepAr
             if (l > 0) {
                 if (first) cp_wait_pending(l - 1);   // this layer's weights
                 tile_dx(gin, ldA, P[l].out, ws + P[l].ws_off, P[l].ws_ld, P[l].in, act(l), ldA, gout, ldA,
-                        P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr);
+                        P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr, red);
                 float* t = gin;
                 gin = gout;
                 gout = t;

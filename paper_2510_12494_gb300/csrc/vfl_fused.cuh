@@ -5,7 +5,7 @@
 
 namespace vfl {
 
-constexpr int kFusedThreads = 256;
+constexpr int kFusedThreads = 512;
 constexpr int kFusedRows = 16;                 // rows per row tile
 constexpr int kFusedMaxWidth = 256;            // widest layer input or output
 constexpr int kFusedMaxLayers = 16;
@@ -66,14 +66,16 @@ struct FusedStepArgs {
 
 // Shared memory: every staged weight matrix (w_floats, laid out by ws_off /
 // wts_off) followed by row-tile activation slots of kFusedRows x act_ld.
+// plus 1024 floats for the K-split partial sums of the tile GEMMs (8 tiles x 32 lanes x 4)
+constexpr int kFusedRedFloats = 1024;
 inline size_t fused_smem_fwd(int w_floats, int act_ld) {
-    return (size_t)(w_floats + 2 * kFusedRows * act_ld) * sizeof(float);
+    return (size_t)(w_floats + 2 * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
 inline size_t fused_smem_active(int w_floats, int act_ld, int na, int nt) {
-    return (size_t)(w_floats + (na + nt + 4) * kFusedRows * act_ld) * sizeof(float);
+    return (size_t)(w_floats + (na + nt + 4) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
 inline size_t fused_smem_pbwd(int w_floats, int act_ld, int nl) {
-    return (size_t)(w_floats + (nl + 3) * kFusedRows * act_ld) * sizeof(float);
+    return (size_t)(w_floats + (nl + 3) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
 
 cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s);
