@@ -31,6 +31,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "split-VFL training samples/sec at 1 GB300; % of roofline per kernel"
 FP32_ALU_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12   # SMs x FP32 lanes x FMA x max clock
+TF32_PER_BF16 = 1.1 / 2.25                               # nominal dense TF32 / BF16 tensor throughput
 
 
 def parse():
@@ -231,10 +232,15 @@ def roofline(prof, pk):
     name, (n, ms, flops, nbytes) = max(prof.items(), key=lambda kv: kv[1][1])
     sec = ms / 1e3
     tensor = name.startswith("gemm_tc")
+    tf32x3 = name.startswith("fused_")
     if tensor:
         peak = pk["bf16_tflops_sustained"]
         ach = flops / sec / 1e12
-        compute_bound = True
+        bound, unit = "tensor", "TFLOP/s"
+    elif tf32x3:
+        # fp32 contractions on the TF32 tensor path in 3xTF32 form: three TF32 products per fp32 one
+        peak = pk["bf16_tflops_sustained"] * TF32_PER_BF16 / 3.0
+        ach = flops / sec / 1e12
         bound, unit = "tensor", "TFLOP/s"
     else:
         alu_peak = FP32_ALU_PEAK_TFLOPS
@@ -247,6 +253,8 @@ def roofline(prof, pk):
     return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
             "traffic": None, "launches": n, "avg_us": ms / n * 1e3,
             "peak_src": (f"{pk['src']} sustained bf16 GEMM" if tensor else
+                         f"{pk['src']} sustained bf16 GEMM x {TF32_PER_BF16:.4f} (nominal TF32/BF16) / 3 (3xTF32)"
+                         if tf32x3 else
                          ("derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz" if bound == "alu"
                           else f"{pk['src']} HBM copy")),
             "all_classes_ms": {k: round(v[1], 4) for k, v in sorted(prof.items(), key=lambda kv: -kv[1][1])}}
