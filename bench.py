@@ -42,6 +42,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2, help="workload preset 1..5 (default 2, credit-shaped)")
     ap.add_argument("--rows", type=int, default=0, help="override the preset's row count")
+    ap.add_argument("--workers", type=int, default=0, help="override the preset's worker streams per party")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -55,6 +56,8 @@ def workload(args):
     p = synth.preset(args.config)
     if args.rows:
         p = p.with_(n_rows=args.rows)
+    if args.workers:
+        p = p.with_(workers=args.workers)
     desc = (f"{p.name}: N={p.n_rows}, d_p/d_a={p.d_passive}/{p.d_active}, "
             f"passive {'-'.join(map(str, (p.d_passive,) + p.passive))}, "
             f"active {'-'.join(map(str, (p.d_active,) + p.active))}, "
@@ -232,7 +235,7 @@ def roofline(prof, pk):
     name, (n, ms, flops, nbytes) = max(prof.items(), key=lambda kv: kv[1][1])
     sec = ms / 1e3
     tensor = name.startswith("gemm_tc")
-    tf32x3 = name.startswith("fused_")
+    tf32x3 = name.startswith("fused_") and name != "fused_update"   # fused_update runs on the FP32 lanes
     if tensor:
         peak = pk["bf16_tflops_sustained"]
         ach = flops / sec / 1e12

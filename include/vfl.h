@@ -259,7 +259,7 @@ int64_t vfl_kernel_launches(const vfl_ctx* ctx);
  * vfl_kernel_class_name), the number of launches, their summed duration in ms
  * and their summed algorithmic flops and bytes.
  */
-#define VFL_KERNEL_CLASSES 16
+#define VFL_KERNEL_CLASSES 17
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);
 vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
                            double* bytes);

@@ -1,17 +1,28 @@
-// Fused kernels for narrow fp32 models (every width <= 256, one worker stream
-// per party): each phase of Algorithm 1 is one launch.
+// Fused kernels for narrow fp32 models (every width <= 256): each phase of
+// Algorithm 1 is one row-parallel launch, and each party's weight gradient and
+// SGD step (Eq. 2, delayed form of App. D) is one more.
 //
-//  - passive forward: every CTA stages all of f_p's weights (transposed copies)
-//    into shared memory with cp.async, then runs the bottom chain for its row
-//    tile; the last CTA to finish publishes the channel header.
-//  - active step (cooperative launch): phase 1 is row-parallel -- active bottom
-//    forward, top forward on [z^a | z^p], loss, the input-gradient chain back to
-//    the first active layer, publish dz^p, and each row tile's partial weight
-//    gradient (from the tiles already in shared memory).  After a grid-wide
-//    barrier, phase 2 sums the partials of every parameter over the row tiles
-//    in a fixed order (deterministic) and applies SGD to the master and the new
-//    version's copies; CTA 0 reduces the loss and writes the gradient header.
-//  - passive backward (cooperative launch): the same two phases for f_p.
+//  - passive forward: every CTA stages all of f_p's weights into shared memory
+//    with cp.async, then runs the bottom chain for its 16-row tile; the last CTA
+//    to finish publishes the embedding channel's header.
+//  - active step: active bottom forward, top forward on [z^a | z^p], loss, the
+//    input-gradient chain back to the first active layer; dz^p goes to the
+//    gradient channel (header written by the last CTA), every layer's
+//    d(pre-activation) rows stay in HBM for the update.
+//  - passive backward: the input-gradient chain of f_p from dz^p.
+//  - update (one per party): dW = D^T X over the step's rows for every layer,
+//    an output tile per cluster of 8 CTAs that each take 1/8 of the rows; the 8
+//    partial tiles are summed in rank order through distributed shared memory
+//    (deterministic), and SGD writes the master and the new version's copy.
+//
+// The row-tile GEMMs run on the warp-level tensor cores (mma.sync m16n8k8,
+// TF32) in 3xTF32 form, which keeps fp32 accuracy: x = hi + lo with hi, lo
+// TF32, and a b ~ a_hi b_hi + a_lo b_hi + a_hi b_lo.  Activation tiles that
+// feed a GEMM live in shared memory as their hi and lo planes, split once by
+// the epilogue that writes them and loaded with ldmatrix; weights are split as
+// they are read.  Every tile is zero-padded to a multiple of 8 columns and
+// every staged weight matrix to a multiple of 8 rows, so the GEMM loops need no
+// bounds checks.
 #include <cooperative_groups.h>
 
 #include "vfl_fused.cuh"
@@ -23,12 +34,22 @@ namespace vfl {
 namespace {
 
 constexpr int NT = kFusedThreads;     // 16 warps
+constexpr int NW = NT / 32;
 constexpr int R = kFusedRows;
 static_assert(R == 16, "the MMA tiles cover exactly 16 rows");
+static_assert(NW == R, "row-tile copies give each warp one row");
+
+__device__ __forceinline__ int ceil8(int x) { return (x + 7) & ~7; }
 
 __device__ __forceinline__ void cp16(float* s, const float* g) {
     const unsigned sa = (unsigned)__cvta_generic_to_shared(s);
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sa), "l"(g) : "memory");
+}
+
+// 4 bytes, or zero-fill when !valid (src must still be a valid address)
+__device__ __forceinline__ void cp4(float* s, const float* g, bool valid) {
+    const unsigned sa = (unsigned)__cvta_generic_to_shared(s);
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(sa), "l"(g), "r"(valid ? 4 : 0) : "memory");
 }
 
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
@@ -51,10 +72,10 @@ __device__ __forceinline__ void cp_wait_pending(int n) {
 
 // R rows of `cols` floats (cols % 4 == 0): rows < nrows copied asynchronously
 // from global (row stride ldg), the rest zero-filled; smem row stride lds.
+// Warp r copies row r.
 __device__ void async_rows(float* s, int lds, const float* g, long long ldg, int cols, int nrows) {
-    const int q = cols / 4;
-    for (int i = threadIdx.x; i < R * q; i += NT) {
-        const int r = i / q, c = (i - r * q) * 4;
+    const int r = threadIdx.x >> 5;
+    for (int c = (threadIdx.x & 31) * 4; c < cols; c += 128) {
         if (r < nrows)
             cp16(s + r * lds + c, g + (long long)r * ldg + c);
         else
@@ -64,238 +85,209 @@ __device__ void async_rows(float* s, int lds, const float* g, long long ldg, int
 
 // rows x cols floats (cols % 4 == 0, 16-byte aligned rows) into smem rows of stride lds, asynchronously
 __device__ void async_matrix(float* s, int lds, const float* g, long long ldg, int rows, int cols) {
-    const int q = cols / 4;
-    for (int i = threadIdx.x; i < rows * q; i += NT) {
-        const int r = i / q, c = (i - r * q) * 4;
-        cp16(s + r * lds + c, g + (long long)r * ldg + c);
-    }
+    for (int r = threadIdx.x >> 5; r < rows; r += NW)
+        for (int c = (threadIdx.x & 31) * 4; c < cols; c += 128) cp16(s + r * lds + c, g + (long long)r * ldg + c);
 }
 
+// A staged layer, asynchronously: W's rows (stride ws_ld), zero rows up to
+// ceil8(out), then b over ceil8(out) floats, zero past out.  The version copies keep their
+// columns [in, in_ld) zero, so every staged tile is zero-padded both ways.
 __device__ void stage_layer_weights(float* ws, const FusedLayerArgs& L) {
-    if (L.ws_off >= 0) async_matrix(ws + L.ws_off, L.ws_ld, L.W, L.in_ld, L.out, (int)L.in_ld);
+    if (L.ws_off < 0) return;
+    float* w = ws + L.ws_off;
+    async_matrix(w, L.ws_ld, L.W, L.in_ld, L.out, (int)L.in_ld);
+    const int out8 = ceil8(L.out);
+    for (int r = L.out + (threadIdx.x >> 5); r < out8; r += NW)
+        for (int c = (threadIdx.x & 31) * 4; c < L.in_ld; c += 128)
+            *reinterpret_cast<float4*>(w + r * L.ws_ld + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+    float* b = w + out8 * L.ws_ld;
+    for (int c = threadIdx.x; c < out8; c += NT) cp4(b + c, L.b + (c < L.out ? c : 0), c < L.out);
 }
 
-// ---- warp-level tensor-core tiles: mma.sync m16n8k8 TF32 in 3xTF32 form ----
-// Each fp32 operand x is split into hi = tf32(x) and lo = tf32(x - hi); the
-// product is accumulated as lo*hi + hi*lo + hi*hi in fp32 (the lo*lo term,
-// ~2^-22 relative, is dropped), which keeps fp32-level accuracy.
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-    uint32_t r;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-    return r;
+__device__ __forceinline__ const float* staged_bias(const float* ws, const FusedLayerArgs& L) {
+    return ws + L.ws_off + ceil8(L.out) * L.ws_ld;
 }
+
+// ---- 3xTF32 on mma.sync m16n8k8 ---------------------------------------------
+// TF32 rounding to nearest, ties away from zero, on the bit pattern: adding half
+// an ulp of the 10-bit mantissa to the magnitude bits carries into the exponent
+// exactly when rounding up crosses a binade.
+__device__ __forceinline__ uint32_t to_tf32(float x) { return (__float_as_uint(x) + 0x1000u) & 0xffffe000u; }
 
 __device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
     hi = to_tf32(x);
     lo = to_tf32(x - __uint_as_float(hi));
 }
 
+// d += a b (m16n8k8, TF32 inputs, fp32 accumulation); no side effects, so the
+// compiler may interleave independent MMAs
 __device__ __forceinline__ void mma_tf32(float* d, const uint32_t* a, const uint32_t* b) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+    asm("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// d += a_hi*b_hi and e += a_lo*b_hi + a_hi*b_lo for a 16x8 (A) by 8x8 (B)
-// fragment pair given as fp32 values; the caller adds e into d at the end
-// (two accumulators keep the dependent MMA chain short).
-__device__ __forceinline__ void mma_3xtf32(float* d, float* e, const float* a, const float* b) {
-    uint32_t ah[4], al[4], bh[2], bl[2];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) split_tf32(a[i], ah[i], al[i]);
-    split_tf32(b[0], bh[0], bl[0]);
-    split_tf32(b[1], bh[1], bl[1]);
-    mma_tf32(e, al, bh);
-    mma_tf32(d, ah, bh);
-    mma_tf32(e, ah, bl);
+// A fragment (fp32 bits) of a 16 x 8 block of a 16-row tile: ldmatrix of four
+// 8 x 4 (32-bit) matrices, rows 0-7 / 8-15 by columns k0..k0+3 / k0+4..k0+7.
+// Lane l points at row (l mod 8) + 8 ((l / 8) mod 2), column k0 + 4 (l / 16)
+// (a16_lane_offset); a row stride of 4 mod 32 floats makes it conflict-free.
+__device__ __forceinline__ int a16_lane_offset(int ld) {
+    const int lane = threadIdx.x & 31;
+    return ((lane & 7) + ((lane >> 3) & 1) * 8) * ld + (lane >> 4) * 4;
 }
 
-// One 16x8 output tile of  sum_k A[r][k] B[k][n]  for k in [kbeg, kend), 3xTF32.
-// A is the 16-row tile (row stride lda, columns past K masked); B[k][n] is read
-// as  bm[n * ldb_n + k * ldb_k]  (rows past N / K masked).  Accumulates into d, e.
-__device__ __forceinline__ void mma_tile_range(float* d, float* e, const float* as, int lda, int K, const float* bm,
-                                               int ldb_n, int ldb_k, int n, bool n_ok, int kbeg, int kend) {
+__device__ __forceinline__ void lds_a(uint32_t* a, const float* p) {
+    const unsigned addr = (unsigned)__cvta_generic_to_shared(p);
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+                 : "r"(addr));
+}
+
+constexpr int kTilesPerWarp = 4;
+
+// For the nt <= 4 output blocks at columns 8 j0, 8 (j0 + 1), ...:
+// d += A_lo B_hi + A_hi B_lo + A_hi B_hi (small terms first) over k-steps
+// [ks0, ks1).  Forward (kT = false): B[k][n] = W[n][k]; input gradient
+// (kT = true): B[k][n] = W[k][n]; W in smem, row stride ldw.  One A fragment
+// serves all the warp's blocks, whose MMA chains are independent; the next
+// k-step's operands are loaded before this one's MMAs issue.
+template <bool kT>
+__device__ __forceinline__ void mma_steps(float (*d)[4], const float* A, int lda, const float* W, int ldw, int j0,
+                                          int nt, int ks0, int ks1) {
     const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
-    for (int k0 = kbeg; k0 < kend; k0 += 8) {
-        const int ka = k0 + t, kb = k0 + t + 4;
-        float a[4], b[2];
-        a[0] = ka < K ? as[g * lda + ka] : 0.f;
-        a[1] = ka < K ? as[(g + 8) * lda + ka] : 0.f;
-        a[2] = kb < K ? as[g * lda + kb] : 0.f;
-        a[3] = kb < K ? as[(g + 8) * lda + kb] : 0.f;
-        b[0] = (ka < K && n_ok) ? bm[n * ldb_n + ka * ldb_k] : 0.f;
-        b[1] = (kb < K && n_ok) ? bm[n * ldb_n + kb * ldb_k] : 0.f;
-        mma_3xtf32(d, e, a, b);
+    const float* wb = kT ? W + t * ldw + j0 * 8 + g : W + (j0 * 8 + g) * ldw + t;
+    const int jstep = kT ? 8 : 8 * ldw;
+    const int kstep = kT ? 8 * ldw : 8;
+    const int khalf = kT ? 4 * ldw : 4;
+    const float* ab = A + a16_lane_offset(lda);
+    uint32_t a[4];
+    float b[kTilesPerWarp][2];
+    auto load = [&](int ks) {
+        lds_a(a, ab + ks * 8);
+#pragma unroll
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) {
+                const float* w = wb + i * jstep + ks * kstep;
+                b[i][0] = w[0];
+                b[i][1] = w[khalf];
+            }
+    };
+    if (ks0 < ks1) load(ks0);
+    for (int ks = ks0; ks < ks1; ++ks) {
+        uint32_t ah[4], al[4], bh[kTilesPerWarp][2], bl[kTilesPerWarp][2];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) split_tf32(__uint_as_float(a[i]), ah[i], al[i]);
+#pragma unroll
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) {
+                split_tf32(b[i][0], bh[i][0], bl[i][0]);
+                split_tf32(b[i][1], bh[i][1], bl[i][1]);
+            }
+        if (ks + 1 < ks1) load(ks + 1);
+#pragma unroll
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) mma_tf32(d[i], al, bh[i]);
+#pragma unroll
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) mma_tf32(d[i], ah, bl[i]);
+#pragma unroll
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) mma_tf32(d[i], ah, bh[i]);
     }
 }
 
-// C[16 x N] = A[16 x K] . B over the 16 warps of the block: output tile j (8
-// columns) goes to warp j mod 16; with at most 8 tiles the K range is split
-// between warps w and w + 8 and the second half is added through `red`
-// (fixed order).  The epilogue callback receives (row, col, value) for
-// every in-range output.
-template <typename Epi>
-__device__ void tile_gemm(const float* as, int lda, int K, const float* bm, int ldb_n, int ldb_k, int N, float* red,
-                          Epi epi) {
+// C[16 x 8 ntl] = A[16 x 8 ks] B with the warp mapping `map` (fused_gemm_map):
+// each group of 2^lng warps writes its 16 x 8 ntl partial, row-major (row
+// stride 8 ntl + 8), to `red`; then warp r sums row r's partials in group
+// order and calls epi(r, c, v0, v1) for each column pair c, c+1.  Callers put
+// a barrier before each call.
+static_assert(NW == 16 && R == 16, "the warp mapping assumes 16 warps and 16 rows");
+// The MMA part, out of line (one copy per B layout, with its own registers).
+template <bool kT>
+__device__ __noinline__ void gemm_partials(const float* A, int lda, int ks, const float* W, int ldw, int ntl, int map,
+                                           float* red) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
-    constexpr int NW = NT / 32;
-    const int ntiles = (N + 7) / 8;
-    const bool split = ntiles <= NW / 2;
-    const int ksteps = (K + 7) / 8;
-    const int khalf = ((ksteps + 1) / 2) * 8;
-    float d[2][4] = {}, e[2][4] = {};
-    int mine = 0;
-    if (split) {
-        const int j = warp % (NW / 2), half = warp / (NW / 2);
-        if (j < ntiles) {
-            const int n = j * 8 + g;
-            mma_tile_range(d[0], e[0], as, lda, K, bm, ldb_n, ldb_k, n, n < N, half ? khalf : 0, half ? K : min(K, khalf));
-            mine = 1;
-        }
-        if (mine && half) {
+    const int lng = map & 15, lkg = (map >> 4) & 15, tpw = map >> 8;
+    const int rs = 8 * ntl + 8;
+    const int grp = warp >> lng, j0 = (warp & ((1 << lng) - 1)) * tpw;
+    if (grp < (1 << lkg) && j0 < ntl) {
+        const int nt = min(tpw, ntl - j0);
+        float d[kTilesPerWarp][4] = {};
+        mma_steps<kT>(d, A, lda, W, ldw, j0, nt, (grp * ks) >> lkg, ((grp + 1) * ks) >> lkg);
+        float* pr = red + grp * 16 * rs + g * rs + j0 * 8 + 2 * t;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) red[(j * 32 + lane) * 4 + q] = d[0][q] + e[0][q];
-        }
-        __syncthreads();
-        if (!mine || half) return;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) d[0][q] += e[0][q] + red[(j * 32 + lane) * 4 + q];
-        const int c0 = j * 8 + 2 * t;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int c = c0 + (q & 1);
-            if (c < N) epi(g + 8 * (q >> 1), c, d[0][q]);
-        }
-        return;
-    }
-#pragma unroll
-    for (int jj = 0; jj < 2; ++jj) {
-        const int j = warp + NW * jj;
-        if (j < ntiles) {
-            const int n = j * 8 + g;
-            mma_tile_range(d[jj], e[jj], as, lda, K, bm, ldb_n, ldb_k, n, n < N, 0, K);
-        }
-    }
-#pragma unroll
-    for (int jj = 0; jj < 2; ++jj) {
-        const int j = warp + NW * jj;
-        if (j >= ntiles) break;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int c = j * 8 + 2 * t + (q & 1);
-            if (c < N) epi(g + 8 * (q >> 1), c, d[jj][q] + e[jj][q]);
-        }
+        for (int i = 0; i < kTilesPerWarp; ++i)
+            if (i < nt) {
+                *reinterpret_cast<float2*>(pr + i * 8) = make_float2(d[i][0], d[i][1]);
+                *reinterpret_cast<float2*>(pr + 8 * rs + i * 8) = make_float2(d[i][2], d[i][3]);
+            }
     }
 }
 
-// Y[r][c] = act(sum_k X[r][k] W[c][k] + b[c]) for the 16 rows of a tile (W
-// row-major in smem).  To smem (ldy) and to global rows < nrows when yg is set.
-__device__ void tile_fwd(const float* xs, int ldx, int K, const float* ws, int ldw, const float* __restrict__ bias,
-                         int N, bool relu, float* ys, int ldy, float* yg, long long ldyg, int nrows, float* red) {
-    tile_gemm(xs, ldx, K, ws, ldw, 1, N, red, [&](int r, int c, float v) {
-        float y = v + bias[c];
-        if (relu) y = fmaxf(y, 0.f);
-        ys[r * ldy + c] = y;
-        if (yg && r < nrows) yg[(long long)r * ldyg + c] = y;
+template <bool kT, typename Epi>
+__device__ __forceinline__ void tile_gemm(const float* A, int lda, int ks, const float* W, int ldw, int ntl, int map,
+                                          float* red, Epi epi) {
+    gemm_partials<kT>(A, lda, ks, W, ldw, ntl, map, red);
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int rs = 8 * ntl + 8;
+    const int r = threadIdx.x >> 5, kg = 1 << ((map >> 4) & 15);
+    for (int c = 2 * lane; c < 8 * ntl; c += 64) {
+        const float* src = red + r * rs + c;
+        float2 v = *reinterpret_cast<const float2*>(src);
+#pragma unroll 4
+        for (int q = 1; q < kg; ++q) {
+            const float2 u = *reinterpret_cast<const float2*>(src + q * 16 * rs);
+            v.x += u.x;
+            v.y += u.y;
+        }
+        epi(r, c, v.x, v.y);
+    }
+}
+
+// Hidden-layer forward: Y = ReLU(X W^T + b) -> smem tile `out`, and to global
+// rows < nrows (row stride ldyg >= ceil8(N)) when yg is set.
+__device__ __forceinline__ void tile_fwd(const float* X, int ld, int K, const float* ws, int ldw, const float* bias,
+                                         int N, int map, float* out, float* yg, long long ldyg, int nrows, float* red) {
+    tile_gemm<false>(X, ld, ceil8(K) / 8, ws, ldw, ceil8(N) / 8, map, red, [&](int r, int c, float v0, float v1) {
+        const float2 y = make_float2(fmaxf(v0 + bias[c], 0.f), fmaxf(v1 + bias[c + 1], 0.f));
+        *reinterpret_cast<float2*>(out + r * ld + c) = y;
+        if (yg && r < nrows) *reinterpret_cast<float2*>(yg + (long long)r * ldyg + c) = y;
     });
 }
 
-// dX[r][k] = sum_c dY[r][c] W[c][k], zeroed where prev[r][k] <= 0 (when prev is
-// given).  To smem and to global rows < nrows.
-__device__ void tile_dx(const float* dys, int ldd, int N, const float* ws, int ldw, int K, const float* prev, int ldp,
-                        float* os, int ldo, float* og, long long ldog, int nrows, float* red) {
-    tile_gemm(dys, ldd, N, ws, 1, ldw, K, red, [&](int r, int k, float v) {
-        if (prev && !(prev[r * ldp + k] > 0.f)) v = 0.f;
-        os[r * ldo + k] = v;
-        if (og && r < nrows) og[(long long)r * ldog + k] = v;
+// Input gradient of a hidden layer: dX = (dY W) * [prev > 0] -> smem tile `out`
+// and global rows < nrows.
+__device__ __forceinline__ void tile_dx(const float* dY, int ld, int K, const float* ws, int ldw, int N, int map,
+                                        const float* prev, float* out, float* og, long long ldog, int nrows,
+                                        float* red) {
+    tile_gemm<true>(dY, ld, ceil8(K) / 8, ws, ldw, ceil8(N) / 8, map, red, [&](int r, int c, float v0, float v1) {
+        const float2 m = *reinterpret_cast<const float2*>(prev + r * ld + c);
+        const float2 v = make_float2(m.x > 0.f ? v0 : 0.f, m.y > 0.f ? v1 : 0.f);
+        *reinterpret_cast<float2*>(out + r * ld + c) = v;
+        if (og && r < nrows) *reinterpret_cast<float2*>(og + (long long)r * ldog + c) = v;
     });
-}
-
-// Partial gradient of one layer over the tile's 16 rows, [W | b] flat:
-// part[o*in + k] = sum_r D[r][o] X[r][k] (16-output x 8-input MMA tiles, K = 16
-// rows in two steps) and part[out*in + o] = sum_r D[r][o].  Rows beyond the
-// batch hold D = 0; smem columns past out / in are masked.
-__device__ void tile_partial(const float* Ds, int ldd, const float* Xs, int ldx, int out, int in,
-                             float* __restrict__ part) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
-    const int mt = (out + 15) / 16, nt = (in + 7) / 8;
-    for (int it = warp; it < mt * nt; it += NT / 32) {
-        const int o0 = (it / nt) * 16, i0 = (it % nt) * 8;
-        const int oa = o0 + g, ob = o0 + g + 8, i = i0 + g;
-        float d[4] = {0.f, 0.f, 0.f, 0.f}, e[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int r0 = 0; r0 < R; r0 += 8) {
-            const float* d0 = Ds + (r0 + t) * ldd;
-            const float* d1 = Ds + (r0 + t + 4) * ldd;
-            float a[4], b[2];
-            a[0] = oa < out ? d0[oa] : 0.f;
-            a[1] = ob < out ? d0[ob] : 0.f;
-            a[2] = oa < out ? d1[oa] : 0.f;
-            a[3] = ob < out ? d1[ob] : 0.f;
-            b[0] = i < in ? Xs[(r0 + t) * ldx + i] : 0.f;
-            b[1] = i < in ? Xs[(r0 + t + 4) * ldx + i] : 0.f;
-            mma_3xtf32(d, e, a, b);
-        }
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int o = o0 + g + 8 * (q >> 1), k = i0 + 2 * t + (q & 1);
-            if (o < out && k < in) part[(long long)o * in + k] = d[q] + e[q];
-        }
-    }
-    for (int o = threadIdx.x; o < out; o += NT) {
-        float acc = 0.f;
-#pragma unroll
-        for (int r = 0; r < R; ++r) acc += Ds[r * ldd + o];
-        part[(long long)out * in + o] = acc;
-    }
-}
-
-// Phase 2: every parameter's gradient = sum of the row tiles' partials in tile
-// order, then SGD (Eq. 2) on the master and on both copies of the new version.
-__device__ void reduce_and_sgd(const FusedStepArgs& a, int nl, int ntiles) {
-    for (long long i = blockIdx.x * (long long)NT + threadIdx.x; i < a.ptotal; i += (long long)gridDim.x * NT) {
-        int l = 0;
-        while (l + 1 < nl && i >= a.L[l + 1].poff) ++l;
-        const FusedLayerArgs& L = a.L[l];
-        float g = 0.f;
-#pragma unroll 16
-        for (int t = 0; t < ntiles; ++t) g += __ldcg(a.part + (long long)t * a.ptotal + i);
-        const long long idx = i - L.poff;
-        const long long nw = (long long)L.out * L.in;
-        if (idx < nw) {
-            L.gW[idx] = g;
-            const float w = L.Wm[idx] - a.lr * g;
-            L.Wm[idx] = w;
-            const long long o = idx / L.in, k = idx - o * L.in;
-            L.Wc[o * L.in_ld + k] = w;
-        } else {
-            const long long o = idx - nw;
-            L.gb[o] = g;
-            const float b = L.bm[o] - a.lr * g;
-            L.bm[o] = b;
-            L.bc[o] = b;
-        }
-    }
 }
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedChainArgs a) {
     extern __shared__ __align__(16) float smem[];
+    const int ld = a.act_ld;
     float* ws = smem;
-    float* buf0 = smem + a.w_floats;
-    float* buf1 = buf0 + R * a.act_ld;
-    float* red = buf1 + R * a.act_ld;           // K-split partial sums of tile_gemm
+    float* t0 = smem + a.w_floats;                      // x_p rows, then ping-pong
+    float* t1 = t0 + R * ld;
+    float* t2 = t1 + R * ld;
+    float* red = t2 + R * ld;                           // partial output blocks
     const int ntiles = (a.rows + R - 1) / R;
     bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
         __syncthreads();
-        async_rows(buf0, a.act_ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)a.L[0].in_ld, nr);
+        async_rows(t0, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)a.L[0].in_ld, nr);
         if (first) {
-            // group l holds layer l's weights (group 0 also the first tile), so layer l only
-            // waits for its own weights while the later ones are still arriving
+            // group l holds layer l's weights (group 0 also the rows), so layer l
+            // only waits for its own weights while the later ones are still arriving
             for (int l = 0; l < a.nl; ++l) {
                 stage_layer_weights(ws, a.L[l]);
                 cp_commit();
@@ -303,8 +295,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
         } else {
             cp_commit();
         }
-        float* cur = buf0;
-        float* nxt = buf1;
+        const float* cur = t0;
         for (int l = 0; l < a.nl; ++l) {
             const FusedLayerArgs& L = a.L[l];
             if (first)
@@ -313,14 +304,14 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
                 cp_wait_pending(0);
             else
                 __syncthreads();
-            tile_fwd(cur, a.act_ld, L.in, ws + L.ws_off, L.ws_ld, L.b, L.out, true, nxt, a.act_ld,
+            float* nxt = (l & 1) ? t2 : t1;
+            tile_fwd(cur, ld, L.in, ws + L.ws_off, L.ws_ld, staged_bias(ws, L), L.out, L.fmap, nxt,
                      L.Y + (long long)r0 * L.ldy, L.ldy, nr, red);
-            float* t = cur;
             cur = nxt;
-            nxt = t;
         }
         first = false;
     }
+    if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
     // the last CTA to finish publishes the header after every payload write
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -337,38 +328,60 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
     }
 }
 
+// One CTA's share of the "last CTA publishes" rule: after every CTA's payload
+// writes, the last one to arrive writes the header and re-arms the counter.
+__device__ void publish_when_last(int* counter, ChannelHeader* hdr, long long k, int batch, int version) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const int done = atomicAdd(counter, 1);
+        if (done == (int)gridDim.x - 1) {
+            __threadfence();
+            hdr->k = k;
+            hdr->batch = batch;
+            hdr->version = version;
+            *counter = 0;
+            __threadfence();
+        }
+    }
+}
+
 __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
-    cg::grid_group grid = cg::this_grid();
     const int La = a.na, Lt = a.nt;
-    const int ldA = a.act_ld;
+    const int ld = a.act_ld;
     float* ws = smem;
-    float* acts = smem + a.w_floats;
-    // slots: 0 = x_a; 1..La = f_a outputs; La+1 = [z^a | z^p]; La+2..La+1+Lt = g outputs (last: logits);
-    // La+Lt+2, La+Lt+3 = gradient ping-pong
-    auto act = [&](int i) { return acts + i * R * ldA; };
-    float* g0 = act(La + Lt + 2);
-    float* g1 = act(La + Lt + 3);
-    float* red = act(La + Lt + 4);              // K-split partial sums of tile_gemm
+    // tiles of R x ld floats: 0 = x_a rows (later the logits); 1..La-1 = f_a's hidden
+    // outputs; La = [z^a | z^p]; La+1..La+Lt-1 = g's hidden outputs; La+Lt, La+Lt+1 = gradients
+    float* tiles = smem + a.w_floats;
+    auto slot = [&](int i) { return tiles + i * R * ld; };
+    float* X = slot(0);
+    auto H = [&](int l) { return slot(1 + l); };            // output of f_a layer l < La - 1
+    float* C = slot(La);
+    auto TH = [&](int l) { return slot(La + 1 + l); };      // output of g layer l < Lt - 1
+    float* G0 = slot(La + Lt);
+    float* G1 = slot(La + Lt + 1);
+    float* red = slot(La + Lt + 2);
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* A = a.L;
     const FusedLayerArgs* T = a.L + La;
     const int ea = A[La - 1].out;
     const int ep = T[0].in - ea;
+    const int ep8 = ceil8(ep);
     const int nout = T[Lt - 1].out;
     const int ntiles = (a.rows + R - 1) / R;
     const float inv_b = 1.0f / (float)a.rows;
+    const int Ltot = La + Lt;
     bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
-        float* part = a.part + (long long)tile * a.ptotal;
         __syncthreads();
-        async_rows(act(0), ldA, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
-        async_rows(act(La + 1) + ea, ldA, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep, nr);
+        async_rows(X, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
+        async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
         if (first) {
-            // one commit group per layer, in the order the forward uses them
-            for (int l = 0; l < La + Lt; ++l) {
+            // one commit group per layer, in the order the forward uses them (group 0 also the rows)
+            for (int l = 0; l < Ltot; ++l) {
                 stage_layer_weights(ws, a.L[l]);
                 cp_commit();
             }
@@ -377,32 +390,55 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         }
         for (int l = 0; l < La; ++l) {                                   // z^a = f_a(x^a)
             if (first)
-                cp_wait_pending(La + Lt - 1 - l);
+                cp_wait_pending(Ltot - 1 - l);
             else if (l == 0)
                 cp_wait_pending(0);
             else
                 __syncthreads();
-            tile_fwd(act(l), ldA, A[l].in, ws + A[l].ws_off, A[l].ws_ld, A[l].b, A[l].out, true, act(l + 1), ldA,
-                     A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
+            if (l == 0) {
+                const int r = threadIdx.x >> 5;                          // z^p kept for the update
+                if (r < nr)
+                    for (int c = threadIdx.x & 31; c < ep; c += 32)
+                        a.zpc[(long long)(r0 + r) * a.ldzpc + c] = C[r * ld + ea + c];
+            }
+            tile_fwd(l == 0 ? X : H(l - 1), ld, A[l].in, ws + A[l].ws_off, A[l].ws_ld, staged_bias(ws, A[l]), A[l].out,
+                     A[l].fmap, l == La - 1 ? C : H(l), A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
         }
-        __syncthreads();
-        for (int i = threadIdx.x; i < R * ea; i += NT) {                 // [z^a | z^p]
-            const int r = i / ea, c = i - r * ea;
-            act(La + 1)[r * ldA + c] = act(La)[r * ldA + c];
-        }
-        for (int l = 0; l < Lt; ++l) {                                   // y_hat = g(z^a, z^p)
+        for (int l = 0; l < Lt - 1; ++l) {                               // g's hidden layers on [z^a | z^p]
             if (first)
                 cp_wait_pending(Lt - 1 - l);
             else
                 __syncthreads();
-            tile_fwd(act(La + 1 + l), ldA, T[l].in, ws + T[l].ws_off, T[l].ws_ld, T[l].b, T[l].out, l < Lt - 1,
-                     act(La + 2 + l), ldA, T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
+            tile_fwd(l == 0 ? C : TH(l - 1), ld, T[l].in, ws + T[l].ws_off, T[l].ws_ld, staged_bias(ws, T[l]), T[l].out,
+                     T[l].fmap, TH(l), T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
+        }
+        float* lg = X;                                                   // x_a's tile is free again
+        {                                                                // logits: no activation
+            const FusedLayerArgs& L = T[Lt - 1];
+            if (first)
+                cp_wait_pending(0);
+            else
+                __syncthreads();
+            const float* bias = staged_bias(ws, L);
+            float* yg = L.Y + (long long)r0 * L.ldy;
+            const long long ldy = L.ldy;
+            tile_gemm<false>(Lt == 1 ? C : TH(Lt - 2), ld, ceil8(L.in) / 8, ws + L.ws_off, L.ws_ld, ceil8(nout) / 8, L.fmap, red,
+                             [&](int r, int c, float v0, float v1) {
+                                 v0 += bias[c];
+                                 v1 += bias[c + 1];
+                                 *reinterpret_cast<float2*>(lg + r * ld + c) = make_float2(v0, v1);
+                                 if (r < nr) {
+                                     if (c < nout) yg[(long long)r * ldy + c] = v0;
+                                     if (c + 1 < nout) yg[(long long)r * ldy + c + 1] = v1;
+                                 }
+                             });
         }
         __syncthreads();
         if (threadIdx.x < R) {                                           // loss, d(logits)
             const int r = threadIdx.x;
-            const float* s = act(La + 1 + Lt) + r * ldA;
-            float* d = g0 + r * ldA;
+            const float* s = lg + r * ld;
+            float* d = G0 + r * ld;
+            float* dg = T[Lt - 1].D + (long long)(r0 + r) * T[Lt - 1].ldd;
             if (r < nr) {
                 const int y = a.y[r0 + r];
                 float li;
@@ -420,105 +456,86 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
                     for (int j = 0; j < nout; ++j) d[j] = (expf(s[j] - m) * iz - (j == y ? 1.f : 0.f)) * inv_b;
                 }
                 a.rowloss[r0 + r] = li;
-                for (int j = 0; j < nout; ++j) a.ds[(long long)(r0 + r) * nout + j] = d[j];
+                for (int j = 0; j < nout; ++j) dg[j] = d[j];
             } else {
                 for (int j = 0; j < nout; ++j) d[j] = 0.f;
             }
+            for (int j = nout; j < ceil8(nout); ++j) d[j] = 0.f;
         }
-        // backward through g: partial gradients, input-gradient chain
-        float* gin = g0;
-        float* gout = g1;
-        for (int l = Lt - 1; l >= 0; --l) {
+        // backward through g: the input-gradient chain
+        float* gin = G0;
+        float* gout = G1;
+        for (int l = Lt - 1; l >= 1; --l) {
             __syncthreads();
-            tile_partial(gin, ldA, act(La + 1 + l), ldA, T[l].out, T[l].in, part + T[l].poff);
-            if (l > 0)
-                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, act(La + 1 + l), ldA, gout, ldA,
-                        T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr, red);
-            else
-                tile_dx(gin, ldA, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, nullptr, 0, gout, ldA, nullptr, 0,
-                        nr, red);
+            tile_dx(gin, ld, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, T[l].dmap, TH(l - 1), gout,
+                    T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr, red);
             float* t = gin;
             gin = gout;
             gout = t;
         }
         __syncthreads();
-        // split [dz^a | dz^p]: dz^a * [z^a > 0] is the d(pre) of f_a's last layer; dz^p is published
-        for (int i = threadIdx.x; i < R * (ea + ep); i += NT) {
-            const int r = i / (ea + ep), c = i - r * (ea + ep);
-            float v = gin[r * ldA + c];
-            if (c < ea) {
-                if (!(act(La)[r * ldA + c] > 0.f)) v = 0.f;
-                gout[r * ldA + c] = v;
-                if (r < nr) A[La - 1].D[(long long)(r0 + r) * A[La - 1].ldd + c] = v;
-            } else if (r < nr) {
-                a.gradp[(long long)(r0 + r) * a.ldgp + (c - ea)] = v;
-            }
+        {
+            // g's first layer: [dz^a | dz^p] = dY W; dz^a * [z^a > 0] is the d(pre) of f_a's last
+            // layer, dz^p (no mask: the passive party applies its own) is published
+            const FusedLayerArgs& L = T[0];
+            float* da = A[La - 1].D + (long long)r0 * A[La - 1].ldd;
+            const long long ldda = A[La - 1].ldd;
+            float* gp = a.gradp + (long long)r0 * a.ldgp;
+            const long long ldgp = a.ldgp;
+            float* go = gout;
+            tile_gemm<true>(gin, ld, ceil8(L.out) / 8, ws + L.ws_off, L.ws_ld, ceil8(L.in) / 8, L.dmap, red,
+                            [&](int r, int c, float v0, float v1) {
+                                if (c < ea) {
+                                    const float2 m = *reinterpret_cast<const float2*>(C + r * ld + c);
+                                    const float2 v = make_float2(m.x > 0.f ? v0 : 0.f, m.y > 0.f ? v1 : 0.f);
+                                    *reinterpret_cast<float2*>(go + r * ld + c) = v;
+                                    if (r < nr) *reinterpret_cast<float2*>(da + (long long)r * ldda + c) = v;
+                                } else if (r < nr) {
+                                    *reinterpret_cast<float2*>(gp + (long long)r * ldgp + (c - ea)) = make_float2(v0, v1);
+                                }
+                            });
+            float* t = gin;
+            gin = gout;
+            gout = t;
         }
-        gin = gout;
-        gout = (gin == g0) ? g1 : g0;
-        for (int l = La - 1; l >= 0; --l) {                              // backward through f_a
+        for (int l = La - 1; l >= 1; --l) {                              // backward through f_a
             __syncthreads();
-            tile_partial(gin, ldA, act(l), ldA, A[l].out, A[l].in, part + A[l].poff);
-            if (l > 0) {
-                tile_dx(gin, ldA, A[l].out, ws + A[l].ws_off, A[l].ws_ld, A[l].in, act(l), ldA, gout, ldA,
-                        A[l - 1].D + (long long)r0 * A[l - 1].ldd, A[l - 1].ldd, nr, red);
-                float* t = gin;
-                gin = gout;
-                gout = t;
-            }
+            tile_dx(gin, ld, A[l].out, ws + A[l].ws_off, A[l].ws_ld, A[l].in, A[l].dmap, H(l - 1), gout,
+                    A[l - 1].D + (long long)r0 * A[l - 1].ldd, A[l - 1].ldd, nr, red);
+            float* t = gin;
+            gin = gout;
+            gout = t;
         }
         first = false;
     }
     if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
-    grid.sync();
-    reduce_and_sgd(a, La + Lt, ntiles);
-    if (blockIdx.x == 0) {
-        // mean loss over the batch (fixed order) and the gradient channel's header
-        __syncthreads();
-        float part = 0.f;
-        for (int r = threadIdx.x; r < a.rows; r += NT) part += __ldcg(a.rowloss + r);
-        for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
-        float* red = smem;
-        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = part;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float v = 0.f;
-            for (int w = 0; w < NT / 32; ++w) v += red[w];
-            *a.loss_out = v * inv_b;
-            a.pub_hdr->k = a.k;
-            a.pub_hdr->batch = a.batch;
-            a.pub_hdr->version = a.version;
-            __threadfence();
-        }
-    }
+    publish_when_last(a.counter, a.pub_hdr, a.k, a.batch, a.version);
 }
 
 __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
-    cg::grid_group grid = cg::this_grid();
     const int Lp = a.na;
-    const int ldA = a.act_ld;
+    const int ld = a.act_ld;
     float* ws = smem;
-    float* acts = smem + a.w_floats;
-    // slots: 0 = x_p; 1..Lp = f_p outputs (saved by the forward); Lp+1, Lp+2 = gradients
-    auto act = [&](int i) { return acts + i * R * ldA; };
-    float* g0 = act(Lp + 1);
-    float* g1 = act(Lp + 2);
-    float* red = act(Lp + 3);                   // K-split partial sums of tile_gemm
+    // tiles: 0..Lp-1 = f_p's outputs (saved by the forward), Lp = dz^p rows, Lp+1, Lp+2 = gradients
+    float* tiles = smem + a.w_floats;
+    auto slot = [&](int i) { return tiles + i * R * ld; };
+    float* gs = slot(Lp);
+    float* G0 = slot(Lp + 1);
+    float* G1 = slot(Lp + 2);
+    float* red = slot(Lp + 3);
     if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* P = a.L;
-    const int ep = P[Lp - 1].out;
+    const int ep8 = ceil8(P[Lp - 1].out);
     const int ntiles = (a.rows + R - 1) / R;
     bool first = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int r0 = tile * R;
         const int nr = min(R, a.rows - r0);
-        float* part = a.part + (long long)tile * a.ptotal;
         __syncthreads();
-        async_rows(act(0), ldA, a.x + (long long)r0 * a.ldx, a.ldx, (int)P[0].in_ld, nr);
         for (int l = 0; l < Lp; ++l)
-            async_rows(act(l + 1), ldA, P[l].Y + (long long)r0 * P[l].ldy, P[l].ldy, (int)P[l].out_ld, nr);
-        async_rows(g1, ldA, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
+            async_rows(slot(l), ld, P[l].Y + (long long)r0 * P[l].ldy, P[l].ldy, (int)P[l].out_ld, nr);
+        async_rows(gs, ld, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
         cp_commit();
         if (first) {
             // weights in the order the backward uses them: layer Lp-1 first
@@ -528,31 +545,168 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
             }
         }
         cp_wait_pending(first ? Lp - 1 : 0);
-        for (int i = threadIdx.x; i < R * ep; i += NT) {                 // dz^p * [z^p > 0]
-            const int r = i / ep, c = i - r * ep;
-            const float v = act(Lp)[r * ldA + c] > 0.f ? g1[r * ldA + c] : 0.f;
-            g0[r * ldA + c] = v;
-            if (r < nr) P[Lp - 1].D[(long long)(r0 + r) * P[Lp - 1].ldd + c] = v;
-        }
-        float* gin = g0;
-        float* gout = g1;
-        for (int l = Lp - 1; l >= 0; --l) {
-            __syncthreads();
-            tile_partial(gin, ldA, act(l), ldA, P[l].out, P[l].in, part + P[l].poff);
-            if (l > 0) {
-                if (first) cp_wait_pending(l - 1);   // this layer's weights
-                tile_dx(gin, ldA, P[l].out, ws + P[l].ws_off, P[l].ws_ld, P[l].in, act(l), ldA, gout, ldA,
-                        P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr, red);
-                float* t = gin;
-                gin = gout;
-                gout = t;
+        {                                                                // dz^p * [z^p > 0]
+            const int r = threadIdx.x >> 5;
+            const float* zp = slot(Lp - 1);
+            float* dg = P[Lp - 1].D + (long long)(r0 + r) * P[Lp - 1].ldd;
+            for (int c = (threadIdx.x & 31) * 2; c < ep8; c += 64) {
+                const float2 z = *reinterpret_cast<const float2*>(zp + r * ld + c);
+                const float2 gr = *reinterpret_cast<const float2*>(gs + r * ld + c);
+                const float2 v = make_float2(z.x > 0.f ? gr.x : 0.f, z.y > 0.f ? gr.y : 0.f);
+                *reinterpret_cast<float2*>(G0 + r * ld + c) = v;
+                if (r < nr) *reinterpret_cast<float2*>(dg + c) = v;
             }
+        }
+        float* gin = G0;
+        float* gout = G1;
+        for (int l = Lp - 1; l >= 1; --l) {
+            if (first)
+                cp_wait_pending(l - 1);   // this layer's weights
+            else
+                __syncthreads();
+            tile_dx(gin, ld, P[l].out, ws + P[l].ws_off, P[l].ws_ld, P[l].in, P[l].dmap, slot(l - 1), gout,
+                    P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr, red);
+            float* t = gin;
+            gin = gout;
+            gout = t;
         }
         first = false;
     }
     if (first) cp_wait_pending(0);
-    grid.sync();
-    reduce_and_sgd(a, Lp, ntiles);
+}
+
+// dW = D^T X, db = sum of D's rows, then SGD, for one 32 x 32 output tile per
+// cluster; CTA `rank` of the cluster covers rows [rank c, (rank + 1) c) with
+// c = ceil(rows / 8).  Inside a CTA, 4 row groups x (8 x 8 threads of 4 x 4
+// outputs) accumulate in fp32; the groups, then the 8 ranks, are summed in a
+// fixed order.
+constexpr int kUpdRows = 128;                // rows staged per pass
+constexpr int kUpdLd = kUpdTile + 4;         // smem row stride
+constexpr int kUpdLoads = kUpdRows * kUpdTile / kUpdThreads;
+static_assert(kUpdThreads == 256 && kUpdTile == 32, "the thread map below assumes 256 threads and 32 x 32 tiles");
+static_assert(kUpdRows * kUpdLd >= 4 * kUpdTile * kUpdTile, "the group partials reuse the D stage");
+
+__global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThreads)
+    fused_update_kernel(const FusedUpdArgs a) {
+    __shared__ __align__(16) float Ds[kUpdRows * kUpdLd];
+    __shared__ __align__(16) float Xs[kUpdRows * kUpdLd];
+    __shared__ __align__(16) float Pw[kUpdTile * kUpdTile];   // this CTA's partial dW tile
+    __shared__ float Pb[kUpdTile];                            // and partial db
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int tile = blockIdx.x / kUpdCluster;
+    int l = 0;
+    while (l + 1 < a.nl && tile >= a.L[l + 1].tile0) ++l;
+    const FusedUpdLayer& L = a.L[l];
+    const int t = tile - L.tile0;
+    const int o0 = (t / L.tiles_i) * kUpdTile, i0 = (t % L.tiles_i) * kUpdTile;
+    const int no = min(kUpdTile, L.out - o0), ni = min(kUpdTile, L.in - i0);
+    const bool bias = i0 == 0;
+    const int chunk = (a.rows + kUpdCluster - 1) / kUpdCluster;
+    const int rbeg = min(a.rows, rank * chunk), rend = min(a.rows, rbeg + chunk);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int grp = warp >> 1;                               // row group
+    const int ob = (((warp & 1) << 2) + (lane >> 3)) * 4;    // first of 4 outputs
+    const int ib = (lane & 7) * 4;                           // first of 4 inputs
+    float acc[4][4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+    float bacc = 0.f;                                        // db partial of output tid & 31
+    for (int rb = rbeg; rb < rend; rb += kUpdRows) {
+        const int nr = min(kUpdRows, rend - rb);
+        float dv[kUpdLoads], xv[kUpdLoads];
+#pragma unroll
+        for (int j = 0; j < kUpdLoads; ++j) {                // every load in flight before any store
+            const int e = tid + j * kUpdThreads, r = e >> 5, c = e & 31;
+            const long long gr = rb + r;
+            dv[j] = (r < nr && c < no) ? __ldg(L.D + gr * L.ldd + o0 + c) : 0.f;
+            const int ic = i0 + c;
+            xv[j] = 0.f;
+            if (r < nr && c < ni)
+                xv[j] = ic < L.xsplit ? __ldg(L.X + gr * L.ldx + ic) : __ldg(L.X2 + gr * L.ldx2 + (ic - L.xsplit));
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kUpdLoads; ++j) {
+            const int e = tid + j * kUpdThreads, r = e >> 5, c = e & 31;
+            Ds[r * kUpdLd + c] = dv[j];
+            Xs[r * kUpdLd + c] = xv[j];
+        }
+        __syncthreads();
+        for (int r = grp; r < nr; r += 4) {
+            const float4 d = *reinterpret_cast<const float4*>(Ds + r * kUpdLd + ob);
+            const float4 x = *reinterpret_cast<const float4*>(Xs + r * kUpdLd + ib);
+            const float dd[4] = {d.x, d.y, d.z, d.w}, xx[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+            for (int p = 0; p < 4; ++p)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(dd[p], xx[q], acc[p][q]);
+        }
+        if (bias)
+            for (int r = tid >> 5; r < nr; r += kUpdThreads / 32) bacc += Ds[r * kUpdLd + (tid & 31)];
+    }
+    __syncthreads();
+    float* gpart = Ds;                                       // [4 groups][32][32]
+    float* bpart = Xs;                                       // [8 warps][32]
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+        *reinterpret_cast<float4*>(gpart + grp * kUpdTile * kUpdTile + (ob + p) * kUpdTile + ib) =
+            make_float4(acc[p][0], acc[p][1], acc[p][2], acc[p][3]);
+    bpart[tid] = bacc;
+    __syncthreads();
+    for (int e = tid; e < kUpdTile * kUpdTile; e += kUpdThreads)
+        Pw[e] = ((gpart[e] + gpart[1024 + e]) + gpart[2048 + e]) + gpart[3072 + e];
+    if (tid < kUpdTile) {
+        float s = 0.f;
+        for (int w = 0; w < kUpdThreads / 32; ++w) s += bpart[w * 32 + tid];
+        Pb[tid] = s;
+    }
+    cluster.sync();
+    // rank q sums outputs [128 q, 128 q + 128) of the tile (rows 4q..4q+3) over the ranks in order
+    constexpr int kPer = kUpdTile * kUpdTile / kUpdCluster;
+    if (tid < kPer) {
+        const int e = rank * kPer + tid, o = e / kUpdTile, i = e - o * kUpdTile;
+        if (o < no && i < ni) {
+            float g = 0.f;
+#pragma unroll
+            for (int q = 0; q < kUpdCluster; ++q) g += cluster.map_shared_rank(Pw, q)[e];
+            const long long go = o0 + o, gi = i0 + i;
+            const long long idx = go * L.in + gi;
+            L.gW[idx] = g;
+            const float w = L.Wm[idx] - a.lr * g;
+            L.Wm[idx] = w;
+            L.Wc[go * L.in_ld + gi] = w;
+        }
+    } else if (bias && tid < kPer + kUpdTile / kUpdCluster) {
+        const int o = rank * (kUpdTile / kUpdCluster) + (tid - kPer);
+        if (o < no) {
+            float g = 0.f;
+#pragma unroll
+            for (int q = 0; q < kUpdCluster; ++q) g += cluster.map_shared_rank(Pb, q)[o];
+            const int go = o0 + o;
+            L.gb[go] = g;
+            const float b = L.bm[go] - a.lr * g;
+            L.bm[go] = b;
+            L.bc[go] = b;
+        }
+    }
+    cluster.sync();                                          // peers' shared memory stays valid until here
+    if (blockIdx.x == 0 && a.loss_out) {                     // mean loss of the step, fixed order
+        float s = 0.f;
+        for (int r = tid; r < a.rows; r += kUpdThreads) s += a.rowloss[r];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
+        if (lane == 0) Pb[warp] = s;
+        __syncthreads();
+        if (tid == 0) {
+            float v = 0.f;
+            for (int w = 0; w < kUpdThreads / 32; ++w) v += Pb[w];
+            *a.loss_out = v / (float)a.rows;
+        }
+    }
 }
 
 template <typename K>
@@ -570,31 +724,26 @@ cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_fused_active(const FusedStepArgs& a, int grid, cudaStream_t s) {
+cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s) {
     static cudaError_t attr = set_smem_attr(fused_active_kernel);
     if (attr != cudaSuccess) return attr;
-    void* args[] = {(void*)&a};
-    return cudaLaunchCooperativeKernel((const void*)fused_active_kernel, dim3(grid), dim3(NT), args,
-                                       fused_smem_active(a.w_floats, a.act_ld, a.na, a.nt), s);
+    const int ntiles = (a.rows + R - 1) / R;
+    fused_active_kernel<<<ntiles, NT, fused_smem_active(a.w_floats, a.act_ld, a.na, a.nt), s>>>(a);
+    return cudaGetLastError();
 }
 
-cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, int grid, cudaStream_t s) {
+cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s) {
     static cudaError_t attr = set_smem_attr(fused_passive_bwd_kernel);
     if (attr != cudaSuccess) return attr;
-    void* args[] = {(void*)&a};
-    return cudaLaunchCooperativeKernel((const void*)fused_passive_bwd_kernel, dim3(grid), dim3(NT), args,
-                                       fused_smem_pbwd(a.w_floats, a.act_ld, a.na), s);
+    const int ntiles = (a.rows + R - 1) / R;
+    fused_passive_bwd_kernel<<<ntiles, NT, fused_smem_pbwd(a.w_floats, a.act_ld, a.na), s>>>(a);
+    return cudaGetLastError();
 }
 
-cudaError_t fused_max_grid(int which, size_t smem, int* ctas) {
-    int per_sm = 0, dev = 0, nsm = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    const void* f = which == 0 ? (const void*)fused_active_kernel : (const void*)fused_passive_bwd_kernel;
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedMaxSmem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, f, NT, smem);
-    *ctas = per_sm * nsm;
-    return e;
+cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s) {
+    if (a.ntiles < 1 || a.rows < 1) return cudaErrorInvalidValue;
+    fused_update_kernel<<<a.ntiles * kUpdCluster, kUpdThreads, 0, s>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace vfl

@@ -15,9 +15,29 @@ constexpr size_t kFusedMaxSmem = 227 * 1024;
 // forward's B fragments read 8 rows x 4 columns conflict-free), a 16-byte multiple
 inline int fused_act_stride(long long width) { return (int)(((width + 27) / 32) * 32 + 4); }
 inline int fused_w_stride(long long ld) { return fused_act_stride(ld); }
+// shared-memory floats of a staged layer: W in ceil8(out) rows of fused_w_stride, then b over ceil8(out)
+inline long long fused_layer_floats(int out, long long in_ld) {
+    const long long out8 = (out + 7) / 8 * 8;
+    return out8 * fused_w_stride(in_ld) + out8;
+}
+
+// Warp mapping of a 16-row tile GEMM with ks k-steps and ntl output blocks of 8
+// columns (kFusedThreads = 512, 16 warps): 2^lng warps cover the blocks, up to
+// 4 each (tpw), and 2^lkg groups of them split the k-steps, as many as fit the
+// 16 warps, the k-steps and the partial buffer (16 rows x (8 ntl + 8) floats
+// per group).  Packed as lng | lkg << 4 | tpw << 8.
+constexpr int kFusedRedFloats = 8192;
+inline __host__ __device__ int fused_gemm_map(int ks, int ntl) {
+    const int lng = ntl <= 4 ? 0 : ntl <= 8 ? 1 : ntl <= 16 ? 2 : 3;
+    const int tpw = (ntl + (1 << lng) - 1) >> lng;
+    int lkg = 4 - lng;
+    while (lkg > 0 && ((1 << lkg) > ks || ((16 * (8 * ntl + 8)) << lkg) > kFusedRedFloats)) --lkg;
+    return lng | lkg << 4 | tpw << 8;
+}
 
 struct FusedLayerArgs {
     int in, out;
+    int fmap, dmap;          // fused_gemm_map of the forward and of the input-gradient GEMM
     long long in_ld;         // row stride of W copies
     long long out_ld;        // row stride of activations this layer writes
     const float* W;          // weight version read by this step, [out, in_ld]
@@ -25,11 +45,7 @@ struct FusedLayerArgs {
     int ws_off;              // shared-memory offset (floats) of W, -1 when not staged
     int ws_ld;               // its shared-memory row stride (= 4 mod 32)
     float* Y; long long ldy; // forward output rows of this step (global)
-    float* D; long long ldd; // d(pre-activation) rows of this step (global), written in phase 1
-    long long poff;          // offset of this layer's [W | b] gradient in the flat parameter vector
-    float* Wm; float* bm;    // fp32 master (SGD)
-    float* Wc; float* bc;    // copy of the new version
-    float* gW; float* gb;    // reduced gradient (read back by vfl_get_grads)
+    float* D; long long ldd; // d(pre-activation) rows of this step (global)
 };
 
 // Passive forward of one step.
@@ -43,45 +59,82 @@ struct FusedChainArgs {
     long long k; int batch, version;
 };
 
-// Active step (L[0..na) = f_a, L[na..na+nt) = g) or passive backward (L[0..nl) = f_p).
+// Row-parallel part of the active step (L[0..na) = f_a, L[na..na+nt) = g) or of
+// the passive backward (L[0..na) = f_p, nt = 0): forward and input-gradient
+// chains, one 16-row tile per CTA; the weight gradients come from the update kernel.
 struct FusedStepArgs {
     FusedLayerArgs L[kFusedMaxLayers];
-    int na, nt;                         // passive backward: na = layers of f_p, nt = 0
+    int na, nt;
     int rows, act_ld, w_floats;
-    const float* x; long long ldx;      // active: x_a rows of the step; passive: x_p rows
+    const float* x; long long ldx;      // active: x_a rows of the step
     const int* y;                       // labels of the step's rows (active)
     int loss;
     const float* zp; long long ldzp;    // active: published embedding to read
+    float* zpc; long long ldzpc;        // active: copy of z^p kept for the weight gradient of g's first layer
     float* gradp; long long ldgp;       // active: gradient payload to publish; passive: to read
-    float* ds;                          // active: d(logits) [rows, n_out]
     float* rowloss;                     // active: per-row loss
-    float* loss_out;
-    float* part; long long ptotal;      // per-row-tile partial gradients [tiles][ptotal]
-    float lr;
     const ChannelHeader* chk_hdr;       // header to check (embedding / gradient channel)
     ChannelHeader* pub_hdr;             // header to publish (active: gradient channel)
+    int* counter;                       // active: CTAs done, for the last one to publish
     long long k; int batch, version;
     int* status;
 };
 
-// Shared memory: every staged weight matrix (w_floats, laid out by ws_off /
-// wts_off) followed by row-tile activation slots of kFusedRows x act_ld.
-// plus 1024 floats for the K-split partial sums of the tile GEMMs (8 tiles x 32 lanes x 4)
-constexpr int kFusedRedFloats = 1024;
+// Weight gradient + SGD of a set of layers: dW = D^T X and db = column sums of D
+// over the step's rows, then Eq. 2 on the master and the new version's copy.
+constexpr int kUpdThreads = 256;
+constexpr int kUpdCluster = 8;        // CTAs per output tile, each over 1/8 of the rows
+constexpr int kUpdTile = 32;          // output tile: 32 outputs x 32 inputs
+struct FusedUpdLayer {
+    int out, in;
+    long long in_ld;                  // row stride of the version copy
+    const float* D; long long ldd;    // d(pre-activation) rows [rows, out]
+    const float* X; long long ldx;    // input columns [0, xsplit)
+    const float* X2; long long ldx2;  // input columns [xsplit, in), indexed from 0
+    int xsplit;
+    int tile0, tiles_i;               // first output tile of this layer, tiles along the input
+    float* Wm; float* bm;             // fp32 master
+    float* Wc; float* bc;             // the new version's copy
+    float* gW; float* gb;             // the reduced gradient (read back by vfl_get_grads)
+};
+struct FusedUpdArgs {
+    FusedUpdLayer L[kFusedMaxLayers];
+    int nl, ntiles, rows;
+    float lr;
+    const float* rowloss;             // mean loss of the step from these (nullptr: none)
+    float* loss_out;
+};
+// Fills the tile bookkeeping of L[0..nl) and returns the number of output tiles.
+inline int fused_update_tiles(FusedUpdLayer* L, int nl) {
+    int t = 0;
+    for (int l = 0; l < nl; ++l) {
+        L[l].tile0 = t;
+        L[l].tiles_i = (L[l].in + kUpdTile - 1) / kUpdTile;
+        t += L[l].tiles_i * ((L[l].out + kUpdTile - 1) / kUpdTile);
+    }
+    return t;
+}
+
+// Shared memory: every staged weight matrix (w_floats, laid out by ws_off),
+// then fp32 row tiles of kFusedRows x act_ld floats, then kFusedRedFloats for
+// the partial output blocks of the tile GEMMs.
+// passive forward: x_p rows and a ping-pong pair
 inline size_t fused_smem_fwd(int w_floats, int act_ld) {
-    return (size_t)(w_floats + 2 * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
+    return (size_t)(w_floats + 3 * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
+// active step: x_a rows (later the logits), f_a's hidden outputs, [z^a | z^p],
+// g's hidden outputs, two gradients
 inline size_t fused_smem_active(int w_floats, int act_ld, int na, int nt) {
-    return (size_t)(w_floats + (na + nt + 4) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
+    return (size_t)(w_floats + (na + nt + 2) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
+// passive backward: f_p's saved outputs, dz^p rows, two gradients
 inline size_t fused_smem_pbwd(int w_floats, int act_ld, int nl) {
     return (size_t)(w_floats + (nl + 3) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
 
 cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s);
-cudaError_t launch_fused_active(const FusedStepArgs& a, int grid, cudaStream_t s);
-cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, int grid, cudaStream_t s);
-// Largest cooperative grid of the active (which = 0) or passive-backward (1) kernel with `smem` bytes.
-cudaError_t fused_max_grid(int which, size_t smem, int* ctas);
+cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s);
+cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s);
+cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s);
 
 }  // namespace vfl

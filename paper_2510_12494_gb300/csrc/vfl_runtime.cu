@@ -38,12 +38,12 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
-    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum"};
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update"};
 
 struct ProfRec {
     int cls;
@@ -124,12 +124,9 @@ struct vfl_ctx {
     // fused one-launch-per-phase path (narrow fp32 models)
     bool fused = false;
     int f_act_ld = 0, f_wp = 0, f_wa = 0;       // smem row stride, weight-stage floats per party
-    long long f_ptotal_p = 0, f_ptotal_a = 0;   // flat parameter counts
-    float* f_part_p = nullptr;                  // [tiles][ptotal_p]
-    float* f_part_a = nullptr;                  // [tiles][ptotal_a]
-    float* f_rowloss = nullptr;                 // [B]
-    int* f_counter = nullptr;
-    int f_grid_a = 1, f_grid_p = 1;
+    float* f_rowloss[kMaxWorkers] = {};         // per worker: per-row loss [B]
+    float* f_zpc[kMaxWorkers] = {};             // per worker: z^p rows consumed by the step [B, ld8(e_p)]
+    int* f_counter = nullptr;                   // last-CTA counters: [0, 16) passive fwd, [16, 32) active, per worker
 
     // streams / events
     cudaStream_t ps[kMaxWorkers] = {};
@@ -316,24 +313,22 @@ void choose_split(Layer& L, int B) {
 }
 
 // The fused path serves fp32 models whose every width fits one shared-memory
-// row tile, with one worker stream per party and no DP.
+// row tile, without DP.
 bool fused_eligible(const vfl_config& c) {
-    if (c.dtype != VFL_FP32 || c.workers != 1 || c.dp_clip > 0.f) return false;
+    if (c.dtype != VFL_FP32 || c.dp_clip > 0.f) return false;
     if (c.d_passive > kFusedMaxWidth || c.d_active > kFusedMaxWidth) return false;
     for (int i = 0; i < c.n_passive; ++i) if (c.passive_out[i] > kFusedMaxWidth) return false;
     for (int i = 0; i < c.n_active; ++i) if (c.active_out[i] > kFusedMaxWidth) return false;
     for (int i = 0; i < c.n_top; ++i) if (c.top_out[i] > kFusedMaxWidth) return false;
     if (c.active_out[c.n_active - 1] + c.passive_out[c.n_passive - 1] > kFusedMaxWidth) return false;
     if (c.n_active + c.n_top > kFusedMaxLayers) return false;
-    // the embeddings are copied into the top's input tile with 16-byte copies
-    if (c.active_out[c.n_active - 1] % 4 != 0 || c.passive_out[c.n_passive - 1] % 4 != 0) return false;
+    // z^p lands in the top's input tile after z^a's 8-column blocks, by 16-byte copies
+    if (c.active_out[c.n_active - 1] % 8 != 0 || c.passive_out[c.n_passive - 1] % 4 != 0) return false;
     return true;
 }
 
-// Shared-memory layout of one fused launch: which layers stage W (for input
-// gradients) and W^T (for the forward).  Returns the floats used.
 // Shared-memory layout of the weights one fused launch stages: layers
-// [w_from, n) get W.  Returns the floats used.
+// [w_from, n) get W and b.  Returns the floats used.
 int fused_weight_layout(FusedLayerArgs* L, int n, int w_from) {
     int off = 0;
     for (int l = 0; l < n; ++l) {
@@ -341,7 +336,7 @@ int fused_weight_layout(FusedLayerArgs* L, int n, int w_from) {
         L[l].ws_off = -1;
         if (l >= w_from) {
             L[l].ws_off = off;
-            off += L[l].out * L[l].ws_ld;
+            off += (int)fused_layer_floats(L[l].out, L[l].in_ld);
         }
     }
     return off;
@@ -388,27 +383,20 @@ void build_layers(vfl_ctx* ctx) {
     if (ctx->fused) {
         int maxw = std::max(c.d_passive, c.d_active);
         ctx->f_wp = ctx->f_wa = 0;
-        ctx->f_ptotal_p = ctx->f_ptotal_a = 0;
-        for (const Layer& L : ctx->P) {
-            maxw = std::max(maxw, std::max(L.in, L.out));
-            ctx->f_ptotal_p += (long long)L.out * L.in + L.out;
-        }
+        for (const Layer& L : ctx->P) maxw = std::max(maxw, std::max(L.in, L.out));
         for (auto* v : {&ctx->A, &ctx->T})
-            for (const Layer& L : *v) {
-                maxw = std::max(maxw, std::max(L.in, L.out));
-                ctx->f_ptotal_a += (long long)L.out * L.in + L.out;
-            }
+            for (const Layer& L : *v) maxw = std::max(maxw, std::max(L.in, L.out));
         ctx->f_act_ld = fused_act_stride(ld8(maxw));
         // staged weights per launch (row-major W): every layer of f_p for the forward, every layer of
         // f_a and g for the active step, f_p's layers after the first for the backward
         long long w_pf = 0, w_pb = 0, w_a = 0;
         for (size_t l = 0; l < ctx->P.size(); ++l) {
-            const long long w = (long long)ctx->P[l].out * fused_w_stride(ctx->P[l].in_ld);
+            const long long w = fused_layer_floats(ctx->P[l].out, ctx->P[l].in_ld);
             w_pf += w;
             if (l > 0) w_pb += w;
         }
         for (auto* v : {&ctx->A, &ctx->T})
-            for (const Layer& L : *v) w_a += (long long)L.out * fused_w_stride(L.in_ld);
+            for (const Layer& L : *v) w_a += fused_layer_floats(L.out, L.in_ld);
         ctx->f_wp = (int)std::max(w_pf, w_pb);
         ctx->f_wa = (int)w_a;
         const size_t sa = fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size());
@@ -486,11 +474,11 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
         }
     ctx->scratch_f32 = static_cast<float*>(cv.take(std::max(B * ld8(maxw), maxwt) * 4ull));
     if (ctx->fused) {
-        const long long tiles = (B + kFusedRows - 1) / kFusedRows;
-        ctx->f_part_p = static_cast<float*>(cv.take((unsigned long long)tiles * ctx->f_ptotal_p * 4));
-        ctx->f_part_a = static_cast<float*>(cv.take((unsigned long long)tiles * ctx->f_ptotal_a * 4));
-        ctx->f_rowloss = static_cast<float*>(cv.take(B * 4ull));
-        ctx->f_counter = static_cast<int*>(cv.take(256));
+        for (int w = 0; w < ctx->W; ++w) {
+            ctx->f_rowloss[w] = static_cast<float*>(cv.take(B * 4ull));
+            ctx->f_zpc[w] = static_cast<float*>(cv.take(B * ld8(ctx->P.back().out) * 4ull));
+        }
+        ctx->f_counter = static_cast<int*>(cv.take(2 * kMaxWorkers * sizeof(int)));
     }
     return cv.off + 256;
 }
@@ -672,12 +660,13 @@ vfl_status wait_ev(vfl_ctx* ctx, cudaStream_t s, cudaEvent_t e) {
     } while (0)
 
 // ---- fused path -------------------------------------------------------------
-FusedLayerArgs fused_layer(const Layer& L, int vslot, int new_slot, int w, void* Y, long long ldy, void* D,
-                           long long ldd, long long poff) {
+FusedLayerArgs fused_layer(const Layer& L, int vslot, void* Y, long long ldy, void* D, long long ldd) {
     FusedLayerArgs f;
     std::memset(&f, 0, sizeof f);
     f.in = L.in;
     f.out = L.out;
+    f.fmap = fused_gemm_map((L.in + 7) / 8, (L.out + 7) / 8);
+    f.dmap = fused_gemm_map((L.out + 7) / 8, (L.in + 7) / 8);
     f.in_ld = L.in_ld;
     f.out_ld = ld8(L.out);
     f.W = static_cast<const float*>(L.cW[vslot]);
@@ -686,40 +675,76 @@ FusedLayerArgs fused_layer(const Layer& L, int vslot, int new_slot, int w, void*
     f.ldy = ldy;
     f.D = static_cast<float*>(D);
     f.ldd = ldd;
-    f.poff = poff;
-    f.Wm = L.W;
-    f.bm = L.b;
-    f.Wc = static_cast<float*>(L.cW[new_slot]);
-    f.bc = L.cb[new_slot];
-    f.gW = L.pW[w];
-    f.gb = L.pb[w];
     return f;
 }
 
-double fused_flops(const std::vector<Layer>& v, int rows, bool fwd, bool dx_first, bool dw) {
+// Update of layer L from its d(pre) rows D and input rows [X | X2] (X2 from column xsplit on).
+FusedUpdLayer fused_upd_layer(const Layer& L, int new_slot, int w, const void* D, long long ldd, const void* X,
+                              long long ldx, const void* X2, long long ldx2, int xsplit) {
+    FusedUpdLayer u;
+    std::memset(&u, 0, sizeof u);
+    u.out = L.out;
+    u.in = L.in;
+    u.in_ld = L.in_ld;
+    u.D = static_cast<const float*>(D);
+    u.ldd = ldd;
+    u.X = static_cast<const float*>(X);
+    u.ldx = ldx;
+    u.X2 = static_cast<const float*>(X2 ? X2 : X);
+    u.ldx2 = X2 ? ldx2 : ldx;
+    u.xsplit = X2 ? xsplit : L.in;
+    u.Wm = L.W;
+    u.bm = L.b;
+    u.Wc = static_cast<float*>(L.cW[new_slot]);
+    u.bc = L.cb[new_slot];
+    u.gW = L.pW[w];
+    u.gb = L.pb[w];
+    return u;
+}
+
+// 2 rows in out FLOPs per layer for each of: forward, input gradient (all layers
+// but the first unless dx_first), weight gradient.
+double fused_flops(const std::vector<Layer>& v, int rows, bool fwd, bool dx, bool dx_first, bool dw) {
     double f = 0;
     for (size_t l = 0; l < v.size(); ++l) {
         const double mn = 2.0 * rows * v[l].in * v[l].out;
         if (fwd) f += mn;
+        if (dx && (dx_first || l > 0)) f += mn;
         if (dw) f += mn;
-        if (dx_first || l > 0) f += dw ? mn : 0;
     }
     return f;
 }
 
+vfl_status launch_update(vfl_ctx* ctx, FusedUpdArgs& u, int rows, cudaStream_t s) {
+    u.ntiles = fused_update_tiles(u.L, u.nl);
+    u.rows = rows;
+    u.lr = ctx->cfg.lr;
+    // algorithmic: dW = D^T X per layer; D and X read once, 16 B per parameter
+    // (master read + write, gradient and new copy written)
+    double flops = 0, bytes = 0;
+    for (int l = 0; l < u.nl; ++l) {
+        const FusedUpdLayer& L = u.L[l];
+        flops += 2.0 * rows * L.out * L.in;
+        bytes += (double)rows * (L.out + L.in) * 4 + ((double)L.out * L.in + L.out) * 16;
+    }
+    if (u.loss_out) bytes += rows * 4.0 + 4;
+    PLAUNCH(K_FUSED_UPDATE, flops, bytes, s, launch_fused_update(u, s));
+    return VFL_OK;
+}
+
 vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slot, int vslot, int rows,
-                                 const float* X, cudaStream_t s) {
+                                 const float* X, int w, cudaStream_t s) {
     FusedChainArgs a;
     std::memset(&a, 0, sizeof a);
     a.nl = (int)ctx->P.size();
     for (int l = 0; l < a.nl; ++l)
-        a.L[l] = fused_layer(ctx->P[l], vslot, vslot, 0, ctx->act_p[slot][l], ld8(ctx->P[l].out), nullptr, 0, 0);
+        a.L[l] = fused_layer(ctx->P[l], vslot, ctx->act_p[slot][l], ld8(ctx->P[l].out), nullptr, 0);
     a.x = X;
     a.ldx = ctx->ldxp;
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
     a.w_floats = fused_weight_layout(a.L, a.nl, 0);
-    a.counter = ctx->f_counter;
+    a.counter = ctx->f_counter + w;
     a.hdr = ctx->emb_hdr + slot;
     a.k = k;
     a.batch = (int)(k % ctx->nb);
@@ -727,31 +752,29 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     // algorithmic bytes: the batch's features in, the saved activations out, one read of the weights
     double bytes = (double)rows * ctx->cfg.d_passive * 4;
     for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 4;
-    PLAUNCH(K_FUSED_PFWD, fused_flops(ctx->P, rows, true, false, false), bytes, s, launch_fused_passive_fwd(a, s));
+    PLAUNCH(K_FUSED_PFWD, fused_flops(ctx->P, rows, true, false, false, false), bytes, s,
+            launch_fused_passive_fwd(a, s));
     return VFL_OK;
 }
 
+// Active party, row-parallel part: forward, loss, input gradients, dz^p published.
 vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, int vslot, int rows,
-                             const float* Xa, cudaStream_t s) {
+                             const float* Xa, int w, cudaStream_t s) {
     FusedStepArgs a;
     std::memset(&a, 0, sizeof a);
     const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size();
-    const int new_slot = (int)((k + 1) % ctx->S1);
     const int n_out = ctx->T.back().out;
-    long long off = 0;
     for (int l = 0; l < La; ++l) {
         const Layer& L = ctx->A[l];
-        a.L[l] = fused_layer(L, vslot, new_slot, 0, ctx->act_a[0][l], ld8(L.out), ctx->dpre_a[0][l], ld8(L.out), off);
-        off += (long long)L.out * L.in + L.out;
+        a.L[l] = fused_layer(L, vslot, ctx->act_a[w][l], ld8(L.out), ctx->dpre_a[w][l], ld8(L.out));
     }
     for (int l = 0; l < Lt; ++l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
-        a.L[La + l] = fused_layer(L, vslot, new_slot, 0, last ? (void*)ctx->logits[0] : ctx->act_t[0][l],
-                                  last ? n_out : ld8(L.out), last ? (void*)ctx->ds[0] : ctx->dpre_t[0][l],
-                                  last ? n_out : ld8(L.out), off);
-        off += (long long)L.out * L.in + L.out;
+        a.L[La + l] = fused_layer(L, vslot, last ? (void*)ctx->logits[w] : ctx->act_t[w][l], last ? n_out : ld8(L.out),
+                                  last ? (void*)ctx->ds[w] : ctx->dpre_t[w][l], last ? n_out : ld8(L.out));
     }
+    const int ep = ctx->P.back().out;
     a.na = La;
     a.nt = Lt;
     a.rows = rows;
@@ -764,71 +787,107 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     a.y = ctx->Y + r0;
     a.loss = ctx->cfg.loss;
     a.zp = static_cast<const float*>(ctx->act_p[slot].back());
-    a.ldzp = ld8(ctx->P.back().out);
+    a.ldzp = ld8(ep);
+    a.zpc = ctx->f_zpc[w];
+    a.ldzpc = ld8(ep);
     a.gradp = static_cast<float*>(ctx->grad[slot]);
-    a.ldgp = ld8(ctx->P.back().out);
-    a.ds = ctx->ds[0];
-    a.rowloss = ctx->f_rowloss;
-    a.loss_out = ctx->losses + (k % kLossCap);
-    a.part = ctx->f_part_a;
-    a.ptotal = ctx->f_ptotal_a;
-    a.lr = ctx->cfg.lr;
+    a.ldgp = ld8(ep);
+    a.rowloss = ctx->f_rowloss[w];
     a.chk_hdr = ctx->emb_hdr + slot;
     a.pub_hdr = ctx->grad_hdr + slot;
+    a.counter = ctx->f_counter + kMaxWorkers + w;
     a.k = k;
     a.batch = (int)(k % ctx->nb);
     a.version = (int)v;
     a.status = ctx->status;
-    const int tiles = (rows + kFusedRows - 1) / kFusedRows;
-    const int want = std::max<long long>(tiles, (ctx->f_ptotal_a + kFusedThreads - 1) / kFusedThreads);
-    const int grid = std::max(1, std::min(want, ctx->f_grid_a));
-    const double flops = fused_flops(ctx->A, rows, true, false, true) + fused_flops(ctx->T, rows, true, true, true);
-    // algorithmic bytes: x^a, labels and z^p in, dz^p out; every weight read once,
-    // its master read and written, and the new version's copy written
-    double bytes = (double)rows * (ctx->cfg.d_active + 2.0 * ctx->P.back().out + 1) * 4;
+    const double flops = fused_flops(ctx->A, rows, true, true, false, false) + fused_flops(ctx->T, rows, true, true, true, false);
+    // algorithmic bytes: x^a, labels and z^p in; every layer's output and
+    // d(pre-activation) out, z^p's copy and dz^p out; every weight read once
+    double bytes = (double)rows * (ctx->cfg.d_active + 3.0 * ep + 2) * 4;
     for (auto* vv : {&ctx->A, &ctx->T})
-        for (const Layer& L : *vv) bytes += ((double)L.out * L.in + L.out) * 16;
-    PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, grid, s));
+        for (const Layer& L : *vv) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 4;
+    PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, s));
     return VFL_OK;
 }
 
-vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot, int rows, const float* Xp,
-                                  cudaStream_t s) {
+// Active party's weight gradients of f_a and g, and SGD to version k+1.
+vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float* Xa, int w, cudaStream_t s) {
+    FusedUpdArgs u;
+    std::memset(&u, 0, sizeof u);
+    const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size();
+    const int new_slot = (int)((k + 1) % ctx->S1);
+    const int n_out = ctx->T.back().out;
+    const int ea = ctx->A.back().out, ep = ctx->P.back().out;
+    int n = 0;
+    for (int l = 0; l < La; ++l) {
+        const Layer& L = ctx->A[l];
+        const void* X = l == 0 ? (const void*)Xa : ctx->act_a[w][l - 1];
+        const long long ldx = l == 0 ? ctx->ldxa : ld8(ctx->A[l - 1].out);
+        u.L[n++] = fused_upd_layer(L, new_slot, w, ctx->dpre_a[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
+    }
+    for (int l = 0; l < Lt; ++l) {
+        const Layer& L = ctx->T[l];
+        const bool last = l == Lt - 1;
+        const void* D = last ? (const void*)ctx->ds[w] : ctx->dpre_t[w][l];
+        const long long ldd = last ? n_out : ld8(L.out);
+        if (l == 0)
+            u.L[n++] = fused_upd_layer(L, new_slot, w, D, ldd, ctx->act_a[w][La - 1], ld8(ea), ctx->f_zpc[w], ld8(ep), ea);
+        else
+            u.L[n++] = fused_upd_layer(L, new_slot, w, D, ldd, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr,
+                                       0, 0);
+    }
+    u.nl = n;
+    u.rowloss = ctx->f_rowloss[w];
+    u.loss_out = ctx->losses + (k % kLossCap);
+    return launch_update(ctx, u, rows, s);
+}
+
+// Passive party, row-parallel part of the backward phase: d(pre) of every layer of f_p.
+vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot, int rows, int w, cudaStream_t s) {
     FusedStepArgs a;
     std::memset(&a, 0, sizeof a);
     const int Lp = (int)ctx->P.size();
-    const int new_slot = (int)((k + 1) % ctx->S1);
-    long long off = 0;
     for (int l = 0; l < Lp; ++l) {
         const Layer& L = ctx->P[l];
-        a.L[l] = fused_layer(L, vslot, new_slot, 0, ctx->act_p[slot][l], ld8(L.out), ctx->dpre_p[0][l], ld8(L.out),
-                             off);
-        off += (long long)L.out * L.in + L.out;
+        a.L[l] = fused_layer(L, vslot, ctx->act_p[slot][l], ld8(L.out), ctx->dpre_p[w][l], ld8(L.out));
     }
     a.na = Lp;
     a.nt = 0;
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
     a.w_floats = fused_weight_layout(a.L, Lp, 1);
-    a.x = Xp;
-    a.ldx = ctx->ldxp;
     a.gradp = static_cast<float*>(ctx->grad[slot]);
     a.ldgp = ld8(ctx->P.back().out);
-    a.part = ctx->f_part_p;
-    a.ptotal = ctx->f_ptotal_p;
-    a.lr = ctx->cfg.lr;
     a.chk_hdr = ctx->grad_hdr + slot;
     a.k = k;
     a.status = ctx->status;
-    const int tiles = (rows + kFusedRows - 1) / kFusedRows;
-    const int want = std::max<long long>(tiles, (ctx->f_ptotal_p + kFusedThreads - 1) / kFusedThreads);
-    const int grid = std::max(1, std::min(want, ctx->f_grid_p));
-    // algorithmic bytes: x^p, dz^p and the saved activations in; weights as in the active step
-    double bytes = (double)rows * (ctx->cfg.d_passive + ctx->P.back().out) * 4;
-    for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 16;
-    PLAUNCH(K_FUSED_PBWD, fused_flops(ctx->P, rows, false, false, true), bytes, s,
-            launch_fused_passive_bwd(a, grid, s));
+    // algorithmic bytes: dz^p and the saved activations in, every d(pre) out, weights after the first read once
+    double bytes = (double)rows * ctx->P.back().out * 4;
+    for (size_t l = 0; l < ctx->P.size(); ++l) {
+        const Layer& L = ctx->P[l];
+        bytes += (double)rows * L.out * 8;
+        if (l > 0) bytes += ((double)L.out * L.in + L.out) * 4;
+    }
+    PLAUNCH(K_FUSED_PBWD, fused_flops(ctx->P, rows, false, true, false, false), bytes, s,
+            launch_fused_passive_bwd(a, s));
     return VFL_OK;
+}
+
+// Passive party's weight gradients of f_p and SGD to version k+1.
+vfl_status fused_passive_update(vfl_ctx* ctx, long long k, int slot, int rows, const float* Xp, int w,
+                                cudaStream_t s) {
+    FusedUpdArgs u;
+    std::memset(&u, 0, sizeof u);
+    const int Lp = (int)ctx->P.size();
+    const int new_slot = (int)((k + 1) % ctx->S1);
+    for (int l = 0; l < Lp; ++l) {
+        const Layer& L = ctx->P[l];
+        const void* X = l == 0 ? (const void*)Xp : ctx->act_p[slot][l - 1];
+        const long long ldx = l == 0 ? ctx->ldxp : ld8(ctx->P[l - 1].out);
+        u.L[l] = fused_upd_layer(L, new_slot, w, ctx->dpre_p[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
+    }
+    u.nl = Lp;
+    return launch_update(ctx, u, rows, s);
 }
 
 // ---- the three phases ------------------------------------------------------
@@ -851,7 +910,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
     const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
     if (ctx->fused) {
-        TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), s));
+        TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), (int)(k % ctx->W), s));
         CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
         ctx->fwd_version[slot] = (int)v;
         ctx->slot_step_p[slot] = k;
@@ -898,9 +957,11 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const void* Xa0 = static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * es;
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
-        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
-        TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), s));
+        TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), w, s));
         CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
+        // SGD on theta_1 in step order: version k+1 from version k
+        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+        TRY(fused_active_update(ctx, k, rows, static_cast<const float*>(Xa0), w, s));
         CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
         ctx->grad_step[slot] = k;
         ctx->last_act_step[w] = k;
@@ -1001,9 +1062,11 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
     if (ctx->fused) {
-        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
         const float* Xp = reinterpret_cast<const float*>(static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz);
-        TRY(fused_passive_backward(ctx, k, slot, vslot, rows, Xp, s));
+        TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
+        // SGD on theta_2 in step order
+        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+        TRY(fused_passive_update(ctx, k, slot, rows, Xp, w, s));
         CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
         ctx->n_bwd = k + 1;
         return VFL_OK;
@@ -1135,15 +1198,6 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     if (e == cudaSuccess) e = cudaMemset(workspace, 0, need);
     if (e == cudaSuccess) e = cudaMemset(ctx->emb_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
     if (e == cudaSuccess) e = cudaMemset(ctx->grad_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
-    if (e == cudaSuccess && ctx->fused) {
-        long long w_p = 0;
-        for (size_t l = 1; l < ctx->P.size(); ++l) w_p += (long long)ctx->P[l].out * fused_w_stride(ctx->P[l].in_ld);
-        e = fused_max_grid(0, fused_smem_active(ctx->f_wa, ctx->f_act_ld, (int)ctx->A.size(), (int)ctx->T.size()),
-                           &ctx->f_grid_a);
-        if (e == cudaSuccess)
-            e = fused_max_grid(1, fused_smem_pbwd((int)w_p, ctx->f_act_ld, (int)ctx->P.size()), &ctx->f_grid_p);
-        if (e == cudaSuccess && (ctx->f_grid_a < 1 || ctx->f_grid_p < 1)) e = cudaErrorInvalidConfiguration;
-    }
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         g_global_err = std::string("vfl_create: ") + cudaGetErrorString(e);

@@ -165,7 +165,7 @@ PRESETS = {
     1: VflPreset(1, "tiny-sync", 4096, 10, 10, (32, 16), (32, 16), (32, 1), "bce",
                  256, 1, 0.01, 0, "sync", "fp32", 1),
     2: VflPreset(2, "credit-shaped", 30000, 12, 11, (128, 64), (128, 64), (64, 1), "bce",
-                 1024, 5, 0.01, 2, "seeded", "fp32", 1),
+                 1024, 5, 0.01, 2, "seeded", "fp32", 2),
     3: VflPreset(3, "multiclass", 500000, 27, 27, (256, 256, 128), (256, 256, 128), (256, 7), "ce",
                  4096, 1, 0.01, 2, "seeded", "bf16", 1),
     4: VflPreset(4, "wide-dp", 1000000, 1000, 1000, (512, 256), (512, 256), (256, 1), "bce",

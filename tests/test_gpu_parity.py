@@ -55,13 +55,15 @@ def force_gpu_state(ctx, o, S):
         ctx.set_version(v, oracle_version(o, v))
 
 
-def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None):
+def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=None):
     """Step-by-step comparison.  bf16 presets are teacher-forced: before each
     step the GPU takes the oracle's weight versions, so one step's error is
     measured without the drift of earlier roundings (a bf16 weight copy that
     rounds the other way moves later ReLU masks)."""
     import synth
     p = synth.preset(cid)
+    if workers:
+        p = p.with_(workers=workers)
     q, xp, xa, y, params = setup(p, n_rows)
     nb = -(-n_rows // q.batch)
     steps = steps or nb + 2                      # one epoch and two steps of the next
@@ -91,6 +93,33 @@ def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None):
 def test_step_parity(vfl, cid):
     worst, failures = run_sequential(vfl, cid, CASES[cid])
     assert not failures, f"preset {cid}: {failures[:3]}; worst {sorted(worst.items(), key=lambda t: -t[1])[:6]}"
+
+
+def test_step_parity_worker_streams(vfl):
+    """Several worker streams per party: each step's buffers and gradient
+    partials live with its worker (k mod W), and every step still matches."""
+    worst, failures = run_sequential(vfl, 2, CASES[2], workers=3)
+    assert not failures, f"{failures[:3]}; worst {sorted(worst.items(), key=lambda t: -t[1])[:6]}"
+
+
+@pytest.mark.parametrize("cid", [1, 2])
+def test_worker_streams_equal_one_stream(vfl, cid):
+    """With W worker streams per party the steps that the schedule's staleness
+    allows run concurrently; the result is bit-identical to one stream."""
+    import synth
+    q, xp, xa, y, params = setup(synth.preset(cid), CASES[cid] if cid == 1 else 4 * 1024 + 304)
+    n = 2 * q.steps_per_epoch + 1
+    tp, ta = schedule(q, n)
+    one = new_context(vfl, q.with_(workers=1), xp, xa, y, params)
+    one.train_steps(0, n, tp, ta)
+    for w in (2, 3):
+        many = new_context(vfl, q.with_(workers=w), xp, xa, y, params)
+        many.train_steps(0, n, tp, ta)
+        np.testing.assert_array_equal(many.read_losses(0, n), one.read_losses(0, n))
+        for key, (W, b) in one.get_params().items():
+            W2, b2 = many.get_params()[key]
+            np.testing.assert_array_equal(W, W2)
+            np.testing.assert_array_equal(b, b2)
 
 
 @pytest.mark.parametrize("cid", [1, 2])
@@ -182,12 +211,14 @@ def test_step_parity_generic_kernels(vfl, cid, monkeypatch):
     assert not failures, f"preset {cid}: {failures[:3]}"
 
 
-@pytest.mark.parametrize("cid", [2, 3])
-def test_graph_replay_equals_direct_enqueue(vfl, cid):
+@pytest.mark.parametrize("cid,workers", [(2, 0), (2, 3), (3, 0)])
+def test_graph_replay_equals_direct_enqueue(vfl, cid, workers):
     """A captured CUDA graph of a window of steps replays exactly what the
     direct enqueue computes, advances the cursor, and refuses the wrong cursor."""
     import synth
     p = synth.preset(cid)
+    if workers:
+        p = p.with_(workers=workers)
     q, xp, xa, y, params = setup(p, CASES[cid])
     n = q.steps_per_epoch + 2
     tp, ta = schedule(q, 2 * n)
