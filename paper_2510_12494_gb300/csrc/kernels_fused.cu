@@ -83,8 +83,20 @@ __device__ void async_rows(float* s, int lds, const float* g, long long ldg, int
     }
 }
 
-// rows x cols floats (cols % 4 == 0, 16-byte aligned rows) into smem rows of stride lds, asynchronously
+// rows x cols floats (cols % 4 == 0, 16-byte aligned rows) into smem rows of stride lds, asynchronously.
+// A source whose rows are contiguous (ldg == cols) with a power-of-two number of 16-byte chunks per row
+// is walked chunk by chunk over all lanes (narrow rows would otherwise leave most lanes of each
+// copy instruction idle, and the copies cost per instruction, not per byte).
 __device__ void async_matrix(float* s, int lds, const float* g, long long ldg, int rows, int cols) {
+    const int q = cols >> 2;
+    if (ldg == cols && (q & (q - 1)) == 0) {
+        const int lq = __ffs(q) - 1;
+        for (int i = threadIdx.x; i < rows * q; i += NT) {
+            const int r = i >> lq, c = (i & (q - 1)) << 2;
+            cp16(s + r * lds + c, g + (long long)r * ldg + c);
+        }
+        return;
+    }
     for (int r = threadIdx.x >> 5; r < rows; r += NW)
         for (int c = (threadIdx.x & 31) * 4; c < cols; c += 128) cp16(s + r * lds + c, g + (long long)r * ldg + c);
 }
@@ -346,8 +358,115 @@ __device__ void publish_when_last(int* counter, ChannelHeader* hdr, long long k,
     }
 }
 
+// Loss of one row (Eq. 1 in the stable logit form, or softmax cross-entropy)
+// from its n_out logits s; writes d(logits) = dloss/ds / B to d.
+__device__ __forceinline__ float loss_row(const float* s, int nout, int y, int loss, float inv_b, float* d) {
+    if (loss == VFL_LOSS_BCE) {
+        const float x = s[0];
+        d[0] = (1.0f / (1.0f + expf(-x)) - (float)y) * inv_b;
+        return fmaxf(x, 0.f) - x * (float)y + log1pf(expf(-fabsf(x)));
+    }
+    float m = s[0];
+    for (int j = 1; j < nout; ++j) m = fmaxf(m, s[j]);
+    float z = 0.f;
+    for (int j = 0; j < nout; ++j) z += expf(s[j] - m);
+    const float iz = 1.0f / z;
+    for (int j = 0; j < nout; ++j) d[j] = (expf(s[j] - m) * iz - (j == y ? 1.f : 0.f)) * inv_b;
+    return logf(z) + m - s[y];
+}
+
+// g's last hidden layer Lh (input X) with the output layer Lo (n_out <= kFusedMaxOut),
+// the loss and its gradient folded into the epilogue, warp r for row r:
+// h = ReLU(X Wh^T + bh) -> smem tile `hs` and Lh.Y; s = h Wo^T + bo (fp32 dot
+// products, reduced across the warp) -> Lo.Y; the row's loss -> rowloss;
+// ds = dloss/ds / B -> Lo.D; dh = (ds Wo) * [h > 0] -> smem tile `gs` and Lh.D.
+// The layers' fields come as scalars (Lh: hidden, Lo: output): a struct
+// reference into kernel parameters would be copied to local memory per call.
+struct TopLast {
+    int h_in, h_out, h_map, h_ws_off, h_ws_ld;
+    int o_out, o_ws_off, o_ws_ld;
+    float* h_y; long long h_ldy;
+    float* h_d; long long h_ldd;
+    float* o_y; long long o_ldy;
+    float* o_d; long long o_ldd;
+};
+
+__device__ __noinline__ void top_last_fused(const float* X, int ld, const float* ws, TopLast L, float* hs, float* gs,
+                                            const int* y, int loss, float inv_b, float* rowloss, int r0, int nr,
+                                            float* red) {
+    const int ntl = ceil8(L.h_out) / 8;
+    gemm_partials<false>(X, ld, ceil8(L.h_in) / 8, ws + L.h_ws_off, L.h_ws_ld, ntl, L.h_map, red);
+    __syncthreads();
+    const int lane = threadIdx.x & 31, r = threadIdx.x >> 5;
+    const int rs = 8 * ntl + 8, kg = 1 << ((L.h_map >> 4) & 15);
+    const int nout = L.o_out;
+    const float* bh = ws + L.h_ws_off + ceil8(L.h_out) * L.h_ws_ld;
+    const float* wo = ws + L.o_ws_off;
+    const int ldo = L.o_ws_ld;
+    const bool valid = r < nr;
+    float part[kFusedMaxOut];
+#pragma unroll
+    for (int j = 0; j < kFusedMaxOut; ++j) part[j] = 0.f;
+    for (int c = 2 * lane; c < 8 * ntl; c += 64) {
+        const float* src = red + r * rs + c;
+        float2 v = *reinterpret_cast<const float2*>(src);
+#pragma unroll 4
+        for (int q = 1; q < kg; ++q) {
+            const float2 u = *reinterpret_cast<const float2*>(src + q * 16 * rs);
+            v.x += u.x;
+            v.y += u.y;
+        }
+        const float2 h = make_float2(fmaxf(v.x + bh[c], 0.f), fmaxf(v.y + bh[c + 1], 0.f));
+        *reinterpret_cast<float2*>(hs + r * ld + c) = h;
+        if (valid) *reinterpret_cast<float2*>(L.h_y + (long long)(r0 + r) * L.h_ldy + c) = h;
+#pragma unroll
+        for (int j = 0; j < kFusedMaxOut; ++j)
+            if (j < nout) part[j] = fmaf(h.x, wo[j * ldo + c], fmaf(h.y, wo[j * ldo + c + 1], part[j]));
+    }
+    float sv[kFusedMaxOut], dv[kFusedMaxOut];
+    const float* bo = wo + ceil8(nout) * ldo;
+#pragma unroll
+    for (int j = 0; j < kFusedMaxOut; ++j) {
+        if (j < nout) {
+            float t = part[j];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            sv[j] = t + bo[j];
+        }
+    }
+    const float li = loss_row(sv, nout, valid ? y[r] : 0, loss, inv_b, dv);
+    if (!valid)
+#pragma unroll
+        for (int j = 0; j < kFusedMaxOut; ++j) dv[j] = 0.f;
+    if (valid && lane == 0) {
+        rowloss[r] = li;
+        float* lo = L.o_y + (long long)(r0 + r) * L.o_ldy;
+        float* dl = L.o_d + (long long)(r0 + r) * L.o_ldd;
+        for (int j = 0; j < nout; ++j) {
+            lo[j] = sv[j];
+            dl[j] = dv[j];
+        }
+    }
+    __syncwarp();
+    for (int c = 2 * lane; c < 8 * ntl; c += 64) {
+        float g0 = 0.f, g1 = 0.f;
+#pragma unroll
+        for (int j = 0; j < kFusedMaxOut; ++j)
+            if (j < nout) {
+                g0 = fmaf(dv[j], wo[j * ldo + c], g0);
+                g1 = fmaf(dv[j], wo[j * ldo + c + 1], g1);
+            }
+        const float2 h = *reinterpret_cast<const float2*>(hs + r * ld + c);
+        const float2 gd = make_float2(h.x > 0.f ? g0 : 0.f, h.y > 0.f ? g1 : 0.f);
+        *reinterpret_cast<float2*>(gs + r * ld + c) = gd;
+        if (valid) *reinterpret_cast<float2*>(L.h_d + (long long)(r0 + r) * L.h_ldd + c) = gd;
+    }
+}
+
 __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
+    // the embedding channel's header, checked at the end (a load that nothing waits for until then)
+    const long long hdr_k = threadIdx.x == 0 ? a.chk_hdr->k : 0;
     const int La = a.na, Lt = a.nt;
     const int ld = a.act_ld;
     float* ws = smem;
@@ -362,7 +481,6 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
     float* G0 = slot(La + Lt);
     float* G1 = slot(La + Lt + 1);
     float* red = slot(La + Lt + 2);
-    if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* A = a.L;
     const FusedLayerArgs* T = a.L + La;
     const int ea = A[La - 1].out;
@@ -404,68 +522,67 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
             tile_fwd(l == 0 ? X : H(l - 1), ld, A[l].in, ws + A[l].ws_off, A[l].ws_ld, staged_bias(ws, A[l]), A[l].out,
                      A[l].fmap, l == La - 1 ? C : H(l), A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
         }
+        // with n_out <= kFusedMaxOut, g's output layer, the loss, d(logits) and the output layer's input
+        // gradient ride in the epilogue of g's last hidden layer (one warp per row)
+        const bool fuse_out = Lt >= 2 && nout <= kFusedMaxOut;
         for (int l = 0; l < Lt - 1; ++l) {                               // g's hidden layers on [z^a | z^p]
             if (first)
-                cp_wait_pending(Lt - 1 - l);
+                cp_wait_pending(fuse_out && l == Lt - 2 ? 0 : Lt - 1 - l);
             else
                 __syncthreads();
-            tile_fwd(l == 0 ? C : TH(l - 1), ld, T[l].in, ws + T[l].ws_off, T[l].ws_ld, staged_bias(ws, T[l]), T[l].out,
-                     T[l].fmap, TH(l), T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
-        }
-        float* lg = X;                                                   // x_a's tile is free again
-        {                                                                // logits: no activation
-            const FusedLayerArgs& L = T[Lt - 1];
-            if (first)
-                cp_wait_pending(0);
-            else
-                __syncthreads();
-            const float* bias = staged_bias(ws, L);
-            float* yg = L.Y + (long long)r0 * L.ldy;
-            const long long ldy = L.ldy;
-            tile_gemm<false>(Lt == 1 ? C : TH(Lt - 2), ld, ceil8(L.in) / 8, ws + L.ws_off, L.ws_ld, ceil8(nout) / 8, L.fmap, red,
-                             [&](int r, int c, float v0, float v1) {
-                                 v0 += bias[c];
-                                 v1 += bias[c + 1];
-                                 *reinterpret_cast<float2*>(lg + r * ld + c) = make_float2(v0, v1);
-                                 if (r < nr) {
-                                     if (c < nout) yg[(long long)r * ldy + c] = v0;
-                                     if (c + 1 < nout) yg[(long long)r * ldy + c + 1] = v1;
-                                 }
-                             });
-        }
-        __syncthreads();
-        if (threadIdx.x < R) {                                           // loss, d(logits)
-            const int r = threadIdx.x;
-            const float* s = lg + r * ld;
-            float* d = G0 + r * ld;
-            float* dg = T[Lt - 1].D + (long long)(r0 + r) * T[Lt - 1].ldd;
-            if (r < nr) {
-                const int y = a.y[r0 + r];
-                float li;
-                if (a.loss == VFL_LOSS_BCE) {
-                    const float x = s[0];
-                    li = fmaxf(x, 0.f) - x * (float)y + log1pf(expf(-fabsf(x)));
-                    d[0] = (1.0f / (1.0f + expf(-x)) - (float)y) * inv_b;
-                } else {
-                    float m = s[0];
-                    for (int j = 1; j < nout; ++j) m = fmaxf(m, s[j]);
-                    float z = 0.f;
-                    for (int j = 0; j < nout; ++j) z += expf(s[j] - m);
-                    li = logf(z) + m - s[y];
-                    const float iz = 1.0f / z;
-                    for (int j = 0; j < nout; ++j) d[j] = (expf(s[j] - m) * iz - (j == y ? 1.f : 0.f)) * inv_b;
-                }
-                a.rowloss[r0 + r] = li;
-                for (int j = 0; j < nout; ++j) dg[j] = d[j];
+            if (fuse_out && l == Lt - 2) {
+                const FusedLayerArgs& Lh = T[l];
+                const FusedLayerArgs& Lo = T[Lt - 1];
+                const TopLast tl{Lh.in, Lh.out, Lh.fmap, Lh.ws_off, Lh.ws_ld, Lo.out, Lo.ws_off, Lo.ws_ld,
+                                 Lh.Y, Lh.ldy, Lh.D, Lh.ldd, Lo.Y, Lo.ldy, Lo.D, Lo.ldd};
+                top_last_fused(l == 0 ? C : TH(l - 1), ld, ws, tl, TH(l), G0, a.y + r0, a.loss, inv_b, a.rowloss + r0,
+                               r0, nr, red);
             } else {
-                for (int j = 0; j < nout; ++j) d[j] = 0.f;
+                tile_fwd(l == 0 ? C : TH(l - 1), ld, T[l].in, ws + T[l].ws_off, T[l].ws_ld, staged_bias(ws, T[l]),
+                         T[l].out, T[l].fmap, TH(l), T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
             }
-            for (int j = nout; j < ceil8(nout); ++j) d[j] = 0.f;
         }
-        // backward through g: the input-gradient chain
+        if (!fuse_out) {
+            float* lg = X;                                               // x_a's tile is free again
+            {                                                            // logits: no activation
+                const FusedLayerArgs& L = T[Lt - 1];
+                if (first)
+                    cp_wait_pending(0);
+                else
+                    __syncthreads();
+                const float* bias = staged_bias(ws, L);
+                float* yg = L.Y + (long long)r0 * L.ldy;
+                const long long ldy = L.ldy;
+                tile_gemm<false>(Lt == 1 ? C : TH(Lt - 2), ld, ceil8(L.in) / 8, ws + L.ws_off, L.ws_ld, ceil8(nout) / 8,
+                                 L.fmap, red, [&](int r, int c, float v0, float v1) {
+                                     v0 += bias[c];
+                                     v1 += bias[c + 1];
+                                     *reinterpret_cast<float2*>(lg + r * ld + c) = make_float2(v0, v1);
+                                     if (r < nr) {
+                                         if (c < nout) yg[(long long)r * ldy + c] = v0;
+                                         if (c + 1 < nout) yg[(long long)r * ldy + c + 1] = v1;
+                                     }
+                                 });
+            }
+            __syncthreads();
+            if (threadIdx.x < R) {                                       // loss, d(logits)
+                const int r = threadIdx.x;
+                const float* sr = lg + r * ld;
+                float* d = G0 + r * ld;
+                float* dg = T[Lt - 1].D + (long long)(r0 + r) * T[Lt - 1].ldd;
+                if (r < nr) {
+                    a.rowloss[r0 + r] = loss_row(sr, nout, a.y[r0 + r], a.loss, inv_b, d);
+                    for (int j = 0; j < nout; ++j) dg[j] = d[j];
+                } else {
+                    for (int j = 0; j < nout; ++j) d[j] = 0.f;
+                }
+                for (int j = nout; j < ceil8(nout); ++j) d[j] = 0.f;
+            }
+        }
+        // backward through g: the input-gradient chain (from the last hidden layer when it was fused)
         float* gin = G0;
         float* gout = G1;
-        for (int l = Lt - 1; l >= 1; --l) {
+        for (int l = fuse_out ? Lt - 2 : Lt - 1; l >= 1; --l) {
             __syncthreads();
             tile_dx(gin, ld, T[l].out, ws + T[l].ws_off, T[l].ws_ld, T[l].in, T[l].dmap, TH(l - 1), gout,
                     T[l - 1].D + (long long)r0 * T[l - 1].ldd, T[l - 1].ldd, nr, red);
@@ -509,11 +626,13 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         first = false;
     }
     if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
+    if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
     publish_when_last(a.counter, a.pub_hdr, a.k, a.batch, a.version);
 }
 
 __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
+    const long long hdr_k = threadIdx.x == 0 ? a.chk_hdr->k : 0;   // gradient channel's header, checked at the end
     const int Lp = a.na;
     const int ld = a.act_ld;
     float* ws = smem;
@@ -524,7 +643,6 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
     float* G0 = slot(Lp + 1);
     float* G1 = slot(Lp + 2);
     float* red = slot(Lp + 3);
-    if (threadIdx.x == 0 && a.chk_hdr->k != a.k) atomicOr(a.status, ST_VERSION);
     const FusedLayerArgs* P = a.L;
     const int ep8 = ceil8(P[Lp - 1].out);
     const int ntiles = (a.rows + R - 1) / R;
@@ -573,6 +691,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
         first = false;
     }
     if (first) cp_wait_pending(0);
+    if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
 }
 
 // dW = D^T X, db = sum of D's rows, then SGD, for one 32 x 32 output tile per
@@ -582,7 +701,6 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
 // fixed order.
 constexpr int kUpdRows = 128;                // rows staged per pass
 constexpr int kUpdLd = kUpdTile + 4;         // smem row stride
-constexpr int kUpdLoads = kUpdRows * kUpdTile / kUpdThreads;
 static_assert(kUpdThreads == 256 && kUpdTile == 32, "the thread map below assumes 256 threads and 32 x 32 tiles");
 static_assert(kUpdRows * kUpdLd >= 4 * kUpdTile * kUpdTile, "the group partials reuse the D stage");
 
@@ -595,6 +713,23 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int tile = blockIdx.x / kUpdCluster;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (tile == a.ntiles) {                                  // one extra cluster: mean loss of the step, fixed order
+        if (rank == 0 && a.loss_out) {
+            float s = 0.f;
+            for (int r = tid; r < a.rows; r += kUpdThreads) s += a.rowloss[r];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
+            if (lane == 0) Pb[warp] = s;
+            __syncthreads();
+            if (tid == 0) {
+                float v = 0.f;
+                for (int w = 0; w < kUpdThreads / 32; ++w) v += Pb[w];
+                *a.loss_out = v / (float)a.rows;
+            }
+        }
+        return;
+    }
     int l = 0;
     while (l + 1 < a.nl && tile >= a.L[l + 1].tile0) ++l;
     const FusedUpdLayer& L = a.L[l];
@@ -605,7 +740,6 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     const int chunk = (a.rows + kUpdCluster - 1) / kUpdCluster;
     const int rbeg = min(a.rows, rank * chunk), rend = min(a.rows, rbeg + chunk);
 
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int grp = warp >> 1;                               // row group
     const int ob = (((warp & 1) << 2) + (lane >> 3)) * 4;    // first of 4 outputs
     const int ib = (lane & 7) * 4;                           // first of 4 inputs
@@ -615,27 +749,31 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
 #pragma unroll
         for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
     float bacc = 0.f;                                        // db partial of output tid & 31
+    const bool dvec = (L.ldd & 3) == 0;                      // D rows hold whole 16-byte chunks
     for (int rb = rbeg; rb < rend; rb += kUpdRows) {
         const int nr = min(kUpdRows, rend - rb);
-        float dv[kUpdLoads], xv[kUpdLoads];
-#pragma unroll
-        for (int j = 0; j < kUpdLoads; ++j) {                // every load in flight before any store
-            const int e = tid + j * kUpdThreads, r = e >> 5, c = e & 31;
+        __syncthreads();
+        // rows [rb, rb + nr) of D[:, o0 : o0+32] and X[:, i0 : i0+32] in 16-byte chunks (cp.async), zero
+        // past the layer's columns; X's columns come from X or, from xsplit on (a multiple of 4), from X2
+        for (int e = tid; e < kUpdRows * (kUpdTile / 4); e += kUpdThreads) {
+            const int r = e >> 3, c = (e & 7) * 4;
+            float* ds = Ds + r * kUpdLd + c;
+            float* xs = Xs + r * kUpdLd + c;
             const long long gr = rb + r;
-            dv[j] = (r < nr && c < no) ? __ldg(L.D + gr * L.ldd + o0 + c) : 0.f;
-            const int ic = i0 + c;
-            xv[j] = 0.f;
-            if (r < nr && c < ni)
-                xv[j] = ic < L.xsplit ? __ldg(L.X + gr * L.ldx + ic) : __ldg(L.X2 + gr * L.ldx2 + (ic - L.xsplit));
-        }
-        __syncthreads();
+            if (r < nr && o0 + c < L.out && dvec) {
+                cp16(ds, L.D + gr * L.ldd + o0 + c);
+            } else {
 #pragma unroll
-        for (int j = 0; j < kUpdLoads; ++j) {
-            const int e = tid + j * kUpdThreads, r = e >> 5, c = e & 31;
-            Ds[r * kUpdLd + c] = dv[j];
-            Xs[r * kUpdLd + c] = xv[j];
+                for (int q = 0; q < 4; ++q) ds[q] = (r < nr && o0 + c + q < L.out) ? __ldg(L.D + gr * L.ldd + o0 + c + q) : 0.f;
+            }
+            const int ic = i0 + c;
+            if (r < nr && ic < L.in)
+                cp16(xs, ic < L.xsplit ? L.X + gr * L.ldx + ic : L.X2 + gr * L.ldx2 + (ic - L.xsplit));
+            else
+                *reinterpret_cast<float4*>(xs) = make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        __syncthreads();
+        cp_commit();
+        cp_wait_pending(0);
         for (int r = grp; r < nr; r += 4) {
             const float4 d = *reinterpret_cast<const float4*>(Ds + r * kUpdLd + ob);
             const float4 x = *reinterpret_cast<const float4*>(Xs + r * kUpdLd + ib);
@@ -694,24 +832,15 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
         }
     }
     cluster.sync();                                          // peers' shared memory stays valid until here
-    if (blockIdx.x == 0 && a.loss_out) {                     // mean loss of the step, fixed order
-        float s = 0.f;
-        for (int r = tid; r < a.rows; r += kUpdThreads) s += a.rowloss[r];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
-        if (lane == 0) Pb[warp] = s;
-        __syncthreads();
-        if (tid == 0) {
-            float v = 0.f;
-            for (int w = 0; w < kUpdThreads / 32; ++w) v += Pb[w];
-            *a.loss_out = v / (float)a.rows;
-        }
-    }
 }
 
 template <typename K>
 cudaError_t set_smem_attr(K kernel) {
-    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedMaxSmem);
+    // every fused kernel asks for the largest shared-memory carveout, so an SM
+    // moving from one of them to the next keeps its L1 / shared split
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedMaxSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    return e;
 }
 
 }  // namespace
@@ -741,8 +870,11 @@ cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s) {
+    static cudaError_t attr = cudaFuncSetAttribute(fused_update_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (attr != cudaSuccess) return attr;
     if (a.ntiles < 1 || a.rows < 1) return cudaErrorInvalidValue;
-    fused_update_kernel<<<a.ntiles * kUpdCluster, kUpdThreads, 0, s>>>(a);
+    // one more cluster than output tiles when the step's mean loss is wanted
+    fused_update_kernel<<<(a.ntiles + (a.loss_out ? 1 : 0)) * kUpdCluster, kUpdThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -9,6 +9,7 @@ constexpr int kFusedThreads = 512;
 constexpr int kFusedRows = 16;                 // rows per row tile
 constexpr int kFusedMaxWidth = 256;            // widest layer input or output
 constexpr int kFusedMaxLayers = 16;
+constexpr int kFusedMaxOut = 16;               // n_out up to which the output layer is folded into an epilogue
 constexpr size_t kFusedMaxSmem = 227 * 1024;
 
 // shared-memory row stride >= width, = 4 mod 32 (the MMA A fragments and the
