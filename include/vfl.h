@@ -257,7 +257,11 @@ int64_t vfl_kernel_launches(const vfl_ctx* ctx);
  * synchronizes and folds the records into per-class totals.  vfl_profile_get
  * then returns, for kernel class `cls` (0 .. VFL_KERNEL_CLASSES-1, named by
  * vfl_kernel_class_name), the number of launches, their summed duration in ms
- * and their summed algorithmic flops and bytes.
+ * and their summed algorithmic flops and bytes.  Launches captured into a
+ * graph (vfl_graph_capture) while timing is on carry their event pairs into
+ * the graph: launch it once, then call vfl_profile(ctx, 0); folding before the
+ * graph has run returns VFL_E_STATE.  Such a graph should not be replayed
+ * after the fold (its events go back to the context's pool).
  */
 #define VFL_KERNEL_CLASSES 17
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);

@@ -245,13 +245,15 @@ bool prof_begin(vfl_ctx* ctx, ProfRec* r, int cls, double flops, double bytes, c
     r->e0 = spare_event(ctx);
     r->e1 = spare_event(ctx);
     if (!r->e0 || !r->e1) return false;
-    cudaEventRecord(r->e0, s);
+    // external: under stream capture the record becomes a graph node that records the event when
+    // the graph runs (a plain record would only order the capture's streams)
+    cudaEventRecordWithFlags(r->e0, s, cudaEventRecordExternal);
     return true;
 }
 
 void prof_end(vfl_ctx* ctx, ProfRec* r, bool on, cudaStream_t s) {
     if (!on) return;
-    cudaEventRecord(r->e1, s);
+    cudaEventRecordWithFlags(r->e1, s, cudaEventRecordExternal);
     ctx->prof.push_back(*r);
 }
 
@@ -1511,7 +1513,6 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     if (!ctx || !out) return VFL_E_INVAL;
     *out = nullptr;
     if (ctx->broken) return VFL_E_CUDA;
-    if (ctx->prof_on) return ctx->fail(VFL_E_STATE, "vfl_graph_capture while per-launch timing is on");
     for (int w = 0; w < ctx->W; ++w)
         if (!ctx->ps[w] || !ctx->as[w])
             return ctx->fail(VFL_E_STATE, "graph capture needs the caller's streams (vfl_set_streams)");
@@ -1711,7 +1712,14 @@ vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable) {
     TRY(sync_all(ctx));
     for (ProfRec& r : ctx->prof) {
         float ms = 0.f;
-        CK(cudaEventElapsedTime(&ms, r.e0, r.e1));
+        const cudaError_t e = cudaEventElapsedTime(&ms, r.e0, r.e1);
+        if (e != cudaSuccess) {
+            // launches captured into a graph that has not run yet: nothing to fold
+            cudaGetLastError();
+            ctx->prof.clear();
+            return ctx->fail(VFL_E_STATE, "timed launches have not run (a captured graph not launched?): %s",
+                             cudaGetErrorString(e));
+        }
         ProfAgg& a = ctx->agg[r.cls];
         a.n += 1;
         a.ms += ms;
