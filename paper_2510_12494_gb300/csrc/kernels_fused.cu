@@ -699,15 +699,17 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
 // c = ceil(rows / 8).  Inside a CTA, 4 row groups x (8 x 8 threads of 4 x 4
 // outputs) accumulate in fp32; the groups, then the 8 ranks, are summed in a
 // fixed order.
-constexpr int kUpdRows = 128;                // rows staged per pass
-constexpr int kUpdLd = kUpdTile + 4;         // smem row stride
+constexpr int kUpdRows = 128;                // rows staged per pass: 32 per row group of 2 warps
+constexpr int kUpdLd = kUpdTile + 8;         // smem row stride, 8 mod 32: the MMA fragment loads are conflict-free
 static_assert(kUpdThreads == 256 && kUpdTile == 32, "the thread map below assumes 256 threads and 32 x 32 tiles");
-static_assert(kUpdRows * kUpdLd >= 4 * kUpdTile * kUpdTile, "the group partials reuse the D stage");
+static_assert(kUpdThreads == 256 && kUpdRows == 128, "4 row groups x 2 warps, 32 rows per group");
+static_assert(2 * kUpdRows * kUpdLd >= 4 * kUpdTile * kUpdTile, "the row-group partials reuse the stage");
 
 __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThreads)
     fused_update_kernel(const FusedUpdArgs a) {
-    __shared__ __align__(16) float Ds[kUpdRows * kUpdLd];
-    __shared__ __align__(16) float Xs[kUpdRows * kUpdLd];
+    __shared__ __align__(16) float stage[2 * kUpdRows * kUpdLd];
+    float* Ds = stage;
+    float* Xs = stage + kUpdRows * kUpdLd;
     __shared__ __align__(16) float Pw[kUpdTile * kUpdTile];   // this CTA's partial dW tile
     __shared__ float Pb[kUpdTile];                            // and partial db
     cg::cluster_group cluster = cg::this_cluster();
@@ -740,14 +742,15 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     const int chunk = (a.rows + kUpdCluster - 1) / kUpdCluster;
     const int rbeg = min(a.rows, rank * chunk), rend = min(a.rows, rbeg + chunk);
 
-    const int grp = warp >> 1;                               // row group
-    const int ob = (((warp & 1) << 2) + (lane >> 3)) * 4;    // first of 4 outputs
-    const int ib = (lane & 7) * 4;                           // first of 4 inputs
+    const int fg = lane >> 2, ft = lane & 3;     // MMA fragment row / column lane
+    // the 32 x 32 tile as 2 (outputs) x 4 (inputs) MMA blocks in 3xTF32, A[o][r] = D[r][o],
+    // B[r][i] = X[r][i]: warp w takes output half mt = w mod 2 and the 32 rows of row group w / 2
+    const int mt = warp & 1, rgrp = warp >> 1;
     float acc[4][4];
 #pragma unroll
-    for (int p = 0; p < 4; ++p)
+    for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+        for (int q = 0; q < 4; ++q) acc[nt][q] = 0.f;
     float bacc = 0.f;                                        // db partial of output tid & 31
     const bool dvec = (L.ldd & 3) == 0;                      // D rows hold whole 16-byte chunks
     for (int rb = rbeg; rb < rend; rb += kUpdRows) {
@@ -774,26 +777,42 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
         }
         cp_commit();
         cp_wait_pending(0);
-        for (int r = grp; r < nr; r += 4) {
-            const float4 d = *reinterpret_cast<const float4*>(Ds + r * kUpdLd + ob);
-            const float4 x = *reinterpret_cast<const float4*>(Xs + r * kUpdLd + ib);
-            const float dd[4] = {d.x, d.y, d.z, d.w}, xx[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-            for (int p = 0; p < 4; ++p)
+        for (int kk = 0; kk < 4; ++kk) {
+            const int k0 = rgrp * 32 + kk * 8;               // rows past nr are zero-filled
+            uint32_t ah[4], al[4], bh[4][2], bl[4][2];
+            const float* d0 = Ds + (k0 + ft) * kUpdLd + mt * 16 + fg;
+            const float* d1 = d0 + 4 * kUpdLd;
+            split_tf32(d0[0], ah[0], al[0]);
+            split_tf32(d0[8], ah[1], al[1]);
+            split_tf32(d1[0], ah[2], al[2]);
+            split_tf32(d1[8], ah[3], al[3]);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(dd[p], xx[q], acc[p][q]);
+            for (int nt = 0; nt < 4; ++nt) {
+                const float* x0 = Xs + (k0 + ft) * kUpdLd + nt * 8 + fg;
+                split_tf32(x0[0], bh[nt][0], bl[nt][0]);
+                split_tf32(x0[4 * kUpdLd], bh[nt][1], bl[nt][1]);
+            }
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) mma_tf32(acc[nt], al, bh[nt]);
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) mma_tf32(acc[nt], ah, bl[nt]);
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) mma_tf32(acc[nt], ah, bh[nt]);
         }
         if (bias)
             for (int r = tid >> 5; r < nr; r += kUpdThreads / 32) bacc += Ds[r * kUpdLd + (tid & 31)];
     }
-    __syncthreads();
-    float* gpart = Ds;                                       // [4 groups][32][32]
-    float* bpart = Xs;                                       // [8 warps][32]
-#pragma unroll
-    for (int p = 0; p < 4; ++p)
-        *reinterpret_cast<float4*>(gpart + grp * kUpdTile * kUpdTile + (ob + p) * kUpdTile + ib) =
-            make_float4(acc[p][0], acc[p][1], acc[p][2], acc[p][3]);
+    __shared__ float bpart[kUpdThreads];                     // db partials [8 warps][32]
     bpart[tid] = bacc;
+    __syncthreads();
+    float* gpart = stage;                                    // [4 row groups][32][32]
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+        float* pw = gpart + rgrp * kUpdTile * kUpdTile + (mt * 16 + fg) * kUpdTile + nt * 8 + 2 * ft;
+        *reinterpret_cast<float2*>(pw) = make_float2(acc[nt][0], acc[nt][1]);
+        *reinterpret_cast<float2*>(pw + 8 * kUpdTile) = make_float2(acc[nt][2], acc[nt][3]);
+    }
     __syncthreads();
     for (int e = tid; e < kUpdTile * kUpdTile; e += kUpdThreads)
         Pw[e] = ((gpart[e] + gpart[1024 + e]) + gpart[2048 + e]) + gpart[3072 + e];
