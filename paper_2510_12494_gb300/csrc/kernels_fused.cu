@@ -34,6 +34,15 @@ namespace vfl {
 namespace {
 
 constexpr int NT = kFusedThreads;     // 16 warps
+
+// Programmatic dependent launch.  Inside a graph whose edge into this kernel is
+// programmatic, the kernel may start while its producer still runs:
+// griddep_wait() returns once the producer grid has completed and its writes
+// are visible, so every read of the producer's output comes after it.
+// griddep_trigger() lets this kernel's own programmatic dependents launch.
+// Without such edges both are no-ops.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 constexpr int NW = NT / 32;
 constexpr int R = kFusedRows;
 static_assert(R == 16, "the MMA tiles cover exactly 16 rows");
@@ -284,6 +293,7 @@ __device__ __forceinline__ void tile_dx(const float* dY, int ld, int K, const fl
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedChainArgs a) {
     extern __shared__ __align__(16) float smem[];
+    griddep_trigger();   // the active step may start staging its weights and rows now
     const int ld = a.act_ld;
     float* ws = smem;
     float* t0 = smem + a.w_floats;                      // x_p rows, then ping-pong
@@ -465,8 +475,7 @@ __device__ __noinline__ void top_last_fused(const float* X, int ld, const float*
 
 __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
-    // the embedding channel's header, checked at the end (a load that nothing waits for until then)
-    const long long hdr_k = threadIdx.x == 0 ? a.chk_hdr->k : 0;
+    long long hdr_k = a.k;   // the embedding channel's header, read once the publisher has finished
     const int La = a.na, Lt = a.nt;
     const int ld = a.act_ld;
     float* ws = smem;
@@ -496,29 +505,25 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         const int nr = min(R, a.rows - r0);
         __syncthreads();
         async_rows(X, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
-        async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
         if (first) {
-            // one commit group per layer, in the order the forward uses them (group 0 also the rows)
+            // one commit group per layer, in the order the forward uses them (group 0 also x^a's rows);
+            // only then wait for the publisher, and z^p's rows come last
             for (int l = 0; l < Ltot; ++l) {
                 stage_layer_weights(ws, a.L[l]);
                 cp_commit();
             }
-        } else {
-            cp_commit();
+            griddep_wait();
+            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
         }
+        async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
+        cp_commit();
         for (int l = 0; l < La; ++l) {                                   // z^a = f_a(x^a)
             if (first)
-                cp_wait_pending(Ltot - 1 - l);
+                cp_wait_pending(Ltot - l);   // x^a's rows and layers 0..l; later layers and z^p may be in flight
             else if (l == 0)
-                cp_wait_pending(0);
+                cp_wait_pending(0);          // this tile's x^a and z^p rows
             else
                 __syncthreads();
-            if (l == 0) {
-                const int r = threadIdx.x >> 5;                          // z^p kept for the update
-                if (r < nr)
-                    for (int c = threadIdx.x & 31; c < ep; c += 32)
-                        a.zpc[(long long)(r0 + r) * a.ldzpc + c] = C[r * ld + ea + c];
-            }
             tile_fwd(l == 0 ? X : H(l - 1), ld, A[l].in, ws + A[l].ws_off, A[l].ws_ld, staged_bias(ws, A[l]), A[l].out,
                      A[l].fmap, l == La - 1 ? C : H(l), A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
         }
@@ -526,10 +531,15 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         // gradient ride in the epilogue of g's last hidden layer (one warp per row)
         const bool fuse_out = Lt >= 2 && nout <= kFusedMaxOut;
         for (int l = 0; l < Lt - 1; ++l) {                               // g's hidden layers on [z^a | z^p]
-            if (first)
-                cp_wait_pending(fuse_out && l == Lt - 2 ? 0 : Lt - 1 - l);
-            else
+            if (l == 0) {
+                cp_wait_pending(0);                                      // z^p's rows (and every weight)
+                const int r = threadIdx.x >> 5;                          // z^p kept for the update
+                if (r < nr)
+                    for (int c = threadIdx.x & 31; c < ep; c += 32)
+                        a.zpc[(long long)(r0 + r) * a.ldzpc + c] = C[r * ld + ea + c];
+            } else {
                 __syncthreads();
+            }
             if (fuse_out && l == Lt - 2) {
                 const FusedLayerArgs& Lh = T[l];
                 const FusedLayerArgs& Lo = T[Lt - 1];
@@ -546,10 +556,13 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
             float* lg = X;                                               // x_a's tile is free again
             {                                                            // logits: no activation
                 const FusedLayerArgs& L = T[Lt - 1];
-                if (first)
-                    cp_wait_pending(0);
-                else
-                    __syncthreads();
+                cp_wait_pending(0);
+                if (Lt == 1) {                                           // z^p kept for the update
+                    const int r = threadIdx.x >> 5;
+                    if (r < nr)
+                        for (int c = threadIdx.x & 31; c < ep; c += 32)
+                            a.zpc[(long long)(r0 + r) * a.ldzpc + c] = C[r * ld + ea + c];
+                }
                 const float* bias = staged_bias(ws, L);
                 float* yg = L.Y + (long long)r0 * L.ldy;
                 const long long ldy = L.ldy;
@@ -579,6 +592,7 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
                 for (int j = nout; j < ceil8(nout); ++j) d[j] = 0.f;
             }
         }
+        griddep_trigger();   // the passive backward and the update may launch and stage now
         // backward through g: the input-gradient chain (from the last hidden layer when it was fused)
         float* gin = G0;
         float* gout = G1;
@@ -625,14 +639,18 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         }
         first = false;
     }
-    if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
+    if (first) {                     // CTAs without a row tile have nothing in flight
+        griddep_wait();
+        cp_wait_pending(0);
+    }
     if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
     publish_when_last(a.counter, a.pub_hdr, a.k, a.batch, a.version);
 }
 
 __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedStepArgs a) {
     extern __shared__ __align__(16) float smem[];
-    const long long hdr_k = threadIdx.x == 0 ? a.chk_hdr->k : 0;   // gradient channel's header, checked at the end
+    griddep_trigger();       // the passive update may launch now (it waits for this grid before reading)
+    long long hdr_k = a.k;   // the gradient channel's header, read once the active step has finished
     const int Lp = a.na;
     const int ld = a.act_ld;
     float* ws = smem;
@@ -653,16 +671,20 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
         __syncthreads();
         for (int l = 0; l < Lp; ++l)
             async_rows(slot(l), ld, P[l].Y + (long long)r0 * P[l].ldy, P[l].ldy, (int)P[l].out_ld, nr);
-        async_rows(gs, ld, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
         cp_commit();
         if (first) {
-            // weights in the order the backward uses them: layer Lp-1 first
+            // weights in the order the backward uses them (layer Lp-1 first), then wait for the active
+            // step, whose dz^p comes last
             for (int l = Lp - 1; l >= 1; --l) {
                 stage_layer_weights(ws, P[l]);
                 cp_commit();
             }
+            griddep_wait();
+            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
         }
-        cp_wait_pending(first ? Lp - 1 : 0);
+        async_rows(gs, ld, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
+        cp_commit();
+        cp_wait_pending(0);
         {                                                                // dz^p * [z^p > 0]
             const int r = threadIdx.x >> 5;
             const float* zp = slot(Lp - 1);
@@ -678,10 +700,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
         float* gin = G0;
         float* gout = G1;
         for (int l = Lp - 1; l >= 1; --l) {
-            if (first)
-                cp_wait_pending(l - 1);   // this layer's weights
-            else
-                __syncthreads();
+            __syncthreads();
             tile_dx(gin, ld, P[l].out, ws + P[l].ws_off, P[l].ws_ld, P[l].in, P[l].dmap, slot(l - 1), gout,
                     P[l - 1].D + (long long)r0 * P[l - 1].ldd, P[l - 1].ldd, nr, red);
             float* t = gin;
@@ -690,7 +709,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
         }
         first = false;
     }
-    if (first) cp_wait_pending(0);
+    if (first) griddep_wait();
     if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
 }
 
@@ -712,6 +731,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     float* Xs = stage + kUpdRows * kUpdLd;
     __shared__ __align__(16) float Pw[kUpdTile * kUpdTile];   // this CTA's partial dW tile
     __shared__ float Pb[kUpdTile];                            // and partial db
+    griddep_wait();   // the d(pre-activation) rows, z^p's copy and the row losses come from the row kernel
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int tile = blockIdx.x / kUpdCluster;

@@ -13,6 +13,8 @@
 //    Each party keeps its S+1 most recent weight versions in a ring.
 #include <algorithm>
 #include <cstdarg>
+#include <map>
+#include <utility>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -151,6 +153,11 @@ struct vfl_ctx {
     // it), so waits on the events that produced those versions are skipped -- those events may have
     // been recorded inside a graph capture, where they cannot be waited on from outside
     long long ordered_floor = -1;
+
+    // graph capture of the fused path: the kernel node of each (phase, step), so that the edges a
+    // consumer only needs at a later point of its run become programmatic (see vfl_graph_capture)
+    bool capturing = false;
+    std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
         char buf[512];
@@ -661,6 +668,23 @@ vfl_status wait_ev(vfl_ctx* ctx, cudaStream_t s, cudaEvent_t e) {
         if (st_ != VFL_OK) return st_;  \
     } while (0)
 
+// Fused-path phases whose kernel nodes a capture records.
+enum CapPhase : int { CAP_PFWD, CAP_ACTIVE, CAP_AUPD, CAP_PBWD, CAP_PUPD };
+
+// Under stream capture (and without per-launch timing, whose event nodes would sit in between),
+// remember the kernel node just captured on stream s as phase `ph` of step k.
+void note_node(vfl_ctx* ctx, int ph, long long k, cudaStream_t s) {
+    if (!ctx->capturing || ctx->prof_on) return;
+    cudaStreamCaptureStatus st;
+    const cudaGraphNode_t* deps = nullptr;
+    size_t n = 0;
+    if (cudaStreamGetCaptureInfo(s, &st, nullptr, nullptr, &deps, nullptr, &n) == cudaSuccess &&
+        st == cudaStreamCaptureStatusActive && n == 1)
+        ctx->cap_nodes[{ph, k}] = deps[0];
+    else
+        cudaGetLastError();
+}
+
 // ---- fused path -------------------------------------------------------------
 FusedLayerArgs fused_layer(const Layer& L, int vslot, void* Y, long long ldy, void* D, long long ldd) {
     FusedLayerArgs f;
@@ -913,6 +937,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
     if (ctx->fused) {
         TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), (int)(k % ctx->W), s));
+        note_node(ctx, CAP_PFWD, k, s);
         CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
         ctx->fwd_version[slot] = (int)v;
         ctx->slot_step_p[slot] = k;
@@ -960,10 +985,12 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
         TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), w, s));
+        note_node(ctx, CAP_ACTIVE, k, s);
         CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
         // SGD on theta_1 in step order: version k+1 from version k
         if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
         TRY(fused_active_update(ctx, k, rows, static_cast<const float*>(Xa0), w, s));
+        note_node(ctx, CAP_AUPD, k, s);
         CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
         ctx->grad_step[slot] = k;
         ctx->last_act_step[w] = k;
@@ -1066,9 +1093,11 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     if (ctx->fused) {
         const float* Xp = reinterpret_cast<const float*>(static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz);
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
+        note_node(ctx, CAP_PBWD, k, s);
         // SGD on theta_2 in step order
         if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
         TRY(fused_passive_update(ctx, k, slot, rows, Xp, w, s));
+        note_node(ctx, CAP_PUPD, k, s);
         CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
         ctx->n_bwd = k + 1;
         return VFL_OK;
@@ -1508,6 +1537,46 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
     return VFL_OK;
 }
 
+namespace {
+
+// Replace the plain edge from -> to by a programmatic one: `to` may launch once every CTA of `from`
+// has signalled (griddepcontrol.launch_dependents) and runs its prologue, waiting in griddepcontrol.wait
+// for `from` to complete before it reads from's output.  Left plain when the edge is not a direct one.
+void make_programmatic(cudaGraph_t g, cudaGraphNode_t from, cudaGraphNode_t to) {
+    if (cudaGraphRemoveDependencies(g, &from, &to, nullptr, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    cudaGraphEdgeData ed;
+    std::memset(&ed, 0, sizeof ed);
+    ed.from_port = cudaGraphKernelNodePortProgrammatic;
+    ed.type = cudaGraphDependencyTypeProgrammatic;
+    if (cudaGraphAddDependencies(g, &from, &to, &ed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        cudaGraphAddDependencies(g, &from, &to, nullptr, 1);
+    }
+}
+
+// For each captured step: passive forward -> active step (the active step stages its weights and x^a
+// before reading z^p), active step -> passive backward (weights and saved activations before dz^p),
+// active step -> active update and passive backward -> passive update (launch latency hidden).
+void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n) {
+    auto node = [&](int ph, long long k) -> cudaGraphNode_t {
+        auto it = ctx->cap_nodes.find({ph, k});
+        return it == ctx->cap_nodes.end() ? nullptr : it->second;
+    };
+    for (long long k = k0; k < k0 + n; ++k) {
+        const std::pair<int, int> edges[4] = {
+            {CAP_PFWD, CAP_ACTIVE}, {CAP_ACTIVE, CAP_PBWD}, {CAP_ACTIVE, CAP_AUPD}, {CAP_PBWD, CAP_PUPD}};
+        for (const auto& ed : edges) {
+            cudaGraphNode_t from = node(ed.first, k), to = node(ed.second, k);
+            if (from && to) make_programmatic(g, from, to);
+        }
+    }
+}
+
+}  // namespace
+
 vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
                              vfl_graph** out) {
     if (!ctx || !out) return VFL_E_INVAL;
@@ -1541,7 +1610,10 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     }
     const long long floor_before = ctx->ordered_floor;
     ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k0);
+    ctx->cap_nodes.clear();
+    ctx->capturing = true;
     if (e == cudaSuccess) st = vfl_train_steps(ctx, k0, n_steps, tau_p, tau_a);
+    ctx->capturing = false;
     ctx->ordered_floor = floor_before;
     // join every stream back into the origin, even after a failure, so that capture can end
     int j = 0;
@@ -1555,9 +1627,14 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     }
     cudaError_t e2 = cudaStreamEndCapture(origin, &graph);
     if (e == cudaSuccess) e = e2;
+    if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, graph, k0, n_steps);
+    ctx->cap_nodes.clear();
     const HostState after = save_state(ctx);
     load_state(ctx, before);
     if (st == VFL_OK && e == cudaSuccess) e = cudaGraphInstantiate(&g->exec, graph, 0);
+    // upload now, so that the first replay does not pay for it
+    if (st == VFL_OK && e == cudaSuccess) e = cudaGraphUpload(g->exec, origin);
+    if (st == VFL_OK && e == cudaSuccess) e = cudaStreamSynchronize(origin);
     if (graph) cudaGraphDestroy(graph);
     if (st != VFL_OK || e != cudaSuccess) {
         vfl_graph_destroy(g);
