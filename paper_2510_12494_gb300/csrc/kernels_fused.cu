@@ -308,6 +308,8 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
         __syncthreads();
         async_rows(t0, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)a.L[0].in_ld, nr);
         if (first) {
+            // the weight version comes from an earlier update, which may still be finishing
+            griddep_wait();
             // group l holds layer l's weights (group 0 also the rows), so layer l
             // only waits for its own weights while the later ones are still arriving
             for (int l = 0; l < a.nl; ++l) {
@@ -333,7 +335,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
         }
         first = false;
     }
-    if (first) cp_wait_pending(0);   // CTAs without a row tile have nothing in flight
+    if (first) griddep_wait();       // CTAs without a row tile have nothing in flight
     // the last CTA to finish publishes the header after every payload write
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -507,25 +509,30 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         async_rows(X, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
         if (first) {
             // one commit group per layer, in the order the forward uses them (group 0 also x^a's rows);
-            // only then wait for the publisher, and z^p's rows come last
+            // z^p's rows follow once the publisher has finished, after f_a's forward
             for (int l = 0; l < Ltot; ++l) {
                 stage_layer_weights(ws, a.L[l]);
                 cp_commit();
             }
-            griddep_wait();
-            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
+        } else {
+            async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
+            cp_commit();
         }
-        async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
-        cp_commit();
         for (int l = 0; l < La; ++l) {                                   // z^a = f_a(x^a)
             if (first)
-                cp_wait_pending(Ltot - l);   // x^a's rows and layers 0..l; later layers and z^p may be in flight
+                cp_wait_pending(Ltot - 1 - l);   // x^a's rows and layers 0..l
             else if (l == 0)
-                cp_wait_pending(0);          // this tile's x^a and z^p rows
+                cp_wait_pending(0);              // this tile's x^a and z^p rows
             else
                 __syncthreads();
             tile_fwd(l == 0 ? X : H(l - 1), ld, A[l].in, ws + A[l].ws_off, A[l].ws_ld, staged_bias(ws, A[l]), A[l].out,
                      A[l].fmap, l == La - 1 ? C : H(l), A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
+        }
+        if (first) {
+            griddep_wait();                                              // the embedding's publisher has finished
+            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
+            async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);   // beside z^a's columns
+            cp_commit();
         }
         // with n_out <= kFusedMaxOut, g's output layer, the loss, d(logits) and the output layer's input
         // gradient ride in the epilogue of g's last hidden layer (one warp per row)

@@ -1558,9 +1558,11 @@ void make_programmatic(cudaGraph_t g, cudaGraphNode_t from, cudaGraphNode_t to) 
 }
 
 // For each captured step: passive forward -> active step (the active step stages its weights and x^a
-// before reading z^p), active step -> passive backward (weights and saved activations before dz^p),
-// active step -> active update and passive backward -> passive update (launch latency hidden).
-void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n) {
+// and runs f_a before reading z^p), active step -> passive backward (weights and saved activations
+// before dz^p), active step -> active update and passive backward -> passive update (launch latency
+// hidden), and the passive update that produced the version a passive forward reads -> that forward
+// (rows before the weights).
+void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, const int32_t* tau_p) {
     auto node = [&](int ph, long long k) -> cudaGraphNode_t {
         auto it = ctx->cap_nodes.find({ph, k});
         return it == ctx->cap_nodes.end() ? nullptr : it->second;
@@ -1572,6 +1574,9 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n) 
             cudaGraphNode_t from = node(ed.first, k), to = node(ed.second, k);
             if (from && to) make_programmatic(g, from, to);
         }
+        const long long v = k - tau_p[k];   // version of the forward: made by the update of step v - 1
+        cudaGraphNode_t from = node(CAP_PUPD, v - 1), to = node(CAP_PFWD, k);
+        if (from && to) make_programmatic(g, from, to);
     }
 }
 
@@ -1627,7 +1632,7 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     }
     cudaError_t e2 = cudaStreamEndCapture(origin, &graph);
     if (e == cudaSuccess) e = e2;
-    if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, graph, k0, n_steps);
+    if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, graph, k0, n_steps, tau_p);
     ctx->cap_nodes.clear();
     const HostState after = save_state(ctx);
     load_state(ctx, before);
