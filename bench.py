@@ -238,7 +238,7 @@ def roofline(prof, pk):
     name, (n, ms, flops, nbytes) = max(prof.items(), key=lambda kv: kv[1][1])
     sec = ms / 1e3
     tensor = name.startswith("gemm_tc")
-    tf32x3 = name.startswith("fused_") and name != "fused_update"   # fused_update runs on the FP32 lanes
+    tf32x3 = name.startswith("fused_")      # the fused kernels' contractions: 3xTF32 warp MMAs
     if tensor:
         peak = pk["bf16_tflops_sustained"]
         ach = flops / sec / 1e12
