@@ -263,7 +263,7 @@ int64_t vfl_kernel_launches(const vfl_ctx* ctx);
  * graph has run returns VFL_E_STATE.  Such a graph should not be replayed
  * after the fold (its events go back to the context's pool).
  */
-#define VFL_KERNEL_CLASSES 17
+#define VFL_KERNEL_CLASSES 18
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);
 vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
                            double* bytes);

@@ -23,7 +23,7 @@ FP32, BF16 = 0, 1
 SCHED_SYNC, SCHED_MAX, SCHED_SEEDED = 0, 1, 2
 TAP_EMB, TAP_GRAD, TAP_LOGITS, TAP_ZA, TAP_DZA = range(5)
 PASSIVE, ACTIVE, TOP = 0, 1, 2
-KERNEL_CLASSES = 17
+KERNEL_CLASSES = 18
 
 STATUS_NAMES = {0: "VFL_OK", 1: "VFL_E_INVAL", 2: "VFL_E_OOM", 3: "VFL_E_CUDA", 4: "VFL_E_STATE",
                 5: "VFL_E_VERSION", 6: "VFL_E_TIMEOUT"}

@@ -179,6 +179,162 @@ __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__
 }
 
 // ---------------------------------------------------------------------------
+// Output layer + loss for the bf16 path (see HeadArgs).  256 threads, kHeadRows rows per block:
+// phase 1 gives warp w the rows w, w+8, ...; lane l holds inputs [8l, 8l+8) of a row.  Phase 2
+// gives thread t the inputs [8 (t mod 32), +8) of outputs j = t/32, t/32 + 8.
+constexpr int HEAD_NT = 256;
+static_assert(kHeadMaxK == 32 * 8 && kHeadMaxOut <= 2 * (HEAD_NT / 32), "head thread map");
+
+__global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
+    __shared__ float Ws[kHeadMaxOut * kHeadMaxK];
+    __shared__ __align__(16) __nv_bfloat16 hs[kHeadRows * kHeadMaxK];
+    __shared__ float dss[kHeadRows * kHeadMaxOut];
+    __shared__ float wloss[HEAD_NT / 32];
+    __shared__ bool last;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int K = a.K, nout = a.nout;
+    const int r0 = blockIdx.x * kHeadRows, nr = min(kHeadRows, a.rows - r0);
+    const float inv_b = 1.0f / (float)a.rows;
+    const __nv_bfloat16* W = static_cast<const __nv_bfloat16*>(a.W);
+    for (int i = tid; i < nout * K; i += HEAD_NT) {
+        const int j = i / K, k = i - j * K;
+        Ws[j * kHeadMaxK + k] = __bfloat162float(W[(long long)j * a.ldw + k]);
+    }
+    __syncthreads();
+    const bool kin = lane * 8 < K;
+    float wl = 0.f;                                     // this warp's rows' loss, in row order
+    for (int r = warp; r < kHeadRows; r += HEAD_NT / 32) {
+        float hk[8];
+        uint4 raw = make_uint4(0u, 0u, 0u, 0u);
+        if (r < nr && kin)
+            raw = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.h) + (long long)(r0 + r) * a.ldh + lane * 8);
+        *reinterpret_cast<uint4*>(hs + r * kHeadMaxK + lane * 8) = raw;
+        const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) hk[e] = __bfloat162float(hb[e]);
+        float sv[kHeadMaxOut], dv[kHeadMaxOut];
+#pragma unroll
+        for (int j = 0; j < kHeadMaxOut; ++j) {
+            if (j < nout) {
+                float p = 0.f;
+                const float* w = Ws + j * kHeadMaxK + lane * 8;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) p = fmaf(hk[e], kin ? w[e] : 0.f, p);
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
+                sv[j] = p + a.b[j];
+            }
+        }
+        float li = 0.f;
+        if (r < nr) {
+            const int yl = a.y[r0 + r];
+            if (a.loss == VFL_LOSS_BCE) {
+                const float x = sv[0];
+                li = fmaxf(x, 0.f) - x * (float)yl + log1pf(expf(-fabsf(x)));
+                dv[0] = (1.0f / (1.0f + expf(-x)) - (float)yl) * inv_b;
+            } else {
+                float m = sv[0];
+#pragma unroll
+                for (int j = 1; j < kHeadMaxOut; ++j)
+                    if (j < nout) m = fmaxf(m, sv[j]);
+                float z = 0.f;
+#pragma unroll
+                for (int j = 0; j < kHeadMaxOut; ++j)
+                    if (j < nout) z += expf(sv[j] - m);
+                float sy = 0.f;
+#pragma unroll
+                for (int j = 0; j < kHeadMaxOut; ++j)
+                    if (j < nout && j == yl) sy = sv[j];
+                li = logf(z) + m - sy;
+                const float iz = 1.0f / z;
+#pragma unroll
+                for (int j = 0; j < kHeadMaxOut; ++j)
+                    if (j < nout) dv[j] = (expf(sv[j] - m) * iz - (j == yl ? 1.f : 0.f)) * inv_b;
+            }
+            wl += li;
+            if (lane < nout) {
+                float sl = 0.f, dl = 0.f;
+#pragma unroll
+                for (int j = 0; j < kHeadMaxOut; ++j)
+                    if (j == lane) { sl = sv[j]; dl = dv[j]; }
+                a.logits[(long long)(r0 + r) * nout + lane] = sl;
+                a.ds[(long long)(r0 + r) * nout + lane] = dl;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kHeadMaxOut; ++j) dv[j] = 0.f;
+        }
+        if (lane < nout) {
+            float dl = 0.f;
+#pragma unroll
+            for (int j = 0; j < kHeadMaxOut; ++j)
+                if (j == lane) dl = dv[j];
+            dss[r * kHeadMaxOut + lane] = dl;
+        }
+        if (r < nr && kin) {                            // hidden layer's d(pre-activation), bf16
+            __align__(16) __nv_bfloat16 ob[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                float g = 0.f;
+#pragma unroll
+                for (int j = 0; j < kHeadMaxOut; ++j)
+                    if (j < nout) g = fmaf(dv[j], Ws[j * kHeadMaxK + lane * 8 + e], g);
+                ob[e] = __float2bfloat16_rn(hk[e] > 0.f ? g : 0.f);
+            }
+            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.dh) + (long long)(r0 + r) * a.lddh + lane * 8) =
+                *reinterpret_cast<const uint4*>(ob);
+        }
+    }
+    if (lane == 0) wloss[warp] = wl;
+    __syncthreads();
+    // partial dW and db of this block, rows in order
+    {
+        const int kc = (tid & 31) * 8;
+        const int j0 = tid >> 5;
+        if (kc < K) {
+#pragma unroll
+            for (int jj = 0; jj < 2; ++jj) {
+                const int j = j0 + jj * (HEAD_NT / 32);
+                if (j >= nout) break;
+                float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                for (int r = 0; r < nr; ++r) {
+                    const float d = dss[r * kHeadMaxOut + j];
+                    const uint4 raw = *reinterpret_cast<const uint4*>(hs + r * kHeadMaxK + kc);
+                    const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[e] = fmaf(d, __bfloat162float(hb[e]), acc[e]);
+                }
+                float* pw = a.pW + blockIdx.x * a.pw_stride + (long long)j * K + kc;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) pw[e] = acc[e];
+            }
+        }
+        if (tid < nout) {
+            float sb = 0.f;
+            for (int r = 0; r < nr; ++r) sb += dss[r * kHeadMaxOut + tid];
+            a.pb[blockIdx.x * a.pb_stride + tid] = sb;
+        }
+    }
+    // the step's mean loss: block sums in block order, by the last block to finish
+    if (tid == 0) {
+        float v = 0.f;
+        for (int w = 0; w < HEAD_NT / 32; ++w) v += wloss[w];
+        a.blk_loss[blockIdx.x] = v;
+        __threadfence();
+        last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (last && tid == 0) {
+        __threadfence();
+        float v = 0.f;
+        for (int bb = 0; bb < (int)gridDim.x; ++bb) v += __ldcg(a.blk_loss + bb);
+        *a.loss_out = v * inv_b;
+        *a.counter = 0;
+        __threadfence();
+    }
+}
+
+// ---------------------------------------------------------------------------
 // DP: per-row clip of the per-sample gradient B*dz to norm C, plus sigma*C*N(0,1).
 // ---------------------------------------------------------------------------
 constexpr int DP_NT = 256;
@@ -388,6 +544,14 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask
 cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
                         float* loss_out, cudaStream_t s) {
     loss_kernel<<<1, LOSS_NT, 0, s>>>(logits, y, rows, n_out, loss_kind, ds, loss_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_head(const HeadArgs& a, cudaStream_t s) {
+    if (a.rows < 1 || a.nout < 1 || a.nout > kHeadMaxOut || a.K < 8 || a.K > kHeadMaxK || (a.K & 7) ||
+        a.nblk < head_blocks(a.rows))
+        return cudaErrorInvalidValue;
+    head_kernel<<<a.nblk, HEAD_NT, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -86,6 +86,34 @@ struct SgdArgs {
 };
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s);
 
+// Output layer of g (n_out <= kHeadMaxOut outputs over K <= kHeadMaxK bf16 inputs) with the loss
+// folded in, for the bf16 path: per row the logits s = h W^T + b (fp32), the row's loss and
+// ds = dloss/ds / B (Eq. 1 or softmax cross-entropy), and the hidden layer's d(pre-activation)
+// (ds W) * [h > 0] rounded to bf16; per block of kHeadRows rows the partial dW = ds^T h and
+// db = sum of ds (reduced by the SGD kernel in block order), and the step's mean loss from the
+// block sums in block order (the last block to finish).
+constexpr int kHeadMaxOut = 12;
+constexpr int kHeadMaxK = 256;
+constexpr int kHeadRows = 64;
+struct HeadArgs {
+    const void* h; long long ldh;     // g's last hidden activation rows [rows, ldh], bf16
+    const void* W; long long ldw;     // the output layer's version copy [n_out, ldw], bf16
+    const float* b;                   // its bias, fp32
+    int K, nout, rows, loss;
+    const int* y;
+    float* logits;                    // [rows, n_out]
+    float* ds;                        // [rows, n_out]
+    void* dh; long long lddh;         // hidden layer's d(pre-activation) [rows, lddh], bf16
+    float* pW; long long pw_stride;   // [blocks][n_out * K]
+    float* pb; long long pb_stride;   // [blocks][n_out]
+    int nblk;                         // blocks launched, >= head_blocks(rows); blocks past the rows write zero partials
+    float* blk_loss;                  // [blocks]
+    int* counter;                     // blocks finished (re-armed by the last)
+    float* loss_out;
+};
+inline int head_blocks(int rows) { return (rows + kHeadRows - 1) / kHeadRows; }
+cudaError_t launch_head(const HeadArgs& a, cudaStream_t s);
+
 cudaError_t launch_write_header(ChannelHeader* h, long long k, int batch, int version, cudaStream_t s);
 cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status, cudaStream_t s);
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,

@@ -40,12 +40,12 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_HEAD, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
-    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update"};
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update", "head_loss"};
 
 struct ProfRec {
     int cls;
@@ -129,6 +129,11 @@ struct vfl_ctx {
     float* f_rowloss[kMaxWorkers] = {};         // per worker: per-row loss [B]
     float* f_zpc[kMaxWorkers] = {};             // per worker: z^p rows consumed by the step [B, ld8(e_p)]
     int* f_counter = nullptr;                   // last-CTA counters: [0, 16) passive fwd, [16, 32) active, per worker
+
+    // bf16 path: g's output layer and the loss in one launch (narrow output over a narrow hidden layer)
+    bool head = false;
+    int* h_counter = nullptr;                   // per worker: blocks finished
+    float* h_blk_loss[kMaxWorkers] = {};        // per worker: per-block loss sums
 
     // streams / events
     cudaStream_t ps[kMaxWorkers] = {};
@@ -243,6 +248,24 @@ cudaEvent_t spare_event(vfl_ctx* ctx) {
 }
 
 // Opens a profiled launch: records the start event when profiling is on.
+// Under stream capture the record is made external, so that it becomes a graph node recording
+// the event when the graph runs (a plain record would only order the capture's streams); outside
+// a capture the flag is not accepted.  A failed record is cleared from the last-error state (it
+// must not fail the launch it brackets) and drops the timing record.
+bool prof_record(cudaEvent_t e, cudaStream_t s) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    const unsigned flags = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+    if (cudaEventRecordWithFlags(e, s, flags) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return true;
+}
+
 bool prof_begin(vfl_ctx* ctx, ProfRec* r, int cls, double flops, double bytes, cudaStream_t s) {
     ++ctx->launches;
     if (!ctx->prof_on) return false;
@@ -252,16 +275,12 @@ bool prof_begin(vfl_ctx* ctx, ProfRec* r, int cls, double flops, double bytes, c
     r->e0 = spare_event(ctx);
     r->e1 = spare_event(ctx);
     if (!r->e0 || !r->e1) return false;
-    // external: under stream capture the record becomes a graph node that records the event when
-    // the graph runs (a plain record would only order the capture's streams)
-    cudaEventRecordWithFlags(r->e0, s, cudaEventRecordExternal);
-    return true;
+    return prof_record(r->e0, s);
 }
 
 void prof_end(vfl_ctx* ctx, ProfRec* r, bool on, cudaStream_t s) {
     if (!on) return;
-    cudaEventRecordWithFlags(r->e1, s, cudaEventRecordExternal);
-    ctx->prof.push_back(*r);
+    if (prof_record(r->e1, s)) ctx->prof.push_back(*r);
 }
 
 }  // namespace
@@ -334,6 +353,14 @@ bool fused_eligible(const vfl_config& c) {
     // z^p lands in the top's input tile after z^a's 8-column blocks, by 16-byte copies
     if (c.active_out[c.n_active - 1] % 8 != 0 || c.passive_out[c.n_passive - 1] % 4 != 0) return false;
     return true;
+}
+
+// The bf16 path folds g's output layer and the loss into one kernel when g has a hidden layer
+// of at most kHeadMaxK (a multiple of 8) units and at most kHeadMaxOut outputs.
+bool head_eligible(const vfl_config& c) {
+    if (c.dtype != VFL_BF16 || c.n_top < 2) return false;
+    const int K = c.top_out[c.n_top - 2], n_out = c.top_out[c.n_top - 1];
+    return n_out <= kHeadMaxOut && K >= 8 && K <= kHeadMaxK && K % 8 == 0;
 }
 
 // Shared-memory layout of the weights one fused launch stages: layers
@@ -413,6 +440,13 @@ void build_layers(vfl_ctx* ctx) {
         const size_t sf = fused_smem_fwd((int)w_pf, ctx->f_act_ld);
         if (std::max(sa, std::max(sp, sf)) > kFusedMaxSmem) ctx->fused = false;
     }
+    if (ctx->head) {
+        // one dW / db partial per block of kHeadRows rows, summed by the SGD kernel in block order
+        Layer& H = ctx->T.back();
+        H.nsplit = H.nsplit_b = head_blocks(c.batch);
+        H.kchunk = kHeadRows;
+        H.colsum_bias = false;
+    }
 }
 
 // Lay out every device buffer; with base == nullptr only measures.
@@ -488,6 +522,11 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             ctx->f_zpc[w] = static_cast<float*>(cv.take(B * ld8(ctx->P.back().out) * 4ull));
         }
         ctx->f_counter = static_cast<int*>(cv.take(2 * kMaxWorkers * sizeof(int)));
+    }
+    if (ctx->head) {
+        ctx->h_counter = static_cast<int*>(cv.take(kMaxWorkers * sizeof(int)));
+        for (int w = 0; w < ctx->W; ++w)
+            ctx->h_blk_loss[w] = static_cast<float*>(cv.take(head_blocks(B) * 4ull));
     }
     return cv.off + 256;
 }
@@ -1011,8 +1050,9 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->emb_hdr + slot, k, ctx->status, s));
     const void* Za = ctx->act_a[w][La - 1];
     const void* Zp = ctx->act_p[slot][Lp - 1];
-    // top forward on [z^a | z^p]
-    for (int l = 0; l < Lt; ++l) {
+    // top forward on [z^a | z^p]; with the head kernel, g's output layer runs with the loss
+    const int Lf = ctx->head ? Lt - 1 : Lt;
+    for (int l = 0; l < Lf; ++l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
         void* Y = last ? (void*)ctx->logits[w] : ctx->act_t[w][l];
@@ -1023,12 +1063,37 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
             TRY(linear_fwd(ctx, L, vslot, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0, rows, Y, ldy,
                            !last, last, s));
     }
-    // loss and d(logits)
-    PLAUNCH(K_LOSS, 0, (double)rows * n_out * 8 + rows * 4.0, s,
-            launch_loss(ctx->logits[w], ctx->Y + r0, rows, n_out, c.loss, ctx->ds[w], ctx->losses + (k % kLossCap), s));
-    // top backward
+    if (ctx->head) {
+        // output layer, loss, d(logits), its dW / db partials and the hidden layer's d(pre-activation)
+        const Layer& H = ctx->T[Lt - 1];
+        HeadArgs h;
+        std::memset(&h, 0, sizeof h);
+        h.h = ctx->act_t[w][Lt - 2]; h.ldh = ld8(H.in);
+        h.W = H.cW[vslot]; h.ldw = H.in_ld;
+        h.b = H.cb[vslot];
+        h.K = H.in; h.nout = n_out; h.rows = rows; h.loss = c.loss;
+        h.y = ctx->Y + r0;
+        h.logits = ctx->logits[w]; h.ds = ctx->ds[w];
+        h.dh = ctx->dpre_t[w][Lt - 2]; h.lddh = ld8(H.in);
+        h.pW = H.pW[w]; h.pw_stride = (long long)n_out * H.in;
+        h.pb = H.pb[w]; h.pb_stride = n_out;
+        h.nblk = H.nsplit;
+        h.blk_loss = ctx->h_blk_loss[w];
+        h.counter = ctx->h_counter + w;
+        h.loss_out = ctx->losses + (k % kLossCap);
+        const double hf = 2.0 * rows * n_out * H.in * 3.0;
+        const double hb = (double)rows * H.in * ctx->esz * 2 + (double)n_out * H.in * ctx->esz +
+                          (double)rows * (n_out * 8.0 + 4.0) + 4.0 * H.nsplit * ((double)n_out * H.in + n_out);
+        PLAUNCH(K_HEAD, hf, hb, s, launch_head(h, s));
+    } else {
+        // loss and d(logits)
+        PLAUNCH(K_LOSS, 0, (double)rows * n_out * 8 + rows * 4.0, s,
+                launch_loss(ctx->logits[w], ctx->Y + r0, rows, n_out, c.loss, ctx->ds[w],
+                            ctx->losses + (k % kLossCap), s));
+    }
+    // top backward (the head kernel has done the output layer's part)
     const bool dp = c.dp_clip > 0.f;
-    for (int l = Lt - 1; l >= 0; --l) {
+    for (int l = Lf - 1; l >= 0; --l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
         const void* dpre = last ? (const void*)ctx->ds[w] : ctx->dpre_t[w][l];
@@ -1180,6 +1245,7 @@ vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* 
     tmp.bf16 = cfg->dtype == VFL_BF16;
     tmp.esz = tmp.bf16 ? 2 : 4;
     tmp.fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
+    tmp.head = head_eligible(*cfg) && !getenv("VFL_DISABLE_HEAD");
     build_layers(&tmp);
     *bytes = carve_all(&tmp, nullptr);
     return VFL_OK;
@@ -1210,6 +1276,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
     for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
     ctx->fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
+    ctx->head = head_eligible(*cfg) && !getenv("VFL_DISABLE_HEAD");
     build_layers(ctx);
     const unsigned long long need = carve_all(ctx, nullptr);
     if (workspace_bytes < need) {

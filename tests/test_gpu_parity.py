@@ -211,6 +211,32 @@ def test_step_parity_generic_kernels(vfl, cid, monkeypatch):
     assert not failures, f"preset {cid}: {failures[:3]}"
 
 
+@pytest.mark.parametrize("cid", [3, 5])
+def test_step_parity_generic_head(vfl, cid, monkeypatch):
+    """The bf16 presets fold g's output layer and the loss into one kernel by
+    default; the per-layer GEMMs and loss kernel it replaces must match the
+    oracle too."""
+    monkeypatch.setenv("VFL_DISABLE_HEAD", "1")
+    worst, failures = run_sequential(vfl, cid, CASES[cid], steps=4)
+    assert not failures, f"preset {cid}: {failures[:3]}"
+
+
+@pytest.mark.parametrize("cid", [3, 4, 5])
+def test_head_kernel_runs(vfl, cid):
+    """The bf16 presets' active step runs the folded output-layer kernel once
+    per step, and no separate loss kernel."""
+    import synth
+    q, xp, xa, y, params = setup(synth.preset(cid), CASES[cid])
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    tp, ta = schedule(q, 3)
+    ctx.profile(True)
+    ctx.train_steps(0, 3, tp, ta)
+    ctx.profile(False)
+    summ = ctx.profile_summary()
+    assert summ["head_loss"][0] == 3
+    assert summ.get("loss", (0,))[0] == 0
+
+
 @pytest.mark.parametrize("cid,workers", [(2, 0), (2, 3), (3, 0)])
 def test_graph_replay_equals_direct_enqueue(vfl, cid, workers):
     """A captured CUDA graph of a window of steps replays exactly what the
