@@ -260,6 +260,7 @@ class StepRecord:
     zp: np.ndarray = None        # published embedding  [B_k, e_p]
     za: np.ndarray = None        # active embedding     [B_k, e_a]
     logits: np.ndarray = None    # [B_k, n_out]
+    ds: np.ndarray = None        # d(mean loss)/d(logits) [B_k, n_out]
     dzp: np.ndarray = None       # published gradient   [B_k, e_p]
     dza: np.ndarray = None       # [B_k, e_a]
     grads: dict = None           # (party, layer) -> (dW, db)
@@ -368,6 +369,7 @@ class Oracle:
         rec = StepRecord(k, j, (r0, r1), tau_p, tau_a, vp, va, float(loss))
         if record:
             rec.zp, rec.za, rec.logits, rec.dzp, rec.dza = zp, ha[-1], logits, dzp_f, dza
+            rec.ds = ds
             rec.grads = {}
             for party, g in ((0, gP), (1, gA), (2, gT)):
                 for l, gl in enumerate(g):

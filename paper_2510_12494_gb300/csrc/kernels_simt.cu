@@ -50,7 +50,7 @@ __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
     const TA* A2 = static_cast<const TA*>(g.A2);
     const TB* B = static_cast<const TB*>(g.B);
     float acc[4][4] = {};
-    float bsum[4] = {};
+    double bsum[4] = {};        // db partials in fp64: their per-row terms largely cancel
     const bool want_bsum = g.mode == GEMM_DW && blockIdx.y == 0 && tx == 0 && g.Pb != nullptr;
 
     for (int k0 = kb; k0 < ke; k0 += BK) {
@@ -97,7 +97,7 @@ __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
     for (int i = 0; i < 4; ++i) {
         const int m = m0 + ty * 4 + i;
         if (m >= g.M) continue;
-        if (want_bsum) g.Pb[(long long)blockIdx.z * g.pb_stride + m] = bsum[i];
+        if (want_bsum) g.Pb[(long long)blockIdx.z * g.pb_stride + m] = (float)bsum[i];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int n = n0 + tx * 4 + j;
@@ -423,9 +423,9 @@ __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
             stf(L.cW, r * L.in_ld + c, a.c_bf16, w);
         } else {
             const long long j = idx - nw;
-            float gsum = 0.f;
+            double gsum = 0.0;      // the bias partials largely cancel: sum them in fp64
             for (int z = 0; z < L.nsplit_b; ++z) gsum += L.pb[z * L.pb_stride + j];
-            const float b = L.b[j] - a.lr * gsum;
+            const float b = L.b[j] - a.lr * (float)gsum;
             L.b[j] = b;
             L.cb[j] = b;
         }

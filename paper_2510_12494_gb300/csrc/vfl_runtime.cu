@@ -1434,10 +1434,10 @@ vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t wor
         for (int z = 0; z < L->nsplit; ++z) a += pw[z * nw + i];
         dW[i] = a;
     }
-    for (int i = 0; i < L->out; ++i) {
-        float a = 0.f;
+    for (int i = 0; i < L->out; ++i) {      // as the SGD kernel sums them: fp64, partials in order
+        double a = 0.0;
         for (int z = 0; z < L->nsplit_b; ++z) a += pb[(size_t)z * L->out + i];
-        db[i] = a;
+        db[i] = (float)a;
     }
     return VFL_OK;
 }

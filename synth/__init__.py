@@ -294,9 +294,24 @@ def _label_cfg5(seed, x):
     return np.argmax((x - 0.5) @ w.T, axis=1).astype(np.int32)
 
 
+def _features_custom(seed, r0, r1, d):
+    return _normal_matrix(seed, 20, r0, r1, d)
+
+
+def _label_custom(seed, x, r0, r1, n_out, loss):
+    # a linear teacher over all columns: Bernoulli(sigmoid) for BCE, argmax over n_out classes for CE
+    d = x.shape[1]
+    if loss == "bce":
+        w = _teacher_normal(seed, 20, (d,), math.sqrt(1.0 / d))
+        return _bernoulli(seed, 20, r0, r1, _sigmoid(x @ w))
+    w = _teacher_normal(seed, 21, (n_out, d), math.sqrt(1.0 / d))
+    return np.argmax(x @ w.T, axis=1).astype(np.int32)
+
+
 def make_dataset(p: VflPreset, rows=None, chunk: int | None = None):
     """(x_passive fp32 [n, d_p], x_active fp32 [n, d_a], y int32 [n]) for rows
-    [r0, r1) of preset ``p`` (all rows by default)."""
+    [r0, r1) of preset ``p`` (all rows by default).  cid 0 is a model of any
+    shape: N(0, 1) features and labels from a seeded linear teacher."""
     r0, r1 = (0, p.n_rows) if rows is None else rows
     if not (0 <= r0 <= r1 <= p.n_rows):
         raise ValueError(f"row range {rows} outside [0, {p.n_rows}]")
@@ -315,7 +330,10 @@ def make_dataset(p: VflPreset, rows=None, chunk: int | None = None):
     else:
         for a in range(r0, r1, chunk):
             b = min(r1, a + chunk)
-            if p.cid == 1:
+            if p.cid == 0:
+                x = _features_custom(seed, a, b, p.d_passive + p.d_active)
+                y = _label_custom(seed, x, a, b, p.n_out, p.loss)
+            elif p.cid == 1:
                 x = _features_cfg1(seed, a, b); y = _label_cfg1(seed, x, a, b)
             elif p.cid == 3:
                 x = _features_cfg3(seed, a, b); y = _label_cfg3(seed, x)

@@ -77,12 +77,77 @@ def compare_step(vfl, ctx, rec, tol, check_grads=True):
     errs["loss"] = abs(loss - rec.loss) / max(abs(rec.loss), 1e-30)
     if check_grads:
         g = ctx.get_grads(worker=k % ctx.p.workers)
+        out_layer = (2, len(ctx.p.top) - 1)
         for key, (dW, db) in g.items():
             errs[f"dW{key}"] = tensor_err(dW, rec.grads[key][0], dt)
-            errs[f"db{key}"] = tensor_err(db, rec.grads[key][1], dt)
+            if key == out_layer and dt == "fp32":
+                # db of the output layer is the column sum of d(logits), whose signed per-row terms
+                # cancel as the model calibrates: its error is taken against the sum of the terms'
+                # magnitudes, the scale that bounds the rounding error of a sum
+                scale = float(np.abs(rec.ds).sum(axis=0).max())
+                ref = np.asarray(rec.grads[key][1], np.float64)
+                errs[f"db{key}"] = float(np.abs(np.asarray(db, np.float64) - ref).max() /
+                                         max(np.abs(ref).max(), scale, 1e-30))
+            else:
+                errs[f"db{key}"] = tensor_err(db, rec.grads[key][1], dt)
     params = ctx.get_params()
     for key, (W, b) in params.items():
         errs[f"W{key}"] = tensor_err(W, rec.params[key][0], dt)
         errs[f"b{key}"] = tensor_err(b, rec.params[key][1], dt)
     bad = {name: e for name, e in errs.items() if not e <= tol}
     return errs, bad
+
+
+def oracle_version(o, v):
+    """{(party, layer): (W, b)} of the oracle's stored weight version v."""
+    out = {}
+    for l, (W, b) in enumerate(o.versions_p[v]):
+        out[(0, l)] = (W, b)
+    A, T = o.versions_a[v]
+    for l, (W, b) in enumerate(A):
+        out[(1, l)] = (W, b)
+    for l, (W, b) in enumerate(T):
+        out[(2, l)] = (W, b)
+    return out
+
+
+def force_gpu_state(ctx, o, S):
+    """Put the GPU context into the oracle's state before step o.k: cursor and
+    every stored weight version (oracle -> GPU only)."""
+    k = o.k
+    ctx.set_cursor(k)
+    for v in range(max(0, k - S), k + 1):
+        ctx.set_version(v, oracle_version(o, v))
+
+
+def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=None):
+    """Step-by-step comparison.  bf16 presets are teacher-forced: before each
+    step the GPU takes the oracle's weight versions, so one step's error is
+    measured without the drift of earlier roundings (a bf16 weight copy that
+    rounds the other way moves later ReLU masks)."""
+    p = synth.preset(cid) if isinstance(cid, int) else cid
+    if workers:
+        p = p.with_(workers=workers)
+    q, xp, xa, y, params = setup(p, n_rows)
+    nb = -(-n_rows // q.batch)
+    steps = steps or nb + 2                      # one epoch and two steps of the next
+    if teacher_forced is None:
+        teacher_forced = q.dtype == "bf16"
+    tp, ta = schedule(q, steps)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
+    worst = {}
+    failures = []
+    for k in range(steps):
+        if teacher_forced and k > 0:
+            force_gpu_state(ctx, o, q.staleness)
+        rec = o.step(int(tp[k]), int(ta[k]), record=True)
+        ctx.passive_forward(k, int(tp[k]))
+        ctx.active_step(k, int(ta[k]))
+        ctx.passive_backward(k)
+        errs, bad = compare_step(vfl, ctx, rec, TOL[q.dtype])
+        for name, e in errs.items():
+            worst[name] = max(worst.get(name, 0.0), e)
+        if bad:
+            failures.append((k, bad))
+    return worst, failures

@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 
 import oracle
-from _parity import EPOCH_LOSS_TOL, TOL, compare_step, new_context, rel_err, schedule, setup
+from _parity import EPOCH_LOSS_TOL, TOL, compare_step, new_context, rel_err, run_sequential, schedule, setup
 
 pytestmark = pytest.mark.gpu
 
@@ -31,62 +31,6 @@ CASES = {
     4: 8192 + 576,
     5: 2 * 2048 + 1344,
 }
-
-
-def oracle_version(o, v):
-    """{(party, layer): (W, b)} of the oracle's stored weight version v."""
-    out = {}
-    for l, (W, b) in enumerate(o.versions_p[v]):
-        out[(0, l)] = (W, b)
-    A, T = o.versions_a[v]
-    for l, (W, b) in enumerate(A):
-        out[(1, l)] = (W, b)
-    for l, (W, b) in enumerate(T):
-        out[(2, l)] = (W, b)
-    return out
-
-
-def force_gpu_state(ctx, o, S):
-    """Put the GPU context into the oracle's state before step o.k: cursor and
-    every stored weight version (oracle -> GPU only)."""
-    k = o.k
-    ctx.set_cursor(k)
-    for v in range(max(0, k - S), k + 1):
-        ctx.set_version(v, oracle_version(o, v))
-
-
-def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=None):
-    """Step-by-step comparison.  bf16 presets are teacher-forced: before each
-    step the GPU takes the oracle's weight versions, so one step's error is
-    measured without the drift of earlier roundings (a bf16 weight copy that
-    rounds the other way moves later ReLU masks)."""
-    import synth
-    p = synth.preset(cid)
-    if workers:
-        p = p.with_(workers=workers)
-    q, xp, xa, y, params = setup(p, n_rows)
-    nb = -(-n_rows // q.batch)
-    steps = steps or nb + 2                      # one epoch and two steps of the next
-    if teacher_forced is None:
-        teacher_forced = q.dtype == "bf16"
-    tp, ta = schedule(q, steps)
-    ctx = new_context(vfl, q, xp, xa, y, params)
-    o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
-    worst = {}
-    failures = []
-    for k in range(steps):
-        if teacher_forced and k > 0:
-            force_gpu_state(ctx, o, q.staleness)
-        rec = o.step(int(tp[k]), int(ta[k]), record=True)
-        ctx.passive_forward(k, int(tp[k]))
-        ctx.active_step(k, int(ta[k]))
-        ctx.passive_backward(k)
-        errs, bad = compare_step(vfl, ctx, rec, TOL[q.dtype])
-        for name, e in errs.items():
-            worst[name] = max(worst.get(name, 0.0), e)
-        if bad:
-            failures.append((k, bad))
-    return worst, failures
 
 
 @pytest.mark.parametrize("cid", [1, 2, 3, 4, 5])

@@ -49,3 +49,18 @@ def test_init_params(cid):
         bound = 1 / np.sqrt(fin)
         assert np.abs(W).max() <= bound and np.abs(b).max() <= bound
     assert synth.layer_shapes(p)[len(p.passive) + len(p.active)][3] == p.e_active + p.e_passive
+
+
+def test_custom_shape_recipe():
+    """cid 0: any widths; N(0, 1) features, labels within the classes of the loss."""
+    p = synth.preset(1).with_(cid=0, d_passive=37, d_active=5, n_rows=3000, top=(8, 5), loss="ce")
+    xp, xa, y = synth.make_dataset(p)
+    assert xp.shape == (3000, 37) and xa.shape == (3000, 5)
+    x = np.concatenate([xp, xa], 1)
+    assert abs(x.mean()) < 0.03 and abs(x.std() - 1) < 0.03
+    assert set(np.unique(y)) == set(range(5))
+    a = synth.make_dataset(p, rows=(1000, 1200))
+    for u, v in zip(a, (xp[1000:1200], xa[1000:1200], y[1000:1200])):
+        np.testing.assert_array_equal(u, v)
+    _, _, yb = synth.make_dataset(p.with_(loss="bce", top=(8, 1)))
+    assert set(np.unique(yb)) == {0, 1}
