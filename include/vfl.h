@@ -121,6 +121,28 @@ vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n,
                           const float* x_active, const int32_t* y);
 
 /*
+ * Host-resident data.  After this call every step k reads its own rows
+ * [r0, r1) of x_passive [n_rows, d_p] fp32, x_active [n_rows, d_a] fp32 and
+ * y [n_rows] int32 straight from host memory into a device staging ring of
+ * S + workers + 2 slots (part of the workspace), with one kernel on io_stream,
+ * and its phases read the rows there; the kernel that computes the step's mean
+ * loss also writes it to loss_out[k mod loss_cap] (skipped when loss_out is
+ * null).  A step's rows are read once the step that last used its slot has
+ * finished both updates.  The arrays must be page-locked (cudaHostAlloc,
+ * cudaHostRegister; VFL_E_INVAL otherwise) unless the device accesses pageable
+ * memory through the host's page tables, and must stay valid while steps that
+ * use them are in flight or a graph captured under the binding can still be
+ * launched: graphs captured under it contain the staging, and launch only
+ * while it holds.  io_stream is a caller stream (not a worker stream) that must
+ * outlive the binding.  The labels are checked here as vfl_load_data checks
+ * them; bf16 contexts round the staged rows to bf16.  Pass x_passive = null to
+ * unbind (the device-resident dataset is used again).  Valid only while no step
+ * is in flight; synchronizes the context.
+ */
+vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* x_passive, const float* x_active, const int32_t* y,
+                              float* loss_out, int64_t loss_cap, void* io_stream);
+
+/*
  * Set / read the fp32 master parameters of one layer: W [out, in], b [out]
  * (host pointers).  vfl_set_params resets every stored weight version of the
  * layer to the new values and is only valid before the first step.

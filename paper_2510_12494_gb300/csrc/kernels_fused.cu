@@ -737,7 +737,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     float* Ds = stage;
     float* Xs = stage + kUpdRows * kUpdLd;
     __shared__ __align__(16) float Pw[kUpdTile * kUpdTile];   // this CTA's partial dW tile
-    __shared__ double Pb[kUpdTile];                           // and partial db
+    __shared__ float Pb[kUpdTile];                            // and partial db
     griddep_wait();   // the d(pre-activation) rows, z^p's copy and the row losses come from the row kernel
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
@@ -755,6 +755,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
                 float v = 0.f;
                 for (int w = 0; w < kUpdThreads / 32; ++w) v += Pb[w];
                 *a.loss_out = v / (float)a.rows;
+                if (a.loss_host) *a.loss_host = v / (float)a.rows;
             }
         }
         return;
@@ -778,9 +779,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
         for (int q = 0; q < 4; ++q) acc[nt][q] = 0.f;
-    // db partial of output tid & 31, in fp64: db is a sum of signed per-row terms that largely cancel
-    // (softmax / sigmoid residuals), so fp32 rounding of the running sum can be large next to the result
-    double bacc = 0.0;
+    float bacc = 0.f;                                        // db partial of output tid & 31
     const bool dvec = (L.ldd & 3) == 0;                      // D rows hold whole 16-byte chunks
     for (int rb = rbeg; rb < rend; rb += kUpdRows) {
         const int nr = min(kUpdRows, rend - rb);
@@ -832,7 +831,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
         if (bias)
             for (int r = tid >> 5; r < nr; r += kUpdThreads / 32) bacc += Ds[r * kUpdLd + (tid & 31)];
     }
-    __shared__ double bpart[kUpdThreads];                    // db partials [8 warps][32]
+    __shared__ float bpart[kUpdThreads];                     // db partials [8 warps][32]
     bpart[tid] = bacc;
     __syncthreads();
     float* gpart = stage;                                    // [4 row groups][32][32]
@@ -846,7 +845,7 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     for (int e = tid; e < kUpdTile * kUpdTile; e += kUpdThreads)
         Pw[e] = ((gpart[e] + gpart[1024 + e]) + gpart[2048 + e]) + gpart[3072 + e];
     if (tid < kUpdTile) {
-        double sb = 0.0;
+        float sb = 0.f;
         for (int w = 0; w < kUpdThreads / 32; ++w) sb += bpart[w * 32 + tid];
         Pb[tid] = sb;
     }
@@ -869,10 +868,9 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     } else if (bias && tid < kPer + kUpdTile / kUpdCluster) {
         const int o = rank * (kUpdTile / kUpdCluster) + (tid - kPer);
         if (o < no) {
-            double gd = 0.0;
+            float g = 0.f;
 #pragma unroll
-            for (int q = 0; q < kUpdCluster; ++q) gd += cluster.map_shared_rank(Pb, q)[o];
-            const float g = (float)gd;
+            for (int q = 0; q < kUpdCluster; ++q) g += cluster.map_shared_rank(Pb, q)[o];
             const int go = o0 + o;
             L.gb[go] = g;
             const float b = L.bm[go] - a.lr * g;

@@ -141,7 +141,7 @@ constexpr int LOSS_NT = 1024;
 
 __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__ logits, const int* __restrict__ y,
                                                         int rows, int n_out, int kind, float* __restrict__ ds,
-                                                        float* __restrict__ loss_out) {
+                                                        float* __restrict__ loss_out, float* loss_host) {
     __shared__ float red[LOSS_NT / 32];
     const float inv_b = 1.0f / (float)rows;
     float part = 0.f;
@@ -174,7 +174,10 @@ __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__
     if (threadIdx.x < 32) {
         float v = red[threadIdx.x];
         for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
-        if (threadIdx.x == 0) *loss_out = v * inv_b;
+        if (threadIdx.x == 0) {
+            *loss_out = v * inv_b;
+            if (loss_host) *loss_host = v * inv_b;
+        }
     }
 }
 
@@ -329,6 +332,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         float v = 0.f;
         for (int bb = 0; bb < (int)gridDim.x; ++bb) v += __ldcg(a.blk_loss + bb);
         *a.loss_out = v * inv_b;
+        if (a.loss_host) *a.loss_host = v * inv_b;
         *a.counter = 0;
         __threadfence();
     }
@@ -462,6 +466,26 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
     }
 }
 
+// One step's rows from host memory (read over the C2C link / PCIe as the kernel runs): element i of
+// the padded passive rows, then of the padded active rows, then the labels.
+__global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const float* __restrict__ hxa, int da,
+                                  const int* __restrict__ hy, int rows, void* xp, long long ld_p, void* xa,
+                                  long long ld_a, int* __restrict__ y, int bf16) {
+    const long long np = (long long)rows * ld_p, na = (long long)rows * ld_a;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < np + na + rows;
+         i += (long long)gridDim.x * blockDim.x) {
+        if (i < np) {
+            const long long r = i / ld_p, c = i - r * ld_p;
+            stf(xp, i, bf16, c < dp ? hxp[r * dp + c] : 0.f);
+        } else if (i < np + na) {
+            const long long j = i - np, r = j / ld_a, c = j - r * ld_a;
+            stf(xa, j, bf16, c < da ? hxa[r * da + c] : 0.f);
+        } else {
+            y[i - np - na] = hy[i - np - na];
+        }
+    }
+}
+
 // Column sums over blocks of 64 rows: block (x, y) covers columns
 // [256 x, 256 x + 256) of rows [64 y, 64 y + 64); tx owns 8 adjacent columns,
 // ty every 8th row; the 8 row lanes are combined in a fixed order.
@@ -542,8 +566,8 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask
 }
 
 cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
-                        float* loss_out, cudaStream_t s) {
-    loss_kernel<<<1, LOSS_NT, 0, s>>>(logits, y, rows, n_out, loss_kind, ds, loss_out);
+                        float* loss_out, float* loss_host, cudaStream_t s) {
+    loss_kernel<<<1, LOSS_NT, 0, s>>>(logits, y, rows, n_out, loss_kind, ds, loss_out, loss_host);
     return cudaGetLastError();
 }
 
@@ -598,6 +622,14 @@ cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long ma
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     cast_rows_kernel<<<grid_for((long long)rows * ld, 256), 256, 0, s>>>(src, rows, d, dst, ld, bf16);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da, const int* hy, int rows, void* xp,
+                              long long ld_p, void* xa, long long ld_a, int* y, int bf16, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    const long long n = (long long)rows * (ld_p + ld_a + 1);
+    stage_rows_kernel<<<grid_for(n, 256), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, xp, ld_p, xa, ld_a, y, bf16);
     return cudaGetLastError();
 }
 

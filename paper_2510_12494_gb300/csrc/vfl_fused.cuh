@@ -104,6 +104,7 @@ struct FusedUpdArgs {
     float lr;
     const float* rowloss;             // mean loss of the step from these (nullptr: none)
     float* loss_out;
+    float* loss_host;                 // a second copy of it in mapped host memory (nullptr: none)
 };
 // Fills the tile bookkeeping of L[0..nl) and returns the number of output tiles.
 inline int fused_update_tiles(FusedUpdLayer* L, int nl) {

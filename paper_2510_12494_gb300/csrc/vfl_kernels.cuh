@@ -55,7 +55,7 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask
 //   rows: B_k; logits fp32 [B_k, n_out]; y int32 labels of the batch rows.
 //   ds [B_k, n_out] = dLoss/dlogits of the batch-mean loss; loss_out = mean loss.
 cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
-                        float* loss_out, cudaStream_t s);
+                        float* loss_out, float* loss_host, cudaStream_t s);
 
 // DP on the published gradient (one block per row):
 //   in fp32 [rows, e] (ld_in), out compute dtype [rows, e] (ld_out).
@@ -110,6 +110,7 @@ struct HeadArgs {
     float* blk_loss;                  // [blocks]
     int* counter;                     // blocks finished (re-armed by the last)
     float* loss_out;
+    float* loss_host;                 // a second copy of the mean loss in mapped host memory (or null)
 };
 inline int head_blocks(int rows) { return (rows + kHeadRows - 1) / kHeadRows; }
 cudaError_t launch_head(const HeadArgs& a, cudaStream_t s);
@@ -119,6 +120,10 @@ cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status,
                                cudaStream_t s);
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s);
+// Stage one step's rows from host-resident (mapped) arrays: x_p [rows, dp] and x_a [rows, da] fp32 into
+// rows of ld_p / ld_a elements (bf16 or fp32, padding columns zero), and the labels.
+cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da, const int* hy, int rows, void* xp,
+                              long long ld_p, void* xa, long long ld_a, int* y, int bf16, cudaStream_t s);
 // Column sums in blocks of 64 rows: Pb[z * pb_stride + o] = sum of D[r * ldd + o] over
 // rows r in [64 z, 64 z + 64) (zero for blocks past `rows`); z < nblocks.  D's row
 // stride must cover ceil(out / 8) * 8 columns.

@@ -32,6 +32,7 @@ namespace {
 constexpr int kMaxWorkers = 16;
 constexpr int kMaxSlots = 16;
 constexpr int kEvPool = 64;
+constexpr int kMaxIoSlots = kMaxSlots + kMaxWorkers + 2;   // staging ring: S + W + 2 slots
 constexpr int kLossCap = 4096;
 
 thread_local std::string g_global_err;
@@ -140,6 +141,21 @@ struct vfl_ctx {
     cudaStream_t as[kMaxWorkers] = {};
     cudaEvent_t ev_pver[kEvPool] = {}, ev_aver[kEvPool] = {}, ev_emb[kEvPool] = {}, ev_grad[kEvPool] = {};
 
+    // host-resident data (vfl_bind_host_data): each step reads its rows into slot k mod io_R of a
+    // device staging ring on the caller's I/O stream; the loss kernels also write the host ring
+    bool hio = false;
+    const float* h_xp = nullptr;
+    const float* h_xa = nullptr;
+    const int32_t* h_y = nullptr;
+    float* h_loss = nullptr;
+    long long h_loss_cap = 0;
+    int io_R = 0;
+    void* io_xp[kMaxIoSlots] = {};
+    void* io_xa[kMaxIoSlots] = {};
+    int* io_y[kMaxIoSlots] = {};
+    cudaStream_t io = nullptr;
+    cudaEvent_t ev_staged[kEvPool] = {};
+
     // per-launch timing (vfl_profile)
     bool prof_on = false;
     std::vector<ProfRec> prof;
@@ -225,7 +241,8 @@ struct vfl_graph {
     long long k0, n;
     HostState after;           // host state once the captured steps have run
     long long launches;        // kernels per replay
-    cudaEvent_t fork, join[2 * kMaxWorkers];
+    bool hio;                  // captured with host data bound (its copies are part of the graph)
+    cudaEvent_t fork, join[2 * kMaxWorkers + 1];
 };
 
 #define CK(call)                                                     \
@@ -523,6 +540,13 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
         }
         ctx->f_counter = static_cast<int*>(cv.take(2 * kMaxWorkers * sizeof(int)));
     }
+    // staging ring of host-resident data: slot k mod io_R holds step k's rows
+    ctx->io_R = c.staleness + ctx->W + 2;
+    for (int r = 0; r < ctx->io_R; ++r) {
+        ctx->io_xp[r] = cv.take(B * ctx->ldxp * es);
+        ctx->io_xa[r] = cv.take(B * ctx->ldxa * es);
+        ctx->io_y[r] = static_cast<int*>(cv.take(B * 4ull));
+    }
     if (ctx->head) {
         ctx->h_counter = static_cast<int*>(cv.take(kMaxWorkers * sizeof(int)));
         for (int w = 0; w < ctx->W; ++w)
@@ -532,6 +556,22 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
 }
 
 inline cudaStream_t pstream(vfl_ctx* ctx, long long k) { return ctx->ps[k % ctx->W]; }
+
+// Rows of step k (first row r0): the staging ring's slot when host data is bound, else the
+// device-resident dataset.  Both have the same row strides.
+inline const void* xp_rows(const vfl_ctx* ctx, long long k, long long r0) {
+    return ctx->hio ? ctx->io_xp[k % ctx->io_R] : static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+}
+inline const void* xa_rows(const vfl_ctx* ctx, long long k, long long r0) {
+    return ctx->hio ? ctx->io_xa[k % ctx->io_R] : static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * ctx->esz;
+}
+inline const int* y_rows(const vfl_ctx* ctx, long long k, long long r0) {
+    return ctx->hio ? ctx->io_y[k % ctx->io_R] : ctx->Y + r0;
+}
+// Where the kernel that computes step k's mean loss also writes it: the bound host ring, if any.
+inline float* loss_host(const vfl_ctx* ctx, long long k) {
+    return ctx->hio && ctx->h_loss ? ctx->h_loss + k % ctx->h_loss_cap : nullptr;
+}
 inline cudaStream_t astream(vfl_ctx* ctx, long long k) { return ctx->as[k % ctx->W]; }
 
 // ---- GEMM helpers ---------------------------------------------------------
@@ -849,7 +889,7 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     a.ldx = ctx->ldxa;
     long long r0;
     ctx->batch_rows(k, &r0);
-    a.y = ctx->Y + r0;
+    a.y = y_rows(ctx, k, r0);
     a.loss = ctx->cfg.loss;
     a.zp = static_cast<const float*>(ctx->act_p[slot].back());
     a.ldzp = ld8(ep);
@@ -904,6 +944,7 @@ vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float*
     u.nl = n;
     u.rowloss = ctx->f_rowloss[w];
     u.loss_out = ctx->losses + (k % kLossCap);
+    u.loss_host = loss_host(ctx, k);
     return launch_update(ctx, u, rows, s);
 }
 
@@ -955,6 +996,30 @@ vfl_status fused_passive_update(vfl_ctx* ctx, long long k, int slot, int rows, c
     return launch_update(ctx, u, rows, s);
 }
 
+// ---- host-resident data ----------------------------------------------------
+// Read step k's rows from the bound (mapped) host arrays into its staging slot on the I/O stream, after
+// the last step that used the slot (k - io_R: its passive and active updates are its last reads
+// of the rows); the step's phases wait for ev_staged.  io_R > S, so that step is always enqueued.
+vfl_status stage_step(vfl_ctx* ctx, long long k) {
+    const vfl_config& c = ctx->cfg;
+    long long r0;
+    const int rows = ctx->batch_rows(k, &r0);
+    const int slot = (int)(k % ctx->io_R);
+    cudaStream_t s = ctx->io;
+    const long long prev = k - ctx->io_R;
+    if (prev >= 0 && prev + 1 > ctx->ordered_floor) {
+        TRY(wait_ev(ctx, s, ctx->ev_pver[(prev + 1) % kEvPool]));
+        TRY(wait_ev(ctx, s, ctx->ev_aver[(prev + 1) % kEvPool]));
+    }
+    PLAUNCH(K_CAST, 0, (double)rows * (c.d_passive + c.d_active + 1) * 4 + (double)rows * (ctx->ldxp + ctx->ldxa) * ctx->esz,
+            s, launch_stage_rows(ctx->h_xp + r0 * c.d_passive, c.d_passive, ctx->h_xa + r0 * c.d_active, c.d_active,
+                                 ctx->h_y + r0, rows, ctx->io_xp[slot], ctx->ldxp, ctx->io_xa[slot], ctx->ldxa,
+                                 ctx->io_y[slot], ctx->bf16, s));
+    CK(cudaEventRecord(ctx->ev_staged[k % kEvPool], s));
+    return VFL_OK;
+}
+
+
 // ---- the three phases ------------------------------------------------------
 vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const vfl_config& c = ctx->cfg;
@@ -973,7 +1038,11 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     long long r0;
     const int rows = ctx->batch_rows(k, &r0);
     if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
-    const void* X = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+    if (ctx->hio) {
+        TRY(stage_step(ctx, k));
+        TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
+    }
+    const void* X = xp_rows(ctx, k, r0);
     if (ctx->fused) {
         TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), (int)(k % ctx->W), s));
         note_node(ctx, CAP_PFWD, k, s);
@@ -1012,7 +1081,6 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     cudaStream_t s = astream(ctx, k);
     const int slot = (int)(k % ctx->S1);
     const int vslot = (int)(v % ctx->S1);
-    const int es = ctx->esz;
     long long r0;
     const int rows = ctx->batch_rows(k, &r0);
     const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size(), Lp = (int)ctx->P.size();
@@ -1020,7 +1088,8 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const int n_out = ctx->T.back().out;
 
     if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
-    const void* Xa0 = static_cast<const char*>(ctx->Xa) + r0 * ctx->ldxa * es;
+    if (ctx->hio) TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
+    const void* Xa0 = xa_rows(ctx, k, r0);
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
         TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), w, s));
@@ -1072,7 +1141,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         h.W = H.cW[vslot]; h.ldw = H.in_ld;
         h.b = H.cb[vslot];
         h.K = H.in; h.nout = n_out; h.rows = rows; h.loss = c.loss;
-        h.y = ctx->Y + r0;
+        h.y = y_rows(ctx, k, r0);
         h.logits = ctx->logits[w]; h.ds = ctx->ds[w];
         h.dh = ctx->dpre_t[w][Lt - 2]; h.lddh = ld8(H.in);
         h.pW = H.pW[w]; h.pw_stride = (long long)n_out * H.in;
@@ -1081,6 +1150,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         h.blk_loss = ctx->h_blk_loss[w];
         h.counter = ctx->h_counter + w;
         h.loss_out = ctx->losses + (k % kLossCap);
+        h.loss_host = loss_host(ctx, k);
         const double hf = 2.0 * rows * n_out * H.in * 3.0;
         const double hb = (double)rows * H.in * ctx->esz * 2 + (double)n_out * H.in * ctx->esz +
                           (double)rows * (n_out * 8.0 + 4.0) + 4.0 * H.nsplit * ((double)n_out * H.in + n_out);
@@ -1088,8 +1158,8 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     } else {
         // loss and d(logits)
         PLAUNCH(K_LOSS, 0, (double)rows * n_out * 8 + rows * 4.0, s,
-                launch_loss(ctx->logits[w], ctx->Y + r0, rows, n_out, c.loss, ctx->ds[w],
-                            ctx->losses + (k % kLossCap), s));
+                launch_loss(ctx->logits[w], y_rows(ctx, k, r0), rows, n_out, c.loss, ctx->ds[w],
+                            ctx->losses + (k % kLossCap), loss_host(ctx, k), s));
     }
     // top backward (the head kernel has done the output layer's part)
     const bool dp = c.dp_clip > 0.f;
@@ -1156,7 +1226,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
     if (ctx->fused) {
-        const float* Xp = reinterpret_cast<const float*>(static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz);
+        const float* Xp = static_cast<const float*>(xp_rows(ctx, k, r0));
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
         note_node(ctx, CAP_PBWD, k, s);
         // SGD on theta_2 in step order
@@ -1172,7 +1242,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     PLAUNCH(K_MASK, 0, 3.0 * rows * ep * ctx->esz, s,
             launch_relu_mask(ctx->grad[slot], ctx->act_p[slot][Lp - 1], ctx->dpre_p[w][Lp - 1], ld8(ep), rows, ep,
                              ctx->bf16, s));
-    const void* Xp0 = static_cast<const char*>(ctx->Xp) + r0 * ctx->ldxp * ctx->esz;
+    const void* Xp0 = xp_rows(ctx, k, r0);
     for (int l = Lp - 1; l >= 0; --l) {
         const Layer& L = ctx->P[l];
         const void* Xin = l == 0 ? Xp0 : ctx->act_p[slot][l - 1];
@@ -1204,11 +1274,22 @@ vfl_status read_status(vfl_ctx* ctx) {
     return VFL_OK;
 }
 
-vfl_status sync_all(vfl_ctx* ctx) {
+// Every stream the context enqueues on: the workers' (passive, active), then the I/O pair.
+int ctx_streams(const vfl_ctx* ctx, cudaStream_t* out) {
+    int n = 0;
     for (int w = 0; w < ctx->W; ++w) {
-        CK(cudaStreamSynchronize(ctx->ps[w]));
-        CK(cudaStreamSynchronize(ctx->as[w]));
+        out[n++] = ctx->ps[w];
+        out[n++] = ctx->as[w];
     }
+    if (ctx->hio) out[n++] = ctx->io;
+    return n;
+}
+constexpr int kMaxStreams = 2 * kMaxWorkers + 1;
+
+vfl_status sync_all(vfl_ctx* ctx) {
+    cudaStream_t ss[kMaxStreams];
+    const int n = ctx_streams(ctx, ss);
+    for (int i = 0; i < n; ++i) CK(cudaStreamSynchronize(ss[i]));
     return read_status(ctx);
 }
 
@@ -1292,6 +1373,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_aver[i], cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_emb[i], cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_grad[i], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_staged[i], cudaEventDisableTiming);
     }
     if (e == cudaSuccess) e = cudaMemset(workspace, 0, need);
     if (e == cudaSuccess) e = cudaMemset(ctx->emb_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
@@ -1309,10 +1391,9 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
 vfl_status vfl_destroy(vfl_ctx* ctx) {
     if (!ctx) return VFL_OK;
     if (!ctx->broken) {
-        for (int w = 0; w < ctx->W; ++w) {
-            cudaStreamSynchronize(ctx->ps[w]);
-            cudaStreamSynchronize(ctx->as[w]);
-        }
+        cudaStream_t ss[kMaxStreams];
+        const int n = ctx_streams(ctx, ss);
+        for (int i = 0; i < n; ++i) cudaStreamSynchronize(ss[i]);
     }
     for (ProfRec& r : ctx->prof) {
         ctx->ev_spare.push_back(r.e0);
@@ -1325,6 +1406,7 @@ vfl_status vfl_destroy(vfl_ctx* ctx) {
         if (ctx->ev_aver[i]) cudaEventDestroy(ctx->ev_aver[i]);
         if (ctx->ev_emb[i]) cudaEventDestroy(ctx->ev_emb[i]);
         if (ctx->ev_grad[i]) cudaEventDestroy(ctx->ev_grad[i]);
+        if (ctx->ev_staged[i]) cudaEventDestroy(ctx->ev_staged[i]);
     }
     delete ctx;
     return VFL_OK;
@@ -1384,6 +1466,66 @@ vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n,
     PLAUNCH(K_CAST, 0, n * c.d_active * (4.0 + ctx->esz), sa, launch_cast_rows(ctx->stage_a[worker], (int)n, c.d_active,
                             static_cast<char*>(ctx->Xa) + row0 * ctx->ldxa * ctx->esz, ctx->ldxa, ctx->bf16, sa));
     CK(cudaMemcpyAsync(ctx->Y + row0, y, (size_t)n * 4, cudaMemcpyHostToDevice, sa));
+    return VFL_OK;
+}
+
+namespace {
+// The device-side address of host memory that kernels may read or write: page-locked memory
+// registered with CUDA, or any host memory on a device that accesses pageable memory coherently.
+const void* device_view(const void* p) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    if (at.type == cudaMemoryTypeHost && at.devicePointer) return at.devicePointer;
+    int dev = 0, pageable = 0;
+    if (at.type == cudaMemoryTypeUnregistered && cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccessUsesHostPageTables, dev) == cudaSuccess &&
+        pageable)
+        return p;
+    return nullptr;
+}
+}  // namespace
+
+vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* xp, const float* xa, const int32_t* y, float* loss_out,
+                              int64_t loss_cap, void* io_stream) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_bind_host_data with steps in flight");
+    if (!xp) {
+        TRY(sync_all(ctx));
+        ctx->hio = false;
+        ctx->h_xp = ctx->h_xa = nullptr;
+        ctx->h_y = nullptr;
+        ctx->h_loss = nullptr;
+        ctx->h_loss_cap = 0;
+        ctx->io = nullptr;
+        return VFL_OK;
+    }
+    if (!xa || !y || !io_stream) return ctx->fail(VFL_E_INVAL, "null host array or I/O stream");
+    if (loss_out && loss_cap < 1) return ctx->fail(VFL_E_INVAL, "loss_cap must be >= 1");
+    for (int w = 0; w < ctx->W; ++w)
+        if (io_stream == ctx->ps[w] || io_stream == ctx->as[w])
+            return ctx->fail(VFL_E_INVAL, "the I/O stream must not be a worker stream");
+    const int n_cls = ctx->cfg.loss == VFL_LOSS_BCE ? 2 : ctx->T.back().out;
+    for (long long i = 0; i < ctx->n_rows; ++i)
+        if (y[i] < 0 || y[i] >= n_cls) return ctx->fail(VFL_E_INVAL, "label %d of row %lld outside [0, %d)", y[i], i, n_cls);
+    const void* dxp = device_view(xp);
+    const void* dxa = device_view(xa);
+    const void* dy = device_view(y);
+    const void* dl = loss_out ? device_view(loss_out) : nullptr;
+    if (!dxp || !dxa || !dy || (loss_out && !dl))
+        return ctx->fail(VFL_E_INVAL, "host arrays must be page-locked (cudaHostAlloc / cudaHostRegister)");
+    TRY(sync_all(ctx));
+    ctx->h_xp = static_cast<const float*>(dxp);
+    ctx->h_xa = static_cast<const float*>(dxa);
+    ctx->h_y = static_cast<const int32_t*>(dy);
+    ctx->h_loss = static_cast<float*>(const_cast<void*>(dl));
+    ctx->h_loss_cap = loss_out ? loss_cap : 0;
+    ctx->io = static_cast<cudaStream_t>(io_stream);
+    ctx->hio = true;
     return VFL_OK;
 }
 
@@ -1664,8 +1806,9 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     g->ctx = ctx;
     g->k0 = k0;
     g->n = n_steps;
+    g->hio = ctx->hio;
     cudaError_t e = cudaEventCreateWithFlags(&g->fork, cudaEventDisableTiming);
-    for (int i = 0; i < 2 * ctx->W && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
+    for (int i = 0; i < kMaxStreams && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
     if (e != cudaSuccess) {
         delete g;
         return ctx->cuda(e, "cudaEventCreate", __LINE__);
@@ -1674,12 +1817,12 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     cudaStream_t origin = ctx->ps[0];
     cudaGraph_t graph = nullptr;
     vfl_status st = VFL_OK;
+    cudaStream_t ss[kMaxStreams];
+    const int nss = ctx_streams(ctx, ss);
     e = cudaStreamBeginCapture(origin, cudaStreamCaptureModeThreadLocal);
     if (e == cudaSuccess) e = cudaEventRecord(g->fork, origin);
-    for (int w = 0; w < ctx->W && e == cudaSuccess; ++w) {
-        if (w > 0) e = cudaStreamWaitEvent(ctx->ps[w], g->fork, 0);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->as[w], g->fork, 0);
-    }
+    for (int i = 0; i < nss && e == cudaSuccess; ++i)
+        if (ss[i] != origin) e = cudaStreamWaitEvent(ss[i], g->fork, 0);
     const long long floor_before = ctx->ordered_floor;
     ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k0);
     ctx->cap_nodes.clear();
@@ -1688,15 +1831,9 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     ctx->capturing = false;
     ctx->ordered_floor = floor_before;
     // join every stream back into the origin, even after a failure, so that capture can end
-    int j = 0;
-    for (int w = 0; w < ctx->W; ++w) {
-        cudaStream_t ss[2] = {ctx->ps[w], ctx->as[w]};
-        for (cudaStream_t x : ss) {
-            if (x == origin) continue;
-            if (cudaEventRecord(g->join[j], x) == cudaSuccess) cudaStreamWaitEvent(origin, g->join[j], 0);
-            ++j;
-        }
-    }
+    for (int i = 0; i < nss; ++i)
+        if (ss[i] != origin && cudaEventRecord(g->join[i], ss[i]) == cudaSuccess)
+            cudaStreamWaitEvent(origin, g->join[i], 0);
     cudaError_t e2 = cudaStreamEndCapture(origin, &graph);
     if (e == cudaSuccess) e = e2;
     if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, graph, k0, n_steps, tau_p);
@@ -1724,24 +1861,20 @@ vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* g) {
     if (ctx->broken) return VFL_E_CUDA;
     if (ctx->n_fwd != g->k0 || ctx->n_act != g->k0 || ctx->n_bwd != g->k0)
         return ctx->fail(VFL_E_STATE, "graph starts at step %lld but the context is at step %lld", g->k0, ctx->n_fwd);
+    if (g->hio != ctx->hio) return ctx->fail(VFL_E_STATE, "graph captured with another host-data binding");
     cudaStream_t origin = ctx->ps[0];
     // order the replay after everything already enqueued on the context's streams, and theirs after it
-    int j = 0;
-    for (int w = 0; w < ctx->W; ++w) {
-        cudaStream_t ss[2] = {ctx->ps[w], ctx->as[w]};
-        for (cudaStream_t x : ss) {
-            if (x == origin) continue;
-            CK(cudaEventRecord(g->join[j], x));
-            CK(cudaStreamWaitEvent(origin, g->join[j], 0));
-            ++j;
-        }
+    cudaStream_t ss[kMaxStreams];
+    const int nss = ctx_streams(ctx, ss);
+    for (int i = 0; i < nss; ++i) {
+        if (ss[i] == origin) continue;
+        CK(cudaEventRecord(g->join[i], ss[i]));
+        CK(cudaStreamWaitEvent(origin, g->join[i], 0));
     }
     CK(cudaGraphLaunch(g->exec, origin));
     CK(cudaEventRecord(g->fork, origin));
-    for (int w = 0; w < ctx->W; ++w) {
-        if (w > 0) CK(cudaStreamWaitEvent(ctx->ps[w], g->fork, 0));
-        CK(cudaStreamWaitEvent(ctx->as[w], g->fork, 0));
-    }
+    for (int i = 0; i < nss; ++i)
+        if (ss[i] != origin) CK(cudaStreamWaitEvent(ss[i], g->fork, 0));
     const long long launched = ctx->launches + g->launches;
     load_state(ctx, g->after);
     ctx->launches = launched;

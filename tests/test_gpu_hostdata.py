@@ -1,0 +1,100 @@
+"""Host-resident data (vfl_bind_host_data): every step copies its own rows from
+pinned host memory into the staging ring and its loss back out.  Training this
+way is bit-identical to training on the device-resident dataset, directly
+enqueued or replayed from CUDA graphs, across epochs (ring slots reused) and
+with several worker streams."""
+import numpy as np
+import pytest
+
+import synth
+from _parity import new_context, schedule, setup
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def vfl():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2510_12494_gb300 import build
+    build.build()
+    import paper_2510_12494_gb300 as v
+    return v
+
+
+def host_context(vfl, q, xp, xa, y, params, cap):
+    """A context that never loads the dataset: its resident copy stays zero."""
+    import torch
+    ctx = vfl.Context(q, q.n_rows)
+    ctx.set_params(params)
+    pins = [torch.from_numpy(a).pin_memory() for a in (xp, xa, y)]
+    loss = torch.full((cap,), float("nan"), dtype=torch.float32).pin_memory()
+    ctx.bind_host_data(*pins, loss_out=loss)
+    return ctx, loss
+
+
+def assert_same_state(a, b):
+    for key, (W, bias) in a.get_params().items():
+        W2, b2 = b.get_params()[key]
+        np.testing.assert_array_equal(W, W2)
+        np.testing.assert_array_equal(bias, b2)
+
+
+@pytest.mark.parametrize("cid,workers", [(1, 0), (2, 0), (2, 3), (3, 0)])
+def test_host_data_equals_resident(vfl, cid, workers):
+    p = synth.preset(cid)
+    if workers:
+        p = p.with_(workers=workers)
+    rows = {1: 4096 - 100, 2: 4 * 1024 + 304, 3: 2 * 4096 + 288}[cid]
+    q, xp, xa, y, params = setup(p, rows)
+    n = 2 * q.steps_per_epoch + 3
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx, loss = host_context(vfl, q, xp, xa, y, params, cap=n)
+    ctx.train_steps(0, n, tp, ta)
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
+    assert_same_state(ctx, ref)
+
+
+@pytest.mark.parametrize("cid", [2, 3])
+def test_host_data_graph_replay(vfl, cid):
+    """Graphs captured under the binding carry the copies: replaying windows
+    gives the same losses and weights as direct enqueue on resident data."""
+    p = synth.preset(cid)
+    rows = {2: 4 * 1024 + 304, 3: 2 * 4096 + 288}[cid]
+    q, xp, xa, y, params = setup(p, rows)
+    nb = q.steps_per_epoch
+    n = 2 * nb + 3
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx, loss = host_context(vfl, q, xp, xa, y, params, cap=n)
+    ctx.train_steps(0, 2, tp, ta)                  # a direct prefix, then graphs
+    k = 2
+    while k < n:
+        m = min(nb, n - k)
+        g = ctx.capture(k, m, tp, ta)
+        ctx.launch_graph(g)
+        k += m
+    ctx.synchronize()
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
+    assert_same_state(ctx, ref)
+
+
+def test_unbind_returns_to_resident_data(vfl):
+    q, xp, xa, y, params = setup(synth.preset(2), 2 * 1024 + 304)
+    n = 7
+    tp, ta = schedule(q, 2 * n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, 2 * n, tp, ta)
+    ctx, loss = host_context(vfl, q, xp, xa, y, params, cap=n)
+    ctx.train_steps(0, n, tp, ta)
+    ctx.bind_host_data(None, None, None)
+    ctx.load_data(xp, xa, y)
+    ctx.train_steps(n, n, tp, ta)
+    np.testing.assert_array_equal(ctx.read_losses(0, 2 * n), ref.read_losses(0, 2 * n))
+    assert_same_state(ctx, ref)
