@@ -722,9 +722,10 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
 
 // dW = D^T X, db = sum of D's rows, then SGD, for one 32 x 32 output tile per
 // cluster; CTA `rank` of the cluster covers rows [rank c, (rank + 1) c) with
-// c = ceil(rows / 8).  Inside a CTA, 4 row groups x (8 x 8 threads of 4 x 4
-// outputs) accumulate in fp32; the groups, then the 8 ranks, are summed in a
-// fixed order.
+// c = ceil(rows / 8).  Inside a CTA, 4 row groups accumulate in fp32 and are
+// summed in a fixed order; each CTA then pushes its partial of the 128 outputs
+// rank q owns into q's shared memory (slot = sender's rank), and after one
+// cluster barrier every owner sums its 8 slots in rank order and applies SGD.
 constexpr int kUpdRows = 128;                // rows staged per pass: 32 per row group of 2 warps
 constexpr int kUpdLd = kUpdTile + 8;         // smem row stride, 8 mod 32: the MMA fragment loads are conflict-free
 static_assert(kUpdThreads == 256 && kUpdTile == 32, "the thread map below assumes 256 threads and 32 x 32 tiles");
@@ -736,8 +737,11 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     __shared__ __align__(16) float stage[2 * kUpdRows * kUpdLd];
     float* Ds = stage;
     float* Xs = stage + kUpdRows * kUpdLd;
-    __shared__ __align__(16) float Pw[kUpdTile * kUpdTile];   // this CTA's partial dW tile
-    __shared__ float Pb[kUpdTile];                            // and partial db
+    constexpr int kPer = kUpdTile * kUpdTile / kUpdCluster;   // outputs of the tile each rank owns
+    constexpr int kPerB = kUpdTile / kUpdCluster;             // bias outputs each rank owns
+    __shared__ __align__(16) float Rw[kUpdCluster * kPer];    // partials of the owned outputs, by sender
+    __shared__ float Rb[kUpdCluster * kPerB];
+    __shared__ float Pb[kUpdThreads / 32];                    // the loss cluster's warp sums
     griddep_wait();   // the d(pre-activation) rows, z^p's copy and the row losses come from the row kernel
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
@@ -842,22 +846,25 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
         *reinterpret_cast<float2*>(pw + 8 * kUpdTile) = make_float2(acc[nt][2], acc[nt][3]);
     }
     __syncthreads();
-    for (int e = tid; e < kUpdTile * kUpdTile; e += kUpdThreads)
-        Pw[e] = ((gpart[e] + gpart[1024 + e]) + gpart[2048 + e]) + gpart[3072 + e];
+    // rank q owns outputs [128 q, 128 q + 128) of the tile (rows 4q..4q+3) and bias outputs 4q..4q+3
+    for (int e = tid; e < kUpdTile * kUpdTile; e += kUpdThreads) {
+        const float v = ((gpart[e] + gpart[1024 + e]) + gpart[2048 + e]) + gpart[3072 + e];
+        const int q = e / kPer;
+        cluster.map_shared_rank(Rw, q)[rank * kPer + (e - q * kPer)] = v;
+    }
     if (tid < kUpdTile) {
         float sb = 0.f;
         for (int w = 0; w < kUpdThreads / 32; ++w) sb += bpart[w * 32 + tid];
-        Pb[tid] = sb;
+        const int q = tid / kPerB;
+        cluster.map_shared_rank(Rb, q)[rank * kPerB + (tid - q * kPerB)] = sb;
     }
-    cluster.sync();
-    // rank q sums outputs [128 q, 128 q + 128) of the tile (rows 4q..4q+3) over the ranks in order
-    constexpr int kPer = kUpdTile * kUpdTile / kUpdCluster;
+    cluster.sync();   // every push has landed; no shared memory of another CTA is touched after this
     if (tid < kPer) {
         const int e = rank * kPer + tid, o = e / kUpdTile, i = e - o * kUpdTile;
         if (o < no && i < ni) {
             float g = 0.f;
 #pragma unroll
-            for (int q = 0; q < kUpdCluster; ++q) g += cluster.map_shared_rank(Pw, q)[e];
+            for (int q = 0; q < kUpdCluster; ++q) g += Rw[q * kPer + tid];
             const long long go = o0 + o, gi = i0 + i;
             const long long idx = go * L.in + gi;
             L.gW[idx] = g;
@@ -865,12 +872,12 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
             L.Wm[idx] = w;
             L.Wc[go * L.in_ld + gi] = w;
         }
-    } else if (bias && tid < kPer + kUpdTile / kUpdCluster) {
-        const int o = rank * (kUpdTile / kUpdCluster) + (tid - kPer);
+    } else if (bias && tid < kPer + kPerB) {
+        const int o = rank * kPerB + (tid - kPer);
         if (o < no) {
             float g = 0.f;
 #pragma unroll
-            for (int q = 0; q < kUpdCluster; ++q) g += cluster.map_shared_rank(Pb, q)[o];
+            for (int q = 0; q < kUpdCluster; ++q) g += Rb[q * kPerB + (tid - kPer)];
             const int go = o0 + o;
             L.gb[go] = g;
             const float b = L.bm[go] - a.lr * g;
@@ -878,7 +885,6 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
             L.bc[go] = b;
         }
     }
-    cluster.sync();                                          // peers' shared memory stays valid until here
 }
 
 template <typename K>
