@@ -3,11 +3,11 @@
 // SGD step (Eq. 2, delayed form of App. D) is one more.
 //
 //  - passive forward: every CTA stages all of f_p's weights into shared memory
-//    with cp.async, then runs the bottom chain for its 16-row tile; the last CTA
-//    to finish publishes the embedding channel's header.
+//    with cp.async, then runs the bottom chain for its 16-row tile; CTA 0 writes
+//    the embedding channel's header.
 //  - active step: active bottom forward, top forward on [z^a | z^p], loss, the
 //    input-gradient chain back to the first active layer; dz^p goes to the
-//    gradient channel (header written by the last CTA), every layer's
+//    gradient channel (header written by CTA 0), every layer's
 //    d(pre-activation) rows stay in HBM for the update.
 //  - passive backward: the input-gradient chain of f_p from dz^p.
 //  - update (one per party): dW = D^T X over the step's rows for every layer,
@@ -49,6 +49,18 @@ static_assert(R == 16, "the MMA tiles cover exactly 16 rows");
 static_assert(NW == R, "row-tile copies give each warp one row");
 
 __device__ __forceinline__ int ceil8(int x) { return (x + 7) & ~7; }
+
+// The channel header of a published payload, written by CTA 0.  Every subscriber is ordered after
+// the publishing kernel's completion (stream order, an event, or a programmatic dependency whose
+// wait returns once the grid has completed), which makes all of the grid's payload writes visible
+// with the header; so no CTA needs to wait for the others or fence its writes here.
+__device__ __forceinline__ void publish_header(ChannelHeader* hdr, long long k, int batch, int version) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        hdr->k = k;
+        hdr->batch = batch;
+        hdr->version = version;
+    }
+}
 
 __device__ __forceinline__ void cp16(float* s, const float* g) {
     const unsigned sa = (unsigned)__cvta_generic_to_shared(s);
@@ -336,38 +348,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
         first = false;
     }
     if (first) griddep_wait();       // CTAs without a row tile have nothing in flight
-    // the last CTA to finish publishes the header after every payload write
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const int done = atomicAdd(a.counter, 1);
-        if (done == (int)gridDim.x - 1) {
-            __threadfence();
-            a.hdr->k = a.k;
-            a.hdr->batch = a.batch;
-            a.hdr->version = a.version;
-            *a.counter = 0;
-            __threadfence();
-        }
-    }
-}
-
-// One CTA's share of the "last CTA publishes" rule: after every CTA's payload
-// writes, the last one to arrive writes the header and re-arms the counter.
-__device__ void publish_when_last(int* counter, ChannelHeader* hdr, long long k, int batch, int version) {
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const int done = atomicAdd(counter, 1);
-        if (done == (int)gridDim.x - 1) {
-            __threadfence();
-            hdr->k = k;
-            hdr->batch = batch;
-            hdr->version = version;
-            *counter = 0;
-            __threadfence();
-        }
-    }
+    publish_header(a.hdr, a.k, a.batch, a.version);
 }
 
 // Loss of one row (Eq. 1 in the stable logit form, or softmax cross-entropy)
@@ -651,7 +632,7 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
         cp_wait_pending(0);
     }
     if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
-    publish_when_last(a.counter, a.pub_hdr, a.k, a.batch, a.version);
+    publish_header(a.pub_hdr, a.k, a.batch, a.version);
 }
 
 __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedStepArgs a) {

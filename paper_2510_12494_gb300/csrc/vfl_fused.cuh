@@ -55,7 +55,6 @@ struct FusedChainArgs {
     int nl;
     const float* x; long long ldx;
     int rows, act_ld, w_floats;
-    int* counter;
     ChannelHeader* hdr;
     long long k; int batch, version;
 };
@@ -76,7 +75,6 @@ struct FusedStepArgs {
     float* rowloss;                     // active: per-row loss
     const ChannelHeader* chk_hdr;       // header to check (embedding / gradient channel)
     ChannelHeader* pub_hdr;             // header to publish (active: gradient channel)
-    int* counter;                       // active: CTAs done, for the last one to publish
     long long k; int batch, version;
     int* status;
 };

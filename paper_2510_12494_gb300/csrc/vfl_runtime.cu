@@ -129,7 +129,6 @@ struct vfl_ctx {
     int f_act_ld = 0, f_wp = 0, f_wa = 0;       // smem row stride, weight-stage floats per party
     float* f_rowloss[kMaxWorkers] = {};         // per worker: per-row loss [B]
     float* f_zpc[kMaxWorkers] = {};             // per worker: z^p rows consumed by the step [B, ld8(e_p)]
-    int* f_counter = nullptr;                   // last-CTA counters: [0, 16) passive fwd, [16, 32) active, per worker
 
     // bf16 path: g's output layer and the loss in one launch (narrow output over a narrow hidden layer)
     bool head = false;
@@ -538,7 +537,6 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             ctx->f_rowloss[w] = static_cast<float*>(cv.take(B * 4ull));
             ctx->f_zpc[w] = static_cast<float*>(cv.take(B * ld8(ctx->P.back().out) * 4ull));
         }
-        ctx->f_counter = static_cast<int*>(cv.take(2 * kMaxWorkers * sizeof(int)));
     }
     // staging ring of host-resident data: slot k mod io_R holds step k's rows
     ctx->io_R = c.staleness + ctx->W + 2;
@@ -849,7 +847,6 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     a.rows = rows;
     a.act_ld = ctx->f_act_ld;
     a.w_floats = fused_weight_layout(a.L, a.nl, 0);
-    a.counter = ctx->f_counter + w;
     a.hdr = ctx->emb_hdr + slot;
     a.k = k;
     a.batch = (int)(k % ctx->nb);
@@ -900,7 +897,6 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     a.rowloss = ctx->f_rowloss[w];
     a.chk_hdr = ctx->emb_hdr + slot;
     a.pub_hdr = ctx->grad_hdr + slot;
-    a.counter = ctx->f_counter + kMaxWorkers + w;
     a.k = k;
     a.batch = (int)(k % ctx->nb);
     a.version = (int)v;
