@@ -723,12 +723,14 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     __shared__ __align__(16) float Rw[kUpdCluster * kPer];    // partials of the owned outputs, by sender
     __shared__ float Rb[kUpdCluster * kPerB];
     __shared__ float Pb[kUpdThreads / 32];                    // the loss cluster's warp sums
-    griddep_wait();   // the d(pre-activation) rows, z^p's copy and the row losses come from the row kernel
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int tile = blockIdx.x / kUpdCluster;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // the d(pre-activation) rows, most inputs X and the row losses come from the row kernel this launch
+    // depends on (programmatically, in a graph): griddep_wait() comes before any read of them
     if (tile == a.ntiles) {                                  // one extra cluster: mean loss of the step, fixed order
+        griddep_wait();
         if (rank == 0 && a.loss_out) {
             float s = 0.f;
             for (int r = tid; r < a.rows; r += kUpdThreads) s += a.rowloss[r];
@@ -754,6 +756,31 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     const bool bias = i0 == 0;
     const int chunk = (a.rows + kUpdCluster - 1) / kUpdCluster;
     const int rbeg = min(a.rows, rank * chunk), rend = min(a.rows, rbeg + chunk);
+    // this rank's outputs of the tile: the master of version k was written by the previous update, a
+    // full dependency, so it is read now and its latency hides behind the wait
+    const int eo = rank * kPer + tid, oo = eo / kUpdTile, io = eo - oo * kUpdTile;
+    const bool own_w = tid < kPer && oo < no && io < ni;
+    const long long widx = (long long)(o0 + oo) * L.in + (i0 + io);
+    const float wm = own_w ? L.Wm[widx] : 0.f;
+    const int ob = rank * kPerB + (tid - kPer);
+    const bool own_b = bias && tid >= kPer && tid < kPer + kPerB && ob < no;
+    const float bmv = own_b ? L.bm[o0 + ob] : 0.f;
+    // rows [rb, rb + nr) of X[:, i0 : i0+32] in 16-byte chunks (cp.async), zero past the layer's columns;
+    // X's columns come from X or, from xsplit on (a multiple of 4), from X2
+    auto stage_x = [&](int rb, int nr) {
+        for (int e = tid; e < kUpdRows * (kUpdTile / 4); e += kUpdThreads) {
+            const int r = e >> 3, c = (e & 7) * 4;
+            float* xs = Xs + r * kUpdLd + c;
+            const long long gr = rb + r;
+            const int ic = i0 + c;
+            if (r < nr && ic < L.in)
+                cp16(xs, ic < L.xsplit ? L.X + gr * L.ldx + ic : L.X2 + gr * L.ldx2 + (ic - L.xsplit));
+            else
+                *reinterpret_cast<float4*>(xs) = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    };
+    if (L.x_early && rbeg < rend) stage_x(rbeg, min(kUpdRows, rend - rbeg));
+    griddep_wait();
 
     const int fg = lane >> 2, ft = lane & 3;     // MMA fragment row / column lane
     // the 32 x 32 tile as 2 (outputs) x 4 (inputs) MMA blocks in 3xTF32, A[o][r] = D[r][o],
@@ -768,13 +795,11 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     const bool dvec = (L.ldd & 3) == 0;                      // D rows hold whole 16-byte chunks
     for (int rb = rbeg; rb < rend; rb += kUpdRows) {
         const int nr = min(kUpdRows, rend - rb);
-        __syncthreads();
-        // rows [rb, rb + nr) of D[:, o0 : o0+32] and X[:, i0 : i0+32] in 16-byte chunks (cp.async), zero
-        // past the layer's columns; X's columns come from X or, from xsplit on (a multiple of 4), from X2
+        if (rb > rbeg) __syncthreads();                      // the previous pass has read the stage
+        // rows [rb, rb + nr) of D[:, o0 : o0+32] in 16-byte chunks (cp.async), zero past the layer's columns
         for (int e = tid; e < kUpdRows * (kUpdTile / 4); e += kUpdThreads) {
             const int r = e >> 3, c = (e & 7) * 4;
             float* ds = Ds + r * kUpdLd + c;
-            float* xs = Xs + r * kUpdLd + c;
             const long long gr = rb + r;
             if (r < nr && o0 + c < L.out && dvec) {
                 cp16(ds, L.D + gr * L.ldd + o0 + c);
@@ -782,12 +807,8 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
 #pragma unroll
                 for (int q = 0; q < 4; ++q) ds[q] = (r < nr && o0 + c + q < L.out) ? __ldg(L.D + gr * L.ldd + o0 + c + q) : 0.f;
             }
-            const int ic = i0 + c;
-            if (r < nr && ic < L.in)
-                cp16(xs, ic < L.xsplit ? L.X + gr * L.ldx + ic : L.X2 + gr * L.ldx2 + (ic - L.xsplit));
-            else
-                *reinterpret_cast<float4*>(xs) = make_float4(0.f, 0.f, 0.f, 0.f);
         }
+        if (!(L.x_early && rb == rbeg)) stage_x(rb, nr);
         cp_commit();
         cp_wait_pending(0);
 #pragma unroll
@@ -840,31 +861,23 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
         cluster.map_shared_rank(Rb, q)[rank * kPerB + (tid - q * kPerB)] = sb;
     }
     cluster.sync();   // every push has landed; no shared memory of another CTA is touched after this
-    if (tid < kPer) {
-        const int e = rank * kPer + tid, o = e / kUpdTile, i = e - o * kUpdTile;
-        if (o < no && i < ni) {
-            float g = 0.f;
+    if (own_w) {
+        float g = 0.f;
 #pragma unroll
-            for (int q = 0; q < kUpdCluster; ++q) g += Rw[q * kPer + tid];
-            const long long go = o0 + o, gi = i0 + i;
-            const long long idx = go * L.in + gi;
-            L.gW[idx] = g;
-            const float w = L.Wm[idx] - a.lr * g;
-            L.Wm[idx] = w;
-            L.Wc[go * L.in_ld + gi] = w;
-        }
-    } else if (bias && tid < kPer + kPerB) {
-        const int o = rank * kPerB + (tid - kPer);
-        if (o < no) {
-            float g = 0.f;
+        for (int q = 0; q < kUpdCluster; ++q) g += Rw[q * kPer + tid];
+        L.gW[widx] = g;
+        const float w = wm - a.lr * g;
+        L.Wm[widx] = w;
+        L.Wc[(long long)(o0 + oo) * L.in_ld + (i0 + io)] = w;
+    } else if (own_b) {
+        float g = 0.f;
 #pragma unroll
-            for (int q = 0; q < kUpdCluster; ++q) g += Rb[q * kPerB + (tid - kPer)];
-            const int go = o0 + o;
-            L.gb[go] = g;
-            const float b = L.bm[go] - a.lr * g;
-            L.bm[go] = b;
-            L.bc[go] = b;
-        }
+        for (int q = 0; q < kUpdCluster; ++q) g += Rb[q * kPerB + (tid - kPer)];
+        const int go = o0 + ob;
+        L.gb[go] = g;
+        const float b = bmv - a.lr * g;
+        L.bm[go] = b;
+        L.bc[go] = b;
     }
 }
 

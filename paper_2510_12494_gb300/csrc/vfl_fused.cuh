@@ -91,6 +91,7 @@ struct FusedUpdLayer {
     const float* X; long long ldx;    // input columns [0, xsplit)
     const float* X2; long long ldx2;  // input columns [xsplit, in), indexed from 0
     int xsplit;
+    int x_early;                      // X is not written by the grid this launch depends on programmatically
     int tile0, tiles_i;               // first output tile of this layer, tiles along the input
     float* Wm; float* bm;             // fp32 master
     float* Wc; float* bc;             // the new version's copy

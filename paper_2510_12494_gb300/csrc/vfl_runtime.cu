@@ -926,6 +926,7 @@ vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float*
         const long long ldx = l == 0 ? ctx->ldxa : ld8(ctx->A[l - 1].out);
         u.L[n++] = fused_upd_layer(L, new_slot, w, ctx->dpre_a[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
     }
+    u.L[0].x_early = 1;   // x^a's rows: every other input comes from the active step's row kernel
     for (int l = 0; l < Lt; ++l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
@@ -987,6 +988,7 @@ vfl_status fused_passive_update(vfl_ctx* ctx, long long k, int slot, int rows, c
         const void* X = l == 0 ? (const void*)Xp : ctx->act_p[slot][l - 1];
         const long long ldx = l == 0 ? ctx->ldxp : ld8(ctx->P[l - 1].out);
         u.L[l] = fused_upd_layer(L, new_slot, w, ctx->dpre_p[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
+        u.L[l].x_early = 1;   // x^p's rows and the forward's activations: only D comes from the backward
     }
     u.nl = Lp;
     return launch_update(ctx, u, rows, s);
