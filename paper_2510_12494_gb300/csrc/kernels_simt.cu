@@ -182,16 +182,19 @@ __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__
 }
 
 // ---------------------------------------------------------------------------
-// Output layer + loss for the bf16 path (see HeadArgs).  256 threads, kHeadRows rows per block:
-// phase 1 gives warp w the rows w, w+8, ...; lane l holds inputs [8l, 8l+8) of a row.  Phase 2
-// gives thread t the inputs [8 (t mod 32), +8) of outputs j = t/32, t/32 + 8.
+// Output layer + loss for the bf16 path (see HeadArgs).  256 threads, kHeadRows rows per block.
+// Phase 0 stages W, the block's rows of h and their labels in shared memory with every load in
+// flight at once.  Phase 1 gives warp w the rows w, w+8, ...; lane l holds inputs [8l, 8l+8) of a
+// row, and W sits lane-minor (element (j, 8l+e) at (8j+e)*32 + l) so the warp's reads of it hit 32
+// banks.  Phase 2 gives thread t the inputs [8 (t mod 32), +8) of outputs j = t/32, t/32 + 8.
 constexpr int HEAD_NT = 256;
 static_assert(kHeadMaxK == 32 * 8 && kHeadMaxOut <= 2 * (HEAD_NT / 32), "head thread map");
 
 __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
-    __shared__ float Ws[kHeadMaxOut * kHeadMaxK];
+    __shared__ float Ws[kHeadMaxOut * kHeadMaxK];          // lane-minor: (j, 8l + e) at (8j + e) * 32 + l
     __shared__ __align__(16) __nv_bfloat16 hs[kHeadRows * kHeadMaxK];
     __shared__ float dss[kHeadRows * kHeadMaxOut];
+    __shared__ int ys[kHeadRows];
     __shared__ float wloss[HEAD_NT / 32];
     __shared__ bool last;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -199,19 +202,25 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
     const int r0 = blockIdx.x * kHeadRows, nr = min(kHeadRows, a.rows - r0);
     const float inv_b = 1.0f / (float)a.rows;
     const __nv_bfloat16* W = static_cast<const __nv_bfloat16*>(a.W);
+    const __nv_bfloat16* Hg = static_cast<const __nv_bfloat16*>(a.h);
+    // phase 0: W, the rows (zero past nr and past K) and the labels
     for (int i = tid; i < nout * K; i += HEAD_NT) {
         const int j = i / K, k = i - j * K;
-        Ws[j * kHeadMaxK + k] = __bfloat162float(W[(long long)j * a.ldw + k]);
+        Ws[(j * 8 + (k & 7)) * 32 + (k >> 3)] = __bfloat162float(W[(long long)j * a.ldw + k]);
     }
+    for (int i = tid; i < kHeadRows * (kHeadMaxK / 8); i += HEAD_NT) {
+        const int r = i >> 5, c = (i & 31) * 8;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r < nr && c < K) v = *reinterpret_cast<const uint4*>(Hg + (long long)(r0 + r) * a.ldh + c);
+        *reinterpret_cast<uint4*>(hs + r * kHeadMaxK + c) = v;
+    }
+    if (tid < kHeadRows) ys[tid] = tid < nr ? a.y[r0 + tid] : 0;
     __syncthreads();
     const bool kin = lane * 8 < K;
     float wl = 0.f;                                     // this warp's rows' loss, in row order
     for (int r = warp; r < kHeadRows; r += HEAD_NT / 32) {
         float hk[8];
-        uint4 raw = make_uint4(0u, 0u, 0u, 0u);
-        if (r < nr && kin)
-            raw = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.h) + (long long)(r0 + r) * a.ldh + lane * 8);
-        *reinterpret_cast<uint4*>(hs + r * kHeadMaxK + lane * 8) = raw;
+        const uint4 raw = *reinterpret_cast<const uint4*>(hs + r * kHeadMaxK + lane * 8);
         const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&raw);
 #pragma unroll
         for (int e = 0; e < 8; ++e) hk[e] = __bfloat162float(hb[e]);
@@ -220,9 +229,9 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         for (int j = 0; j < kHeadMaxOut; ++j) {
             if (j < nout) {
                 float p = 0.f;
-                const float* w = Ws + j * kHeadMaxK + lane * 8;
+                const float* w = Ws + j * kHeadMaxK + lane;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) p = fmaf(hk[e], kin ? w[e] : 0.f, p);
+                for (int e = 0; e < 8; ++e) p = fmaf(hk[e], kin ? w[e * 32] : 0.f, p);
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
                 sv[j] = p + a.b[j];
@@ -230,7 +239,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         }
         float li = 0.f;
         if (r < nr) {
-            const int yl = a.y[r0 + r];
+            const int yl = ys[r];
             if (a.loss == VFL_LOSS_BCE) {
                 const float x = sv[0];
                 li = fmaxf(x, 0.f) - x * (float)yl + log1pf(expf(-fabsf(x)));
@@ -281,7 +290,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
                 float g = 0.f;
 #pragma unroll
                 for (int j = 0; j < kHeadMaxOut; ++j)
-                    if (j < nout) g = fmaf(dv[j], Ws[j * kHeadMaxK + lane * 8 + e], g);
+                    if (j < nout) g = fmaf(dv[j], Ws[(j * 8 + e) * 32 + lane], g);
                 ob[e] = __float2bfloat16_rn(hk[e] > 0.f ? g : 0.f);
             }
             *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.dh) + (long long)(r0 + r) * a.lddh + lane * 8) =
