@@ -94,7 +94,7 @@ cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s);
 // block sums in block order (the last block to finish).
 constexpr int kHeadMaxOut = 12;
 constexpr int kHeadMaxK = 256;
-constexpr int kHeadRows = 64;
+constexpr int kHeadRows = 32;
 struct HeadArgs {
     const void* h; long long ldh;     // g's last hidden activation rows [rows, ldh], bf16
     const void* W; long long ldw;     // the output layer's version copy [n_out, ldw], bf16
