@@ -8,11 +8,12 @@ Pinned by ``tests/test_oracle_*.py``: Philox known-answer vectors and constant
 derivations, finite differences, the split = block-diagonal monolithic MLP
 invariant, zero staleness = synchronous SGD (against torch autograd on CPU),
 brute-force delayed SGD over every realisable schedule on tiny runs, closed
-forms (logistic regression, eta = 0, DP reductions) and bf16 rounding against
-torch's cast.  Parity unpinned: nothing.
+forms (logistic regression, eta = 0, DP reductions, the embedding mechanism's
+straight-through backward against torch autograd with the clip factor held
+constant) and bf16 rounding against torch's cast.  Parity unpinned: nothing.
 """
 from .vfl_oracle import (  # noqa: F401
-    PHILOX_M, PHILOX_W, TAG_DP, TAG_SCHED, SCHED_SYNC, SCHED_MAX, SCHED_SEEDED,
+    PHILOX_M, PHILOX_W, TAG_DP, TAG_DPE, TAG_SCHED, SCHED_SYNC, SCHED_MAX, SCHED_SEEDED,
     philox, make_schedule, bf16_round, mlp_forward, mlp_backward, loss_and_dlogits,
-    dp_normals, dp_clip_noise, Oracle, StepRecord,
+    dp_normals, dp_clip_noise, dp_embed, gdp_sigma, Oracle, StepRecord,
 )

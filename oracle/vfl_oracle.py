@@ -40,10 +40,19 @@ Readings where the paper is silent (each is listed in the design doc):
   clipped to L2 norm C and N(0, (sigma C)^2 I) noise is added, then divided by
   B_k again.  Noise: Philox4x32-10 with key (seed lo, seed hi) and counter
   (col // 4, row in batch, k, 0x4450); Box-Muller on 24-bit uniforms.
+* DP variant on the published embedding (App. C, the paper's own target): per
+  row c_i = min(1, C/||z_i||) (1 for a zero row) and the published embedding is
+  c_i z_i + sigma C xi_i, xi from the same generator with counter word 3 =
+  0x4445.  The backward is straight-through: the passive party scales the
+  received gradient by c_i (the Jacobian of c_i and of the noise are ignored)
+  before its own ReLU mask on the clean z.  sigma for a target mu-GDP level
+  follows Eq. 25 with the O(.)'s constant taken as 1.
 * bf16 presets round to bf16 (round-to-nearest-even, via fp32) at: the inputs,
   each weight version's compute copy (biases stay fp32), every stored hidden
   activation and embedding, and every activation gradient handed from one layer
-  to the next (including both published cut-layer gradients).  Logits, loss and
+  to the next (including both published cut-layer gradients, the noisy
+  published embedding and the scaled gradient the passive backward starts
+  from).  Logits, loss and
   d(logits) stay unrounded; master weights and weight gradients are never
   rounded.
 """
@@ -61,7 +70,8 @@ PHILOX_M = (0xD2511F53, 0xCD9E8D57)
 PHILOX_W = (0x9E3779B9, 0xBB67AE85)
 _U32 = 0xFFFFFFFF
 TAG_SCHED = 0x5343      # counter word 3 of the staleness-schedule draws
-TAG_DP = 0x4450         # counter word 3 of the DP noise draws
+TAG_DP = 0x4450         # counter word 3 of the DP noise draws on the published gradient
+TAG_DPE = 0x4445        # counter word 3 of the DP noise draws on the published embedding
 
 
 def philox(ctr, key):
@@ -205,15 +215,15 @@ def loss_and_dlogits(s, y, loss: str):
     return li.mean(), ds, li
 
 
-def dp_normals(seed: int, k: int, rows: int, cols: int):
+def dp_normals(seed: int, k: int, rows: int, cols: int, tag: int = TAG_DP):
     """N(0,1) draws xi[i, c] for the DP noise of step k (App. C, Assumption 5):
-    Philox4x32-10, key (seed lo, seed hi), counter (c // 4, i, k, TAG_DP); the
+    Philox4x32-10, key (seed lo, seed hi), counter (c // 4, i, k, tag); the
     block's words (x0, x1) give columns 4q, 4q+1 and (x2, x3) columns 4q+2,
     4q+3 by Box-Muller with u1 = ((x >> 8) + 1) 2^-24, u2 = (y >> 8) 2^-24."""
     nq = (cols + 3) // 4
     q = np.arange(nq, dtype=np.uint64)[None, :]
     i = np.arange(rows, dtype=np.uint64)[:, None]
-    x = philox((q, i, np.uint64(k & _U32), np.uint64(TAG_DP)), (seed & _U32, (seed >> 32) & _U32))
+    x = philox((q, i, np.uint64(k & _U32), np.uint64(tag)), (seed & _U32, (seed >> 32) & _U32))
     out = np.empty((rows, nq, 4))
     for pair in (0, 1):
         a, b = x[2 * pair], x[2 * pair + 1]
@@ -238,6 +248,26 @@ def dp_clip_noise(dz, k: int, clip: float, sigma: float, seed: int):
     if sigma != 0.0:
         g = g + sigma * clip * dp_normals(seed, k, B, dz.shape[1])
     return g / B
+
+
+def dp_embed(z, k: int, clip: float, sigma: float, seed: int):
+    """Gaussian mechanism on the published embedding (App. C): per row
+    c_i = min(1, C/||z_i||) (1 for a zero row), z~_i = c_i z_i + sigma C xi_i.
+    Returns (z~, c)."""
+    norm = np.sqrt((z * z).sum(axis=1))
+    with np.errstate(divide="ignore", invalid="ignore"):
+        c = np.where(norm > clip, clip / norm, 1.0)
+    out = z * c[:, None]
+    if sigma != 0.0:
+        out = out + sigma * clip * dp_normals(seed, k, z.shape[0], z.shape[1], TAG_DPE)
+    return out, c
+
+
+def gdp_sigma(mu: float, batch: int, n: int, queries: int) -> float:
+    """Noise multiplier for mu-GDP on the published embedding, Eq. 25 with the
+    O(.)'s constant taken as 1: sigma = N_m sqrt(K) / (mu N), N_m the minibatch
+    size, N the whole dataset, K the number of batches the worker processes."""
+    return batch * math.sqrt(queries) / (mu * n)
 
 
 # ---------------------------------------------------------------------------
@@ -284,6 +314,7 @@ class Oracle:
     versions_a: dict = field(default_factory=dict)
     channel_e: dict = field(default_factory=dict)
     channel_g: dict = field(default_factory=dict)
+    emb_scale: dict = field(default_factory=dict)   # step -> per-row clip factors of its published embedding
 
     def __post_init__(self):
         c = self.cfg
@@ -322,7 +353,13 @@ class Oracle:
         # Publisher phase (passive): z^p = f_p(x^p; theta_2^(k - tau_p)), publish to C_e[B_j].
         P = self._compute(self.versions_p[vp])
         hp = mlp_forward(P, self.xp_c[r0:r1], True, self.dtype)
-        self.channel_e[k] = (hp[-1], j, vp)
+        emb_dp = c.dp_clip > 0.0 and getattr(c, "dp_target", "grad") == "emb"
+        if emb_dp:   # App. C: Gaussian noise on the published embedding
+            zpub, self.emb_scale[k] = dp_embed(hp[-1], k, c.dp_clip, c.dp_sigma, self.dp_seed)
+            zpub = _store(zpub, self.dtype)
+        else:
+            zpub = hp[-1]
+        self.channel_e[k] = (zpub, j, vp)
 
         # Subscriber phase (active): fetch z^p, z^a = f_a(x^a), y_hat = g(z^a, z^p),
         # loss, grads wrt theta_1 and z^p; publish grad to C_g[B_j].
@@ -338,7 +375,7 @@ class Oracle:
         ea = ha[-1].shape[1]
         dza = _store(dtop[:, :ea], self.dtype)
         dzp = dtop[:, ea:]
-        if c.dp_clip > 0.0:
+        if c.dp_clip > 0.0 and not emb_dp:
             dzp = dp_clip_noise(dzp, k, c.dp_clip, c.dp_sigma, self.dp_seed)
         dzp = _store(dzp, self.dtype)
         gA, _ = mlp_backward(A, ha, dza, True, self.dtype, need_dx=False)
@@ -348,7 +385,9 @@ class Oracle:
         # passive version with the saved activations.
         dzp_f, j_g, _ = self.channel_g.pop(k)
         assert j_g == j
-        gP, _ = mlp_backward(P, hp, dzp_f, True, self.dtype, need_dx=False)
+        # straight-through backward of the embedding mechanism: scale by c_i, ignore its Jacobian
+        dzp_in = _store(self.emb_scale.pop(k)[:, None] * dzp_f, self.dtype) if emb_dp else dzp_f
+        gP, _ = mlp_backward(P, hp, dzp_in, True, self.dtype, need_dx=False)
 
         # Gradient descent (Eq. 2) in the delayed form of App. D:
         # theta^(k+1) = theta^(k) - eta * g evaluated at theta^(k - tau).

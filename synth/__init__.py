@@ -135,9 +135,10 @@ class VflPreset:
     schedule: str           # "sync" | "seeded"
     dtype: str              # "fp32" | "bf16"
     workers: int            # worker streams per party
-    dp_clip: float = 0.0    # > 0 enables DP on the published embedding gradient
+    dp_clip: float = 0.0    # > 0 enables DP on the exchanged tensor named by dp_target
     dp_sigma: float = 0.0
     seed: int = 0
+    dp_target: str = "grad" # "grad": the published embedding gradient; "emb": the published embedding
 
     @property
     def n_out(self) -> int:
