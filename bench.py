@@ -43,6 +43,10 @@ def parse():
     ap.add_argument("--config", type=int, default=2, help="workload preset 1..5 (default 2, credit-shaped)")
     ap.add_argument("--rows", type=int, default=0, help="override the preset's row count")
     ap.add_argument("--workers", type=int, default=0, help="override the preset's worker streams per party")
+    ap.add_argument("--dp-target", choices=["grad", "emb"], default=None,
+                    help="with DP: the published gradient (the preset's) or the published embedding (App. C)")
+    ap.add_argument("--dp", type=float, nargs=2, default=None, metavar=("CLIP", "SIGMA"),
+                    help="enable DP with this clip norm and noise multiplier")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -58,12 +62,18 @@ def workload(args):
         p = p.with_(n_rows=args.rows)
     if args.workers:
         p = p.with_(workers=args.workers)
+    if args.dp:
+        p = p.with_(dp_clip=args.dp[0], dp_sigma=args.dp[1])
+    if args.dp_target:
+        p = p.with_(dp_target=args.dp_target)
     desc = (f"{p.name}: N={p.n_rows}, d_p/d_a={p.d_passive}/{p.d_active}, "
             f"passive {'-'.join(map(str, (p.d_passive,) + p.passive))}, "
             f"active {'-'.join(map(str, (p.d_active,) + p.active))}, "
             f"top {'-'.join(map(str, (p.e_active + p.e_passive,) + p.top))} {p.loss.upper()}, "
             f"B={p.batch}, S={p.staleness} ({p.schedule} schedule), {p.dtype}, "
-            f"{p.workers} worker stream(s) per party" + (f", DP C={p.dp_clip} sigma={p.dp_sigma}" if p.dp_clip else ""))
+            f"{p.workers} worker stream(s) per party" +
+            (f", DP on the {'embedding' if p.dp_target == 'emb' else 'embedding gradient'} C={p.dp_clip} "
+             f"sigma={p.dp_sigma}" if p.dp_clip else ""))
     return p, desc
 
 

@@ -51,6 +51,9 @@ typedef int32_t vfl_status;
 #define VFL_FP32 0        /* fp32 storage and arithmetic                               */
 #define VFL_BF16 1        /* bf16 weights copies / activations, fp32 accumulate+master */
 
+#define VFL_DP_GRAD 0     /* DP on the published embedding gradient dLoss/dz^p          */
+#define VFL_DP_EMB 1      /* DP on the published embedding z^p (App. C)                 */
+
 #define VFL_SCHED_SYNC 0  /* tau = 0                                                    */
 #define VFL_SCHED_MAX 1   /* tau(k) = min(k, S)                                         */
 #define VFL_SCHED_SEEDED 2
@@ -75,10 +78,30 @@ typedef struct vfl_config {
     float lr;                               /* SGD step size eta (Eq. 2)                 */
     int32_t staleness;                      /* bound S on tau; channels hold S+1 slots   */
     int32_t workers;                        /* worker streams per party (1..16)          */
-    float dp_clip;                          /* > 0 enables DP on the published gradient  */
+    float dp_clip;                          /* > 0 enables DP on the tensor dp_target names */
     float dp_sigma;                         /* noise multiplier; noise std = sigma * clip */
     uint64_t dp_seed;                       /* Philox key of the DP noise                */
+    int32_t dp_target;                      /* VFL_DP_GRAD | VFL_DP_EMB (see below)       */
 } vfl_config;
+
+/*
+ * DP mechanisms (App. C), both per row of the batch, with N(0,1) draws from
+ * Philox4x32-10 keyed by dp_seed (counter (col / 4, row, k, tag), Box-Muller):
+ *  - VFL_DP_GRAD: the published gradient, g_i = B_k dz_i clipped to L2 norm C,
+ *    plus sigma C xi_i, divided by B_k (tag 0x4450);
+ *  - VFL_DP_EMB: the published embedding, c_i = min(1, C / ||z_i||) (1 for a
+ *    zero row), published c_i z_i + sigma C xi_i (tag 0x4445); the passive
+ *    backward scales the gradient it receives by c_i before its ReLU mask on
+ *    the clean z (straight-through: the Jacobians of c_i and the noise are
+ *    ignored).
+ * Either sends the model through the per-layer kernels.
+ */
+
+/* Noise multiplier for mu-GDP on the published embedding, Eq. 25 with the O(.)
+ * constant taken as 1: sigma = batch sqrt(queries) / (mu n_rows), queries = the
+ * batches the worker processes.  VFL_E_INVAL unless mu > 0, batch >= 1,
+ * n_rows >= 1 and queries >= 1. */
+vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queries, double* sigma);
 
 typedef struct vfl_ctx vfl_ctx;
 

@@ -20,6 +20,7 @@ VFL_OK, VFL_E_INVAL, VFL_E_OOM, VFL_E_CUDA, VFL_E_STATE, VFL_E_VERSION, VFL_E_TI
 MAX_LAYERS = 8
 LOSS_BCE, LOSS_CE = 0, 1
 FP32, BF16 = 0, 1
+DP_GRAD, DP_EMB = 0, 1
 SCHED_SYNC, SCHED_MAX, SCHED_SEEDED = 0, 1, 2
 TAP_EMB, TAP_GRAD, TAP_LOGITS, TAP_ZA, TAP_DZA = range(5)
 PASSIVE, ACTIVE, TOP = 0, 1, 2
@@ -44,6 +45,7 @@ class VflConfig(ctypes.Structure):
         ("loss", ctypes.c_int32), ("dtype", ctypes.c_int32), ("batch", ctypes.c_int32),
         ("lr", ctypes.c_float), ("staleness", ctypes.c_int32), ("workers", ctypes.c_int32),
         ("dp_clip", ctypes.c_float), ("dp_sigma", ctypes.c_float), ("dp_seed", ctypes.c_uint64),
+        ("dp_target", ctypes.c_int32),
     ]
 
 
@@ -71,6 +73,8 @@ EXPORTS = {
     "vfl_set_cursor": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
     "vfl_set_version": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
                                          ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_gdp_sigma": (ctypes.c_int32, [ctypes.c_double, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                       ctypes.POINTER(ctypes.c_double)]),
     "vfl_make_schedule": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
                                            ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_passive_forward": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32]),
@@ -148,7 +152,15 @@ def make_config(p) -> VflConfig:
     c.dp_clip = p.dp_clip
     c.dp_sigma = p.dp_sigma
     c.dp_seed = getattr(p, "dp_seed", getattr(p, "seed", 0))
+    c.dp_target = DP_EMB if getattr(p, "dp_target", "grad") == "emb" else DP_GRAD
     return c
+
+
+def gdp_sigma(mu: float, batch: int, n_rows: int, queries: int) -> float:
+    """Noise multiplier for mu-GDP on the published embedding (Eq. 25, see vfl_gdp_sigma)."""
+    out = ctypes.c_double()
+    _check(lib().vfl_gdp_sigma(mu, batch, n_rows, queries, ctypes.byref(out)))
+    return out.value
 
 
 def make_schedule(seed: int, S: int, kind: int, n_steps: int):

@@ -26,6 +26,7 @@
 #include <cooperative_groups.h>
 
 #include "vfl_fused.cuh"
+#include "vfl_philox.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -344,6 +345,32 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
             tile_fwd(cur, ld, L.in, ws + L.ws_off, L.ws_ld, staged_bias(ws, L), L.out, L.fmap, nxt,
                      L.Y + (long long)r0 * L.ldy, L.ldy, nr, red);
             cur = nxt;
+        }
+        if (a.dp_out) {
+            // DP on the published embedding: warp r takes row r of the tile (the clean z stays in L.Y)
+            __syncthreads();
+            const int r = threadIdx.x >> 5, lane = threadIdx.x & 31;
+            const int e = a.L[a.nl - 1].out;
+            if (r < nr) {
+                const float* zr = cur + r * ld;
+                float ss = 0.f;
+                for (int c = lane; c < e; c += 32) ss = fmaf(zr[c], zr[c], ss);
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+                const float norm = sqrtf(ss);
+                const float f = norm > a.dp_clip ? a.dp_clip / norm : 1.0f;
+                if (lane == 0) a.dp_scale[r0 + r] = f;
+                const float noise = a.dp_sigma * a.dp_clip;
+                const uint2 key = make_uint2((unsigned)(a.dp_seed & 0xFFFFFFFFull), (unsigned)(a.dp_seed >> 32));
+                float* out = a.dp_out + (long long)(r0 + r) * a.ld_dp;
+                for (int q = lane; 4 * q < e; q += 32) {
+                    float xi[4] = {0.f, 0.f, 0.f, 0.f};
+                    if (noise != 0.f) dp_normals4(q, r0 + r, a.k, 0x4445u, key, xi);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        if (4 * q + j < e) out[4 * q + j] = fmaf(zr[4 * q + j], f, noise * xi[j]);
+                }
+            }
         }
         first = false;
     }
@@ -675,12 +702,14 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
         cp_wait_pending(0);
         {                                                                // dz^p * [z^p > 0]
             const int r = threadIdx.x >> 5;
+            // DP on the embedding: the straight-through backward scales the received gradient by c
+            const float sc = a.rowscale && r < nr ? a.rowscale[r0 + r] : 1.0f;
             const float* zp = slot(Lp - 1);
             float* dg = P[Lp - 1].D + (long long)(r0 + r) * P[Lp - 1].ldd;
             for (int c = (threadIdx.x & 31) * 2; c < ep8; c += 64) {
                 const float2 z = *reinterpret_cast<const float2*>(zp + r * ld + c);
                 const float2 gr = *reinterpret_cast<const float2*>(gs + r * ld + c);
-                const float2 v = make_float2(z.x > 0.f ? gr.x : 0.f, z.y > 0.f ? gr.y : 0.f);
+                const float2 v = make_float2(z.x > 0.f ? sc * gr.x : 0.f, z.y > 0.f ? sc * gr.y : 0.f);
                 *reinterpret_cast<float2*>(G0 + r * ld + c) = v;
                 if (r < nr) *reinterpret_cast<float2*>(dg + c) = v;
             }

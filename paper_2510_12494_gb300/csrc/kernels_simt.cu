@@ -2,6 +2,7 @@
 // for narrow layers, the fused loss, DP clip+noise, ReLU mask, fused SGD,
 // channel headers and data casts.
 #include "vfl_kernels.cuh"
+#include "vfl_philox.cuh"
 
 namespace vfl {
 
@@ -20,20 +21,6 @@ __device__ __forceinline__ void stf(void* base, long long idx, int bf16, float v
 __device__ __forceinline__ float ldany(const void* base, long long idx, int bf16) {
     return bf16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(base)[idx])
                 : static_cast<const float*>(base)[idx];
-}
-
-// Philox4x32-10 (Salmon et al., SC'11): ten rounds of two 32x32->64 products,
-// key bumped by the Weyl increments between rounds.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 key) {
-#pragma unroll
-    for (int r = 0; r < 10; ++r) {
-        const unsigned lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
-        const unsigned lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-        c = make_uint4(hi1 ^ c.y ^ key.x, lo1, hi0 ^ c.w ^ key.y, lo0);
-        key.x += 0x9E3779B9u;
-        key.y += 0xBB67AE85u;
-    }
-    return c;
 }
 
 constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
@@ -380,19 +367,8 @@ __global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in,
     const uint2 key = make_uint2((unsigned)(seed & 0xFFFFFFFFull), (unsigned)(seed >> 32));
     const float scale = sigma * clip;
     for (int q = threadIdx.x; q * 4 < e; q += DP_NT) {
-        const uint4 w = philox4x32_10(make_uint4((unsigned)q, (unsigned)r, (unsigned)(k & 0xFFFFFFFFll), 0x4450u), key);
-        const unsigned xs[4] = {w.x, w.y, w.z, w.w};
         float z[4];
-#pragma unroll
-        for (int p = 0; p < 2; ++p) {
-            const float u1 = (float)((xs[2 * p] >> 8) + 1u) * 0x1p-24f;
-            const float u2 = (float)(xs[2 * p + 1] >> 8) * 0x1p-24f;
-            const float rad = sqrtf(-2.0f * logf(u1));
-            float sn, cs;
-            sincospif(2.0f * u2, &sn, &cs);
-            z[2 * p] = rad * cs;
-            z[2 * p + 1] = rad * sn;
-        }
+        dp_normals4(q, r, k, 0x4450u, key, z);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int c = 4 * q + j;
@@ -405,14 +381,56 @@ __global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in,
     }
 }
 
+// DP on the published embedding (App. C): per row c = min(1, C / ||z||) (1 for a zero row), the
+// payload c z + sigma C N(0,1) (tag 0x4445) in the compute dtype, and c kept for the backward.
+__global__ void __launch_bounds__(DP_NT) dp_emb_kernel(const void* z, long long ld, int bf16, void* out,
+                                                        float* __restrict__ scale_out, int e, float clip, float sigma,
+                                                        unsigned long long seed, long long k) {
+    __shared__ float red[DP_NT / 32];
+    __shared__ float s_factor;
+    const int r = blockIdx.x;
+    const long long base = (long long)r * ld;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < e; c += DP_NT) {
+        const float v = ldany(z, base + c, bf16);
+        ss = fmaf(v, v, ss);
+    }
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_down_sync(0xffffffffu, ss, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float v = threadIdx.x < DP_NT / 32 ? red[threadIdx.x] : 0.f;
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+        if (threadIdx.x == 0) {
+            const float norm = sqrtf(v);
+            s_factor = norm > clip ? clip / norm : 1.0f;
+            scale_out[r] = s_factor;
+        }
+    }
+    __syncthreads();
+    const float factor = s_factor;
+    const uint2 key = make_uint2((unsigned)(seed & 0xFFFFFFFFull), (unsigned)(seed >> 32));
+    const float noise = sigma * clip;
+    for (int q = threadIdx.x; q * 4 < e; q += DP_NT) {
+        float xi[4] = {0.f, 0.f, 0.f, 0.f};
+        if (noise != 0.f) dp_normals4(q, r, k, 0x4445u, key, xi);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int c = 4 * q + j;
+            if (c < e) stf(out, base + c, bf16, fmaf(ldany(z, base + c, bf16), factor, noise * xi[j]));
+        }
+    }
+}
+
+// out = g * [z > 0], with g first scaled by rs[row] when rs is given (rounded to T)
 template <typename T>
 __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ z, T* __restrict__ out,
-                                 long long ld, int rows, int e) {
+                                 long long ld, int rows, int e, const float* __restrict__ rs) {
     const long long n = (long long)rows * e;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
         const long long r = i / e, c = i % e;
         const long long idx = r * ld + c;
-        out[idx] = ldf(z + idx) > 0.f ? g[idx] : T(0.f);
+        out[idx] = ldf(z + idx) > 0.f ? (rs ? T(rs[r] * ldf(g + idx)) : g[idx]) : T(0.f);
     }
 }
 
@@ -596,15 +614,22 @@ cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_
 }
 
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
-                             cudaStream_t s) {
+                             const float* row_scale, cudaStream_t s) {
     const int nb = grid_for((long long)rows * e, 256);
     if (bf16)
         relu_mask_kernel<__nv_bfloat16><<<nb, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(g),
                                                            static_cast<const __nv_bfloat16*>(z),
-                                                           static_cast<__nv_bfloat16*>(out), ld, rows, e);
+                                                           static_cast<__nv_bfloat16*>(out), ld, rows, e, row_scale);
     else
         relu_mask_kernel<float><<<nb, 256, 0, s>>>(static_cast<const float*>(g), static_cast<const float*>(z),
-                                                   static_cast<float*>(out), ld, rows, e);
+                                                   static_cast<float*>(out), ld, rows, e, row_scale);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, float* scale_out, int rows, int e,
+                          float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    dp_emb_kernel<<<rows, DP_NT, 0, s>>>(z, ld, bf16, out, scale_out, e, clip, sigma, seed, k);
     return cudaGetLastError();
 }
 

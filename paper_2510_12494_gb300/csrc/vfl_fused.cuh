@@ -57,6 +57,12 @@ struct FusedChainArgs {
     int rows, act_ld, w_floats;
     ChannelHeader* hdr;
     long long k; int batch, version;
+    // DP on the published embedding (App. C), when dp_out is set: per row c = min(1, C / ||z||), the
+    // payload c z + sigma C N(0,1) (Philox tag 0x4445) to dp_out, c to dp_scale
+    float* dp_out; long long ld_dp;
+    float* dp_scale;
+    float dp_clip, dp_sigma;
+    unsigned long long dp_seed;
 };
 
 // Row-parallel part of the active step (L[0..na) = f_a, L[na..na+nt) = g) or of
@@ -77,6 +83,7 @@ struct FusedStepArgs {
     ChannelHeader* pub_hdr;             // header to publish (active: gradient channel)
     long long k; int batch, version;
     int* status;
+    const float* rowscale;              // passive, DP on the embedding: the rows' clip factors (else null)
 };
 
 // Weight gradient + SGD of a set of layers: dW = D^T X and db = column sums of D

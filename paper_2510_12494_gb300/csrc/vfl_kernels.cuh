@@ -62,9 +62,15 @@ cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, 
 cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_out, int out_bf16, int rows,
                       int e, float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s);
 
-// out[r, c] = g[r, c] * (z[r, c] > 0), compute dtype, [rows, e] with leading dim ld.
+// DP on the published embedding (one block per row): z and out in the compute dtype [rows, e] (ld),
+// out = c z + sigma clip N(0,1) with c = min(1, clip / ||z||) per row, written to scale_out[rows].
+cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, float* scale_out, int rows, int e,
+                          float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s);
+
+// out[r, c] = g[r, c] * (z[r, c] > 0), compute dtype, [rows, e] with leading dim ld; with row_scale,
+// g[r, c] is first multiplied by row_scale[r] (and rounded to the compute dtype).
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
-                             cudaStream_t s);
+                             const float* row_scale, cudaStream_t s);
 
 struct SgdLayer {
     float* W; float* b;           // fp32 master

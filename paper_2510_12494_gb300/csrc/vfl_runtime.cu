@@ -12,6 +12,7 @@
 //    computed with weights of version k - tau(k); updates apply in step order.
 //    Each party keeps its S+1 most recent weight versions in a ring.
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <map>
 #include <utility>
@@ -117,6 +118,8 @@ struct vfl_ctx {
     float* ds[kMaxWorkers] = {};
     float* dzp32[kMaxWorkers] = {};
     void* grad[kMaxSlots] = {};
+    void* emb_pub[kMaxSlots] = {};      // DP on the embedding: the published (noisy) payload per slot
+    float* emb_c[kMaxSlots] = {};       // and its per-row clip factors [B], for the passive backward
     ChannelHeader* emb_hdr = nullptr;   // [S1]
     ChannelHeader* grad_hdr = nullptr;  // [S1]
     float* losses = nullptr;            // [kLossCap]
@@ -341,6 +344,7 @@ vfl_status check_config(const vfl_config* c, long long n_rows, std::string* why)
     if (c->staleness + 1 + c->workers + 2 > kEvPool) return bad("staleness + workers too large");
     if (!(c->lr >= 0.f)) return bad("lr must be >= 0");
     if (c->dp_clip < 0.f || c->dp_sigma < 0.f) return bad("dp_clip / dp_sigma must be >= 0");
+    if (c->dp_target != VFL_DP_GRAD && c->dp_target != VFL_DP_EMB) return bad("unknown dp_target");
     if (c->n_active + c->n_top > kMaxSgdLayers || c->n_passive > kMaxSgdLayers) return bad("too many layers");
     (void)buf;
     return VFL_OK;
@@ -359,7 +363,7 @@ void choose_split(Layer& L, int B) {
 // The fused path serves fp32 models whose every width fits one shared-memory
 // row tile, without DP.
 bool fused_eligible(const vfl_config& c) {
-    if (c.dtype != VFL_FP32 || c.dp_clip > 0.f) return false;
+    if (c.dtype != VFL_FP32 || (c.dp_clip > 0.f && c.dp_target != VFL_DP_EMB)) return false;
     if (c.d_passive > kFusedMaxWidth || c.d_active > kFusedMaxWidth) return false;
     for (int i = 0; i < c.n_passive; ++i) if (c.passive_out[i] > kFusedMaxWidth) return false;
     for (int i = 0; i < c.n_active; ++i) if (c.active_out[i] > kFusedMaxWidth) return false;
@@ -498,6 +502,10 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
         ctx->act_p[s].clear();
         for (const Layer& L : ctx->P) ctx->act_p[s].push_back(cv.take(B * ld8(L.out) * es));
         ctx->grad[s] = cv.take(B * ld8(ctx->P.back().out) * es);
+        if (c.dp_clip > 0.f && c.dp_target == VFL_DP_EMB) {
+            ctx->emb_pub[s] = cv.take(B * ld8(ctx->P.back().out) * es);
+            ctx->emb_c[s] = static_cast<float*>(cv.take(B * 4ull));
+        }
     }
     const int n_out = ctx->T.back().out;
     for (int w = 0; w < ctx->W; ++w) {
@@ -554,6 +562,9 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
 }
 
 inline cudaStream_t pstream(vfl_ctx* ctx, long long k) { return ctx->ps[k % ctx->W]; }
+
+// DP on the published embedding (App. C) rather than on its gradient
+inline bool emb_dp(const vfl_ctx* ctx) { return ctx->cfg.dp_clip > 0.f && ctx->cfg.dp_target == VFL_DP_EMB; }
 
 // Rows of step k (first row r0): the staging ring's slot when host data is bound, else the
 // device-resident dataset.  Both have the same row strides.
@@ -848,6 +859,14 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     a.act_ld = ctx->f_act_ld;
     a.w_floats = fused_weight_layout(a.L, a.nl, 0);
     a.hdr = ctx->emb_hdr + slot;
+    if (emb_dp(ctx)) {
+        a.dp_out = static_cast<float*>(ctx->emb_pub[slot]);
+        a.ld_dp = ld8(ctx->P.back().out);
+        a.dp_scale = ctx->emb_c[slot];
+        a.dp_clip = ctx->cfg.dp_clip;
+        a.dp_sigma = ctx->cfg.dp_sigma;
+        a.dp_seed = ctx->cfg.dp_seed;
+    }
     a.k = k;
     a.batch = (int)(k % ctx->nb);
     a.version = (int)v;
@@ -888,7 +907,7 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     ctx->batch_rows(k, &r0);
     a.y = y_rows(ctx, k, r0);
     a.loss = ctx->cfg.loss;
-    a.zp = static_cast<const float*>(ctx->act_p[slot].back());
+    a.zp = static_cast<const float*>(emb_dp(ctx) ? ctx->emb_pub[slot] : ctx->act_p[slot].back());
     a.ldzp = ld8(ep);
     a.zpc = ctx->f_zpc[w];
     a.ldzpc = ld8(ep);
@@ -964,6 +983,7 @@ vfl_status fused_passive_backward(vfl_ctx* ctx, long long k, int slot, int vslot
     a.chk_hdr = ctx->grad_hdr + slot;
     a.k = k;
     a.status = ctx->status;
+    a.rowscale = emb_dp(ctx) ? ctx->emb_c[slot] : nullptr;
     // algorithmic bytes: dz^p and the saved activations in, every d(pre) out, weights after the first read once
     double bytes = (double)rows * ctx->P.back().out * 4;
     for (size_t l = 0; l < ctx->P.size(); ++l) {
@@ -1059,6 +1079,12 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
         X = Y;
         ldx = ld8(L.out);
     }
+    if (emb_dp(ctx)) {   // App. C: the published embedding is clipped and noised; z stays for the backward
+        const int ep = ctx->P.back().out;
+        PLAUNCH(K_DP, 0, (double)rows * ep * 2 * ctx->esz + rows * 4.0, s,
+                launch_dp_emb(ctx->act_p[slot].back(), ld8(ep), ctx->bf16, ctx->emb_pub[slot], ctx->emb_c[slot], rows,
+                              ep, c.dp_clip, c.dp_sigma, c.dp_seed, k, s));
+    }
     PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)(k % ctx->nb), (int)v, s));
     CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
     ctx->fwd_version[slot] = (int)v;
@@ -1116,7 +1142,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
     PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->emb_hdr + slot, k, ctx->status, s));
     const void* Za = ctx->act_a[w][La - 1];
-    const void* Zp = ctx->act_p[slot][Lp - 1];
+    const void* Zp = emb_dp(ctx) ? ctx->emb_pub[slot] : ctx->act_p[slot][Lp - 1];
     // top forward on [z^a | z^p]; with the head kernel, g's output layer runs with the loss
     const int Lf = ctx->head ? Lt - 1 : Lt;
     for (int l = 0; l < Lf; ++l) {
@@ -1160,7 +1186,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
                             ctx->losses + (k % kLossCap), loss_host(ctx, k), s));
     }
     // top backward (the head kernel has done the output layer's part)
-    const bool dp = c.dp_clip > 0.f;
+    const bool dp = c.dp_clip > 0.f && c.dp_target == VFL_DP_GRAD;
     for (int l = Lf - 1; l >= 0; --l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
@@ -1236,10 +1262,11 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
         return VFL_OK;
     }
     PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->grad_hdr + slot, k, ctx->status, s));
-    // dpre of the cut layer = dLoss/dz^p * [z^p > 0]
+    // dpre of the cut layer = dLoss/dz^p * [z^p > 0]; with DP on the embedding the received gradient is
+    // first scaled by the row's clip factor (straight-through backward of the mechanism)
     PLAUNCH(K_MASK, 0, 3.0 * rows * ep * ctx->esz, s,
             launch_relu_mask(ctx->grad[slot], ctx->act_p[slot][Lp - 1], ctx->dpre_p[w][Lp - 1], ld8(ep), rows, ep,
-                             ctx->bf16, s));
+                             ctx->bf16, emb_dp(ctx) ? ctx->emb_c[slot] : nullptr, s));
     const void* Xp0 = xp_rows(ctx, k, r0);
     for (int l = Lp - 1; l >= 0; --l) {
         const Layer& L = ctx->P[l];
@@ -1654,6 +1681,12 @@ vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
     return VFL_OK;
 }
 
+vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queries, double* sigma) {
+    if (!sigma || !(mu > 0.0) || batch < 1 || n_rows < 1 || queries < 1) return VFL_E_INVAL;
+    *sigma = (double)batch * std::sqrt((double)queries) / (mu * (double)n_rows);
+    return VFL_OK;
+}
+
 vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_steps, int32_t* tau_p,
                              int32_t* tau_a) {
     if (S < 0 || n_steps < 0 || (n_steps > 0 && (!tau_p || !tau_a))) {
@@ -1932,7 +1965,7 @@ vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out) {
     switch (what) {
         case VFL_TAP_EMB:
             if (ctx->slot_step_p[slot] != k) return ctx->fail(VFL_E_STATE, "embedding of step %lld is not stored", (long long)k);
-            src = ctx->act_p[slot].back(); ld = ld8(ep); cols = ep;
+            src = emb_dp(ctx) ? ctx->emb_pub[slot] : ctx->act_p[slot].back(); ld = ld8(ep); cols = ep;
             break;
         case VFL_TAP_GRAD:
             if (ctx->grad_step[slot] != k) return ctx->fail(VFL_E_STATE, "gradient of step %lld is not stored", (long long)k);

@@ -38,9 +38,11 @@ def test_library_exports_every_declared_function(vfl):
 
 
 def test_config_struct_layout_matches_header(vfl):
-    # 5 + 3*8 int32, then loss, dtype, batch, lr, staleness, workers, clip, sigma (4 bytes each), then u64
-    assert ctypes.sizeof(vfl.VflConfig) == (5 + 24 + 8) * 4 + 4 + 8
+    # 5 + 3*8 int32, then loss, dtype, batch, lr, staleness, workers, clip, sigma (4 bytes each), then u64,
+    # then the int32 dp_target and 4 bytes of tail padding
+    assert ctypes.sizeof(vfl.VflConfig) == (5 + 24 + 8) * 4 + 4 + 8 + 8
     assert vfl.VflConfig.dp_seed.offset % 8 == 0
+    assert vfl.VflConfig.dp_target.offset == vfl.VflConfig.dp_seed.offset + 8
 
 
 @pytest.mark.parametrize("S", [0, 1, 2, 4, 7])
@@ -70,6 +72,14 @@ def test_workspace_sizes(vfl, cid):
     assert b < 64 * 2 ** 30
 
 
+def test_gdp_sigma_matches_the_oracle(vfl):
+    import oracle
+    for args in ((1.0, 1024, 30000, 150), (0.25, 256, 4096, 16), (3.0, 8192, 1000000, 123)):
+        assert vfl.gdp_sigma(*args) == pytest.approx(oracle.gdp_sigma(*args), rel=1e-15)
+    with pytest.raises(vfl.VflError):
+        vfl.gdp_sigma(0.0, 1024, 30000, 150)
+
+
 def test_invalid_configs_are_rejected(vfl):
     p = synth.preset(1)
     for bad in (dict(batch=0), dict(staleness=-1), dict(staleness=40), dict(workers=0), dict(workers=17),
@@ -78,3 +88,8 @@ def test_invalid_configs_are_rejected(vfl):
             vfl.workspace_bytes(p.with_(**bad), 100)
     with pytest.raises(vfl.VflError):
         vfl.workspace_bytes(p, 0)
+    cfg = vfl.make_config(p.with_(dp_clip=1.0, dp_target="emb"))
+    assert cfg.dp_target == vfl.DP_EMB
+    cfg.dp_target = 7
+    out = ctypes.c_uint64()
+    assert vfl.lib().vfl_workspace_bytes(ctypes.byref(cfg), 100, ctypes.byref(out)) == vfl.VFL_E_INVAL
