@@ -37,7 +37,7 @@ TF32_PER_BF16 = 1.1 / 2.25                               # nominal dense TF32 / 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=150)
+    ap.add_argument("--steps", type=int, default=1500)
     ap.add_argument("--warmup", type=int, default=30)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2, help="workload preset 1..5 (default 2, credit-shaped)")
@@ -146,8 +146,7 @@ CPU_SNIPPET = r"""
 import sys, time, json, os
 sys.path.insert(0, {root!r})
 import numpy as np, synth, oracle
-p = synth.preset({cid})
-if {rows}: p = p.with_(n_rows={rows})
+p = synth.VflPreset(**{fields!r})      # the workload exactly as the GPU arm runs it
 n_steps = {n_steps}
 nb = p.steps_per_epoch
 last = min(n_steps, nb) * p.batch
@@ -175,8 +174,8 @@ def run_oracle(p, args, n_steps, budget):
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         env[v] = str(cores)
     env["CUDA_VISIBLE_DEVICES"] = ""
-    code = CPU_SNIPPET.format(root=ROOT, cid=p.cid, rows=args.rows, n_steps=n_steps, kind=sched_kind(p),
-                              budget=budget)
+    fields = {f: getattr(p, f) for f in p.__dataclass_fields__}
+    code = CPU_SNIPPET.format(root=ROOT, fields=fields, n_steps=n_steps, kind=sched_kind(p), budget=budget)
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle timing failed: {r.stderr[-2000:]}")
