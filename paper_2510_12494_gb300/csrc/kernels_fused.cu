@@ -395,7 +395,8 @@ __device__ __forceinline__ float loss_row(const float* s, int nout, int y, int l
     return logf(z) + m - s[y];
 }
 
-// g's last hidden layer Lh (input X) with the output layer Lo (n_out <= kFusedMaxOut),
+// g's last hidden layer Lh (input X) with the output layer Lo (n_out <= MO <= kFusedMaxOut;
+// MO = 1 for the BCE logit, so the per-output loops carry no predicated-off work),
 // the loss and its gradient folded into the epilogue, warp r for row r:
 // h = ReLU(X Wh^T + bh) -> smem tile `hs` and Lh.Y; s = h Wo^T + bo (fp32 dot
 // products, reduced across the warp) -> Lo.Y; the row's loss -> rowloss;
@@ -411,6 +412,7 @@ struct TopLast {
     float* o_d; long long o_ldd;
 };
 
+template <int MO>
 __device__ __noinline__ void top_last_fused(const float* X, int ld, const float* ws, TopLast L, float* hs, float* gs,
                                             const int* y, int loss, float inv_b, float* rowloss, int r0, int nr,
                                             float* red) {
@@ -424,9 +426,9 @@ __device__ __noinline__ void top_last_fused(const float* X, int ld, const float*
     const float* wo = ws + L.o_ws_off;
     const int ldo = L.o_ws_ld;
     const bool valid = r < nr;
-    float part[kFusedMaxOut];
+    float part[MO];
 #pragma unroll
-    for (int j = 0; j < kFusedMaxOut; ++j) part[j] = 0.f;
+    for (int j = 0; j < MO; ++j) part[j] = 0.f;
     for (int c = 2 * lane; c < 8 * ntl; c += 64) {
         const float* src = red + r * rs + c;
         float2 v = *reinterpret_cast<const float2*>(src);
@@ -440,13 +442,13 @@ __device__ __noinline__ void top_last_fused(const float* X, int ld, const float*
         *reinterpret_cast<float2*>(hs + r * ld + c) = h;
         if (valid) *reinterpret_cast<float2*>(L.h_y + (long long)(r0 + r) * L.h_ldy + c) = h;
 #pragma unroll
-        for (int j = 0; j < kFusedMaxOut; ++j)
+        for (int j = 0; j < MO; ++j)
             if (j < nout) part[j] = fmaf(h.x, wo[j * ldo + c], fmaf(h.y, wo[j * ldo + c + 1], part[j]));
     }
-    float sv[kFusedMaxOut], dv[kFusedMaxOut];
+    float sv[MO], dv[MO];
     const float* bo = wo + ceil8(nout) * ldo;
 #pragma unroll
-    for (int j = 0; j < kFusedMaxOut; ++j) {
+    for (int j = 0; j < MO; ++j) {
         if (j < nout) {
             float t = part[j];
 #pragma unroll
@@ -457,7 +459,7 @@ __device__ __noinline__ void top_last_fused(const float* X, int ld, const float*
     const float li = loss_row(sv, nout, valid ? y[r] : 0, loss, inv_b, dv);
     if (!valid)
 #pragma unroll
-        for (int j = 0; j < kFusedMaxOut; ++j) dv[j] = 0.f;
+        for (int j = 0; j < MO; ++j) dv[j] = 0.f;
     if (valid && lane == 0) {
         rowloss[r] = li;
         float* lo = L.o_y + (long long)(r0 + r) * L.o_ldy;
@@ -471,7 +473,7 @@ __device__ __noinline__ void top_last_fused(const float* X, int ld, const float*
     for (int c = 2 * lane; c < 8 * ntl; c += 64) {
         float g0 = 0.f, g1 = 0.f;
 #pragma unroll
-        for (int j = 0; j < kFusedMaxOut; ++j)
+        for (int j = 0; j < MO; ++j)
             if (j < nout) {
                 g0 = fmaf(dv[j], wo[j * ldo + c], g0);
                 g1 = fmaf(dv[j], wo[j * ldo + c + 1], g1);
@@ -560,8 +562,12 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
                 const FusedLayerArgs& Lo = T[Lt - 1];
                 const TopLast tl{Lh.in, Lh.out, Lh.fmap, Lh.ws_off, Lh.ws_ld, Lo.out, Lo.ws_off, Lo.ws_ld,
                                  Lh.Y, Lh.ldy, Lh.D, Lh.ldd, Lo.Y, Lo.ldy, Lo.D, Lo.ldd};
-                top_last_fused(l == 0 ? C : TH(l - 1), ld, ws, tl, TH(l), G0, a.y + r0, a.loss, inv_b, a.rowloss + r0,
-                               r0, nr, red);
+                if (nout == 1)
+                    top_last_fused<1>(l == 0 ? C : TH(l - 1), ld, ws, tl, TH(l), G0, a.y + r0, a.loss, inv_b,
+                                      a.rowloss + r0, r0, nr, red);
+                else
+                    top_last_fused<kFusedMaxOut>(l == 0 ? C : TH(l - 1), ld, ws, tl, TH(l), G0, a.y + r0, a.loss,
+                                                 inv_b, a.rowloss + r0, r0, nr, red);
             } else {
                 tile_fwd(l == 0 ? C : TH(l - 1), ld, T[l].in, ws + T[l].ws_off, T[l].ws_ld, staged_bias(ws, T[l]),
                          T[l].out, T[l].fmap, TH(l), T[l].Y + (long long)r0 * T[l].ldy, T[l].ldy, nr, red);
