@@ -34,7 +34,7 @@ FP32_ALU_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12   # SMs x FP32 lanes x FMA
 TF32_PER_BF16 = 1.1 / 2.25                               # nominal dense TF32 / BF16 tensor throughput
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=1500)
@@ -52,7 +52,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-graphs", action="store_true", help="enqueue every step directly instead of replaying "
                     "a CUDA graph captured before each timed iteration")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def workload(args):
@@ -275,6 +275,24 @@ def roofline(prof, pk):
             "all_classes_ms": {k: round(v[1], 4) for k, v in sorted(prof.items(), key=lambda kv: -kv[1][1])}}
 
 
+def slowest_rank(x: float) -> float:
+    """The maximum of x over the ranks of the default process group (x itself
+    without one): a multi-GPU job is as fast as its slowest replica."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(samples_per_rank: int, world: int, slowest_seconds: float) -> float:
+    """Whole-job samples/s: every rank's samples over the slowest rank's time."""
+    return samples_per_rank * world / slowest_seconds
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -360,12 +378,8 @@ def run_ours(args):
     launches = ctx.launches - l0
     torch.cuda.synchronize()
     clk = clocks.stop()
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    n_samp = samples(p, W, K) * world
-    value = n_samp / (ms / 1e3)
+    ms = slowest_rank(ms)
+    value = job_throughput(samples(p, W, K), world, ms / 1e3)
 
     # per-kernel timing: the same workload again, every launch bracketed by CUDA events (recorded
     # inside the replayed graphs when graphs are on, so each duration is the kernel as the step runs it)
@@ -389,11 +403,11 @@ def run_ours(args):
         t0 = time.perf_counter()
         ctx.train_steps(k0, K, tp, ta)
         ctx.synchronize()
-        dt = time.perf_counter() - t0
+        dt = slowest_rank(time.perf_counter() - t0)
         ctx.bind_host_data(None, None, None)
         assert np.isfinite(loss_host.numpy()).all()
         h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
-        e2e = {"value": samples(p, k0, K) * world / dt, "unit": "samples/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": job_throughput(samples(p, k0, K), world, dt), "unit": "samples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": 4}
 
     if rank == 0:
