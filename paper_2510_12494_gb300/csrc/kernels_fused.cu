@@ -758,6 +758,9 @@ __global__ void __cluster_dims__(kUpdCluster, 1, 1) __launch_bounds__(kUpdThread
     __shared__ __align__(16) float Rw[kUpdCluster * kPer];    // partials of the owned outputs, by sender
     __shared__ float Rb[kUpdCluster * kPerB];
     __shared__ float Pb[kUpdThreads / 32];                    // the loss cluster's warp sums
+    // a passive forward that reads the version this update writes may launch now and fetch its rows; it
+    // waits for this grid before it reads the weights
+    griddep_trigger();
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int tile = blockIdx.x / kUpdCluster;
