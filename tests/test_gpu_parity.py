@@ -104,6 +104,33 @@ def test_fp32_epoch_loss_and_dag_equals_sequential(vfl, cid):
         np.testing.assert_array_equal(b, b2)
 
 
+def test_full_size_in_the_bench_configuration(vfl):
+    """The credit-shaped workload at full size as bench.py times it: one CUDA
+    graph per epoch (captured, then replayed), two worker streams per party,
+    five epochs; epoch losses within 1e-3 of the oracle and the final weights
+    within 1e-3."""
+    import synth
+    q, xp, xa, y, params = setup(synth.preset(2))
+    nb = q.steps_per_epoch
+    n_steps = nb * q.epochs
+    tp, ta = schedule(q, n_steps)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    for e in range(q.epochs):
+        g = ctx.capture(e * nb, nb, tp, ta)
+        ctx.launch_graph(g)
+    ctx.synchronize()
+    losses = ctx.read_losses(0, n_steps)
+    o = oracle.Oracle(q, xp, xa, y, params)
+    ref, _ = o.run(tp, ta, n_steps)
+    for e in range(q.epochs):
+        got = o.epoch_loss(losses[e * nb:(e + 1) * nb], e * nb)
+        want = o.epoch_loss(ref[e * nb:(e + 1) * nb], e * nb)
+        assert abs(got - want) <= EPOCH_LOSS_TOL * abs(want), (e, got, want)
+    for key, (W, b) in ctx.get_params().items():
+        assert rel_err(W, o.current_params()[key][0]) < 1e-3
+        assert rel_err(b, o.current_params()[key][1]) < 1e-3
+
+
 @pytest.mark.parametrize("cid", [3, 5])
 def test_bf16_free_running_epoch_loss(vfl, cid):
     """Without teacher forcing, a whole bf16 epoch stays within 2e-2 of the
