@@ -511,39 +511,30 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
     const int ntiles = (a.rows + R - 1) / R;
     const float inv_b = 1.0f / (float)a.rows;
     const int Ltot = La + Lt;
-    bool first = true;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int r0 = tile * R;
+    // one 16-row tile per CTA (the launch has one CTA per tile)
+    if ((int)blockIdx.x >= ntiles) {
+        griddep_wait();
+        return;
+    }
+    {
+        const int r0 = blockIdx.x * R;
         const int nr = min(R, a.rows - r0);
-        __syncthreads();
         async_rows(X, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)A[0].in_ld, nr);
-        if (first) {
-            // one commit group per layer, in the order the forward uses them (group 0 also x^a's rows);
-            // z^p's rows follow once the publisher has finished, after f_a's forward
-            for (int l = 0; l < Ltot; ++l) {
-                stage_layer_weights(ws, a.L[l]);
-                cp_commit();
-            }
-        } else {
-            async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);
+        // one commit group per layer, in the order the forward uses them (group 0 also x^a's rows);
+        // z^p's rows follow once the publisher has finished, after f_a's forward
+        for (int l = 0; l < Ltot; ++l) {
+            stage_layer_weights(ws, a.L[l]);
             cp_commit();
         }
         for (int l = 0; l < La; ++l) {                                   // z^a = f_a(x^a)
-            if (first)
-                cp_wait_pending(Ltot - 1 - l);   // x^a's rows and layers 0..l
-            else if (l == 0)
-                cp_wait_pending(0);              // this tile's x^a and z^p rows
-            else
-                __syncthreads();
+            cp_wait_pending(Ltot - 1 - l);       // x^a's rows and layers 0..l
             tile_fwd(l == 0 ? X : H(l - 1), ld, A[l].in, ws + A[l].ws_off, A[l].ws_ld, staged_bias(ws, A[l]), A[l].out,
                      A[l].fmap, l == La - 1 ? C : H(l), A[l].Y + (long long)r0 * A[l].ldy, A[l].ldy, nr, red);
         }
-        if (first) {
-            griddep_wait();                                              // the embedding's publisher has finished
-            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
-            async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);   // beside z^a's columns
-            cp_commit();
-        }
+        griddep_wait();                                                  // the embedding's publisher has finished
+        if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
+        async_rows(C + ea, ld, a.zp + (long long)r0 * a.ldzp, a.ldzp, ep8, nr);   // beside z^a's columns
+        cp_commit();
         // with n_out <= kFusedMaxOut, g's output layer, the loss, d(logits) and the output layer's input
         // gradient ride in the epilogue of g's last hidden layer (one warp per row)
         const bool fuse_out = Lt >= 2 && nout <= kFusedMaxOut;
@@ -658,11 +649,6 @@ __global__ void __launch_bounds__(NT, 1) fused_active_kernel(const FusedStepArgs
             gin = gout;
             gout = t;
         }
-        first = false;
-    }
-    if (first) {                     // CTAs without a row tile have nothing in flight
-        griddep_wait();
-        cp_wait_pending(0);
     }
     if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
     publish_header(a.pub_hdr, a.k, a.batch, a.version);
