@@ -314,33 +314,27 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
     float* t2 = t1 + R * ld;
     float* red = t2 + R * ld;                           // partial output blocks
     const int ntiles = (a.rows + R - 1) / R;
-    bool first = true;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int r0 = tile * R;
+    // one 16-row tile per CTA (the launch has one CTA per tile)
+    if ((int)blockIdx.x >= ntiles) {
+        griddep_wait();
+        return;
+    }
+    {
+        const int r0 = blockIdx.x * R;
         const int nr = min(R, a.rows - r0);
-        __syncthreads();
         async_rows(t0, ld, a.x + (long long)r0 * a.ldx, a.ldx, (int)a.L[0].in_ld, nr);
-        if (first) {
-            // the weight version comes from an earlier update, which may still be finishing
-            griddep_wait();
-            // group l holds layer l's weights (group 0 also the rows), so layer l
-            // only waits for its own weights while the later ones are still arriving
-            for (int l = 0; l < a.nl; ++l) {
-                stage_layer_weights(ws, a.L[l]);
-                cp_commit();
-            }
-        } else {
+        // the weight version comes from an earlier update, which may still be finishing
+        griddep_wait();
+        // group l holds layer l's weights (group 0 also the rows), so layer l
+        // only waits for its own weights while the later ones are still arriving
+        for (int l = 0; l < a.nl; ++l) {
+            stage_layer_weights(ws, a.L[l]);
             cp_commit();
         }
         const float* cur = t0;
         for (int l = 0; l < a.nl; ++l) {
             const FusedLayerArgs& L = a.L[l];
-            if (first)
-                cp_wait_pending(a.nl - 1 - l);
-            else if (l == 0)
-                cp_wait_pending(0);
-            else
-                __syncthreads();
+            cp_wait_pending(a.nl - 1 - l);
             float* nxt = (l & 1) ? t2 : t1;
             tile_fwd(cur, ld, L.in, ws + L.ws_off, L.ws_ld, staged_bias(ws, L), L.out, L.fmap, nxt,
                      L.Y + (long long)r0 * L.ldy, L.ldy, nr, red);
@@ -372,9 +366,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_fwd_kernel(const FusedCha
                 }
             }
         }
-        first = false;
     }
-    if (first) griddep_wait();       // CTAs without a row tile have nothing in flight
     publish_header(a.hdr, a.k, a.batch, a.version);
 }
 
@@ -671,24 +663,25 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
     const FusedLayerArgs* P = a.L;
     const int ep8 = ceil8(P[Lp - 1].out);
     const int ntiles = (a.rows + R - 1) / R;
-    bool first = true;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int r0 = tile * R;
+    // one 16-row tile per CTA (the launch has one CTA per tile)
+    if ((int)blockIdx.x >= ntiles) {
+        griddep_wait();
+        return;
+    }
+    {
+        const int r0 = blockIdx.x * R;
         const int nr = min(R, a.rows - r0);
-        __syncthreads();
         for (int l = 0; l < Lp; ++l)
             async_rows(slot(l), ld, P[l].Y + (long long)r0 * P[l].ldy, P[l].ldy, (int)P[l].out_ld, nr);
         cp_commit();
-        if (first) {
-            // weights in the order the backward uses them (layer Lp-1 first), then wait for the active
-            // step, whose dz^p comes last
-            for (int l = Lp - 1; l >= 1; --l) {
-                stage_layer_weights(ws, P[l]);
-                cp_commit();
-            }
-            griddep_wait();
-            if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
+        // weights in the order the backward uses them (layer Lp-1 first), then wait for the active
+        // step, whose dz^p comes last
+        for (int l = Lp - 1; l >= 1; --l) {
+            stage_layer_weights(ws, P[l]);
+            cp_commit();
         }
+        griddep_wait();
+        if (threadIdx.x == 0) hdr_k = a.chk_hdr->k;
         async_rows(gs, ld, a.gradp + (long long)r0 * a.ldgp, a.ldgp, (int)P[Lp - 1].out_ld, nr);
         cp_commit();
         cp_wait_pending(0);
@@ -716,9 +709,7 @@ __global__ void __launch_bounds__(NT, 1) fused_passive_bwd_kernel(const FusedSte
             gin = gout;
             gout = t;
         }
-        first = false;
     }
-    if (first) griddep_wait();
     if (threadIdx.x == 0 && hdr_k != a.k) atomicOr(a.status, ST_VERSION);
 }
 
