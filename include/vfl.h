@@ -17,7 +17,8 @@
  *  - Party ids: 0 = passive bottom f_p (theta_2), 1 = active bottom f_a,
  *    2 = top model g (1 and 2 together are theta_1).
  *  - "Host pointer" arguments are read or written before the call returns
- *    (except vfl_stage_rows, which is asynchronous); the caller keeps ownership.
+ *    (except vfl_fetch_loss and the arrays bound by vfl_bind_host_data, which
+ *    are used asynchronously); the caller keeps ownership.
  *  - Device memory comes from the caller: vfl_workspace_bytes() says how much,
  *    vfl_create() carves every device buffer out of that one allocation.
  *  - Work is enqueued on caller-provided CUDA streams (vfl_set_streams);
@@ -131,17 +132,6 @@ vfl_status vfl_set_streams(vfl_ctx* ctx, int32_t n, void* const* streams);
  * [0, n_out)).  Synchronous.  bf16 contexts round the features to bf16 here.
  */
 vfl_status vfl_load_data(vfl_ctx* ctx, const float* x_passive, const float* x_active, const int32_t* y);
-
-/*
- * Asynchronously copy rows [row0, row0+n) of the dataset from host memory
- * (pinned for true asynchrony) into the device copy: the passive rows on the
- * passive stream of worker `worker`, the active rows and labels on the active
- * one.  The host buffers hold only those n rows and must stay valid until the
- * streams pass this point.  Work enqueued afterwards on the same workers sees
- * the new rows.
- */
-vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n, const float* x_passive,
-                          const float* x_active, const int32_t* y);
 
 /*
  * Host-resident data.  After this call every step k reads its own rows

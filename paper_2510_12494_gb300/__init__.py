@@ -57,8 +57,6 @@ EXPORTS = {
     "vfl_destroy": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_set_streams": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]),
     "vfl_load_data": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
-    "vfl_stage_rows": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64,
-                                        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_bind_host_data": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                             ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_set_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
@@ -239,14 +237,6 @@ class Context:
         y = np.ascontiguousarray(y, np.int32)
         assert xp.shape == (self.n_rows, self.p.d_passive) and xa.shape == (self.n_rows, self.p.d_active)
         self._call(lib().vfl_load_data, _ptr(xp), _ptr(xa), _ptr(y))
-
-    def stage_rows(self, worker, row0, xp, xa, y):
-        """Asynchronous host->device copy of rows [row0, row0+len(y)); the arrays
-        (ideally pinned) must stay alive until the worker streams pass this point."""
-        def addr(a):
-            return a.data_ptr() if hasattr(a, "data_ptr") else a.ctypes.data
-        self._call(lib().vfl_stage_rows, worker, row0, len(y), ctypes.c_void_p(addr(xp)), ctypes.c_void_p(addr(xa)),
-                   ctypes.c_void_p(addr(y)))
 
     def bind_host_data(self, xp, xa, y, loss_out=None):
         """Every later step reads its rows from these host tensors (pinned torch

@@ -108,8 +108,8 @@ struct vfl_ctx {
     // device buffers
     void* Xp = nullptr; void* Xa = nullptr; int* Y = nullptr;
     long long ldxp = 0, ldxa = 0;
-    float* stage_p[kMaxWorkers] = {};
-    float* stage_a[kMaxWorkers] = {};
+    float* stage_p = nullptr;                    // fp32 rows on their way into the dataset (vfl_load_data)
+    float* stage_a = nullptr;
     std::vector<void*> act_p[kMaxSlots];          // per slot, per passive layer [B, ld8(out)]
     std::vector<void*> dpre_p[kMaxWorkers];       // per worker, per passive layer
     std::vector<void*> act_a[kMaxWorkers], dpre_a[kMaxWorkers];
@@ -480,10 +480,8 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
     ctx->Xp = cv.take((unsigned long long)ctx->n_rows * ctx->ldxp * es);
     ctx->Xa = cv.take((unsigned long long)ctx->n_rows * ctx->ldxa * es);
     ctx->Y = static_cast<int*>(cv.take((unsigned long long)ctx->n_rows * 4));
-    for (int w = 0; w < ctx->W; ++w) {
-        ctx->stage_p[w] = static_cast<float*>(cv.take(B * c.d_passive * 4ull));
-        ctx->stage_a[w] = static_cast<float*>(cv.take(B * c.d_active * 4ull));
-    }
+    ctx->stage_p = static_cast<float*>(cv.take(B * c.d_passive * 4ull));
+    ctx->stage_a = static_cast<float*>(cv.take(B * c.d_active * 4ull));
     for (std::vector<Layer>* v : {&ctx->P, &ctx->A, &ctx->T}) {
         for (Layer& L : *v) {
             L.W = static_cast<float*>(cv.take((unsigned long long)L.out * L.in * 4));
@@ -1463,34 +1461,15 @@ vfl_status vfl_load_data(vfl_ctx* ctx, const float* xp, const float* xa, const i
     cudaStream_t s = ctx->ps[0];
     for (long long r = 0; r < ctx->n_rows; r += c.batch) {
         const int n = (int)std::min<long long>(c.batch, ctx->n_rows - r);
-        CK(cudaMemcpyAsync(ctx->stage_p[0], xp + r * c.d_passive, (size_t)n * c.d_passive * 4, cudaMemcpyHostToDevice, s));
-        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_p[0], n, c.d_passive,
+        CK(cudaMemcpyAsync(ctx->stage_p, xp + r * c.d_passive, (size_t)n * c.d_passive * 4, cudaMemcpyHostToDevice, s));
+        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_p, n, c.d_passive,
                                 static_cast<char*>(ctx->Xp) + r * ctx->ldxp * ctx->esz, ctx->ldxp, ctx->bf16, s));
-        CK(cudaMemcpyAsync(ctx->stage_a[0], xa + r * c.d_active, (size_t)n * c.d_active * 4, cudaMemcpyHostToDevice, s));
-        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_a[0], n, c.d_active,
+        CK(cudaMemcpyAsync(ctx->stage_a, xa + r * c.d_active, (size_t)n * c.d_active * 4, cudaMemcpyHostToDevice, s));
+        PLAUNCH(K_CAST, 0, 0, s, launch_cast_rows(ctx->stage_a, n, c.d_active,
                                 static_cast<char*>(ctx->Xa) + r * ctx->ldxa * ctx->esz, ctx->ldxa, ctx->bf16, s));
         CK(cudaStreamSynchronize(s));
     }
     CK(cudaMemcpy(ctx->Y, y, (size_t)ctx->n_rows * 4, cudaMemcpyHostToDevice));
-    return VFL_OK;
-}
-
-vfl_status vfl_stage_rows(vfl_ctx* ctx, int32_t worker, int64_t row0, int64_t n, const float* xp, const float* xa,
-                          const int32_t* y) {
-    if (!ctx || !xp || !xa || !y) return ctx ? ctx->fail(VFL_E_INVAL, "null data pointer") : VFL_E_INVAL;
-    if (ctx->broken) return VFL_E_CUDA;
-    const vfl_config& c = ctx->cfg;
-    if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
-    if (row0 < 0 || n < 1 || n > c.batch || row0 + n > ctx->n_rows)
-        return ctx->fail(VFL_E_INVAL, "rows [%lld, %lld) invalid (at most one batch)", (long long)row0, (long long)(row0 + n));
-    cudaStream_t sp = ctx->ps[worker], sa = ctx->as[worker];
-    CK(cudaMemcpyAsync(ctx->stage_p[worker], xp, (size_t)n * c.d_passive * 4, cudaMemcpyHostToDevice, sp));
-    PLAUNCH(K_CAST, 0, n * c.d_passive * (4.0 + ctx->esz), sp, launch_cast_rows(ctx->stage_p[worker], (int)n, c.d_passive,
-                            static_cast<char*>(ctx->Xp) + row0 * ctx->ldxp * ctx->esz, ctx->ldxp, ctx->bf16, sp));
-    CK(cudaMemcpyAsync(ctx->stage_a[worker], xa, (size_t)n * c.d_active * 4, cudaMemcpyHostToDevice, sa));
-    PLAUNCH(K_CAST, 0, n * c.d_active * (4.0 + ctx->esz), sa, launch_cast_rows(ctx->stage_a[worker], (int)n, c.d_active,
-                            static_cast<char*>(ctx->Xa) + row0 * ctx->ldxa * ctx->esz, ctx->ldxa, ctx->bf16, sa));
-    CK(cudaMemcpyAsync(ctx->Y + row0, y, (size_t)n * 4, cudaMemcpyHostToDevice, sa));
     return VFL_OK;
 }
 

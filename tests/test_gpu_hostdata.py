@@ -98,3 +98,19 @@ def test_unbind_returns_to_resident_data(vfl):
     ctx.train_steps(n, n, tp, ta)
     np.testing.assert_array_equal(ctx.read_losses(0, 2 * n), ref.read_losses(0, 2 * n))
     assert_same_state(ctx, ref)
+
+
+def test_fetch_loss_copies_each_step_loss(vfl):
+    """vfl_fetch_loss: an asynchronous copy of one step's mean loss into pinned
+    host memory, valid once the step's active worker stream passes it."""
+    import torch
+    q, xp, xa, y, params = setup(synth.preset(2), 2 * 1024 + 304)
+    n = 6
+    tp, ta = schedule(q, n)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    out = torch.full((n,), float("nan"), dtype=torch.float32).pin_memory()
+    ctx.train_steps(0, n, tp, ta)
+    for k in range(n):
+        ctx.fetch_loss(k, out.data_ptr() + 4 * k)
+    ctx.synchronize()
+    np.testing.assert_array_equal(out.numpy(), ctx.read_losses(0, n))
