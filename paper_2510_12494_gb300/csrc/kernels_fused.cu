@@ -11,16 +11,17 @@
 //    d(pre-activation) rows stay in HBM for the update.
 //  - passive backward: the input-gradient chain of f_p from dz^p.
 //  - update (one per party): dW = D^T X over the step's rows for every layer,
-//    an output tile per cluster of 8 CTAs that each take 1/8 of the rows; the 8
-//    partial tiles are summed in rank order through distributed shared memory
-//    (deterministic), and SGD writes the master and the new version's copy.
+//    an output tile per cluster of 8 CTAs that each take 1/8 of the rows; each
+//    CTA pushes its partial of the outputs another rank owns into that rank's
+//    shared memory, the owners sum the 8 partials in rank order (deterministic)
+//    and SGD writes the master and the new version's copy.
 //
 // The row-tile GEMMs run on the warp-level tensor cores (mma.sync m16n8k8,
 // TF32) in 3xTF32 form, which keeps fp32 accuracy: x = hi + lo with hi, lo
-// TF32, and a b ~ a_hi b_hi + a_lo b_hi + a_hi b_lo.  Activation tiles that
-// feed a GEMM live in shared memory as their hi and lo planes, split once by
-// the epilogue that writes them and loaded with ldmatrix; weights are split as
-// they are read.  Every tile is zero-padded to a multiple of 8 columns and
+// TF32, and a b ~ a_hi b_hi + a_lo b_hi + a_hi b_lo.  Activation tiles live in
+// shared memory in fp32; their A fragments are loaded with ldmatrix and split
+// in registers, and weights are split as they are read.  Every tile is
+// zero-padded to a multiple of 8 columns and
 // every staged weight matrix to a multiple of 8 rows, so the GEMM loops need no
 // bounds checks.
 #include <cooperative_groups.h>
