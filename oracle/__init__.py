@@ -15,5 +15,5 @@ constant) and bf16 rounding against torch's cast.  Parity unpinned: nothing.
 from .vfl_oracle import (  # noqa: F401
     PHILOX_M, PHILOX_W, TAG_DP, TAG_DPE, TAG_SCHED, SCHED_SYNC, SCHED_MAX, SCHED_SEEDED,
     philox, make_schedule, bf16_round, mlp_forward, mlp_backward, loss_and_dlogits,
-    dp_normals, dp_clip_noise, dp_embed, gdp_sigma, Oracle, StepRecord,
+    dp_normals, dp_clip_noise, dp_embed, gdp_sigma, ps_interval, ps_aggregates_after, Oracle, StepRecord,
 )

@@ -47,6 +47,14 @@ Readings where the paper is silent (each is listed in the design doc):
   received gradient by c_i (the Jacobian of c_i and of the noise are ignored)
   before its own ReLU mask on the clean z.  sigma for a target mu-GDP level
   follows Eq. 25 with the O(.)'s constant taken as 1.
+* Intra-party semi-asynchronous parameter server (Sec. 4.2, Eq. 5, Algorithm
+  1), when cfg.ps_dt0 > 0: each party keeps one replica of its parameters per
+  worker (cfg.workers of them); step k is served by worker pair k mod W, whose
+  replicas it reads (the latest: no staleness within a replica's chain) and
+  updates.  After epoch t (1-based) each party's replicas are averaged (sum over
+  the workers in order, divided by W) and every replica takes the average when
+  t mod Delta T_t == 0, Delta T_t = ceil(Delta T_0 / 2 tanh(2 t / Delta T_0 - 2)
+  + Delta T_0 / 2) (Eq. 5).
 * bf16 presets round to bf16 (round-to-nearest-even, via fp32) at: the inputs,
   each weight version's compute copy (biases stay fp32), every stored hidden
   activation and embedding, and every activation gradient handed from one layer
@@ -263,6 +271,17 @@ def dp_embed(z, k: int, clip: float, sigma: float, seed: int):
     return out, c
 
 
+def ps_interval(t: int, dt0: int) -> int:
+    """Synchronization interval Delta T_t of the intra-party parameter server
+    after epoch t (Eq. 5)."""
+    return math.ceil(dt0 / 2.0 * math.tanh(2.0 * t / dt0 - 2.0) + dt0 / 2.0)
+
+
+def ps_aggregates_after(t: int, dt0: int) -> bool:
+    """Whether the replicas are averaged at the end of epoch t (1-based): t mod Delta T_t == 0."""
+    return t % ps_interval(t, dt0) == 0
+
+
 def gdp_sigma(mu: float, batch: int, n: int, queries: int) -> float:
     """Noise multiplier for mu-GDP on the published embedding, Eq. 25 with the
     O(.)'s constant taken as 1: sigma = N_m sqrt(K) / (mu N), N_m the minibatch
@@ -315,6 +334,7 @@ class Oracle:
     channel_e: dict = field(default_factory=dict)
     channel_g: dict = field(default_factory=dict)
     emb_scale: dict = field(default_factory=dict)   # step -> per-row clip factors of its published embedding
+    replicas: list = None                            # parameter-server mode: [(P, A, T)] per worker
 
     def __post_init__(self):
         c = self.cfg
@@ -331,6 +351,11 @@ class Oracle:
         T = [tuple(np.asarray(v, np.float64) for v in self.params[(2, l)]) for l in range(lt)]
         self.versions_p = {0: P}
         self.versions_a = {0: (A, T)}
+        self.ps = getattr(c, "ps_dt0", 0) > 0
+        if self.ps:
+            if c.staleness != 0:
+                raise ValueError("the parameter-server mode reads each replica's latest version (staleness 0)")
+            self.replicas = [(_copy_params(P), _copy_params(A), _copy_params(T)) for _ in range(c.workers)]
 
     # compute copies of a stored version (bf16 presets round W, never b)
     def _compute(self, layers):
@@ -349,6 +374,10 @@ class Oracle:
         j, r0, r1 = self.batch_rows(k)
         Bk = r1 - r0
         vp, va = k - tau_p, k - tau_a
+        if self.ps:   # worker pair k mod W serves the step with its own replicas
+            w = k % c.workers
+            self.versions_p[vp] = self.replicas[w][0]
+            self.versions_a[va] = (self.replicas[w][1], self.replicas[w][2])
 
         # Publisher phase (passive): z^p = f_p(x^p; theta_2^(k - tau_p)), publish to C_e[B_j].
         P = self._compute(self.versions_p[vp])
@@ -397,6 +426,11 @@ class Oracle:
         newP = [(W - lr * dW, b - lr * db) for (W, b), (dW, db) in zip(curP, gP)]
         newA = [(W - lr * dW, b - lr * db) for (W, b), (dW, db) in zip(curA, gA)]
         newT = [(W - lr * dW, b - lr * db) for (W, b), (dW, db) in zip(curT, gT)]
+        if self.ps:
+            self.replicas[k % c.workers] = (newP, newA, newT)
+            if (k + 1) % self.nb == 0 and ps_aggregates_after((k + 1) // self.nb, c.ps_dt0):
+                self._ps_average()
+            newP, newA, newT = self.replicas[0]      # the stored version: replica 0 (see current_params)
         self.versions_p[k + 1] = newP
         self.versions_a[k + 1] = (newA, newT)
         # only the last S+1 versions can ever be read again
@@ -413,10 +447,34 @@ class Oracle:
             for party, g in ((0, gP), (1, gA), (2, gT)):
                 for l, gl in enumerate(g):
                     rec.grads[(party, l)] = gl
-            rec.params = self.current_params()
+            rec.params = self.replica_params(k % c.workers) if self.ps else self.current_params()
         return rec
 
+    def _ps_average(self):
+        """Every party's replicas take their mean (sum over the workers in order, divided by W)."""
+        W = len(self.replicas)
+        avg = []
+        for part in range(3):
+            layers = []
+            for l in range(len(self.replicas[0][part])):
+                Ws = sum(self.replicas[w][part][l][0] for w in range(W)) / W
+                bs = sum(self.replicas[w][part][l][1] for w in range(W)) / W
+                layers.append((Ws, bs))
+            avg.append(layers)
+        self.replicas = [tuple(_copy_params(p) for p in avg) for _ in range(W)]
+
+    def replica_params(self, w: int):
+        """Parameter-server mode: replica w's parameters {(party, layer): (W, b)}."""
+        out = {}
+        for party, layers in enumerate(self.replicas[w]):
+            for l, (W, b) in enumerate(layers):
+                out[(party, l)] = (W.copy(), b.copy())
+        return out
+
     def current_params(self):
+        """The parameters after the last step (parameter-server mode: replica 0's)."""
+        if self.ps:
+            return self.replica_params(0)
         out = {}
         P = self.versions_p[self.k]
         A, T = self.versions_a[self.k]

@@ -139,6 +139,7 @@ class VflPreset:
     dp_sigma: float = 0.0
     seed: int = 0
     dp_target: str = "grad" # "grad": the published embedding gradient; "emb": the published embedding
+    ps_dt0: int = 0         # > 0: per-worker replicas averaged after the epochs Eq. 5 selects (Delta T_0)
 
     @property
     def n_out(self) -> int:
