@@ -47,6 +47,9 @@ def parse(argv=None):
                     help="with DP: the published gradient (the preset's) or the published embedding (App. C)")
     ap.add_argument("--dp", type=float, nargs=2, default=None, metavar=("CLIP", "SIGMA"),
                     help="enable DP with this clip norm and noise multiplier")
+    ap.add_argument("--ps-dt0", type=int, default=0, metavar="DT0",
+                    help="intra-party parameter server (Eq. 5): per-worker replicas averaged per Delta T_0 = DT0 "
+                         "(sets the staleness to 0)")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -66,6 +69,8 @@ def workload(args):
         p = p.with_(dp_clip=args.dp[0], dp_sigma=args.dp[1])
     if args.dp_target:
         p = p.with_(dp_target=args.dp_target)
+    if args.ps_dt0:
+        p = p.with_(ps_dt0=args.ps_dt0, staleness=0, schedule="sync")
     desc = (f"{p.name}: N={p.n_rows}, d_p/d_a={p.d_passive}/{p.d_active}, "
             f"passive {'-'.join(map(str, (p.d_passive,) + p.passive))}, "
             f"active {'-'.join(map(str, (p.d_active,) + p.active))}, "
@@ -73,7 +78,9 @@ def workload(args):
             f"B={p.batch}, S={p.staleness} ({p.schedule} schedule), {p.dtype}, "
             f"{p.workers} worker stream(s) per party" +
             (f", DP on the {'embedding' if p.dp_target == 'emb' else 'embedding gradient'} C={p.dp_clip} "
-             f"sigma={p.dp_sigma}" if p.dp_clip else ""))
+             f"sigma={p.dp_sigma}" if p.dp_clip else "") +
+            (f", parameter server per worker (replicas averaged per Eq. 5, Delta T_0={p.ps_dt0})"
+             if p.ps_dt0 else ""))
     return p, desc
 
 

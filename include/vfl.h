@@ -83,6 +83,7 @@ typedef struct vfl_config {
     float dp_sigma;                         /* noise multiplier; noise std = sigma * clip */
     uint64_t dp_seed;                       /* Philox key of the DP noise                */
     int32_t dp_target;                      /* VFL_DP_GRAD | VFL_DP_EMB (see below)       */
+    int32_t ps_dt0;                         /* > 0: intra-party parameter server, Delta T_0 (see below) */
 } vfl_config;
 
 /*
@@ -97,6 +98,26 @@ typedef struct vfl_config {
  *    ignored).
  * Either sends the model through the per-layer kernels.
  */
+
+/*
+ * Intra-party semi-asynchronous parameter server (Sec. 4.2, Eq. 5), enabled by
+ * ps_dt0 > 0 (requires staleness == 0).  Each party keeps one replica of its
+ * parameters (fp32 master and compute copy) per worker; step k runs on worker
+ * w = k mod workers, reads replica w as it stands and applies its SGD update to
+ * replica w only, so the workers' chains run concurrently on their own stream
+ * pairs.  After the last step of epoch t (t = 1, 2, ...; an epoch is
+ * ceil(n_rows / batch) steps) every party's replicas are replaced by their mean
+ * (fp32 sum over the workers in order 0..W-1, then divided by W) when
+ * t mod Delta T_t == 0, Delta T_t = ceil(Delta T_0 / 2 tanh(2 t / Delta T_0 - 2)
+ * + Delta T_0 / 2).  vfl_get_params reads replica 0; vfl_get_replica /
+ * vfl_set_replica read and write any replica (they replace the version API,
+ * which answers VFL_E_STATE in this mode).
+ */
+
+/* Delta T_t of Eq. 5 for epoch t >= 1 and Delta T_0 = dt0 >= 1 (host only, pure): the
+ * parameter-server mode averages the replicas after epoch t when t mod Delta T_t == 0.
+ * VFL_E_INVAL for t < 1, dt0 < 1 or a null output. */
+vfl_status vfl_ps_interval(int64_t t, int32_t dt0, int64_t* interval);
 
 /* Noise multiplier for mu-GDP on the published embedding, Eq. 25 with the O(.)
  * constant taken as 1: sigma = batch sqrt(queries) / (mu n_rows), queries = the
@@ -188,6 +209,16 @@ vfl_status vfl_step_cursor(vfl_ctx* ctx, int64_t* k);
 vfl_status vfl_get_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, float* W, float* b);
 vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k);
 vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, const float* W, const float* b);
+
+/*
+ * Parameter-server mode only (VFL_E_STATE otherwise): the fp32 master of one
+ * layer of replica `worker` (0 <= worker < workers), host pointers W [out, in]
+ * and b [out].  Both synchronize the context and need no step in flight;
+ * vfl_set_replica also rewrites the replica's compute copy (rounded to the
+ * compute dtype).  A checkpoint in this mode is the cursor plus every replica.
+ */
+vfl_status vfl_get_replica(vfl_ctx* ctx, int32_t worker, int32_t party, int32_t layer, float* W, float* b);
+vfl_status vfl_set_replica(vfl_ctx* ctx, int32_t worker, int32_t party, int32_t layer, const float* W, const float* b);
 
 /*
  * Staleness schedule (host only, pure).  tau_p[k], tau_a[k] for k < n_steps:
@@ -298,7 +329,7 @@ int64_t vfl_kernel_launches(const vfl_ctx* ctx);
  * graph has run returns VFL_E_STATE.  Such a graph should not be replayed
  * after the fold (its events go back to the context's pool).
  */
-#define VFL_KERNEL_CLASSES 18
+#define VFL_KERNEL_CLASSES 19
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);
 vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
                            double* bytes);

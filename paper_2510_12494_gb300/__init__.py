@@ -24,7 +24,7 @@ DP_GRAD, DP_EMB = 0, 1
 SCHED_SYNC, SCHED_MAX, SCHED_SEEDED = 0, 1, 2
 TAP_EMB, TAP_GRAD, TAP_LOGITS, TAP_ZA, TAP_DZA = range(5)
 PASSIVE, ACTIVE, TOP = 0, 1, 2
-KERNEL_CLASSES = 18
+KERNEL_CLASSES = 19
 
 STATUS_NAMES = {0: "VFL_OK", 1: "VFL_E_INVAL", 2: "VFL_E_OOM", 3: "VFL_E_CUDA", 4: "VFL_E_STATE",
                 5: "VFL_E_VERSION", 6: "VFL_E_TIMEOUT"}
@@ -45,7 +45,7 @@ class VflConfig(ctypes.Structure):
         ("loss", ctypes.c_int32), ("dtype", ctypes.c_int32), ("batch", ctypes.c_int32),
         ("lr", ctypes.c_float), ("staleness", ctypes.c_int32), ("workers", ctypes.c_int32),
         ("dp_clip", ctypes.c_float), ("dp_sigma", ctypes.c_float), ("dp_seed", ctypes.c_uint64),
-        ("dp_target", ctypes.c_int32),
+        ("dp_target", ctypes.c_int32), ("ps_dt0", ctypes.c_int32),
     ]
 
 
@@ -71,6 +71,11 @@ EXPORTS = {
     "vfl_set_cursor": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
     "vfl_set_version": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
                                          ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_get_replica": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                         ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_set_replica": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                         ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_ps_interval": (ctypes.c_int32, [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64)]),
     "vfl_gdp_sigma": (ctypes.c_int32, [ctypes.c_double, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                        ctypes.POINTER(ctypes.c_double)]),
     "vfl_make_schedule": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
@@ -151,7 +156,15 @@ def make_config(p) -> VflConfig:
     c.dp_sigma = p.dp_sigma
     c.dp_seed = getattr(p, "dp_seed", getattr(p, "seed", 0))
     c.dp_target = DP_EMB if getattr(p, "dp_target", "grad") == "emb" else DP_GRAD
+    c.ps_dt0 = getattr(p, "ps_dt0", 0)
     return c
+
+
+def ps_interval(t: int, dt0: int) -> int:
+    """Delta T_t of Eq. 5 as the runtime computes it (see vfl_ps_interval)."""
+    out = ctypes.c_int64()
+    _check(lib().vfl_ps_interval(t, dt0, ctypes.byref(out)))
+    return out.value
 
 
 def gdp_sigma(mu: float, batch: int, n_rows: int, queries: int) -> float:
@@ -313,6 +326,24 @@ class Context:
                 out[(party, l)] = (W, b)
         return out
 
+    def get_replica(self, w: int):
+        """Parameter-server mode: {(party, layer): (W, b)} of worker w's replica (fp32 masters)."""
+        out = {}
+        for party, widths in ((0, self.p.passive), (1, self.p.active), (2, self.p.top)):
+            for l in range(len(widths)):
+                o, i = self._shape(party, l)
+                W = np.zeros((o, i), np.float32)
+                b = np.zeros(o, np.float32)
+                self._call(lib().vfl_get_replica, w, party, l, _ptr(W), _ptr(b))
+                out[(party, l)] = (W, b)
+        return out
+
+    def set_replica(self, w: int, params: dict):
+        for (party, l), (W, b) in params.items():
+            W = np.ascontiguousarray(W, np.float32)
+            b = np.ascontiguousarray(b, np.float32)
+            self._call(lib().vfl_set_replica, w, party, l, _ptr(W), _ptr(b))
+
     def set_cursor(self, k: int):
         self._call(lib().vfl_set_cursor, k)
 
@@ -324,15 +355,26 @@ class Context:
             b = np.ascontiguousarray(b, np.float32)
             self._call(lib().vfl_set_version, party, l, v, _ptr(W), _ptr(b))
 
+    @property
+    def ps(self) -> bool:
+        return self.cfg.ps_dt0 > 0
+
     def checkpoint(self):
-        """(k, {version: params}, fp32 masters of version k)."""
+        """(k, {version: params}, fp32 masters of version k); in the parameter-server
+        mode (k, {worker: replica}, None)."""
         k = self.cursor()
+        if self.ps:
+            return k, {w: self.get_replica(w) for w in range(self.p.workers)}, None
         vers = {v: self.get_version(v) for v in range(max(0, k - self.p.staleness), k + 1)}
         return k, vers, self.get_params()
 
     def restore(self, ckpt):
         k, vers, master = ckpt
         self.set_cursor(k)
+        if self.ps:
+            for w, params in vers.items():
+                self.set_replica(w, params)
+            return
         for v, params in vers.items():
             self.set_version(v, master if v == k else params)
 

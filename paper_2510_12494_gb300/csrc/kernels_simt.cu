@@ -463,6 +463,37 @@ __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
     }
 }
 
+__global__ void __launch_bounds__(256) ps_average_kernel(const PsAvgLayer* __restrict__ tab, int n_layers,
+                                                         long long total, int nrep, int c_bf16) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        int l = 0;
+        while (l + 1 < n_layers && i >= tab[l + 1].begin) ++l;
+        const PsAvgLayer& L = tab[l];
+        const long long idx = i - L.begin;
+        const long long nw = (long long)L.out * L.in;
+        if (idx < nw) {
+            float acc = 0.f;
+            for (int w = 0; w < nrep; ++w) acc += L.Wr[w][idx];
+            const float v = __fdiv_rn(acc, (float)nrep);
+            const long long r = idx / L.in, c = idx % L.in;
+            for (int w = 0; w < nrep; ++w) {
+                L.Wr[w][idx] = v;
+                stf(L.cW[w], r * L.in_ld + c, c_bf16, v);
+            }
+        } else {
+            const long long j = idx - nw;
+            float acc = 0.f;
+            for (int w = 0; w < nrep; ++w) acc += L.br[w][j];
+            const float v = __fdiv_rn(acc, (float)nrep);
+            for (int w = 0; w < nrep; ++w) {
+                L.br[w][j] = v;
+                L.cb[w][j] = v;
+            }
+        }
+    }
+}
+
 __global__ void write_header_kernel(ChannelHeader* h, long long k, int batch, int version) {
     h->k = k;
     h->batch = batch;
@@ -635,6 +666,13 @@ cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, floa
 
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
     sgd_kernel<<<grid_for(a.total, 256), 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ps_average(const PsAvgLayer* tab, int n_layers, long long total, int nrep, int c_bf16,
+                              cudaStream_t s) {
+    if (total <= 0) return cudaSuccess;
+    ps_average_kernel<<<grid_for(total, 256), 256, 0, s>>>(tab, n_layers, total, nrep, c_bf16);
     return cudaGetLastError();
 }
 

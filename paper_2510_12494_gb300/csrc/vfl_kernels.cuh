@@ -92,6 +92,21 @@ struct SgdArgs {
 };
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s);
 
+// Parameter-server aggregation (Sec. 4.2): every replica of a party's layers takes the mean of the
+// replicas, summed in fp32 in replica order and divided by nrep (IEEE division); the fp32 masters
+// and the compute copies [out, in_ld] (padding columns untouched) are all rewritten.  The layer
+// table lives in device memory; layer l covers flat indices [begin, begin + out * in + out).
+constexpr int kPsMaxRep = 16;
+struct PsAvgLayer {
+    float* Wr[kPsMaxRep]; float* br[kPsMaxRep];   // fp32 masters per replica
+    void* cW[kPsMaxRep]; float* cb[kPsMaxRep];    // compute copies per replica
+    int out, in;
+    long long in_ld;
+    long long begin;
+};
+cudaError_t launch_ps_average(const PsAvgLayer* tab, int n_layers, long long total, int nrep, int c_bf16,
+                              cudaStream_t s);
+
 // Output layer of g (n_out <= kHeadMaxOut outputs over K <= kHeadMaxK bf16 inputs) with the loss
 // folded in, for the bf16 path: per row the logits s = h W^T + b (fp32), the row's loss and
 // ds = dloss/ds / B (Eq. 1 or softmax cross-entropy), and the hidden layer's d(pre-activation)

@@ -11,6 +11,9 @@
 //  - App. D (Assumption 4, theorem): the gradient applied at step k was
 //    computed with weights of version k - tau(k); updates apply in step order.
 //    Each party keeps its S+1 most recent weight versions in a ring.
+//  - Sec. 4.2 / Eq. 5 (ps_dt0 > 0): one replica of each party's parameters per
+//    worker, each worker's steps chained on its own stream pair, the replicas
+//    averaged after the epochs Eq. 5 selects.
 #include <algorithm>
 #include <cmath>
 #include <cstdarg>
@@ -42,12 +45,13 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_HEAD, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_HEAD, K_PS_AVG, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
-    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update", "head_loss"};
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update", "head_loss",
+    "ps_average"};
 
 struct ProfRec {
     int cls;
@@ -66,6 +70,8 @@ struct Layer {
     long long in_ld = 0;                  // leading dim of the compute copy of W
     float* W = nullptr;                   // fp32 master [out, in]
     float* b = nullptr;                   // fp32 master [out]
+    float* Wr[kMaxWorkers] = {};          // parameter-server mode: replica w's master (Wr[0] = W)
+    float* br[kMaxWorkers] = {};
     void* cW[kMaxSlots] = {};             // version copies [out, in_ld], compute dtype
     float* cb[kMaxSlots] = {};            // version copies of b, fp32
     float* pW[kMaxWorkers] = {};          // split-K partial dW [nsplit][out*in]
@@ -94,7 +100,7 @@ struct Carver {
 struct vfl_ctx {
     vfl_config cfg{};
     long long n_rows = 0;
-    int S1 = 1;                 // slots = staleness + 1
+    int S1 = 1;                 // slots = staleness + 1 (parameter-server mode: one per worker)
     int W = 1;                  // workers per party
     int esz = 4;                // bytes per compute element
     int bf16 = 0;
@@ -132,6 +138,12 @@ struct vfl_ctx {
     int f_act_ld = 0, f_wp = 0, f_wa = 0;       // smem row stride, weight-stage floats per party
     float* f_rowloss[kMaxWorkers] = {};         // per worker: per-row loss [B]
     float* f_zpc[kMaxWorkers] = {};             // per worker: z^p rows consumed by the step [B, ld8(e_p)]
+
+    // parameter-server mode (Sec. 4.2): replicas per worker, averaged per Eq. 5
+    bool psmode = false;
+    PsAvgLayer* ps_tab = nullptr;               // device table: P's layers, then A's, then T's
+    long long ps_total[2] = {};                 // flat parameter counts: passive, active (f_a and g)
+    cudaEvent_t ev_pavg[kEvPool] = {}, ev_aavg[kEvPool] = {};   // per aggregation step: averaging done
 
     // bf16 path: g's output layer and the loss in one launch (narrow output over a narrow hidden layer)
     bool head = false;
@@ -345,6 +357,9 @@ vfl_status check_config(const vfl_config* c, long long n_rows, std::string* why)
     if (!(c->lr >= 0.f)) return bad("lr must be >= 0");
     if (c->dp_clip < 0.f || c->dp_sigma < 0.f) return bad("dp_clip / dp_sigma must be >= 0");
     if (c->dp_target != VFL_DP_GRAD && c->dp_target != VFL_DP_EMB) return bad("unknown dp_target");
+    if (c->ps_dt0 < 0) return bad("ps_dt0 must be >= 0");
+    if (c->ps_dt0 > 0 && c->staleness != 0)
+        return bad("the parameter-server mode reads each replica's latest version: staleness must be 0");
     if (c->n_active + c->n_top > kMaxSgdLayers || c->n_passive > kMaxSgdLayers) return bad("too many layers");
     (void)buf;
     return VFL_OK;
@@ -486,6 +501,12 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
         for (Layer& L : *v) {
             L.W = static_cast<float*>(cv.take((unsigned long long)L.out * L.in * 4));
             L.b = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
+            L.Wr[0] = L.W;
+            L.br[0] = L.b;
+            for (int w = 1; ctx->psmode && w < ctx->W; ++w) {
+                L.Wr[w] = static_cast<float*>(cv.take((unsigned long long)L.out * L.in * 4));
+                L.br[w] = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
+            }
             for (int s = 0; s < ctx->S1; ++s) {
                 L.cW[s] = cv.take((unsigned long long)L.out * L.in_ld * es);
                 L.cb[s] = static_cast<float*>(cv.take((unsigned long long)L.out * 4));
@@ -528,6 +549,9 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
     ctx->emb_hdr = static_cast<ChannelHeader*>(cv.take(sizeof(ChannelHeader) * ctx->S1));
     ctx->grad_hdr = static_cast<ChannelHeader*>(cv.take(sizeof(ChannelHeader) * ctx->S1));
     ctx->losses = static_cast<float*>(cv.take(kLossCap * 4ull));
+    if (ctx->psmode)
+        ctx->ps_tab = static_cast<PsAvgLayer*>(
+            cv.take(sizeof(PsAvgLayer) * (ctx->P.size() + ctx->A.size() + ctx->T.size())));
     ctx->status = static_cast<int*>(cv.take(256));
     // scratch for taps and version reads/writes: a [B, widest] activation or a whole weight matrix
     long long maxw = std::max<long long>(c.d_passive, c.d_active);
@@ -563,6 +587,38 @@ inline cudaStream_t pstream(vfl_ctx* ctx, long long k) { return ctx->ps[k % ctx-
 
 // DP on the published embedding (App. C) rather than on its gradient
 inline bool emb_dp(const vfl_ctx* ctx) { return ctx->cfg.dp_clip > 0.f && ctx->cfg.dp_target == VFL_DP_EMB; }
+
+// ---- parameter-server mode (Sec. 4.2) ------------------------------------------------
+// Synchronization interval after epoch t (1-based), Eq. 5:
+// Delta T_t = ceil(Delta T_0 / 2 * tanh(2 t / Delta T_0 - 2) + Delta T_0 / 2).
+long long ps_interval(long long t, int dt0) {
+    const double h = dt0 / 2.0;
+    const long long v = (long long)std::ceil(h * std::tanh(2.0 * (double)t / dt0 - 2.0) + h);
+    return std::max<long long>(1, v);
+}
+// Whether the replicas are averaged right after step e: e ends epoch t and t mod Delta T_t == 0.
+bool ps_agg_at(const vfl_ctx* ctx, long long e) {
+    if (!ctx->psmode || e < 0 || (e + 1) % ctx->nb != 0) return false;
+    const long long t = (e + 1) / ctx->nb;
+    return t % ps_interval(t, ctx->cfg.ps_dt0) == 0;
+}
+// The latest averaging step a < k that step k must follow (a >= k - W: older ones are ordered
+// through the worker's own stream), or -1.
+long long ps_last_agg(const vfl_ctx* ctx, long long k) {
+    for (long long e = (k / ctx->nb) * ctx->nb - 1; e >= 0 && e >= k - ctx->W; e -= ctx->nb)
+        if (ps_agg_at(ctx, e)) return e;
+    return -1;
+}
+// Passive updates that must be enqueued before step k's publisher: its worker's previous step, and
+// the averaging it follows.
+long long ps_need_bwd(const vfl_ctx* ctx, long long k) {
+    return std::max(k - ctx->W + 1, ps_last_agg(ctx, k) + 1);
+}
+// Replica and version slot step k's worker reads and updates (the single master and ring otherwise).
+inline int ps_rep(const vfl_ctx* ctx, long long k) { return ctx->psmode ? (int)(k % ctx->W) : 0; }
+inline int new_version_slot(const vfl_ctx* ctx, long long k) {
+    return ctx->psmode ? (int)(k % ctx->W) : (int)((k + 1) % ctx->S1);
+}
 
 // Rows of step k (first row r0): the staging ring's slot when host data is bound, else the
 // device-resident dataset.  Both have the same row strides.
@@ -707,7 +763,8 @@ vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, l
     return VFL_OK;
 }
 
-vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w, int new_slot, cudaStream_t s) {
+vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w, int rep, int new_slot,
+               cudaStream_t s) {
     SgdArgs args;
     std::memset(&args, 0, sizeof args);
     long long off = 0;
@@ -716,7 +773,7 @@ vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w
         if (!v) continue;
         for (Layer& L : *v) {
             SgdLayer& d = args.L[n++];
-            d.W = L.W; d.b = L.b;
+            d.W = L.Wr[rep]; d.b = L.br[rep];
             d.pW = L.pW[w]; d.pb = L.pb[w];
             d.pW_stride = (long long)L.out * L.in;
             d.pb_stride = L.out;
@@ -791,8 +848,8 @@ FusedLayerArgs fused_layer(const Layer& L, int vslot, void* Y, long long ldy, vo
 }
 
 // Update of layer L from its d(pre) rows D and input rows [X | X2] (X2 from column xsplit on).
-FusedUpdLayer fused_upd_layer(const Layer& L, int new_slot, int w, const void* D, long long ldd, const void* X,
-                              long long ldx, const void* X2, long long ldx2, int xsplit) {
+FusedUpdLayer fused_upd_layer(const Layer& L, int new_slot, int rep, int w, const void* D, long long ldd,
+                              const void* X, long long ldx, const void* X2, long long ldx2, int xsplit) {
     FusedUpdLayer u;
     std::memset(&u, 0, sizeof u);
     u.out = L.out;
@@ -805,8 +862,8 @@ FusedUpdLayer fused_upd_layer(const Layer& L, int new_slot, int w, const void* D
     u.X2 = static_cast<const float*>(X2 ? X2 : X);
     u.ldx2 = X2 ? ldx2 : ldx;
     u.xsplit = X2 ? xsplit : L.in;
-    u.Wm = L.W;
-    u.bm = L.b;
+    u.Wm = L.Wr[rep];
+    u.bm = L.br[rep];
     u.Wc = static_cast<float*>(L.cW[new_slot]);
     u.bc = L.cb[new_slot];
     u.gW = L.pW[w];
@@ -933,7 +990,7 @@ vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float*
     FusedUpdArgs u;
     std::memset(&u, 0, sizeof u);
     const int La = (int)ctx->A.size(), Lt = (int)ctx->T.size();
-    const int new_slot = (int)((k + 1) % ctx->S1);
+    const int new_slot = new_version_slot(ctx, k), rp = ps_rep(ctx, k);
     const int n_out = ctx->T.back().out;
     const int ea = ctx->A.back().out, ep = ctx->P.back().out;
     int n = 0;
@@ -941,7 +998,7 @@ vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float*
         const Layer& L = ctx->A[l];
         const void* X = l == 0 ? (const void*)Xa : ctx->act_a[w][l - 1];
         const long long ldx = l == 0 ? ctx->ldxa : ld8(ctx->A[l - 1].out);
-        u.L[n++] = fused_upd_layer(L, new_slot, w, ctx->dpre_a[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
+        u.L[n++] = fused_upd_layer(L, new_slot, rp, w, ctx->dpre_a[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
     }
     u.L[0].x_early = 1;   // x^a's rows: every other input comes from the active step's row kernel
     for (int l = 0; l < Lt; ++l) {
@@ -950,10 +1007,11 @@ vfl_status fused_active_update(vfl_ctx* ctx, long long k, int rows, const float*
         const void* D = last ? (const void*)ctx->ds[w] : ctx->dpre_t[w][l];
         const long long ldd = last ? n_out : ld8(L.out);
         if (l == 0)
-            u.L[n++] = fused_upd_layer(L, new_slot, w, D, ldd, ctx->act_a[w][La - 1], ld8(ea), ctx->f_zpc[w], ld8(ep), ea);
+            u.L[n++] = fused_upd_layer(L, new_slot, rp, w, D, ldd, ctx->act_a[w][La - 1], ld8(ea), ctx->f_zpc[w],
+                                       ld8(ep), ea);
         else
-            u.L[n++] = fused_upd_layer(L, new_slot, w, D, ldd, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr,
-                                       0, 0);
+            u.L[n++] = fused_upd_layer(L, new_slot, rp, w, D, ldd, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out),
+                                       nullptr, 0, 0);
     }
     u.nl = n;
     u.rowloss = ctx->f_rowloss[w];
@@ -1000,12 +1058,12 @@ vfl_status fused_passive_update(vfl_ctx* ctx, long long k, int slot, int rows, c
     FusedUpdArgs u;
     std::memset(&u, 0, sizeof u);
     const int Lp = (int)ctx->P.size();
-    const int new_slot = (int)((k + 1) % ctx->S1);
+    const int new_slot = new_version_slot(ctx, k), rp = ps_rep(ctx, k);
     for (int l = 0; l < Lp; ++l) {
         const Layer& L = ctx->P[l];
         const void* X = l == 0 ? (const void*)Xp : ctx->act_p[slot][l - 1];
         const long long ldx = l == 0 ? ctx->ldxp : ld8(ctx->P[l - 1].out);
-        u.L[l] = fused_upd_layer(L, new_slot, w, ctx->dpre_p[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
+        u.L[l] = fused_upd_layer(L, new_slot, rp, w, ctx->dpre_p[w][l], ld8(L.out), X, ldx, nullptr, 0, 0);
         u.L[l].x_early = 1;   // x^p's rows and the forward's activations: only D comes from the backward
     }
     u.nl = Lp;
@@ -1036,6 +1094,46 @@ vfl_status stage_step(vfl_ctx* ctx, long long k) {
 }
 
 
+// ---- parameter-server aggregation ---------------------------------------------
+// After step e's update on its worker's stream s: wait for every other worker's latest update
+// (steps e-W+1 .. e-1; workers that have not run yet still hold the initial replica), then replace
+// the party's replicas by their mean.  The steps of the next W that read a replica wait for ev_*avg.
+vfl_status ps_average(vfl_ctx* ctx, long long e, bool passive, cudaStream_t s) {
+    cudaEvent_t* ev = passive ? ctx->ev_pver : ctx->ev_aver;
+    for (long long j = std::max(0ll, e - ctx->W + 1); j < e; ++j)
+        if (j + 1 > ctx->ordered_floor) TRY(wait_ev(ctx, s, ev[(j + 1) % kEvPool]));
+    const int first = passive ? 0 : (int)ctx->P.size();
+    const int n = passive ? (int)ctx->P.size() : (int)(ctx->A.size() + ctx->T.size());
+    const long long total = ctx->ps_total[passive ? 0 : 1];
+    // algorithmic bytes: every replica's master read and written, every compute copy written
+    const double bytes = (double)total * ctx->W * (8.0 + ctx->esz);
+    PLAUNCH(K_PS_AVG, (double)total * ctx->W, bytes, s,
+            launch_ps_average(ctx->ps_tab + first, n, total, ctx->W, ctx->bf16, s));
+    CK(cudaEventRecord((passive ? ctx->ev_pavg : ctx->ev_aavg)[e % kEvPool], s));
+    return VFL_OK;
+}
+
+// Before step k's first launch on party stream s: in the parameter-server mode, wait for the
+// averaging it follows (its replica's own chain is ordered by the stream); otherwise for the
+// update that produced version v.
+vfl_status wait_version(vfl_ctx* ctx, long long k, long long v, bool passive, cudaStream_t s) {
+    if (ctx->psmode) {
+        const long long a = ps_last_agg(ctx, k);
+        if (a >= 0 && a + 1 > ctx->ordered_floor)
+            TRY(wait_ev(ctx, s, (passive ? ctx->ev_pavg : ctx->ev_aavg)[a % kEvPool]));
+        return VFL_OK;
+    }
+    if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, (passive ? ctx->ev_pver : ctx->ev_aver)[v % kEvPool]));
+    return VFL_OK;
+}
+
+// Before step k's update on s: updates apply in step order (App. D); in the parameter-server mode
+// the replica's previous update ran on the same stream.
+vfl_status wait_update_order(vfl_ctx* ctx, long long k, bool passive, cudaStream_t s) {
+    if (ctx->psmode || k <= 0 || k <= ctx->ordered_floor) return VFL_OK;
+    return wait_ev(ctx, s, (passive ? ctx->ev_pver : ctx->ev_aver)[k % kEvPool]);
+}
+
 // ---- the three phases ------------------------------------------------------
 vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     const vfl_config& c = ctx->cfg;
@@ -1044,16 +1142,21 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
         return ctx->fail(VFL_E_STATE, "passive_forward(%lld): tau_p=%d outside [0, min(k, S=%d)]", k, tau_p, c.staleness);
     const long long v = k - tau_p;
     const long long u = ctx->n_bwd;  // passive updates enqueued
-    if (v > u)
+    if (ctx->psmode) {
+        if (u < ps_need_bwd(ctx, k))
+            return ctx->fail(VFL_E_STATE, "passive_forward(%lld): the update or averaging its replica follows is not "
+                             "enqueued yet (%lld updates)", k, u);
+    } else if (v > u) {
         return ctx->fail(VFL_E_STATE, "passive_forward(%lld): passive version %lld not produced yet (%lld updates)", k, v, u);
-    if (v < u - c.staleness)
+    } else if (v < u - c.staleness) {
         return ctx->fail(VFL_E_STATE, "passive_forward(%lld): passive version %lld no longer stored", k, v);
+    }
     cudaStream_t s = pstream(ctx, k);
     const int slot = (int)(k % ctx->S1);
     const int vslot = (int)(v % ctx->S1);
     long long r0;
     const int rows = ctx->batch_rows(k, &r0);
-    if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[v % kEvPool]));
+    TRY(wait_version(ctx, k, v, true, s));
     if (ctx->hio) {
         TRY(stage_step(ctx, k));
         TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
@@ -1109,7 +1212,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const int ea = ctx->A.back().out, ep = ctx->P.back().out;
     const int n_out = ctx->T.back().out;
 
-    if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[v % kEvPool]));
+    TRY(wait_version(ctx, k, v, false, s));
     if (ctx->hio) TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
     const void* Xa0 = xa_rows(ctx, k, r0);
     if (ctx->fused) {
@@ -1118,10 +1221,11 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         note_node(ctx, CAP_ACTIVE, k, s);
         CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
         // SGD on theta_1 in step order: version k+1 from version k
-        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
+        TRY(wait_update_order(ctx, k, false, s));
         TRY(fused_active_update(ctx, k, rows, static_cast<const float*>(Xa0), w, s));
         note_node(ctx, CAP_AUPD, k, s);
         CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
+        if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
         ctx->grad_step[slot] = k;
         ctx->last_act_step[w] = k;
         ctx->n_act = k + 1;
@@ -1227,9 +1331,10 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         }
     }
     // SGD on theta_1 in step order: version k+1 from version k
-    if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_aver[k % kEvPool]));
-    TRY(sgd(ctx, &ctx->A, &ctx->T, w, (int)((k + 1) % ctx->S1), s));
+    TRY(wait_update_order(ctx, k, false, s));
+    TRY(sgd(ctx, &ctx->A, &ctx->T, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
     CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
+    if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
     ctx->last_act_step[w] = k;
     ctx->n_act = k + 1;
     return VFL_OK;
@@ -1252,10 +1357,11 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
         note_node(ctx, CAP_PBWD, k, s);
         // SGD on theta_2 in step order
-        if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
+        TRY(wait_update_order(ctx, k, true, s));
         TRY(fused_passive_update(ctx, k, slot, rows, Xp, w, s));
         note_node(ctx, CAP_PUPD, k, s);
         CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
+        if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, true, s));
         ctx->n_bwd = k + 1;
         return VFL_OK;
     }
@@ -1277,9 +1383,10 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
                           ctx->act_p[slot][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
     }
-    if (k > 0 && k > ctx->ordered_floor) TRY(wait_ev(ctx, s, ctx->ev_pver[k % kEvPool]));
-    TRY(sgd(ctx, &ctx->P, nullptr, w, (int)((k + 1) % ctx->S1), s));
+    TRY(wait_update_order(ctx, k, true, s));
+    TRY(sgd(ctx, &ctx->P, nullptr, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
     CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
+    if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, true, s));
     ctx->n_bwd = k + 1;
     return VFL_OK;
 }
@@ -1344,8 +1451,9 @@ vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* 
     vfl_ctx tmp;
     tmp.cfg = *cfg;
     tmp.n_rows = n_rows;
-    tmp.S1 = cfg->staleness + 1;
+    tmp.psmode = cfg->ps_dt0 > 0;
     tmp.W = cfg->workers;
+    tmp.S1 = tmp.psmode ? tmp.W : cfg->staleness + 1;
     tmp.bf16 = cfg->dtype == VFL_BF16;
     tmp.esz = tmp.bf16 ? 2 : 4;
     tmp.fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
@@ -1372,8 +1480,9 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     vfl_ctx* ctx = new vfl_ctx();
     ctx->cfg = *cfg;
     ctx->n_rows = n_rows;
-    ctx->S1 = cfg->staleness + 1;
+    ctx->psmode = cfg->ps_dt0 > 0;
     ctx->W = cfg->workers;
+    ctx->S1 = ctx->psmode ? ctx->W : cfg->staleness + 1;
     ctx->bf16 = cfg->dtype == VFL_BF16;
     ctx->esz = ctx->bf16 ? 2 : 4;
     ctx->nb = (int)((n_rows + cfg->batch - 1) / cfg->batch);
@@ -1397,10 +1506,36 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_emb[i], cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_grad[i], cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_staged[i], cudaEventDisableTiming);
+        if (e == cudaSuccess && ctx->psmode) e = cudaEventCreateWithFlags(&ctx->ev_pavg[i], cudaEventDisableTiming);
+        if (e == cudaSuccess && ctx->psmode) e = cudaEventCreateWithFlags(&ctx->ev_aavg[i], cudaEventDisableTiming);
     }
     if (e == cudaSuccess) e = cudaMemset(workspace, 0, need);
     if (e == cudaSuccess) e = cudaMemset(ctx->emb_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
     if (e == cudaSuccess) e = cudaMemset(ctx->grad_hdr, 0xFF, sizeof(ChannelHeader) * ctx->S1);
+    if (e == cudaSuccess && ctx->psmode) {
+        // the averaging kernel's layer table: per party, flat offsets from 0
+        std::vector<PsAvgLayer> tab;
+        for (std::vector<Layer>* v : {&ctx->P, &ctx->A, &ctx->T}) {
+            long long& total = ctx->ps_total[v == &ctx->P ? 0 : 1];
+            for (const Layer& L : *v) {
+                PsAvgLayer t;
+                std::memset(&t, 0, sizeof t);
+                for (int w = 0; w < ctx->W; ++w) {
+                    t.Wr[w] = L.Wr[w];
+                    t.br[w] = L.br[w];
+                    t.cW[w] = L.cW[w];
+                    t.cb[w] = L.cb[w];
+                }
+                t.out = L.out;
+                t.in = L.in;
+                t.in_ld = L.in_ld;
+                t.begin = total;
+                total += (long long)L.out * L.in + L.out;
+                tab.push_back(t);
+            }
+        }
+        e = cudaMemcpy(ctx->ps_tab, tab.data(), sizeof(PsAvgLayer) * tab.size(), cudaMemcpyHostToDevice);
+    }
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         g_global_err = std::string("vfl_create: ") + cudaGetErrorString(e);
@@ -1430,6 +1565,8 @@ vfl_status vfl_destroy(vfl_ctx* ctx) {
         if (ctx->ev_emb[i]) cudaEventDestroy(ctx->ev_emb[i]);
         if (ctx->ev_grad[i]) cudaEventDestroy(ctx->ev_grad[i]);
         if (ctx->ev_staged[i]) cudaEventDestroy(ctx->ev_staged[i]);
+        if (ctx->ev_pavg[i]) cudaEventDestroy(ctx->ev_pavg[i]);
+        if (ctx->ev_aavg[i]) cudaEventDestroy(ctx->ev_aavg[i]);
     }
     delete ctx;
     return VFL_OK;
@@ -1541,8 +1678,11 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
     if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
     TRY(sync_all(ctx));
     const size_t nw = (size_t)L->out * L->in;
-    CK(cudaMemcpy(L->W, W, nw * 4, cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(L->b, b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    // every replica (one unless in the parameter-server mode) starts from the same master
+    for (int w = 0; w < (ctx->psmode ? ctx->W : 1); ++w) {
+        CK(cudaMemcpy(L->Wr[w], W, nw * 4, cudaMemcpyHostToDevice));
+        CK(cudaMemcpy(L->br[w], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    }
     // every version slot gets the same compute copy (padding columns stay zero)
     for (int s = 0; s < ctx->S1; ++s) {
         CK(cudaMemset(L->cW[s], 0, (size_t)L->out * L->in_ld * ctx->esz));
@@ -1618,6 +1758,7 @@ vfl_status vfl_get_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
     if (ctx->broken) return VFL_E_CUDA;
     Layer* L = find_layer(ctx, party, layer);
     if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    if (ctx->psmode) return ctx->fail(VFL_E_STATE, "the parameter-server mode stores replicas: use vfl_get_replica");
     int64_t k = 0;
     TRY(vfl_step_cursor(ctx, &k));
     if (v < std::max<int64_t>(0, k - ctx->cfg.staleness) || v > k)
@@ -1637,6 +1778,7 @@ vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
     if (ctx->broken) return VFL_E_CUDA;
     Layer* L = find_layer(ctx, party, layer);
     if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    if (ctx->psmode) return ctx->fail(VFL_E_STATE, "the parameter-server mode stores replicas: use vfl_set_replica");
     int64_t k = 0;
     TRY(vfl_step_cursor(ctx, &k));
     if (v < std::max<int64_t>(0, k - ctx->cfg.staleness) || v > k)
@@ -1657,6 +1799,49 @@ vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v
         CK(cudaMemcpy(L->b, b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
     }
     CK(cudaDeviceSynchronize());
+    return VFL_OK;
+}
+
+vfl_status vfl_get_replica(vfl_ctx* ctx, int32_t worker, int32_t party, int32_t layer, float* W, float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null output pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (!ctx->psmode) return ctx->fail(VFL_E_STATE, "replicas exist only in the parameter-server mode");
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
+    int64_t k = 0;
+    TRY(vfl_step_cursor(ctx, &k));
+    TRY(sync_all(ctx));
+    CK(cudaMemcpy(W, L->Wr[worker], (size_t)L->out * L->in * 4, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(b, L->br[worker], (size_t)L->out * 4, cudaMemcpyDeviceToHost));
+    return VFL_OK;
+}
+
+vfl_status vfl_set_replica(vfl_ctx* ctx, int32_t worker, int32_t party, int32_t layer, const float* W, const float* b) {
+    if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null parameter pointer") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (!ctx->psmode) return ctx->fail(VFL_E_STATE, "replicas exist only in the parameter-server mode");
+    Layer* L = find_layer(ctx, party, layer);
+    if (!L) return ctx->fail(VFL_E_INVAL, "no layer %d of party %d", layer, party);
+    if (worker < 0 || worker >= ctx->W) return ctx->fail(VFL_E_INVAL, "worker %d out of range", worker);
+    int64_t k = 0;
+    TRY(vfl_step_cursor(ctx, &k));
+    TRY(sync_all(ctx));
+    const size_t nw = (size_t)L->out * L->in;
+    CK(cudaMemcpy(L->Wr[worker], W, nw * 4, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(L->br[worker], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    // replica w's compute copy is version slot w, the cast of its master
+    CK(cudaMemset(L->cW[worker], 0, (size_t)L->out * L->in_ld * ctx->esz));
+    ++ctx->launches;
+    CK(launch_cast_rows(L->Wr[worker], L->out, L->in, L->cW[worker], L->in_ld, ctx->bf16, 0));
+    CK(cudaMemcpy(L->cb[worker], b, (size_t)L->out * 4, cudaMemcpyHostToDevice));
+    CK(cudaDeviceSynchronize());
+    return VFL_OK;
+}
+
+vfl_status vfl_ps_interval(int64_t t, int32_t dt0, int64_t* interval) {
+    if (t < 1 || dt0 < 1 || !interval) return VFL_E_INVAL;
+    *interval = ps_interval(t, dt0);
     return VFL_OK;
 }
 
@@ -1739,7 +1924,7 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
     // is queued ahead of the backward of step k whenever tau_p permits.
     while (ctx->n_bwd < end) {
         bool progressed = false;
-        while (ctx->n_fwd < end && ctx->n_fwd - tau_p[ctx->n_fwd] <= ctx->n_bwd) {
+        while (ctx->n_fwd < end && (ctx->psmode ? ps_need_bwd(ctx, ctx->n_fwd) : ctx->n_fwd - tau_p[ctx->n_fwd]) <= ctx->n_bwd) {
             TRY(do_passive_forward(ctx, ctx->n_fwd, tau_p[ctx->n_fwd]));
             progressed = true;
         }
@@ -1793,8 +1978,10 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
             cudaGraphNode_t from = node(ed.first, k), to = node(ed.second, k);
             if (from && to) make_programmatic(g, from, to);
         }
-        const long long v = k - tau_p[k];   // version of the forward: made by the update of step v - 1
-        cudaGraphNode_t from = node(CAP_PUPD, v - 1), to = node(CAP_PFWD, k);
+        // the update that made the forward's weights: step v - 1 for version v = k - tau_p, the previous
+        // step of the worker in the parameter-server mode (no edge when an averaging sits in between)
+        const long long src = ctx->psmode ? k - ctx->W : k - tau_p[k] - 1;
+        cudaGraphNode_t from = node(CAP_PUPD, src), to = node(CAP_PFWD, k);
         if (from && to) make_programmatic(g, from, to);
     }
 }

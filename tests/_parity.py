@@ -90,7 +90,8 @@ def compare_step(vfl, ctx, rec, tol, check_grads=True):
                                          max(np.abs(ref).max(), scale, 1e-30))
             else:
                 errs[f"db{key}"] = tensor_err(db, rec.grads[key][1], dt)
-    params = ctx.get_params()
+    # the parameter-server mode: the replica the step updated (the oracle records the same one)
+    params = ctx.get_replica(k % ctx.p.workers) if ctx.ps else ctx.get_params()
     for key, (W, b) in params.items():
         errs[f"W{key}"] = tensor_err(W, rec.params[key][0], dt)
         errs[f"b{key}"] = tensor_err(b, rec.params[key][1], dt)
@@ -113,9 +114,14 @@ def oracle_version(o, v):
 
 def force_gpu_state(ctx, o, S):
     """Put the GPU context into the oracle's state before step o.k: cursor and
-    every stored weight version (oracle -> GPU only)."""
+    every stored weight version, or every replica in the parameter-server mode
+    (oracle -> GPU only)."""
     k = o.k
     ctx.set_cursor(k)
+    if ctx.ps:
+        for w in range(ctx.p.workers):
+            ctx.set_replica(w, o.replica_params(w))
+        return
     for v in range(max(0, k - S), k + 1):
         ctx.set_version(v, oracle_version(o, v))
 

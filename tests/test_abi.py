@@ -39,10 +39,11 @@ def test_library_exports_every_declared_function(vfl):
 
 def test_config_struct_layout_matches_header(vfl):
     # 5 + 3*8 int32, then loss, dtype, batch, lr, staleness, workers, clip, sigma (4 bytes each), then u64,
-    # then the int32 dp_target and 4 bytes of tail padding
+    # then the int32 dp_target and ps_dt0
     assert ctypes.sizeof(vfl.VflConfig) == (5 + 24 + 8) * 4 + 4 + 8 + 8
     assert vfl.VflConfig.dp_seed.offset % 8 == 0
     assert vfl.VflConfig.dp_target.offset == vfl.VflConfig.dp_seed.offset + 8
+    assert vfl.VflConfig.ps_dt0.offset == vfl.VflConfig.dp_target.offset + 4
 
 
 @pytest.mark.parametrize("S", [0, 1, 2, 4, 7])
@@ -88,8 +89,34 @@ def test_invalid_configs_are_rejected(vfl):
             vfl.workspace_bytes(p.with_(**bad), 100)
     with pytest.raises(vfl.VflError):
         vfl.workspace_bytes(p, 0)
+    for bad in (dict(ps_dt0=-1), dict(ps_dt0=4, staleness=1, workers=2)):
+        with pytest.raises(vfl.VflError):
+            vfl.workspace_bytes(p.with_(**bad), 100)
     cfg = vfl.make_config(p.with_(dp_clip=1.0, dp_target="emb"))
     assert cfg.dp_target == vfl.DP_EMB
     cfg.dp_target = 7
     out = ctypes.c_uint64()
     assert vfl.lib().vfl_workspace_bytes(ctypes.byref(cfg), 100, ctypes.byref(out)) == vfl.VFL_E_INVAL
+
+
+@pytest.mark.parametrize("dt0", [1, 2, 3, 4, 5, 8, 13, 40])
+def test_ps_interval_matches_the_oracle(vfl, dt0):
+    for t in range(1, 6 * dt0 + 3):
+        assert vfl.ps_interval(t, dt0) == oracle.ps_interval(t, dt0), (t, dt0)
+    with pytest.raises(vfl.VflError):
+        vfl.ps_interval(0, dt0)
+    with pytest.raises(vfl.VflError):
+        vfl.ps_interval(1, 0)
+
+
+def test_ps_workspace_holds_a_master_per_replica(vfl):
+    p = synth.preset(2).with_(workers=4, staleness=0)
+    base = vfl.workspace_bytes(p, p.n_rows)
+    with_ps = vfl.workspace_bytes(p.with_(ps_dt0=4), p.n_rows)
+    n_params = 0
+    for widths, d_in in ((p.passive, p.d_passive), (p.active, p.d_active), (p.top, p.e_active + p.e_passive)):
+        for o in widths:
+            n_params += o * d_in + o
+            d_in = o
+    # three more fp32 masters (and the version ring grows from one slot to one per worker)
+    assert with_ps - base >= 3 * n_params * 4
