@@ -596,9 +596,10 @@ long long ps_interval(long long t, int dt0) {
     const long long v = (long long)std::ceil(h * std::tanh(2.0 * (double)t / dt0 - 2.0) + h);
     return std::max<long long>(1, v);
 }
-// Whether the replicas are averaged right after step e: e ends epoch t and t mod Delta T_t == 0.
+// Whether the replicas are averaged right after step e: e ends epoch t and t mod Delta T_t == 0
+// (with one worker the mean is the replica itself and nothing is launched).
 bool ps_agg_at(const vfl_ctx* ctx, long long e) {
-    if (!ctx->psmode || e < 0 || (e + 1) % ctx->nb != 0) return false;
+    if (!ctx->psmode || ctx->W < 2 || e < 0 || (e + 1) % ctx->nb != 0) return false;
     const long long t = (e + 1) / ctx->nb;
     return t % ps_interval(t, ctx->cfg.ps_dt0) == 0;
 }
