@@ -55,6 +55,16 @@ Readings where the paper is silent (each is listed in the design doc):
   the workers in order, divided by W) and every replica takes the average when
   t mod Delta T_t == 0, Delta T_t = ceil(Delta T_0 / 2 tanh(2 t / Delta T_0 - 2)
   + Delta T_0 / 2) (Eq. 5).
+* Waiting deadline and buffer overflow (Sec. 4.1, Algorithm 1's subscriber
+  branch): a step whose embedding the subscriber does not get (deadline passed,
+  or dropped oldest-first from a full buffer) is dropped: its publisher's work
+  is discarded, nothing else runs, no loss is recorded and neither party's
+  parameters change (version k+1 = version k), and its batch is reassigned to
+  the next step.  Step k therefore trains batch j = (k - D(k)) mod nb, D(k) the
+  drops before k; an epoch ends with the step that completes batch nb - 1.
+  Drops come in as a per-step 0/1 input; make_drops draws them: step k drops
+  when word 0 of Philox(key=(seed lo, seed hi), ctr=(k lo, k hi, 2, 0x4452)) is
+  below floor(rate 2^32).
 * bf16 presets round to bf16 (round-to-nearest-even, via fp32) at: the inputs,
   each weight version's compute copy (biases stay fp32), every stored hidden
   activation and embedding, and every activation gradient handed from one layer
@@ -80,6 +90,7 @@ _U32 = 0xFFFFFFFF
 TAG_SCHED = 0x5343      # counter word 3 of the staleness-schedule draws
 TAG_DP = 0x4450         # counter word 3 of the DP noise draws on the published gradient
 TAG_DPE = 0x4445        # counter word 3 of the DP noise draws on the published embedding
+TAG_DROP = 0x4452       # counter word 3 of the waiting-deadline drop draws
 
 
 def philox(ctr, key):
@@ -271,6 +282,19 @@ def dp_embed(z, k: int, clip: float, sigma: float, seed: int):
     return out, c
 
 
+def make_drops(seed: int, rate: float, n_steps: int):
+    """uint8 [n_steps]: 1 where the step is dropped (waiting deadline), drawn as
+    word 0 of Philox(key=(seed lo, seed hi), ctr=(k lo, k hi, 2, TAG_DROP)) below
+    floor(rate * 2^32), rate in [0, 1]."""
+    if not (0.0 <= rate <= 1.0) or n_steps < 0:
+        raise ValueError("rate must be in [0, 1] and n_steps >= 0")
+    k = np.arange(n_steps, dtype=np.uint64)
+    u = philox((k & np.uint64(_U32), k >> np.uint64(32), np.uint64(2), np.uint64(TAG_DROP)),
+               (seed & _U32, (seed >> 32) & _U32))[0]
+    thr = min(1 << 32, int(math.floor(rate * 4294967296.0)))
+    return (u.astype(np.uint64) < np.uint64(thr)).astype(np.uint8) if thr < (1 << 32) else np.ones(n_steps, np.uint8)
+
+
 def ps_interval(t: int, dt0: int) -> int:
     """Synchronization interval Delta T_t of the intra-party parameter server
     after epoch t (Eq. 5)."""
@@ -314,6 +338,7 @@ class StepRecord:
     dza: np.ndarray = None       # [B_k, e_a]
     grads: dict = None           # (party, layer) -> (dW, db)
     params: dict = None          # (party, layer) -> (W, b) after this step
+    dropped: bool = False        # waiting deadline: nothing trained, batch reassigned to the next step
 
 
 @dataclass
@@ -335,6 +360,7 @@ class Oracle:
     channel_g: dict = field(default_factory=dict)
     emb_scale: dict = field(default_factory=dict)   # step -> per-row clip factors of its published embedding
     replicas: list = None                            # parameter-server mode: [(P, A, T)] per worker
+    n_done: int = 0                                  # batches trained (steps not dropped)
 
     def __post_init__(self):
         c = self.cfg
@@ -361,17 +387,33 @@ class Oracle:
     def _compute(self, layers):
         return [(_store(W, self.dtype), b) for W, b in layers]
 
-    def batch_rows(self, k: int):
-        j = k % self.nb
+    def batch_rows(self, k: int = None):
+        """Batch id and rows of the next step (the batch after the last one trained;
+        without drops, step k's batch is k mod nb)."""
+        j = self.n_done % self.nb if k is None or k == self.k else k % self.nb
         r0 = j * self.cfg.batch
         return j, r0, min(self.n, r0 + self.cfg.batch)
 
-    def step(self, tau_p: int, tau_a: int, record: bool = False) -> StepRecord:
+    def step(self, tau_p: int, tau_a: int, record: bool = False, drop: bool = False) -> StepRecord:
         c = self.cfg
         k = self.k
         if not (0 <= tau_p <= min(k, c.staleness) and 0 <= tau_a <= min(k, c.staleness)):
             raise ValueError(f"step {k}: staleness ({tau_p}, {tau_a}) outside [0, min(k, S={c.staleness})]")
-        j, r0, r1 = self.batch_rows(k)
+        j, r0, r1 = self.batch_rows()
+        if drop:
+            # the subscriber gave up on the embedding: no loss, no update, the batch goes to step k+1
+            self.versions_p[k + 1] = self.versions_p[k]
+            self.versions_a[k + 1] = self.versions_a[k]
+            for d in (self.versions_p, self.versions_a):
+                for v in [v for v in d if v < k + 1 - c.staleness]:
+                    del d[v]
+            self.k = k + 1
+            rec = StepRecord(k, j, (r0, r1), tau_p, tau_a, k - tau_p, k - tau_a, float("nan"), dropped=True)
+            if record and self.ps:
+                rec.params = self.replica_params(k % c.workers)
+            elif record:
+                rec.params = self.current_params()
+            return rec
         Bk = r1 - r0
         vp, va = k - tau_p, k - tau_a
         if self.ps:   # worker pair k mod W serves the step with its own replicas
@@ -428,7 +470,7 @@ class Oracle:
         newT = [(W - lr * dW, b - lr * db) for (W, b), (dW, db) in zip(curT, gT)]
         if self.ps:
             self.replicas[k % c.workers] = (newP, newA, newT)
-            if (k + 1) % self.nb == 0 and ps_aggregates_after((k + 1) // self.nb, c.ps_dt0):
+            if j == self.nb - 1 and ps_aggregates_after((self.n_done + 1) // self.nb, c.ps_dt0):
                 self._ps_average()
             newP, newA, newT = self.replicas[0]      # the stored version: replica 0 (see current_params)
         self.versions_p[k + 1] = newP
@@ -438,6 +480,7 @@ class Oracle:
             for v in [v for v in d if v < k + 1 - c.staleness]:
                 del d[v]
         self.k = k + 1
+        self.n_done += 1
 
         rec = StepRecord(k, j, (r0, r1), tau_p, tau_a, vp, va, float(loss))
         if record:
@@ -483,13 +526,14 @@ class Oracle:
                 out[(party, l)] = (W.copy(), b.copy())
         return out
 
-    def run(self, tau_p, tau_a, n_steps: int, record_steps=()):
-        """n_steps steps from the current k; returns (per-step mean losses, records)."""
+    def run(self, tau_p, tau_a, n_steps: int, record_steps=(), drops=None):
+        """n_steps steps from the current k; returns (per-step mean losses, NaN for a
+        dropped step; records)."""
         losses, recs = [], {}
         rs = set(record_steps)
         for _ in range(n_steps):
             k = self.k
-            r = self.step(int(tau_p[k]), int(tau_a[k]), record=k in rs)
+            r = self.step(int(tau_p[k]), int(tau_a[k]), record=k in rs, drop=drops is not None and bool(drops[k]))
             losses.append(r.loss)
             if k in rs:
                 recs[k] = r
