@@ -50,6 +50,9 @@ def parse(argv=None):
     ap.add_argument("--ps-dt0", type=int, default=0, metavar="DT0",
                     help="intra-party parameter server (Eq. 5): per-worker replicas averaged per Delta T_0 = DT0 "
                          "(sets the staleness to 0)")
+    ap.add_argument("--drop-rate", type=float, default=0.0, metavar="R",
+                    help="waiting-deadline drops: each step's subscriber gives up with probability R (seeded draws); "
+                         "dropped steps train nothing and count no samples")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -80,7 +83,9 @@ def workload(args):
             (f", DP on the {'embedding' if p.dp_target == 'emb' else 'embedding gradient'} C={p.dp_clip} "
              f"sigma={p.dp_sigma}" if p.dp_clip else "") +
             (f", parameter server per worker (replicas averaged per Eq. 5, Delta T_0={p.ps_dt0})"
-             if p.ps_dt0 else ""))
+             if p.ps_dt0 else "") +
+            (f", waiting-deadline drops at rate {args.drop_rate} (batch reassigned to the next step)"
+             if getattr(args, "drop_rate", 0.0) else ""))
     return p, desc
 
 
@@ -94,8 +99,16 @@ def rows_of(p, k):
     return r0, min(p.n_rows, r0 + p.batch)
 
 
-def samples(p, k0, n):
-    return sum(rows_of(p, k)[1] - rows_of(p, k)[0] for k in range(k0, k0 + n))
+def samples(p, k0, n, drops=None):
+    """Rows trained by steps [k0, k0+n): a dropped step trains none and hands its batch to the next."""
+    if drops is None:
+        return sum(rows_of(p, k)[1] - rows_of(p, k)[0] for k in range(k0, k0 + n))
+    tot = 0
+    for k in range(k0, k0 + n):
+        if not drops[k]:
+            r0, r1 = rows_of(p, k - int(drops[:k].sum()))
+            tot += r1 - r0
+    return tot
 
 
 def sched_kind(p):
@@ -163,11 +176,12 @@ xp, xa, y = synth.make_dataset(p, rows=(0, rows))
 q = p.with_(n_rows=rows)
 params = synth.init_params(q)
 tp, ta = oracle.make_schedule(q.seed, q.staleness, {kind}, n_steps)
+drops = oracle.make_drops(q.seed, {drop_rate}, n_steps)
 o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
 t0 = time.perf_counter(); done = 0; nsamp = 0
 while done < n_steps:
-    r = o.step(int(tp[done]), int(ta[done]))
-    nsamp += r.rows[1] - r.rows[0]
+    r = o.step(int(tp[done]), int(ta[done]), drop=bool(drops[done]))
+    nsamp += 0 if r.dropped else r.rows[1] - r.rows[0]
     done += 1
     if time.perf_counter() - t0 > {budget}: break
 dt = time.perf_counter() - t0
@@ -182,7 +196,8 @@ def run_oracle(p, args, n_steps, budget):
         env[v] = str(cores)
     env["CUDA_VISIBLE_DEVICES"] = ""
     fields = {f: getattr(p, f) for f in p.__dataclass_fields__}
-    code = CPU_SNIPPET.format(root=ROOT, fields=fields, n_steps=n_steps, kind=sched_kind(p), budget=budget)
+    code = CPU_SNIPPET.format(root=ROOT, fields=fields, n_steps=n_steps, kind=sched_kind(p), budget=budget,
+                              drop_rate=float(args.drop_rate))
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle timing failed: {r.stderr[-2000:]}")
@@ -326,6 +341,7 @@ def run_ours(args):
     W, K = args.warmup, args.steps
     total = W + 3 * K
     tp, ta = vfl.make_schedule(p.seed, p.staleness, sched_kind(p), total)
+    drops = vfl.make_drops(p.seed, args.drop_rate, total) if args.drop_rate > 0 else None
     ctx = vfl.Context(p, p.n_rows)
     ctx.load_data(xp, xa, y)
     ctx.set_params(params)
@@ -344,7 +360,7 @@ def run_ours(args):
             ctx.profile(True)
         while k < k0 + n:
             m = min(nb, k0 + n - k)
-            graph = ctx.capture(k, m, tp, ta) if use_graphs else None
+            graph = ctx.capture(k, m, tp, ta, drops) if use_graphs else None
             with torch.cuda.stream(main):
                 flush.zero_()
                 # keep the GPU busy while the host enqueues this iteration, so that the host's launch
@@ -358,7 +374,7 @@ def run_ours(args):
             if graph is not None:
                 ctx.launch_graph(graph)
             else:
-                ctx.train_steps(k, m, tp, ta)
+                ctx.train_steps(k, m, tp, ta, drops)
             for s in ctx.streams:
                 ev = torch.cuda.Event()
                 ev.record(s)
@@ -374,7 +390,7 @@ def run_ours(args):
         return total_ms, prof
 
     # warm-up
-    ctx.train_steps(0, W, tp, ta)
+    ctx.train_steps(0, W, tp, ta, drops)
     ctx.synchronize()
     if world > 1:
         torch.distributed.barrier()
@@ -386,7 +402,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = slowest_rank(ms)
-    value = job_throughput(samples(p, W, K), world, ms / 1e3)
+    value = job_throughput(samples(p, W, K, drops), world, ms / 1e3)
 
     # per-kernel timing: the same workload again, every launch bracketed by CUDA events (recorded
     # inside the replayed graphs when graphs are on, so each duration is the kernel as the step runs it)
@@ -408,13 +424,14 @@ def run_ours(args):
         k0 = W + 2 * K
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        ctx.train_steps(k0, K, tp, ta)
+        ctx.train_steps(k0, K, tp, ta, drops)
         ctx.synchronize()
         dt = slowest_rank(time.perf_counter() - t0)
         ctx.bind_host_data(None, None, None)
-        assert np.isfinite(loss_host.numpy()).all()
+        kept = np.ones(K, bool) if drops is None else drops[k0:k0 + K] == 0
+        assert np.isfinite(loss_host.numpy()[kept]).all() and np.isnan(loss_host.numpy()[~kept]).all()
         h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
-        e2e = {"value": job_throughput(samples(p, k0, K), world, dt), "unit": "samples/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": job_throughput(samples(p, k0, K, drops), world, dt), "unit": "samples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": 4}
 
     if rank == 0:

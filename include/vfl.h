@@ -257,14 +257,41 @@ vfl_status vfl_active_step(vfl_ctx* ctx, int64_t k, int32_t tau_a);
 vfl_status vfl_passive_backward(vfl_ctx* ctx, int64_t k);
 
 /*
+ * Waiting deadline / buffer overflow (Sec. 4.1; Algorithm 1's subscriber branch):
+ * the subscriber of step k gives up on its embedding (it did not arrive within
+ * the deadline, or a full buffer discarded it oldest-first).  Called instead of
+ * vfl_active_step(k): step k trains nothing, records a NaN loss, and both
+ * parties' version k+1 equals version k; vfl_passive_backward(k) is still called
+ * (the passive party is notified: it skips its backward and carries its version
+ * forward).  The batch of step k is reassigned to step k+1: step k trains batch
+ * (k - D) mod nb, D the drops before k.  Valid when step k is the next active
+ * step and no later step has been published (its batch would change); if step
+ * k was never published, its publish is skipped.
+ * vfl_get_drops / vfl_set_drops read and (with no step in flight, for restoring
+ * a checkpoint after vfl_set_cursor) set D for the next step.
+ */
+vfl_status vfl_drop_step(vfl_ctx* ctx, int64_t k);
+vfl_status vfl_get_drops(vfl_ctx* ctx, int64_t* n_drops);
+vfl_status vfl_set_drops(vfl_ctx* ctx, int64_t n_drops);
+
+/*
+ * Seeded drop draws (host only, pure): drop[k] = 1 when word 0 of
+ * Philox4x32-10(key = (seed lo, seed hi), counter = (k lo, k hi, 2, 0x4452)) is
+ * below floor(rate * 2^32) (every step when rate == 1).  VFL_E_INVAL unless
+ * 0 <= rate <= 1.
+ */
+vfl_status vfl_make_drops(uint64_t seed, double rate, int64_t n_steps, uint8_t* drop);
+
+/*
  * Enqueue steps [k0, k0 + n_steps) as one dependency graph across the worker
  * streams: each publisher phase runs as soon as its weight version exists, so
  * the parties overlap as far as tau allows.  tau_p / tau_a are host arrays
- * indexed by absolute step (length >= k0 + n_steps).  Same contract as the three
- * per-phase calls.
+ * indexed by absolute step (length >= k0 + n_steps).  `drop` (NULL: none) marks
+ * the steps whose subscriber gives up (see vfl_drop_step), indexed the same way.
+ * Same contract as the per-phase calls.
  */
 vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
-                           const int32_t* tau_a);
+                           const int32_t* tau_a, const uint8_t* drop);
 
 /*
  * CUDA-graph replay of a window of steps.  vfl_graph_capture records steps
@@ -275,10 +302,12 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
  * after all work already on the context's streams, and advances the cursor to
  * k0 + n_steps.  Capture needs caller streams (vfl_set_streams) and per-launch
  * timing off.  A graph belongs to one context; destroy it before the context.
+ * `drop` as for vfl_train_steps; the batches are baked in, so a replay also
+ * needs the drop count the capture started from.
  */
 typedef struct vfl_graph vfl_graph;
 vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
-                             const int32_t* tau_a, vfl_graph** out);
+                             const int32_t* tau_a, const uint8_t* drop, vfl_graph** out);
 vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* graph);
 vfl_status vfl_graph_destroy(vfl_graph* graph);
 

@@ -84,9 +84,13 @@ EXPORTS = {
     "vfl_active_step": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32]),
     "vfl_passive_backward": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
     "vfl_train_steps": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
-                                         ctypes.c_void_p]),
+                                         ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_graph_capture": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
-                                           ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
+                                           ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
+    "vfl_drop_step": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_get_drops": (ctypes.c_int32, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)]),
+    "vfl_set_drops": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_make_drops": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_double, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_graph_launch": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_graph_destroy": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_synchronize": (ctypes.c_int32, [ctypes.c_void_p]),
@@ -180,6 +184,21 @@ def make_schedule(seed: int, S: int, kind: int, n_steps: int):
     ta = np.zeros(max(n_steps, 1), np.int32)
     _check(lib().vfl_make_schedule(seed, S, kind, n_steps, _ptr(tp), _ptr(ta)))
     return tp[:n_steps], ta[:n_steps]
+
+
+def make_drops(seed: int, rate: float, n_steps: int):
+    """uint8 drop marks from the library's seeded draws (see vfl_make_drops)."""
+    out = np.zeros(max(n_steps, 1), np.uint8)
+    _check(lib().vfl_make_drops(seed, rate, n_steps, _ptr(out)))
+    return out[:n_steps]
+
+
+def _drops_ptr(drops, end):
+    if drops is None:
+        return None, None
+    d = np.ascontiguousarray(drops, np.uint8)
+    assert len(d) >= end
+    return d, _ptr(d)
 
 
 def weight_grad_noalloc(dpre, x, dW, db, dtype: int, stream=None):
@@ -360,17 +379,18 @@ class Context:
         return self.cfg.ps_dt0 > 0
 
     def checkpoint(self):
-        """(k, {version: params}, fp32 masters of version k); in the parameter-server
-        mode (k, {worker: replica}, None)."""
+        """(k, {version: params}, fp32 masters of version k, dropped steps so far); in
+        the parameter-server mode (k, {worker: replica}, None, dropped steps)."""
         k = self.cursor()
         if self.ps:
-            return k, {w: self.get_replica(w) for w in range(self.p.workers)}, None
+            return k, {w: self.get_replica(w) for w in range(self.p.workers)}, None, self.drops()
         vers = {v: self.get_version(v) for v in range(max(0, k - self.p.staleness), k + 1)}
-        return k, vers, self.get_params()
+        return k, vers, self.get_params(), self.drops()
 
     def restore(self, ckpt):
-        k, vers, master = ckpt
+        k, vers, master, drops = ckpt
         self.set_cursor(k)
+        self.set_drops(drops)
         if self.ps:
             for w, params in vers.items():
                 self.set_replica(w, params)
@@ -388,19 +408,33 @@ class Context:
     def passive_backward(self, k):
         self._call(lib().vfl_passive_backward, k)
 
-    def train_steps(self, k0, n, tau_p, tau_a):
+    def drop_step(self, k):
+        """The subscriber of step k gives up on its embedding (see vfl_drop_step)."""
+        self._call(lib().vfl_drop_step, k)
+
+    def drops(self) -> int:
+        n = ctypes.c_int64()
+        self._call(lib().vfl_get_drops, ctypes.byref(n))
+        return n.value
+
+    def set_drops(self, n: int):
+        self._call(lib().vfl_set_drops, n)
+
+    def train_steps(self, k0, n, tau_p, tau_a, drops=None):
         tau_p = np.ascontiguousarray(tau_p, np.int32)
         tau_a = np.ascontiguousarray(tau_a, np.int32)
         assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
-        self._call(lib().vfl_train_steps, k0, n, _ptr(tau_p), _ptr(tau_a))
+        d, dp = _drops_ptr(drops, k0 + n)
+        self._call(lib().vfl_train_steps, k0, n, _ptr(tau_p), _ptr(tau_a), dp)
 
-    def capture(self, k0, n, tau_p, tau_a):
+    def capture(self, k0, n, tau_p, tau_a, drops=None):
         """A CUDA graph of steps [k0, k0+n) (see vfl_graph_capture); replay with launch_graph."""
         tau_p = np.ascontiguousarray(tau_p, np.int32)
         tau_a = np.ascontiguousarray(tau_a, np.int32)
         assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
+        d, dp = _drops_ptr(drops, k0 + n)
         g = ctypes.c_void_p()
-        self._call(lib().vfl_graph_capture, k0, n, _ptr(tau_p), _ptr(tau_a), ctypes.byref(g))
+        self._call(lib().vfl_graph_capture, k0, n, _ptr(tau_p), _ptr(tau_a), dp, ctypes.byref(g))
         self._graphs = getattr(self, "_graphs", []) + [g]
         return g
 

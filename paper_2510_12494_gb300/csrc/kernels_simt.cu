@@ -494,6 +494,12 @@ __global__ void __launch_bounds__(256) ps_average_kernel(const PsAvgLayer* __res
     }
 }
 
+__global__ void mark_dropped_kernel(float* loss, float* loss_host) {
+    const float nan = __int_as_float(0x7FC00000);
+    *loss = nan;
+    if (loss_host) *loss_host = nan;
+}
+
 __global__ void write_header_kernel(ChannelHeader* h, long long k, int batch, int version) {
     h->k = k;
     h->batch = batch;
@@ -673,6 +679,11 @@ cudaError_t launch_ps_average(const PsAvgLayer* tab, int n_layers, long long tot
                               cudaStream_t s) {
     if (total <= 0) return cudaSuccess;
     ps_average_kernel<<<grid_for(total, 256), 256, 0, s>>>(tab, n_layers, total, nrep, c_bf16);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mark_dropped(float* loss, float* loss_host, cudaStream_t s) {
+    mark_dropped_kernel<<<1, 1, 0, s>>>(loss, loss_host);
     return cudaGetLastError();
 }
 

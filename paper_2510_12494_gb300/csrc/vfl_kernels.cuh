@@ -54,6 +54,8 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask
 // Loss + d(logits) over one batch (single block, deterministic reduction):
 //   rows: B_k; logits fp32 [B_k, n_out]; y int32 labels of the batch rows.
 //   ds [B_k, n_out] = dLoss/dlogits of the batch-mean loss; loss_out = mean loss.
+// A dropped step's loss: NaN in the loss ring slot and, when given, in the host ring slot.
+cudaError_t launch_mark_dropped(float* loss, float* loss_host, cudaStream_t s);
 cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
                         float* loss_out, float* loss_host, cudaStream_t s);
 

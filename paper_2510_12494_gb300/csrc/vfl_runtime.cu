@@ -11,6 +11,8 @@
 //  - App. D (Assumption 4, theorem): the gradient applied at step k was
 //    computed with weights of version k - tau(k); updates apply in step order.
 //    Each party keeps its S+1 most recent weight versions in a ring.
+//  - Sec. 4.1 waiting deadline / buffer overflow: a dropped step trains nothing
+//    (both parties copy version k to k+1) and hands its batch to the next step.
 //  - Sec. 4.2 / Eq. 5 (ps_dt0 > 0): one replica of each party's parameters per
 //    worker, each worker's steps chained on its own stream pair, the replicas
 //    averaged after the epochs Eq. 5 selects.
@@ -38,6 +40,7 @@ constexpr int kMaxSlots = 16;
 constexpr int kEvPool = 64;
 constexpr int kMaxIoSlots = kMaxSlots + kMaxWorkers + 2;   // staging ring: S + W + 2 slots
 constexpr int kLossCap = 4096;
+constexpr int kInfoRing = 64;   // per-step host records (batch, drop) of the steps in flight
 
 thread_local std::string g_global_err;
 
@@ -178,6 +181,11 @@ struct vfl_ctx {
 
     // host-side ordering state
     long long n_fwd = 0, n_act = 0, n_bwd = 0;
+    long long n_drops = 0;                      // dropped steps among those published
+    long long step_id[kInfoRing];               // per step k (slot k mod kInfoRing): its index,
+    long long step_batch[kInfoRing];            // batch id,
+    long long step_trained[kInfoRing];          // batches trained before it,
+    unsigned char step_drop[kInfoRing] = {};    // dropped (waiting deadline)
     int fwd_version[kMaxSlots] = {};
     long long slot_step_p[kMaxSlots];
     long long grad_step[kMaxSlots];
@@ -207,8 +215,17 @@ struct vfl_ctx {
     vfl_status cuda(cudaError_t e, const char* what, int line) {
         return fail(VFL_E_CUDA, "%s failed (line %d): %s", what, line, cudaGetErrorString(e));
     }
+    // Batch of step k: (k - drops before k) mod nb, recorded when the step is published.
+    long long batch_of(long long k) const {
+        const int i = (int)(k % kInfoRing);
+        return step_id[i] == k ? step_batch[i] : (k - n_drops) % nb;
+    }
+    bool dropped(long long k) const {
+        const int i = (int)(k % kInfoRing);
+        return step_id[i] == k && step_drop[i];
+    }
     int batch_rows(long long k, long long* r0) const {
-        const long long j = k % nb;
+        const long long j = batch_of(k);
         *r0 = j * cfg.batch;
         return (int)std::min<long long>(cfg.batch, n_rows - *r0);
     }
@@ -216,7 +233,9 @@ struct vfl_ctx {
 
 // Host-side ordering state of a context (saved around graph capture).
 struct HostState {
-    long long n_fwd, n_act, n_bwd;
+    long long n_fwd, n_act, n_bwd, n_drops;
+    long long step_id[kInfoRing], step_batch[kInfoRing], step_trained[kInfoRing];
+    unsigned char step_drop[kInfoRing];
     int fwd_version[kMaxSlots];
     long long slot_step_p[kMaxSlots], grad_step[kMaxSlots], last_act_step[kMaxWorkers];
     bool started;
@@ -228,6 +247,11 @@ static HostState save_state(const vfl_ctx* c) {
     h.n_fwd = c->n_fwd;
     h.n_act = c->n_act;
     h.n_bwd = c->n_bwd;
+    h.n_drops = c->n_drops;
+    std::memcpy(h.step_id, c->step_id, sizeof h.step_id);
+    std::memcpy(h.step_batch, c->step_batch, sizeof h.step_batch);
+    std::memcpy(h.step_trained, c->step_trained, sizeof h.step_trained);
+    std::memcpy(h.step_drop, c->step_drop, sizeof h.step_drop);
     std::memcpy(h.fwd_version, c->fwd_version, sizeof h.fwd_version);
     std::memcpy(h.slot_step_p, c->slot_step_p, sizeof h.slot_step_p);
     std::memcpy(h.grad_step, c->grad_step, sizeof h.grad_step);
@@ -241,6 +265,11 @@ static void load_state(vfl_ctx* c, const HostState& h) {
     c->n_fwd = h.n_fwd;
     c->n_act = h.n_act;
     c->n_bwd = h.n_bwd;
+    c->n_drops = h.n_drops;
+    std::memcpy(c->step_id, h.step_id, sizeof h.step_id);
+    std::memcpy(c->step_batch, h.step_batch, sizeof h.step_batch);
+    std::memcpy(c->step_trained, h.step_trained, sizeof h.step_trained);
+    std::memcpy(c->step_drop, h.step_drop, sizeof h.step_drop);
     std::memcpy(c->fwd_version, h.fwd_version, sizeof h.fwd_version);
     std::memcpy(c->slot_step_p, h.slot_step_p, sizeof h.slot_step_p);
     std::memcpy(c->grad_step, h.grad_step, sizeof h.grad_step);
@@ -253,6 +282,7 @@ struct vfl_graph {
     vfl_ctx* ctx;
     cudaGraphExec_t exec;
     long long k0, n;
+    long long drops0;          // drop count the captured steps' batches start from
     HostState after;           // host state once the captured steps have run
     long long launches;        // kernels per replay
     bool hio;                  // captured with host data bound (its copies are part of the graph)
@@ -598,15 +628,17 @@ long long ps_interval(long long t, int dt0) {
 }
 // Whether the replicas are averaged right after step e: e ends epoch t and t mod Delta T_t == 0
 // (with one worker the mean is the replica itself and nothing is launched).
+// Epochs count trained batches: with drops, epoch t ends at the step that trains batch nb-1 for the
+// t-th time.
 bool ps_agg_at(const vfl_ctx* ctx, long long e) {
-    if (!ctx->psmode || ctx->W < 2 || e < 0 || (e + 1) % ctx->nb != 0) return false;
-    const long long t = (e + 1) / ctx->nb;
+    if (!ctx->psmode || ctx->W < 2 || e < 0 || ctx->dropped(e) || ctx->batch_of(e) != ctx->nb - 1) return false;
+    const long long t = ctx->step_trained[e % kInfoRing] / ctx->nb + 1;
     return t % ps_interval(t, ctx->cfg.ps_dt0) == 0;
 }
 // The latest averaging step a < k that step k must follow (a >= k - W: older ones are ordered
 // through the worker's own stream), or -1.
 long long ps_last_agg(const vfl_ctx* ctx, long long k) {
-    for (long long e = (k / ctx->nb) * ctx->nb - 1; e >= 0 && e >= k - ctx->W; e -= ctx->nb)
+    for (long long e = k - 1; e >= 0 && e >= k - ctx->W; --e)
         if (ps_agg_at(ctx, e)) return e;
     return -1;
 }
@@ -924,7 +956,7 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
         a.dp_seed = ctx->cfg.dp_seed;
     }
     a.k = k;
-    a.batch = (int)(k % ctx->nb);
+    a.batch = (int)ctx->batch_of(k);
     a.version = (int)v;
     // algorithmic bytes: the batch's features in, the saved activations out, one read of the weights
     double bytes = (double)rows * ctx->cfg.d_passive * 4;
@@ -973,7 +1005,7 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     a.chk_hdr = ctx->emb_hdr + slot;
     a.pub_hdr = ctx->grad_hdr + slot;
     a.k = k;
-    a.batch = (int)(k % ctx->nb);
+    a.batch = (int)ctx->batch_of(k);
     a.version = (int)v;
     a.status = ctx->status;
     const double flops = fused_flops(ctx->A, rows, true, true, false, false) + fused_flops(ctx->T, rows, true, true, true, false);
@@ -1136,7 +1168,45 @@ vfl_status wait_update_order(vfl_ctx* ctx, long long k, bool passive, cudaStream
 }
 
 // ---- the three phases ------------------------------------------------------
-vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
+// Host record of step k at its publish: its batch (the next untrained one) and whether it is dropped.
+void record_step(vfl_ctx* ctx, long long k, bool drop) {
+    const int i = (int)(k % kInfoRing);
+    ctx->step_id[i] = k;
+    ctx->step_trained[i] = k - ctx->n_drops;
+    ctx->step_batch[i] = (k - ctx->n_drops) % ctx->nb;
+    ctx->step_drop[i] = drop ? 1 : 0;
+    if (drop) ++ctx->n_drops;
+}
+
+// A dropped step's version k+1 = version k: copy the compute copies of one party's layers from
+// slot k mod S1 to slot (k+1) mod S1 on s, after version k exists (the masters already hold it).
+// With one slot, or one per worker (parameter-server mode), there is nothing to copy.
+vfl_status copy_version_forward(vfl_ctx* ctx, long long k, bool passive, cudaStream_t s) {
+    if (k > 0 && k > ctx->ordered_floor && !ctx->psmode)
+        TRY(wait_ev(ctx, s, (passive ? ctx->ev_pver : ctx->ev_aver)[k % kEvPool]));
+    const int from = (int)(k % ctx->S1), to = new_version_slot(ctx, k);
+    if (from != to && !ctx->psmode)
+        for (std::vector<Layer>* v : passive ? std::vector<std::vector<Layer>*>{&ctx->P}
+                                             : std::vector<std::vector<Layer>*>{&ctx->A, &ctx->T})
+            for (Layer& L : *v) {
+                CK(cudaMemcpyAsync(L.cW[to], L.cW[from], (size_t)L.out * L.in_ld * ctx->esz, cudaMemcpyDeviceToDevice, s));
+                CK(cudaMemcpyAsync(L.cb[to], L.cb[from], (size_t)L.out * 4, cudaMemcpyDeviceToDevice, s));
+            }
+    CK(cudaEventRecord((passive ? ctx->ev_pver : ctx->ev_aver)[(k + 1) % kEvPool], s));
+    return VFL_OK;
+}
+
+// The subscriber's side of a dropped step (waiting deadline): no active work, the loss slot(s) NaN,
+// the active version carried forward.
+vfl_status do_drop_active(vfl_ctx* ctx, long long k) {
+    cudaStream_t s = astream(ctx, k);
+    PLAUNCH(K_LOSS, 0, 8, s, launch_mark_dropped(ctx->losses + (k % kLossCap), loss_host(ctx, k), s));
+    TRY(copy_version_forward(ctx, k, false, s));
+    ctx->n_act = k + 1;
+    return VFL_OK;
+}
+
+vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = false) {
     const vfl_config& c = ctx->cfg;
     if (k != ctx->n_fwd) return ctx->fail(VFL_E_STATE, "passive_forward(%lld): next publish is step %lld", k, ctx->n_fwd);
     if (tau_p < 0 || tau_p > c.staleness || tau_p > k)
@@ -1152,6 +1222,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
     } else if (v < u - c.staleness) {
         return ctx->fail(VFL_E_STATE, "passive_forward(%lld): passive version %lld no longer stored", k, v);
     }
+    record_step(ctx, k, drop);
     cudaStream_t s = pstream(ctx, k);
     const int slot = (int)(k % ctx->S1);
     const int vslot = (int)(v % ctx->S1);
@@ -1187,7 +1258,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p) {
                 launch_dp_emb(ctx->act_p[slot].back(), ld8(ep), ctx->bf16, ctx->emb_pub[slot], ctx->emb_c[slot], rows,
                               ep, c.dp_clip, c.dp_sigma, c.dp_seed, k, s));
     }
-    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)(k % ctx->nb), (int)v, s));
+    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
     CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
     ctx->fwd_version[slot] = (int)v;
     ctx->slot_step_p[slot] = k;
@@ -1200,6 +1271,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const vfl_config& c = ctx->cfg;
     if (k != ctx->n_act) return ctx->fail(VFL_E_STATE, "active_step(%lld): next active step is %lld", k, ctx->n_act);
     if (k >= ctx->n_fwd) return ctx->fail(VFL_E_STATE, "active_step(%lld): embedding not published yet", k);
+    if (ctx->dropped(k)) return do_drop_active(ctx, k);
     if (tau_a < 0 || tau_a > c.staleness || tau_a > k)
         return ctx->fail(VFL_E_STATE, "active_step(%lld): tau_a=%d outside [0, min(k, S=%d)]", k, tau_a, c.staleness);
     const long long v = k - tau_a;
@@ -1316,7 +1388,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
                 launch_dp(ctx->dzp32[w], ld8(ep), ctx->grad[slot], ld8(ep), ctx->bf16, rows, ep, c.dp_clip,
                           c.dp_sigma, c.dp_seed, k, s));
     // publish the gradient
-    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)(k % ctx->nb), (int)v, s));
+    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
     CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
     ctx->grad_step[slot] = k;
     // active bottom backward
@@ -1344,6 +1416,11 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
 vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     if (k != ctx->n_bwd) return ctx->fail(VFL_E_STATE, "passive_backward(%lld): next backward is %lld", k, ctx->n_bwd);
     if (k >= ctx->n_act) return ctx->fail(VFL_E_STATE, "passive_backward(%lld): gradient not published yet", k);
+    if (ctx->dropped(k)) {   // notified of the drop: no backward, the passive version carried forward
+        TRY(copy_version_forward(ctx, k, true, pstream(ctx, k)));
+        ctx->n_bwd = k + 1;
+        return VFL_OK;
+    }
     const int w = (int)(k % ctx->W);
     cudaStream_t s = pstream(ctx, k);
     const int slot = (int)(k % ctx->S1);
@@ -1489,6 +1566,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     ctx->nb = (int)((n_rows + cfg->batch - 1) / cfg->batch);
     for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
     for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
+    for (int i = 0; i < kInfoRing; ++i) ctx->step_id[i] = -1;
     ctx->fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
     ctx->head = head_eligible(*cfg) && !getenv("VFL_DISABLE_HEAD");
     build_layers(ctx);
@@ -1747,6 +1825,8 @@ vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k) {
         return ctx->fail(VFL_E_STATE, "vfl_set_cursor with steps in flight");
     TRY(sync_all(ctx));
     ctx->n_fwd = ctx->n_act = ctx->n_bwd = k;
+    ctx->n_drops = 0;   // the batches trained so far are k unless vfl_set_drops says otherwise
+    for (int i = 0; i < kInfoRing; ++i) ctx->step_id[i] = -1;
     ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k);
     for (int s = 0; s < kMaxSlots; ++s) ctx->slot_step_p[s] = ctx->grad_step[s] = -1;
     for (int w = 0; w < kMaxWorkers; ++w) ctx->last_act_step[w] = -1;
@@ -1852,6 +1932,38 @@ vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queri
     return VFL_OK;
 }
 
+namespace {
+// Word 0 of Philox4x32-10 with counter (k lo, k hi, c2, c3) and key (seed lo, seed hi).
+uint32_t philox_word0(uint64_t seed, int64_t k, uint32_t c2, uint32_t c3) {
+    uint32_t c[4] = {(uint32_t)(k & 0xFFFFFFFFu), (uint32_t)((uint64_t)k >> 32), c2, c3};
+    uint32_t key[2] = {(uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32)};
+    for (int r = 0; r < 10; ++r) {
+        const uint64_t p0 = (uint64_t)0xD2511F53u * c[0];
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * c[2];
+        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ key[0];
+        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ key[1];
+        c[0] = n0;
+        c[1] = (uint32_t)p1;
+        c[2] = n2;
+        c[3] = (uint32_t)p0;
+        key[0] += 0x9E3779B9u;
+        key[1] += 0xBB67AE85u;
+    }
+    return c[0];
+}
+}  // namespace
+
+vfl_status vfl_make_drops(uint64_t seed, double rate, int64_t n_steps, uint8_t* drop) {
+    if (!(rate >= 0.0 && rate <= 1.0) || n_steps < 0 || (n_steps > 0 && !drop)) {
+        g_global_err = "vfl_make_drops: invalid argument";
+        return VFL_E_INVAL;
+    }
+    const uint64_t thr = rate >= 1.0 ? (1ull << 32) : (uint64_t)std::floor(rate * 4294967296.0);
+    for (int64_t k = 0; k < n_steps; ++k)
+        drop[k] = thr >= (1ull << 32) || (uint64_t)philox_word0(seed, k, 2u, 0x4452u) < thr ? 1 : 0;
+    return VFL_OK;
+}
+
 vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_steps, int32_t* tau_p,
                              int32_t* tau_a) {
     if (S < 0 || n_steps < 0 || (n_steps > 0 && (!tau_p || !tau_a))) {
@@ -1862,7 +1974,6 @@ vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_s
         g_global_err = "vfl_make_schedule: unknown kind";
         return VFL_E_INVAL;
     }
-    const uint32_t k0 = (uint32_t)(seed & 0xFFFFFFFFu), k1 = (uint32_t)(seed >> 32);
     for (int party = 0; party < 2; ++party) {
         int32_t* tau = party == 0 ? tau_p : tau_a;
         int32_t prev = 0;
@@ -1872,21 +1983,7 @@ vfl_status vfl_make_schedule(uint64_t seed, int32_t S, int32_t kind, int64_t n_s
                 t = (int32_t)std::min<int64_t>(k, S);
             } else if (kind == VFL_SCHED_SEEDED && k > 0) {
                 // Philox4x32-10, counter (k lo, k hi, party, 0x5343), key (seed lo, seed hi); word 0
-                uint32_t c[4] = {(uint32_t)(k & 0xFFFFFFFFu), (uint32_t)((uint64_t)k >> 32), (uint32_t)party, 0x5343u};
-                uint32_t key[2] = {k0, k1};
-                for (int r = 0; r < 10; ++r) {
-                    const uint64_t p0 = (uint64_t)0xD2511F53u * c[0];
-                    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c[2];
-                    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ key[0];
-                    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ key[1];
-                    c[0] = n0;
-                    c[1] = (uint32_t)p1;
-                    c[2] = n2;
-                    c[3] = (uint32_t)p0;
-                    key[0] += 0x9E3779B9u;
-                    key[1] += 0xBB67AE85u;
-                }
-                const int64_t u = (int64_t)(c[0] % (uint32_t)(S + 1));
+                const int64_t u = (int64_t)(philox_word0(seed, k, (uint32_t)party, 0x5343u) % (uint32_t)(S + 1));
                 t = (int32_t)std::min<int64_t>(std::min<int64_t>(k, S), std::min<int64_t>(prev + 1, u));
             }
             tau[k] = t;
@@ -1908,13 +2005,49 @@ vfl_status vfl_active_step(vfl_ctx* ctx, int64_t k, int32_t tau_a) {
     return do_active_step(ctx, k, tau_a);
 }
 
+vfl_status vfl_drop_step(vfl_ctx* ctx, int64_t k) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (k != ctx->n_act) return ctx->fail(VFL_E_STATE, "drop_step(%lld): next active step is %lld", (long long)k, ctx->n_act);
+    if (ctx->n_fwd > k + 1)
+        return ctx->fail(VFL_E_STATE, "drop_step(%lld): step %lld is already published with the next batch",
+                         (long long)k, ctx->n_fwd - 1);
+    if (ctx->n_fwd == k) {   // the embedding never arrived: nothing was published for step k
+        record_step(ctx, k, true);
+        ctx->n_fwd = k + 1;
+        ctx->started = true;
+    } else if (!ctx->dropped(k)) {
+        ctx->step_drop[k % kInfoRing] = 1;
+        ++ctx->n_drops;
+    }
+    return do_drop_active(ctx, k);
+}
+
+vfl_status vfl_get_drops(vfl_ctx* ctx, int64_t* n) {
+    if (!ctx || !n) return VFL_E_INVAL;
+    *n = ctx->n_drops;
+    return VFL_OK;
+}
+
+vfl_status vfl_set_drops(vfl_ctx* ctx, int64_t n) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_set_drops with steps in flight");
+    if (n < 0 || n > ctx->n_fwd) return ctx->fail(VFL_E_INVAL, "drop count %lld outside [0, %lld]", (long long)n, ctx->n_fwd);
+    ctx->n_drops = n;
+    for (int i = 0; i < kInfoRing; ++i) ctx->step_id[i] = -1;
+    return VFL_OK;
+}
+
 vfl_status vfl_passive_backward(vfl_ctx* ctx, int64_t k) {
     if (!ctx) return VFL_E_INVAL;
     if (ctx->broken) return VFL_E_CUDA;
     return do_passive_backward(ctx, k);
 }
 
-vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a) {
+vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
+                           const uint8_t* drop) {
     if (!ctx) return VFL_E_INVAL;
     if (ctx->broken) return VFL_E_CUDA;
     if (n_steps < 0 || (n_steps > 0 && (!tau_p || !tau_a))) return ctx->fail(VFL_E_INVAL, "invalid schedule arguments");
@@ -1926,7 +2059,7 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
     while (ctx->n_bwd < end) {
         bool progressed = false;
         while (ctx->n_fwd < end && (ctx->psmode ? ps_need_bwd(ctx, ctx->n_fwd) : ctx->n_fwd - tau_p[ctx->n_fwd]) <= ctx->n_bwd) {
-            TRY(do_passive_forward(ctx, ctx->n_fwd, tau_p[ctx->n_fwd]));
+            TRY(do_passive_forward(ctx, ctx->n_fwd, tau_p[ctx->n_fwd], drop && drop[ctx->n_fwd]));
             progressed = true;
         }
         while (ctx->n_act < ctx->n_fwd) {
@@ -1990,6 +2123,7 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
 }  // namespace
 
 vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
+                             const uint8_t* drop,
                              vfl_graph** out) {
     if (!ctx || !out) return VFL_E_INVAL;
     *out = nullptr;
@@ -2004,6 +2138,7 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     g->ctx = ctx;
     g->k0 = k0;
     g->n = n_steps;
+    g->drops0 = ctx->n_drops;
     g->hio = ctx->hio;
     cudaError_t e = cudaEventCreateWithFlags(&g->fork, cudaEventDisableTiming);
     for (int i = 0; i < kMaxStreams && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
@@ -2025,7 +2160,7 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     ctx->ordered_floor = std::max<long long>(ctx->ordered_floor, k0);
     ctx->cap_nodes.clear();
     ctx->capturing = true;
-    if (e == cudaSuccess) st = vfl_train_steps(ctx, k0, n_steps, tau_p, tau_a);
+    if (e == cudaSuccess) st = vfl_train_steps(ctx, k0, n_steps, tau_p, tau_a, drop);
     ctx->capturing = false;
     ctx->ordered_floor = floor_before;
     // join every stream back into the origin, even after a failure, so that capture can end
@@ -2060,6 +2195,9 @@ vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* g) {
     if (ctx->n_fwd != g->k0 || ctx->n_act != g->k0 || ctx->n_bwd != g->k0)
         return ctx->fail(VFL_E_STATE, "graph starts at step %lld but the context is at step %lld", g->k0, ctx->n_fwd);
     if (g->hio != ctx->hio) return ctx->fail(VFL_E_STATE, "graph captured with another host-data binding");
+    if (g->drops0 != ctx->n_drops)
+        return ctx->fail(VFL_E_STATE, "graph captured after %lld dropped steps, the context has %lld", g->drops0,
+                         ctx->n_drops);
     cudaStream_t origin = ctx->ps[0];
     // order the replay after everything already enqueued on the context's streams, and theirs after it
     cudaStream_t ss[kMaxStreams];

@@ -118,6 +118,7 @@ def force_gpu_state(ctx, o, S):
     (oracle -> GPU only)."""
     k = o.k
     ctx.set_cursor(k)
+    ctx.set_drops(o.k - o.n_done)
     if ctx.ps:
         for w in range(ctx.p.workers):
             ctx.set_replica(w, o.replica_params(w))
@@ -126,11 +127,23 @@ def force_gpu_state(ctx, o, S):
         ctx.set_version(v, oracle_version(o, v))
 
 
-def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=None):
+def compare_dropped(ctx, rec, tol):
+    """A dropped step: NaN loss, and the parameters (or the step's replica) the oracle kept."""
+    errs = {"loss_nan": 0.0 if np.isnan(ctx.read_losses(rec.k, 1)[0]) else 1.0}
+    params = ctx.get_replica(rec.k % ctx.p.workers) if ctx.ps else ctx.get_params()
+    for key, (W, b) in params.items():
+        errs[f"W{key}"] = tensor_err(W, rec.params[key][0], ctx.p.dtype)
+        errs[f"b{key}"] = tensor_err(b, rec.params[key][1], ctx.p.dtype)
+    return errs, {name: e for name, e in errs.items() if not e <= tol}
+
+
+def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=None, drops=None, publish_dropped=True):
     """Step-by-step comparison.  bf16 presets are teacher-forced: before each
     step the GPU takes the oracle's weight versions, so one step's error is
     measured without the drift of earlier roundings (a bf16 weight copy that
-    rounds the other way moves later ReLU masks)."""
+    rounds the other way moves later ReLU masks).  `drops` marks steps whose
+    subscriber gives up (vfl_drop_step); with publish_dropped False their
+    publisher never runs."""
     p = synth.preset(cid) if isinstance(cid, int) else cid
     if workers:
         p = p.with_(workers=workers)
@@ -147,11 +160,19 @@ def run_sequential(vfl, cid, n_rows, steps=None, teacher_forced=None, workers=No
     for k in range(steps):
         if teacher_forced and k > 0:
             force_gpu_state(ctx, o, q.staleness)
-        rec = o.step(int(tp[k]), int(ta[k]), record=True)
-        ctx.passive_forward(k, int(tp[k]))
-        ctx.active_step(k, int(ta[k]))
-        ctx.passive_backward(k)
-        errs, bad = compare_step(vfl, ctx, rec, TOL[q.dtype])
+        dropped = drops is not None and bool(drops[k])
+        rec = o.step(int(tp[k]), int(ta[k]), record=True, drop=dropped)
+        if dropped:
+            if publish_dropped:
+                ctx.passive_forward(k, int(tp[k]))
+            ctx.drop_step(k)
+            ctx.passive_backward(k)
+            errs, bad = compare_dropped(ctx, rec, TOL[q.dtype])
+        else:
+            ctx.passive_forward(k, int(tp[k]))
+            ctx.active_step(k, int(ta[k]))
+            ctx.passive_backward(k)
+            errs, bad = compare_step(vfl, ctx, rec, TOL[q.dtype])
         for name, e in errs.items():
             worst[name] = max(worst.get(name, 0.0), e)
         if bad:

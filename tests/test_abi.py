@@ -120,3 +120,15 @@ def test_ps_workspace_holds_a_master_per_replica(vfl):
             d_in = o
     # three more fp32 masters (and the version ring grows from one slot to one per worker)
     assert with_ps - base >= 3 * n_params * 4
+
+
+@pytest.mark.parametrize("rate", [0.0, 0.01, 0.3, 0.999, 1.0])
+@pytest.mark.parametrize("seed", [0, 7, 0xDEADBEEF12345])
+def test_drop_draws_match_oracle_bit_exactly(vfl, rate, seed):
+    np.testing.assert_array_equal(vfl.make_drops(seed, rate, 3000), oracle.make_drops(seed, rate, 3000))
+
+
+def test_drop_draws_reject_bad_rates(vfl):
+    for rate in (-0.1, 1.5, float("nan")):
+        with pytest.raises(vfl.VflError):
+            vfl.make_drops(0, rate, 5)
