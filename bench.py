@@ -428,7 +428,10 @@ def run_ours(args):
         ctx.synchronize()
         dt = slowest_rank(time.perf_counter() - t0)
         ctx.bind_host_data(None, None, None)
-        kept = np.ones(K, bool) if drops is None else drops[k0:k0 + K] == 0
+        kept = np.ones(K, bool)            # the host ring's slot k mod K holds step k's loss
+        if drops is not None:
+            steps = np.arange(k0, k0 + K)
+            kept[steps % K] = drops[steps] == 0
         assert np.isfinite(loss_host.numpy()[kept]).all() and np.isnan(loss_host.numpy()[~kept]).all()
         h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
         e2e = {"value": job_throughput(samples(p, k0, K, drops), world, dt), "unit": "samples/s", "h2d_bytes_per_step": h2d,

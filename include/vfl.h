@@ -325,8 +325,13 @@ vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out);
  */
 vfl_status vfl_fetch_loss(vfl_ctx* ctx, int64_t k, float* host_out);
 
-/* Copy a channel slot or a per-worker buffer of step k to host fp32 (see VFL_TAP_*); synchronizes. */
-vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out);
+/* Copy a channel slot or a per-worker buffer of step k to host fp32 (see VFL_TAP_*): rows x cols
+ * floats, rows as vfl_step_rows gives; VFL_E_INVAL when that exceeds out_elems.  Synchronizes. */
+vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out, int64_t out_elems);
+
+/* First row and row count of the batch step k trains (published steps in flight, or the next
+ * step): batch (k - drops before k) mod nb. */
+vfl_status vfl_step_rows(vfl_ctx* ctx, int64_t k, int64_t* r0, int32_t* rows);
 
 /*
  * Fault probe: a bounded device-side wait (at most max_iters polls) for the

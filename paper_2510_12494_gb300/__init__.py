@@ -95,7 +95,9 @@ EXPORTS = {
     "vfl_graph_destroy": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_synchronize": (ctypes.c_int32, [ctypes.c_void_p]),
     "vfl_read_losses": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]),
-    "vfl_tap": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p]),
+    "vfl_tap": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_step_rows": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.POINTER(ctypes.c_int64),
+                                       ctypes.POINTER(ctypes.c_int32)]),
     "vfl_fetch_loss": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_wait_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64]),
     "vfl_check_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64]),
@@ -454,16 +456,18 @@ class Context:
         self._call(lib().vfl_fetch_loss, k, ctypes.c_void_p(host_ptr))
 
     def batch_rows(self, k):
-        j = k % self.nb
-        r0 = j * self.p.batch
-        return r0, min(self.n_rows, r0 + self.p.batch)
+        """(first row, end row) of the batch step k trains, as the library assigns it."""
+        r0 = ctypes.c_int64()
+        n = ctypes.c_int32()
+        self._call(lib().vfl_step_rows, k, ctypes.byref(r0), ctypes.byref(n))
+        return r0.value, r0.value + n.value
 
     def tap(self, k, what):
         r0, r1 = self.batch_rows(k)
         cols = {TAP_EMB: self.p.e_passive, TAP_GRAD: self.p.e_passive, TAP_LOGITS: self.p.n_out,
                 TAP_ZA: self.p.e_active, TAP_DZA: self.p.e_active}[what]
         out = np.zeros((r1 - r0, cols), np.float32)
-        self._call(lib().vfl_tap, k, what, _ptr(out))
+        self._call(lib().vfl_tap, k, what, _ptr(out), out.size)
         return out
 
     def wait_channel(self, which, k, max_iters):

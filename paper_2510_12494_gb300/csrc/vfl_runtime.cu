@@ -2255,7 +2255,16 @@ vfl_status vfl_fetch_loss(vfl_ctx* ctx, int64_t k, float* host_out) {
     return VFL_OK;
 }
 
-vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out) {
+vfl_status vfl_step_rows(vfl_ctx* ctx, int64_t k, int64_t* r0, int32_t* rows) {
+    if (!ctx || !r0 || !rows) return VFL_E_INVAL;
+    if (k < 0) return ctx->fail(VFL_E_INVAL, "step %lld < 0", (long long)k);
+    long long r;
+    *rows = ctx->batch_rows(k, &r);
+    *r0 = r;
+    return VFL_OK;
+}
+
+vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out, int64_t out_elems) {
     if (!ctx || !out) return VFL_E_INVAL;
     if (ctx->broken) return VFL_E_CUDA;
     TRY(sync_all(ctx));
@@ -2287,6 +2296,9 @@ vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out) {
         default:
             return ctx->fail(VFL_E_INVAL, "unknown tap %d", what);
     }
+    if ((long long)rows * cols > out_elems)
+        return ctx->fail(VFL_E_INVAL, "tap of step %lld needs %lld floats, the buffer holds %lld", (long long)k,
+                         (long long)rows * cols, (long long)out_elems);
     ++ctx->launches;
     CK(launch_to_f32(src, ld, rows, cols, bf, ctx->scratch_f32, 0));
     CK(cudaMemcpy(out, ctx->scratch_f32, (size_t)rows * cols * 4, cudaMemcpyDeviceToHost));
