@@ -125,6 +125,47 @@ vfl_status vfl_ps_interval(int64_t t, int32_t dt0, int64_t* interval);
  * n_rows >= 1 and queries >= 1. */
 vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queries, double* sigma);
 
+/*
+ * System planning (Sec. 4.3-4.4, Eq. 7-17, Algorithm 2).  Host only, pure.
+ * Delay model of one iteration, each term coef * B^exp * w / C (Eq. 7-9):
+ *   T_A = (lambda_a B^gamma_a + phi_a B^beta_a + lambda_top B^gamma_top + phi_top B^beta_top) w_a / C_a
+ *   T_P = (lambda_p B^gamma_p + phi_p B^beta_p) w_p / C_p
+ *   O(w_a, w_p, B) = max(T_A, T_P) + (E + G) / B_b,  E = G = B * bytes_per_row   (Eq. 10, 17)
+ * Memory per worker M(B) = M0 + rho B^chi, so B <= B_max = min over the two parties of
+ * ((M_max - M0) / rho)^(1/chi) (Eq. 14-15; a party with rho <= 0 sets no bound).
+ */
+typedef struct vfl_plan_model {
+    double lambda_a, gamma_a, phi_a, beta_a;          /* active bottom forward / backward        */
+    double lambda_top, gamma_top, phi_top, beta_top;  /* top model forward / backward (Eq. 9)    */
+    double lambda_p, gamma_p, phi_p, beta_p;          /* passive bottom forward / backward       */
+    double C_a, C_p;                                  /* compute units of each party (> 0)       */
+    double bytes_per_row;                             /* cut-layer payload per row, each direction */
+    double bandwidth;                                 /* B_b (> 0), bytes per time unit          */
+    double M_A0, rho_A, M_A_max;                      /* active memory model per worker          */
+    double M_P0, rho_P, M_P_max;                      /* passive memory model per worker         */
+    double chi;                                       /* memory exponent (> 0)                   */
+} vfl_plan_model;
+
+/* B_max of Eq. 15 (+inf when neither party bounds it; VFL_E_INVAL when a bound is negative). */
+vfl_status vfl_plan_bmax(const vfl_plan_model* m, double* bmax);
+
+/* O(w_a, w_p, B) of Eq. 17 for one configuration. */
+vfl_status vfl_plan_delay(const vfl_plan_model* m, int32_t w_a, int32_t w_p, double batch, double* delay);
+
+/*
+ * Algorithm 2: the (w_a, w_p, B) minimising O over w_a in [wa_lo, wa_hi], w_p in
+ * [wp_lo, wp_hi] and the candidate batches (n_batches of them) with B <= B_max.
+ * Scan order: batches as given, then w_a, then w_p ascending; the first strict
+ * minimum wins.  VFL_E_INVAL when no candidate is feasible or a range is empty.
+ */
+vfl_status vfl_plan(const vfl_plan_model* m, int32_t wa_lo, int32_t wa_hi, int32_t wp_lo, int32_t wp_hi,
+                    const int32_t* batches, int32_t n_batches, int32_t* w_a, int32_t* w_p, int32_t* batch,
+                    double* delay);
+
+/* Least-squares fit of t = coef * x^expo in log space over n >= 2 points (x, t > 0, not all x equal):
+ * the profiling step that turns measured delays into the constants of Eq. 7-9. */
+vfl_status vfl_fit_power(const double* x, const double* t, int32_t n, double* coef, double* expo);
+
 typedef struct vfl_ctx vfl_ctx;
 
 /* Bytes of device workspace vfl_create() needs for `cfg` and a dataset of n_rows rows. */

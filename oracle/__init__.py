@@ -12,10 +12,12 @@ forms (logistic regression, eta = 0, DP reductions, the embedding mechanism's
 straight-through backward against torch autograd with the clip factor held
 constant), bf16 rounding against torch's cast, the parameter server against
 independent torch replicas, and dropped steps against a brute force that
-replays the reassigned batches.  Parity unpinned: nothing.
+replays the reassigned batches, and the planner (Eq. 7-17, Algorithm 2) on
+cases whose optimum is worked out by hand.  Parity unpinned: nothing.
 """
 from .vfl_oracle import (  # noqa: F401
     PHILOX_M, PHILOX_W, TAG_DP, TAG_DPE, TAG_DROP, TAG_SCHED, SCHED_SYNC, SCHED_MAX, SCHED_SEEDED,
     philox, make_schedule, bf16_round, mlp_forward, mlp_backward, loss_and_dlogits,
     dp_normals, dp_clip_noise, dp_embed, gdp_sigma, make_drops, ps_interval, ps_aggregates_after, Oracle, StepRecord,
 )
+from .planner import FIELDS as PLAN_FIELDS, fit_power, plan, plan_bmax, plan_delay  # noqa: F401

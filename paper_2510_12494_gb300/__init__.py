@@ -49,6 +49,14 @@ class VflConfig(ctypes.Structure):
     ]
 
 
+class VflPlanModel(ctypes.Structure):
+    """vfl_plan_model: the delay, communication and memory constants of Eq. 7-15."""
+    _fields_ = [(f, ctypes.c_double) for f in (
+        "lambda_a", "gamma_a", "phi_a", "beta_a", "lambda_top", "gamma_top", "phi_top", "beta_top",
+        "lambda_p", "gamma_p", "phi_p", "beta_p", "C_a", "C_p", "bytes_per_row", "bandwidth",
+        "M_A0", "rho_A", "M_A_max", "M_P0", "rho_P", "M_P_max", "chi")]
+
+
 EXPORTS = {
     # name: (restype, argtypes)
     "vfl_workspace_bytes": (ctypes.c_int32, [ctypes.POINTER(VflConfig), ctypes.c_int64, ctypes.POINTER(ctypes.c_uint64)]),
@@ -76,6 +84,15 @@ EXPORTS = {
     "vfl_set_replica": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                          ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_ps_interval": (ctypes.c_int32, [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64)]),
+    "vfl_plan_bmax": (ctypes.c_int32, [ctypes.POINTER(VflPlanModel), ctypes.POINTER(ctypes.c_double)]),
+    "vfl_plan_delay": (ctypes.c_int32, [ctypes.POINTER(VflPlanModel), ctypes.c_int32, ctypes.c_int32, ctypes.c_double,
+                                        ctypes.POINTER(ctypes.c_double)]),
+    "vfl_plan": (ctypes.c_int32, [ctypes.POINTER(VflPlanModel), ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                  ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
+                                  ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
+                                  ctypes.POINTER(ctypes.c_double)]),
+    "vfl_fit_power": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_double),
+                                       ctypes.POINTER(ctypes.c_double)]),
     "vfl_gdp_sigma": (ctypes.c_int32, [ctypes.c_double, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                        ctypes.POINTER(ctypes.c_double)]),
     "vfl_make_schedule": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
@@ -186,6 +203,45 @@ def make_schedule(seed: int, S: int, kind: int, n_steps: int):
     ta = np.zeros(max(n_steps, 1), np.int32)
     _check(lib().vfl_make_schedule(seed, S, kind, n_steps, _ptr(tp), _ptr(ta)))
     return tp[:n_steps], ta[:n_steps]
+
+
+def plan_model(**kw) -> VflPlanModel:
+    """A vfl_plan_model from keyword constants (unnamed ones 0; C_a, C_p, bandwidth and chi default 1)."""
+    m = VflPlanModel()
+    m.C_a = m.C_p = m.bandwidth = m.chi = 1.0
+    for k, v in kw.items():
+        setattr(m, k, float(v))
+    return m
+
+
+def plan_bmax(m: VflPlanModel) -> float:
+    out = ctypes.c_double()
+    _check(lib().vfl_plan_bmax(ctypes.byref(m), ctypes.byref(out)))
+    return out.value
+
+
+def plan_delay(m: VflPlanModel, w_a: int, w_p: int, batch: float) -> float:
+    out = ctypes.c_double()
+    _check(lib().vfl_plan_delay(ctypes.byref(m), w_a, w_p, batch, ctypes.byref(out)))
+    return out.value
+
+
+def plan(m: VflPlanModel, wa_range, wp_range, batches):
+    """Algorithm 2 (vfl_plan): (w_a, w_p, B, O)."""
+    b = np.ascontiguousarray(batches, np.int32)
+    wa, wp, bb, o = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32(), ctypes.c_double()
+    _check(lib().vfl_plan(ctypes.byref(m), wa_range[0], wa_range[1], wp_range[0], wp_range[1], _ptr(b), len(b),
+                          ctypes.byref(wa), ctypes.byref(wp), ctypes.byref(bb), ctypes.byref(o)))
+    return wa.value, wp.value, bb.value, o.value
+
+
+def fit_power(x, t):
+    """(coef, expo) of t = coef * x^expo (vfl_fit_power)."""
+    x = np.ascontiguousarray(x, np.float64)
+    t = np.ascontiguousarray(t, np.float64)
+    c, e = ctypes.c_double(), ctypes.c_double()
+    _check(lib().vfl_fit_power(_ptr(x), _ptr(t), len(x), ctypes.byref(c), ctypes.byref(e)))
+    return c.value, e.value
 
 
 def make_drops(seed: int, rate: float, n_steps: int):

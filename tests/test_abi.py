@@ -132,3 +132,55 @@ def test_drop_draws_reject_bad_rates(vfl):
     for rate in (-0.1, 1.5, float("nan")):
         with pytest.raises(vfl.VflError):
             vfl.make_drops(0, rate, 5)
+
+
+def _rand_plan_model(vfl, rng):
+    kw = {f: float(rng.uniform(0.01, 2.0)) for f in ("lambda_a", "phi_a", "lambda_top", "phi_top", "lambda_p", "phi_p")}
+    kw.update({f: float(rng.uniform(-1.2, 0.4)) for f in ("gamma_a", "beta_a", "gamma_top", "beta_top", "gamma_p",
+                                                           "beta_p")})
+    kw.update(C_a=float(rng.uniform(1, 64)), C_p=float(rng.uniform(1, 64)), bytes_per_row=float(rng.uniform(0, 2e-3)),
+              bandwidth=float(rng.uniform(1, 10)), M_A0=1.0, rho_A=float(rng.uniform(1e-4, 1e-2)),
+              M_A_max=float(rng.uniform(5, 50)), M_P0=2.0, rho_P=float(rng.uniform(1e-4, 1e-2)),
+              M_P_max=float(rng.uniform(5, 50)), chi=float(rng.uniform(0.8, 1.5)))
+    return kw
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_planner_matches_oracle(vfl, seed):
+    from types import SimpleNamespace
+    rng = np.random.default_rng(100 + seed)
+    kw = _rand_plan_model(vfl, rng)
+    m, om = vfl.plan_model(**kw), SimpleNamespace(**kw)
+    assert vfl.plan_bmax(m) == pytest.approx(oracle.plan_bmax(om), rel=1e-13)
+    for wa, wp, b in ((1, 1, 16.0), (3, 7, 333.0), (50, 2, 1024.0)):
+        assert vfl.plan_delay(m, wa, wp, b) == pytest.approx(oracle.plan_delay(om, wa, wp, b), rel=1e-13)
+    batches = [16, 32, 64, 128, 256, 512, 1024, 2048, 4096]
+    try:
+        want = oracle.plan(om, (1, 6), (2, 5), batches)
+    except ValueError:
+        with pytest.raises(vfl.VflError):
+            vfl.plan(m, (1, 6), (2, 5), batches)
+        return
+    got = vfl.plan(m, (1, 6), (2, 5), batches)
+    assert got[:3] == want[:3]
+    assert got[3] == pytest.approx(want[3], rel=1e-13)
+    x = np.array([16, 64, 256, 1024, 4096], np.float64)
+    t = 0.5 * x ** 0.8 * np.exp(rng.normal(0, 0.05, x.size))
+    c1, e1 = vfl.fit_power(x, t)
+    c2, e2 = oracle.fit_power(x, t)
+    assert c1 == pytest.approx(c2, rel=1e-10) and e1 == pytest.approx(e2, rel=1e-10)
+
+
+def test_planner_rejects_bad_arguments(vfl):
+    m = vfl.plan_model(lambda_a=1.0)
+    for args in (((2, 1), (1, 1), [16]), ((0, 1), (1, 1), [16]), ((1, 1), (1, 1), [])):
+        with pytest.raises(vfl.VflError):
+            vfl.plan(m, *args)
+    with pytest.raises(vfl.VflError):
+        vfl.plan(vfl.plan_model(lambda_a=1.0, C_a=0.0), (1, 1), (1, 1), [16])
+    with pytest.raises(vfl.VflError):
+        vfl.plan_bmax(vfl.plan_model(M_A0=5.0, rho_A=1.0, M_A_max=1.0))
+    with pytest.raises(vfl.VflError):
+        vfl.fit_power([4.0, 4.0], [1.0, 2.0])
+    with pytest.raises(vfl.VflError):
+        vfl.fit_power([1.0, 2.0], [1.0, -2.0])
