@@ -338,7 +338,9 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
  * CUDA-graph replay of a window of steps.  vfl_graph_capture records steps
  * [k0, k0 + n_steps) -- the same kernels and cross-stream events
  * vfl_train_steps would enqueue -- into an executable graph without running
- * them; the context must be idle at cursor k0 and stays there.
+ * them; every step before k0 must be enqueued (it may still be running, e.g. a
+ * replayed graph: the host can capture the next window meanwhile) and the
+ * cursor stays at k0.
  * vfl_graph_launch replays it once (the context must be at cursor k0), ordered
  * after all work already on the context's streams, and advances the cursor to
  * k0 + n_steps.  Capture needs caller streams (vfl_set_streams) and per-launch

@@ -2133,7 +2133,8 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
             return ctx->fail(VFL_E_STATE, "graph capture needs the caller's streams (vfl_set_streams)");
     if (k0 != ctx->n_fwd || k0 != ctx->n_act || k0 != ctx->n_bwd)
         return ctx->fail(VFL_E_STATE, "vfl_graph_capture(%lld): steps before k0 are not all enqueued", (long long)k0);
-    TRY(sync_all(ctx));
+    // no synchronisation: earlier steps (a graph being replayed) may still run while the host captures the
+    // next window; the capture records work without executing it and its replay is ordered after them
     vfl_graph* g = new vfl_graph();
     g->ctx = ctx;
     g->k0 = k0;
@@ -2174,9 +2175,8 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     const HostState after = save_state(ctx);
     load_state(ctx, before);
     if (st == VFL_OK && e == cudaSuccess) e = cudaGraphInstantiate(&g->exec, graph, 0);
-    // upload now, so that the first replay does not pay for it
+    // upload now (ordered on the origin stream, without waiting), so that the first replay does not pay for it
     if (st == VFL_OK && e == cudaSuccess) e = cudaGraphUpload(g->exec, origin);
-    if (st == VFL_OK && e == cudaSuccess) e = cudaStreamSynchronize(origin);
     if (graph) cudaGraphDestroy(graph);
     if (st != VFL_OK || e != cudaSuccess) {
         vfl_graph_destroy(g);
