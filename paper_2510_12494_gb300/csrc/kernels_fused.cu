@@ -906,39 +906,67 @@ cudaError_t set_smem_attr(K kernel) {
     return e;
 }
 
+// Launch with the programmatic-launch attributes of `o` (a plain launch when it asks for none).
+template <typename Args>
+cudaError_t launch_with(void (*kernel)(const Args), const Args& a, int grid, int block, size_t smem, cudaStream_t s,
+                        const LaunchOpt& o) {
+    if (!o.serialize && !o.pevent) {
+        kernel<<<grid, block, smem, s>>>(a);
+        return cudaGetLastError();
+    }
+    cudaLaunchAttribute at[2];
+    int n = 0;
+    if (o.serialize) {
+        at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (o.pevent) {
+        at[n].id = cudaLaunchAttributeProgrammaticEvent;
+        at[n].val.programmaticEvent.event = o.pevent;
+        at[n].val.programmaticEvent.flags = 0;
+        at[n].val.programmaticEvent.triggerAtBlockStart = 0;
+        ++n;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = n;
+    return cudaLaunchKernelEx(&cfg, kernel, a);
+}
+
 }  // namespace
 
-cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s) {
+cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s, const LaunchOpt& o) {
     static cudaError_t attr = set_smem_attr(fused_passive_fwd_kernel);
     if (attr != cudaSuccess) return attr;
     const int ntiles = (a.rows + R - 1) / R;
-    fused_passive_fwd_kernel<<<ntiles, NT, fused_smem_fwd(a.w_floats, a.act_ld), s>>>(a);
-    return cudaGetLastError();
+    return launch_with(fused_passive_fwd_kernel, a, ntiles, NT, fused_smem_fwd(a.w_floats, a.act_ld), s, o);
 }
 
-cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s) {
+cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s, const LaunchOpt& o) {
     static cudaError_t attr = set_smem_attr(fused_active_kernel);
     if (attr != cudaSuccess) return attr;
     const int ntiles = (a.rows + R - 1) / R;
-    fused_active_kernel<<<ntiles, NT, fused_smem_active(a.w_floats, a.act_ld, a.na, a.nt), s>>>(a);
-    return cudaGetLastError();
+    return launch_with(fused_active_kernel, a, ntiles, NT, fused_smem_active(a.w_floats, a.act_ld, a.na, a.nt), s, o);
 }
 
-cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s) {
+cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s, const LaunchOpt& o) {
     static cudaError_t attr = set_smem_attr(fused_passive_bwd_kernel);
     if (attr != cudaSuccess) return attr;
     const int ntiles = (a.rows + R - 1) / R;
-    fused_passive_bwd_kernel<<<ntiles, NT, fused_smem_pbwd(a.w_floats, a.act_ld, a.na), s>>>(a);
-    return cudaGetLastError();
+    return launch_with(fused_passive_bwd_kernel, a, ntiles, NT, fused_smem_pbwd(a.w_floats, a.act_ld, a.na), s, o);
 }
 
-cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s) {
+cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s, const LaunchOpt& o) {
     static cudaError_t attr = cudaFuncSetAttribute(fused_update_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (attr != cudaSuccess) return attr;
     if (a.ntiles < 1 || a.rows < 1) return cudaErrorInvalidValue;
     // one more cluster than output tiles when the step's mean loss is wanted
-    fused_update_kernel<<<(a.ntiles + (a.loss_out ? 1 : 0)) * kUpdCluster, kUpdThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_with(fused_update_kernel, a, (a.ntiles + (a.loss_out ? 1 : 0)) * kUpdCluster, kUpdThreads, 0, s, o);
 }
 
 }  // namespace vfl

@@ -140,9 +140,19 @@ inline size_t fused_smem_pbwd(int w_floats, int act_ld, int nl) {
     return (size_t)(w_floats + (nl + 3) * kFusedRows * act_ld + kFusedRedFloats) * sizeof(float);
 }
 
-cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s);
-cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s);
-cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s);
-cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s);
+// Programmatic dependent launch outside CUDA graphs (a captured graph gets the same dependencies as
+// programmatic edges instead).  serialize: the kernel may launch once the previous kernel on its
+// stream has triggered (it waits for that grid before reading its output).  pevent: an event recorded
+// by the launch that fires once every CTA of this kernel has triggered; a kernel on another stream
+// that waits on it may launch then and waits for this grid before reading its output.
+struct LaunchOpt {
+    int serialize = 0;
+    cudaEvent_t pevent = nullptr;
+};
+
+cudaError_t launch_fused_passive_fwd(const FusedChainArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
+cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
+cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
+cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
 
 }  // namespace vfl

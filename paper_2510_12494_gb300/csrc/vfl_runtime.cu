@@ -200,6 +200,7 @@ struct vfl_ctx {
     // graph capture of the fused path: the kernel node of each (phase, step), so that the edges a
     // consumer only needs at a later point of its run become programmatic (see vfl_graph_capture)
     bool capturing = false;
+    bool direct_pdl = true;     // programmatic launches outside graphs (VFL_DISABLE_DIRECT_PDL turns them off)
     std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
@@ -862,6 +863,11 @@ void note_node(vfl_ctx* ctx, int ph, long long k, cudaStream_t s) {
 }
 
 // ---- fused path -------------------------------------------------------------
+// Direct enqueue (not captured, not timed per launch) gives the fused kernels the programmatic
+// dependencies a captured graph gets as edges: the passive forward and the active step record their
+// channel events programmatically, and each update launches behind its row kernel on the same stream.
+inline bool use_direct_pdl(const vfl_ctx* ctx) { return ctx->direct_pdl && !ctx->capturing && !ctx->prof_on; }
+
 FusedLayerArgs fused_layer(const Layer& L, int vslot, void* Y, long long ldy, void* D, long long ldd) {
     FusedLayerArgs f;
     std::memset(&f, 0, sizeof f);
@@ -930,7 +936,9 @@ vfl_status launch_update(vfl_ctx* ctx, FusedUpdArgs& u, int rows, cudaStream_t s
         bytes += (double)rows * (L.out + L.in) * 4 + ((double)L.out * L.in + L.out) * 16;
     }
     if (u.loss_out) bytes += rows * 4.0 + 4;
-    PLAUNCH(K_FUSED_UPDATE, flops, bytes, s, launch_fused_update(u, s));
+    LaunchOpt o;
+    o.serialize = use_direct_pdl(ctx) ? 1 : 0;   // behind its row kernel on the same stream
+    PLAUNCH(K_FUSED_UPDATE, flops, bytes, s, launch_fused_update(u, s, o));
     return VFL_OK;
 }
 
@@ -961,8 +969,10 @@ vfl_status fused_passive_forward(vfl_ctx* ctx, long long k, long long v, int slo
     // algorithmic bytes: the batch's features in, the saved activations out, one read of the weights
     double bytes = (double)rows * ctx->cfg.d_passive * 4;
     for (const Layer& L : ctx->P) bytes += (double)rows * L.out * 4 + ((double)L.out * L.in + L.out) * 4;
+    LaunchOpt o;
+    if (use_direct_pdl(ctx)) o.pevent = ctx->ev_emb[k % kEvPool];
     PLAUNCH(K_FUSED_PFWD, fused_flops(ctx->P, rows, true, false, false, false), bytes, s,
-            launch_fused_passive_fwd(a, s));
+            launch_fused_passive_fwd(a, s, o));
     return VFL_OK;
 }
 
@@ -1014,7 +1024,9 @@ vfl_status fused_active_step(vfl_ctx* ctx, long long k, long long v, int slot, i
     double bytes = (double)rows * (ctx->cfg.d_active + 3.0 * ep + 2) * 4;
     for (auto* vv : {&ctx->A, &ctx->T})
         for (const Layer& L : *vv) bytes += (double)rows * L.out * 8 + ((double)L.out * L.in + L.out) * 4;
-    PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, s));
+    LaunchOpt o;
+    if (use_direct_pdl(ctx)) o.pevent = ctx->ev_grad[k % kEvPool];
+    PLAUNCH(K_FUSED_ACTIVE, flops, bytes, s, launch_fused_active(a, s, o));
     return VFL_OK;
 }
 
@@ -1235,9 +1247,10 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
     }
     const void* X = xp_rows(ctx, k, r0);
     if (ctx->fused) {
+        const bool pdl = use_direct_pdl(ctx);
         TRY(fused_passive_forward(ctx, k, v, slot, vslot, rows, static_cast<const float*>(X), (int)(k % ctx->W), s));
         note_node(ctx, CAP_PFWD, k, s);
-        CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
+        if (!pdl) CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
         ctx->fwd_version[slot] = (int)v;
         ctx->slot_step_p[slot] = k;
         ctx->n_fwd = k + 1;
@@ -1290,9 +1303,10 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const void* Xa0 = xa_rows(ctx, k, r0);
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
+        const bool pdl = use_direct_pdl(ctx);
         TRY(fused_active_step(ctx, k, v, slot, vslot, rows, static_cast<const float*>(Xa0), w, s));
         note_node(ctx, CAP_ACTIVE, k, s);
-        CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
+        if (!pdl) CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
         // SGD on theta_1 in step order: version k+1 from version k
         TRY(wait_update_order(ctx, k, false, s));
         TRY(fused_active_update(ctx, k, rows, static_cast<const float*>(Xa0), w, s));
@@ -1569,6 +1583,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     for (int i = 0; i < kInfoRing; ++i) ctx->step_id[i] = -1;
     ctx->fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
     ctx->head = head_eligible(*cfg) && !getenv("VFL_DISABLE_HEAD");
+    ctx->direct_pdl = !getenv("VFL_DISABLE_DIRECT_PDL");
     build_layers(ctx);
     const unsigned long long need = carve_all(ctx, nullptr);
     if (workspace_bytes < need) {
