@@ -203,3 +203,14 @@ def test_deadline_from_a_missing_publish(vfl):
     assert np.isnan(got[3]) and np.isnan(ref[3])
     keep = drops == 0
     assert np.abs(got[keep] - ref[keep]).max() / np.abs(ref[keep]).max() < 1e-5
+
+
+@pytest.mark.parametrize("target", ["grad", "emb"])
+def test_drops_with_dp(vfl, target):
+    """Drops with either DP mechanism: the noise of a step is keyed by its step index, so the draws of the
+    steps after a drop are the oracle's."""
+    q = synth.preset(1).with_(n_rows=3 * 256 + 37, staleness=1, schedule="seeded", dp_clip=1.0, dp_sigma=0.7,
+                              dp_target=target)
+    drops = np.zeros(10, np.uint8)
+    drops[[2, 7]] = 1
+    assert_parity(vfl, q, 10, drops)

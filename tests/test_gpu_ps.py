@@ -165,3 +165,31 @@ def test_ps_average_matches_the_replica_mean(vfl):
             np.testing.assert_array_equal(r[w][key][1], r[0][key][1])
         assert rel_err(r[0][key][0], o.replica_params(0)[key][0]) < TOL["fp32"]
         assert rel_err(r[0][key][1], o.replica_params(0)[key][1]) < TOL["fp32"]
+
+
+def test_ps_with_embedding_dp(vfl):
+    """The parameter server with DP on the published embedding (fused kernels), against the oracle."""
+    q = ps_preset(1, 2, 1, 3 * 256 + 37, dp_clip=1.0, dp_sigma=0.5, dp_target="emb")
+    assert_parity(vfl, q, steps=9)
+
+
+def test_ps_host_data_equals_resident(vfl):
+    """Replicas trained from pinned host rows equal the device-resident run bit for bit."""
+    import torch
+    q = ps_preset(2, 3, 2, 4 * 1024 + 304)
+    steps = 3 * 5 + 2
+    ref = train(vfl, q, steps, "train_steps")
+    q2, xp, xa, y, params = setup(q, q.n_rows)
+    tp, ta = schedule(q2, steps)
+    ctx = vfl.Context(q2, q2.n_rows)
+    ctx.set_params(params)
+    pins = [torch.from_numpy(a).pin_memory() for a in (xp, xa, y)]
+    loss = torch.full((steps,), float("nan"), dtype=torch.float32).pin_memory()
+    ctx.bind_host_data(*pins, loss_out=loss)
+    ctx.train_steps(0, steps, tp, ta)
+    ctx.synchronize()
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, steps))
+    for w in range(3):
+        for key, (W, b) in ctx.get_replica(w).items():
+            np.testing.assert_array_equal(W, ref.get_replica(w)[key][0])
+            np.testing.assert_array_equal(b, ref.get_replica(w)[key][1])
