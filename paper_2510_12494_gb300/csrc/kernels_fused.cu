@@ -969,4 +969,11 @@ cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s, const Lau
     return launch_with(fused_update_kernel, a, (a.ntiles + (a.loss_out ? 1 : 0)) * kUpdCluster, kUpdThreads, 0, s, o);
 }
 
+bool is_fused_kernel(const void* func) {
+    return func == reinterpret_cast<const void*>(fused_passive_fwd_kernel) ||
+           func == reinterpret_cast<const void*>(fused_active_kernel) ||
+           func == reinterpret_cast<const void*>(fused_passive_bwd_kernel) ||
+           func == reinterpret_cast<const void*>(fused_update_kernel);
+}
+
 }  // namespace vfl

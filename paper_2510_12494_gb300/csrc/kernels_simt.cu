@@ -3,6 +3,7 @@
 // channel headers and data casts.
 #include "vfl_kernels.cuh"
 #include "vfl_philox.cuh"
+#include "vfl_pdl.cuh"
 
 namespace vfl {
 
@@ -27,6 +28,7 @@ constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
 
 template <typename TA, typename TB, typename TM>
 __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
+    pdl_entry();
     __shared__ float As[BK][BM + 1];
     __shared__ float Bs[BK][BN + 1];
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -129,6 +131,7 @@ constexpr int LOSS_NT = 1024;
 __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__ logits, const int* __restrict__ y,
                                                         int rows, int n_out, int kind, float* __restrict__ ds,
                                                         float* __restrict__ loss_out, float* loss_host) {
+    pdl_entry();
     __shared__ float red[LOSS_NT / 32];
     const float inv_b = 1.0f / (float)rows;
     float part = 0.f;
@@ -178,6 +181,7 @@ constexpr int HEAD_NT = 256;
 static_assert(kHeadMaxK == 32 * 8 && kHeadMaxOut <= 2 * (HEAD_NT / 32), "head thread map");
 
 __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
+    pdl_entry();
     __shared__ float Ws[kHeadMaxOut * kHeadMaxK];          // lane-minor: (j, 8l + e) at (8j + e) * 32 + l
     __shared__ __align__(16) __nv_bfloat16 hs[kHeadRows * kHeadMaxK];
     __shared__ float dss[kHeadRows * kHeadMaxOut];
@@ -342,6 +346,7 @@ constexpr int DP_NT = 256;
 __global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in, long long ld_in, void* out,
                                                     long long ld_out, int out_bf16, int e, float clip, float sigma,
                                                     unsigned long long seed, long long k, float bk) {
+    pdl_entry();
     __shared__ float red[DP_NT / 32];
     __shared__ float s_factor;
     const int r = blockIdx.x;
@@ -386,6 +391,7 @@ __global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in,
 __global__ void __launch_bounds__(DP_NT) dp_emb_kernel(const void* z, long long ld, int bf16, void* out,
                                                         float* __restrict__ scale_out, int e, float clip, float sigma,
                                                         unsigned long long seed, long long k) {
+    pdl_entry();
     __shared__ float red[DP_NT / 32];
     __shared__ float s_factor;
     const int r = blockIdx.x;
@@ -426,6 +432,7 @@ __global__ void __launch_bounds__(DP_NT) dp_emb_kernel(const void* z, long long 
 template <typename T>
 __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ z, T* __restrict__ out,
                                  long long ld, int rows, int e, const float* __restrict__ rs) {
+    pdl_entry();
     const long long n = (long long)rows * e;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
         const long long r = i / e, c = i % e;
@@ -438,6 +445,7 @@ __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ 
 // SGD (Eq. 2): master -= lr * sum_z partial[z]; write the new version's copy.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
+    pdl_entry();
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < a.total;
          i += (long long)gridDim.x * blockDim.x) {
         int l = 0;
@@ -465,6 +473,7 @@ __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
 
 __global__ void __launch_bounds__(256) ps_average_kernel(const PsAvgLayer* __restrict__ tab, int n_layers,
                                                          long long total, int nrep, int c_bf16) {
+    pdl_entry();
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         int l = 0;
@@ -495,12 +504,14 @@ __global__ void __launch_bounds__(256) ps_average_kernel(const PsAvgLayer* __res
 }
 
 __global__ void mark_dropped_kernel(float* loss, float* loss_host) {
+    pdl_entry();
     const float nan = __int_as_float(0x7FC00000);
     *loss = nan;
     if (loss_host) *loss_host = nan;
 }
 
 __global__ void write_header_kernel(ChannelHeader* h, long long k, int batch, int version) {
+    pdl_entry();
     h->k = k;
     h->batch = batch;
     h->version = version;
@@ -508,11 +519,13 @@ __global__ void write_header_kernel(ChannelHeader* h, long long k, int batch, in
 }
 
 __global__ void check_header_kernel(const ChannelHeader* h, long long k, int* status) {
+    pdl_entry();
     if (h->k != k) atomicOr(status, ST_VERSION);
 }
 
 // Bounded poll: gives up after max_iters reads and records ST_TIMEOUT.
 __global__ void wait_header_kernel(const ChannelHeader* h, long long k, long long max_iters, int* status) {
+    pdl_entry();
     const volatile long long* pk = &h->k;
     for (long long it = 0; it < max_iters; ++it) {
         if (*pk == k) return;
@@ -522,6 +535,7 @@ __global__ void wait_header_kernel(const ChannelHeader* h, long long k, long lon
 }
 
 __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d, void* dst, long long ld, int bf16) {
+    pdl_entry();
     const long long n = (long long)rows * ld;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
         const long long r = i / ld, c = i % ld;
@@ -535,6 +549,7 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
 __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const float* __restrict__ hxa, int da,
                                   const int* __restrict__ hy, int rows, void* xp, long long ld_p, void* xa,
                                   long long ld_a, int* __restrict__ y, int bf16) {
+    pdl_entry();
     const long long np = (long long)rows * ld_p, na = (long long)rows * ld_a;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < np + na + rows;
          i += (long long)gridDim.x * blockDim.x) {
@@ -556,6 +571,7 @@ __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const f
 // Reads 8 columns at a time, so D's row stride must cover ceil(out/8)*8 columns.
 __global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16,
                                                      float* __restrict__ Pb, long long pb_stride) {
+    pdl_entry();
     __shared__ float red[8][257];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int c0 = blockIdx.x * 256 + tx * 8;
@@ -597,6 +613,7 @@ __global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ld
 }
 
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
+    pdl_entry();
     const long long n = (long long)rows * cols;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
         const long long r = i / cols, c = i % cols;

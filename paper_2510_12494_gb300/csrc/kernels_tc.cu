@@ -23,6 +23,7 @@
 #include <mutex>
 
 #include "vfl_tc.cuh"
+#include "vfl_pdl.cuh"
 
 namespace vfl {
 
@@ -159,6 +160,7 @@ __device__ __forceinline__ float bf16_at(const void* base, long long idx) {
 __global__ void __launch_bounds__(THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap ta2,
                    const __grid_constant__ CUtensorMap tb, const __grid_constant__ CUtensorMap tb2, const TcParams p) {
+    pdl_entry();
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;

@@ -155,4 +155,8 @@ cudaError_t launch_fused_active(const FusedStepArgs& a, cudaStream_t s, const La
 cudaError_t launch_fused_passive_bwd(const FusedStepArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
 cudaError_t launch_fused_update(const FusedUpdArgs& a, cudaStream_t s, const LaunchOpt& o = LaunchOpt());
 
+// Whether a kernel (its function pointer, as a graph kernel node records it) is one of the fused kernels
+// above, which place their programmatic waits themselves; every other kernel of the library waits at entry.
+bool is_fused_kernel(const void* func);
+
 }  // namespace vfl

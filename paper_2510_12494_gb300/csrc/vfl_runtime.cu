@@ -2133,6 +2133,35 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
         cudaGraphNode_t from = node(CAP_PUPD, src), to = node(CAP_PFWD, k);
         if (from && to) make_programmatic(g, from, to);
     }
+    // every other kernel starts by waiting for its producer (pdl_entry), so any remaining plain edge
+    // between two kernel nodes whose target is not a fused kernel can be programmatic as well
+    size_t ne = 0;
+    if (cudaGraphGetEdges(g, nullptr, nullptr, nullptr, &ne) != cudaSuccess || ne == 0) {
+        cudaGetLastError();
+        return;
+    }
+    std::vector<cudaGraphNode_t> from(ne), to(ne);
+    std::vector<cudaGraphEdgeData> ed(ne);
+    if (cudaGraphGetEdges(g, from.data(), to.data(), ed.data(), &ne) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    auto kernel_func = [](cudaGraphNode_t n) -> const void* {
+        cudaGraphNodeType t;
+        cudaKernelNodeParams kp;
+        if (cudaGraphNodeGetType(n, &t) != cudaSuccess || t != cudaGraphNodeTypeKernel ||
+            cudaGraphKernelNodeGetParams(n, &kp) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        return kp.func;
+    };
+    for (size_t i = 0; i < ne; ++i) {
+        if (ed[i].type == cudaGraphDependencyTypeProgrammatic) continue;
+        const void* ff = kernel_func(from[i]);
+        const void* tf = kernel_func(to[i]);
+        if (ff && tf && !is_fused_kernel(tf)) make_programmatic(g, from[i], to[i]);
+    }
 }
 
 }  // namespace
