@@ -227,6 +227,15 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
 vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, float* b);
 
 /*
+ * Seeded initial parameters for every layer, as vfl_set_params would take them: each entry of
+ * layer l of party q (W row-major, then b) is (2u - 1) / sqrt(fan_in) in double, rounded to fp32,
+ * u = word i * 2^-32 of the stream Philox4x32-10(key = (seed lo, seed hi), counter = (i / 4 lo,
+ * i / 4 hi, (q << 8) | l, 0x49)) word i mod 4 -- U(-1/sqrt(fan_in), 1/sqrt(fan_in)).  Only valid
+ * before the first step.
+ */
+vfl_status vfl_init_params(vfl_ctx* ctx, uint64_t seed);
+
+/*
  * Gradient dLoss/dW [out, in] and dLoss/db [out] of one layer from the most
  * recent step of that party on worker `worker` (before the SGD update used
  * it).  Synchronizes the context.
@@ -360,6 +369,16 @@ vfl_status vfl_synchronize(vfl_ctx* ctx);
 /* Mean loss of steps [k0, k0+n) (float per step) into host memory; synchronizes.
  * Only the last 4096 steps are kept. */
 vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out);
+
+/*
+ * One epoch: steps [epoch * nb, (epoch + 1) * nb) (nb = ceil(n_rows / batch)) through
+ * vfl_train_steps (same arrays, indexed by absolute step; `drop` may be NULL), then, when
+ * mean_loss_out is not NULL, a synchronize and the epoch's mean loss per sample: each trained
+ * step's mean loss weighted by its rows (dropped steps count none).  The steps before the epoch
+ * must all be enqueued.
+ */
+vfl_status vfl_train_epoch(vfl_ctx* ctx, int64_t epoch, const int32_t* tau_p, const int32_t* tau_a,
+                           const uint8_t* drop, float* mean_loss_out);
 
 /*
  * Enqueue an asynchronous copy of the mean loss of step k (already enqueued)

@@ -105,6 +105,9 @@ EXPORTS = {
     "vfl_graph_capture": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
                                            ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
     "vfl_drop_step": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_init_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_uint64]),
+    "vfl_train_epoch": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
+                                         ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "vfl_get_drops": (ctypes.c_int32, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)]),
     "vfl_set_drops": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
     "vfl_make_drops": (ctypes.c_int32, [ctypes.c_uint64, ctypes.c_double, ctypes.c_int64, ctypes.c_void_p]),
@@ -465,6 +468,21 @@ class Context:
 
     def passive_backward(self, k):
         self._call(lib().vfl_passive_backward, k)
+
+    def init_params(self, seed: int):
+        """Seeded initial parameters (vfl_init_params; the recipe of synth.init_params)."""
+        self._call(lib().vfl_init_params, seed)
+
+    def train_epoch(self, epoch, tau_p, tau_a, drops=None, mean_loss=True):
+        """Steps of one epoch (vfl_train_epoch); returns the epoch's mean loss per sample (or None)."""
+        tau_p = np.ascontiguousarray(tau_p, np.int32)
+        tau_a = np.ascontiguousarray(tau_a, np.int32)
+        end = (epoch + 1) * self.nb
+        assert len(tau_p) >= end and len(tau_a) >= end
+        d, dp = _drops_ptr(drops, end)
+        out = ctypes.c_float()
+        self._call(lib().vfl_train_epoch, epoch, _ptr(tau_p), _ptr(tau_a), dp, ctypes.byref(out) if mean_loss else None)
+        return out.value if mean_loss else None
 
     def drop_step(self, k):
         """The subscriber of step k gives up on its embedding (see vfl_drop_step)."""

@@ -19,6 +19,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdarg>
+#include <limits>
 #include <map>
 #include <utility>
 #include <cstdio>
@@ -1527,6 +1528,32 @@ namespace vfl {
 void set_global_error(const char* msg) { g_global_err = msg; }
 }  // namespace vfl
 
+namespace {
+// Philox4x32-10 with counter (k lo, k hi, c2, c3) and key (seed lo, seed hi): the four output words.
+void philox4(uint64_t seed, int64_t k, uint32_t c2, uint32_t c3, uint32_t out[4]) {
+    uint32_t c[4] = {(uint32_t)(k & 0xFFFFFFFFu), (uint32_t)((uint64_t)k >> 32), c2, c3};
+    uint32_t key[2] = {(uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32)};
+    for (int r = 0; r < 10; ++r) {
+        const uint64_t p0 = (uint64_t)0xD2511F53u * c[0];
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * c[2];
+        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ key[0];
+        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ key[1];
+        c[0] = n0;
+        c[1] = (uint32_t)p1;
+        c[2] = n2;
+        c[3] = (uint32_t)p0;
+        key[0] += 0x9E3779B9u;
+        key[1] += 0xBB67AE85u;
+    }
+    for (int j = 0; j < 4; ++j) out[j] = c[j];
+}
+uint32_t philox_word0(uint64_t seed, int64_t k, uint32_t c2, uint32_t c3) {
+    uint32_t w[4];
+    philox4(seed, k, c2, c3, w);
+    return w[0];
+}
+}  // namespace
+
 // ============================================================================
 // C ABI
 // ============================================================================
@@ -1787,6 +1814,29 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
     return VFL_OK;
 }
 
+vfl_status vfl_init_params(vfl_ctx* ctx, uint64_t seed) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (ctx->started) return ctx->fail(VFL_E_STATE, "vfl_init_params after the first step");
+    for (std::vector<Layer>* v : {&ctx->P, &ctx->A, &ctx->T})
+        for (const Layer& L : *v) {
+            const long long nw = (long long)L.out * L.in, n = nw + L.out;
+            std::vector<float> vals((size_t)n);
+            const uint32_t sub = ((uint32_t)L.party << 8) | (uint32_t)L.idx;
+            const double scale = 1.0 / std::sqrt((double)L.in);
+            for (long long blk = 0; blk * 4 < n; ++blk) {
+                uint32_t w[4];
+                philox4(seed, blk, sub, 0x49u, w);
+                for (int j = 0; j < 4 && blk * 4 + j < n; ++j) {
+                    const double u = (double)w[j] * (1.0 / 4294967296.0);
+                    vals[(size_t)(blk * 4 + j)] = (float)((2.0 * u - 1.0) * scale);
+                }
+            }
+            TRY(vfl_set_params(ctx, L.party, L.idx, vals.data(), vals.data() + nw));
+        }
+    return VFL_OK;
+}
+
 vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, float* b) {
     if (!ctx || !W || !b) return ctx ? ctx->fail(VFL_E_INVAL, "null output pointer") : VFL_E_INVAL;
     if (ctx->broken) return VFL_E_CUDA;
@@ -1947,26 +1997,6 @@ vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queri
     return VFL_OK;
 }
 
-namespace {
-// Word 0 of Philox4x32-10 with counter (k lo, k hi, c2, c3) and key (seed lo, seed hi).
-uint32_t philox_word0(uint64_t seed, int64_t k, uint32_t c2, uint32_t c3) {
-    uint32_t c[4] = {(uint32_t)(k & 0xFFFFFFFFu), (uint32_t)((uint64_t)k >> 32), c2, c3};
-    uint32_t key[2] = {(uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32)};
-    for (int r = 0; r < 10; ++r) {
-        const uint64_t p0 = (uint64_t)0xD2511F53u * c[0];
-        const uint64_t p1 = (uint64_t)0xCD9E8D57u * c[2];
-        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ key[0];
-        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ key[1];
-        c[0] = n0;
-        c[1] = (uint32_t)p1;
-        c[2] = n2;
-        c[3] = (uint32_t)p0;
-        key[0] += 0x9E3779B9u;
-        key[1] += 0xBB67AE85u;
-    }
-    return c[0];
-}
-}  // namespace
 
 vfl_status vfl_make_drops(uint64_t seed, double rate, int64_t n_steps, uint8_t* drop) {
     if (!(rate >= 0.0 && rate <= 1.0) || n_steps < 0 || (n_steps > 0 && !drop)) {
@@ -2087,6 +2117,28 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
         }
         if (!progressed) return ctx->fail(VFL_E_STATE, "schedule cannot make progress at step %lld", ctx->n_bwd);
     }
+    return VFL_OK;
+}
+
+vfl_status vfl_train_epoch(vfl_ctx* ctx, int64_t epoch, const int32_t* tau_p, const int32_t* tau_a,
+                           const uint8_t* drop, float* mean_loss_out) {
+    if (!ctx) return VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    if (epoch < 0) return ctx->fail(VFL_E_INVAL, "epoch %lld < 0", (long long)epoch);
+    const long long k0 = epoch * ctx->nb;
+    TRY(vfl_train_steps(ctx, k0, ctx->nb, tau_p, tau_a, drop));
+    if (!mean_loss_out) return VFL_OK;
+    std::vector<float> loss((size_t)ctx->nb);
+    TRY(vfl_read_losses(ctx, k0, ctx->nb, loss.data()));
+    double tot = 0.0, rows = 0.0;
+    for (long long i = 0; i < ctx->nb; ++i) {
+        if (ctx->dropped(k0 + i)) continue;
+        long long r0;
+        const int n = ctx->batch_rows(k0 + i, &r0);
+        tot += (double)loss[(size_t)i] * n;
+        rows += n;
+    }
+    *mean_loss_out = rows > 0 ? (float)(tot / rows) : std::numeric_limits<float>::quiet_NaN();
     return VFL_OK;
 }
 

@@ -1,0 +1,55 @@
+"""The library's seeded parameter initialisation and its epoch call: the
+initial parameters equal the input generator's bit for bit (the same Philox
+stream), and vfl_train_epoch runs the epoch's steps and returns the mean loss
+per sample over the steps it trained, against the oracle."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _parity import new_context, schedule, setup
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def vfl():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2510_12494_gb300 import build
+    build.build()
+    import paper_2510_12494_gb300 as v
+    return v
+
+
+@pytest.mark.parametrize("cid,seed", [(1, 0), (2, 7), (5, 123456789012)])
+def test_init_params_equal_the_generator(vfl, cid, seed):
+    p = synth.preset(cid).with_(n_rows=4096)
+    ctx = vfl.Context(p, p.n_rows)
+    ctx.init_params(seed)
+    want = synth.init_params(p, seed)
+    for key, (W, b) in ctx.get_params().items():
+        np.testing.assert_array_equal(W, want[key][0])
+        np.testing.assert_array_equal(b, want[key][1])
+
+
+@pytest.mark.parametrize("with_drops", [False, True])
+def test_train_epoch_mean_loss(vfl, with_drops):
+    q, xp, xa, y, params = setup(synth.preset(2), 3 * 1024 + 304)
+    nb = q.steps_per_epoch
+    tp, ta = schedule(q, 2 * nb)
+    drops = None
+    if with_drops:
+        drops = np.zeros(2 * nb, np.uint8)
+        drops[[1, nb + 2]] = 1
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    got = [ctx.train_epoch(e, tp, ta, drops) for e in range(2)]
+    o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
+    for e in range(2):
+        losses, recs = o.run(tp, ta, nb, record_steps=range(e * nb, (e + 1) * nb), drops=drops)
+        rows = np.array([0 if r.dropped else r.rows[1] - r.rows[0] for r in (recs[k] for k in sorted(recs))])
+        want = np.nansum(losses * rows) / rows.sum()
+        assert abs(got[e] - want) / abs(want) < 1e-5
+        mine = ctx.read_losses(e * nb, nb)
+        assert np.isnan(mine).sum() == (0 if drops is None else int(drops[e * nb:(e + 1) * nb].sum()))
