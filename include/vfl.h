@@ -361,6 +361,28 @@ typedef struct vfl_graph vfl_graph;
 vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p,
                              const int32_t* tau_a, const uint8_t* drop, vfl_graph** out);
 vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* graph);
+
+/*
+ * Re-record `graph` for steps [k0, k0 + n_steps) (same preconditions as vfl_graph_capture) and update
+ * its executable graph in place (cudaGraphExecUpdate): far cheaper than a new capture's
+ * instantiation when the new window has the same shape.  Launches already in flight keep their old
+ * contents.  VFL_E_STATE when the shape differs (the graph is then unchanged and still replays its
+ * old window); windows of one length have one shape in the uniform order (vfl_set_order) without
+ * drops or parameter-server averaging.
+ */
+vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* graph, int64_t k0, int64_t n_steps, const int32_t* tau_p,
+                            const int32_t* tau_a, const uint8_t* drop);
+
+/*
+ * Dependency order of the enqueued steps.  VFL_ORDER_OVERLAP (default): a step waits only for the
+ * version it reads, so steps overlap as far as tau allows.  VFL_ORDER_UNIFORM: every step waits for
+ * all updates before it and is published after the previous backward, as if tau were 0, while
+ * still computing with versions k - tau -- the same results, less overlap, but one graph shape for
+ * every window (vfl_graph_update).  Only with no step in flight.
+ */
+#define VFL_ORDER_OVERLAP 0
+#define VFL_ORDER_UNIFORM 1
+vfl_status vfl_set_order(vfl_ctx* ctx, int32_t order);
 vfl_status vfl_graph_destroy(vfl_graph* graph);
 
 /* Wait for all enqueued work; returns VFL_E_VERSION / VFL_E_TIMEOUT recorded by kernels. */

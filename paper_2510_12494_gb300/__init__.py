@@ -105,6 +105,9 @@ EXPORTS = {
     "vfl_graph_capture": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
                                            ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
     "vfl_drop_step": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64]),
+    "vfl_graph_update": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+                                          ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
+    "vfl_set_order": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32]),
     "vfl_init_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_uint64]),
     "vfl_train_epoch": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
                                          ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
@@ -513,6 +516,22 @@ class Context:
         self._call(lib().vfl_graph_capture, k0, n, _ptr(tau_p), _ptr(tau_a), dp, ctypes.byref(g))
         self._graphs = getattr(self, "_graphs", []) + [g]
         return g
+
+    def update_graph(self, g, k0, n, tau_p, tau_a, drops=None) -> bool:
+        """Re-record g for steps [k0, k0+n) in place (vfl_graph_update); False when the shape differs."""
+        tau_p = np.ascontiguousarray(tau_p, np.int32)
+        tau_a = np.ascontiguousarray(tau_a, np.int32)
+        assert len(tau_p) >= k0 + n and len(tau_a) >= k0 + n
+        d, dp = _drops_ptr(drops, k0 + n)
+        st = lib().vfl_graph_update(self.h, g, k0, n, _ptr(tau_p), _ptr(tau_a), dp)
+        if st == VFL_E_STATE:
+            return False
+        _check(st, self.h)
+        return True
+
+    def set_order(self, uniform: bool):
+        """VFL_ORDER_UNIFORM (True) or VFL_ORDER_OVERLAP (False), see vfl_set_order."""
+        self._call(lib().vfl_set_order, 1 if uniform else 0)
 
     def launch_graph(self, g):
         self._call(lib().vfl_graph_launch, g)

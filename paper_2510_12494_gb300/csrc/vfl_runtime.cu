@@ -202,6 +202,10 @@ struct vfl_ctx {
     // consumer only needs at a later point of its run become programmatic (see vfl_graph_capture)
     bool capturing = false;
     bool direct_pdl = true;     // programmatic launches outside graphs (VFL_DISABLE_DIRECT_PDL turns them off)
+    // uniform dependency order (vfl_set_order): every step waits for the previous step's updates and is
+    // published after the previous backward, whatever its staleness, so that windows of steps have one
+    // graph shape (vfl_graph_update); the arithmetic, with its stale versions, is unchanged
+    bool uniform = false;
     std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
@@ -1169,6 +1173,7 @@ vfl_status wait_version(vfl_ctx* ctx, long long k, long long v, bool passive, cu
             TRY(wait_ev(ctx, s, (passive ? ctx->ev_pavg : ctx->ev_aavg)[a % kEvPool]));
         return VFL_OK;
     }
+    if (ctx->uniform) v = k;   // version k exists only after every version before it
     if (v > 0 && v > ctx->ordered_floor) TRY(wait_ev(ctx, s, (passive ? ctx->ev_pver : ctx->ev_aver)[v % kEvPool]));
     return VFL_OK;
 }
@@ -2068,6 +2073,15 @@ vfl_status vfl_drop_step(vfl_ctx* ctx, int64_t k) {
     return do_drop_active(ctx, k);
 }
 
+vfl_status vfl_set_order(vfl_ctx* ctx, int32_t order) {
+    if (!ctx) return VFL_E_INVAL;
+    if (order != VFL_ORDER_OVERLAP && order != VFL_ORDER_UNIFORM) return ctx->fail(VFL_E_INVAL, "unknown order %d", order);
+    if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "vfl_set_order with steps in flight");
+    ctx->uniform = order == VFL_ORDER_UNIFORM;
+    return VFL_OK;
+}
+
 vfl_status vfl_get_drops(vfl_ctx* ctx, int64_t* n) {
     if (!ctx || !n) return VFL_E_INVAL;
     *n = ctx->n_drops;
@@ -2103,7 +2117,8 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
     // is queued ahead of the backward of step k whenever tau_p permits.
     while (ctx->n_bwd < end) {
         bool progressed = false;
-        while (ctx->n_fwd < end && (ctx->psmode ? ps_need_bwd(ctx, ctx->n_fwd) : ctx->n_fwd - tau_p[ctx->n_fwd]) <= ctx->n_bwd) {
+        while (ctx->n_fwd < end && (ctx->psmode ? ps_need_bwd(ctx, ctx->n_fwd)
+                                    : ctx->uniform ? ctx->n_fwd : ctx->n_fwd - tau_p[ctx->n_fwd]) <= ctx->n_bwd) {
             TRY(do_passive_forward(ctx, ctx->n_fwd, tau_p[ctx->n_fwd], drop && drop[ctx->n_fwd]));
             progressed = true;
         }
@@ -2218,38 +2233,22 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
 
 }  // namespace
 
-vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
-                             const uint8_t* drop,
-                             vfl_graph** out) {
-    if (!ctx || !out) return VFL_E_INVAL;
-    *out = nullptr;
-    if (ctx->broken) return VFL_E_CUDA;
-    for (int w = 0; w < ctx->W; ++w)
-        if (!ctx->ps[w] || !ctx->as[w])
-            return ctx->fail(VFL_E_STATE, "graph capture needs the caller's streams (vfl_set_streams)");
-    if (k0 != ctx->n_fwd || k0 != ctx->n_act || k0 != ctx->n_bwd)
-        return ctx->fail(VFL_E_STATE, "vfl_graph_capture(%lld): steps before k0 are not all enqueued", (long long)k0);
-    // no synchronisation: earlier steps (a graph being replayed) may still run while the host captures the
-    // next window; the capture records work without executing it and its replay is ordered after them
-    vfl_graph* g = new vfl_graph();
-    g->ctx = ctx;
-    g->k0 = k0;
-    g->n = n_steps;
-    g->drops0 = ctx->n_drops;
-    g->hio = ctx->hio;
-    cudaError_t e = cudaEventCreateWithFlags(&g->fork, cudaEventDisableTiming);
-    for (int i = 0; i < kMaxStreams && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
-    if (e != cudaSuccess) {
-        delete g;
-        return ctx->cuda(e, "cudaEventCreate", __LINE__);
-    }
+}  // extern "C"
+
+namespace {
+
+// Record steps [k0, k0 + n) into a new cudaGraph (through vfl_train_steps on the context's streams in
+// capture mode, the fused kernels' programmatic edges added) without running them.  The context's host
+// state is left at k0; *after is the state once the captured steps have run.
+vfl_status capture_window(vfl_ctx* ctx, vfl_graph* g, long long k0, long long n_steps, const int32_t* tau_p,
+                          const int32_t* tau_a, const uint8_t* drop, cudaGraph_t* graph, HostState* after) {
+    *graph = nullptr;
     const HostState before = save_state(ctx);
     cudaStream_t origin = ctx->ps[0];
-    cudaGraph_t graph = nullptr;
     vfl_status st = VFL_OK;
     cudaStream_t ss[kMaxStreams];
     const int nss = ctx_streams(ctx, ss);
-    e = cudaStreamBeginCapture(origin, cudaStreamCaptureModeThreadLocal);
+    cudaError_t e = cudaStreamBeginCapture(origin, cudaStreamCaptureModeThreadLocal);
     if (e == cudaSuccess) e = cudaEventRecord(g->fork, origin);
     for (int i = 0; i < nss && e == cudaSuccess; ++i)
         if (ss[i] != origin) e = cudaStreamWaitEvent(ss[i], g->fork, 0);
@@ -2264,24 +2263,108 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
     for (int i = 0; i < nss; ++i)
         if (ss[i] != origin && cudaEventRecord(g->join[i], ss[i]) == cudaSuccess)
             cudaStreamWaitEvent(origin, g->join[i], 0);
-    cudaError_t e2 = cudaStreamEndCapture(origin, &graph);
+    cudaError_t e2 = cudaStreamEndCapture(origin, graph);
     if (e == cudaSuccess) e = e2;
-    if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, graph, k0, n_steps, tau_p);
+    if (st == VFL_OK && e == cudaSuccess) programmatic_edges(ctx, *graph, k0, n_steps, tau_p);
     ctx->cap_nodes.clear();
-    const HostState after = save_state(ctx);
+    *after = save_state(ctx);
+    after->launches -= before.launches;   // kernels per replay
     load_state(ctx, before);
-    if (st == VFL_OK && e == cudaSuccess) e = cudaGraphInstantiate(&g->exec, graph, 0);
-    // upload now (ordered on the origin stream, without waiting), so that the first replay does not pay for it
-    if (st == VFL_OK && e == cudaSuccess) e = cudaGraphUpload(g->exec, origin);
-    if (graph) cudaGraphDestroy(graph);
     if (st != VFL_OK || e != cudaSuccess) {
-        vfl_graph_destroy(g);
+        if (*graph) cudaGraphDestroy(*graph);
+        *graph = nullptr;
         if (st != VFL_OK) return st;
         return ctx->cuda(e, "graph capture", __LINE__);
     }
+    return VFL_OK;
+}
+
+vfl_status check_capture(vfl_ctx* ctx, long long k0) {
+    for (int w = 0; w < ctx->W; ++w)
+        if (!ctx->ps[w] || !ctx->as[w])
+            return ctx->fail(VFL_E_STATE, "graph capture needs the caller's streams (vfl_set_streams)");
+    if (k0 != ctx->n_fwd || k0 != ctx->n_act || k0 != ctx->n_bwd)
+        return ctx->fail(VFL_E_STATE, "graph capture at %lld: steps before it are not all enqueued", k0);
+    return VFL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int32_t* tau_p, const int32_t* tau_a,
+                             const uint8_t* drop,
+                             vfl_graph** out) {
+    if (!ctx || !out) return VFL_E_INVAL;
+    *out = nullptr;
+    if (ctx->broken) return VFL_E_CUDA;
+    TRY(check_capture(ctx, k0));
+    // no synchronisation: earlier steps (a graph being replayed) may still run while the host captures the
+    // next window; the capture records work without executing it and its replay is ordered after them
+    vfl_graph* g = new vfl_graph();
+    g->ctx = ctx;
+    g->k0 = k0;
+    g->n = n_steps;
+    g->drops0 = ctx->n_drops;
+    g->hio = ctx->hio;
+    cudaError_t e = cudaEventCreateWithFlags(&g->fork, cudaEventDisableTiming);
+    for (int i = 0; i < kMaxStreams && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&g->join[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        vfl_graph_destroy(g);
+        return ctx->cuda(e, "cudaEventCreate", __LINE__);
+    }
+    cudaGraph_t graph = nullptr;
+    HostState after;
+    vfl_status st = capture_window(ctx, g, k0, n_steps, tau_p, tau_a, drop, &graph, &after);
+    if (st != VFL_OK) {
+        vfl_graph_destroy(g);
+        return st;
+    }
+    e = cudaGraphInstantiate(&g->exec, graph, 0);
+    // upload now (ordered on the origin stream, without waiting), so that the first replay does not pay for it
+    if (e == cudaSuccess) e = cudaGraphUpload(g->exec, ctx->ps[0]);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+        vfl_graph_destroy(g);
+        return ctx->cuda(e, "graph instantiate", __LINE__);
+    }
     g->after = after;
-    g->launches = after.launches - before.launches;
+    g->launches = after.launches;
+    g->after.launches = 0;
     *out = g;
+    return VFL_OK;
+}
+
+vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* g, int64_t k0, int64_t n_steps, const int32_t* tau_p,
+                            const int32_t* tau_a, const uint8_t* drop) {
+    if (!ctx || !g || g->ctx != ctx) return ctx ? ctx->fail(VFL_E_INVAL, "graph of another context") : VFL_E_INVAL;
+    if (ctx->broken) return VFL_E_CUDA;
+    TRY(check_capture(ctx, k0));
+    cudaGraph_t graph = nullptr;
+    HostState after;
+    TRY(capture_window(ctx, g, k0, n_steps, tau_p, tau_a, drop, &graph, &after));
+    cudaGraphExecUpdateResultInfo info;
+    cudaError_t e = cudaGraphExecUpdate(g->exec, graph, &info);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        // a different shape of graph: the executable graph is unchanged and still valid for its old window
+        if (info.result == cudaGraphExecUpdateErrorTopologyChanged || info.result == cudaGraphExecUpdateErrorNodeTypeChanged ||
+            info.result == cudaGraphExecUpdateErrorFunctionChanged || info.result == cudaGraphExecUpdateErrorParametersChanged ||
+            info.result == cudaGraphExecUpdateErrorNotSupported || info.result == cudaGraphExecUpdateErrorAttributesChanged ||
+            info.result == cudaGraphExecUpdateErrorUnsupportedFunctionChange)
+            return ctx->fail(VFL_E_STATE, "steps [%lld, %lld) do not fit the graph's shape (update result %d)",
+                             (long long)k0, (long long)(k0 + n_steps), (int)info.result);
+        return ctx->cuda(e, "cudaGraphExecUpdate", __LINE__);
+    }
+    CK(cudaGraphUpload(g->exec, ctx->ps[0]));
+    g->k0 = k0;
+    g->n = n_steps;
+    g->drops0 = ctx->n_drops;
+    g->hio = ctx->hio;
+    g->launches = after.launches;
+    g->after = after;
+    g->after.launches = 0;
     return VFL_OK;
 }
 

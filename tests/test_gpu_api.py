@@ -53,3 +53,34 @@ def test_train_epoch_mean_loss(vfl, with_drops):
         assert abs(got[e] - want) / abs(want) < 1e-5
         mine = ctx.read_losses(e * nb, nb)
         assert np.isnan(mine).sum() == (0 if drops is None else int(drops[e * nb:(e + 1) * nb].sum()))
+
+
+@pytest.mark.parametrize("cid", [2, 3])
+def test_uniform_order_and_graph_updates(vfl, cid):
+    """The uniform dependency order computes exactly what the overlapping order does, and in it one
+    graph updated in place per epoch (vfl_graph_update) replays every epoch of a seeded schedule."""
+    rows = {2: 4 * 1024 + 304, 3: 2 * 4096 + 288}[cid]
+    q, xp, xa, y, params = setup(synth.preset(cid), rows)
+    nb = q.steps_per_epoch
+    n = 4 * nb
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    uni = new_context(vfl, q, xp, xa, y, params)
+    uni.set_order(True)
+    uni.train_steps(0, n, tp, ta)
+    np.testing.assert_array_equal(uni.read_losses(0, n), ref.read_losses(0, n))
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    ctx.set_order(True)
+    g = ctx.capture(0, nb, tp, ta)
+    ctx.launch_graph(g)
+    for e in range(1, 4):
+        assert ctx.update_graph(g, e * nb, nb, tp, ta), f"epoch {e} did not fit the graph"
+        ctx.launch_graph(g)
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+    for key, (W, b) in ctx.get_params().items():
+        np.testing.assert_array_equal(W, ref.get_params()[key][0])
+        np.testing.assert_array_equal(b, ref.get_params()[key][1])
+    with pytest.raises(vfl.VflError):
+        ctx.set_order(2)
