@@ -431,12 +431,17 @@ def run_ours(args):
             t0 = time.perf_counter()
             if graphs:
                 ctx.set_order(True)
-                g, gm = None, 0
+                cache = {}      # (window length, first worker) -> graph; a window's shape depends on both
                 k = k0
                 while k < k0 + K:
                     m = min(nb, k0 + K - k)
-                    if g is None or m != gm or not ctx.update_graph(g, k, m, tp, ta, drops):
-                        g, gm = ctx.capture(k, m, tp, ta, drops), m
+                    key = (m, k % p.workers)
+                    g = cache.get(key)
+                    if g is not None and ctx.update_graph(g, k, m, tp, ta, drops):
+                        counts["updated"] += 1
+                    else:
+                        g = cache[key] = ctx.capture(k, m, tp, ta, drops)
+                        counts["captured"] += 1
                     ctx.launch_graph(g)
                     k += m
             else:
@@ -451,12 +456,14 @@ def run_ours(args):
             assert np.isfinite(loss_host.numpy()[kept]).all() and np.isnan(loss_host.numpy()[~kept]).all()
             return job_throughput(samples(p, k0, K, drops), world, dt)
 
+        counts = {"updated": 0, "captured": 0}
         direct = e2e_run(W + 2 * K, False)
         piped = e2e_run(W + 3 * K, True) if use_graphs else None
         ctx.bind_host_data(None, None, None)
         h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
         e2e = {"value": max(direct, piped or 0.0), "unit": "samples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": 4, "direct_enqueue": direct, "uniform_order_graph_updates": piped,
+               "graph_windows": counts,
                "method": "uniform-order graphs updated in flight" if piped and piped > direct else "direct enqueue"}
 
     if rank == 0:

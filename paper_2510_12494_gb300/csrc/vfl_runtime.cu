@@ -2196,7 +2196,8 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
         }
         // the update that made the forward's weights: step v - 1 for version v = k - tau_p, the previous
         // step of the worker in the parameter-server mode (no edge when an averaging sits in between)
-        const long long src = ctx->psmode ? k - ctx->W : k - tau_p[k] - 1;
+        // (in the uniform order the forward waits for the previous step's update, whatever it reads)
+        const long long src = ctx->psmode ? k - ctx->W : ctx->uniform ? k - 1 : k - tau_p[k] - 1;
         cudaGraphNode_t from = node(CAP_PUPD, src), to = node(CAP_PFWD, k);
         if (from && to) make_programmatic(g, from, to);
     }
