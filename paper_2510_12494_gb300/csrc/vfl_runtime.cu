@@ -1181,7 +1181,8 @@ vfl_status wait_version(vfl_ctx* ctx, long long k, long long v, bool passive, cu
 // Before step k's update on s: updates apply in step order (App. D); in the parameter-server mode
 // the replica's previous update ran on the same stream.
 vfl_status wait_update_order(vfl_ctx* ctx, long long k, bool passive, cudaStream_t s) {
-    if (ctx->psmode || k <= 0 || k <= ctx->ordered_floor) return VFL_OK;
+    // in the uniform order the step's first launch on this stream already waited for update k-1
+    if (ctx->psmode || ctx->uniform || k <= 0 || k <= ctx->ordered_floor) return VFL_OK;
     return wait_ev(ctx, s, (passive ? ctx->ev_pver : ctx->ev_aver)[k % kEvPool]);
 }
 
@@ -2358,7 +2359,6 @@ vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* g, int64_t k0, int64_t n_st
                              (long long)k0, (long long)(k0 + n_steps), (int)info.result);
         return ctx->cuda(e, "cudaGraphExecUpdate", __LINE__);
     }
-    CK(cudaGraphUpload(g->exec, ctx->ps[0]));
     g->k0 = k0;
     g->n = n_steps;
     g->drops0 = ctx->n_drops;
