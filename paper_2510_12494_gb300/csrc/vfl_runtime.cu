@@ -1306,7 +1306,9 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     const int n_out = ctx->T.back().out;
 
     TRY(wait_version(ctx, k, v, false, s));
-    if (ctx->hio) TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
+    // the per-layer path reads x^a's staged rows before it subscribes; the fused kernel launches behind the
+    // publisher, which itself waited for the staging
+    if (ctx->hio && !ctx->fused) TRY(wait_ev(ctx, s, ctx->ev_staged[k % kEvPool]));
     const void* Xa0 = xa_rows(ctx, k, r0);
     if (ctx->fused) {
         TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
