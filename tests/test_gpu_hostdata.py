@@ -114,3 +114,29 @@ def test_fetch_loss_copies_each_step_loss(vfl):
         ctx.fetch_loss(k, out.data_ptr() + 4 * k)
     ctx.synchronize()
     np.testing.assert_array_equal(out.numpy(), ctx.read_losses(0, n))
+
+
+def test_host_data_uniform_order_graph_updates(vfl):
+    """The end-to-end path: host-resident rows, the uniform dependency order, one graph per epoch updated
+    in place -- the same losses and weights as direct enqueue on resident data."""
+    p = synth.preset(2)
+    rows = 4 * 1024 + 304
+    q, xp, xa, y, params = setup(p, rows)
+    nb = q.steps_per_epoch
+    n = 4 * nb
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx, loss = host_context(vfl, q, xp, xa, y, params, cap=n)
+    ctx.set_order(True)
+    graphs = {}
+    for e in range(4):
+        w = (e * nb) % q.workers
+        if w not in graphs:
+            graphs[w] = ctx.capture(e * nb, nb, tp, ta)
+        else:
+            assert ctx.update_graph(graphs[w], e * nb, nb, tp, ta)
+        ctx.launch_graph(graphs[w])
+    ctx.synchronize()
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
+    assert_same_state(ctx, ref)
