@@ -569,13 +569,13 @@ __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const f
 // [256 x, 256 x + 256) of rows [64 y, 64 y + 64); tx owns 8 adjacent columns,
 // ty every 8th row; the 8 row lanes are combined in a fixed order.
 // Reads 8 columns at a time, so D's row stride must cover ceil(out/8)*8 columns.
-__global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16,
-                                                     float* __restrict__ Pb, long long pb_stride) {
-    pdl_entry();
+// Column block bx (256 columns) of row block by (64 rows) of one column-sum job.
+__device__ __forceinline__ void colsum_block(const void* D, long long ldd, int rows, int out, int bf16,
+                                             float* __restrict__ Pb, long long pb_stride, int bx, int by) {
     __shared__ float red[8][257];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-    const int c0 = blockIdx.x * 256 + tx * 8;
-    const int rb = blockIdx.y * 64;
+    const int c0 = bx * 256 + tx * 8;
+    const int rb = by * 64;
     float acc[8] = {};
     if (c0 < out) {
 #pragma unroll
@@ -603,13 +603,27 @@ __global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ld
 #pragma unroll
     for (int q = 0; q < 8; ++q) red[ty][tx * 8 + q] = acc[q];
     __syncthreads();
-    const int c = blockIdx.x * 256 + threadIdx.x;
+    const int c = bx * 256 + threadIdx.x;
     if (c < out) {
         float t = 0.f;
 #pragma unroll
         for (int y = 0; y < 8; ++y) t += red[y][threadIdx.x];
-        Pb[(long long)blockIdx.y * pb_stride + c] = t;
+        Pb[(long long)by * pb_stride + c] = t;
     }
+}
+
+__global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16,
+                                                     float* __restrict__ Pb, long long pb_stride) {
+    pdl_entry();
+    colsum_block(D, ldd, rows, out, bf16, Pb, pb_stride, blockIdx.x, blockIdx.y);
+}
+
+// Several layers' column sums in one launch: job blockIdx.z, blocks outside the job's grid return.
+__global__ void __launch_bounds__(256) colsum_batch_kernel(const ColsumBatch b) {
+    pdl_entry();
+    const ColsumJob& j = b.j[blockIdx.z];
+    if ((int)blockIdx.x >= (j.out + 255) / 256 || (int)blockIdx.y >= j.nblocks) return;
+    colsum_block(j.D, j.ldd, j.rows, j.out, j.bf16, j.Pb, j.pb_stride, blockIdx.x, blockIdx.y);
 }
 
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
@@ -738,6 +752,19 @@ cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int b
     if (nblocks < 1) return cudaErrorInvalidValue;
     dim3 grid((out + 255) / 256, nblocks);
     colsum_kernel<<<grid, 256, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_colsum_batch(const ColsumBatch& b, cudaStream_t s) {
+    if (b.n < 1) return cudaSuccess;
+    if (b.n > kMaxColsumJobs) return cudaErrorInvalidValue;
+    int gx = 1, gy = 1;
+    for (int i = 0; i < b.n; ++i) {
+        if (b.j[i].nblocks < 1) return cudaErrorInvalidValue;
+        gx = max(gx, (b.j[i].out + 255) / 256);
+        gy = max(gy, b.j[i].nblocks);
+    }
+    colsum_batch_kernel<<<dim3(gx, gy, b.n), 256, 0, s>>>(b);
     return cudaGetLastError();
 }
 

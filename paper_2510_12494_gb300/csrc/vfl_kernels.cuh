@@ -152,6 +152,18 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
 // stride must cover ceil(out / 8) * 8 columns.
 cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
                           int nblocks, cudaStream_t s);
+// The same column sums for several layers in one launch (jobs in any order; each as launch_colsum).
+struct ColsumJob {
+    const void* D; long long ldd;
+    int rows, out, bf16, nblocks;
+    float* Pb; long long pb_stride;
+};
+constexpr int kMaxColsumJobs = 16;
+struct ColsumBatch {
+    ColsumJob j[kMaxColsumJobs];
+    int n;
+};
+cudaError_t launch_colsum_batch(const ColsumBatch& b, cudaStream_t s);
 
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);

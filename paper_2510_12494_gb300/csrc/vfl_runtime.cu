@@ -206,6 +206,9 @@ struct vfl_ctx {
     // published after the previous backward, whatever its staleness, so that windows of steps have one
     // graph shape (vfl_graph_update); the arithmetic, with its stale versions, is unchanged
     bool uniform = false;
+    // bias column sums of the per-layer path, gathered over a party's backward and launched as one batch
+    // before its SGD (the d(pre) buffers stay until then)
+    ColsumBatch cs_pending{};
     std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
@@ -294,6 +297,12 @@ struct vfl_graph {
     bool hio;                  // captured with host data bound (its copies are part of the graph)
     cudaEvent_t fork, join[2 * kMaxWorkers + 1];
 };
+
+#define TRY(x)                          \
+    do {                                \
+        vfl_status st_ = (x);           \
+        if (st_ != VFL_OK) return st_;  \
+    } while (0)
 
 #define CK(call)                                                     \
     do {                                                             \
@@ -719,6 +728,28 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
     return VFL_OK;
 }
 
+// Launch the gathered column sums as one batch on s (before the SGD that reads them).
+vfl_status flush_colsum(vfl_ctx* ctx, cudaStream_t s) {
+    ColsumBatch& b = ctx->cs_pending;
+    if (b.n == 0) return VFL_OK;
+    double bytes = 0;
+    for (int i = 0; i < b.n; ++i)
+        bytes += (double)b.j[i].rows * b.j[i].out * (b.j[i].bf16 ? 2 : 4) + (double)b.j[i].nblocks * b.j[i].out * 4;
+    PLAUNCH(K_COLSUM, 0, bytes, s, launch_colsum_batch(b, s));
+    b.n = 0;
+    return VFL_OK;
+}
+
+// Queue one layer's bias column sums (64-row block partials) for the party's batch.
+vfl_status defer_colsum(vfl_ctx* ctx, const void* D, long long ldd, int rows, int out, int bf16, float* Pb,
+                        long long pb_stride, int nblocks, cudaStream_t s) {
+    if (ctx->cs_pending.n == kMaxColsumJobs) TRY(flush_colsum(ctx, s));
+    ColsumJob& j = ctx->cs_pending.j[ctx->cs_pending.n++];
+    j.D = D; j.ldd = ldd; j.rows = rows; j.out = out; j.bf16 = bf16; j.nblocks = nblocks;
+    j.Pb = Pb; j.pb_stride = pb_stride;
+    return VFL_OK;
+}
+
 // Partial dW, db of layer L for the step on worker w:
 //   dW[out, in] = dpre^T X, dpre [rows, out] (leading dim ldd, fp32 when dpre_f32).
 //   X may be [X1 | X2] split at column ka (then two GEMMs write the two column blocks).
@@ -740,8 +771,7 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
         t.nsplit = L.nsplit; t.kchunk = L.kchunk;
         t.err = ctx->status;
         PLAUNCH(K_TC_DW, flops, bytes, s, launch_tc_gemm(t, s));
-        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz + (double)L.nsplit_b * L.out * 4, s,
-                launch_colsum(dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit_b, s));
+        TRY(defer_colsum(ctx, dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit_b, s));
         return VFL_OK;
     }
     const int n1 = X2 ? ka : L.in;
@@ -753,9 +783,7 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
     g.kchunk = L.kchunk;
     const double f1 = X2 ? flops * n1 / L.in : flops, b1 = X2 ? bytes * n1 / L.in : bytes;
     PLAUNCH(K_SIMT_DW, f1, b1, s, launch_gemm_simt(g, a_bf, bf, bf, L.nsplit, s));
-    if (L.colsum_bias)
-        PLAUNCH(K_COLSUM, 0, (double)rows * L.out * ctx->esz, s,
-                launch_colsum(dpre, ldd, rows, L.out, a_bf, L.pb[w], L.out, L.nsplit_b, s));
+    if (L.colsum_bias) TRY(defer_colsum(ctx, dpre, ldd, rows, L.out, a_bf, L.pb[w], L.out, L.nsplit_b, s));
     if (X2) {
         GemmArgs g2 = gemm_base(GEMM_DW, L.out, L.in - ka, rows);
         g2.A = dpre; g2.a_rs = 1; g2.a_cs = ldd;
@@ -844,11 +872,6 @@ vfl_status wait_ev(vfl_ctx* ctx, cudaStream_t s, cudaEvent_t e) {
     return VFL_OK;
 }
 
-#define TRY(x)                          \
-    do {                                \
-        vfl_status st_ = (x);           \
-        if (st_ != VFL_OK) return st_;  \
-    } while (0)
 
 // Fused-path phases whose kernel nodes a capture records.
 enum CapPhase : int { CAP_PFWD, CAP_ACTIVE, CAP_AUPD, CAP_PBWD, CAP_PUPD };
@@ -1428,6 +1451,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     }
     // SGD on theta_1 in step order: version k+1 from version k
     TRY(wait_update_order(ctx, k, false, s));
+    TRY(flush_colsum(ctx, s));
     TRY(sgd(ctx, &ctx->A, &ctx->T, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
     CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
@@ -1485,6 +1509,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
         }
     }
     TRY(wait_update_order(ctx, k, true, s));
+    TRY(flush_colsum(ctx, s));
     TRY(sgd(ctx, &ctx->P, nullptr, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
     CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, true, s));
