@@ -29,6 +29,7 @@ constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
 template <typename TA, typename TB, typename TM>
 __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
     pdl_entry();
+    header_check(g.hdr);
     __shared__ float As[BK][BM + 1];
     __shared__ float Bs[BK][BN + 1];
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -112,6 +113,7 @@ __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
             }
         }
     }
+    header_publish(g.hdr);
 }
 
 template <typename TA, typename TB>
@@ -431,8 +433,9 @@ __global__ void __launch_bounds__(DP_NT) dp_emb_kernel(const void* z, long long 
 // out = g * [z > 0], with g first scaled by rs[row] when rs is given (rounded to T)
 template <typename T>
 __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ z, T* __restrict__ out,
-                                 long long ld, int rows, int e, const float* __restrict__ rs) {
+                                 long long ld, int rows, int e, const float* __restrict__ rs, const HeaderOps hdr) {
     pdl_entry();
+    header_check(hdr);
     const long long n = (long long)rows * e;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
         const long long r = i / e, c = i % e;
@@ -682,15 +685,16 @@ cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_
 }
 
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
-                             const float* row_scale, cudaStream_t s) {
+                             const float* row_scale, const HeaderOps& hdr, cudaStream_t s) {
     const int nb = grid_for((long long)rows * e, 256);
     if (bf16)
         relu_mask_kernel<__nv_bfloat16><<<nb, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(g),
                                                            static_cast<const __nv_bfloat16*>(z),
-                                                           static_cast<__nv_bfloat16*>(out), ld, rows, e, row_scale);
+                                                           static_cast<__nv_bfloat16*>(out), ld, rows, e, row_scale,
+                                                           hdr);
     else
         relu_mask_kernel<float><<<nb, 256, 0, s>>>(static_cast<const float*>(g), static_cast<const float*>(z),
-                                                   static_cast<float*>(out), ld, rows, e, row_scale);
+                                                   static_cast<float*>(out), ld, rows, e, row_scale, hdr);
     return cudaGetLastError();
 }
 

@@ -58,6 +58,7 @@ struct TcParams {
     float* P;
     long long p_stride;
     int* err;
+    HeaderOps hdr;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -161,6 +162,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap ta2,
                    const __grid_constant__ CUtensorMap tb, const __grid_constant__ CUtensorMap tb2, const TcParams p) {
     pdl_entry();
+    header_check(p.hdr);
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;
@@ -382,6 +384,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
     }
+    header_publish(p.hdr);
 }
 
 // ---------------------------------------------------------------------------
@@ -465,6 +468,7 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
     p.N = g.N;
     p.K = g.K;
     p.err = g.err;
+    p.hdr = g.hdr;
     CUtensorMap ta, ta2, tb, tb2;
     std::memset(&ta, 0, sizeof ta);
     std::memset(&ta2, 0, sizeof ta2);

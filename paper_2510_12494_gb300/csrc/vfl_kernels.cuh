@@ -30,6 +30,32 @@ enum GemmMode : int { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
 //        columns n >= n_split to C2 at column n - n_split (masked by mask2 when set).
 //   DW : split-K partial: P[z * p_stride + m * ldc + n] = sum over k in chunk z;
 //        Pb[z * pb_stride + m] = sum_k A(m, k) over the chunk (bias gradient).
+// Channel-header work folded into a kernel of the step (instead of a one-thread kernel of its own):
+// thread 0 of CTA 0 checks `chk` at entry (another step's header sets ST_VERSION in *status) and writes
+// `pub` = {k, batch, version} when it ends; readers of `pub` wait for the whole grid to complete first.
+struct HeaderOps {
+    ChannelHeader* pub;
+    const ChannelHeader* chk;
+    long long k;
+    int batch, version;
+    int* status;
+};
+#ifdef __CUDACC__
+__device__ __forceinline__ bool first_thread_of_grid() {
+    return blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0;
+}
+__device__ __forceinline__ void header_check(const HeaderOps& h) {
+    if (h.chk && first_thread_of_grid() && h.chk->k != h.k) atomicOr(h.status, ST_VERSION);
+}
+__device__ __forceinline__ void header_publish(const HeaderOps& h) {
+    if (h.pub && first_thread_of_grid()) {
+        h.pub->k = h.k;
+        h.pub->batch = h.batch;
+        h.pub->version = h.version;
+    }
+}
+#endif
+
 struct GemmArgs {
     int mode;
     int M, N, K;
@@ -44,6 +70,7 @@ struct GemmArgs {
     float* P; long long p_stride;
     float* Pb; long long pb_stride;
     int kchunk;
+    HeaderOps hdr;
 };
 
 // Launch the SIMT GEMM (fp32 FFMA).  a_bf16 / b_bf16 select operand element
@@ -72,7 +99,7 @@ cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, floa
 // out[r, c] = g[r, c] * (z[r, c] > 0), compute dtype, [rows, e] with leading dim ld; with row_scale,
 // g[r, c] is first multiplied by row_scale[r] (and rounded to the compute dtype).
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
-                             const float* row_scale, cudaStream_t s);
+                             const float* row_scale, const HeaderOps& hdr, cudaStream_t s);
 
 struct SgdLayer {
     float* W; float* b;           // fp32 master

@@ -700,7 +700,7 @@ GemmArgs gemm_base(int mode, int M, int N, int K) {
 // Y[rows, out] = act(X W^T + b); X may be [X1 | X2] split at column ka.
 vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, long long ldx, const void* X2,
                       long long ldx2, int ka, int rows, void* Y, long long ldy, bool relu, bool y_f32,
-                      cudaStream_t s) {
+                      cudaStream_t s, const HeaderOps* hdr = nullptr) {
     const int in_bf = ctx->bf16;
     const double flops = 2.0 * rows * L.out * L.in;
     const double bytes = ((double)rows * L.in + (double)L.out * L.in) * ctx->esz +
@@ -714,6 +714,7 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
         t.bias = L.cb[slot]; t.relu = relu;
         t.C = Y; t.ldc = ldy;
         t.err = ctx->status;
+        if (hdr) t.hdr = *hdr;
         PLAUNCH(K_TC_FWD, flops, bytes, s, launch_tc_gemm(t, s));
         return VFL_OK;
     }
@@ -724,6 +725,7 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
     g.bias = L.cb[slot];
     g.relu = relu ? 1 : 0;
     g.C = Y; g.ldc = ldy; g.c_bf16 = y_f32 ? 0 : in_bf;
+    if (hdr) g.hdr = *hdr;
     PLAUNCH(K_SIMT_FWD, flops, bytes, s, launch_gemm_simt(g, in_bf, in_bf, in_bf, 1, s));
     return VFL_OK;
 }
@@ -800,7 +802,7 @@ vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long
 // mask1 > 0), the rest -> C2 (masked by mask2 when given).
 vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, long long ldd, bool dpre_f32,
                      int rows, void* C, long long ldc, const void* mask1, int n_split, void* C2, long long ldc2,
-                     bool c2_f32, const void* mask2, cudaStream_t s) {
+                     bool c2_f32, const void* mask2, cudaStream_t s, const HeaderOps* hdr = nullptr) {
     const int bf = ctx->bf16;
     const double flops = 2.0 * rows * L.out * L.in;
     const double bytes = (double)rows * L.out * (dpre_f32 ? 4 : ctx->esz) + (double)L.out * L.in * ctx->esz +
@@ -815,6 +817,7 @@ vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, l
         t.n_split = n_split; t.C2 = C2; t.ldc2 = ldc2; t.mask2 = mask2;
         t.c2_f32 = c2_f32 ? 1 : 0;
         t.err = ctx->status;
+        if (hdr) t.hdr = *hdr;
         PLAUNCH(K_TC_DX, flops, bytes, s, launch_tc_gemm(t, s));
         return VFL_OK;
     }
@@ -826,6 +829,7 @@ vfl_status linear_dx(vfl_ctx* ctx, const Layer& L, int slot, const void* dpre, l
     g.n_split = n_split;
     g.C2 = C2; g.ldc2 = ldc2; g.c2_bf16 = c2_f32 ? 0 : bf;
     g.mask2 = mask2; g.mask2_ld = ldc2;
+    if (hdr) g.hdr = *hdr;
     PLAUNCH(K_SIMT_DX, flops, bytes, s, launch_gemm_simt(g, dpre_f32 ? 0 : bf, bf, bf, 1, s));
     return VFL_OK;
 }
@@ -1288,10 +1292,17 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
         return VFL_OK;
     }
     long long ldx = ctx->ldxp;
+    // the embedding's header is published by the kernel that writes the payload last
+    HeaderOps pub{};
+    pub.pub = ctx->emb_hdr + slot;
+    pub.k = k;
+    pub.batch = (int)ctx->batch_of(k);
+    pub.version = (int)v;
     for (size_t l = 0; l < ctx->P.size(); ++l) {
         const Layer& L = ctx->P[l];
         void* Y = ctx->act_p[slot][l];
-        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, Y, ld8(L.out), true, false, s));
+        const bool publish = l + 1 == ctx->P.size() && !emb_dp(ctx);
+        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, Y, ld8(L.out), true, false, s, publish ? &pub : nullptr));
         X = Y;
         ldx = ld8(L.out);
     }
@@ -1300,8 +1311,8 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
         PLAUNCH(K_DP, 0, (double)rows * ep * 2 * ctx->esz + rows * 4.0, s,
                 launch_dp_emb(ctx->act_p[slot].back(), ld8(ep), ctx->bf16, ctx->emb_pub[slot], ctx->emb_c[slot], rows,
                               ep, c.dp_clip, c.dp_sigma, c.dp_seed, k, s));
+        PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
     }
-    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->emb_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
     CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
     ctx->fwd_version[slot] = (int)v;
     ctx->slot_step_p[slot] = k;
@@ -1359,9 +1370,12 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         X = ctx->act_a[w][l];
         ldx = ld8(L.out);
     }
-    // subscribe: wait for the embedding of step k, check its header
+    // subscribe: wait for the embedding of step k; the first kernel that reads it checks its header
     TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
-    PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->emb_hdr + slot, k, ctx->status, s));
+    HeaderOps sub{};
+    sub.chk = ctx->emb_hdr + slot;
+    sub.k = k;
+    sub.status = ctx->status;
     const void* Za = ctx->act_a[w][La - 1];
     const void* Zp = emb_dp(ctx) ? ctx->emb_pub[slot] : ctx->act_p[slot][Lp - 1];
     // top forward on [z^a | z^p]; with the head kernel, g's output layer runs with the loss
@@ -1372,7 +1386,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         void* Y = last ? (void*)ctx->logits[w] : ctx->act_t[w][l];
         const long long ldy = last ? n_out : ld8(L.out);
         if (l == 0)
-            TRY(linear_fwd(ctx, L, vslot, Za, ld8(ea), Zp, ld8(ep), ea, rows, Y, ldy, !last, last, s));
+            TRY(linear_fwd(ctx, L, vslot, Za, ld8(ea), Zp, ld8(ep), ea, rows, Y, ldy, !last, last, s, &sub));
         else
             TRY(linear_fwd(ctx, L, vslot, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0, rows, Y, ldy,
                            !last, last, s));
@@ -1424,17 +1438,24 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
                           L.in, nullptr, 0, false, nullptr, s));
         } else {
             // split: dz^a (masked -> dpre of the active cut layer), dz^p -> gradient channel (or fp32 for DP)
+            // without DP this kernel writes the published gradient and its header
             void* C2 = dp ? (void*)ctx->dzp32[w] : ctx->grad[slot];
+            HeaderOps gpub{};
+            gpub.pub = ctx->grad_hdr + slot;
+            gpub.k = k;
+            gpub.batch = (int)ctx->batch_of(k);
+            gpub.version = (int)v;
             TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_a[w][La - 1], ld8(ea), Za, ea, C2,
-                          ld8(ep), dp, nullptr, s));
+                          ld8(ep), dp, nullptr, s, dp ? nullptr : &gpub));
         }
     }
-    if (dp)
+    if (dp) {
         PLAUNCH(K_DP, 0, (double)rows * ep * (4 + ctx->esz), s,
                 launch_dp(ctx->dzp32[w], ld8(ep), ctx->grad[slot], ld8(ep), ctx->bf16, rows, ep, c.dp_clip,
                           c.dp_sigma, c.dp_seed, k, s));
+        PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
+    }
     // publish the gradient
-    PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
     CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
     ctx->grad_step[slot] = k;
     // active bottom backward
@@ -1490,12 +1511,16 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
         ctx->n_bwd = k + 1;
         return VFL_OK;
     }
-    PLAUNCH(K_HEADER, 0, 16, s, launch_check_header(ctx->grad_hdr + slot, k, ctx->status, s));
     // dpre of the cut layer = dLoss/dz^p * [z^p > 0]; with DP on the embedding the received gradient is
-    // first scaled by the row's clip factor (straight-through backward of the mechanism)
+    // first scaled by the row's clip factor (straight-through backward of the mechanism); the kernel checks
+    // the gradient's header
+    HeaderOps sub{};
+    sub.chk = ctx->grad_hdr + slot;
+    sub.k = k;
+    sub.status = ctx->status;
     PLAUNCH(K_MASK, 0, 3.0 * rows * ep * ctx->esz, s,
             launch_relu_mask(ctx->grad[slot], ctx->act_p[slot][Lp - 1], ctx->dpre_p[w][Lp - 1], ld8(ep), rows, ep,
-                             ctx->bf16, emb_dp(ctx) ? ctx->emb_c[slot] : nullptr, s));
+                             ctx->bf16, emb_dp(ctx) ? ctx->emb_c[slot] : nullptr, sub, s));
     const void* Xp0 = xp_rows(ctx, k, r0);
     for (int l = Lp - 1; l >= 0; --l) {
         const Layer& L = ctx->P[l];

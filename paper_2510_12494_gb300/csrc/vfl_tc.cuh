@@ -34,6 +34,7 @@ struct TcGemm {
     float* Pb; long long pb_stride;
     int nsplit, kchunk;
     int* err;                   // status word: ST_KERNEL_TIMEOUT when a bounded wait gave up
+    HeaderOps hdr;              // channel header checked at entry / published at the end (or none)
 };
 
 // The driver's tensor-map encoder is reachable (false on machines without a driver).

@@ -88,3 +88,21 @@ def test_uniform_order_and_graph_updates(vfl, cid):
         np.testing.assert_array_equal(W, ref.get_params()[key][0])
         np.testing.assert_array_equal(b, ref.get_params()[key][1])
     assert vfl.lib().vfl_set_order(ctx.h, 2) == vfl.VFL_E_INVAL
+
+
+@pytest.mark.parametrize("cid", [3, 4])
+def test_per_layer_path_headers_ride_in_the_kernels(vfl, cid):
+    """On the per-layer path the payload's last writer publishes the channel header and the first reader
+    checks it: no header kernels run unless a DP kernel writes the payload (wide-dp perturbs the gradient),
+    and the published headers are the steps' own."""
+    rows = {3: 2 * 4096 + 288, 4: 8192 + 576}[cid]
+    q, xp, xa, y, params = setup(synth.preset(cid), rows)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    tp, ta = schedule(q, 4)
+    ctx.profile(True)
+    ctx.train_steps(0, 4, tp, ta)
+    ctx.profile(False)
+    used = {k: v[0] for k, v in ctx.profile_summary().items()}
+    assert used.get("channel_header", 0) == (4 if cid == 4 else 0), used
+    ctx.check_channel(0, 3)
+    ctx.check_channel(1, 3)
