@@ -397,8 +397,10 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = Clocks(local)
     l0 = ctx.launches
+    x0 = ctx.exchange_bytes()
     ms, _ = timed_block(W, K)
     launches = ctx.launches - l0
+    x1 = ctx.exchange_bytes()
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = slowest_rank(ms)
@@ -478,6 +480,8 @@ def run_ours(args):
                        else "direct enqueue",
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU, 2 parties on separate streams"},
             "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roof, "cpu_baseline": cpu,
+            # Sec. 5's communication cost: payload bytes through the two channels per timed step
+            "exchange_bytes_per_step": {"embedding": (x1[0] - x0[0]) / K, "gradient": (x1[1] - x0[1]) / K},
         }
         print(json.dumps(line))
     ctx.close()

@@ -435,6 +435,11 @@ vfl_status vfl_check_channel(vfl_ctx* ctx, int32_t which, int64_t k);
 /* Number of kernels this context has launched so far (for launch accounting). */
 int64_t vfl_kernel_launches(const vfl_ctx* ctx);
 
+/* Communication cost (Sec. 5's metric): payload bytes published so far through the embedding and
+ * gradient channels (B_k x e_p elements of the compute dtype per publish; a dropped step publishes
+ * its embedding, if its publisher ran, and no gradient).  Host counters, no synchronisation. */
+vfl_status vfl_exchange_bytes(const vfl_ctx* ctx, int64_t* emb, int64_t* grad);
+
 /*
  * Per-launch timing.  vfl_profile(ctx, 1) starts recording a CUDA event pair
  * around every kernel launch, on the launch's stream; vfl_profile(ctx, 0)

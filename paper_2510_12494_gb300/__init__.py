@@ -125,6 +125,8 @@ EXPORTS = {
     "vfl_wait_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64]),
     "vfl_check_channel": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64]),
     "vfl_kernel_launches": (ctypes.c_int64, [ctypes.c_void_p]),
+    "vfl_exchange_bytes": (ctypes.c_int32, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64),
+                                            ctypes.POINTER(ctypes.c_int64)]),
     "vfl_profile": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32]),
     "vfl_profile_get": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64),
                                          ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
@@ -572,6 +574,12 @@ class Context:
     @property
     def launches(self) -> int:
         return lib().vfl_kernel_launches(self.h)
+
+    def exchange_bytes(self):
+        """(embedding, gradient) payload bytes published so far (vfl_exchange_bytes)."""
+        e, g = ctypes.c_int64(), ctypes.c_int64()
+        _check(lib().vfl_exchange_bytes(self.h, ctypes.byref(e), ctypes.byref(g)), self.h)
+        return e.value, g.value
 
     def profile(self, enable: bool):
         self._call(lib().vfl_profile, 1 if enable else 0)

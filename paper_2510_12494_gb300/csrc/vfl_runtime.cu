@@ -183,6 +183,7 @@ struct vfl_ctx {
     // host-side ordering state
     long long n_fwd = 0, n_act = 0, n_bwd = 0;
     long long n_drops = 0;                      // dropped steps among those published
+    long long x_emb = 0, x_grad = 0;            // payload bytes published through the two channels
     long long step_id[kInfoRing];               // per step k (slot k mod kInfoRing): its index,
     long long step_batch[kInfoRing];            // batch id,
     long long step_trained[kInfoRing];          // batches trained before it,
@@ -242,7 +243,7 @@ struct vfl_ctx {
 
 // Host-side ordering state of a context (saved around graph capture).
 struct HostState {
-    long long n_fwd, n_act, n_bwd, n_drops;
+    long long n_fwd, n_act, n_bwd, n_drops, x_emb, x_grad;
     long long step_id[kInfoRing], step_batch[kInfoRing], step_trained[kInfoRing];
     unsigned char step_drop[kInfoRing];
     int fwd_version[kMaxSlots];
@@ -257,6 +258,8 @@ static HostState save_state(const vfl_ctx* c) {
     h.n_act = c->n_act;
     h.n_bwd = c->n_bwd;
     h.n_drops = c->n_drops;
+    h.x_emb = c->x_emb;
+    h.x_grad = c->x_grad;
     std::memcpy(h.step_id, c->step_id, sizeof h.step_id);
     std::memcpy(h.step_batch, c->step_batch, sizeof h.step_batch);
     std::memcpy(h.step_trained, c->step_trained, sizeof h.step_trained);
@@ -275,6 +278,8 @@ static void load_state(vfl_ctx* c, const HostState& h) {
     c->n_act = h.n_act;
     c->n_bwd = h.n_bwd;
     c->n_drops = h.n_drops;
+    c->x_emb = h.x_emb;
+    c->x_grad = h.x_grad;
     std::memcpy(c->step_id, h.step_id, sizeof h.step_id);
     std::memcpy(c->step_batch, h.step_batch, sizeof h.step_batch);
     std::memcpy(c->step_trained, h.step_trained, sizeof h.step_trained);
@@ -1287,6 +1292,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
         if (!pdl) CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
         ctx->fwd_version[slot] = (int)v;
         ctx->slot_step_p[slot] = k;
+        ctx->x_emb += (long long)rows * ctx->P.back().out * ctx->esz;
         ctx->n_fwd = k + 1;
         ctx->started = true;
         return VFL_OK;
@@ -1316,6 +1322,7 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
     CK(cudaEventRecord(ctx->ev_emb[k % kEvPool], s));
     ctx->fwd_version[slot] = (int)v;
     ctx->slot_step_p[slot] = k;
+    ctx->x_emb += (long long)rows * ctx->P.back().out * ctx->esz;
     ctx->n_fwd = k + 1;
     ctx->started = true;
     return VFL_OK;
@@ -1357,6 +1364,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
         if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
         ctx->grad_step[slot] = k;
+        ctx->x_grad += (long long)rows * ep * ctx->esz;
         ctx->last_act_step[w] = k;
         ctx->n_act = k + 1;
         return VFL_OK;
@@ -1458,6 +1466,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     // publish the gradient
     CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
     ctx->grad_step[slot] = k;
+    ctx->x_grad += (long long)rows * ep * ctx->esz;
     // active bottom backward
     for (int l = La - 1; l >= 0; --l) {
         const Layer& L = ctx->A[l];
@@ -2559,6 +2568,13 @@ vfl_status vfl_check_channel(vfl_ctx* ctx, int32_t which, int64_t k) {
 }
 
 int64_t vfl_kernel_launches(const vfl_ctx* ctx) { return ctx ? ctx->launches : 0; }
+
+vfl_status vfl_exchange_bytes(const vfl_ctx* ctx, int64_t* emb, int64_t* grad) {
+    if (!ctx || !emb || !grad) return VFL_E_INVAL;
+    *emb = ctx->x_emb;
+    *grad = ctx->x_grad;
+    return VFL_OK;
+}
 
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable) {
     if (!ctx) return VFL_E_INVAL;

@@ -106,3 +106,16 @@ def test_per_layer_path_headers_ride_in_the_kernels(vfl, cid):
     assert used.get("channel_header", 0) == (4 if cid == 4 else 0), used
     ctx.check_channel(0, 3)
     ctx.check_channel(1, 3)
+
+
+def test_exchange_bytes_count_the_published_payloads(vfl):
+    q, xp, xa, y, params = setup(synth.preset(2), 3 * 1024 + 304)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    n = 2 * q.steps_per_epoch
+    tp, ta = schedule(q, n)
+    drops = np.zeros(n, np.uint8)
+    drops[3] = 1
+    ctx.train_steps(0, n, tp, ta, drops)
+    rows = sum(ctx.batch_rows(k)[1] - ctx.batch_rows(k)[0] for k in range(n))
+    rows_kept = sum(ctx.batch_rows(k)[1] - ctx.batch_rows(k)[0] for k in range(n) if not drops[k])
+    assert ctx.exchange_bytes() == (rows * q.e_passive * 4, rows_kept * q.e_passive * 4)
