@@ -1369,6 +1369,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         ctx->n_act = k + 1;
         return VFL_OK;
     }
+    ctx->cs_pending.n = 0;   // nothing left over from a phase that failed part-way
     // active bottom forward: z^a = f_a(x^a)
     const void* X = Xa0;
     long long ldx = ctx->ldxa;
@@ -1507,6 +1508,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int Lp = (int)ctx->P.size();
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
+    ctx->cs_pending.n = 0;
     if (ctx->fused) {
         const float* Xp = static_cast<const float*>(xp_rows(ctx, k, r0));
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
