@@ -119,3 +119,25 @@ def test_exchange_bytes_count_the_published_payloads(vfl):
     rows = sum(ctx.batch_rows(k)[1] - ctx.batch_rows(k)[0] for k in range(n))
     rows_kept = sum(ctx.batch_rows(k)[1] - ctx.batch_rows(k)[0] for k in range(n) if not drops[k])
     assert ctx.exchange_bytes() == (rows * q.e_passive * 4, rows_kept * q.e_passive * 4)
+
+
+def test_graph_update_refuses_another_shape_and_keeps_the_graph(vfl):
+    """A window whose graph has another shape (here: a dropped step) is refused by vfl_graph_update, and the
+    graph still replays the window it holds."""
+    q, xp, xa, y, params = setup(synth.preset(2), 4 * 1024 + 304)
+    nb = q.steps_per_epoch
+    n = 2 * nb
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.set_order(True)
+    ref.train_steps(0, n, tp, ta)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    ctx.set_order(True)
+    g = ctx.capture(0, nb, tp, ta)
+    drops = np.zeros(n, np.uint8)
+    drops[1] = 1
+    assert not ctx.update_graph(g, 0, nb, tp, ta, drops)
+    ctx.launch_graph(g)
+    ctx.train_steps(nb, nb, tp, ta)
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
