@@ -2411,17 +2411,13 @@ vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* g, int64_t k0, int64_t n_st
     cudaGraphExecUpdateResultInfo info;
     cudaError_t e = cudaGraphExecUpdate(g->exec, graph, &info);
     cudaGraphDestroy(graph);
-    if (e != cudaSuccess) {
+    if (e == cudaErrorGraphExecUpdateFailure) {
+        // not performed (another shape of graph): the executable graph still holds its old window
         cudaGetLastError();
-        // a different shape of graph: the executable graph is unchanged and still valid for its old window
-        if (info.result == cudaGraphExecUpdateErrorTopologyChanged || info.result == cudaGraphExecUpdateErrorNodeTypeChanged ||
-            info.result == cudaGraphExecUpdateErrorFunctionChanged || info.result == cudaGraphExecUpdateErrorParametersChanged ||
-            info.result == cudaGraphExecUpdateErrorNotSupported || info.result == cudaGraphExecUpdateErrorAttributesChanged ||
-            info.result == cudaGraphExecUpdateErrorUnsupportedFunctionChange)
-            return ctx->fail(VFL_E_STATE, "steps [%lld, %lld) do not fit the graph's shape (update result %d)",
-                             (long long)k0, (long long)(k0 + n_steps), (int)info.result);
-        return ctx->cuda(e, "cudaGraphExecUpdate", __LINE__);
+        return ctx->fail(VFL_E_STATE, "steps [%lld, %lld) do not fit the graph's shape (update result %d)",
+                         (long long)k0, (long long)(k0 + n_steps), (int)info.result);
     }
+    if (e != cudaSuccess) return ctx->cuda(e, "cudaGraphExecUpdate", __LINE__);
     g->k0 = k0;
     g->n = n_steps;
     g->drops0 = ctx->n_drops;
