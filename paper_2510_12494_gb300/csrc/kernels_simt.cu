@@ -1,6 +1,7 @@
 // SIMT kernels of the split-VFL step: the fp32 GEMM used for fp32 contexts and
-// for narrow layers, the fused loss, DP clip+noise, ReLU mask, fused SGD,
-// channel headers and data casts.
+// for narrow layers, the fused loss, DP clip+noise, ReLU mask, fused SGD, batched
+// bias column sums, the parameter-server average, channel headers (behind a DP
+// kernel; otherwise the GEMMs carry them) and data casts.
 #include "vfl_kernels.cuh"
 #include "vfl_philox.cuh"
 #include "vfl_pdl.cuh"

@@ -15,7 +15,9 @@
 //   DX   C[rows, in]  = D[rows, out] . W[out, in]      A K-major,  B MN-major
 //   DW   P[out, in]   = D[rows, out]^T . X[rows, in]   A MN-major, B MN-major
 // Every wait is bounded: on timeout the CTA records an error bit, drains what
-// it issued (again bounded), frees its TMEM and returns.
+// it issued (again bounded), frees its TMEM and returns.  The kernel starts with
+// pdl_entry() (a captured graph may launch it programmatically) and thread 0 of
+// CTA 0 checks / publishes a channel header when the step asks it to.
 #include <cuda.h>
 
 #include <algorithm>

@@ -6,8 +6,9 @@
 //  - Algorithm 1: vfl_passive_forward = publisher phase, vfl_active_step =
 //    subscriber phase, vfl_passive_backward = backward phase.
 //  - Sec. 4.1 channels keyed by batch id with bounded buffers: here HBM rings of
-//    S+1 slots with a header {k, batch, version}; a CUDA event per publish
-//    orders the subscriber's stream after the publisher's.
+//    S+1 slots with a header {k, batch, version}, written by the kernel that
+//    writes the payload last and checked by the first kernel that reads it; a
+//    CUDA event per publish orders the subscriber's stream after the publisher's.
 //  - App. D (Assumption 4, theorem): the gradient applied at step k was
 //    computed with weights of version k - tau(k); updates apply in step order.
 //    Each party keeps its S+1 most recent weight versions in a ring.
