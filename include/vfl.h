@@ -394,7 +394,9 @@ vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out);
 
 /*
  * One epoch: steps [epoch * nb, (epoch + 1) * nb) (nb = ceil(n_rows / batch)) through
- * vfl_train_steps (same arrays, indexed by absolute step; `drop` may be NULL), then, when
+ * vfl_train_steps (same arrays, indexed by absolute step; `drop` may be NULL) -- in the uniform order
+ * (vfl_set_order) without drops, as a CUDA graph the context keeps per epoch shape and updates in
+ * place for every later epoch (vfl_graph_update) -- then, when
  * mean_loss_out is not NULL, a synchronize and the epoch's mean loss per sample: each trained
  * step's mean loss weighted by its rows (dropped steps count none).  The steps before the epoch
  * must all be enqueued.

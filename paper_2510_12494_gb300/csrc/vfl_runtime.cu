@@ -211,6 +211,8 @@ struct vfl_ctx {
     // bias column sums of the per-layer path, gathered over a party's backward and launched as one batch
     // before its SGD (the d(pre) buffers stay until then)
     ColsumBatch cs_pending{};
+    // vfl_train_epoch in the uniform order: one epoch graph per first worker, updated in place every epoch
+    vfl_graph* epoch_graph[kMaxWorkers] = {};
     std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
 
     vfl_status fail(vfl_status st, const char* fmt, ...) {
@@ -1744,6 +1746,10 @@ vfl_status vfl_destroy(vfl_ctx* ctx) {
         const int n = ctx_streams(ctx, ss);
         for (int i = 0; i < n; ++i) cudaStreamSynchronize(ss[i]);
     }
+    for (vfl_graph*& g : ctx->epoch_graph) {
+        vfl_graph_destroy(g);
+        g = nullptr;
+    }
     for (ProfRec& r : ctx->prof) {
         ctx->ev_spare.push_back(r.e0);
         ctx->ev_spare.push_back(r.e1);
@@ -2206,7 +2212,21 @@ vfl_status vfl_train_epoch(vfl_ctx* ctx, int64_t epoch, const int32_t* tau_p, co
     if (ctx->broken) return VFL_E_CUDA;
     if (epoch < 0) return ctx->fail(VFL_E_INVAL, "epoch %lld < 0", (long long)epoch);
     const long long k0 = epoch * ctx->nb;
-    TRY(vfl_train_steps(ctx, k0, ctx->nb, tau_p, tau_a, drop));
+    bool own_streams = true;
+    for (int w = 0; w < ctx->W; ++w) own_streams = own_streams && ctx->ps[w] && ctx->as[w];
+    if (ctx->uniform && !drop && own_streams && !ctx->prof_on) {
+        // the epoch replays as a graph: the cached one of its shape updated in place, else a new capture
+        vfl_graph*& g = ctx->epoch_graph[k0 % ctx->W];
+        if (!g || g->n != ctx->nb || vfl_graph_update(ctx, g, k0, ctx->nb, tau_p, tau_a, nullptr) != VFL_OK) {
+            if (ctx->broken) return VFL_E_CUDA;
+            if (g) vfl_graph_destroy(g);
+            g = nullptr;
+            TRY(vfl_graph_capture(ctx, k0, ctx->nb, tau_p, tau_a, nullptr, &g));
+        }
+        TRY(vfl_graph_launch(ctx, g));
+    } else {
+        TRY(vfl_train_steps(ctx, k0, ctx->nb, tau_p, tau_a, drop));
+    }
     if (!mean_loss_out) return VFL_OK;
     std::vector<float> loss((size_t)ctx->nb);
     TRY(vfl_read_losses(ctx, k0, ctx->nb, loss.data()));

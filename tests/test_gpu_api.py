@@ -141,3 +141,28 @@ def test_graph_update_refuses_another_shape_and_keeps_the_graph(vfl):
     ctx.train_steps(nb, nb, tp, ta)
     ctx.synchronize()
     np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+
+
+@pytest.mark.parametrize("cid", [2, 3])
+def test_train_epoch_as_updated_graphs(vfl, cid):
+    """In the uniform order vfl_train_epoch replays each epoch as a graph it keeps and updates in place;
+    the epochs equal direct enqueue in the overlapping order bit for bit."""
+    rows = {2: 4 * 1024 + 304, 3: 2 * 4096 + 288}[cid]
+    q, xp, xa, y, params = setup(synth.preset(cid), rows)
+    nb = q.steps_per_epoch
+    n = 5 * nb
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx = new_context(vfl, q, xp, xa, y, params)
+    ctx.set_order(True)
+    launches = []
+    for e in range(5):
+        l0 = ctx.launches
+        ctx.train_epoch(e, tp, ta, mean_loss=(e == 4))
+        launches.append(ctx.launches - l0)
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+    for key, (W, b) in ctx.get_params().items():
+        np.testing.assert_array_equal(W, ref.get_params()[key][0])
+    assert len(set(launches)) == 1, launches      # every epoch's graph runs the same kernels
