@@ -2287,7 +2287,10 @@ void programmatic_edges(vfl_ctx* ctx, cudaGraph_t g, long long k0, long long n, 
         if (from && to) make_programmatic(g, from, to);
     }
     // every other kernel starts by waiting for its producer (pdl_entry), so any remaining plain edge
-    // between two kernel nodes whose target is not a fused kernel can be programmatic as well
+    // between two kernel nodes whose target is not a fused kernel can be programmatic as well (the fused
+    // path's few other kernels -- staging, averaging -- are off its critical chain: the per-edge queries
+    // are skipped there, they cost the host more than they save)
+    if (ctx->fused) return;
     size_t ne = 0;
     if (cudaGraphGetEdges(g, nullptr, nullptr, nullptr, &ne) != cudaSuccess || ne == 0) {
         cudaGetLastError();
