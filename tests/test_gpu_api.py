@@ -166,3 +166,16 @@ def test_train_epoch_as_updated_graphs(vfl, cid):
     for key, (W, b) in ctx.get_params().items():
         np.testing.assert_array_equal(W, ref.get_params()[key][0])
     assert len(set(launches)) == 1, launches      # every epoch's graph runs the same kernels
+
+
+def test_planner_calibration_tool(vfl):
+    """The calibration tool fits Eq. 7-8's constants from a synchronous run on this GPU and Algorithm 2
+    picks a candidate of the search space."""
+    from paper_2510_12494_gb300 import plan as planner
+    p = synth.preset(1)
+    model, meas = planner.calibrate(vfl, p, [128, 256, 512], steps=6, warmup=2)
+    assert sorted(meas) == [128, 256, 512]
+    assert all(v > 0 for b in meas for v in meas[b].values())
+    assert model["lambda_a"] > 0 and model["lambda_p"] > 0 and model["phi_p"] > 0
+    wa, wp, b, o = vfl.plan(vfl.plan_model(**model), (1, 2), (1, 2), [128, 256, 512])
+    assert (wa, wp) == (1, 1) and b in (128, 256, 512) and o > 0
