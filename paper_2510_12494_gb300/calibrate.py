@@ -24,7 +24,7 @@ whole pipelined step (CUDA graphs, every worker count and batch size of the
 search space, w_a = w_p since the library runs one worker count per party)
 and reports the measured throughput next to the model's prediction.
 
-Run: python -m paper_2510_12494_gb300.plan [--config N] [--batches ...] [--workers ...]
+Run: python -m paper_2510_12494_gb300.calibrate [--config N] [--batches ...] [--workers ...]
 """
 from __future__ import annotations
 

@@ -171,7 +171,7 @@ def test_train_epoch_as_updated_graphs(vfl, cid):
 def test_planner_calibration_tool(vfl):
     """The calibration tool fits Eq. 7-8's constants from a synchronous run on this GPU and Algorithm 2
     picks a candidate of the search space."""
-    from paper_2510_12494_gb300 import plan as planner
+    from paper_2510_12494_gb300 import calibrate as planner
     p = synth.preset(1)
     model, meas = planner.calibrate(vfl, p, [128, 256, 512], steps=6, warmup=2)
     assert sorted(meas) == [128, 256, 512]
