@@ -128,3 +128,13 @@ def test_bf16_head_limit(vfl, n_out, head):
     used = kernels_used(vfl, q)
     assert ("head_loss" in used) == head and ("loss" in used) != head, used
     assert_parity(vfl, q, steps=4)
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_unit_dimensions(vfl, dtype):
+    """Every GEMM dimension at 1 somewhere: one feature per party, width-1 layers and cut layers, one logit
+    (M = 1 is the single-row batch case above)."""
+    base = synth.preset(1) if dtype == "fp32" else SMALL_BF16.with_(loss="bce")
+    q = base.with_(cid=0, name=f"unit-{dtype}", d_passive=1, d_active=1, passive=(1,), active=(3, 1), top=(1, 1),
+                   loss="bce", n_rows=300, batch=128)
+    assert_parity(vfl, q, steps=5)
