@@ -214,3 +214,10 @@ def test_drops_with_dp(vfl, target):
     drops = np.zeros(10, np.uint8)
     drops[[2, 7]] = 1
     assert_parity(vfl, q, 10, drops)
+
+
+def test_drops_at_the_largest_staleness_bound(vfl):
+    """S = 15 (16 version slots) with three worker streams and a drop in four."""
+    q = synth.preset(1).with_(n_rows=5 * 256 + 37, staleness=15, schedule="seeded", workers=3)
+    drops = oracle.make_drops(5, 0.25, 30)
+    assert_parity(vfl, q, 30, drops)

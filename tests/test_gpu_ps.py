@@ -193,3 +193,9 @@ def test_ps_host_data_equals_resident(vfl):
         for key, (W, b) in ctx.get_replica(w).items():
             np.testing.assert_array_equal(W, ref.get_replica(w)[key][0])
             np.testing.assert_array_equal(b, ref.get_replica(w)[key][1])
+
+
+def test_ps_at_the_worker_limit(vfl):
+    """16 workers (one version slot and one replica each, the library's limit), averaged every epoch."""
+    q = ps_preset(1, 16, 1, 20 * 64 + 9, batch=64)
+    assert_parity(vfl, q, steps=2 * 21 + 3)
