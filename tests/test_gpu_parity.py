@@ -105,19 +105,17 @@ def test_fp32_epoch_loss_and_dag_equals_sequential(vfl, cid):
 
 
 def test_full_size_in_the_bench_configuration(vfl):
-    """The credit-shaped workload at full size as bench.py times it: one CUDA
-    graph per epoch (captured, then replayed), two worker streams per party,
-    five epochs; epoch losses within 1e-3 of the oracle and the final weights
-    within 1e-3."""
+    """The credit-shaped workload at full size as bench.py times it: the whole
+    training run (five epochs) as one CUDA graph, captured then replayed, two
+    worker streams per party; epoch losses within 1e-3 of the oracle and the
+    final weights within 1e-3."""
     import synth
     q, xp, xa, y, params = setup(synth.preset(2))
     nb = q.steps_per_epoch
     n_steps = nb * q.epochs
     tp, ta = schedule(q, n_steps)
     ctx = new_context(vfl, q, xp, xa, y, params)
-    for e in range(q.epochs):
-        g = ctx.capture(e * nb, nb, tp, ta)
-        ctx.launch_graph(g)
+    ctx.launch_graph(ctx.capture(0, n_steps, tp, ta))
     ctx.synchronize()
     losses = ctx.read_losses(0, n_steps)
     o = oracle.Oracle(q, xp, xa, y, params)
