@@ -100,7 +100,7 @@ typedef struct vfl_config {
  */
 
 /*
- * Intra-party semi-asynchronous parameter server (Sec. 4.2, Eq. 5), enabled by
+ * Intra-party semi-asynchronous parameter server (Sec. 4.1, Eq. 5), enabled by
  * ps_dt0 > 0 (requires staleness == 0).  Each party keeps one replica of its
  * parameters (fp32 master and compute copy) per worker; step k runs on worker
  * w = k mod workers, reads replica w as it stands and applies its SGD update to
@@ -126,7 +126,7 @@ vfl_status vfl_ps_interval(int64_t t, int32_t dt0, int64_t* interval);
 vfl_status vfl_gdp_sigma(double mu, int64_t batch, int64_t n_rows, int64_t queries, double* sigma);
 
 /*
- * System planning (Sec. 4.3-4.4, Eq. 7-17, Algorithm 2).  Host only, pure.
+ * System planning (Sec. 4.2-4.3, Eq. 7-17, Algorithm 2).  Host only, pure.
  * Delay model of one iteration, each term coef * B^exp * w / C (Eq. 7-9):
  *   T_A = (lambda_a B^gamma_a + phi_a B^beta_a + lambda_top B^gamma_top + phi_top B^beta_top) w_a / C_a
  *   T_P = (lambda_p B^gamma_p + phi_p B^beta_p) w_p / C_p
@@ -168,20 +168,30 @@ vfl_status vfl_fit_power(const double* x, const double* t, int32_t n, double* co
 
 typedef struct vfl_ctx vfl_ctx;
 
-/* Bytes of device workspace vfl_create() needs for `cfg` and a dataset of n_rows rows. */
+/* Bytes of device workspace vfl_create() needs for `cfg` and a dataset of n_rows rows: both parties'
+ * feature partitions and the labels (Sec. 3), the S+1 weight versions each party keeps (App. D,
+ * Assumption 4), the embedding and gradient channel buffers (Sec. 4.1) and the per-worker scratch. */
 vfl_status vfl_workspace_bytes(const vfl_config* cfg, int64_t n_rows, uint64_t* bytes);
 
 /*
- * Create a context on the current CUDA device.  `workspace` is a device pointer
+ * Create a context on the current CUDA device for the problem of Sec. 3: the passive party's d_p
+ * features and bottom model f_p, the active party's d_a features, labels, bottom model f_a and top
+ * model g, the loss (Eq. 1 for BCE), the step size of Eq. 2, the staleness bound of App. D
+ * (Assumption 4), the channels of Sec. 4.1 (S+1 slots each) and the workers per party (Fig. 2).
+ * VFL_E_INVAL for a configuration outside the limits above, VFL_E_OOM for a short workspace.  `workspace` is a device pointer
  * (256-byte aligned) of at least vfl_workspace_bytes() bytes; it stays owned by
  * the caller and must outlive the context.  Parameters start at zero: set them
  * with vfl_set_params() before training.
  */
 vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, uint64_t workspace_bytes,
                       vfl_ctx** out);
+/* Release the context (the paper has no counterpart).  Waits for its work; the workspace and the
+ * borrowed streams stay the caller's.  Valid in every state, including after VFL_E_CUDA. */
 vfl_status vfl_destroy(vfl_ctx* ctx);
 
 /*
+ * The workers of each party (Sec. 4.1, Fig. 2: each party runs several workers that publish and
+ * subscribe concurrently) are CUDA streams here.
  * Borrow 2*workers CUDA streams (cudaStream_t passed as void*): entries
  * [0, workers) run the passive party's work, [workers, 2*workers) the active
  * party's.  Steps go to worker k mod workers.  The streams must outlive the context.
@@ -189,6 +199,8 @@ vfl_status vfl_destroy(vfl_ctx* ctx);
 vfl_status vfl_set_streams(vfl_ctx* ctx, int32_t n, void* const* streams);
 
 /*
+ * The vertically partitioned dataset of Sec. 3: the passive party holds x^p, the active party x^a
+ * and the labels y, row i of each belonging to the same sample (rows aligned by construction).
  * Copy the whole dataset from host memory: x_passive [n_rows, d_p] and
  * x_active [n_rows, d_a] fp32, y [n_rows] int32 (BCE: 0/1, CE: class id in
  * [0, n_out)).  Synchronous.  bf16 contexts round the features to bf16 here.
@@ -196,7 +208,8 @@ vfl_status vfl_set_streams(vfl_ctx* ctx, int32_t n, void* const* streams);
 vfl_status vfl_load_data(vfl_ctx* ctx, const float* x_passive, const float* x_active, const int32_t* y);
 
 /*
- * Host-resident data.  After this call every step k reads its own rows
+ * Host-resident data (the same partitioned dataset of Sec. 3, left in host memory; the paper has no
+ * counterpart for the staging).  After this call every step k reads its own rows
  * [r0, r1) of x_passive [n_rows, d_p] fp32, x_active [n_rows, d_a] fp32 and
  * y [n_rows] int32 straight from host memory into a device staging ring of
  * S + workers + 2 slots (part of the workspace), with one kernel on io_stream,
@@ -218,6 +231,7 @@ vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* x_passive, const float*
                               float* loss_out, int64_t loss_cap, void* io_stream);
 
 /*
+ * The parameters theta_2 (f_p) and theta_1 (f_a and g) of Sec. 3 that Eq. 2 updates.
  * Set / read the fp32 master parameters of one layer: W [out, in], b [out]
  * (host pointers).  vfl_set_params resets every stored weight version of the
  * layer to the new values and is only valid before the first step.
@@ -227,6 +241,8 @@ vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const floa
 vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, float* b);
 
 /*
+ * Algorithm 1 starts from random weights theta_1, theta_2 without naming a distribution; this
+ * library's reading is a uniform fan-in draw.
  * Seeded initial parameters for every layer, as vfl_set_params would take them: each entry of
  * layer l of party q (W row-major, then b) is (2u - 1) / sqrt(fan_in) in double, rounded to fp32,
  * u = word i * 2^-32 of the stream Philox4x32-10(key = (seed lo, seed hi), counter = (i / 4 lo,
@@ -236,6 +252,7 @@ vfl_status vfl_get_params(vfl_ctx* ctx, int32_t party, int32_t layer, float* W, 
 vfl_status vfl_init_params(vfl_ctx* ctx, uint64_t seed);
 
 /*
+ * The gradients grad_theta_1 L and grad_theta_2 L of Sec. 3's backward pass (Eq. 2 applies them).
  * Gradient dLoss/dW [out, in] and dLoss/db [out] of one layer from the most
  * recent step of that party on worker `worker` (before the SGD update used
  * it).  Synchronizes the context.
@@ -243,7 +260,9 @@ vfl_status vfl_init_params(vfl_ctx* ctx, uint64_t seed);
 vfl_status vfl_get_grads(vfl_ctx* ctx, int32_t party, int32_t layer, int32_t worker, float* dW, float* db);
 
 /*
- * Checkpoint / restore.  Valid only while no step is in flight (every enqueued
+ * Checkpoint / restore of the state the delayed update of App. D reads: the step counter and the
+ * stored weight versions theta^(k - tau), tau <= S (the paper has no checkpoint format).
+ * Valid only while no step is in flight (every enqueued
  * step has run all three phases).
  *  - vfl_step_cursor: number of finished steps k = the current weight version.
  *  - vfl_get_version: the stored compute copy of weight version v
@@ -333,6 +352,8 @@ vfl_status vfl_set_drops(vfl_ctx* ctx, int64_t n_drops);
 vfl_status vfl_make_drops(uint64_t seed, double rate, int64_t n_steps, uint8_t* drop);
 
 /*
+ * Algorithm 1's three phases (publisher, subscriber, backward) for a window of steps, each step's
+ * versions fixed by the staleness schedule (App. D).
  * Enqueue steps [k0, k0 + n_steps) as one dependency graph across the worker
  * streams: each publisher phase runs as soon as its weight version exists, so
  * the parties overlap as far as tau allows.  tau_p / tau_a are host arrays
@@ -344,7 +365,8 @@ vfl_status vfl_train_steps(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const int3
                            const int32_t* tau_a, const uint8_t* drop);
 
 /*
- * CUDA-graph replay of a window of steps.  vfl_graph_capture records steps
+ * CUDA-graph replay of a window of steps (the paper has no counterpart: the same phases of
+ * Algorithm 1 as vfl_train_steps, recorded once and replayed).  vfl_graph_capture records steps
  * [k0, k0 + n_steps) -- the same kernels and cross-stream events
  * vfl_train_steps would enqueue -- into an executable graph without running
  * them; every step before k0 must be enqueued (it may still be running, e.g. a
@@ -363,6 +385,7 @@ vfl_status vfl_graph_capture(vfl_ctx* ctx, int64_t k0, int64_t n_steps, const in
 vfl_status vfl_graph_launch(vfl_ctx* ctx, vfl_graph* graph);
 
 /*
+ * (No counterpart in the paper; an update of a vfl_graph_capture graph.)
  * Re-record `graph` for steps [k0, k0 + n_steps) (same preconditions as vfl_graph_capture) and update
  * its executable graph in place (cudaGraphExecUpdate): far cheaper than a new capture's
  * instantiation when the new window has the same shape.  Launches already in flight keep their old
@@ -374,7 +397,8 @@ vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* graph, int64_t k0, int64_t 
                             const int32_t* tau_a, const uint8_t* drop);
 
 /*
- * Dependency order of the enqueued steps.  VFL_ORDER_OVERLAP (default): a step waits only for the
+ * Dependency order of the enqueued steps (no counterpart in the paper: both orders compute what
+ * App. D's delayed update defines).  VFL_ORDER_OVERLAP (default): a step waits only for the
  * version it reads, so steps overlap as far as tau allows.  VFL_ORDER_UNIFORM: every step waits for
  * all updates before it and is published after the previous backward, as if tau were 0, while
  * still computing with versions k - tau -- the same results, less overlap, but one graph shape for
@@ -385,14 +409,17 @@ vfl_status vfl_graph_update(vfl_ctx* ctx, vfl_graph* graph, int64_t k0, int64_t 
 vfl_status vfl_set_order(vfl_ctx* ctx, int32_t order);
 vfl_status vfl_graph_destroy(vfl_graph* graph);
 
-/* Wait for all enqueued work; returns VFL_E_VERSION / VFL_E_TIMEOUT recorded by kernels. */
+/* Wait for all enqueued work (no counterpart in the paper); returns VFL_E_VERSION (a channel header
+ * of Sec. 4.1 named another step) or VFL_E_TIMEOUT recorded by kernels. */
 vfl_status vfl_synchronize(vfl_ctx* ctx);
 
-/* Mean loss of steps [k0, k0+n) (float per step) into host memory; synchronizes.
+/* The loss of Eq. 1 (BCE) or softmax cross-entropy, averaged over each step's rows: steps
+ * [k0, k0+n) (float per step, NaN for a dropped step) into host memory; synchronizes.
  * Only the last 4096 steps are kept. */
 vfl_status vfl_read_losses(vfl_ctx* ctx, int64_t k0, int64_t n, float* out);
 
 /*
+ * Algorithm 1's epoch loop (global epoch t: every batch B_j once, through the three phases).
  * One epoch: steps [epoch * nb, (epoch + 1) * nb) (nb = ceil(n_rows / batch)) through
  * vfl_train_steps (same arrays, indexed by absolute step; `drop` may be NULL) -- in the uniform order
  * (vfl_set_order) without drops, as a CUDA graph the context keeps per epoch shape and updates in
@@ -405,21 +432,26 @@ vfl_status vfl_train_epoch(vfl_ctx* ctx, int64_t epoch, const int32_t* tau_p, co
                            const uint8_t* drop, float* mean_loss_out);
 
 /*
+ * The loss of Eq. 1 for one step, read without a synchronisation.
  * Enqueue an asynchronous copy of the mean loss of step k (already enqueued)
  * into host memory `host_out` (pinned for asynchrony) on the stream of the
  * step's active worker; valid once that stream passes this point.
  */
 vfl_status vfl_fetch_loss(vfl_ctx* ctx, int64_t k, float* host_out);
 
-/* Copy a channel slot or a per-worker buffer of step k to host fp32 (see VFL_TAP_*): rows x cols
+/* Parity probe of Algorithm 1's exchanged tensors (z^p in C_e[B_j], grad_z^p L in C_g[B_j]) and of
+ * the active party's z^a, grad_z^a L and logits (Sec. 3).
+ * Copy a channel slot or a per-worker buffer of step k to host fp32 (see VFL_TAP_*): rows x cols
  * floats, rows as vfl_step_rows gives; VFL_E_INVAL when that exceeds out_elems.  Synchronizes. */
 vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out, int64_t out_elems);
 
-/* First row and row count of the batch step k trains (published steps in flight, or the next
+/* Batch B_j of step k (Algorithm 1's sampled batch; its id labels the channels, Sec. 4.1).
+ * First row and row count of the batch step k trains (published steps in flight, or the next
  * step): batch (k - drops before k) mod nb. */
 vfl_status vfl_step_rows(vfl_ctx* ctx, int64_t k, int64_t* r0, int32_t* rows);
 
 /*
+ * Sec. 4.1's waiting deadline T_ddl as a device-side probe.
  * Fault probe: a bounded device-side wait (at most max_iters polls) for the
  * embedding (which = 0) or gradient (which = 1) channel slot of step k to carry
  * header k.  Returns VFL_OK or VFL_E_TIMEOUT; never blocks indefinitely.
@@ -427,6 +459,7 @@ vfl_status vfl_step_rows(vfl_ctx* ctx, int64_t k, int64_t* r0, int32_t* rows);
 vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_iters);
 
 /*
+ * Sec. 4.1's batch-ID labelled channels: the subscriber's check of the slot's label.
  * Non-blocking subscriber check: does the embedding (which = 0) or gradient
  * (which = 1) channel slot of step k carry the header of step k?  VFL_OK or
  * VFL_E_VERSION (the same device-side check the subscriber phases run).
@@ -434,7 +467,7 @@ vfl_status vfl_wait_channel(vfl_ctx* ctx, int32_t which, int64_t k, int64_t max_
  */
 vfl_status vfl_check_channel(vfl_ctx* ctx, int32_t which, int64_t k);
 
-/* Number of kernels this context has launched so far (for launch accounting). */
+/* Number of kernels this context has launched so far (launch accounting; no counterpart in the paper). */
 int64_t vfl_kernel_launches(const vfl_ctx* ctx);
 
 /* Communication cost (Sec. 5's metric): payload bytes published so far through the embedding and
@@ -443,7 +476,8 @@ int64_t vfl_kernel_launches(const vfl_ctx* ctx);
 vfl_status vfl_exchange_bytes(const vfl_ctx* ctx, int64_t* emb, int64_t* grad);
 
 /*
- * Per-launch timing.  vfl_profile(ctx, 1) starts recording a CUDA event pair
+ * Per-launch timing: the measurements Sec. 4.2 (System Profiling) fits the delay model of
+ * Eq. 7-9 to.  vfl_profile(ctx, 1) starts recording a CUDA event pair
  * around every kernel launch, on the launch's stream; vfl_profile(ctx, 0)
  * synchronizes and folds the records into per-class totals.  vfl_profile_get
  * then returns, for kernel class `cls` (0 .. VFL_KERNEL_CLASSES-1, named by
@@ -480,17 +514,20 @@ const char* vfl_kernel_class_name(int32_t cls);
  *   stream  cudaStream_t to enqueue on (NULL: legacy default stream); the call
  *         returns before the work finishes.
  *
- * Limit: out*in + out <= 4,194,304; larger layers get VFL_E_INVAL with the
- * reason in vfl_last_error(NULL).  The first call on a device looks up the
- * array's device address (cudaGetSymbolAddress); make that first call before
- * any stream capture.  All calls share the array and it keeps the last call's
+ * Limits: out*in + out <= 4,194,304 and in <= 4,194,240 (65535 blocks of 64
+ * inputs); larger layers get VFL_E_INVAL with the reason in
+ * vfl_last_error(NULL).  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress) and the SM count; make that first
+ * call before any stream capture.  The address stays cached for the process,
+ * so a device reset (cudaDeviceReset) after the first call is not supported.  All calls share the array and it keeps the last call's
  * partial sums (each call overwrites everything it reads, so nothing needs
  * clearing); calls that can overlap on the GPU race on it, so serialize them.
  */
 vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, int32_t rows, int32_t out, int32_t in,
                                    int32_t dtype, float* dW, float* db, void* stream);
 
-/* Last error message of the context (or of the last failed vfl_create / vfl_make_schedule when ctx is NULL). */
+/* Last error message of the context (or of the last failed vfl_create / vfl_make_schedule when ctx is NULL);
+ * error reporting has no counterpart in the paper. */
 const char* vfl_last_error(const vfl_ctx* ctx);
 
 #ifdef __cplusplus

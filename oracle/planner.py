@@ -1,4 +1,4 @@
-"""System planning of PubSub-VFL (Sec. 4.3-4.4) -- TEST INFRASTRUCTURE ONLY.
+"""System planning of PubSub-VFL (Sec. 4.2-4.3) -- TEST INFRASTRUCTURE ONLY.
 
 The delay model of one iteration (Eq. 7-9): every term is coef * B^exp * w / C,
   T_A = (lambda_a B^gamma_a + phi_a B^beta_a + lambda_top B^gamma_top + phi_top B^beta_top) w_a / C_a,

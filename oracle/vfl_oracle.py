@@ -23,7 +23,7 @@ What it computes, in the paper's order (Algorithm 1, Sec. 3, App. C, App. D):
   and the update is theta_{t+1} = theta_t - eta * (g_{t - tau(t)} + xi_dp).
 * App. C / Assumption 5: Gaussian noise on the exchanged tensor.
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent:
 
 * Two lags per step: tau_p(k) is the age of the passive weights that produced
   the embedding of step k; tau_a(k) the age of the active + top weights that
@@ -47,7 +47,7 @@ Readings where the paper is silent (each is listed in the design doc):
   received gradient by c_i (the Jacobian of c_i and of the noise are ignored)
   before its own ReLU mask on the clean z.  sigma for a target mu-GDP level
   follows Eq. 25 with the O(.)'s constant taken as 1.
-* Intra-party semi-asynchronous parameter server (Sec. 4.2, Eq. 5, Algorithm
+* Intra-party semi-asynchronous parameter server (Sec. 4.1, Eq. 5, Algorithm
   1), when cfg.ps_dt0 > 0: each party keeps one replica of its parameters per
   worker (cfg.workers of them); step k is served by worker pair k mod W, whose
   replicas it reads (the latest: no staleness within a replica's chain) and

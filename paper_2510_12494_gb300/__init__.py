@@ -273,9 +273,26 @@ def weight_grad_noalloc(dpre, x, dW, db, dtype: int, stream=None):
     fixed scratch instead of any allocation.  Enqueued on ``stream`` (a
     torch.cuda.Stream; default: the current stream)."""
     import torch
+    if dtype not in (FP32, BF16):
+        raise ValueError(f"dtype must be FP32 or BF16, got {dtype}")
+    if dpre.dim() != 2 or x.dim() != 2 or dW.dim() != 2 or db.dim() != 1:
+        raise ValueError("dpre, x and dW must be matrices and db a vector")
     rows, out = dpre.shape
-    assert x.shape[0] == rows and dW.shape == (out, x.shape[1]) and db.shape == (out,)
+    if x.shape[0] != rows or tuple(dW.shape) != (out, x.shape[1]) or tuple(db.shape) != (out,):
+        raise ValueError(f"shapes disagree: dpre {tuple(dpre.shape)}, x {tuple(x.shape)}, dW {tuple(dW.shape)}, "
+                         f"db {tuple(db.shape)}")
+    # the kernel reads and writes raw row-major buffers of these element types: anything else would be
+    # read or written past its end
+    want = torch.float32 if dtype == FP32 else torch.bfloat16
+    for name, t, dt in (("dpre", dpre, want), ("x", x, want), ("dW", dW, torch.float32), ("db", db, torch.float32)):
+        if t.dtype != dt:
+            raise ValueError(f"{name} must be {dt}, got {t.dtype}")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous (row-major)")
     s = stream if stream is not None else torch.cuda.current_stream()
+    for name, t in (("dpre", dpre), ("x", x), ("dW", dW), ("db", db)):
+        if t.device.type != "cuda" or t.device.index != s.device.index:
+            raise ValueError(f"{name} must be on {s.device}, the stream's device (got {t.device})")
     _check(lib().vfl_weight_grad_noalloc(ctypes.c_void_p(dpre.data_ptr()), ctypes.c_void_p(x.data_ptr()), rows, out,
                                          x.shape[1], dtype, ctypes.c_void_p(dW.data_ptr()),
                                          ctypes.c_void_p(db.data_ptr()), ctypes.c_void_p(s.cuda_stream)))

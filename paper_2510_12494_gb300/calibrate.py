@@ -1,4 +1,4 @@
-"""Calibrate the system planner (Sec. 4.3-4.4) on this GPU and check its choice.
+"""Calibrate the system planner (Sec. 4.2-4.3) on this GPU and check its choice.
 
 The paper estimates the pipelined system's delays from a synchronous run:
 each phase of a step timed alone, at several batch sizes, fitted to the power

@@ -23,12 +23,18 @@ constexpr unsigned long long kNoAllocScratchBytes = 16ull << 20;   // 16 MiB
 constexpr long long kNoAllocScratchFloats = (long long)(kNoAllocScratchBytes / sizeof(float));
 static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
 
-// Device address of g_noalloc_scratch, looked up once per device.  In host
-// code the array's name is only a host-side stand-in, so kernels must be given
-// this address instead.
+// Device address of g_noalloc_scratch and the device's SM count, looked up
+// once per device.  In host code the array's name is only a host-side
+// stand-in, so kernels must be given this address instead.  The address is
+// cached for the life of the process: a device reset (cudaDeviceReset) after
+// the first call is not supported.
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 float* g_scratch_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+
+// The SIMT GEMM tiles the layer's inputs in blocks of 64 along grid.y.
+constexpr long long kMaxIn = 65535LL * 64;
 
 // dW[i] = sum_z P[z * stride + i] (i < n_w); db[j] = sum_z Pb[z * n_b + j], in z order.
 __global__ void reduce_partials_kernel(const float* __restrict__ P, long long stride, long long n_w,
@@ -69,15 +75,13 @@ extern "C" vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, i
                              .c_str());
         return VFL_E_INVAL;
     }
-    const long long tiles = (long long)((out + 63) / 64) * ((in + 63) / 64);
-    long long nsplit = std::max<long long>(1, 2 * 152 / std::max<long long>(1, tiles));
-    nsplit = std::min<long long>(nsplit, std::max(1, rows / 64));
-    nsplit = std::min<long long>(nsplit, 32);
-    nsplit = std::min<long long>(nsplit, kNoAllocScratchFloats / per_split);
-    const int kchunk = (int)(((rows + nsplit - 1) / nsplit + 15) / 16 * 16);
-    nsplit = (rows + kchunk - 1) / kchunk;
+    if (in > kMaxIn) {
+        set_global_error(("vfl_weight_grad_noalloc: in = " + std::to_string(in) + " exceeds the largest supported "
+                          "input width " + std::to_string(kMaxIn)).c_str());
+        return VFL_E_INVAL;
+    }
 
-    // One-time set-up on the current device: the scratch array's device address.
+    // One-time set-up on the current device: the scratch array's device address and the SM count.
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
@@ -85,6 +89,7 @@ extern "C" vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, i
         return VFL_E_CUDA;
     }
     float* scratch = nullptr;
+    int sm_count = 0;
     {
         std::lock_guard<std::mutex> lock(g_mu);
         if (!g_scratch_ptr[dev]) {
@@ -95,10 +100,27 @@ extern "C" vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, i
                                   cudaGetErrorString(e)).c_str());
                 return VFL_E_CUDA;
             }
+            int sms = 0;
+            e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (e != cudaSuccess || sms < 1) {
+                set_global_error((std::string("vfl_weight_grad_noalloc: SM count query failed: ") +
+                                  cudaGetErrorString(e)).c_str());
+                return VFL_E_CUDA;
+            }
+            g_sm_count[dev] = sms;
             g_scratch_ptr[dev] = static_cast<float*>(p);
         }
         scratch = g_scratch_ptr[dev];
+        sm_count = g_sm_count[dev];
     }
+    // Split the rows so that about two blocks per SM run, within the scratch.
+    const long long tiles = (long long)((out + 63) / 64) * ((in + 63) / 64);
+    long long nsplit = std::max<long long>(1, 2LL * sm_count / std::max<long long>(1, tiles));
+    nsplit = std::min<long long>(nsplit, std::max(1, rows / 64));
+    nsplit = std::min<long long>(nsplit, 32);
+    nsplit = std::min<long long>(nsplit, kNoAllocScratchFloats / per_split);
+    const int kchunk = (int)(((rows + nsplit - 1) / nsplit + 15) / 16 * 16);
+    nsplit = (rows + kchunk - 1) / kchunk;
     float* P = scratch;
     float* Pb = scratch + nsplit * (long long)out * in;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -122,7 +144,7 @@ extern "C" vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, i
     e = launch_gemm_simt(g, bf, bf, bf, (int)nsplit, s);
     if (e == cudaSuccess) {
         const long long n = (long long)out * in + out;
-        long long blocks = std::min<long long>((n + 255) / 256, 152 * 8);
+        long long blocks = std::min<long long>((n + 255) / 256, (long long)sm_count * 8);
         reduce_partials_kernel<<<(int)blocks, 256, 0, s>>>(P, (long long)out * in, (long long)out * in, Pb, out,
                                                             (int)nsplit, dW, db);
         e = cudaGetLastError();

@@ -1,4 +1,4 @@
-// System planning of PubSub-VFL (Sec. 4.3-4.4): the delay model of Eq. 7-12, the memory bound of
+// System planning of PubSub-VFL (Sec. 4.2-4.3): the delay model of Eq. 7-12, the memory bound of
 // Eq. 14-15, the objective of Eq. 17 and the exhaustive search of Algorithm 2, plus the power-law
 // fit that turns measured delays into the model's constants.  Host code only.
 #include <algorithm>

@@ -121,7 +121,7 @@ struct SgdArgs {
 };
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s);
 
-// Parameter-server aggregation (Sec. 4.2): every replica of a party's layers takes the mean of the
+// Parameter-server aggregation (Sec. 4.1, Eq. 5): every replica of a party's layers takes the mean of the
 // replicas, summed in fp32 in replica order and divided by nrep (IEEE division); the fp32 masters
 // and the compute copies [out, in_ld] (padding columns untouched) are all rewritten.  The layer
 // table lives in device memory; layer l covers flat indices [begin, begin + out * in + out).

@@ -14,7 +14,7 @@
 //    Each party keeps its S+1 most recent weight versions in a ring.
 //  - Sec. 4.1 waiting deadline / buffer overflow: a dropped step trains nothing
 //    (both parties copy version k to k+1) and hands its batch to the next step.
-//  - Sec. 4.2 / Eq. 5 (ps_dt0 > 0): one replica of each party's parameters per
+//  - Sec. 4.1 / Eq. 5 (ps_dt0 > 0): one replica of each party's parameters per
 //    worker, each worker's steps chained on its own stream pair, the replicas
 //    averaged after the epochs Eq. 5 selects.
 #include <algorithm>
@@ -144,7 +144,7 @@ struct vfl_ctx {
     float* f_rowloss[kMaxWorkers] = {};         // per worker: per-row loss [B]
     float* f_zpc[kMaxWorkers] = {};             // per worker: z^p rows consumed by the step [B, ld8(e_p)]
 
-    // parameter-server mode (Sec. 4.2): replicas per worker, averaged per Eq. 5
+    // parameter-server mode (Sec. 4.1, Eq. 5): replicas per worker, averaged per Eq. 5
     bool psmode = false;
     PsAvgLayer* ps_tab = nullptr;               // device table: P's layers, then A's, then T's
     long long ps_total[2] = {};                 // flat parameter counts: passive, active (f_a and g)
@@ -641,7 +641,7 @@ inline cudaStream_t pstream(vfl_ctx* ctx, long long k) { return ctx->ps[k % ctx-
 // DP on the published embedding (App. C) rather than on its gradient
 inline bool emb_dp(const vfl_ctx* ctx) { return ctx->cfg.dp_clip > 0.f && ctx->cfg.dp_target == VFL_DP_EMB; }
 
-// ---- parameter-server mode (Sec. 4.2) ------------------------------------------------
+// ---- parameter-server mode (Sec. 4.1, Eq. 5) ------------------------------------------------
 // Synchronization interval after epoch t (1-based), Eq. 5:
 // Delta T_t = ceil(Delta T_0 / 2 * tanh(2 t / Delta T_0 - 2) + Delta T_0 / 2).
 long long ps_interval(long long t, int dt0) {

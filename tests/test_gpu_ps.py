@@ -1,4 +1,4 @@
-"""GPU parity of the intra-party semi-asynchronous parameter server (Sec. 4.2,
+"""GPU parity of the intra-party semi-asynchronous parameter server (Sec. 4.1,
 Eq. 5): per-worker replicas updated by their own steps and averaged after the
 epochs Eq. 5 selects, against the oracle on the same seeded inputs, step by
 step (every tap, gradient and the updated replica); then the concurrent

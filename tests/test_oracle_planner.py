@@ -1,4 +1,4 @@
-"""Pins of the oracle's system planner (Sec. 4.3-4.4, Eq. 7-17, Algorithm 2):
+"""Pins of the oracle's system planner (Sec. 4.2-4.3, Eq. 7-17, Algorithm 2):
 optima worked out by hand (the crossing of a falling and a rising delay, the
 memory bound of Eq. 15, the communication term), the monotonicity the model
 implies in the worker counts, and the power-law fit recovering known

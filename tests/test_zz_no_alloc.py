@@ -83,3 +83,36 @@ def test_noalloc_rejects_layers_beyond_its_scratch(vfl):
         vfl.weight_grad_noalloc(dpre, x, dW, db, vfl.FP32)
     assert ei.value.status == vfl.VFL_E_INVAL
     assert "fixed scratch" in str(ei.value)
+
+
+def test_noalloc_layer_at_the_scratch_limit(vfl):
+    """A layer whose partial sums need the whole fixed scratch in one split
+    (out*in + out == 4,194,304): accepted, and equal to a float64 matmul and
+    column sum of the same bf16 inputs."""
+    import torch
+    out, fin, rows = 2048, 2047, 3000
+    assert out * fin + out == 4 * 2 ** 20
+    g = torch.Generator().manual_seed(7)
+    dpre = torch.randn(rows, out, generator=g).to(torch.bfloat16)
+    x = torch.rand(rows, fin, generator=g).to(torch.bfloat16)
+    ref_w = (dpre.double().T @ x.double()).numpy()
+    ref_b = dpre.double().sum(0).numpy()
+    dW = torch.full((out, fin), float("nan"), device="cuda")
+    db = torch.full((out,), float("nan"), device="cuda")
+    vfl.weight_grad_noalloc(dpre.cuda(), x.cuda(), dW, db, vfl.BF16)
+    torch.cuda.synchronize()
+    assert rel_err(dW.cpu().numpy(), ref_w) <= TOL["fp32"]
+    assert rel_err(db.cpu().numpy(), ref_b) <= TOL["fp32"]
+
+
+def test_noalloc_rejects_too_wide_inputs(vfl):
+    import torch
+    fin = 65535 * 64 + 1
+    dpre = torch.zeros((1, 1), device="cuda")
+    x = torch.zeros((1, fin), device="cuda")
+    dW = torch.zeros((1, fin), device="cuda")
+    db = torch.zeros((1,), device="cuda")
+    with pytest.raises(vfl.VflError) as ei:
+        vfl.weight_grad_noalloc(dpre, x, dW, db, vfl.FP32)
+    assert ei.value.status == vfl.VFL_E_INVAL
+    assert "input width" in str(ei.value)
