@@ -5,8 +5,13 @@ One "step" is one training mini-batch through the whole path: passive bottom
 forward, publish, active bottom forward, top forward, loss, backward, publish
 the cut-layer gradient, both bottoms' backward and the SGD updates (Algorithm 1
 with the delayed update of App. D).  Default workload: the credit-shaped
-preset (30000 rows, 12/11 features, 12/11-128-64 bottoms, top 128-64-1, BCE,
-batch 1024, staleness 2 on the seeded schedule, fp32).  Prints one JSON line.
+preset with the most rows, bytes and FLOPs per epoch: wide-dp (1,000,000 rows,
+1000/1000 binary features, 1000-512-256 bottoms, top 512-256-1, BCE, batch
+8192, staleness 4 on the seeded schedule, bf16 with fp32 accumulation, DP
+clipping + Gaussian noise on the published gradient).  Prints one JSON line.
+
+Timing: the K timed steps run as R >= 5 windows (one epoch each when K allows),
+the L2 flushed before each; value and ms_per_step are the median window's.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config C]
 
@@ -37,10 +42,10 @@ TF32_PER_BF16 = 1.1 / 2.25                               # nominal dense TF32 / 
 def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1500)
-    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--steps", type=int, default=0, help="timed steps (default: 5 epochs of the workload)")
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=2, help="workload preset 1..5 (default 2, credit-shaped)")
+    ap.add_argument("--config", type=int, default=4, help="workload preset 1..5 (default 4, wide-dp)")
     ap.add_argument("--rows", type=int, default=0, help="override the preset's row count")
     ap.add_argument("--workers", type=int, default=0, help="override the preset's worker streams per party")
     ap.add_argument("--dp-target", choices=["grad", "emb"], default=None,
@@ -167,17 +172,23 @@ import sys, time, json, os
 sys.path.insert(0, {root!r})
 import numpy as np, synth, oracle
 p = synth.VflPreset(**{fields!r})      # the workload exactly as the GPU arm runs it
-n_steps = {n_steps}
 nb = p.steps_per_epoch
-last = min(n_steps, nb) * p.batch
-rows = min(p.n_rows, last)
-if n_steps > nb: rows = p.n_rows
-xp, xa, y = synth.make_dataset(p, rows=(0, rows))
-q = p.with_(n_rows=rows)
-params = synth.init_params(q)
-tp, ta = oracle.make_schedule(q.seed, q.staleness, {kind}, n_steps)
-drops = oracle.make_drops(q.seed, {drop_rate}, n_steps)
-o = oracle.Oracle(q, xp, xa, y, params, dp_seed=q.seed)
+
+def build(n_steps):
+    # the rows the first n_steps steps train (step k < nb trains batch k): the sample's steps see
+    # exactly the batches, versions and schedule of the full workload
+    rows = p.n_rows if n_steps >= nb else n_steps * p.batch
+    xp, xa, y = synth.make_dataset(p, rows=(0, rows))
+    q = p.with_(n_rows=rows)
+    tp, ta = oracle.make_schedule(q.seed, q.staleness, {kind}, n_steps)
+    drops = oracle.make_drops(q.seed, {drop_rate}, n_steps)
+    return oracle.Oracle(q, xp, xa, y, synth.init_params(q), dp_seed=q.seed), tp, ta, drops
+
+# size the sample from one probe step, so that only the rows it trains are generated
+o, tp, ta, drops = build(1)
+t0 = time.perf_counter(); o.step(0, 0); t_probe = time.perf_counter() - t0
+n_steps = max(1, min({n_steps}, int({budget} / max(t_probe, 1e-6)) + 1))
+o, tp, ta, drops = build(n_steps)
 t0 = time.perf_counter(); done = 0; nsamp = 0
 while done < n_steps:
     r = o.step(int(tp[done]), int(ta[done]), drop=bool(drops[done]))
@@ -189,8 +200,30 @@ print(json.dumps(dict(steps=done, samples=nsamp, seconds=dt)))
 """
 
 
-def run_oracle(p, args, n_steps, budget):
-    cores = os.cpu_count() or 1
+def cpu_model():
+    """The host CPU's model name (lscpu; /proc/cpuinfo as a fallback)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def run_oracle(p, args, n_steps, budget, threads=None):
+    """The oracle as it stands, timed in a subprocess (no CUDA) with `threads` BLAS threads (default:
+    every host core): at most n_steps steps and about `budget` seconds of the workload's first steps."""
+    cores = threads or os.cpu_count() or 1
     env = dict(os.environ)
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         env[v] = str(cores)
@@ -206,11 +239,20 @@ def run_oracle(p, args, n_steps, budget):
     return res
 
 
-def cpu_baseline(p, args):
-    res = run_oracle(p, args, args.warmup + args.steps, args.cpu_seconds)
-    return {"value": res["samples"] / res["seconds"], "unit": "samples/s", "cores": res["cores"], "kind": "oracle",
-            "sample": f"first {res['steps']} training steps ({res['samples']} samples) of the same workload, "
-                      f"float64 numpy oracle, {res['seconds']:.2f} s, BLAS threads={res['cores']}"}
+def cpu_baseline(p, args, n_steps):
+    """The oracle on the host cores, all of them and one: value = the all-cores figure."""
+    model = cpu_model()
+    full = run_oracle(p, args, n_steps, args.cpu_seconds)
+    one = run_oracle(p, args, n_steps, args.cpu_seconds, threads=1)
+
+    def leg(res):
+        return {"value": res["samples"] / res["seconds"], "threads": res["cores"], "steps": res["steps"],
+                "samples": res["samples"], "seconds": round(res["seconds"], 3)}
+    return {"value": full["samples"] / full["seconds"], "unit": "samples/s", "cores": full["cores"], "kind": "oracle",
+            "cpu_model": model, "all_cores": leg(full), "single_thread": leg(one),
+            "sample": f"first {full['steps']} training steps ({full['samples']} samples) of the same workload "
+                      f"(single thread: {one['steps']} steps), float64 numpy oracle, {full['seconds']:.2f} s with "
+                      f"BLAS threads={full['cores']} on {model}"}
 
 
 # --------------------------------------------------------------------------
@@ -315,6 +357,22 @@ def job_throughput(samples_per_rank: int, world: int, slowest_seconds: float) ->
     return samples_per_rank * world / slowest_seconds
 
 
+def plan(p, args):
+    """(W, K, window, n_e2e): warm-up and timed steps, steps per timed window (R >= 5 windows of one
+    training run of the workload each when K allows), and the end-to-end leg's steps per method (at
+    least one epoch, so that its per-epoch graph updates amortise)."""
+    nb = p.steps_per_epoch
+    run_len = nb * max(1, p.epochs)
+    K = args.steps or 5 * run_len
+    window = run_len if K >= 5 * run_len else max(1, -(-K // 5))
+    return max(args.warmup, 3), K, window, max(nb, K)
+
+
+def config_of(desc, world):
+    """The `config` object both arms print: the workload and how it is spread over devices."""
+    return {"workload": desc, "parallelism": f"replicas x{world} (one per GPU)" if world > 1 else "single device"}
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -332,14 +390,14 @@ def run_ours(args):
     build.build()
 
     p, desc = workload(args)
+    W, K, window, n_e2e = plan(p, args)
     cpu = None
     if rank == 0 and world == 1 and not args.skip_cpu:
-        cpu = cpu_baseline(p, args)          # before the GPU work: the oracle runs on idle host cores
+        cpu = cpu_baseline(p, args, W + K)   # before the GPU work: the oracle runs on idle host cores
 
     xp, xa, y = synth.make_dataset(p)
     params = synth.init_params(p)
-    W, K = args.warmup, args.steps
-    total = W + 4 * K
+    total = W + 2 * K + 2 * n_e2e
     tp, ta = vfl.make_schedule(p.seed, p.staleness, sched_kind(p), total)
     drops = vfl.make_drops(p.seed, args.drop_rate, total) if args.drop_rate > 0 else None
     ctx = vfl.Context(p, p.n_rows)
@@ -348,25 +406,22 @@ def run_ours(args):
     main = torch.cuda.Stream()
     flush = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")   # > 129 MB L2
     nb = p.steps_per_epoch
-    # a timed iteration is one training run of the workload (its epochs; the data stays in L2 from one epoch
-    # to the next, as in a real run); the L2 is flushed between iterations
-    run_len = nb * max(1, p.epochs)
-
     use_graphs = not args.no_graphs
 
     def timed_block(k0, n, profile=False):
-        """Time steps [k0, k0+n) in iterations of one epoch each; L2 flushed before each.
-        With graphs, each iteration's graph is captured (untimed) just before it runs."""
-        total_ms = 0.0
+        """Time steps [k0, k0+n) in windows of `window` steps, the L2 flushed before each; with graphs
+        each window's graph is captured (untimed) just before it runs.  Returns [(steps, samples, ms)]
+        per window and the per-class profile when asked."""
+        out = []
         k = k0
         if profile:
             ctx.profile(True)
         while k < k0 + n:
-            m = min(run_len, k0 + n - k)
+            m = min(window, k0 + n - k)
             graph = ctx.capture(k, m, tp, ta, drops) if use_graphs else None
             with torch.cuda.stream(main):
                 flush.zero_()
-                # keep the GPU busy while the host enqueues this iteration, so that the host's launch
+                # keep the GPU busy while the host enqueues this window, so that the host's launch
                 # latency stays outside the device-timed interval that starts at e0
                 torch.cuda._sleep(HOST_ENQUEUE_CYCLES)
                 e0 = torch.cuda.Event(enable_timing=True)
@@ -384,13 +439,13 @@ def run_ours(args):
                 main.wait_event(ev)
             e1.record(main)
             main.synchronize()
-            total_ms += e0.elapsed_time(e1)
+            out.append((m, samples(p, k, m, drops), e0.elapsed_time(e1)))
             k += m
         prof = None
         if profile:
             ctx.profile(False)
             prof = ctx.profile_summary()
-        return total_ms, prof
+        return out, prof
 
     # warm-up
     ctx.train_steps(0, W, tp, ta, drops)
@@ -401,13 +456,17 @@ def run_ours(args):
     clocks = Clocks(local)
     l0 = ctx.launches
     x0 = ctx.exchange_bytes()
-    ms, _ = timed_block(W, K)
+    wins, _ = timed_block(W, K)
     launches = ctx.launches - l0
     x1 = ctx.exchange_bytes()
     torch.cuda.synchronize()
     clk = clocks.stop()
-    ms = slowest_rank(ms)
-    value = job_throughput(samples(p, W, K, drops), world, ms / 1e3)
+    # the median window (by samples/s) decides; max over ranks of its per-sample time
+    rates = sorted(wins, key=lambda t: t[1] / t[2])
+    mid = rates[len(rates) // 2]
+    ms_med = slowest_rank(mid[2])
+    value = job_throughput(mid[1], world, ms_med / 1e3)
+    ms_per_step = ms_med / mid[0]
 
     # per-kernel timing: the same workload again, every launch bracketed by CUDA events (recorded
     # inside the replayed graphs when graphs are on, so each duration is the kernel as the step runs it)
@@ -424,24 +483,23 @@ def run_ours(args):
         pin_xp = torch.from_numpy(xp).pin_memory()
         pin_xa = torch.from_numpy(xa).pin_memory()
         pin_y = torch.from_numpy(y).pin_memory()
-        loss_host = torch.full((K,), float("nan"), dtype=torch.float32).pin_memory()
+        loss_host = torch.full((n_e2e,), float("nan"), dtype=torch.float32).pin_memory()
         ctx.bind_host_data(pin_xp, pin_xa, pin_y, loss_out=loss_host)
 
         def e2e_run(k0, graphs):
-            """Wall time of steps [k0, k0+K): enqueued directly, or in the uniform dependency order as one
-            graph per epoch, re-recorded and updated in place by the host while the previous epoch's replay
-            runs (a new capture only when the window's shape changes; all of it timed)."""
+            """Wall time of steps [k0, k0+n_e2e): enqueued directly, or in the uniform dependency order as
+            one graph per epoch, re-recorded and updated in place by the host while the previous epoch's
+            replay runs (a new capture only when the window's shape changes; all of it timed)."""
             loss_host.fill_(float("nan"))
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             if graphs:
                 ctx.set_order(True)
-                # (window length, first worker) -> graph: a window's shape depends on both (two graphs used in
-                # turn, so that the host never updates the one being replayed, measured slower: 36.5 M)
+                # (window length, first worker) -> graph: a window's shape depends on both
                 cache = {}
                 k = k0
-                while k < k0 + K:
-                    m = min(nb, k0 + K - k)
+                while k < k0 + n_e2e:
+                    m = min(nb, k0 + n_e2e - k)
                     key = (m, k % p.workers)
                     g = cache.get(key)
                     if g is not None and ctx.update_graph(g, k, m, tp, ta, drops):
@@ -452,38 +510,41 @@ def run_ours(args):
                     ctx.launch_graph(g)
                     k += m
             else:
-                ctx.train_steps(k0, K, tp, ta, drops)
+                ctx.train_steps(k0, n_e2e, tp, ta, drops)
             ctx.synchronize()
             dt = slowest_rank(time.perf_counter() - t0)
             ctx.set_order(False)
-            kept = np.ones(K, bool)            # the host ring's slot k mod K holds step k's loss
+            kept = np.ones(n_e2e, bool)        # the host ring's slot k mod n_e2e holds step k's loss
             if drops is not None:
-                steps = np.arange(k0, k0 + K)
-                kept[steps % K] = drops[steps] == 0
+                steps = np.arange(k0, k0 + n_e2e)
+                kept[steps % n_e2e] = drops[steps] == 0
             assert np.isfinite(loss_host.numpy()[kept]).all() and np.isnan(loss_host.numpy()[~kept]).all()
-            return job_throughput(samples(p, k0, K, drops), world, dt)
+            return job_throughput(samples(p, k0, n_e2e, drops), world, dt)
 
         counts = {"updated": 0, "captured": 0}
         direct = e2e_run(W + 2 * K, False)
-        piped = e2e_run(W + 3 * K, True) if use_graphs else None
+        piped = e2e_run(W + 2 * K + n_e2e, True) if use_graphs else None
         ctx.bind_host_data(None, None, None)
         h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
         e2e = {"value": max(direct, piped or 0.0), "unit": "samples/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": 4, "direct_enqueue": direct, "uniform_order_graph_updates": piped,
-               "graph_windows": counts,
+               "d2h_bytes_per_step": 4, "steps": n_e2e, "direct_enqueue": direct,
+               "uniform_order_graph_updates": piped, "graph_windows": counts,
                "method": "uniform-order graphs updated in flight" if piped and piped > direct else "direct enqueue"}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "samples/s", "n_gpus": world, "steps": K, "warmup": W,
-            "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": dtype_tag(p), "data": "synthetic (seeded stand-in for the paper's tabular data)",
-            "config": {"workload": desc,
-                       "l2": f"flushed (256 MiB write) before each timed iteration: one training run ({max(1, p.epochs)} "
-                             f"epoch(s), {run_len} steps)",
-                       "launch": "CUDA graph per training run, captured before its timed iteration" if use_graphs
+            "config": config_of(desc, world),
+            "timing": {"windows": len(wins), "steps_per_window": window,
+                       "window_ms": [round(t[2], 4) for t in wins],
+                       "window_samples_per_s": [t[1] / t[2] * 1e3 for t in wins],
+                       "statistic": "median window (value, ms_per_step); max over ranks",
+                       "l2": "flushed (256 MiB write) before each window; inputs larger than L2",
+                       "launch": "CUDA graph per window, captured before it runs (untimed)" if use_graphs
                        else "direct enqueue",
-                       "parallelism": f"replicas x{world}" if world > 1 else "1 GPU, 2 parties on separate streams"},
+                       "streams": f"{p.workers} worker stream(s) per party"},
             "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roof, "cpu_baseline": cpu,
             # Sec. 5's communication cost: payload bytes through the two channels per timed step
             "exchange_bytes_per_step": {"embedding": (x1[0] - x0[0]) / K, "gradient": (x1[1] - x0[1]) / K},
@@ -501,20 +562,22 @@ def run_reference(args):
     if rank != 0:
         return
     p, desc = workload(args)
+    W, K, _, _ = plan(p, args)
     budget = 60.0
     t0 = time.perf_counter()
     # warm-up steps, then the timed steps, each a bounded sample of the workload
-    run_oracle(p, args, max(args.warmup, 1), 20.0)
-    res = run_oracle(p, args, args.steps, budget)
+    run_oracle(p, args, max(W, 1), 20.0)
+    res = run_oracle(p, args, K, budget)
     value = res["samples"] / res["seconds"]
-    cpu = {"value": value, "unit": "samples/s", "cores": res["cores"], "kind": "oracle",
-           "sample": f"first {res['steps']} of {args.steps} training steps ({res['samples']} samples), "
-                     f"float64 numpy oracle, {res['seconds']:.2f} s"}
+    model = cpu_model()
+    cpu = {"value": value, "unit": "samples/s", "cores": res["cores"], "kind": "oracle", "cpu_model": model,
+           "sample": f"first {res['steps']} of {K} training steps ({res['samples']} samples), "
+                     f"float64 numpy oracle, {res['seconds']:.2f} s with BLAS threads={res['cores']} on {model}"}
     line = {"metric": METRIC, "value": value, "unit": "samples/s", "n_gpus": world, "steps": res["steps"],
-            "warmup": args.warmup, "ms_per_step": res["seconds"] / max(res["steps"], 1) * 1e3,
+            "warmup": W, "ms_per_step": res["seconds"] / max(res["steps"], 1) * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded stand-in for the paper's tabular data)", "impl": "reference",
-            "config": {"workload": desc, "parallelism": "CPU oracle, host cores"},
+            "config": config_of(desc, world),
             "cpu_baseline": cpu, "e2e": {"value": value, "unit": "samples/s", "h2d_bytes_per_step": 0,
                                          "d2h_bytes_per_step": 0},
             "wall_s": time.perf_counter() - t0}
