@@ -330,14 +330,22 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
     }
     __syncthreads();
-    if (last && tid == 0) {
+    if (last) {
+        // thread t sums blocks t, t + HEAD_NT, ... in order, then a fixed shuffle tree and the warps in order
         __threadfence();
         float v = 0.f;
-        for (int bb = 0; bb < (int)gridDim.x; ++bb) v += __ldcg(a.blk_loss + bb);
-        *a.loss_out = v * inv_b;
-        if (a.loss_host) *a.loss_host = v * inv_b;
-        *a.counter = 0;
-        __threadfence();
+        for (int bb = tid; bb < (int)gridDim.x; bb += HEAD_NT) v += __ldcg(a.blk_loss + bb);
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) wloss[warp] = v;
+        __syncthreads();
+        if (tid == 0) {
+            float t = 0.f;
+            for (int w = 0; w < HEAD_NT / 32; ++w) t += wloss[w];
+            *a.loss_out = t * inv_b;
+            if (a.loss_host) *a.loss_host = t * inv_b;
+            *a.counter = 0;
+            __threadfence();
+        }
     }
 }
 
@@ -345,133 +353,222 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
 // DP: per-row clip of the per-sample gradient B*dz to norm C, plus sigma*C*N(0,1).
 // ---------------------------------------------------------------------------
 constexpr int DP_NT = 256;
+constexpr int DP_ROWS = DP_NT / 32;            // one warp per row
 
+// Sum over the warp's lanes in a fixed shuffle order.
+__device__ __forceinline__ float warp_sum(float v) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Four consecutive values of a row (fp32 or bf16) starting at column c (c + 4 <= e, 16- / 8-byte aligned).
+__device__ __forceinline__ void ld4(const void* base, long long idx, int bf16, float v[4]) {
+    if (bf16) {
+        const uint2 w = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(base) + idx);
+        const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w.x));
+        const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w.y));
+        v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+    } else {
+        const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(base) + idx);
+        v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
+    }
+}
+
+__device__ __forceinline__ void st4(void* base, long long idx, int bf16, const float v[4]) {
+    if (bf16) {
+        const __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
+        uint2 w;
+        w.x = *reinterpret_cast<const uint32_t*>(&a);
+        w.y = *reinterpret_cast<const uint32_t*>(&b);
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(base) + idx) = w;
+    } else {
+        *reinterpret_cast<float4*>(static_cast<float*>(base) + idx) = make_float4(v[0], v[1], v[2], v[3]);
+    }
+}
+
+// DP on the published gradient (App. C reading): per row g = B_k dz, factor = min(1, C / ||g||),
+// out = (g factor + sigma C N(0,1)) / B_k.  One warp per row; lane l takes the 4-column groups
+// q = l, l + 32, ... (the Philox block of group q gives its four normals).  Rows are 16-byte aligned
+// (leading dims are multiples of 8 elements).
 __global__ void __launch_bounds__(DP_NT) dp_kernel(const float* __restrict__ in, long long ld_in, void* out,
-                                                    long long ld_out, int out_bf16, int e, float clip, float sigma,
-                                                    unsigned long long seed, long long k, float bk) {
+                                                    long long ld_out, int out_bf16, int rows, int e, float clip,
+                                                    float sigma, unsigned long long seed, long long k, float bk) {
     pdl_entry();
-    __shared__ float red[DP_NT / 32];
-    __shared__ float s_factor;
-    const int r = blockIdx.x;
+    const int lane = threadIdx.x & 31;
+    const int r = blockIdx.x * DP_ROWS + (threadIdx.x >> 5);
+    if (r >= rows) return;
     const float* row = in + (long long)r * ld_in;
     float ss = 0.f;
-    for (int c = threadIdx.x; c < e; c += DP_NT) {
-        const float gv = row[c] * bk;
-        ss = fmaf(gv, gv, ss);
-    }
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_down_sync(0xffffffffu, ss, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
-    __syncthreads();
-    if (threadIdx.x < 32) {
-        float v = threadIdx.x < DP_NT / 32 ? red[threadIdx.x] : 0.f;
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
-        if (threadIdx.x == 0) {
-            const float norm = sqrtf(v);
-            s_factor = norm > clip ? clip / norm : 1.0f;
+    for (int q = lane; 4 * q < e; q += 32) {
+        float v[4];
+        if (4 * q + 4 <= e) {
+            ld4(row, 4 * q, 0, v);
+        } else {
+            for (int j = 0; j < 4; ++j) v[j] = 4 * q + j < e ? row[4 * q + j] : 0.f;
+        }
+        for (int j = 0; j < 4; ++j) {
+            const float gv = v[j] * bk;
+            ss = fmaf(gv, gv, ss);
         }
     }
-    __syncthreads();
-    const float factor = s_factor;
+    const float norm = sqrtf(warp_sum(ss));
+    const float factor = norm > clip ? clip / norm : 1.0f;
     const uint2 key = make_uint2((unsigned)(seed & 0xFFFFFFFFull), (unsigned)(seed >> 32));
     const float scale = sigma * clip;
-    for (int q = threadIdx.x; q * 4 < e; q += DP_NT) {
-        float z[4];
+    for (int q = lane; 4 * q < e; q += 32) {
+        float z[4], v[4];
         dp_normals4(q, r, k, 0x4450u, key, z);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int c = 4 * q + j;
-            if (c < e) {
-                const float gv = row[c] * bk;
-                const float v = (gv * factor + scale * z[j]) / bk;
-                stf(out, (long long)r * ld_out + c, out_bf16, v);
-            }
+        const bool whole = 4 * q + 4 <= e;
+        if (whole) {
+            ld4(row, 4 * q, 0, v);
+        } else {
+            for (int j = 0; j < 4; ++j) v[j] = 4 * q + j < e ? row[4 * q + j] : 0.f;
+        }
+        for (int j = 0; j < 4; ++j) v[j] = (v[j] * bk * factor + scale * z[j]) / bk;
+        if (whole) {
+            st4(out, (long long)r * ld_out + 4 * q, out_bf16, v);
+        } else {
+            for (int j = 0; j < 4 && 4 * q + j < e; ++j) stf(out, (long long)r * ld_out + 4 * q + j, out_bf16, v[j]);
         }
     }
 }
 
 // DP on the published embedding (App. C): per row c = min(1, C / ||z||) (1 for a zero row), the
 // payload c z + sigma C N(0,1) (tag 0x4445) in the compute dtype, and c kept for the backward.
+// One warp per row, as dp_kernel.
 __global__ void __launch_bounds__(DP_NT) dp_emb_kernel(const void* z, long long ld, int bf16, void* out,
-                                                        float* __restrict__ scale_out, int e, float clip, float sigma,
-                                                        unsigned long long seed, long long k) {
+                                                        float* __restrict__ scale_out, int rows, int e, float clip,
+                                                        float sigma, unsigned long long seed, long long k) {
     pdl_entry();
-    __shared__ float red[DP_NT / 32];
-    __shared__ float s_factor;
-    const int r = blockIdx.x;
+    const int lane = threadIdx.x & 31;
+    const int r = blockIdx.x * DP_ROWS + (threadIdx.x >> 5);
+    if (r >= rows) return;
     const long long base = (long long)r * ld;
     float ss = 0.f;
-    for (int c = threadIdx.x; c < e; c += DP_NT) {
-        const float v = ldany(z, base + c, bf16);
-        ss = fmaf(v, v, ss);
-    }
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_down_sync(0xffffffffu, ss, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
-    __syncthreads();
-    if (threadIdx.x < 32) {
-        float v = threadIdx.x < DP_NT / 32 ? red[threadIdx.x] : 0.f;
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
-        if (threadIdx.x == 0) {
-            const float norm = sqrtf(v);
-            s_factor = norm > clip ? clip / norm : 1.0f;
-            scale_out[r] = s_factor;
+    for (int q = lane; 4 * q < e; q += 32) {
+        float v[4];
+        if (4 * q + 4 <= e) {
+            ld4(z, base + 4 * q, bf16, v);
+        } else {
+            for (int j = 0; j < 4; ++j) v[j] = 4 * q + j < e ? ldany(z, base + 4 * q + j, bf16) : 0.f;
         }
+        for (int j = 0; j < 4; ++j) ss = fmaf(v[j], v[j], ss);
     }
-    __syncthreads();
-    const float factor = s_factor;
+    const float norm = sqrtf(warp_sum(ss));
+    const float factor = norm > clip ? clip / norm : 1.0f;
+    if (lane == 0) scale_out[r] = factor;
     const uint2 key = make_uint2((unsigned)(seed & 0xFFFFFFFFull), (unsigned)(seed >> 32));
     const float noise = sigma * clip;
-    for (int q = threadIdx.x; q * 4 < e; q += DP_NT) {
-        float xi[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int q = lane; 4 * q < e; q += 32) {
+        float xi[4] = {0.f, 0.f, 0.f, 0.f}, v[4];
         if (noise != 0.f) dp_normals4(q, r, k, 0x4445u, key, xi);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int c = 4 * q + j;
-            if (c < e) stf(out, base + c, bf16, fmaf(ldany(z, base + c, bf16), factor, noise * xi[j]));
+        const bool whole = 4 * q + 4 <= e;
+        if (whole) {
+            ld4(z, base + 4 * q, bf16, v);
+        } else {
+            for (int j = 0; j < 4; ++j) v[j] = 4 * q + j < e ? ldany(z, base + 4 * q + j, bf16) : 0.f;
+        }
+        for (int j = 0; j < 4; ++j) v[j] = fmaf(v[j], factor, noise * xi[j]);
+        if (whole) {
+            st4(out, base + 4 * q, bf16, v);
+        } else {
+            for (int j = 0; j < 4 && 4 * q + j < e; ++j) stf(out, base + 4 * q + j, bf16, v[j]);
         }
     }
 }
 
-// out = g * [z > 0], with g first scaled by rs[row] when rs is given (rounded to T)
+// out = g * [z > 0], with g first scaled by rs[row] when rs is given (rounded to T); each thread takes
+// four consecutive columns of one row (rows are 16-byte aligned: ld is a multiple of 8 elements)
 template <typename T>
 __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ z, T* __restrict__ out,
                                  long long ld, int rows, int e, const float* __restrict__ rs, const HeaderOps hdr) {
     pdl_entry();
     header_check(hdr);
-    const long long n = (long long)rows * e;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
-        const long long r = i / e, c = i % e;
-        const long long idx = r * ld + c;
-        out[idx] = ldf(z + idx) > 0.f ? (rs ? T(rs[r] * ldf(g + idx)) : g[idx]) : T(0.f);
+    const int bf = sizeof(T) == 2;
+    const int gq = (e + 3) / 4;
+    const int n = rows * gq;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        const int r = i / gq, c = (i - r * gq) * 4;
+        const long long idx = (long long)r * ld + c;
+        if (c + 4 <= e) {
+            float gv[4], zv[4], o[4];
+            ld4(g, idx, bf, gv);
+            ld4(z, idx, bf, zv);
+            for (int j = 0; j < 4; ++j) {
+                float v = gv[j];
+                if (rs) v = (float)T(rs[r] * v);
+                o[j] = zv[j] > 0.f ? v : 0.f;
+            }
+            st4(out, idx, bf, o);
+        } else {
+            for (int j = 0; c + j < e; ++j)
+                out[idx + j] = ldf(z + idx + j) > 0.f ? (rs ? T(rs[r] * ldf(g + idx + j)) : g[idx + j]) : T(0.f);
+        }
     }
 }
 
 // ---------------------------------------------------------------------------
 // SGD (Eq. 2): master -= lr * sum_z partial[z]; write the new version's copy.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ int sgd_layer_of(const SgdArgs& a, long long i) {
+    int l = 0;
+    while (l + 1 < a.n_layers && i >= a.L[l + 1].begin) ++l;
+    return l;
+}
+
+__device__ __forceinline__ void sgd_apply(const SgdArgs& a, const SgdLayer& L, long long idx, float gsum, double bsum) {
+    const long long nw = (long long)L.out * L.in;
+    if (idx < nw) {
+        const float w = L.W[idx] - a.lr * gsum;
+        L.W[idx] = w;
+        const long long r = idx / L.in, c = idx % L.in;
+        stf(L.cW, r * L.in_ld + c, a.c_bf16, w);
+    } else {
+        const long long j = idx - nw;
+        const float b = L.b[j] - a.lr * (float)bsum;
+        L.b[j] = b;
+        L.cb[j] = b;
+    }
+}
+
+// One thread per parameter: its partials summed in order (the bias partials in fp64: they largely cancel).
 __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
     pdl_entry();
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < a.total;
          i += (long long)gridDim.x * blockDim.x) {
-        int l = 0;
-        while (l + 1 < a.n_layers && i >= a.L[l + 1].begin) ++l;
-        const SgdLayer& L = a.L[l];
+        const SgdLayer& L = a.L[sgd_layer_of(a, i)];
         const long long idx = i - L.begin;
         const long long nw = (long long)L.out * L.in;
-        if (idx < nw) {
-            float gsum = 0.f;
+        float gsum = 0.f;
+        double bsum = 0.0;
+        if (idx < nw)
             for (int z = 0; z < L.nsplit; ++z) gsum += L.pW[z * L.pW_stride + idx];
-            const float w = L.W[idx] - a.lr * gsum;
-            L.W[idx] = w;
-            const long long r = idx / L.in, c = idx % L.in;
-            stf(L.cW, r * L.in_ld + c, a.c_bf16, w);
+        else
+            for (int z = 0; z < L.nsplit_b; ++z) bsum += L.pb[z * L.pb_stride + (idx - nw)];
+        sgd_apply(a, L, idx, gsum, bsum);
+    }
+}
+
+// One warp per parameter, for layers with many partials (a folded output layer's per-block partials):
+// lane l sums partials l, l + 32, ... in order, then a fixed shuffle tree.
+__global__ void __launch_bounds__(256) sgd_warp_kernel(const SgdArgs a) {
+    pdl_entry();
+    const int lane = threadIdx.x & 31;
+    const long long nwarps = (long long)gridDim.x * (blockDim.x / 32);
+    for (long long i = blockIdx.x * (long long)(blockDim.x / 32) + (threadIdx.x >> 5); i < a.total; i += nwarps) {
+        const SgdLayer& L = a.L[sgd_layer_of(a, i)];
+        const long long idx = i - L.begin;
+        const long long nw = (long long)L.out * L.in;
+        float gsum = 0.f;
+        double bsum = 0.0;
+        if (idx < nw) {
+            for (int z = lane; z < L.nsplit; z += 32) gsum += L.pW[z * L.pW_stride + idx];
+            for (int o = 16; o > 0; o >>= 1) gsum += __shfl_xor_sync(0xffffffffu, gsum, o);
         } else {
-            const long long j = idx - nw;
-            double gsum = 0.0;      // the bias partials largely cancel: sum them in fp64
-            for (int z = 0; z < L.nsplit_b; ++z) gsum += L.pb[z * L.pb_stride + j];
-            const float b = L.b[j] - a.lr * (float)gsum;
-            L.b[j] = b;
-            L.cb[j] = b;
+            for (int z = lane; z < L.nsplit_b; z += 32) bsum += L.pb[z * L.pb_stride + (idx - nw)];
+            for (int o = 16; o > 0; o >>= 1) bsum += __shfl_xor_sync(0xffffffffu, bsum, o);
         }
+        if (lane == 0) sgd_apply(a, L, idx, gsum, bsum);
     }
 }
 
@@ -569,67 +666,6 @@ __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const f
     }
 }
 
-// Column sums over blocks of 64 rows: block (x, y) covers columns
-// [256 x, 256 x + 256) of rows [64 y, 64 y + 64); tx owns 8 adjacent columns,
-// ty every 8th row; the 8 row lanes are combined in a fixed order.
-// Reads 8 columns at a time, so D's row stride must cover ceil(out/8)*8 columns.
-// Column block bx (256 columns) of row block by (64 rows) of one column-sum job.
-__device__ __forceinline__ void colsum_block(const void* D, long long ldd, int rows, int out, int bf16,
-                                             float* __restrict__ Pb, long long pb_stride, int bx, int by) {
-    __shared__ float red[8][257];
-    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-    const int c0 = bx * 256 + tx * 8;
-    const int rb = by * 64;
-    float acc[8] = {};
-    if (c0 < out) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int r = rb + ty + 8 * i;
-            if (r < rows) {
-                if (bf16) {
-                    const uint4 w = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(D) +
-                                                                    (long long)r * ldd + c0);
-                    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float2 f = __bfloat1622float2(h[q]);
-                        acc[2 * q] += f.x;
-                        acc[2 * q + 1] += f.y;
-                    }
-                } else {
-                    const float* row = static_cast<const float*>(D) + (long long)r * ldd + c0;
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) acc[q] += row[q];
-                }
-            }
-        }
-    }
-#pragma unroll
-    for (int q = 0; q < 8; ++q) red[ty][tx * 8 + q] = acc[q];
-    __syncthreads();
-    const int c = bx * 256 + threadIdx.x;
-    if (c < out) {
-        float t = 0.f;
-#pragma unroll
-        for (int y = 0; y < 8; ++y) t += red[y][threadIdx.x];
-        Pb[(long long)by * pb_stride + c] = t;
-    }
-}
-
-__global__ void __launch_bounds__(256) colsum_kernel(const void* D, long long ldd, int rows, int out, int bf16,
-                                                     float* __restrict__ Pb, long long pb_stride) {
-    pdl_entry();
-    colsum_block(D, ldd, rows, out, bf16, Pb, pb_stride, blockIdx.x, blockIdx.y);
-}
-
-// Several layers' column sums in one launch: job blockIdx.z, blocks outside the job's grid return.
-__global__ void __launch_bounds__(256) colsum_batch_kernel(const ColsumBatch b) {
-    pdl_entry();
-    const ColsumJob& j = b.j[blockIdx.z];
-    if ((int)blockIdx.x >= (j.out + 255) / 256 || (int)blockIdx.y >= j.nblocks) return;
-    colsum_block(j.D, j.ldd, j.rows, j.out, j.bf16, j.Pb, j.pb_stride, blockIdx.x, blockIdx.y);
-}
-
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
     pdl_entry();
     const long long n = (long long)rows * cols;
@@ -681,13 +717,14 @@ cudaError_t launch_head(const HeadArgs& a, cudaStream_t s) {
 cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_out, int out_bf16, int rows, int e,
                       float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
-    dp_kernel<<<rows, DP_NT, 0, s>>>(in, ld_in, out, ld_out, out_bf16, e, clip, sigma, seed, k, (float)rows);
+    dp_kernel<<<(rows + DP_ROWS - 1) / DP_ROWS, DP_NT, 0, s>>>(in, ld_in, out, ld_out, out_bf16, rows, e, clip, sigma,
+                                                               seed, k, (float)rows);
     return cudaGetLastError();
 }
 
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
                              const float* row_scale, const HeaderOps& hdr, cudaStream_t s) {
-    const int nb = grid_for((long long)rows * e, 256);
+    const int nb = grid_for((long long)rows * ((e + 3) / 4), 256);
     if (bf16)
         relu_mask_kernel<__nv_bfloat16><<<nb, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(g),
                                                            static_cast<const __nv_bfloat16*>(z),
@@ -702,12 +739,18 @@ cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long 
 cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, float* scale_out, int rows, int e,
                           float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
-    dp_emb_kernel<<<rows, DP_NT, 0, s>>>(z, ld, bf16, out, scale_out, e, clip, sigma, seed, k);
+    dp_emb_kernel<<<(rows + DP_ROWS - 1) / DP_ROWS, DP_NT, 0, s>>>(z, ld, bf16, out, scale_out, rows, e, clip, sigma,
+                                                                   seed, k);
     return cudaGetLastError();
 }
 
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
-    sgd_kernel<<<grid_for(a.total, 256), 256, 0, s>>>(a);
+    int most = 1;
+    for (int l = 0; l < a.n_layers; ++l) most = max(most, max(a.L[l].nsplit, a.L[l].nsplit_b));
+    if (most >= 16)
+        sgd_warp_kernel<<<grid_for(a.total * 32, 256), 256, 0, s>>>(a);
+    else
+        sgd_kernel<<<grid_for(a.total, 256), 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -752,26 +795,6 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
     return cudaGetLastError();
 }
 
-cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
-                          int nblocks, cudaStream_t s) {
-    if (nblocks < 1) return cudaErrorInvalidValue;
-    dim3 grid((out + 255) / 256, nblocks);
-    colsum_kernel<<<grid, 256, 0, s>>>(D, ldd, rows, out, bf16, Pb, pb_stride);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_colsum_batch(const ColsumBatch& b, cudaStream_t s) {
-    if (b.n < 1) return cudaSuccess;
-    if (b.n > kMaxColsumJobs) return cudaErrorInvalidValue;
-    int gx = 1, gy = 1;
-    for (int i = 0; i < b.n; ++i) {
-        if (b.j[i].nblocks < 1) return cudaErrorInvalidValue;
-        gx = max(gx, (b.j[i].out + 255) / 256);
-        gy = max(gy, b.j[i].nblocks);
-    }
-    colsum_batch_kernel<<<dim3(gx, gy, b.n), 256, 0, s>>>(b);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_to_f32(const void* src, long long ld, int rows, int cols, int bf16, float* dst, cudaStream_t s) {
     if (rows <= 0 || cols <= 0) return cudaSuccess;

@@ -1,64 +1,125 @@
 // tcgen05 GEMMs for the bf16 Linear layers of the split-VFL step.
 //
-// One CTA computes one 128 x 128 fp32 accumulator tile in tensor memory:
-//   warp 0     TMA producer: 128B-swizzled bf16 tiles of A and B into a
-//              4-stage shared-memory ring (mbarrier full/empty pairs)
-//   warp 1     allocates TMEM and issues tcgen05.mma (M=128, N=128, K=16) from
-//              one thread; tcgen05.commit frees each stage and finally
-//              signals the epilogue
-//   warps 2-5  epilogue: tcgen05.ld of their 32-lane quarter, fused
-//              bias+ReLU (forward), ReLU-mask + column split (input gradient)
-//              or fp32 split-K partial store (weight gradient)
+// Forward and input-gradient GEMMs (tc_gemm_kernel) are persistent: the grid is
+// at most one CTA per SM and each CTA walks its 128 x BN output tiles (BN = 128
+// or 256, chosen per shape) in a static round-robin order.  Warp roles:
+//   warp 0     TMA producer: 128B-swizzled bf16 tiles of A and B into a ring
+//              of shared-memory stages (mbarrier full / empty pairs)
+//   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = BN, K = 16)
+//              from one thread; tcgen05.commit frees each stage and, after a
+//              tile's last k-block, marks its accumulator full
+//   warps 2-9  epilogue: tcgen05.ld of their 32-lane quarter and column half,
+//              fused bias + ReLU (forward) or ReLU-mask + column split (input
+//              gradient), bf16 rows straight to global memory
+// Two accumulators live in TMEM (2 x BN columns), so the epilogue of one tile
+// runs while the MMAs of the next tile fill the other.
+//
+// The weight gradient (tc_dw_kernel) splits the batch rows over the CTAs of a
+// thread-block cluster: every CTA accumulates its row chunk of one 128 x BN
+// tile of dW = D^T X in TMEM and writes it to its slice of an L2-resident
+// workspace; after a cluster barrier (release / acquire) the CTA that owns each
+// 128 / cluster-size rows of the tile sums the slices in rank order
+// (deterministic).  The owner writes the reduced dW and, for parties with one
+// worker stream, applies the SGD step of Eq. 2 in the same epilogue (fp32
+// master and the new version's bf16 copy).  The bias gradient (column sums of
+// D) is taken by the epilogue warps from the A stages in shared memory while
+// the MMAs run, and reduced with the tile.
+//
 // Operands are K-major (k contiguous) or MN-major (m / n contiguous); the
 // shared-memory descriptors describe both, so no transposed copies are needed:
 //   FWD  C[rows, out] = X[rows, in] . W[out, in]^T     A K-major,  B K-major
 //   DX   C[rows, in]  = D[rows, out] . W[out, in]      A K-major,  B MN-major
 //   DW   P[out, in]   = D[rows, out]^T . X[rows, in]   A MN-major, B MN-major
 // Every wait is bounded: on timeout the CTA records an error bit, drains what
-// it issued (again bounded), frees its TMEM and returns.  The kernel starts with
-// pdl_entry() (a captured graph may launch it programmatically) and thread 0 of
-// CTA 0 checks / publishes a channel header when the step asks it to.
+// it issued (again bounded), frees its TMEM and returns.  Thread 0 of CTA 0
+// checks / publishes a channel header when the step asks it to.
 #include <cuda.h>
+#include <cooperative_groups.h>
 
 #include <algorithm>
 #include <cstring>
 #include <mutex>
 
 #include "vfl_tc.cuh"
-#include "vfl_pdl.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace vfl {
 
 namespace {
 
-constexpr int BM = 128, BN = 128, BK = 64, STAGES = 4;
-constexpr int THREADS = 192;
-constexpr uint32_t TILE_BYTES = BM * BK * 2;              // 16 KB per operand per stage
-constexpr uint32_t BOX_BYTES = 64 * 64 * 2;               // one MN-major box (64 mn x 64 k)
-constexpr size_t SMEM_BYTES = 1024 + 2 * STAGES * TILE_BYTES + 256;
-constexpr uint32_t TMEM_COLS = 128;
+constexpr int BM = 128, BK = 64;                          // K-major stages: 64 k (one 128-byte row)
+constexpr int EPI_WARPS = 8;
+constexpr int THREADS = 64 + 32 * EPI_WARPS;             // producer, MMA issuer, epilogue
+constexpr int DW_KS = 128;                                // weight-gradient stages: 128 k (MN-major boxes)
 constexpr long long WAIT_LIMIT = 1ll << 26;               // polls before a wait is declared hung
+constexpr int MAX_CLUSTER = 16;
+
+// A ring of STAGES shared-memory stages, each one 128 x KS bf16 tile of A and one BN x KS tile of B.
+// K-major operands come as one box (KS = 64: the 128-byte swizzle row); MN-major operands as boxes of
+// 64 m / n columns by KS k rows.
+template <int BN, int STAGES_, int KS_ = BK>
+struct Ring {
+    static constexpr int STAGES = STAGES_;
+    static constexpr int N = BN;
+    static constexpr int KS = KS_;
+    static constexpr uint32_t A_BYTES = BM * KS * 2;
+    static constexpr uint32_t B_BYTES = BN * KS * 2;
+    static constexpr uint32_t BOX_BYTES = 64 * KS * 2;
+    static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr uint32_t RING_BYTES = STAGES * STAGE_BYTES;
+    static constexpr uint32_t CTRL_BYTES = 256;   // barriers, TMEM slot, abort flag
+};
+
+// Forward / input gradient: four (256-wide) or six (128-wide) stages keep the MMAs fed with every SM busy,
+// and leave room for each epilogue warp's output staging (32 rows x 64 bytes).
+template <int BN>
+struct GemmCfg : Ring<BN, BN == 256 ? 4 : 6> {
+    using R = Ring<BN, BN == 256 ? 4 : 6>;
+    static constexpr uint32_t WARP_BYTES = 2048;
+    static constexpr size_t SMEM = 1024 + R::RING_BYTES + R::CTRL_BYTES + EPI_WARPS * WARP_BYTES;
+};
+
+// Weight gradient: 128-wide tiles, stages of 128 k rows (two MN-major boxes per operand: a stage's TMA
+// work covers two 64-row k-blocks), three stages; after the mainloop the ring holds the fp32
+// accumulator tile.  Column-sum scratch: 4 x 128 partials, 128 sums.
+struct DwCfg : Ring<128, 3, DW_KS> {
+    using R = Ring<128, 3, DW_KS>;
+    static constexpr uint32_t CSUM_BYTES = (4 * 128 + 128) * 4;
+    static constexpr size_t SMEM = 1024 + R::RING_BYTES + R::CTRL_BYTES + CSUM_BYTES;
+    static_assert((size_t)128 * (128 + 4) * 4 <= R::RING_BYTES, "the accumulator tile must fit the ring");
+};
 
 struct TcParams {
     int mode;
     int M, N, K;
-    int a_mn, b_mn;          // 1: operand is MN-major in global memory
+    int tiles_m, tiles_n;
+    int a_mn, b_mn;
     int ka;                  // FWD: K index where A switches to the second map
     int kb;                  // DW: N index where B switches to the second map
-    int kchunk;              // DW: K range per split
+    int kchunk;              // DW: rows per cluster rank
     const float* bias;
     int relu;
     void* C;
     long long ldc;
-    int c_f32;
     const void* mask1;
     int n_split;
     void* C2;
     long long ldc2;
     int c2_f32;
     const void* mask2;
-    float* P;
-    long long p_stride;
+    // DW outputs
+    float* P;                // reduced dW [M, N] (row stride ldp), or null
+    long long ldp;
+    float* Pb;               // reduced db [M], or null (no bias gradient)
+    float* ws;               // per-rank partial tiles [cs][tiles][128][BN] (L2-resident exchange)
+    float* wsb;              // per-rank bias partials [cs][tiles_m][128]
+    float* Wm;               // fused SGD: fp32 master [M, N] (row stride N), or null
+    float* bm;               //            fp32 bias master [M]
+    void* cW;                //            new version's bf16 copy [M, cw_ld]
+    long long cw_ld;
+    float* cb;               //            new version's bias copy [M]
+    float lr;
     int* err;
     HeaderOps hdr;
 };
@@ -71,6 +132,10 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
@@ -112,7 +177,8 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo_bytes,
     return d;
 }
 
-// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, M = 128, N = 128.
+// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, M = 128, N = BN.
+template <int BN>
 __device__ __forceinline__ uint32_t instr_desc(int a_mn, int b_mn) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
            ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
@@ -160,42 +226,242 @@ __device__ __forceinline__ float bf16_at(const void* base, long long idx) {
     return __bfloat162float(static_cast<const __nv_bfloat16*>(base)[idx]);
 }
 
+// ---------------------------------------------------------------------------
+// Producer: the k-blocks [kb0, kb0 + nk) of one tile into the ring, continuing
+// the ring position `it` (one count per k-block over the CTA's whole run).
+// ---------------------------------------------------------------------------
+template <typename C>
+__device__ __forceinline__ bool produce_tile(const TcParams& p, const CUtensorMap* ta, const CUtensorMap* ta2,
+                                             const CUtensorMap* mb, int nb0, int m0, int kbeg, int nk, uint8_t* ring,
+                                             uint64_t* full, uint64_t* empty, uint32_t& it, volatile int* abort_flag) {
+    constexpr int BN = C::N;
+    for (int kt = 0; kt < nk; ++kt, ++it) {
+        const int s = it % C::STAGES;
+        if (!mbar_wait(smem_u32(&empty[s]), ((it / C::STAGES) & 1) ^ 1, abort_flag)) return false;
+        const uint32_t bar = smem_u32(&full[s]);
+        mbar_expect_tx(bar, C::STAGE_BYTES);
+        const int k = kbeg + kt * C::KS;
+        const uint32_t dA = smem_u32(ring + s * C::STAGE_BYTES), dB = dA + C::A_BYTES;
+        if (!p.a_mn) {
+            if (k < p.ka)
+                tma_load_2d(dA, ta, k, m0, bar);
+            else
+                tma_load_2d(dA, ta2, k - p.ka, m0, bar);
+        } else {
+            tma_load_2d(dA, ta, m0, k, bar);
+            tma_load_2d(dA + C::BOX_BYTES, ta, m0 + 64, k, bar);
+        }
+        if (!p.b_mn) {
+            tma_load_2d(dB, mb, k, nb0, bar);
+        } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) tma_load_2d(dB + j * C::BOX_BYTES, mb, nb0 + 64 * j, k, bar);
+        }
+    }
+    return true;
+}
+
+// After an abort: wait (bounded) for the loads of the last STAGES ring positions before the CTA exits.
+template <typename C>
+__device__ __forceinline__ void drain_loads(uint64_t* full, uint32_t issued) {
+    const uint32_t first = issued > (uint32_t)C::STAGES ? issued - C::STAGES : 0;
+    for (uint32_t i = first; i < issued; ++i) {
+        const uint32_t bar = smem_u32(&full[i % C::STAGES]);
+        for (long long t = 0; t < WAIT_LIMIT && !mbar_try(bar, (i / C::STAGES) & 1); ++t) {
+        }
+    }
+}
+
+// MMA issue for one tile's k-blocks into accumulator `acc`.
+template <typename C>
+__device__ __forceinline__ bool mma_tile(const TcParams& p, uint32_t acc, int nk, uint8_t* ring, uint64_t* full,
+                                         uint64_t* empty, uint32_t& it, volatile int* abort_flag) {
+    const uint32_t idesc = instr_desc<C::N>(p.a_mn, p.b_mn);
+    for (int kt = 0; kt < nk; ++kt, ++it) {
+        const int s = it % C::STAGES;
+        if (!mbar_wait(smem_u32(&full[s]), (it / C::STAGES) & 1, abort_flag)) return false;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t aB = smem_u32(ring + s * C::STAGE_BYTES), bB = aB + C::A_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < C::KS / 16; ++kk) {
+            // K-major: the 16-element slice starts 32 bytes further along each 128-byte row;
+            // MN-major: it starts 16 rows (2048 bytes) further down each box of KS rows.
+            const uint64_t ad =
+                p.a_mn ? smem_desc(aB + kk * 2048, C::BOX_BYTES, 1024) : smem_desc(aB + kk * 32, 16, 1024);
+            const uint64_t bd =
+                p.b_mn ? smem_desc(bB + kk * 2048, C::BOX_BYTES, 1024) : smem_desc(bB + kk * 32, 16, 1024);
+            mma_bf16(acc, ad, bd, idesc, (kt > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(smem_u32(&empty[s]));
+    }
+    return true;
+}
+
+// Input-gradient epilogue of one 32-column chunk for row m, one row per lane: the passes that straddle
+// the split column between C and C2.
+__device__ __forceinline__ void epilogue_chunk(const TcParams& p, int m, int nbase, float* v) {
+    const bool to_c = nbase + 32 <= min(p.N, p.n_split);
+    const bool to_c2 = nbase >= p.n_split && nbase + 32 <= p.N && ((nbase - p.n_split) & 7) == 0;
+    if (to_c || to_c2) {
+        const long long idx = to_c ? (long long)m * p.ldc + nbase : (long long)m * p.ldc2 + (nbase - p.n_split);
+        const void* mask = to_c ? p.mask1 : p.mask2;
+        if (mask) {
+            const uint4* mk = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mask) + idx);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 w = mk[q];
+                const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                    if (!bf16_positive(ws[h] & 0xFFFFu)) v[8 * q + 2 * h] = 0.f;
+                    if (!bf16_positive(ws[h] >> 16)) v[8 * q + 2 * h + 1] = 0.f;
+                }
+            }
+        }
+        if (to_c2 && p.c2_f32) {
+            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C2) + idx);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        } else {
+            uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2) + idx);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                dst[q] = make_uint4(pack_bf16(v[8 * q], v[8 * q + 1]), pack_bf16(v[8 * q + 2], v[8 * q + 3]),
+                                    pack_bf16(v[8 * q + 4], v[8 * q + 5]), pack_bf16(v[8 * q + 6], v[8 * q + 7]));
+        }
+    } else {
+        for (int i = 0; i < 32; ++i) {
+            const int n = nbase + i;
+            if (n >= p.N) break;
+            float x = v[i];
+            if (n < p.n_split) {
+                const long long idx = (long long)m * p.ldc + n;
+                if (p.mask1 && !(bf16_at(p.mask1, idx) > 0.f)) x = 0.f;
+                static_cast<__nv_bfloat16*>(p.C)[idx] = __float2bfloat16_rn(x);
+            } else {
+                const long long idx = (long long)m * p.ldc2 + (n - p.n_split);
+                if (p.mask2 && !(bf16_at(p.mask2, idx) > 0.f)) x = 0.f;
+                if (p.c2_f32)
+                    static_cast<float*>(p.C2)[idx] = x;
+                else
+                    static_cast<__nv_bfloat16*>(p.C2)[idx] = __float2bfloat16_rn(x);
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Staged epilogue.  A warp owns 32 accumulator rows (its TMEM lane quarter); per pass it takes 32 columns
+// (16 for fp32 output), writes them row per lane into its 32 x 64-byte staging buffer, then reads them
+// back so that four lanes cover one row's 64 bytes and stores whole row segments: every store
+// instruction writes eight full 64-byte pieces of rows.  Two rows share a 128-byte line; the line's
+// eight 16-byte units are XOR-swizzled by the line index, so both directions are conflict-free.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4* stage_unit(uint8_t* stage, int r, int ch) {
+    const int line = r >> 1;
+    const int unit = (((r & 1) << 2) | ch) ^ (line & 7);
+    return reinterpret_cast<uint4*>(stage + line * 128 + unit * 16);
+}
+
+// Read back the staged 32 x 32 bf16 block and store rows [r0, r0 + 32) x columns [n, n + 32) of a bf16
+// matrix (row stride ld, `cols` valid columns from n), masked by mask[idx] > 0 when mask is set.
+__device__ __forceinline__ void store_bf16_block(uint8_t* stage, int lane, __nv_bfloat16* C, long long ld,
+                                                 const __nv_bfloat16* mask, int r0, int rows, int n, int cols) {
+    const int ch = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = i * 8 + (lane >> 2);
+        if (r0 + r >= rows) continue;
+        uint4 d = *stage_unit(stage, r, ch);
+        const int c = ch * 8;
+        const long long idx = (long long)(r0 + r) * ld + n + c;
+        if (c + 8 <= cols) {
+            if (mask) {
+                const uint4 mk = *reinterpret_cast<const uint4*>(mask + idx);
+                const uint32_t mw[4] = {mk.x, mk.y, mk.z, mk.w};
+                uint32_t dw[4] = {d.x, d.y, d.z, d.w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                    if (!bf16_positive(mw[h] & 0xFFFFu)) dw[h] &= 0xFFFF0000u;
+                    if (!bf16_positive(mw[h] >> 16)) dw[h] &= 0x0000FFFFu;
+                }
+                d = make_uint4(dw[0], dw[1], dw[2], dw[3]);
+            }
+            *reinterpret_cast<uint4*>(C + idx) = d;
+        } else {
+            const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&d);
+            for (int e = 0; e < 8 && c + e < cols; ++e) {
+                __nv_bfloat16 x = h[e];
+                if (mask && !(__bfloat162float(mask[idx + e]) > 0.f)) x = __float2bfloat16_rn(0.f);
+                C[idx + e] = x;
+            }
+        }
+    }
+}
+
+// The same for 16 fp32 columns per pass (64 bytes a row): v[16] of row `lane` into the staging buffer,
+// then rows [r0, r0 + 32) x columns [n, n + 16) of an fp32 matrix, masked by a bf16 mask when set.
+__device__ __forceinline__ void store_f32_block(uint8_t* stage, int lane, const float* v, float* C, long long ld,
+                                                const __nv_bfloat16* mask, int r0, int rows, int n, int cols) {
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+        *reinterpret_cast<float4*>(stage_unit(stage, lane, c)) = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+    __syncwarp();
+    const int ch = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = i * 8 + (lane >> 2);
+        if (r0 + r >= rows) continue;
+        const float4 d = *reinterpret_cast<const float4*>(stage_unit(stage, r, ch));
+        const int c = ch * 4;
+        const long long idx = (long long)(r0 + r) * ld + n + c;
+        float dv[4] = {d.x, d.y, d.z, d.w};
+        for (int e = 0; e < 4; ++e)
+            if (mask && c + e < cols && !(__bfloat162float(mask[idx + e]) > 0.f)) dv[e] = 0.f;
+        if (c + 4 <= cols)
+            *reinterpret_cast<float4*>(C + idx) = make_float4(dv[0], dv[1], dv[2], dv[3]);
+        else
+            for (int e = 0; e < 4 && c + e < cols; ++e) C[idx + e] = dv[e];
+    }
+    __syncwarp();
+}
+
+// ---------------------------------------------------------------------------
+// Persistent forward / input-gradient GEMM.
+// ---------------------------------------------------------------------------
+template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap ta2,
-                   const __grid_constant__ CUtensorMap tb, const __grid_constant__ CUtensorMap tb2, const TcParams p) {
-    pdl_entry();
-    header_check(p.hdr);
+                   const __grid_constant__ CUtensorMap tb, const TcParams p) {
+    using C = GemmCfg<BN>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sA = smem;
-    uint8_t* sB = smem + STAGES * TILE_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * STAGES * TILE_BYTES);
-    // bars[0..S) full, [S..2S) empty, [2S] accumulator ready, [2S+1] drain
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2);
+    uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(ring + C::RING_BYTES);
+    uint64_t* empty = full + C::STAGES;
+    uint64_t* acc_full = empty + C::STAGES;      // [2]
+    uint64_t* acc_empty = acc_full + 2;          // [2]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
-    int kbeg = 0, kend = p.K;
-    if (p.mode == GEMM_DW) {
-        kbeg = blockIdx.z * p.kchunk;
-        kend = min(p.K, kbeg + p.kchunk);
-    }
-    const int nk = kend > kbeg ? (kend - kbeg + BK - 1) / BK : 0;
+    const int ntiles = p.tiles_m * p.tiles_n;
+    const int nk = (p.K + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(smem_u32(&bars[s]), 1);
-            mbar_init(smem_u32(&bars[STAGES + s]), 1);
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), 1);
         }
-        mbar_init(smem_u32(&bars[2 * STAGES]), 1);
-        mbar_init(smem_u32(&bars[2 * STAGES + 1]), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), EPI_WARPS);
+        }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(TMEM_COLS)
+                     "r"(2 * BN)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -203,190 +469,356 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_slot;
+    // set-up above overlaps the previous kernel's tail (this CTA's shared memory and TMEM are its own:
+    // no other tensor-core CTA fits the SM beside it); inputs are read only after that kernel completes
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    header_check(p.hdr);
 
-    if (warp == 0 && lane == 0 && nk > 0) {
+    if (warp == 0 && lane == 0) {
         // ---------------- TMA producer ----------------
-        // B tiles of a DW tile that lies past the concat split come from the second map
-        const CUtensorMap* mb = &tb;
-        int nb0 = n0;
-        if (p.mode == GEMM_DW && n0 >= p.kb) {
-            mb = &tb2;
-            nb0 = n0 - p.kb;
+        uint32_t it = 0;
+        for (int t = blockIdx.x; t < ntiles && nk > 0; t += gridDim.x) {
+            const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
+            if (!produce_tile<C>(p, &ta, &ta2, &tb, n0, m0, 0, nk, ring, full, empty, it, abort_flag)) break;
         }
-        int issued = 0;
-        for (int kt = 0; kt < nk; ++kt) {
-            const int s = kt % STAGES;
-            const uint32_t it = kt / STAGES;
-            if (!mbar_wait(smem_u32(&bars[STAGES + s]), (it & 1) ^ 1, abort_flag)) break;
-            const uint32_t full = smem_u32(&bars[s]);
-            mbar_expect_tx(full, 2 * TILE_BYTES);
-            const int k = kbeg + kt * BK;
-            const uint32_t dA = smem_u32(sA + s * TILE_BYTES), dB = smem_u32(sB + s * TILE_BYTES);
-            if (!p.a_mn) {
-                if (k < p.ka)
-                    tma_load_2d(dA, &ta, k, m0, full);
-                else
-                    tma_load_2d(dA, &ta2, k - p.ka, m0, full);
-            } else {
-                tma_load_2d(dA, &ta, m0, k, full);
-                tma_load_2d(dA + BOX_BYTES, &ta, m0 + 64, k, full);
-            }
-            if (!p.b_mn) {
-                tma_load_2d(dB, mb, k, nb0, full);
-            } else {
-                tma_load_2d(dB, mb, nb0, k, full);
-                tma_load_2d(dB + BOX_BYTES, mb, nb0 + 64, k, full);
-            }
-            issued = kt + 1;
-        }
-        // on abort, wait (bounded) for the loads already issued before the CTA exits
-        if (*abort_flag) {
-            for (int kt = (issued > STAGES ? issued - STAGES : 0); kt < issued; ++kt) {
-                const uint32_t bar = smem_u32(&bars[kt % STAGES]);
-                for (long long t = 0; t < WAIT_LIMIT && !mbar_try(bar, (kt / STAGES) & 1); ++t) {
-                }
-            }
-        }
-    } else if (warp == 1 && lane == 0 && nk > 0) {
+        if (*abort_flag) drain_loads<C>(full, it);
+    } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
-        const uint32_t idesc = instr_desc(p.a_mn, p.b_mn);
-        bool ok = true;
-        for (int kt = 0; kt < nk && ok; ++kt) {
-            const int s = kt % STAGES;
-            if (!mbar_wait(smem_u32(&bars[s]), (kt / STAGES) & 1, abort_flag)) {
-                ok = false;
-                break;
-            }
+        uint32_t it = 0;
+        int i = 0;
+        for (int t = blockIdx.x; t < ntiles && nk > 0; t += gridDim.x, ++i) {
+            const int b = i & 1;
+            if (!mbar_wait(smem_u32(&acc_empty[b]), ((i >> 1) & 1) ^ 1, abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t aB = smem_u32(sA + s * TILE_BYTES), bB = smem_u32(sB + s * TILE_BYTES);
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) {
-                // K-major: the 16-element slice starts 32 bytes further along each 128-byte row;
-                // MN-major: it starts 16 rows (2048 bytes) further down the 64-row box.
-                const uint64_t ad = p.a_mn ? smem_desc(aB + kk * 2048, BOX_BYTES, 1024) : smem_desc(aB + kk * 32, 16, 1024);
-                const uint64_t bd = p.b_mn ? smem_desc(bB + kk * 2048, BOX_BYTES, 1024) : smem_desc(bB + kk * 32, 16, 1024);
-                mma_bf16(tmem, ad, bd, idesc, (kt > 0 || kk > 0) ? 1u : 0u);
-            }
-            mma_commit(smem_u32(&bars[STAGES + s]));
+            const bool ok = mma_tile<C>(p, tmem + (uint32_t)(b * BN), nk, ring, full, empty, it, abort_flag);
+            // mark the accumulator full (also after an abort, so that in-flight MMAs finish before TMEM is freed)
+            mma_commit(smem_u32(&acc_full[b]));
+            if (!ok) break;
         }
-        // signal the epilogue (also after an abort, so that in-flight MMAs finish before TMEM is freed)
-        mma_commit(smem_u32(&bars[2 * STAGES]));
     } else if (warp >= 2) {
         // ---------------- epilogue ----------------
-        const int quarter = warp & 3;
-        const int row = quarter * 32 + lane;
-        const int m = m0 + row;
-        bool have = nk > 0;
-        if (have) {
-            have = mbar_wait(smem_u32(&bars[2 * STAGES]), 0, abort_flag);
+        const int quarter = warp & 3;            // TMEM lanes this warp may read
+        const int half = (warp - 2) >> 2;        // column half of the tile
+        const int cbeg = half * (BN / 2);
+        uint8_t* stage = ring + C::RING_BYTES + C::CTRL_BYTES + (warp - 2) * C::WARP_BYTES;
+        int i = 0;
+        for (int t = blockIdx.x; t < ntiles && nk > 0; t += gridDim.x, ++i) {
+            const int b = i & 1;
+            const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
+            // this warp's columns' bias (lane j of pass q holds column cbeg + 32 q + j), loaded while the
+            // tile's MMAs run
+            float bias[BN / 64];
+#pragma unroll
+            for (int q = 0; q < BN / 64; ++q) {
+                const int n = n0 + cbeg + 32 * q + lane;
+                bias[q] = p.mode == GEMM_FWD && n < p.N ? __ldg(p.bias + n) : 0.f;
+            }
+            if (!mbar_wait(smem_u32(&acc_full[b]), (i >> 1) & 1, abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        }
-        for (int c0 = 0; c0 < BN; c0 += 32) {
-            float v[32];
-            if (have) {
-                tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
-            } else {
+            const int r0 = m0 + quarter * 32;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = 0.f;
-            }
-            if (*abort_flag || m >= p.M) continue;
-            const int nbase = n0 + c0;
-            if (p.mode == GEMM_FWD) {
-                __nv_bfloat16* C = static_cast<__nv_bfloat16*>(p.C) + (long long)m * p.ldc + nbase;
-                if (nbase + 32 <= p.N) {
-                    const float4* b4 = reinterpret_cast<const float4*>(p.bias + nbase);
-                    uint32_t packed[16];
+            for (int q = 0; q < BN / 64; ++q) {
+                const int c0 = cbeg + 32 * q;
+                float v[32];
+                tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * BN + c0), v);
+                const int nb = n0 + c0;
+                if (__any_sync(0xffffffffu, *abort_flag != 0) || nb >= p.N) continue;
+                const int cols = min(32, p.N - nb);
+                if (p.mode == GEMM_FWD) {
+                    uint32_t u[16];
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        const float4 bq = b4[q];
-                        float x0 = v[4 * q] + bq.x, x1 = v[4 * q + 1] + bq.y, x2 = v[4 * q + 2] + bq.z,
-                              x3 = v[4 * q + 3] + bq.w;
+                    for (int j = 0; j < 16; ++j) {
+                        float x0 = v[2 * j] + __shfl_sync(0xffffffffu, bias[q], 2 * j);
+                        float x1 = v[2 * j + 1] + __shfl_sync(0xffffffffu, bias[q], 2 * j + 1);
                         if (p.relu) {
-                            x0 = fmaxf(x0, 0.f); x1 = fmaxf(x1, 0.f); x2 = fmaxf(x2, 0.f); x3 = fmaxf(x3, 0.f);
+                            x0 = fmaxf(x0, 0.f);
+                            x1 = fmaxf(x1, 0.f);
                         }
-                        packed[2 * q] = pack_bf16(x0, x1);
-                        packed[2 * q + 1] = pack_bf16(x2, x3);
+                        u[j] = pack_bf16(x0, x1);
                     }
-                    uint4* dst = reinterpret_cast<uint4*>(C);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
-                } else {
-                    for (int i = 0; i < 32 && nbase + i < p.N; ++i) {
-                        float x = v[i] + p.bias[nbase + i];
-                        if (p.relu) x = fmaxf(x, 0.f);
-                        C[i] = __float2bfloat16_rn(x);
-                    }
-                }
-            } else if (p.mode == GEMM_DX) {
-                const bool to_c = nbase + 32 <= min(p.N, p.n_split);
-                const bool to_c2 = nbase >= p.n_split && nbase + 32 <= p.N && ((nbase - p.n_split) & 7) == 0;
-                if (to_c || to_c2) {
-                    const long long idx = to_c ? (long long)m * p.ldc + nbase : (long long)m * p.ldc2 + (nbase - p.n_split);
-                    const void* mask = to_c ? p.mask1 : p.mask2;
-                    if (mask) {
-                        const uint4* mk = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mask) + idx);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const uint4 w = mk[q];
-                            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                            for (int h = 0; h < 4; ++h) {
-                                if (!bf16_positive(ws[h] & 0xFFFFu)) v[8 * q + 2 * h] = 0.f;
-                                if (!bf16_positive(ws[h] >> 16)) v[8 * q + 2 * h + 1] = 0.f;
-                            }
-                        }
-                    }
-                    if (to_c2 && p.c2_f32) {
-                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C2) + idx);
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                    for (int c = 0; c < 4; ++c)
+                        *stage_unit(stage, lane, c) = make_uint4(u[4 * c], u[4 * c + 1], u[4 * c + 2], u[4 * c + 3]);
+                    __syncwarp();
+                    store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(p.C), p.ldc, nullptr, r0, p.M, nb, cols);
+                    __syncwarp();
+                } else if (nb + cols <= p.n_split || (nb >= p.n_split && ((nb - p.n_split) & 7) == 0)) {
+                    // the input gradient: columns < n_split to C (masked by mask1), the rest to C2
+                    const bool to_c = nb < p.n_split;
+                    const __nv_bfloat16* mk = static_cast<const __nv_bfloat16*>(to_c ? p.mask1 : p.mask2);
+                    if (!to_c && p.c2_f32) {
+                        store_f32_block(stage, lane, v, static_cast<float*>(p.C2), p.ldc2, mk, r0, p.M,
+                                        nb - p.n_split, min(16, cols));
+                        if (cols > 16)
+                            store_f32_block(stage, lane, v + 16, static_cast<float*>(p.C2), p.ldc2, mk, r0, p.M,
+                                            nb + 16 - p.n_split, cols - 16);
                     } else {
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2) + idx);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q)
-                            dst[q] = make_uint4(pack_bf16(v[8 * q], v[8 * q + 1]), pack_bf16(v[8 * q + 2], v[8 * q + 3]),
-                                                pack_bf16(v[8 * q + 4], v[8 * q + 5]), pack_bf16(v[8 * q + 6], v[8 * q + 7]));
+                        for (int c = 0; c < 4; ++c)
+                            *stage_unit(stage, lane, c) =
+                                make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                           pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+                        __syncwarp();
+                        store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2),
+                                         to_c ? p.ldc : p.ldc2, mk, r0, p.M, to_c ? nb : nb - p.n_split, cols);
+                        __syncwarp();
                     }
-                } else {
-                    for (int i = 0; i < 32; ++i) {
-                        const int n = nbase + i;
-                        if (n >= p.N) break;
-                        float x = v[i];
-                        if (n < p.n_split) {
-                            const long long idx = (long long)m * p.ldc + n;
-                            if (p.mask1 && !(bf16_at(p.mask1, idx) > 0.f)) x = 0.f;
-                            static_cast<__nv_bfloat16*>(p.C)[idx] = __float2bfloat16_rn(x);
-                        } else {
-                            const long long idx = (long long)m * p.ldc2 + (n - p.n_split);
-                            if (p.mask2 && !(bf16_at(p.mask2, idx) > 0.f)) x = 0.f;
-                            if (p.c2_f32)
-                                static_cast<float*>(p.C2)[idx] = x;
-                            else
-                                static_cast<__nv_bfloat16*>(p.C2)[idx] = __float2bfloat16_rn(x);
-                        }
-                    }
-                }
-            } else {
-                float* P = p.P + (long long)blockIdx.z * p.p_stride + (long long)m * p.ldc + nbase;
-                if (nbase + 32 <= p.N && (p.ldc & 3) == 0) {
-                    float4* dst = reinterpret_cast<float4*>(P);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                } else {
-                    for (int i = 0; i < 32 && nbase + i < p.N; ++i) P[i] = v[i];
+                } else if (r0 + lane < p.M) {
+                    // a pass across the split column: one row per lane
+                    epilogue_chunk(p, r0 + lane, nb, v);
                 }
             }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&acc_empty[b]));
         }
     }
+    // the next kernel of the stream may start its launch while this grid drains
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (*abort_flag && threadIdx.x == 0) atomicOr(p.err, ST_KERNEL_TIMEOUT);
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN) : "memory");
     }
     header_publish(p.hdr);
+}
+
+// ---------------------------------------------------------------------------
+// Weight gradient with the split-K reduction in the cluster (and the SGD).
+// Grid (cluster size, tiles_n, tiles_m); cluster (cluster size, 1, 1).
+// ---------------------------------------------------------------------------
+constexpr int DW_BN = 128;
+constexpr int DW_SLD = DW_BN + 4;   // accumulator rows in shared memory, padded (conflict-free 16-byte stores)
+
+// Owner phase: rows [r_lo, r_lo + rpo) of the tile, four columns a thread, the CS ranks' partial tiles
+// (own slice included: every rank wrote its slice before the cluster barrier) summed in rank order; the
+// CS loads of a group are issued together.  Writes dW and, with the SGD, the master and the new version's
+// bf16 copy.
+template <int CS>
+__device__ __forceinline__ void dw_owner(const TcParams& p, const float* __restrict__ ws, size_t zstride, int r_lo,
+                                         int rpo, int m0, int n0) {
+    float* __restrict__ Wm = p.Wm;
+    const int nq = rpo * (DW_BN / 4);
+    for (int e = threadIdx.x; e < nq; e += THREADS) {
+        const int r = r_lo + e / (DW_BN / 4), c = (e % (DW_BN / 4)) * 4;
+        const int m = m0 + r, n = n0 + c;
+        if (m >= p.M || n >= p.N) continue;
+        const int nn = min(4, p.N - n);
+        float w[4] = {0.f, 0.f, 0.f, 0.f};
+        if (Wm)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (j < nn) w[j] = Wm[(long long)m * p.N + n + j];
+        const float4* src = reinterpret_cast<const float4*>(ws + (size_t)r * DW_BN + c);
+        float4 t[CS];
+#pragma unroll
+        for (int z = 0; z < CS; ++z) t[z] = __ldcg(src + z * (zstride / 4));
+        float g[4] = {t[0].x, t[0].y, t[0].z, t[0].w};
+#pragma unroll
+        for (int z = 1; z < CS; ++z) {
+            g[0] += t[z].x; g[1] += t[z].y; g[2] += t[z].z; g[3] += t[z].w;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (j >= nn) break;
+            if (p.P) p.P[(long long)m * p.ldp + n + j] = g[j];
+            if (Wm) {
+                const float wn = w[j] - p.lr * g[j];
+                Wm[(long long)m * p.N + n + j] = wn;
+                static_cast<__nv_bfloat16*>(p.cW)[(long long)m * p.cw_ld + n + j] = __float2bfloat16_rn(wn);
+            }
+        }
+    }
+}
+
+// The single-rank case: the tile straight from shared memory.
+__device__ __forceinline__ void dw_owner_local(const TcParams& p, const float* S, int m0, int n0) {
+    for (int e = threadIdx.x; e < BM * DW_BN; e += THREADS) {
+        const int r = e / DW_BN, c = e % DW_BN;
+        const int m = m0 + r, n = n0 + c;
+        if (m >= p.M || n >= p.N) continue;
+        const float g = S[r * DW_SLD + c];
+        if (p.P) p.P[(long long)m * p.ldp + n] = g;
+        if (p.Wm) {
+            const long long idx = (long long)m * p.N + n;
+            const float wn = p.Wm[idx] - p.lr * g;
+            p.Wm[idx] = wn;
+            static_cast<__nv_bfloat16*>(p.cW)[(long long)m * p.cw_ld + n] = __float2bfloat16_rn(wn);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    tc_dw_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                 const __grid_constant__ CUtensorMap tb2, const TcParams p) {
+    using C = DwCfg;
+    constexpr int BN = DW_BN;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(ring + C::RING_BYTES);
+    uint64_t* empty = full + C::STAGES;
+    uint64_t* acc_full = empty + C::STAGES;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    float* csum_part = reinterpret_cast<float*>(ring + C::RING_BYTES + C::CTRL_BYTES);   // [4][128]
+    float* csum = csum_part + 4 * 128;                                                     // [128]
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int cs = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int rpo = BM / cs;                     // tile rows each rank owns in the reduction
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.z * BM, n0 = blockIdx.y * BN;
+    const int kbeg = rank * p.kchunk;
+    const int kend = min(p.K, kbeg + p.kchunk);
+    const int nk = kend > kbeg ? (kend - kbeg + C::KS - 1) / C::KS : 0;
+    const bool bias = p.Pb != nullptr && blockIdx.y == 0;   // one column of tiles takes db
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), bias ? 1 + EPI_WARPS : 1);
+        }
+        mbar_init(smem_u32(&acc_full[0]), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(BN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_slot;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
+    if (warp == 0 && lane == 0) {
+        // B tiles past the concat split come from the second map
+        const CUtensorMap* mb = &tb;
+        int nb0 = n0;
+        if (n0 >= p.kb) {
+            mb = &tb2;
+            nb0 = n0 - p.kb;
+        }
+        uint32_t it = 0;
+        if (nk > 0) produce_tile<C>(p, &ta, &ta, mb, nb0, m0, kbeg, nk, ring, full, empty, it, abort_flag);
+        if (*abort_flag) drain_loads<C>(full, it);
+    } else if (warp == 1 && lane == 0) {
+        uint32_t it = 0;
+        if (nk > 0) mma_tile<C>(p, tmem, nk, ring, full, empty, it, abort_flag);
+        mma_commit(smem_u32(&acc_full[0]));
+    } else if (warp >= 2 && bias) {
+        // column sums of the A stages (D[rows, m] MN-major: two 64-column boxes of KS rows x 128 bytes,
+        // 16-byte chunks swizzled by row mod 8): thread e takes columns 2 (e mod 64), +1 over the
+        // KS/4-row quarter e / 64 of each stage
+        const int e = threadIdx.x - 64;
+        const int mp = e & 63, kq = e >> 6;
+        const int mcol = 2 * mp, box = mcol >> 6, mb = mcol & 63;
+        constexpr int QR = C::KS / 4;
+        float s0 = 0.f, s1 = 0.f;
+        for (int kt = 0; kt < nk; ++kt) {
+            const int s = kt % C::STAGES;
+            if (!mbar_wait(smem_u32(&full[s]), (kt / C::STAGES) & 1, abort_flag)) break;
+            const uint8_t* a = ring + s * C::STAGE_BYTES + box * C::BOX_BYTES;
+#pragma unroll 8
+            for (int r = kq * QR; r < kq * QR + QR; ++r) {
+                const uint32_t chunk = ((uint32_t)(mb >> 3) ^ (uint32_t)(r & 7));
+                const __nv_bfloat162 h =
+                    *reinterpret_cast<const __nv_bfloat162*>(a + r * 128 + (chunk << 4) + ((mb & 7) << 1));
+                const float2 f = __bfloat1622float2(h);
+                s0 += f.x;
+                s1 += f.y;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
+        }
+        csum_part[kq * 128 + mcol] = s0;
+        csum_part[kq * 128 + mcol + 1] = s1;
+    }
+    if (warp >= 2) {
+        if (!mbar_wait(smem_u32(&acc_full[0]), 0, abort_flag)) {
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    }
+    __syncthreads();
+    if (bias && threadIdx.x < BM)
+        csum[threadIdx.x] = csum_part[threadIdx.x] + csum_part[128 + threadIdx.x] + csum_part[256 + threadIdx.x] +
+                            csum_part[384 + threadIdx.x];
+
+    // the accumulator tile into shared memory (the ring is free: every MMA and every load is complete),
+    // one row per thread
+    float* S = reinterpret_cast<float*>(ring);
+    if (warp >= 2) {
+        const int quarter = warp & 3, half = (warp - 2) >> 2;
+        const int row = quarter * 32 + lane;
+#pragma unroll 1
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+            float v[32];
+            if (nk > 0 && !*abort_flag) {
+                tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 32; ++q) v[q] = 0.f;
+            }
+            float4* d4 = reinterpret_cast<float4*>(S + row * DW_SLD + c0);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+
+    const int tiles = p.tiles_m * p.tiles_n;
+    const int tile = blockIdx.z * p.tiles_n + blockIdx.y;
+    if (cs == 1) {
+        dw_owner_local(p, S, m0, n0);
+    } else {
+        // the tile into this rank's workspace slice (row-major 128 x BN, L2-resident, coalesced), then a
+        // cluster barrier (release / acquire) before the owners read the slices
+        float4* dst = reinterpret_cast<float4*>(p.ws + ((size_t)rank * tiles + tile) * BM * BN);
+        for (int e = threadIdx.x; e < BM * BN / 4; e += THREADS) {
+            const int r = e / (BN / 4), c = (e % (BN / 4)) * 4;
+            dst[e] = *reinterpret_cast<const float4*>(S + r * DW_SLD + c);
+        }
+        if (bias)
+            for (int r = threadIdx.x; r < BM; r += THREADS) p.wsb[((size_t)rank * p.tiles_m + blockIdx.z) * BM + r] = csum[r];
+        cluster.sync();
+        const size_t zstride = (size_t)tiles * BM * BN;
+        const float* ws = p.ws + (size_t)tile * BM * BN;
+        switch (cs) {
+            case 2: dw_owner<2>(p, ws, zstride, rank * rpo, rpo, m0, n0); break;
+            case 4: dw_owner<4>(p, ws, zstride, rank * rpo, rpo, m0, n0); break;
+            case 8: dw_owner<8>(p, ws, zstride, rank * rpo, rpo, m0, n0); break;
+            default: dw_owner<16>(p, ws, zstride, rank * rpo, rpo, m0, n0); break;
+        }
+    }
+    if (bias && threadIdx.x < rpo) {
+        const int r = rank * rpo + threadIdx.x;
+        const int m = m0 + r;
+        if (m < p.M) {
+            double g = 0.0;       // the bias partials largely cancel: sum them in fp64
+            for (int z = 0; z < cs; ++z)
+                g += z == rank ? csum[r] : __ldcg(p.wsb + ((size_t)z * p.tiles_m + blockIdx.z) * BM + r);
+            p.Pb[m] = (float)g;
+            if (p.bm) {
+                const float b = p.bm[m] - p.lr * (float)g;
+                p.bm[m] = b;
+                p.cb[m] = b;
+            }
+        }
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) atomicOr(p.err, ST_KERNEL_TIMEOUT);
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN) : "memory");
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -424,6 +856,43 @@ bool make_map(CUtensorMap* m, const void* base, long long inner, long long rows,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int sm_count() {
+    static int n = 0;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        int dev = 0, v = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0)
+            n = v;
+        else
+            n = 148;
+        cudaGetLastError();
+    });
+    return n;
+}
+
+template <typename K>
+cudaError_t set_smem(K kernel, size_t bytes, bool cluster) {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess && cluster) e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+}
+
+// Relative cost of one 128 x BN tile's k-block: 128-wide tiles read A and B from shared memory
+// for half the MMA work of 256-wide ones.
+constexpr double kCost128 = 0.62, kCost256 = 1.0;
+
+// Shared-memory sizes (and cluster sizes past 8) the kernels need, set once.
+cudaError_t kernel_attrs() {
+    static cudaError_t attr = [] {
+        cudaError_t e = set_smem(tc_gemm_kernel<128>, GemmCfg<128>::SMEM, false);
+        if (e == cudaSuccess) e = set_smem(tc_gemm_kernel<256>, GemmCfg<256>::SMEM, false);
+        if (e == cudaSuccess) e = set_smem(tc_dw_kernel, DwCfg::SMEM, true);
+        return e;
+    }();
+    return attr;
+}
+
 }  // namespace
 
 bool tc_available() { return encode_fn() != nullptr; }
@@ -443,24 +912,97 @@ bool tc_supported_dx(int in, int out, int n_split, bool c2_f32) {
 
 bool tc_shape_dw(int out, int in, bool concat, int kb) {
     if (out < 16 || in < 1) return false;
-    return !(concat && kb % BN != 0);
+    return !(concat && kb % DW_BN != 0);
 }
 
 bool tc_supported_dw(int out, int in, bool concat, int kb) { return tc_shape_dw(out, in, concat, kb) && tc_available(); }
 
 void tc_choose_split(int out, int in, int rows, int* nsplit, int* kchunk) {
-    const long long tiles = (long long)((out + BM - 1) / BM) * ((in + BN - 1) / BN);
-    long long ns = std::max<long long>(1, (152 + tiles / 2) / std::max<long long>(1, tiles));
-    ns = std::min<long long>(ns, std::max(1, rows / 256));
-    ns = std::min<long long>(ns, 16);
-    int kc = (int)(((rows + ns - 1) / ns + BK - 1) / BK * BK);
-    *kchunk = kc;
-    *nsplit = (rows + kc - 1) / kc;
+    // the cluster reduces its ranks' partials: one reduced gradient per layer
+    (void)out;
+    (void)in;
+    *nsplit = 1;
+    *kchunk = rows;
+}
+
+namespace {
+
+// How many clusters of `cs` weight-gradient CTAs this device can run at once (its SMs per GPC and the
+// kernel's shared memory decide); 0 when such a cluster cannot be scheduled.
+int active_clusters(int cs) {
+    static int cache[5];
+    static std::once_flag once;
+    std::call_once(once, [] {
+        for (int j = 0; j < 5; ++j) cache[j] = 0;
+        if (kernel_attrs() != cudaSuccess) return;
+        for (int j = 0; j < 5; ++j) {
+            const int c = 1 << j;
+            cudaLaunchConfig_t lc;
+            std::memset(&lc, 0, sizeof lc);
+            lc.gridDim = dim3(c, 1, 1);
+            lc.blockDim = dim3(THREADS, 1, 1);
+            lc.dynamicSmemBytes = DwCfg::SMEM;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = c;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            lc.attrs = at;
+            lc.numAttrs = 1;
+            int n = 0;
+            const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, tc_dw_kernel, &lc);
+            cudaGetLastError();
+            cache[j] = e == cudaSuccess ? n : 0;
+        }
+    });
+    int j = 0;
+    while ((1 << j) < cs && j < 4) ++j;
+    return cache[j];
+}
+
+// Workspace floats a cs-rank weight-gradient launch exchanges its partials through.
+long long dw_ws_need(int out, int in, int cs) {
+    const long long tm = (out + BM - 1) / BM, tn = (in + DW_BN - 1) / DW_BN;
+    return (long long)cs * tm * tn * BM * DW_BN + (long long)cs * tm * BM;
+}
+
+}  // namespace
+
+long long tc_dw_ws_floats(int out, int in, int rows) {
+    const int stages = (rows + DW_KS - 1) / DW_KS;
+    const int cs_max = std::min(MAX_CLUSTER, std::max(1, stages / 2));
+    return dw_ws_need(out, in, cs_max);
+}
+
+// Cluster size of the weight gradient: the one with the least estimated time, counting the waves of
+// clusters the device can co-schedule, the 128-row stages each rank streams (about 0.33 us each, bound by
+// their four TMA boxes) and a fixed cost per CTA (set-up, exchange, epilogue) of about 2.5 us; ranks keep
+// at least two stages and the exchange fits the workspace.  The tile width is 128.
+void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_floats, int* bn_out, int* cs_out) {
+    (void)concat;
+    (void)kb;
+    const int stages = std::max(1, (rows + DW_KS - 1) / DW_KS);
+    const long long tiles = (long long)((out + BM - 1) / BM) * ((in + DW_BN - 1) / DW_BN);
+    double best = 1e30;
+    int bcs = 1;
+    for (int cs = 1; cs <= MAX_CLUSTER; cs *= 2) {
+        if (cs > 1 && stages < 2 * cs) break;
+        if (dw_ws_need(out, in, cs) > ws_floats) break;
+        const long long slots = cs == 1 ? (long long)sm_count() : active_clusters(cs);
+        if (slots < 1) continue;
+        const double waves = (double)((tiles + slots - 1) / slots);
+        const double t = waves * ((double)((stages + cs - 1) / cs) * 0.33 + 2.5);
+        if (t < best - 1e-9) {
+            best = t;
+            bcs = cs;
+        }
+    }
+    *bn_out = DW_BN;
+    *cs_out = bcs;
 }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
-    static cudaError_t attr = cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   (int)SMEM_BYTES);
+    const cudaError_t attr = kernel_attrs();
     if (attr != cudaSuccess) return attr;
     if (g.M <= 0 || g.N <= 0) return cudaSuccess;
     TcParams p;
@@ -477,7 +1019,62 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
     std::memset(&tb, 0, sizeof tb);
     std::memset(&tb2, 0, sizeof tb2);
     bool ok = true;
-    dim3 grid((g.M + BM - 1) / BM, (g.N + BN - 1) / BN, 1);
+    if (g.mode == GEMM_DW) {
+        // A(m = out, k = row) = D[row, out], B(n = in, k = row) = X[row, in]: both MN-major, boxes of
+        // 64 columns by 128 rows
+        int bn = DW_BN, cs = 1;
+        tc_dw_plan(g.M, g.N, g.K, g.B2 != nullptr, g.kb, g.ws_floats, &bn, &cs);
+        if (!g.ws || dw_ws_need(g.M, g.N, cs) > g.ws_floats) return cudaErrorInvalidValue;
+        if (g.B2 && g.kb % DW_BN != 0) return cudaErrorInvalidValue;
+        p.a_mn = 1;
+        p.b_mn = 1;
+        p.ka = 1 << 30;
+        p.kb = g.B2 ? g.kb : (1 << 30);
+        ok &= make_map(&ta, g.A, g.lda, g.K, g.lda, 64, DW_KS);
+        const long long n1 = g.B2 ? g.kb : g.ldb;
+        ok &= make_map(&tb, g.B, n1, g.K, g.ldb, 64, DW_KS);
+        tb2 = tb;
+        if (g.B2) ok &= make_map(&tb2, g.B2, g.ldb2, g.K, g.ldb2, 64, DW_KS);
+        if (!ok) return cudaErrorInvalidValue;
+        p.kchunk = ((g.K + cs - 1) / cs + DW_KS - 1) / DW_KS * DW_KS;
+        p.P = g.P;
+        p.ldp = g.ldc;
+        p.Pb = g.Pb;
+        p.ws = g.ws;
+        p.Wm = g.Wm;
+        p.bm = g.bm;
+        p.cW = g.cW;
+        p.cw_ld = g.cw_ld;
+        p.cb = g.cb;
+        p.lr = g.lr;
+        p.tiles_m = (g.M + BM - 1) / BM;
+        p.tiles_n = (g.N + DW_BN - 1) / DW_BN;
+        p.wsb = g.ws + (long long)cs * p.tiles_m * p.tiles_n * BM * DW_BN;
+        cudaLaunchConfig_t lc;
+        std::memset(&lc, 0, sizeof lc);
+        lc.gridDim = dim3(cs, p.tiles_n, p.tiles_m);
+        lc.blockDim = dim3(THREADS, 1, 1);
+        lc.dynamicSmemBytes = DwCfg::SMEM;
+        lc.stream = s;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = cs;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        lc.attrs = at;
+        lc.numAttrs = 1;
+        return cudaLaunchKernelEx(&lc, tc_dw_kernel, ta, tb, tb2, p);
+    }
+    // forward / input gradient: 256-wide tiles unless 128-wide ones finish the grid in fewer
+    // cost-weighted rounds of the SMs
+    const int tm = (g.M + BM - 1) / BM;
+    const long long t128 = (long long)tm * ((g.N + 127) / 128), t256 = (long long)tm * ((g.N + 255) / 256);
+    const int sms = sm_count();
+    const double c128 = (double)((t128 + sms - 1) / sms) * kCost128;
+    const double c256 = (double)((t256 + sms - 1) / sms) * kCost256;
+    const int bn = (g.N > 128 && c256 <= c128) ? 256 : 128;
+    p.tiles_m = tm;
+    p.tiles_n = (g.N + bn - 1) / bn;
     if (g.mode == GEMM_FWD) {
         // A = X [rows, K] (two maps when concatenated along K), B = W [out, K]
         p.a_mn = 0;
@@ -487,13 +1084,12 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
         ok &= make_map(&ta, g.A, k1, g.M, g.lda, 64, BM);
         ta2 = ta;
         if (g.A2) ok &= make_map(&ta2, g.A2, g.lda2, g.M, g.lda2, 64, BM);
-        ok &= make_map(&tb, g.B, g.ldb, g.N, g.ldb, 64, BN);
-        tb2 = tb;
+        ok &= make_map(&tb, g.B, g.ldb, g.N, g.ldb, 64, bn);
         p.bias = g.bias;
         p.relu = g.relu;
         p.C = g.C;
         p.ldc = g.ldc;
-    } else if (g.mode == GEMM_DX) {
+    } else {
         // A = D [rows, K = out], B(n, k) = W[k, n]: W [out rows, in_ld] is MN-major
         p.a_mn = 0;
         p.b_mn = 1;
@@ -501,7 +1097,6 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
         ok &= make_map(&ta, g.A, g.lda, g.M, g.lda, 64, BM);
         ta2 = ta;
         ok &= make_map(&tb, g.B, g.ldb, g.K, g.ldb, 64, 64);
-        tb2 = tb;
         p.C = g.C;
         p.ldc = g.ldc;
         p.mask1 = g.mask1;
@@ -510,26 +1105,14 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
         p.ldc2 = g.ldc2;
         p.c2_f32 = g.c2_f32;
         p.mask2 = g.mask2;
-    } else {
-        // A(m = out, k = row) = D[row, out], B(n = in, k = row) = X[row, in]: both MN-major
-        p.a_mn = 1;
-        p.b_mn = 1;
-        p.ka = 1 << 30;
-        p.kb = g.B2 ? g.kb : (1 << 30);
-        ok &= make_map(&ta, g.A, g.lda, g.K, g.lda, 64, 64);
-        ta2 = ta;
-        const long long n1 = g.B2 ? g.kb : g.ldb;
-        ok &= make_map(&tb, g.B, n1, g.K, g.ldb, 64, 64);
-        tb2 = tb;
-        if (g.B2) ok &= make_map(&tb2, g.B2, g.ldb2, g.K, g.ldb2, 64, 64);
-        p.kchunk = g.kchunk;
-        p.P = g.P;
-        p.p_stride = g.p_stride;
-        p.ldc = g.ldc;
-        grid.z = g.nsplit;
     }
     if (!ok) return cudaErrorInvalidValue;
-    tc_gemm_kernel<<<grid, THREADS, SMEM_BYTES, s>>>(ta, ta2, tb, tb2, p);
+    const long long tiles = (long long)p.tiles_m * p.tiles_n;
+    const int grid = (int)std::min<long long>(tiles, sms);
+    if (bn == 256)
+        tc_gemm_kernel<256><<<grid, THREADS, GemmCfg<256>::SMEM, s>>>(ta, ta2, tb, p);
+    else
+        tc_gemm_kernel<128><<<grid, THREADS, GemmCfg<128>::SMEM, s>>>(ta, ta2, tb, p);
     return cudaGetLastError();
 }
 

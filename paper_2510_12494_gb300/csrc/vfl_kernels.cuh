@@ -174,24 +174,6 @@ cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long 
 // rows of ld_p / ld_a elements (bf16 or fp32, padding columns zero), and the labels.
 cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da, const int* hy, int rows, void* xp,
                               long long ld_p, void* xa, long long ld_a, int* y, int bf16, cudaStream_t s);
-// Column sums in blocks of 64 rows: Pb[z * pb_stride + o] = sum of D[r * ldd + o] over
-// rows r in [64 z, 64 z + 64) (zero for blocks past `rows`); z < nblocks.  D's row
-// stride must cover ceil(out / 8) * 8 columns.
-cudaError_t launch_colsum(const void* D, long long ldd, int rows, int out, int bf16, float* Pb, long long pb_stride,
-                          int nblocks, cudaStream_t s);
-// The same column sums for several layers in one launch (jobs in any order; each as launch_colsum).
-struct ColsumJob {
-    const void* D; long long ldd;
-    int rows, out, bf16, nblocks;
-    float* Pb; long long pb_stride;
-};
-constexpr int kMaxColsumJobs = 16;
-struct ColsumBatch {
-    ColsumJob j[kMaxColsumJobs];
-    int n;
-};
-cudaError_t launch_colsum_batch(const ColsumBatch& b, cudaStream_t s);
-
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);
 

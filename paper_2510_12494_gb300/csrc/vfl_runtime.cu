@@ -50,13 +50,13 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_COLSUM, K_FUSED_UPDATE, K_HEAD, K_PS_AVG, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_FUSED_UPDATE, K_HEAD, K_PS_AVG, K_TC_DW_SGD, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
-    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "bias_colsum", "fused_update", "head_loss",
-    "ps_average"};
+    "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "fused_update", "head_loss",
+    "ps_average", "gemm_tc_dw_sgd"};
 
 struct ProfRec {
     int cls;
@@ -83,8 +83,11 @@ struct Layer {
     float* pb[kMaxWorkers] = {};          // partial db [nsplit][out]
     int nsplit = 1;                       // weight-gradient partials
     int nsplit_b = 1;                     // bias-gradient partials
-    bool colsum_bias = false;             // db from 64-row column-sum blocks (tensor-core dW layers)
     int kchunk = 0;
+    bool tc_dw = false;                   // dW, db on the tensor-core cluster kernel (one reduced partial)
+    bool sgd_in_dw = false;               // ... which also applies this layer's SGD step
+    float* dw_ws[kMaxWorkers] = {};       // ... and exchanges its partial tiles through this workspace
+    long long dw_ws_floats = 0;
 };
 
 // Bump allocator over the caller's workspace (dry run when base == nullptr).
@@ -150,6 +153,9 @@ struct vfl_ctx {
     long long ps_total[2] = {};                 // flat parameter counts: passive, active (f_a and g)
     cudaEvent_t ev_pavg[kEvPool] = {}, ev_aavg[kEvPool] = {};   // per aggregation step: averaging done
 
+    // bf16 path: weight-gradient kernels that also apply the SGD step (one worker stream per party)
+    bool sgd_in_dw = false;
+
     // bf16 path: g's output layer and the loss in one launch (narrow output over a narrow hidden layer)
     bool head = false;
     int* h_counter = nullptr;                   // per worker: blocks finished
@@ -208,9 +214,6 @@ struct vfl_ctx {
     // published after the previous backward, whatever its staleness, so that windows of steps have one
     // graph shape (vfl_graph_update); the arithmetic, with its stale versions, is unchanged
     bool uniform = false;
-    // bias column sums of the per-layer path, gathered over a party's backward and launched as one batch
-    // before its SGD (the d(pre) buffers stay until then)
-    ColsumBatch cs_pending{};
     // vfl_train_epoch in the uniform order: one epoch graph per first worker, updated in place every epoch
     vfl_graph* epoch_graph[kMaxWorkers] = {};
     std::map<std::pair<int, long long>, cudaGraphNode_t> cap_nodes;
@@ -478,7 +481,6 @@ void build_layers(vfl_ctx* ctx) {
             L.out = outs[l];
             L.in_ld = ld8(d_in);
             choose_split(L, c.batch);
-            if (c.dtype == VFL_BF16) tc_choose_split(L.out, L.in, c.batch, &L.nsplit, &L.kchunk);
             L.nsplit_b = L.nsplit;
             if (ctx->fused) {
                 L.nsplit = 1;
@@ -499,8 +501,13 @@ void build_layers(vfl_ctx* ctx) {
                 const bool last_top = v == &ctx->T && l + 1 == v->size();
                 const bool concat = v == &ctx->T && l == 0;
                 if (!last_top && tc_shape_dw(L.out, L.in, concat, ea)) {
-                    L.colsum_bias = true;
-                    L.nsplit_b = (c.batch + 63) / 64;
+                    // the cluster kernel reduces the batch on chip: one gradient, its bias column sums
+                    // and, with one worker stream per party (updates ordered by the stream), the SGD
+                    L.tc_dw = true;
+                    tc_choose_split(L.out, L.in, c.batch, &L.nsplit, &L.kchunk);
+                    L.nsplit_b = 1;
+                    L.sgd_in_dw = ctx->W == 1;
+                    ctx->sgd_in_dw = ctx->sgd_in_dw || L.sgd_in_dw;
                 }
             }
     }
@@ -533,7 +540,7 @@ void build_layers(vfl_ctx* ctx) {
         Layer& H = ctx->T.back();
         H.nsplit = H.nsplit_b = head_blocks(c.batch);
         H.kchunk = kHeadRows;
-        H.colsum_bias = false;
+        H.tc_dw = H.sgd_in_dw = false;
     }
 }
 
@@ -567,6 +574,10 @@ unsigned long long carve_all(vfl_ctx* ctx, void* base) {
             for (int w = 0; w < ctx->W; ++w) {
                 L.pW[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit * L.out * L.in * 4));
                 L.pb[w] = static_cast<float*>(cv.take((unsigned long long)L.nsplit_b * L.out * 4));
+                if (L.tc_dw) {
+                    L.dw_ws_floats = tc_dw_ws_floats(L.out, L.in, ctx->cfg.batch);
+                    L.dw_ws[w] = static_cast<float*>(cv.take((unsigned long long)L.dw_ws_floats * 4));
+                }
             }
         }
     }
@@ -738,62 +749,52 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
     return VFL_OK;
 }
 
-// Launch the gathered column sums as one batch on s (before the SGD that reads them).
-vfl_status flush_colsum(vfl_ctx* ctx, cudaStream_t s) {
-    ColsumBatch& b = ctx->cs_pending;
-    if (b.n == 0) return VFL_OK;
-    double bytes = 0;
-    for (int i = 0; i < b.n; ++i)
-        bytes += (double)b.j[i].rows * b.j[i].out * (b.j[i].bf16 ? 2 : 4) + (double)b.j[i].nblocks * b.j[i].out * 4;
-    PLAUNCH(K_COLSUM, 0, bytes, s, launch_colsum_batch(b, s));
-    b.n = 0;
-    return VFL_OK;
-}
-
-// Queue one layer's bias column sums (64-row block partials) for the party's batch.
-vfl_status defer_colsum(vfl_ctx* ctx, const void* D, long long ldd, int rows, int out, int bf16, float* Pb,
-                        long long pb_stride, int nblocks, cudaStream_t s) {
-    if (ctx->cs_pending.n == kMaxColsumJobs) TRY(flush_colsum(ctx, s));
-    ColsumJob& j = ctx->cs_pending.j[ctx->cs_pending.n++];
-    j.D = D; j.ldd = ldd; j.rows = rows; j.out = out; j.bf16 = bf16; j.nblocks = nblocks;
-    j.Pb = Pb; j.pb_stride = pb_stride;
-    return VFL_OK;
-}
-
 // Partial dW, db of layer L for the step on worker w:
 //   dW[out, in] = dpre^T X, dpre [rows, out] (leading dim ldd, fp32 when dpre_f32).
 //   X may be [X1 | X2] split at column ka (then two GEMMs write the two column blocks).
+// On the tensor-core cluster kernel (L.tc_dw) the one reduced dW and db land in the partial buffers, and
+// with L.sgd_in_dw the same kernel applies the SGD step to replica `rep` and writes version slot `new_slot`.
 vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long long ldd, bool dpre_f32,
-                     const void* X, long long ldx, const void* X2, long long ldx2, int ka, int rows, cudaStream_t s) {
+                     const void* X, long long ldx, const void* X2, long long ldx2, int ka, int rows, cudaStream_t s,
+                     int rep = 0, int new_slot = 0) {
     const int bf = ctx->bf16;
     const int a_bf = dpre_f32 ? 0 : bf;
     const double flops = 2.0 * rows * L.out * L.in;
-    const double bytes = (double)rows * L.out * (dpre_f32 ? 4 : ctx->esz) + (double)rows * L.in * ctx->esz +
-                         (double)L.nsplit * ((double)L.out * L.in + L.out) * 4;
-    if (bf && !dpre_f32 && tc_supported_dw(L.out, L.in, X2 != nullptr, ka)) {
+    if (L.tc_dw && !dpre_f32) {
+        if (!tc_available()) return ctx->fail(VFL_E_CUDA, "tensor-core weight gradient: no tensor-map encoder");
         TcGemm t = {};
         t.mode = GEMM_DW;
         t.M = L.out; t.N = L.in; t.K = rows;
         t.A = dpre; t.lda = ldd;
         t.B = X; t.ldb = ldx; t.B2 = X2; t.ldb2 = ldx2; t.kb = X2 ? ka : L.in;
-        t.P = L.pW[w]; t.p_stride = (long long)L.out * L.in; t.ldc = L.in;
-        t.Pb = L.pb[w]; t.pb_stride = L.out;
-        t.nsplit = L.nsplit; t.kchunk = L.kchunk;
+        t.P = L.pW[w]; t.ldc = L.in;
+        t.Pb = L.pb[w];
+        t.ws = L.dw_ws[w]; t.ws_floats = L.dw_ws_floats;
+        if (L.sgd_in_dw) {
+            t.Wm = L.Wr[rep]; t.bm = L.br[rep];
+            t.cW = L.cW[new_slot]; t.cw_ld = L.in_ld; t.cb = L.cb[new_slot];
+            t.lr = ctx->cfg.lr;
+        }
         t.err = ctx->status;
-        PLAUNCH(K_TC_DW, flops, bytes, s, launch_tc_gemm(t, s));
-        TRY(defer_colsum(ctx, dpre, ldd, rows, L.out, bf, L.pb[w], L.out, L.nsplit_b, s));
+        // D and X once, dW and db written; with the SGD the masters read and written and the copies written
+        const double np_ = (double)L.out * L.in + L.out;
+        const double bytes = (double)rows * L.out * ctx->esz + (double)rows * L.in * ctx->esz + np_ * 4 +
+                             (L.sgd_in_dw ? np_ * 8 + (double)L.out * L.in * ctx->esz + L.out * 4.0 : 0.0);
+        PLAUNCH(L.sgd_in_dw ? K_TC_DW_SGD : K_TC_DW, flops + (L.sgd_in_dw ? 2.0 * np_ : 0.0), bytes, s,
+                launch_tc_gemm(t, s));
         return VFL_OK;
     }
+    const double bytes = (double)rows * L.out * (dpre_f32 ? 4 : ctx->esz) + (double)rows * L.in * ctx->esz +
+                         (double)L.nsplit * ((double)L.out * L.in + L.out) * 4;
     const int n1 = X2 ? ka : L.in;
     GemmArgs g = gemm_base(GEMM_DW, L.out, n1, rows);
     g.A = dpre; g.a_rs = 1; g.a_cs = ldd;
     g.B = X; g.b_rs = 1; g.b_cs = ldx;
     g.P = L.pW[w]; g.p_stride = (long long)L.out * L.in; g.ldc = L.in;
-    g.Pb = L.colsum_bias ? nullptr : L.pb[w]; g.pb_stride = L.out;
+    g.Pb = L.pb[w]; g.pb_stride = L.out;
     g.kchunk = L.kchunk;
     const double f1 = X2 ? flops * n1 / L.in : flops, b1 = X2 ? bytes * n1 / L.in : bytes;
     PLAUNCH(K_SIMT_DW, f1, b1, s, launch_gemm_simt(g, a_bf, bf, bf, L.nsplit, s));
-    if (L.colsum_bias) TRY(defer_colsum(ctx, dpre, ldd, rows, L.out, a_bf, L.pb[w], L.out, L.nsplit_b, s));
     if (X2) {
         GemmArgs g2 = gemm_base(GEMM_DW, L.out, L.in - ka, rows);
         g2.A = dpre; g2.a_rs = 1; g2.a_cs = ldd;
@@ -851,6 +852,7 @@ vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w
     for (std::vector<Layer>* v : {a, b}) {
         if (!v) continue;
         for (Layer& L : *v) {
+            if (L.sgd_in_dw) continue;
             SgdLayer& d = args.L[n++];
             d.W = L.Wr[rep]; d.b = L.br[rep];
             d.pW = L.pW[w]; d.pb = L.pb[w];
@@ -864,6 +866,7 @@ vfl_status sgd(vfl_ctx* ctx, std::vector<Layer>* a, std::vector<Layer>* b, int w
             off += (long long)L.out * L.in + L.out;
         }
     }
+    if (n == 0) return VFL_OK;
     args.n_layers = n;
     args.total = off;
     args.lr = ctx->cfg.lr;
@@ -1372,7 +1375,6 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         ctx->n_act = k + 1;
         return VFL_OK;
     }
-    ctx->cs_pending.n = 0;   // nothing left over from a phase that failed part-way
     // active bottom forward: z^a = f_a(x^a)
     const void* X = Xa0;
     long long ldx = ctx->ldxa;
@@ -1432,61 +1434,65 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
                 launch_loss(ctx->logits[w], y_rows(ctx, k, r0), rows, n_out, c.loss, ctx->ds[w],
                             ctx->losses + (k % kLossCap), loss_host(ctx, k), s));
     }
-    // top backward (the head kernel has done the output layer's part)
+    // top backward (the head kernel has done the output layer's part).  Each layer's input gradient runs
+    // before its weight gradient: a weight-gradient kernel that applies the SGD step may write the version
+    // slot the input gradient reads (tau_a = S), and the published gradient goes out first.
     const bool dp = c.dp_clip > 0.f && c.dp_target == VFL_DP_GRAD;
+    const int rep = ps_rep(ctx, k), nslot = new_version_slot(ctx, k);
+    // SGD in step order (App. D): a weight-gradient kernel that applies it follows update k-1
+    if (ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, false, s));
     for (int l = Lf - 1; l >= 0; --l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
         const void* dpre = last ? (const void*)ctx->ds[w] : ctx->dpre_t[w][l];
         const long long ldd = last ? n_out : ld8(L.out);
-        if (l == 0)
-            TRY(linear_dw(ctx, L, w, dpre, ldd, last, Za, ld8(ea), Zp, ld8(ep), ea, rows, s));
-        else
-            TRY(linear_dw(ctx, L, w, dpre, ldd, last, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0,
-                          rows, s));
         if (l > 0) {
             const long long ldo = ld8(ctx->T[l - 1].out);
             TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_t[w][l - 1], ldo, ctx->act_t[w][l - 1],
                           L.in, nullptr, 0, false, nullptr, s));
-        } else {
-            // split: dz^a (masked -> dpre of the active cut layer), dz^p -> gradient channel (or fp32 for DP)
-            // without DP this kernel writes the published gradient and its header
-            void* C2 = dp ? (void*)ctx->dzp32[w] : ctx->grad[slot];
-            HeaderOps gpub{};
-            gpub.pub = ctx->grad_hdr + slot;
-            gpub.k = k;
-            gpub.batch = (int)ctx->batch_of(k);
-            gpub.version = (int)v;
-            TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_a[w][La - 1], ld8(ea), Za, ea, C2,
-                          ld8(ep), dp, nullptr, s, dp ? nullptr : &gpub));
+            TRY(linear_dw(ctx, L, w, dpre, ldd, last, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0,
+                          rows, s, rep, nslot));
+            continue;
         }
+        // split: dz^a (masked -> dpre of the active cut layer), dz^p -> gradient channel (or fp32 for DP)
+        // without DP this kernel writes the published gradient and its header
+        void* C2 = dp ? (void*)ctx->dzp32[w] : ctx->grad[slot];
+        HeaderOps gpub{};
+        gpub.pub = ctx->grad_hdr + slot;
+        gpub.k = k;
+        gpub.batch = (int)ctx->batch_of(k);
+        gpub.version = (int)v;
+        TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_a[w][La - 1], ld8(ea), Za, ea, C2,
+                      ld8(ep), dp, nullptr, s, dp ? nullptr : &gpub));
+        if (dp) {
+            PLAUNCH(K_DP, 0, (double)rows * ep * (4 + ctx->esz), s,
+                    launch_dp(ctx->dzp32[w], ld8(ep), ctx->grad[slot], ld8(ep), ctx->bf16, rows, ep, c.dp_clip,
+                              c.dp_sigma, c.dp_seed, k, s));
+            PLAUNCH(K_HEADER, 0, 16, s,
+                    launch_write_header(ctx->grad_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
+        }
+        // publish the gradient
+        CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
+        ctx->grad_step[slot] = k;
+        ctx->x_grad += (long long)rows * ep * ctx->esz;
+        TRY(linear_dw(ctx, L, w, dpre, ldd, last, Za, ld8(ea), Zp, ld8(ep), ea, rows, s, rep, nslot));
     }
-    if (dp) {
-        PLAUNCH(K_DP, 0, (double)rows * ep * (4 + ctx->esz), s,
-                launch_dp(ctx->dzp32[w], ld8(ep), ctx->grad[slot], ld8(ep), ctx->bf16, rows, ep, c.dp_clip,
-                          c.dp_sigma, c.dp_seed, k, s));
-        PLAUNCH(K_HEADER, 0, 16, s, launch_write_header(ctx->grad_hdr + slot, k, (int)ctx->batch_of(k), (int)v, s));
-    }
-    // publish the gradient
-    CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
-    ctx->grad_step[slot] = k;
-    ctx->x_grad += (long long)rows * ep * ctx->esz;
     // active bottom backward
     for (int l = La - 1; l >= 0; --l) {
         const Layer& L = ctx->A[l];
         const void* Xin = l == 0 ? Xa0 : ctx->act_a[w][l - 1];
         const long long ldin = l == 0 ? ctx->ldxa : ld8(ctx->A[l - 1].out);
-        TRY(linear_dw(ctx, L, w, ctx->dpre_a[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s));
         if (l > 0) {
             const long long ldo = ld8(ctx->A[l - 1].out);
             TRY(linear_dx(ctx, L, vslot, ctx->dpre_a[w][l], ld8(L.out), false, rows, ctx->dpre_a[w][l - 1], ldo,
                           ctx->act_a[w][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
+        TRY(linear_dw(ctx, L, w, ctx->dpre_a[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s, rep, nslot));
     }
-    // SGD on theta_1 in step order: version k+1 from version k
-    TRY(wait_update_order(ctx, k, false, s));
-    TRY(flush_colsum(ctx, s));
-    TRY(sgd(ctx, &ctx->A, &ctx->T, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
+    // SGD on theta_1 in step order: version k+1 from version k (the layers the weight-gradient kernels
+    // did not update)
+    if (!ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, false, s));
+    TRY(sgd(ctx, &ctx->A, &ctx->T, w, rep, nslot, s));
     CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
     ctx->last_act_step[w] = k;
@@ -1511,7 +1517,6 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
     const int Lp = (int)ctx->P.size();
     const int ep = ctx->P.back().out;
     TRY(wait_ev(ctx, s, ctx->ev_grad[k % kEvPool]));
-    ctx->cs_pending.n = 0;
     if (ctx->fused) {
         const float* Xp = static_cast<const float*>(xp_rows(ctx, k, r0));
         TRY(fused_passive_backward(ctx, k, slot, vslot, rows, w, s));
@@ -1536,20 +1541,22 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
             launch_relu_mask(ctx->grad[slot], ctx->act_p[slot][Lp - 1], ctx->dpre_p[w][Lp - 1], ld8(ep), rows, ep,
                              ctx->bf16, emb_dp(ctx) ? ctx->emb_c[slot] : nullptr, sub, s));
     const void* Xp0 = xp_rows(ctx, k, r0);
+    const int rep = ps_rep(ctx, k), nslot = new_version_slot(ctx, k);
+    if (ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, true, s));
     for (int l = Lp - 1; l >= 0; --l) {
         const Layer& L = ctx->P[l];
         const void* Xin = l == 0 ? Xp0 : ctx->act_p[slot][l - 1];
         const long long ldin = l == 0 ? ctx->ldxp : ld8(ctx->P[l - 1].out);
-        TRY(linear_dw(ctx, L, w, ctx->dpre_p[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s));
+        // the input gradient reads the version the forward used, which this step's SGD may overwrite
         if (l > 0) {
             const long long ldo = ld8(ctx->P[l - 1].out);
             TRY(linear_dx(ctx, L, vslot, ctx->dpre_p[w][l], ld8(L.out), false, rows, ctx->dpre_p[w][l - 1], ldo,
                           ctx->act_p[slot][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
+        TRY(linear_dw(ctx, L, w, ctx->dpre_p[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s, rep, nslot));
     }
-    TRY(wait_update_order(ctx, k, true, s));
-    TRY(flush_colsum(ctx, s));
-    TRY(sgd(ctx, &ctx->P, nullptr, w, ps_rep(ctx, k), new_version_slot(ctx, k), s));
+    if (!ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, true, s));
+    TRY(sgd(ctx, &ctx->P, nullptr, w, rep, nslot, s));
     CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, true, s));
     ctx->n_bwd = k + 1;

@@ -13,9 +13,11 @@ namespace vfl {
 //  DX : C[rows, N=in] = A[rows, K=out] W, B = W [out, ldb] (MN-major operand);
 //       columns < n_split -> C masked by mask1 > 0; the rest -> C2 (bf16),
 //       masked by mask2 when given.
-//  DW : P[z][M=out, N=in] = sum over rows of chunk z of A[rows, out]^T B[rows, in]
-//       (both MN-major operands), B may be [B | B2] split at column kb;
-//       Pb[z][out] = column sums of A over the chunk.
+//  DW : P[M=out, N=in] = A[rows, out]^T B[rows, in] (row stride ldc), reduced over
+//       the batch inside a thread-block cluster (partials through `ws`); B may be [B | B2] split at column
+//       kb; Pb[out] = column sums of A (when Pb is set).  With Wm set, the SGD step
+//       of Eq. 2 follows in the same kernel: Wm -= lr P, bm -= lr Pb (fp32
+//       masters), cW [out, cw_ld] = bf16(Wm) and cb = bm (the new version's copies).
 struct TcGemm {
     int mode;
     int M, N, K;
@@ -30,17 +32,26 @@ struct TcGemm {
     void* C2; long long ldc2;
     const void* mask2;
     int c2_f32;                 // DX: C2 is fp32 (the DP path perturbs it before publishing)
-    float* P; long long p_stride;
-    float* Pb; long long pb_stride;
-    int nsplit, kchunk;
+    float* P;
+    float* Pb;
+    float* ws; long long ws_floats;   // DW: partial-tile exchange (tc_dw_ws_floats(M, N, K) floats)
+    float* Wm; float* bm;       // DW with the SGD step: fp32 masters (null: gradient only)
+    void* cW; long long cw_ld;  // the new version's bf16 copy of W
+    float* cb;                  // and of b
+    float lr;
     int* err;                   // status word: ST_KERNEL_TIMEOUT when a bounded wait gave up
     HeaderOps hdr;              // channel header checked at entry / published at the end (or none)
 };
 
 // The driver's tensor-map encoder is reachable (false on machines without a driver).
 bool tc_available();
-// Split-K factor and chunk (a multiple of 64 rows) of a tensor-core weight gradient over `rows`.
+// Split-K factor and chunk of a tensor-core weight gradient over `rows` as the workspace sees it:
+// one reduced gradient (the cluster reduces its ranks' partials on chip).
 void tc_choose_split(int out, int in, int rows, int* nsplit, int* kchunk);
+// Tensor-core weight gradient: the workspace (floats) its partial tiles go through for a batch of `rows`
+// (enough for every plan tc_dw_plan can pick), and its tile width and cluster size.
+long long tc_dw_ws_floats(int out, int in, int rows);
+void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_floats, int* bn, int* cs);
 // Shape rule for the tensor-core weight gradient (independent of the driver).
 bool tc_shape_dw(int out, int in, bool concat, int kb);
 bool tc_supported_fwd(int in, int out, bool concat, int ka, bool out_f32);
