@@ -2,6 +2,8 @@
 // for narrow layers, the fused loss, DP clip+noise, ReLU mask, fused SGD, batched
 // bias column sums, the parameter-server average, channel headers (behind a DP
 // kernel; otherwise the GEMMs carry them) and data casts.
+#include <algorithm>
+
 #include "vfl_kernels.cuh"
 #include "vfl_philox.cuh"
 #include "vfl_pdl.cuh"
@@ -510,65 +512,58 @@ __global__ void relu_mask_kernel(const T* __restrict__ g, const T* __restrict__ 
 // ---------------------------------------------------------------------------
 // SGD (Eq. 2): master -= lr * sum_z partial[z]; write the new version's copy.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ int sgd_layer_of(const SgdArgs& a, long long i) {
-    int l = 0;
-    while (l + 1 < a.n_layers && i >= a.L[l + 1].begin) ++l;
-    return l;
+__device__ __forceinline__ void sgd_apply_w(const SgdArgs& a, const SgdLayer& L, int r, int c, float g) {
+    const long long idx = (long long)r * L.in + c;
+    const float w = L.W[idx] - a.lr * g;
+    L.W[idx] = w;
+    stf(L.cW, (long long)r * L.in_ld + c, a.c_bf16, w);
 }
 
-__device__ __forceinline__ void sgd_apply(const SgdArgs& a, const SgdLayer& L, long long idx, float gsum, double bsum) {
-    const long long nw = (long long)L.out * L.in;
-    if (idx < nw) {
-        const float w = L.W[idx] - a.lr * gsum;
-        L.W[idx] = w;
-        const long long r = idx / L.in, c = idx % L.in;
-        stf(L.cW, r * L.in_ld + c, a.c_bf16, w);
-    } else {
-        const long long j = idx - nw;
-        const float b = L.b[j] - a.lr * (float)bsum;
-        L.b[j] = b;
-        L.cb[j] = b;
-    }
+__device__ __forceinline__ void sgd_apply_b(const SgdArgs& a, const SgdLayer& L, int j, double g) {
+    const float b = L.b[j] - a.lr * (float)g;
+    L.b[j] = b;
+    L.cb[j] = b;
 }
 
-// One thread per parameter: its partials summed in order (the bias partials in fp64: they largely cancel).
+// SGD (Eq. 2) for every layer of a party: layer blockIdx.y, its out * in weights then its out biases
+// spread over the x blocks.  A layer with few partials takes one thread per parameter (partials summed in
+// order; the bias partials in fp64, they largely cancel); one with many (a folded output layer's
+// per-block partials) one warp per parameter: lane l sums partials l, l + 32, ... in order, then a fixed
+// shuffle tree.
 __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
     pdl_entry();
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < a.total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const SgdLayer& L = a.L[sgd_layer_of(a, i)];
-        const long long idx = i - L.begin;
-        const long long nw = (long long)L.out * L.in;
-        float gsum = 0.f;
-        double bsum = 0.0;
-        if (idx < nw)
-            for (int z = 0; z < L.nsplit; ++z) gsum += L.pW[z * L.pW_stride + idx];
-        else
-            for (int z = 0; z < L.nsplit_b; ++z) bsum += L.pb[z * L.pb_stride + (idx - nw)];
-        sgd_apply(a, L, idx, gsum, bsum);
-    }
-}
-
-// One warp per parameter, for layers with many partials (a folded output layer's per-block partials):
-// lane l sums partials l, l + 32, ... in order, then a fixed shuffle tree.
-__global__ void __launch_bounds__(256) sgd_warp_kernel(const SgdArgs a) {
-    pdl_entry();
-    const int lane = threadIdx.x & 31;
-    const long long nwarps = (long long)gridDim.x * (blockDim.x / 32);
-    for (long long i = blockIdx.x * (long long)(blockDim.x / 32) + (threadIdx.x >> 5); i < a.total; i += nwarps) {
-        const SgdLayer& L = a.L[sgd_layer_of(a, i)];
-        const long long idx = i - L.begin;
-        const long long nw = (long long)L.out * L.in;
-        float gsum = 0.f;
-        double bsum = 0.0;
-        if (idx < nw) {
-            for (int z = lane; z < L.nsplit; z += 32) gsum += L.pW[z * L.pW_stride + idx];
-            for (int o = 16; o > 0; o >>= 1) gsum += __shfl_xor_sync(0xffffffffu, gsum, o);
-        } else {
-            for (int z = lane; z < L.nsplit_b; z += 32) bsum += L.pb[z * L.pb_stride + (idx - nw)];
-            for (int o = 16; o > 0; o >>= 1) bsum += __shfl_xor_sync(0xffffffffu, bsum, o);
+    const SgdLayer& L = a.L[blockIdx.y];
+    const int nw = L.out * L.in, np = nw + L.out;
+    if (L.nsplit < 16 && L.nsplit_b < 16) {
+        for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < np; i += gridDim.x * blockDim.x) {
+            if (i < nw) {
+                float g = 0.f;
+                for (int z = 0; z < L.nsplit; ++z) g += L.pW[z * L.pW_stride + i];
+                const int r = i / L.in;
+                sgd_apply_w(a, L, r, i - r * L.in, g);
+            } else {
+                double g = 0.0;
+                for (int z = 0; z < L.nsplit_b; ++z) g += L.pb[z * L.pb_stride + (i - nw)];
+                sgd_apply_b(a, L, i - nw, g);
+            }
         }
-        if (lane == 0) sgd_apply(a, L, idx, gsum, bsum);
+        return;
+    }
+    const int lane = threadIdx.x & 31;
+    const int nwarps = gridDim.x * (blockDim.x / 32);
+    for (int i = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); i < np; i += nwarps) {
+        if (i < nw) {
+            float g = 0.f;
+            for (int z = lane; z < L.nsplit; z += 32) g += L.pW[z * L.pW_stride + i];
+            for (int o = 16; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o);
+            const int r = i / L.in;
+            if (lane == 0) sgd_apply_w(a, L, r, i - r * L.in, g);
+        } else {
+            double g = 0.0;
+            for (int z = lane; z < L.nsplit_b; z += 32) g += L.pb[z * L.pb_stride + (i - nw)];
+            for (int o = 16; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o);
+            if (lane == 0) sgd_apply_b(a, L, i - nw, g);
+        }
     }
 }
 
@@ -647,23 +642,62 @@ __global__ void cast_rows_kernel(const float* __restrict__ src, int rows, int d,
 
 // One step's rows from host memory (read over the C2C link / PCIe as the kernel runs): element i of
 // the padded passive rows, then of the padded active rows, then the labels.
+// One party's block of rows [rows, d] fp32 (contiguous in host memory) into staging rows of ld elements
+// (bf16 or fp32), padding columns zero.  Four consecutive values a thread when d is a multiple of 4 and
+// the block is 16-byte aligned, four such groups loaded before any is stored (the loads cross the
+// host link: as many as possible in flight).
+__device__ __forceinline__ void stage_block(const float* __restrict__ h, int d, int rows, void* dst, long long ld,
+                                            int bf16, int tid, int nthreads) {
+    const int n = rows * d;
+    if ((d & 3) == 0 && (reinterpret_cast<uintptr_t>(h) & 15) == 0 && (ld & 3) == 0) {
+        const int nq = n / 4;
+        constexpr int U = 4;
+        for (int q0 = tid; q0 < nq; q0 += nthreads * U) {
+            float4 v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = q0 + u * nthreads;
+                if (q < nq) v[u] = __ldcs(reinterpret_cast<const float4*>(h) + q);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = q0 + u * nthreads;
+                if (q >= nq) break;
+                const int f = 4 * q, r = f / d, c = f - r * d;
+                const float vals[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+                if (bf16) {
+                    const __nv_bfloat162 a = __floats2bfloat162_rn(vals[0], vals[1]), b = __floats2bfloat162_rn(vals[2], vals[3]);
+                    uint2 w;
+                    w.x = *reinterpret_cast<const uint32_t*>(&a);
+                    w.y = *reinterpret_cast<const uint32_t*>(&b);
+                    *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(dst) + (long long)r * ld + c) = w;
+                } else {
+                    *reinterpret_cast<float4*>(static_cast<float*>(dst) + (long long)r * ld + c) = v[u];
+                }
+            }
+        }
+    } else {
+        for (int i = tid; i < n; i += nthreads) {
+            const int r = i / d, c = i - r * d;
+            stf(dst, (long long)r * ld + c, bf16, h[i]);
+        }
+    }
+    // padding columns
+    const int pad = (int)(ld - d);
+    for (int i = tid; i < rows * pad; i += nthreads) {
+        const int r = i / pad, c = d + (i - r * pad);
+        stf(dst, (long long)r * ld + c, bf16, 0.f);
+    }
+}
+
 __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const float* __restrict__ hxa, int da,
                                   const int* __restrict__ hy, int rows, void* xp, long long ld_p, void* xa,
                                   long long ld_a, int* __restrict__ y, int bf16) {
     pdl_entry();
-    const long long np = (long long)rows * ld_p, na = (long long)rows * ld_a;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < np + na + rows;
-         i += (long long)gridDim.x * blockDim.x) {
-        if (i < np) {
-            const long long r = i / ld_p, c = i - r * ld_p;
-            stf(xp, i, bf16, c < dp ? hxp[r * dp + c] : 0.f);
-        } else if (i < np + na) {
-            const long long j = i - np, r = j / ld_a, c = j - r * ld_a;
-            stf(xa, j, bf16, c < da ? hxa[r * da + c] : 0.f);
-        } else {
-            y[i - np - na] = hy[i - np - na];
-        }
-    }
+    const int tid = blockIdx.x * blockDim.x + threadIdx.x, nt = gridDim.x * blockDim.x;
+    stage_block(hxp, dp, rows, xp, ld_p, bf16, tid, nt);
+    stage_block(hxa, da, rows, xa, ld_a, bf16, tid, nt);
+    for (int i = tid; i < rows; i += nt) y[i] = hy[i];
 }
 
 __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols, int bf16, float* dst) {
@@ -745,12 +779,17 @@ cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, floa
 }
 
 cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
-    int most = 1;
-    for (int l = 0; l < a.n_layers; ++l) most = max(most, max(a.L[l].nsplit, a.L[l].nsplit_b));
-    if (most >= 16)
-        sgd_warp_kernel<<<grid_for(a.total * 32, 256), 256, 0, s>>>(a);
-    else
-        sgd_kernel<<<grid_for(a.total, 256), 256, 0, s>>>(a);
+    if (a.n_layers < 1) return cudaSuccess;
+    // enough x blocks for the largest layer (a warp per parameter where partials are many), within a
+    // few waves of the SMs over all layers
+    long long most = 1;
+    for (int l = 0; l < a.n_layers; ++l) {
+        const long long np = (long long)a.L[l].out * a.L[l].in + a.L[l].out;
+        const bool warp = a.L[l].nsplit >= 16 || a.L[l].nsplit_b >= 16;
+        most = std::max(most, warp ? np * 32 : np);
+    }
+    const long long bx = std::min<long long>((most + 255) / 256, std::max(1, 152 * 8 / a.n_layers));
+    sgd_kernel<<<dim3((unsigned)bx, a.n_layers), 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -144,7 +144,7 @@ cudaError_t launch_ps_average(const PsAvgLayer* tab, int n_layers, long long tot
 // block sums in block order (the last block to finish).
 constexpr int kHeadMaxOut = 12;
 constexpr int kHeadMaxK = 256;
-constexpr int kHeadRows = 32;
+constexpr int kHeadRows = 16;
 struct HeadArgs {
     const void* h; long long ldh;     // g's last hidden activation rows [rows, ldh], bf16
     const void* W; long long ldw;     // the output layer's version copy [n_out, ldw], bf16
