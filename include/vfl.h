@@ -65,6 +65,10 @@ typedef int32_t vfl_status;
 #define VFL_TAP_LOGITS 2  /* logits of the last active step run on k's worker, [B_k, n_out] */
 #define VFL_TAP_ZA 3      /* active embedding z^a of that step, [B_k, e_a]              */
 #define VFL_TAP_DZA 4     /* dLoss/dz^a of that step, [B_k, e_a]                        */
+/* the output of Linear+ReLU layer `layer` of `party` for step k, [B_k, width] (per-layer kernels only:
+ * VFL_E_STATE on a context that runs the fused fp32 kernels): party 0 = f_p (its last layer is z^p before
+ * any DP), 1 = f_a, 2 = the hidden layers of g */
+#define VFL_TAP_ACT(party, layer) (16 + 16 * (party) + (layer))
 
 typedef struct vfl_config {
     int32_t d_passive;                      /* passive feature count d_p                 */

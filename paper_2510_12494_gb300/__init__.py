@@ -23,6 +23,11 @@ FP32, BF16 = 0, 1
 DP_GRAD, DP_EMB = 0, 1
 SCHED_SYNC, SCHED_MAX, SCHED_SEEDED = 0, 1, 2
 TAP_EMB, TAP_GRAD, TAP_LOGITS, TAP_ZA, TAP_DZA = range(5)
+
+
+def TAP_ACT(party: int, layer: int) -> int:
+    """Tap code of the output of Linear+ReLU layer `layer` of `party` (0 passive, 1 active, 2 top hidden)."""
+    return 16 + 16 * party + layer
 PASSIVE, ACTIVE, TOP = 0, 1, 2
 KERNEL_CLASSES = 19
 
@@ -576,8 +581,12 @@ class Context:
 
     def tap(self, k, what):
         r0, r1 = self.batch_rows(k)
-        cols = {TAP_EMB: self.p.e_passive, TAP_GRAD: self.p.e_passive, TAP_LOGITS: self.p.n_out,
-                TAP_ZA: self.p.e_active, TAP_DZA: self.p.e_active}[what]
+        if what >= 16:
+            party, layer = divmod(what - 16, 16)
+            cols = (self.p.passive, self.p.active, self.p.top)[party][layer]
+        else:
+            cols = {TAP_EMB: self.p.e_passive, TAP_GRAD: self.p.e_passive, TAP_LOGITS: self.p.n_out,
+                    TAP_ZA: self.p.e_active, TAP_DZA: self.p.e_active}[what]
         out = np.zeros((r1 - r0, cols), np.float32)
         self._call(lib().vfl_tap, k, what, _ptr(out), out.size)
         return out

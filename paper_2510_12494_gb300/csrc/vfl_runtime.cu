@@ -2563,8 +2563,28 @@ vfl_status vfl_tap(vfl_ctx* ctx, int64_t k, int32_t what, float* out, int64_t ou
             else if (what == VFL_TAP_ZA) { src = ctx->act_a[w].back(); ld = ld8(ea); cols = ea; }
             else { src = ctx->dpre_a[w].back(); ld = ld8(ea); cols = ea; }
             break;
-        default:
-            return ctx->fail(VFL_E_INVAL, "unknown tap %d", what);
+        default: {
+            const int party = (what - 16) / 16, layer = (what - 16) % 16;
+            if (what < 16 || party > 2) return ctx->fail(VFL_E_INVAL, "unknown tap %d", what);
+            if (ctx->fused) return ctx->fail(VFL_E_STATE, "hidden activations are kept by the per-layer kernels only");
+            if (party == 0) {
+                if (layer >= (int)ctx->P.size()) return ctx->fail(VFL_E_INVAL, "no passive layer %d", layer);
+                if (ctx->slot_step_p[slot] != k)
+                    return ctx->fail(VFL_E_STATE, "passive activations of step %lld are not stored", (long long)k);
+                src = ctx->act_p[slot][layer];
+                cols = ctx->P[layer].out;
+            } else {
+                const std::vector<Layer>& v = party == 1 ? ctx->A : ctx->T;
+                const int n = party == 1 ? (int)v.size() : (int)v.size() - 1;
+                if (layer >= n) return ctx->fail(VFL_E_INVAL, "no stored layer %d of party %d", layer, party);
+                if (ctx->last_act_step[w] != k)
+                    return ctx->fail(VFL_E_STATE, "active buffers of step %lld are not stored", (long long)k);
+                src = party == 1 ? ctx->act_a[w][layer] : ctx->act_t[w][layer];
+                cols = v[layer].out;
+            }
+            ld = ld8(cols);
+            break;
+        }
     }
     if ((long long)rows * cols > out_elems)
         return ctx->fail(VFL_E_INVAL, "tap of step %lld needs %lld floats, the buffer holds %lld", (long long)k,
