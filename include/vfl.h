@@ -530,6 +530,19 @@ const char* vfl_kernel_class_name(int32_t cls);
 vfl_status vfl_weight_grad_noalloc(const void* dpre, const void* x, int32_t rows, int32_t out, int32_t in,
                                    int32_t dtype, float* dW, float* db, void* stream);
 
+/*
+ * Roofline denominators of the fp32 kernels (measurement only; the paper has no counterpart): the
+ * device's FP32 FMA throughput (VFL_PEAK_FFMA: eight independent FMA chains per thread) or its TF32
+ * warp-MMA throughput (VFL_PEAK_TF32_MMA: eight independent m16n8k8 accumulators per warp), eight
+ * 256-thread blocks per SM, `iters` iterations.  One warm-up launch, then one timed launch on the
+ * legacy default stream of the current device: *flops its floating-point operations, *ms its
+ * CUDA-event time.  Allocates and frees a small output buffer.  VFL_E_INVAL for an unknown kind or
+ * iters < 1; the reason in vfl_last_error(NULL).
+ */
+#define VFL_PEAK_FFMA 0
+#define VFL_PEAK_TF32_MMA 1
+vfl_status vfl_measure_peak(int32_t kind, int64_t iters, double* flops, float* ms);
+
 /* Last error message of the context (or of the last failed vfl_create / vfl_make_schedule when ctx is NULL);
  * error reporting has no counterpart in the paper. */
 const char* vfl_last_error(const vfl_ctx* ctx);

@@ -140,8 +140,11 @@ EXPORTS = {
     "vfl_weight_grad_noalloc": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                                  ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
                                                  ctypes.c_void_p]),
+    "vfl_measure_peak": (ctypes.c_int32, [ctypes.c_int32, ctypes.c_int64, ctypes.POINTER(ctypes.c_double),
+                                          ctypes.POINTER(ctypes.c_float)]),
     "vfl_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
 }
+PEAK_FFMA, PEAK_TF32_MMA = 0, 1
 
 _lib = None
 
@@ -255,6 +258,13 @@ def fit_power(x, t):
     c, e = ctypes.c_double(), ctypes.c_double()
     _check(lib().vfl_fit_power(_ptr(x), _ptr(t), len(x), ctypes.byref(c), ctypes.byref(e)))
     return c.value, e.value
+
+
+def measure_peak(kind: int, iters: int):
+    """(flop, ms) of one timed throughput launch (vfl_measure_peak) on the current device."""
+    f, ms = ctypes.c_double(), ctypes.c_float()
+    _check(lib().vfl_measure_peak(kind, iters, ctypes.byref(f), ctypes.byref(ms)))
+    return f.value, float(ms.value)
 
 
 def make_drops(seed: int, rate: float, n_steps: int):
