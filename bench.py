@@ -47,7 +47,8 @@ def parse(argv=None):
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=4, help="workload preset 1..5 (default 4, wide-dp)")
     ap.add_argument("--rows", type=int, default=0, help="override the preset's row count")
-    ap.add_argument("--workers", type=int, default=0, help="override the preset's worker streams per party")
+    ap.add_argument("--workers", type=int, default=0, help="worker streams per party (default: the preset's, or "
+                    "BENCH_WORKERS where the workload leaves them open)")
     ap.add_argument("--dp-target", choices=["grad", "emb"], default=None,
                     help="with DP: the published gradient (the preset's) or the published embedding (App. C)")
     ap.add_argument("--dp", type=float, nargs=2, default=None, metavar=("CLIP", "SIGMA"),
@@ -66,6 +67,11 @@ def parse(argv=None):
     return ap.parse_args(argv)
 
 
+# Worker streams per party (the paper's w_a = w_p) where the workload leaves them open: the count measured
+# fastest on GB300 (results do not depend on it: every step computes the same thing on any stream).
+BENCH_WORKERS = {3: 2, 4: 3}
+
+
 def workload(args):
     import synth
     p = synth.preset(args.config)
@@ -73,6 +79,8 @@ def workload(args):
         p = p.with_(n_rows=args.rows)
     if args.workers:
         p = p.with_(workers=args.workers)
+    elif args.config in BENCH_WORKERS and not args.ps_dt0:
+        p = p.with_(workers=BENCH_WORKERS[args.config])
     if args.dp:
         p = p.with_(dp_clip=args.dp[0], dp_sigma=args.dp[1])
     if args.dp_target:

@@ -504,8 +504,10 @@ void build_layers(vfl_ctx* ctx) {
                 const bool last_top = v == &ctx->T && l + 1 == v->size();
                 const bool concat = v == &ctx->T && l == 0;
                 if (!last_top && tc_shape_dw(L.out, L.in, concat, ea)) {
-                    // the cluster kernel reduces the batch on chip: one gradient, its bias column sums
-                    // and, with one worker stream per party (updates ordered by the stream), the SGD
+                    // the cluster kernel reduces the batch: one gradient, its bias column sums and, with one
+                    // worker stream per party, the SGD step (a step's first such kernel waits for the party's
+                    // previous update; with several workers that wait would hold every weight-gradient kernel
+                    // of the step back, so there the SGD stays a separate launch behind them)
                     L.tc_dw = true;
                     tc_choose_split(L.out, L.in, c.batch, &L.nsplit, &L.kchunk);
                     L.nsplit_b = 1;
@@ -756,7 +758,8 @@ vfl_status linear_fwd(vfl_ctx* ctx, const Layer& L, int slot, const void* X, lon
 //   dW[out, in] = dpre^T X, dpre [rows, out] (leading dim ldd, fp32 when dpre_f32).
 //   X may be [X1 | X2] split at column ka (then two GEMMs write the two column blocks).
 // On the tensor-core cluster kernel (L.tc_dw) the one reduced dW and db land in the partial buffers, and
-// with L.sgd_in_dw the same kernel applies the SGD step to replica `rep` and writes version slot `new_slot`.
+// with L.sgd_in_dw the same kernel applies the SGD step to replica `rep` and writes version slot `new_slot`
+// (the caller orders it after update k-1 of the party: wait_update_order before the step's first such kernel).
 vfl_status linear_dw(vfl_ctx* ctx, const Layer& L, int w, const void* dpre, long long ldd, bool dpre_f32,
                      const void* X, long long ldx, const void* X2, long long ldx2, int ka, int rows, cudaStream_t s,
                      int rep = 0, int new_slot = 0) {
@@ -1442,8 +1445,14 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     // slot the input gradient reads (tau_a = S), and the published gradient goes out first.
     const bool dp = c.dp_clip > 0.f && c.dp_target == VFL_DP_GRAD;
     const int rep = ps_rep(ctx, k), nslot = new_version_slot(ctx, k);
-    // SGD in step order (App. D): a weight-gradient kernel that applies it follows update k-1
-    if (ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, false, s));
+    // SGD in step order (App. D): the first weight-gradient kernel that applies it follows update k-1
+    // (the input gradients and the published gradient before it do not wait)
+    bool waited = false;
+    auto dw_order = [&]() -> vfl_status {
+        if (waited || !ctx->sgd_in_dw) return VFL_OK;
+        waited = true;
+        return wait_update_order(ctx, k, false, s);
+    };
     for (int l = Lf - 1; l >= 0; --l) {
         const Layer& L = ctx->T[l];
         const bool last = l == Lt - 1;
@@ -1453,6 +1462,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
             const long long ldo = ld8(ctx->T[l - 1].out);
             TRY(linear_dx(ctx, L, vslot, dpre, ldd, last, rows, ctx->dpre_t[w][l - 1], ldo, ctx->act_t[w][l - 1],
                           L.in, nullptr, 0, false, nullptr, s));
+            TRY(dw_order());
             TRY(linear_dw(ctx, L, w, dpre, ldd, last, ctx->act_t[w][l - 1], ld8(ctx->T[l - 1].out), nullptr, 0, 0,
                           rows, s, rep, nslot));
             continue;
@@ -1478,6 +1488,7 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
         CK(cudaEventRecord(ctx->ev_grad[k % kEvPool], s));
         ctx->grad_step[slot] = k;
         ctx->x_grad += (long long)rows * ep * ctx->esz;
+        TRY(dw_order());
         TRY(linear_dw(ctx, L, w, dpre, ldd, last, Za, ld8(ea), Zp, ld8(ep), ea, rows, s, rep, nslot));
     }
     // active bottom backward
@@ -1490,11 +1501,12 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
             TRY(linear_dx(ctx, L, vslot, ctx->dpre_a[w][l], ld8(L.out), false, rows, ctx->dpre_a[w][l - 1], ldo,
                           ctx->act_a[w][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
+        TRY(dw_order());
         TRY(linear_dw(ctx, L, w, ctx->dpre_a[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s, rep, nslot));
     }
     // SGD on theta_1 in step order: version k+1 from version k (the layers the weight-gradient kernels
     // did not update)
-    if (!ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, false, s));
+    if (!waited) TRY(wait_update_order(ctx, k, false, s));
     TRY(sgd(ctx, &ctx->A, &ctx->T, w, rep, nslot, s));
     CK(cudaEventRecord(ctx->ev_aver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, false, s));
@@ -1545,7 +1557,7 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
                              ctx->bf16, emb_dp(ctx) ? ctx->emb_c[slot] : nullptr, sub, s));
     const void* Xp0 = xp_rows(ctx, k, r0);
     const int rep = ps_rep(ctx, k), nslot = new_version_slot(ctx, k);
-    if (ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, true, s));
+    bool waited = false;
     for (int l = Lp - 1; l >= 0; --l) {
         const Layer& L = ctx->P[l];
         const void* Xin = l == 0 ? Xp0 : ctx->act_p[slot][l - 1];
@@ -1556,9 +1568,14 @@ vfl_status do_passive_backward(vfl_ctx* ctx, long long k) {
             TRY(linear_dx(ctx, L, vslot, ctx->dpre_p[w][l], ld8(L.out), false, rows, ctx->dpre_p[w][l - 1], ldo,
                           ctx->act_p[slot][l - 1], L.in, nullptr, 0, false, nullptr, s));
         }
+        // SGD in step order (App. D): the first weight-gradient kernel that applies it follows update k-1
+        if (ctx->sgd_in_dw && !waited) {
+            waited = true;
+            TRY(wait_update_order(ctx, k, true, s));
+        }
         TRY(linear_dw(ctx, L, w, ctx->dpre_p[w][l], ld8(L.out), false, Xin, ldin, nullptr, 0, 0, rows, s, rep, nslot));
     }
-    if (!ctx->sgd_in_dw) TRY(wait_update_order(ctx, k, true, s));
+    if (!waited) TRY(wait_update_order(ctx, k, true, s));
     TRY(sgd(ctx, &ctx->P, nullptr, w, rep, nslot, s));
     CK(cudaEventRecord(ctx->ev_pver[(k + 1) % kEvPool], s));
     if (ps_agg_at(ctx, k)) TRY(ps_average(ctx, k, true, s));
