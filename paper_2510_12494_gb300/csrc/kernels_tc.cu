@@ -82,10 +82,10 @@ struct GemmCfg : Ring<BN, BN == 256 ? 4 : 6> {
 
 // Weight gradient: 128-wide tiles, stages of 128 k rows (two MN-major boxes per operand: a stage's TMA
 // work covers two 64-row k-blocks), three stages; after the mainloop the ring holds the fp32
-// accumulator tile.  Column-sum scratch: 4 x 128 partials, 128 sums.
+// accumulator tile.  Column-sum scratch: 16 x 128 partials, 128 sums.
 struct DwCfg : Ring<128, 3, DW_KS> {
     using R = Ring<128, 3, DW_KS>;
-    static constexpr uint32_t CSUM_BYTES = (4 * 128 + 128) * 4;
+    static constexpr uint32_t CSUM_BYTES = (16 * 128 + 128) * 4;
     static constexpr size_t SMEM = 1024 + R::RING_BYTES + R::CTRL_BYTES + CSUM_BYTES;
     static_assert((size_t)128 * (128 + 4) * 4 <= R::RING_BYTES, "the accumulator tile must fit the ring");
 };
@@ -662,8 +662,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint64_t* acc_full = empty + C::STAGES;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 2);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-    float* csum_part = reinterpret_cast<float*>(ring + C::RING_BYTES + C::CTRL_BYTES);   // [4][128]
-    float* csum = csum_part + 4 * 128;                                                     // [128]
+    float* csum_part = reinterpret_cast<float*>(ring + C::RING_BYTES + C::CTRL_BYTES);   // [16][128]
+    float* csum = csum_part + 16 * 128;                                                    // [128]
 
     cg::cluster_group cluster = cg::this_cluster();
     const int cs = (int)cluster.num_blocks();
@@ -714,31 +714,32 @@ __global__ void __launch_bounds__(THREADS, 1)
         mma_commit(smem_u32(&acc_full[0]));
     } else if (warp >= 2 && bias) {
         // column sums of the A stages (D[rows, m] MN-major: two 64-column boxes of KS rows x 128 bytes,
-        // 16-byte chunks swizzled by row mod 8): thread e takes columns 2 (e mod 64), +1 over the
-        // KS/4-row quarter e / 64 of each stage
+        // 16-byte chunks swizzled by row mod 8): thread e takes the 8 columns of chunk e mod 16 over the
+        // rows r = e / 16 + 16 i of each stage, one 16-byte load a row
         const int e = threadIdx.x - 64;
-        const int mp = e & 63, kq = e >> 6;
-        const int mcol = 2 * mp, box = mcol >> 6, mb = mcol & 63;
-        constexpr int QR = C::KS / 4;
-        float s0 = 0.f, s1 = 0.f;
+        const int cg = e & 15, rg = e >> 4;
+        const int box = cg >> 3, c8 = cg & 7;
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         for (int kt = 0; kt < nk; ++kt) {
             const int s = kt % C::STAGES;
             if (!mbar_wait(smem_u32(&full[s]), (kt / C::STAGES) & 1, abort_flag)) break;
             const uint8_t* a = ring + s * C::STAGE_BYTES + box * C::BOX_BYTES;
-#pragma unroll 8
-            for (int r = kq * QR; r < kq * QR + QR; ++r) {
-                const uint32_t chunk = ((uint32_t)(mb >> 3) ^ (uint32_t)(r & 7));
-                const __nv_bfloat162 h =
-                    *reinterpret_cast<const __nv_bfloat162*>(a + r * 128 + (chunk << 4) + ((mb & 7) << 1));
-                const float2 f = __bfloat1622float2(h);
-                s0 += f.x;
-                s1 += f.y;
+#pragma unroll
+            for (int r = rg; r < C::KS; r += 16) {
+                const uint4 w = *reinterpret_cast<const uint4*>(a + r * 128 + ((c8 ^ (r & 7)) << 4));
+                const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 f = __bfloat1622float2(h[q]);
+                    acc[2 * q] += f.x;
+                    acc[2 * q + 1] += f.y;
+                }
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
         }
-        csum_part[kq * 128 + mcol] = s0;
-        csum_part[kq * 128 + mcol + 1] = s1;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) csum_part[rg * 128 + cg * 8 + q] = acc[q];
     }
     if (warp >= 2) {
         if (!mbar_wait(smem_u32(&acc_full[0]), 0, abort_flag)) {
@@ -746,9 +747,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     }
     __syncthreads();
-    if (bias && threadIdx.x < BM)
-        csum[threadIdx.x] = csum_part[threadIdx.x] + csum_part[128 + threadIdx.x] + csum_part[256 + threadIdx.x] +
-                            csum_part[384 + threadIdx.x];
+    if (bias && threadIdx.x < BM) {
+        float t = 0.f;
+        for (int g = 0; g < 16; ++g) t += csum_part[g * 128 + threadIdx.x];   // row groups in order
+        csum[threadIdx.x] = t;
+    }
 
     // the accumulator tile into shared memory (the ring is free: every MMA and every load is complete),
     // one row per thread
