@@ -35,8 +35,6 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "split-VFL training samples/sec at 1 GB300; % of roofline per kernel"
-FP32_ALU_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12   # SMs x FP32 lanes x FMA x max clock
-TF32_PER_BF16 = 1.1 / 2.25                               # nominal dense TF32 / BF16 tensor throughput
 
 
 def parse(argv=None):
@@ -267,84 +265,141 @@ def cpu_baseline(p, args, n_steps):
 # the GPU arm
 # --------------------------------------------------------------------------
 def peaks():
-    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    """Roofline denominators: HBM copy and bf16 GEMM from MEASURED_PEAKS.json, the FP32 FMA and TF32
+    warp-MMA peaks from profiles/peaks.json (python -m paper_2510_12494_gb300.peaks)."""
+    out = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
     try:
-        with open(path) as f:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             d = json.load(f)
-        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
-                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "src": "measured"}
+        out = {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+               "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "src": "measured"}
     except (OSError, KeyError, ValueError):
-        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
-
-
-# kernel class -> source file whose ncu counters the committed summaries hold
-KERNEL_SOURCES = {"fused_": "kernels_fused.cu", "gemm_tc": "kernels_tc.cu", "gemm_simt": "kernels_simt.cu"}
-
-
-def profiled_traffic(kernel, workload_name, launch_units):
-    """DRAM bytes per launch of `kernel` from a committed ncu summary in
-    profiles/, scaled to this launch's units; None when no summary matches or
-    the kernel's source changed since the counters were taken."""
-    import hashlib
-    src = next((f for pre, f in KERNEL_SOURCES.items() if kernel.startswith(pre)), None)
-    if src is None:
-        return None
-    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload_name}.md")
-    if not os.path.exists(path):
-        return None
-    meta = {}
-    with open(path) as f:
-        for line in f:
-            if line.startswith("- ") and ":" in line:
-                k, v = line[2:].split(":", 1)
-                meta[k.strip()] = v.strip().strip("`")
-    with open(os.path.join(ROOT, "paper_2510_12494_gb300", "csrc", src), "rb") as f:
-        digest = hashlib.sha256(f.read()).hexdigest()
-    if meta.get("source_sha256") != digest:
-        return None
+        pass
     try:
-        per_unit = float(meta["dram_bytes_per_launch"]) / float(meta["units_per_launch"])
-    except (KeyError, ValueError, ZeroDivisionError):
+        with open(os.path.join(ROOT, "profiles", "peaks.json")) as f:
+            d = json.load(f)
+        out["ffma_tflops"], out["x3tf32_tflops"] = d["fp32_ffma"]["tflops"], d["fp32_3xtf32_tflops"]
+        out["fp32_src"] = "measured"
+    except (OSError, KeyError, ValueError):
+        # nominal: 152 SMs x 128 FP32 lanes x 2 x 2070 MHz; TF32 at 1.1/2.25 of the bf16 peak, / 3 for 3xTF32
+        out["ffma_tflops"], out["x3tf32_tflops"] = 80.5, out["bf16_tflops_sustained"] * 1.1 / 2.25 / 3
+        out["fp32_src"] = "nominal"
+    return out
+
+
+# event class -> the kernel function that runs it (the launch list and the ncu captures are per function)
+KERNEL_OF_CLASS = {
+    "gemm_tc_fwd": "tc_gemm_kernel", "gemm_tc_dx": "tc_gemm_kernel", "gemm_tc_dw": "tc_dw_kernel",
+    "gemm_tc_dw_sgd": "tc_dw_kernel", "gemm_simt_fwd": "gemm_simt_kernel", "gemm_simt_dx": "gemm_simt_kernel",
+    "gemm_simt_dw": "gemm_simt_kernel", "head_loss": "head_kernel", "loss": "loss_kernel",
+    "dp_clip_noise": "dp_kernel", "relu_mask": "relu_mask_kernel", "sgd": "sgd_kernel",
+    "channel_header": "write_header_kernel", "cast": "cast_rows_kernel",
+    "fused_passive_fwd": "fused_passive_fwd_kernel", "fused_active_step": "fused_active_kernel",
+    "fused_passive_bwd": "fused_passive_bwd_kernel", "fused_update": "fused_update_kernel",
+    "ps_average": "ps_average_kernel"}
+KERNEL_SOURCE = {"tc_": "kernels_tc.cu", "fused_": "kernels_fused.cu"}   # everything else: kernels_simt.cu
+
+
+def file_digest(src):
+    import hashlib
+    with open(os.path.join(ROOT, "paper_2510_12494_gb300", "csrc", src), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def source_digest(kernel):
+    return file_digest(next((f for pre, f in KERNEL_SOURCE.items() if kernel.startswith(pre)), "kernels_simt.cu"))
+
+
+def profile_record(name):
+    try:
+        with open(os.path.join(ROOT, "profiles", name)) as f:
+            return json.load(f)
+    except (OSError, ValueError):
         return None
-    return per_unit * launch_units
+
+
+def profiled_traffic(kernel, classes, workload_name, launch_units):
+    """DRAM bytes (read + write) per launch of `kernel` from the committed ncu captures
+    (profiles/kernels.json): the captured launches of the same event classes on the same workload,
+    per unit, scaled to `launch_units`; None when nothing matches or the kernel's source has changed
+    since the counters were taken."""
+    rec = profile_record("kernels.json")
+    if not rec:
+        return None
+    for k in rec["kernels"]:
+        if k["kernel"] != kernel or k["workload"] != workload_name or k["source_sha256"] != source_digest(kernel):
+            continue
+        ls = [x for x in k["launches"] if x.get("class") in classes] or k["launches"]
+        dram = [(x["dram_read"] or 0) + (x["dram_write"] or 0) for x in ls]
+        per_unit = sum(dram) / len(dram) / k["units_per_launch"]
+        return {"bytes_per_launch": per_unit * launch_units, "captured_launches": len(ls),
+                "source": "profiles/" + k["file"]}
+    return None
+
+
+def launch_list_check(kernel, workload_name, flops_per_launch, bytes_per_launch, bound, peak):
+    """The dominant kernel seen from the committed ncu launch list of the same workload
+    (profiles/launches.json: serialised launches, kernel time only): its share of all kernel time,
+    whether it is the largest there too, and its roofline fraction on the launch list's warm duration."""
+    rec = profile_record("launches.json")
+    if not rec or workload_name not in rec.get("workloads", {}):
+        return None
+    w = rec["workloads"][workload_name]
+    stale = [f for f, h in w.get("sources_sha256", {}).items() if h != file_digest(f)]
+    ks = w["kernels"]
+    top = max(ks, key=lambda n: ks[n]["warm_share"])
+    me = ks.get(kernel)
+    out = {"largest_warm": top, "agrees": top == kernel, "stale_sources": stale, "command": w["command"]}
+    if me:
+        sec = me["warm_avg_us"] * 1e-6
+        ach = (flops_per_launch / sec / 1e12) if bound in ("tensor", "alu") else (bytes_per_launch / sec / 1e9)
+        out.update({"warm_share": me["warm_share"], "cold_share": me["cold_share"],
+                    "warm_avg_us": me["warm_avg_us"], "cold_avg_us": me["cold_avg_us"],
+                    "achieved": ach, "frac": ach / peak})
+    return out
 
 
 HOST_ENQUEUE_CYCLES = 1_000_000       # ~0.5 ms of GPU spin before each timed iteration (not timed)
 
 
-def roofline(prof, pk):
-    """Dominant kernel class (largest summed time) against its bound."""
+def roofline(prof, pk, workload_name, units):
+    """The dominant kernel (largest summed event time over its classes) against its bound.  Its
+    achieved rate is the algorithmic work per launch over the event-timed launch duration, and again
+    over the kernel-only duration of the committed ncu launch list."""
     if not prof:
         return None
-    name, (n, ms, flops, nbytes) = max(prof.items(), key=lambda kv: kv[1][1])
+    by_kernel = {}
+    for cls, (n, ms, flops, nbytes) in prof.items():
+        k = KERNEL_OF_CLASS.get(cls, cls)
+        a = by_kernel.setdefault(k, [0, 0.0, 0.0, 0.0, []])
+        a[0] += n; a[1] += ms; a[2] += flops; a[3] += nbytes; a[4].append(cls)
+    name, (n, ms, flops, nbytes, classes) = max(by_kernel.items(), key=lambda kv: kv[1][1])
     sec = ms / 1e3
-    tensor = name.startswith("gemm_tc")
-    tf32x3 = name.startswith("fused_")      # the fused kernels' contractions: 3xTF32 warp MMAs
-    if tensor:
-        peak = pk["bf16_tflops_sustained"]
-        ach = flops / sec / 1e12
-        bound, unit = "tensor", "TFLOP/s"
-    elif tf32x3:
+    if name.startswith("tc_"):
+        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
+        peak_src = f"{pk['src']} sustained bf16 GEMM"
+    elif name.startswith("fused_"):
         # fp32 contractions on the TF32 tensor path in 3xTF32 form: three TF32 products per fp32 one
-        peak = pk["bf16_tflops_sustained"] * TF32_PER_BF16 / 3.0
-        ach = flops / sec / 1e12
-        bound, unit = "tensor", "TFLOP/s"
+        bound, peak, unit = "tensor", pk["x3tf32_tflops"], "TFLOP/s"
+        peak_src = f"{pk['fp32_src']} TF32 warp-MMA peak / 3 (3xTF32)"
     else:
-        alu_peak = FP32_ALU_PEAK_TFLOPS
-        balance = alu_peak * 1e12 / (pk["hbm_gbs"] * 1e9)
-        compute_bound = flops > 0 and flops / max(nbytes, 1.0) > balance
-        if compute_bound:
-            peak, ach, bound, unit = alu_peak, flops / sec / 1e12, "alu", "TFLOP/s"
+        balance = pk["ffma_tflops"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+        if flops > 0 and flops / max(nbytes, 1.0) > balance:
+            bound, peak, unit = "alu", pk["ffma_tflops"], "TFLOP/s"
+            peak_src = f"{pk['fp32_src']} FFMA peak"
         else:
-            peak, ach, bound, unit = pk["hbm_gbs"], nbytes / sec / 1e9, "hbm", "GB/s"
-    return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
-            "traffic": None, "launches": n, "avg_us": ms / n * 1e3,
-            "peak_src": (f"{pk['src']} sustained bf16 GEMM" if tensor else
-                         f"{pk['src']} sustained bf16 GEMM x {TF32_PER_BF16:.4f} (nominal TF32/BF16) / 3 (3xTF32)"
-                         if tf32x3 else
-                         ("derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz" if bound == "alu"
-                          else f"{pk['src']} HBM copy")),
-            "all_classes_ms": {k: round(v[1], 4) for k, v in sorted(prof.items(), key=lambda kv: -kv[1][1])}}
+            bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
+            peak_src = f"{pk['src']} HBM copy"
+    ach = flops / sec / 1e12 if unit == "TFLOP/s" else nbytes / sec / 1e9
+    tr = profiled_traffic(name, classes, workload_name, units)
+    ll = launch_list_check(name, workload_name, flops / n, nbytes / n, "tensor" if unit == "TFLOP/s" else "hbm",
+                           peak)
+    return {"kernel": name, "classes": classes, "bound": bound, "achieved": ach, "peak": peak, "unit": unit,
+            "frac": ach / peak, "traffic": tr["bytes_per_launch"] if tr else None,
+            "traffic_source": tr, "algorithmic_per_launch": {"flops": flops / n, "bytes": nbytes / n},
+            "launches": n, "avg_us": ms / n * 1e3, "timing": "CUDA event pair around each launch, on its stream",
+            "peak_src": peak_src, "launch_list": ll,
+            "all_kernels_ms": {k: round(v[1], 4) for k, v in sorted(by_kernel.items(), key=lambda kv: -kv[1][1])}}
 
 
 def slowest_rank(x: float) -> float:
@@ -479,10 +534,8 @@ def run_ours(args):
     # per-kernel timing: the same workload again, every launch bracketed by CUDA events (recorded
     # inside the replayed graphs when graphs are on, so each duration is the kernel as the step runs it)
     _, prof = timed_block(W + K, K, profile=True)
-    roof = roofline(prof, peaks())
-    if roof:
-        # samples per launch of the dominant kernel: a fused kernel or GEMM processes one batch per launch
-        roof["traffic"] = profiled_traffic(roof["kernel"], p.name, p.batch)
+    # units per launch of the dominant kernel: every kernel of the step processes one batch per launch
+    roof = roofline(prof, peaks(), p.name, p.batch)
 
     # end to end through the public API with host buffers: the dataset stays in pinned host memory,
     # every step copies its rows in and its loss out (vfl_bind_host_data) inside the timed region

@@ -119,12 +119,30 @@ __global__ void __launch_bounds__(NT) gemm_simt_kernel(const GemmArgs g) {
     header_publish(g.hdr);
 }
 
+// Every kernel of the library asks for the shared-memory-heavy split of the SM's L1 / shared storage that
+// the tcgen05 and fused kernels need: kernels of both kinds alternate within a step, and an SM whose split
+// changes between two kernels has to drain before the next one starts.  Set once per kernel, on its first
+// launch.
+template <typename F>
+inline bool prefer_shared_split(F* kernel) {
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                (int)cudaSharedmemCarveoutMaxShared) == cudaSuccess;
+}
+#define SHARED_SPLIT(k)                                          \
+    do {                                                         \
+        static const bool split_set_ = prefer_shared_split(k);  \
+        (void)split_set_;                                        \
+    } while (0)
+
 template <typename TA, typename TB>
 cudaError_t gemm_dispatch_mask(const GemmArgs& g, int mask_bf16, dim3 grid, cudaStream_t s) {
-    if (mask_bf16)
+    if (mask_bf16) {
+        SHARED_SPLIT((gemm_simt_kernel<TA, TB, __nv_bfloat16>));
         gemm_simt_kernel<TA, TB, __nv_bfloat16><<<grid, NT, 0, s>>>(g);
-    else
+    } else {
+        SHARED_SPLIT((gemm_simt_kernel<TA, TB, float>));
         gemm_simt_kernel<TA, TB, float><<<grid, NT, 0, s>>>(g);
+    }
     return cudaGetLastError();
 }
 
@@ -736,6 +754,7 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, int a_bf16, int b_bf16, int mask
 
 cudaError_t launch_loss(const float* logits, const int* y, int rows, int n_out, int loss_kind, float* ds,
                         float* loss_out, float* loss_host, cudaStream_t s) {
+    SHARED_SPLIT(loss_kernel);
     loss_kernel<<<1, LOSS_NT, 0, s>>>(logits, y, rows, n_out, loss_kind, ds, loss_out, loss_host);
     return cudaGetLastError();
 }
@@ -744,6 +763,7 @@ cudaError_t launch_head(const HeadArgs& a, cudaStream_t s) {
     if (a.rows < 1 || a.nout < 1 || a.nout > kHeadMaxOut || a.K < 8 || a.K > kHeadMaxK || (a.K & 7) ||
         a.nblk < head_blocks(a.rows))
         return cudaErrorInvalidValue;
+    SHARED_SPLIT(head_kernel);
     head_kernel<<<a.nblk, HEAD_NT, 0, s>>>(a);
     return cudaGetLastError();
 }
@@ -751,6 +771,7 @@ cudaError_t launch_head(const HeadArgs& a, cudaStream_t s) {
 cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_out, int out_bf16, int rows, int e,
                       float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
+    SHARED_SPLIT(dp_kernel);
     dp_kernel<<<(rows + DP_ROWS - 1) / DP_ROWS, DP_NT, 0, s>>>(in, ld_in, out, ld_out, out_bf16, rows, e, clip, sigma,
                                                                seed, k, (float)rows);
     return cudaGetLastError();
@@ -759,20 +780,24 @@ cudaError_t launch_dp(const float* in, long long ld_in, void* out, long long ld_
 cudaError_t launch_relu_mask(const void* g, const void* z, void* out, long long ld, int rows, int e, int bf16,
                              const float* row_scale, const HeaderOps& hdr, cudaStream_t s) {
     const int nb = grid_for((long long)rows * ((e + 3) / 4), 256);
-    if (bf16)
+    if (bf16) {
+        SHARED_SPLIT(relu_mask_kernel<__nv_bfloat16>);
         relu_mask_kernel<__nv_bfloat16><<<nb, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(g),
                                                            static_cast<const __nv_bfloat16*>(z),
                                                            static_cast<__nv_bfloat16*>(out), ld, rows, e, row_scale,
                                                            hdr);
-    else
+    } else {
+        SHARED_SPLIT(relu_mask_kernel<float>);
         relu_mask_kernel<float><<<nb, 256, 0, s>>>(static_cast<const float*>(g), static_cast<const float*>(z),
                                                    static_cast<float*>(out), ld, rows, e, row_scale, hdr);
+    }
     return cudaGetLastError();
 }
 
 cudaError_t launch_dp_emb(const void* z, long long ld, int bf16, void* out, float* scale_out, int rows, int e,
                           float clip, float sigma, unsigned long long seed, long long k, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
+    SHARED_SPLIT(dp_emb_kernel);
     dp_emb_kernel<<<(rows + DP_ROWS - 1) / DP_ROWS, DP_NT, 0, s>>>(z, ld, bf16, out, scale_out, rows, e, clip, sigma,
                                                                    seed, k);
     return cudaGetLastError();
@@ -789,6 +814,7 @@ cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
         most = std::max(most, warp ? np * 32 : np);
     }
     const long long bx = std::min<long long>((most + 255) / 256, std::max(1, 152 * 8 / a.n_layers));
+    SHARED_SPLIT(sgd_kernel);
     sgd_kernel<<<dim3((unsigned)bx, a.n_layers), 256, 0, s>>>(a);
     return cudaGetLastError();
 }
@@ -796,32 +822,38 @@ cudaError_t launch_sgd(const SgdArgs& a, cudaStream_t s) {
 cudaError_t launch_ps_average(const PsAvgLayer* tab, int n_layers, long long total, int nrep, int c_bf16,
                               cudaStream_t s) {
     if (total <= 0) return cudaSuccess;
+    SHARED_SPLIT(ps_average_kernel);
     ps_average_kernel<<<grid_for(total, 256), 256, 0, s>>>(tab, n_layers, total, nrep, c_bf16);
     return cudaGetLastError();
 }
 
 cudaError_t launch_mark_dropped(float* loss, float* loss_host, cudaStream_t s) {
+    SHARED_SPLIT(mark_dropped_kernel);
     mark_dropped_kernel<<<1, 1, 0, s>>>(loss, loss_host);
     return cudaGetLastError();
 }
 
 cudaError_t launch_write_header(ChannelHeader* h, long long k, int batch, int version, cudaStream_t s) {
+    SHARED_SPLIT(write_header_kernel);
     write_header_kernel<<<1, 1, 0, s>>>(h, k, batch, version);
     return cudaGetLastError();
 }
 
 cudaError_t launch_check_header(const ChannelHeader* h, long long k, int* status, cudaStream_t s) {
+    SHARED_SPLIT(check_header_kernel);
     check_header_kernel<<<1, 1, 0, s>>>(h, k, status);
     return cudaGetLastError();
 }
 
 cudaError_t launch_wait_header(const ChannelHeader* h, long long k, long long max_iters, int* status, cudaStream_t s) {
+    SHARED_SPLIT(wait_header_kernel);
     wait_header_kernel<<<1, 1, 0, s>>>(h, k, max_iters, status);
     return cudaGetLastError();
 }
 
 cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long long ld, int bf16, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
+    SHARED_SPLIT(cast_rows_kernel);
     cast_rows_kernel<<<grid_for((long long)rows * ld, 256), 256, 0, s>>>(src, rows, d, dst, ld, bf16);
     return cudaGetLastError();
 }
@@ -830,6 +862,7 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
                               long long ld_p, void* xa, long long ld_a, int* y, int bf16, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     const long long n = (long long)rows * (ld_p + ld_a + 1);
+    SHARED_SPLIT(stage_rows_kernel);
     stage_rows_kernel<<<grid_for(n, 256), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, xp, ld_p, xa, ld_a, y, bf16);
     return cudaGetLastError();
 }
@@ -837,6 +870,7 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
 
 cudaError_t launch_to_f32(const void* src, long long ld, int rows, int cols, int bf16, float* dst, cudaStream_t s) {
     if (rows <= 0 || cols <= 0) return cudaSuccess;
+    SHARED_SPLIT(to_f32_kernel);
     to_f32_kernel<<<grid_for((long long)rows * cols, 256), 256, 0, s>>>(src, ld, rows, cols, bf16, dst);
     return cudaGetLastError();
 }

@@ -357,28 +357,69 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int m, int nba
 // instruction writes eight full 64-byte pieces of rows.  Two rows share a 128-byte line; the line's
 // eight 16-byte units are XOR-swizzled by the line index, so both directions are conflict-free.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint4* stage_unit(uint8_t* stage, int r, int ch) {
+__device__ __forceinline__ uint32_t stage_unit(uint32_t stage, int r, int ch) {
     const int line = r >> 1;
     const int unit = (((r & 1) << 2) | ch) ^ (line & 7);
-    return reinterpret_cast<uint4*>(stage + line * 128 + unit * 16);
+    return stage + (uint32_t)(line * 128 + unit * 16);
+}
+__device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+}
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
+    return v;
+}
+
+// The bf16 ReLU mask an input-gradient pass of 32 columns from nb applies, with its row stride and first
+// column (masks share the layout of the matrix they gate); null for forward, fp32-output or straddling passes.
+__device__ __forceinline__ const __nv_bfloat16* dx_pass_mask(const TcParams& p, int nb, long long* ld, int* n) {
+    if (p.mode == GEMM_FWD || nb >= p.N) return nullptr;
+    const int cols = min(32, p.N - nb);
+    if (nb + cols <= p.n_split) {
+        *ld = p.ldc;
+        *n = nb;
+        return static_cast<const __nv_bfloat16*>(p.mask1);
+    }
+    if (nb >= p.n_split && ((nb - p.n_split) & 7) == 0 && !p.c2_f32) {
+        *ld = p.ldc2;
+        *n = nb - p.n_split;
+        return static_cast<const __nv_bfloat16*>(p.mask2);
+    }
+    return nullptr;
+}
+
+// This lane's four 8-column mask units of a 32 x 32 block (the units store_bf16_block writes), read
+// ahead of the stores so that their latency overlaps the accumulator wait or the previous pass.
+__device__ __forceinline__ void load_mask_block(const __nv_bfloat16* mask, long long ld, int lane, int r0, int rows,
+                                                int n, int cols, uint4 (&mk)[4]) {
+    const int c = (lane & 3) * 8;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = i * 8 + (lane >> 2);
+        mk[i] = make_uint4(0u, 0u, 0u, 0u);
+        if (mask && r0 + r < rows && c + 8 <= cols)
+            mk[i] = __ldg(reinterpret_cast<const uint4*>(mask + (long long)(r0 + r) * ld + n + c));
+    }
 }
 
 // Read back the staged 32 x 32 bf16 block and store rows [r0, r0 + 32) x columns [n, n + 32) of a bf16
-// matrix (row stride ld, `cols` valid columns from n), masked by mask[idx] > 0 when mask is set.
-__device__ __forceinline__ void store_bf16_block(uint8_t* stage, int lane, __nv_bfloat16* C, long long ld,
-                                                 const __nv_bfloat16* mask, int r0, int rows, int n, int cols) {
+// matrix (row stride ld, `cols` valid columns from n), masked by mask > 0 when mask is set: full 8-column
+// units take the mask from mk (load_mask_block), a ragged last unit reads it element by element.
+__device__ __forceinline__ void store_bf16_block(uint32_t stage, int lane, __nv_bfloat16* C, long long ld,
+                                                 const __nv_bfloat16* mask, const uint4 (&mk)[4], int r0, int rows,
+                                                 int n, int cols) {
     const int ch = lane & 3;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int r = i * 8 + (lane >> 2);
         if (r0 + r >= rows) continue;
-        uint4 d = *stage_unit(stage, r, ch);
+        uint4 d = lds128(stage_unit(stage, r, ch));
         const int c = ch * 8;
         const long long idx = (long long)(r0 + r) * ld + n + c;
         if (c + 8 <= cols) {
             if (mask) {
-                const uint4 mk = *reinterpret_cast<const uint4*>(mask + idx);
-                const uint32_t mw[4] = {mk.x, mk.y, mk.z, mk.w};
+                const uint32_t mw[4] = {mk[i].x, mk[i].y, mk[i].z, mk[i].w};
                 uint32_t dw[4] = {d.x, d.y, d.z, d.w};
 #pragma unroll
                 for (int h = 0; h < 4; ++h) {
@@ -401,18 +442,20 @@ __device__ __forceinline__ void store_bf16_block(uint8_t* stage, int lane, __nv_
 
 // The same for 16 fp32 columns per pass (64 bytes a row): v[16] of row `lane` into the staging buffer,
 // then rows [r0, r0 + 32) x columns [n, n + 16) of an fp32 matrix, masked by a bf16 mask when set.
-__device__ __forceinline__ void store_f32_block(uint8_t* stage, int lane, const float* v, float* C, long long ld,
+__device__ __forceinline__ void store_f32_block(uint32_t stage, int lane, const float* v, float* C, long long ld,
                                                 const __nv_bfloat16* mask, int r0, int rows, int n, int cols) {
 #pragma unroll
     for (int c = 0; c < 4; ++c)
-        *reinterpret_cast<float4*>(stage_unit(stage, lane, c)) = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+        sts128(stage_unit(stage, lane, c), make_uint4(__float_as_uint(v[4 * c]), __float_as_uint(v[4 * c + 1]),
+                                                      __float_as_uint(v[4 * c + 2]), __float_as_uint(v[4 * c + 3])));
     __syncwarp();
     const int ch = lane & 3;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int r = i * 8 + (lane >> 2);
         if (r0 + r >= rows) continue;
-        const float4 d = *reinterpret_cast<const float4*>(stage_unit(stage, r, ch));
+        const uint4 du = lds128(stage_unit(stage, r, ch));
+        const float4 d = make_float4(__uint_as_float(du.x), __uint_as_float(du.y), __uint_as_float(du.z), __uint_as_float(du.w));
         const int c = ch * 4;
         const long long idx = (long long)(r0 + r) * ld + n + c;
         float dv[4] = {d.x, d.y, d.z, d.w};
@@ -500,7 +543,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int quarter = warp & 3;            // TMEM lanes this warp may read
         const int half = (warp - 2) >> 2;        // column half of the tile
         const int cbeg = half * (BN / 2);
-        uint8_t* stage = ring + C::RING_BYTES + C::CTRL_BYTES + (warp - 2) * C::WARP_BYTES;
+        const uint32_t stage = smem_u32(ring + C::RING_BYTES + C::CTRL_BYTES + (warp - 2) * C::WARP_BYTES);
         int i = 0;
         for (int t = blockIdx.x; t < ntiles && nk > 0; t += gridDim.x, ++i) {
             const int b = i & 1;
@@ -513,14 +556,37 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int n = n0 + cbeg + 32 * q + lane;
                 bias[q] = p.mode == GEMM_FWD && n < p.N ? __ldg(p.bias + n) : 0.f;
             }
+            const int r0 = m0 + quarter * 32;
+            // input gradient: the ReLU mask of pass 0 is read while the MMAs run, that of pass q + 1 while
+            // pass q is stored
+            uint4 mk[4];
+            {
+                long long mld = 0;
+                int mn = 0;
+                const __nv_bfloat16* mp = dx_pass_mask(p, n0 + cbeg, &mld, &mn);
+                load_mask_block(mp, mld, lane, r0, p.M, mn, min(32, p.N - (n0 + cbeg)), mk);
+            }
             if (!mbar_wait(smem_u32(&acc_full[b]), (i >> 1) & 1, abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const int r0 = m0 + quarter * 32;
-#pragma unroll
+            // one copy of the pass body, run BN / 64 times: the epilogue's code stays small enough to be
+            // resident in the instruction cache after the first pass
+#pragma unroll 1
             for (int q = 0; q < BN / 64; ++q) {
                 const int c0 = cbeg + 32 * q;
                 float v[32];
                 tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * BN + c0), v);
+                float bq = bias[0];
+#pragma unroll
+                for (int z = 1; z < BN / 64; ++z)
+                    if (q == z) bq = bias[z];
+                const uint4 cur[4] = {mk[0], mk[1], mk[2], mk[3]};
+                if (q + 1 < BN / 64) {
+                    long long mld = 0;
+                    int mn = 0;
+                    const int nn = n0 + c0 + 32;
+                    const __nv_bfloat16* mp = dx_pass_mask(p, nn, &mld, &mn);
+                    load_mask_block(mp, mld, lane, r0, p.M, mn, min(32, p.N - nn), mk);
+                }
                 const int nb = n0 + c0;
                 if (__any_sync(0xffffffffu, *abort_flag != 0) || nb >= p.N) continue;
                 const int cols = min(32, p.N - nb);
@@ -528,8 +594,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     uint32_t u[16];
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        float x0 = v[2 * j] + __shfl_sync(0xffffffffu, bias[q], 2 * j);
-                        float x1 = v[2 * j + 1] + __shfl_sync(0xffffffffu, bias[q], 2 * j + 1);
+                        float x0 = v[2 * j] + __shfl_sync(0xffffffffu, bq, 2 * j);
+                        float x1 = v[2 * j + 1] + __shfl_sync(0xffffffffu, bq, 2 * j + 1);
                         if (p.relu) {
                             x0 = fmaxf(x0, 0.f);
                             x1 = fmaxf(x1, 0.f);
@@ -538,29 +604,31 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
 #pragma unroll
                     for (int c = 0; c < 4; ++c)
-                        *stage_unit(stage, lane, c) = make_uint4(u[4 * c], u[4 * c + 1], u[4 * c + 2], u[4 * c + 3]);
+                        sts128(stage_unit(stage, lane, c), make_uint4(u[4 * c], u[4 * c + 1], u[4 * c + 2], u[4 * c + 3]));
                     __syncwarp();
-                    store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(p.C), p.ldc, nullptr, r0, p.M, nb, cols);
+                    store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(p.C), p.ldc, nullptr, cur, r0, p.M, nb,
+                                     cols);
                     __syncwarp();
                 } else if (nb + cols <= p.n_split || (nb >= p.n_split && ((nb - p.n_split) & 7) == 0)) {
                     // the input gradient: columns < n_split to C (masked by mask1), the rest to C2
                     const bool to_c = nb < p.n_split;
-                    const __nv_bfloat16* mk = static_cast<const __nv_bfloat16*>(to_c ? p.mask1 : p.mask2);
+                    const __nv_bfloat16* mk_ptr = static_cast<const __nv_bfloat16*>(to_c ? p.mask1 : p.mask2);
                     if (!to_c && p.c2_f32) {
-                        store_f32_block(stage, lane, v, static_cast<float*>(p.C2), p.ldc2, mk, r0, p.M,
+                        store_f32_block(stage, lane, v, static_cast<float*>(p.C2), p.ldc2, mk_ptr, r0, p.M,
                                         nb - p.n_split, min(16, cols));
                         if (cols > 16)
-                            store_f32_block(stage, lane, v + 16, static_cast<float*>(p.C2), p.ldc2, mk, r0, p.M,
+                            store_f32_block(stage, lane, v + 16, static_cast<float*>(p.C2), p.ldc2, mk_ptr, r0, p.M,
                                             nb + 16 - p.n_split, cols - 16);
                     } else {
 #pragma unroll
                         for (int c = 0; c < 4; ++c)
-                            *stage_unit(stage, lane, c) =
-                                make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                                           pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+                            sts128(stage_unit(stage, lane, c),
+                                   make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                              pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7])));
                         __syncwarp();
                         store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2),
-                                         to_c ? p.ldc : p.ldc2, mk, r0, p.M, to_c ? nb : nb - p.n_split, cols);
+                                         to_c ? p.ldc : p.ldc2, mk_ptr, cur, r0, p.M,
+                                         to_c ? nb : nb - p.n_split, cols);
                         __syncwarp();
                     }
                 } else if (r0 + lane < p.M) {
@@ -877,6 +945,8 @@ int sm_count() {
 template <typename K>
 cudaError_t set_smem(K kernel, size_t bytes, bool cluster) {
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
     if (e == cudaSuccess && cluster) e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     return e;
 }
