@@ -8,9 +8,9 @@
 //   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = BN, K = 16)
 //              from one thread; tcgen05.commit frees each stage and, after a
 //              tile's last k-block, marks its accumulator full
-//   warps 2-9  epilogue: tcgen05.ld of their 32-lane quarter and column half,
+//   warps 2-17 epilogue: tcgen05.ld of their 32-lane quarter and column quarter,
 //              fused bias + ReLU (forward) or ReLU-mask + column split (input
-//              gradient), bf16 rows straight to global memory
+//              gradient), staged in shared memory and stored as row segments
 // Two accumulators live in TMEM (2 x BN columns), so the epilogue of one tile
 // runs while the MMAs of the next tile fill the other.
 //
@@ -49,8 +49,10 @@ namespace vfl {
 namespace {
 
 constexpr int BM = 128, BK = 64;                          // K-major stages: 64 k (one 128-byte row)
-constexpr int EPI_WARPS = 8;
+constexpr int EPI_WARPS = 8;                              // weight gradient: epilogue / column-sum warps
 constexpr int THREADS = 64 + 32 * EPI_WARPS;             // producer, MMA issuer, epilogue
+constexpr int GEMM_EPI_WARPS = 16;                        // forward / input gradient: four per TMEM lane quarter
+constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
 constexpr int DW_KS = 128;                                // weight-gradient stages: 128 k (MN-major boxes)
 constexpr long long WAIT_LIMIT = 1ll << 26;               // polls before a wait is declared hung
 constexpr int MAX_CLUSTER = 16;
@@ -77,7 +79,7 @@ template <int BN>
 struct GemmCfg : Ring<BN, BN == 256 ? 4 : 6> {
     using R = Ring<BN, BN == 256 ? 4 : 6>;
     static constexpr uint32_t WARP_BYTES = 2048;
-    static constexpr size_t SMEM = 1024 + R::RING_BYTES + R::CTRL_BYTES + EPI_WARPS * WARP_BYTES;
+    static constexpr size_t SMEM = 1024 + R::RING_BYTES + R::CTRL_BYTES + GEMM_EPI_WARPS * WARP_BYTES;
 };
 
 // Weight gradient: 128-wide tiles, stages of 128 k rows (two MN-major boxes per operand: a stage's TMA
@@ -158,6 +160,19 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
     return false;
 }
 
+// The same for a wait that spans a whole mainloop (epilogue warps waiting for a tile's MMAs): a short
+// sleep between polls leaves the issue slots and the shared-memory pipe to the producer and the MMA
+// issuer.  Bounded like mbar_wait (about a second of sleeping).
+__device__ __forceinline__ bool mbar_wait_idle(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+    for (long long it = 0; it < (WAIT_LIMIT >> 3); ++it) {
+        if (mbar_try(bar, parity)) return true;
+        if (*abort_flag) return false;
+        __nanosleep(128);
+    }
+    *abort_flag = 1;
+    return false;
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -215,6 +230,17 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
 // bf16 bit pattern h (low 16 bits) is > 0: positive, non-zero, not NaN
 __device__ __forceinline__ bool bf16_positive(uint32_t h) {
     return !(h & 0x8000u) && (h & 0x7FFFu) != 0 && (h & 0x7FFFu) <= 0x7F80u;
+}
+
+// Per 16-bit half of a bf16x2 word: 0xFFFF where that bf16 is > 0 (non-zero magnitude, sign clear, not
+// NaN), else 0 -- bf16_positive for both halves at once, without branches.  Magnitudes are at most
+// 0x7FFF, so neither addition carries out of its half.
+__device__ __forceinline__ uint32_t bf16x2_positive_mask(uint32_t w) {
+    const uint32_t m = w & 0x7FFF7FFFu;
+    const uint32_t nonzero = (m + 0x7FFF7FFFu) & 0x80008000u;
+    const uint32_t nan = (m + 0x007F007Fu) & 0x80008000u;
+    const uint32_t keep = nonzero & ~nan & ~w & 0x80008000u;
+    return (keep >> 15) * 0xFFFFu;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -419,14 +445,10 @@ __device__ __forceinline__ void store_bf16_block(uint32_t stage, int lane, __nv_
         const long long idx = (long long)(r0 + r) * ld + n + c;
         if (c + 8 <= cols) {
             if (mask) {
-                const uint32_t mw[4] = {mk[i].x, mk[i].y, mk[i].z, mk[i].w};
-                uint32_t dw[4] = {d.x, d.y, d.z, d.w};
-#pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    if (!bf16_positive(mw[h] & 0xFFFFu)) dw[h] &= 0xFFFF0000u;
-                    if (!bf16_positive(mw[h] >> 16)) dw[h] &= 0x0000FFFFu;
-                }
-                d = make_uint4(dw[0], dw[1], dw[2], dw[3]);
+                d.x &= bf16x2_positive_mask(mk[i].x);
+                d.y &= bf16x2_positive_mask(mk[i].y);
+                d.z &= bf16x2_positive_mask(mk[i].z);
+                d.w &= bf16x2_positive_mask(mk[i].w);
             }
             *reinterpret_cast<uint4*>(C + idx) = d;
         } else {
@@ -473,7 +495,7 @@ __device__ __forceinline__ void store_f32_block(uint32_t stage, int lane, const 
 // Persistent forward / input-gradient GEMM.
 // ---------------------------------------------------------------------------
 template <int BN>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap ta2,
                    const __grid_constant__ CUtensorMap tb, const TcParams p) {
     using C = GemmCfg<BN>;
@@ -497,7 +519,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
-            mbar_init(smem_u32(&acc_empty[b]), EPI_WARPS);
+            mbar_init(smem_u32(&acc_empty[b]), GEMM_EPI_WARPS);
         }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -540,53 +562,38 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
     } else if (warp >= 2) {
         // ---------------- epilogue ----------------
-        const int quarter = warp & 3;            // TMEM lanes this warp may read
-        const int half = (warp - 2) >> 2;        // column half of the tile
-        const int cbeg = half * (BN / 2);
+        // 16 warps: warp w reads TMEM lane quarter w mod 4 (the only lanes it may access) and one quarter
+        // of the tile's columns, NP passes of 32
+        constexpr int NP = BN / 128;
+        const int quarter = warp & 3;
+        const int group = (warp - 2) >> 2;
+        const int cbeg = group * (BN / 4);
         const uint32_t stage = smem_u32(ring + C::RING_BYTES + C::CTRL_BYTES + (warp - 2) * C::WARP_BYTES);
         int i = 0;
         for (int t = blockIdx.x; t < ntiles && nk > 0; t += gridDim.x, ++i) {
             const int b = i & 1;
             const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
-            // this warp's columns' bias (lane j of pass q holds column cbeg + 32 q + j), loaded while the
-            // tile's MMAs run
-            float bias[BN / 64];
-#pragma unroll
-            for (int q = 0; q < BN / 64; ++q) {
-                const int n = n0 + cbeg + 32 * q + lane;
-                bias[q] = p.mode == GEMM_FWD && n < p.N ? __ldg(p.bias + n) : 0.f;
-            }
             const int r0 = m0 + quarter * 32;
-            // input gradient: the ReLU mask of pass 0 is read while the MMAs run, that of pass q + 1 while
-            // pass q is stored
-            uint4 mk[4];
-            {
+            // read while the tile's MMAs run: this warp's columns' bias (lane j of pass q holds column
+            // cbeg + 32 q + j) and, for the input gradient, the ReLU masks of its passes
+            float bias[NP];
+            uint4 mk[NP][4];
+#pragma unroll
+            for (int q = 0; q < NP; ++q) {
+                const int nq = n0 + cbeg + 32 * q;
+                bias[q] = p.mode == GEMM_FWD && nq + lane < p.N ? __ldg(p.bias + nq + lane) : 0.f;
                 long long mld = 0;
                 int mn = 0;
-                const __nv_bfloat16* mp = dx_pass_mask(p, n0 + cbeg, &mld, &mn);
-                load_mask_block(mp, mld, lane, r0, p.M, mn, min(32, p.N - (n0 + cbeg)), mk);
+                const __nv_bfloat16* mp = dx_pass_mask(p, nq, &mld, &mn);
+                load_mask_block(mp, mld, lane, r0, p.M, mn, min(32, p.N - nq), mk[q]);
             }
-            if (!mbar_wait(smem_u32(&acc_full[b]), (i >> 1) & 1, abort_flag)) break;
+            if (!mbar_wait_idle(smem_u32(&acc_full[b]), (i >> 1) & 1, abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            // one copy of the pass body, run BN / 64 times: the epilogue's code stays small enough to be
-            // resident in the instruction cache after the first pass
-#pragma unroll 1
-            for (int q = 0; q < BN / 64; ++q) {
+#pragma unroll
+            for (int q = 0; q < NP; ++q) {
                 const int c0 = cbeg + 32 * q;
                 float v[32];
                 tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * BN + c0), v);
-                float bq = bias[0];
-#pragma unroll
-                for (int z = 1; z < BN / 64; ++z)
-                    if (q == z) bq = bias[z];
-                const uint4 cur[4] = {mk[0], mk[1], mk[2], mk[3]};
-                if (q + 1 < BN / 64) {
-                    long long mld = 0;
-                    int mn = 0;
-                    const int nn = n0 + c0 + 32;
-                    const __nv_bfloat16* mp = dx_pass_mask(p, nn, &mld, &mn);
-                    load_mask_block(mp, mld, lane, r0, p.M, mn, min(32, p.N - nn), mk);
-                }
                 const int nb = n0 + c0;
                 if (__any_sync(0xffffffffu, *abort_flag != 0) || nb >= p.N) continue;
                 const int cols = min(32, p.N - nb);
@@ -594,8 +601,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     uint32_t u[16];
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        float x0 = v[2 * j] + __shfl_sync(0xffffffffu, bq, 2 * j);
-                        float x1 = v[2 * j + 1] + __shfl_sync(0xffffffffu, bq, 2 * j + 1);
+                        float x0 = v[2 * j] + __shfl_sync(0xffffffffu, bias[q], 2 * j);
+                        float x1 = v[2 * j + 1] + __shfl_sync(0xffffffffu, bias[q], 2 * j + 1);
                         if (p.relu) {
                             x0 = fmaxf(x0, 0.f);
                             x1 = fmaxf(x1, 0.f);
@@ -606,8 +613,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int c = 0; c < 4; ++c)
                         sts128(stage_unit(stage, lane, c), make_uint4(u[4 * c], u[4 * c + 1], u[4 * c + 2], u[4 * c + 3]));
                     __syncwarp();
-                    store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(p.C), p.ldc, nullptr, cur, r0, p.M, nb,
-                                     cols);
+                    store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(p.C), p.ldc, nullptr, mk[q], r0, p.M,
+                                     nb, cols);
                     __syncwarp();
                 } else if (nb + cols <= p.n_split || (nb >= p.n_split && ((nb - p.n_split) & 7) == 0)) {
                     // the input gradient: columns < n_split to C (masked by mask1), the rest to C2
@@ -627,7 +634,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                               pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7])));
                         __syncwarp();
                         store_bf16_block(stage, lane, static_cast<__nv_bfloat16*>(to_c ? p.C : p.C2),
-                                         to_c ? p.ldc : p.ldc2, mk_ptr, cur, r0, p.M,
+                                         to_c ? p.ldc : p.ldc2, mk_ptr, mk[q], r0, p.M,
                                          to_c ? nb : nb - p.n_split, cols);
                         __syncwarp();
                     }
@@ -810,7 +817,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int q = 0; q < 8; ++q) csum_part[rg * 128 + cg * 8 + q] = acc[q];
     }
     if (warp >= 2) {
-        if (!mbar_wait(smem_u32(&acc_full[0]), 0, abort_flag)) {
+        if (!mbar_wait_idle(smem_u32(&acc_full[0]), 0, abort_flag)) {
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     }
@@ -1183,9 +1190,9 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
     const long long tiles = (long long)p.tiles_m * p.tiles_n;
     const int grid = (int)std::min<long long>(tiles, sms);
     if (bn == 256)
-        tc_gemm_kernel<256><<<grid, THREADS, GemmCfg<256>::SMEM, s>>>(ta, ta2, tb, p);
+        tc_gemm_kernel<256><<<grid, GEMM_THREADS, GemmCfg<256>::SMEM, s>>>(ta, ta2, tb, p);
     else
-        tc_gemm_kernel<128><<<grid, THREADS, GemmCfg<128>::SMEM, s>>>(ta, ta2, tb, p);
+        tc_gemm_kernel<128><<<grid, GEMM_THREADS, GemmCfg<128>::SMEM, s>>>(ta, ta2, tb, p);
     return cudaGetLastError();
 }
 
