@@ -203,11 +203,14 @@ __global__ void __launch_bounds__(LOSS_NT) loss_kernel(const float* __restrict__
 constexpr int HEAD_NT = 256;
 static_assert(kHeadMaxK == 32 * 8 && kHeadMaxOut <= 2 * (HEAD_NT / 32), "head thread map");
 
+// NOUT: the output width the kernel is compiled for (1 for the BCE head, kHeadMaxOut otherwise); the
+// arrays sized by it stay in registers, and the single-logit kernel needs far fewer of them.
+template <int NOUT>
 __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
     pdl_entry();
-    __shared__ float Ws[kHeadMaxOut * kHeadMaxK];          // lane-minor: (j, 8l + e) at (8j + e) * 32 + l
+    __shared__ float Ws[NOUT * kHeadMaxK];          // lane-minor: (j, 8l + e) at (8j + e) * 32 + l
     __shared__ __align__(16) __nv_bfloat16 hs[kHeadRows * kHeadMaxK];
-    __shared__ float dss[kHeadRows * kHeadMaxOut];
+    __shared__ float dss[kHeadRows * NOUT];
     __shared__ int ys[kHeadRows];
     __shared__ float wloss[HEAD_NT / 32];
     __shared__ bool last;
@@ -238,9 +241,9 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&raw);
 #pragma unroll
         for (int e = 0; e < 8; ++e) hk[e] = __bfloat162float(hb[e]);
-        float sv[kHeadMaxOut], dv[kHeadMaxOut];
+        float sv[NOUT], dv[NOUT];
 #pragma unroll
-        for (int j = 0; j < kHeadMaxOut; ++j) {
+        for (int j = 0; j < NOUT; ++j) {
             if (j < nout) {
                 float p = 0.f;
                 const float* w = Ws + j * kHeadMaxK + lane;
@@ -261,41 +264,41 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
             } else {
                 float m = sv[0];
 #pragma unroll
-                for (int j = 1; j < kHeadMaxOut; ++j)
+                for (int j = 1; j < NOUT; ++j)
                     if (j < nout) m = fmaxf(m, sv[j]);
                 float z = 0.f;
 #pragma unroll
-                for (int j = 0; j < kHeadMaxOut; ++j)
+                for (int j = 0; j < NOUT; ++j)
                     if (j < nout) z += expf(sv[j] - m);
                 float sy = 0.f;
 #pragma unroll
-                for (int j = 0; j < kHeadMaxOut; ++j)
+                for (int j = 0; j < NOUT; ++j)
                     if (j < nout && j == yl) sy = sv[j];
                 li = logf(z) + m - sy;
                 const float iz = 1.0f / z;
 #pragma unroll
-                for (int j = 0; j < kHeadMaxOut; ++j)
+                for (int j = 0; j < NOUT; ++j)
                     if (j < nout) dv[j] = (expf(sv[j] - m) * iz - (j == yl ? 1.f : 0.f)) * inv_b;
             }
             wl += li;
             if (lane < nout) {
                 float sl = 0.f, dl = 0.f;
 #pragma unroll
-                for (int j = 0; j < kHeadMaxOut; ++j)
+                for (int j = 0; j < NOUT; ++j)
                     if (j == lane) { sl = sv[j]; dl = dv[j]; }
                 a.logits[(long long)(r0 + r) * nout + lane] = sl;
                 a.ds[(long long)(r0 + r) * nout + lane] = dl;
             }
         } else {
 #pragma unroll
-            for (int j = 0; j < kHeadMaxOut; ++j) dv[j] = 0.f;
+            for (int j = 0; j < NOUT; ++j) dv[j] = 0.f;
         }
         if (lane < nout) {
             float dl = 0.f;
 #pragma unroll
-            for (int j = 0; j < kHeadMaxOut; ++j)
+            for (int j = 0; j < NOUT; ++j)
                 if (j == lane) dl = dv[j];
-            dss[r * kHeadMaxOut + lane] = dl;
+            dss[r * NOUT + lane] = dl;
         }
         if (r < nr && kin) {                            // hidden layer's d(pre-activation), bf16
             __align__(16) __nv_bfloat16 ob[8];
@@ -303,7 +306,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
             for (int e = 0; e < 8; ++e) {
                 float g = 0.f;
 #pragma unroll
-                for (int j = 0; j < kHeadMaxOut; ++j)
+                for (int j = 0; j < NOUT; ++j)
                     if (j < nout) g = fmaf(dv[j], Ws[(j * 8 + e) * 32 + lane], g);
                 ob[e] = __float2bfloat16_rn(hk[e] > 0.f ? g : 0.f);
             }
@@ -324,7 +327,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
                 if (j >= nout) break;
                 float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
                 for (int r = 0; r < nr; ++r) {
-                    const float d = dss[r * kHeadMaxOut + j];
+                    const float d = dss[r * NOUT + j];
                     const uint4 raw = *reinterpret_cast<const uint4*>(hs + r * kHeadMaxK + kc);
                     const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&raw);
 #pragma unroll
@@ -337,7 +340,7 @@ __global__ void __launch_bounds__(HEAD_NT) head_kernel(const HeadArgs a) {
         }
         if (tid < nout) {
             float sb = 0.f;
-            for (int r = 0; r < nr; ++r) sb += dss[r * kHeadMaxOut + tid];
+            for (int r = 0; r < nr; ++r) sb += dss[r * NOUT + tid];
             a.pb[blockIdx.x * a.pb_stride + tid] = sb;
         }
     }
@@ -552,6 +555,40 @@ __global__ void __launch_bounds__(256) sgd_kernel(const SgdArgs a) {
     pdl_entry();
     const SgdLayer& L = a.L[blockIdx.y];
     const int nw = L.out * L.in, np = nw + L.out;
+    if (L.nsplit < 16 && L.nsplit_b < 16 && (L.in & 3) == 0 && (L.in_ld & 3) == 0) {
+        // rows of a multiple of four: four weights a thread (16-byte master and partial loads, 16-byte
+        // master stores, 8- or 16-byte copy stores), the same fp32 sums in partial order
+        const int nw4 = nw >> 2;
+        const long long st4 = L.pW_stride >> 2;
+        const float4* __restrict__ pW4 = reinterpret_cast<const float4*>(L.pW);
+        float4* __restrict__ W4 = reinterpret_cast<float4*>(L.W);
+        const int t0 = blockIdx.x * blockDim.x + threadIdx.x, nt = gridDim.x * blockDim.x;
+        for (int i = t0; i < nw4; i += nt) {
+            float4 g = pW4[i];
+            for (int z = 1; z < L.nsplit; ++z) {
+                const float4 h = pW4[z * st4 + i];
+                g.x += h.x; g.y += h.y; g.z += h.z; g.w += h.w;
+            }
+            float4 w = W4[i];
+            w.x -= a.lr * g.x; w.y -= a.lr * g.y; w.z -= a.lr * g.z; w.w -= a.lr * g.w;
+            W4[i] = w;
+            const int r = (4 * i) / L.in, c = 4 * i - r * L.in;
+            const long long o = (long long)r * L.in_ld + c;
+            if (a.c_bf16) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(w.x, w.y), hi = __floats2bfloat162_rn(w.z, w.w);
+                *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(L.cW) + o) =
+                    make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+            } else {
+                *reinterpret_cast<float4*>(static_cast<float*>(L.cW) + o) = w;
+            }
+        }
+        for (int j = t0; j < L.out; j += nt) {
+            double g = 0.0;
+            for (int z = 0; z < L.nsplit_b; ++z) g += L.pb[z * L.pb_stride + j];
+            sgd_apply_b(a, L, j, g);
+        }
+        return;
+    }
     if (L.nsplit < 16 && L.nsplit_b < 16) {
         for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < np; i += gridDim.x * blockDim.x) {
             if (i < nw) {
@@ -763,8 +800,13 @@ cudaError_t launch_head(const HeadArgs& a, cudaStream_t s) {
     if (a.rows < 1 || a.nout < 1 || a.nout > kHeadMaxOut || a.K < 8 || a.K > kHeadMaxK || (a.K & 7) ||
         a.nblk < head_blocks(a.rows))
         return cudaErrorInvalidValue;
-    SHARED_SPLIT(head_kernel);
-    head_kernel<<<a.nblk, HEAD_NT, 0, s>>>(a);
+    if (a.nout == 1) {
+        SHARED_SPLIT(head_kernel<1>);
+        head_kernel<1><<<a.nblk, HEAD_NT, 0, s>>>(a);
+    } else {
+        SHARED_SPLIT(head_kernel<kHeadMaxOut>);
+        head_kernel<kHeadMaxOut><<<a.nblk, HEAD_NT, 0, s>>>(a);
+    }
     return cudaGetLastError();
 }
 

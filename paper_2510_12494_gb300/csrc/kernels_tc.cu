@@ -668,41 +668,74 @@ constexpr int DW_BN = 128;
 constexpr int DW_SLD = DW_BN + 4;   // accumulator rows in shared memory, padded (conflict-free 16-byte stores)
 
 // Owner phase: rows [r_lo, r_lo + rpo) of the tile, four columns a thread, the CS ranks' partial tiles
-// (own slice included: every rank wrote its slice before the cluster barrier) summed in rank order; the
-// CS loads of a group are issued together.  Writes dW and, with the SGD, the master and the new version's
-// bf16 copy.
+// (own slice included: every rank wrote its slice before the cluster barrier) summed in rank order.  A
+// thread takes its groups two at a time and issues every load of both (the CS slices and, with the SGD,
+// the masters) before it stores anything.  Writes dW and, with the SGD, the master and the new version's
+// bf16 copy, 16 bytes (8 for the copy) a store where the row layout allows.
 template <int CS>
 __device__ __forceinline__ void dw_owner(const TcParams& p, const float* __restrict__ ws, size_t zstride, int r_lo,
                                          int rpo, int m0, int n0) {
     float* __restrict__ Wm = p.Wm;
+    float* __restrict__ P = p.P;
+    __nv_bfloat16* __restrict__ cW = static_cast<__nv_bfloat16*>(p.cW);
     const int nq = rpo * (DW_BN / 4);
-    for (int e = threadIdx.x; e < nq; e += THREADS) {
-        const int r = r_lo + e / (DW_BN / 4), c = (e % (DW_BN / 4)) * 4;
-        const int m = m0 + r, n = n0 + c;
-        if (m >= p.M || n >= p.N) continue;
-        const int nn = min(4, p.N - n);
-        float w[4] = {0.f, 0.f, 0.f, 0.f};
-        if (Wm)
+    const bool vec = (p.N & 3) == 0 && (p.ldp & 3) == 0 && (p.cw_ld & 3) == 0;
+    for (int e0 = threadIdx.x; e0 < nq; e0 += 2 * THREADS) {
+        float4 t[2][CS];
+        float4 w[2];
+        int m[2], n[2], nn[2];
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                if (j < nn) w[j] = Wm[(long long)m * p.N + n + j];
-        const float4* src = reinterpret_cast<const float4*>(ws + (size_t)r * DW_BN + c);
-        float4 t[CS];
+        for (int h = 0; h < 2; ++h) {
+            const int e = e0 + h * THREADS;
+            const int r = r_lo + e / (DW_BN / 4), c = (e % (DW_BN / 4)) * 4;
+            m[h] = m0 + r;
+            n[h] = n0 + c;
+            nn[h] = (e < nq && m[h] < p.M && n[h] < p.N) ? min(4, p.N - n[h]) : 0;
+            w[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (nn[h] == 0) continue;
+            const float4* src = reinterpret_cast<const float4*>(ws + (size_t)r * DW_BN + c);
 #pragma unroll
-        for (int z = 0; z < CS; ++z) t[z] = __ldcg(src + z * (zstride / 4));
-        float g[4] = {t[0].x, t[0].y, t[0].z, t[0].w};
-#pragma unroll
-        for (int z = 1; z < CS; ++z) {
-            g[0] += t[z].x; g[1] += t[z].y; g[2] += t[z].z; g[3] += t[z].w;
+            for (int z = 0; z < CS; ++z) t[h][z] = __ldcg(src + z * (zstride / 4));
+            if (Wm) {
+                const float* wp = Wm + (long long)m[h] * p.N + n[h];
+                if (vec && nn[h] == 4) {
+                    w[h] = *reinterpret_cast<const float4*>(wp);
+                } else {
+                    w[h].x = wp[0];
+                    if (nn[h] > 1) w[h].y = wp[1];
+                    if (nn[h] > 2) w[h].z = wp[2];
+                    if (nn[h] > 3) w[h].w = wp[3];
+                }
+            }
         }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            if (j >= nn) break;
-            if (p.P) p.P[(long long)m * p.ldp + n + j] = g[j];
-            if (Wm) {
-                const float wn = w[j] - p.lr * g[j];
-                Wm[(long long)m * p.N + n + j] = wn;
-                static_cast<__nv_bfloat16*>(p.cW)[(long long)m * p.cw_ld + n + j] = __float2bfloat16_rn(wn);
+        for (int h = 0; h < 2; ++h) {
+            if (nn[h] == 0) continue;
+            float4 g = t[h][0];
+#pragma unroll
+            for (int z = 1; z < CS; ++z) {
+                g.x += t[h][z].x; g.y += t[h][z].y; g.z += t[h][z].z; g.w += t[h][z].w;
+            }
+            const float gv[4] = {g.x, g.y, g.z, g.w};
+            const float wv[4] = {w[h].x - p.lr * g.x, w[h].y - p.lr * g.y, w[h].z - p.lr * g.z, w[h].w - p.lr * g.w};
+            if (vec && nn[h] == 4) {
+                if (P) *reinterpret_cast<float4*>(P + (long long)m[h] * p.ldp + n[h]) = g;
+                if (Wm) {
+                    *reinterpret_cast<float4*>(Wm + (long long)m[h] * p.N + n[h]) =
+                        make_float4(wv[0], wv[1], wv[2], wv[3]);
+                    *reinterpret_cast<uint2*>(cW + (long long)m[h] * p.cw_ld + n[h]) =
+                        make_uint2(pack_bf16(wv[0], wv[1]), pack_bf16(wv[2], wv[3]));
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (j >= nn[h]) break;
+                    if (P) P[(long long)m[h] * p.ldp + n[h] + j] = gv[j];
+                    if (Wm) {
+                        Wm[(long long)m[h] * p.N + n[h] + j] = wv[j];
+                        cW[(long long)m[h] * p.cw_ld + n[h] + j] = __float2bfloat16_rn(wv[j]);
+                    }
+                }
             }
         }
     }
