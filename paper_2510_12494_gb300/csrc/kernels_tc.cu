@@ -994,6 +994,7 @@ cudaError_t set_smem(K kernel, size_t bytes, bool cluster) {
 // Relative cost of one 128 x BN tile's k-block: 128-wide tiles read A and B from shared memory
 // for half the MMA work of 256-wide ones.
 constexpr double kCost128 = 0.62, kCost256 = 1.0;
+constexpr long long kMinTiles256 = 48;
 
 // Shared-memory sizes (and cluster sizes past 8) the kernels need, set once.
 cudaError_t kernel_attrs() {
@@ -1178,14 +1179,16 @@ cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s) {
         lc.numAttrs = 1;
         return cudaLaunchKernelEx(&lc, tc_dw_kernel, ta, tb, tb2, p);
     }
-    // forward / input gradient: 256-wide tiles unless 128-wide ones finish the grid in fewer
-    // cost-weighted rounds of the SMs
+    // forward / input gradient: 256-wide tiles when they still give at least kMinTiles256 CTAs (they do twice
+    // the work per TMA stage, so they take half the SM time of 128-wide ones: the step runs its worker
+    // streams' kernels side by side), else unless 128-wide ones finish the grid in fewer cost-weighted
+    // rounds of the SMs
     const int tm = (g.M + BM - 1) / BM;
     const long long t128 = (long long)tm * ((g.N + 127) / 128), t256 = (long long)tm * ((g.N + 255) / 256);
     const int sms = sm_count();
     const double c128 = (double)((t128 + sms - 1) / sms) * kCost128;
     const double c256 = (double)((t256 + sms - 1) / sms) * kCost256;
-    const int bn = (g.N > 128 && c256 <= c128) ? 256 : 128;
+    const int bn = (g.N > 128 && (t256 >= kMinTiles256 || c256 <= c128)) ? 256 : 128;
     p.tiles_m = tm;
     p.tiles_n = (g.N + bn - 1) / bn;
     if (g.mode == GEMM_FWD) {
