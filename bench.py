@@ -345,7 +345,8 @@ def launch_list_check(kernel, workload_name, flops_per_launch, bytes_per_launch,
     if not rec or workload_name not in rec.get("workloads", {}):
         return None
     w = rec["workloads"][workload_name]
-    stale = [f for f, h in w.get("sources_sha256", {}).items() if h != file_digest(f)]
+    mine = next((f for pre, f in KERNEL_SOURCE.items() if kernel.startswith(pre)), "kernels_simt.cu")
+    stale = [f for f, h in w.get("sources_sha256", {}).items() if h != file_digest(f) and f == mine]
     ks = w["kernels"]
     top = max(ks, key=lambda n: ks[n]["warm_share"])
     me = ks.get(kernel)
@@ -378,7 +379,8 @@ def roofline(prof, pk, workload_name, units):
     # the largest summed event time
     rec = profile_record("launches.json")
     wl = (rec or {}).get("workloads", {}).get(workload_name)
-    fresh = wl is not None and all(h == file_digest(f) for f, h in wl.get("sources_sha256", {}).items())
+    srcs = {next((f for pre, f in KERNEL_SOURCE.items() if k.startswith(pre)), "kernels_simt.cu") for k in by_kernel}
+    fresh = wl is not None and all(wl.get("sources_sha256", {}).get(f) == file_digest(f) for f in srcs)
     if fresh and any(k in wl["kernels"] for k in by_kernel):
         name = max((k for k in by_kernel if k in wl["kernels"]), key=lambda k: wl["kernels"][k]["warm_share"])
         selected_by = "largest warm share of the committed ncu launch list"

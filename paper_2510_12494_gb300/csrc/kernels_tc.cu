@@ -1092,6 +1092,7 @@ long long tc_dw_ws_floats(int out, int in, int rows) {
 // clusters the device can co-schedule, the 128-row stages each rank streams (about 0.33 us each, bound by
 // their four TMA boxes) and a fixed cost per CTA (set-up, exchange, epilogue) of about 2.5 us; ranks keep
 // at least two stages and the exchange fits the workspace.  The tile width is 128.
+constexpr long long kDwMaxCtas = 1ll << 30;   // CTAs a weight gradient may spread over
 void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_floats, int* bn_out, int* cs_out) {
     (void)concat;
     (void)kb;
@@ -1101,6 +1102,7 @@ void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_flo
     int bcs = 1;
     for (int cs = 1; cs <= MAX_CLUSTER; cs *= 2) {
         if (cs > 1 && stages < 2 * cs) break;
+        if (cs > 1 && tiles * cs > kDwMaxCtas) break;
         if (dw_ws_need(out, in, cs) > ws_floats) break;
         const long long slots = cs == 1 ? (long long)sm_count() : active_clusters(cs);
         if (slots < 1) continue;
