@@ -1091,8 +1091,11 @@ long long tc_dw_ws_floats(int out, int in, int rows) {
 // Cluster size of the weight gradient: the one with the least estimated time, counting the waves of
 // clusters the device can co-schedule, the 128-row stages each rank streams (about 0.33 us each, bound by
 // their four TMA boxes) and a fixed cost per CTA (set-up, exchange, epilogue) of about 2.5 us; ranks keep
-// at least two stages and the exchange fits the workspace.  The tile width is 128.
-constexpr long long kDwMaxCtas = 1ll << 30;   // CTAs a weight gradient may spread over
+// at least kDwMinStages stages, the kernel spreads over at most kDwMaxCtas CTAs (the worker streams' kernels
+// share the SMs: a weight gradient that holds fewer SMs a little longer leaves more to the others, which
+// measured faster on every bf16 workload) and the exchange fits the workspace.  The tile width is 128.
+constexpr long long kDwMaxCtas = 64;   // CTAs a weight gradient may spread over
+constexpr int kDwMinStages = 4;       // 128-row stages each rank streams at least
 void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_floats, int* bn_out, int* cs_out) {
     (void)concat;
     (void)kb;
@@ -1101,7 +1104,7 @@ void tc_dw_plan(int out, int in, int rows, bool concat, int kb, long long ws_flo
     double best = 1e30;
     int bcs = 1;
     for (int cs = 1; cs <= MAX_CLUSTER; cs *= 2) {
-        if (cs > 1 && stages < 2 * cs) break;
+        if (cs > 1 && stages < kDwMinStages * cs) break;
         if (cs > 1 && tiles * cs > kDwMaxCtas) break;
         if (dw_ws_need(out, in, cs) > ws_floats) break;
         const long long slots = cs == 1 ? (long long)sm_count() : active_clusters(cs);
