@@ -67,7 +67,7 @@ def parse(argv=None):
 
 # Worker streams per party (the paper's w_a = w_p) where the workload leaves them open: the count measured
 # fastest on GB300 (results do not depend on it: every step computes the same thing on any stream).
-BENCH_WORKERS = {3: 2, 4: 3}
+BENCH_WORKERS = {3: 3, 4: 3}
 
 
 def workload(args):
