@@ -555,8 +555,14 @@ def run_ours(args):
     # every step copies its rows in and its loss out (vfl_bind_host_data) inside the timed region
     e2e = None
     if not args.skip_e2e:
+        # the host keeps the features in the compute dtype (bf16 presets: rounded once here, untimed, exactly
+        # as the resident load rounds them), so the copy engines move them straight into the staging ring
+        host_bf16 = p.dtype == "bf16"
         pin_xp = torch.from_numpy(xp).pin_memory()
         pin_xa = torch.from_numpy(xa).pin_memory()
+        if host_bf16:
+            pin_xp = pin_xp.to(torch.bfloat16).pin_memory()
+            pin_xa = pin_xa.to(torch.bfloat16).pin_memory()
         pin_y = torch.from_numpy(y).pin_memory()
         loss_host = torch.full((n_e2e,), float("nan"), dtype=torch.float32).pin_memory()
         ctx.bind_host_data(pin_xp, pin_xa, pin_y, loss_out=loss_host)
@@ -600,8 +606,9 @@ def run_ours(args):
         direct = e2e_run(W + 2 * K, False)
         piped = e2e_run(W + 2 * K + n_e2e, True) if use_graphs else None
         ctx.bind_host_data(None, None, None)
-        h2d = p.batch * (p.d_passive + p.d_active) * 4 + p.batch * 4
+        h2d = p.batch * (p.d_passive + p.d_active) * (2 if host_bf16 else 4) + p.batch * 4
         e2e = {"value": max(direct, piped or 0.0), "unit": "samples/s", "h2d_bytes_per_step": h2d,
+               "host_features": "bf16" if host_bf16 else "fp32",
                "d2h_bytes_per_step": 4, "steps": n_e2e, "direct_enqueue": direct,
                "uniform_order_graph_updates": piped, "graph_windows": counts,
                "method": "uniform-order graphs updated in flight" if piped and piped > direct else "direct enqueue"}

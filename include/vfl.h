@@ -235,6 +235,17 @@ vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* x_passive, const float*
                               float* loss_out, int64_t loss_cap, void* io_stream);
 
 /*
+ * The same binding for a bf16 context whose host dataset is already in its compute dtype (the same
+ * partitioned dataset of Sec. 3; no counterpart in the paper): x_passive [n_rows, d_p] and
+ * x_active [n_rows, d_a] hold bf16 bit patterns (round-to-nearest-even of the fp32 features gives the
+ * rows vfl_load_data would store), y [n_rows] int32; VFL_E_INVAL for an fp32 context.  Each step's
+ * staging kernel then copies its rows without rounding: half the bytes over the host link of the fp32
+ * binding.  Everything else is as for vfl_bind_host_data; x_passive = null unbinds.
+ */
+vfl_status vfl_bind_host_data_bf16(vfl_ctx* ctx, const uint16_t* x_passive, const uint16_t* x_active,
+                                   const int32_t* y, float* loss_out, int64_t loss_cap, void* io_stream);
+
+/*
  * The parameters theta_2 (f_p) and theta_1 (f_a and g) of Sec. 3 that Eq. 2 updates.
  * Set / read the fp32 master parameters of one layer: W [out, in], b [out]
  * (host pointers).  vfl_set_params resets every stored weight version of the

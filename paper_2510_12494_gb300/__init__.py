@@ -72,6 +72,8 @@ EXPORTS = {
     "vfl_load_data": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "vfl_bind_host_data": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                             ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
+    "vfl_bind_host_data_bf16": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                                 ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_set_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
                                         ctypes.c_void_p]),
     "vfl_get_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
@@ -370,7 +372,8 @@ class Context:
 
     def bind_host_data(self, xp, xa, y, loss_out=None):
         """Every later step reads its rows from these host tensors (pinned torch
-        tensors [n_rows, d_p] / [n_rows, d_a] fp32 and [n_rows] int32) on an I/O
+        tensors [n_rows, d_p] / [n_rows, d_a] fp32, or bf16 for a bf16 context
+        (vfl_bind_host_data_bf16), and [n_rows] int32) on an I/O
         stream of the context, and writes its mean loss into loss_out[k % len(loss_out)]
         (a pinned fp32 tensor, optional); see vfl_bind_host_data.
         bind_host_data(None, None, None) unbinds.  The tensors stay referenced while bound."""
@@ -381,13 +384,14 @@ class Context:
             return
         assert tuple(xp.shape) == (self.n_rows, self.p.d_passive) and tuple(xa.shape) == (self.n_rows, self.p.d_active)
         assert tuple(y.shape) == (self.n_rows,)
-        assert xp.dtype == torch.float32 and xa.dtype == torch.float32 and y.dtype == torch.int32
+        assert xp.dtype == xa.dtype and xp.dtype in (torch.float32, torch.bfloat16) and y.dtype == torch.int32
         assert xp.is_contiguous() and xa.is_contiguous() and y.is_contiguous()
         if not hasattr(self, "_io_stream"):
             self._io_stream = torch.cuda.Stream()
         lp = ctypes.c_void_p(loss_out.data_ptr()) if loss_out is not None else None
         cap = len(loss_out) if loss_out is not None else 0
-        self._call(lib().vfl_bind_host_data, ctypes.c_void_p(xp.data_ptr()), ctypes.c_void_p(xa.data_ptr()),
+        fn = lib().vfl_bind_host_data_bf16 if xp.dtype == torch.bfloat16 else lib().vfl_bind_host_data
+        self._call(fn, ctypes.c_void_p(xp.data_ptr()), ctypes.c_void_p(xa.data_ptr()),
                    ctypes.c_void_p(y.data_ptr()), lp, cap, ctypes.c_void_p(self._io_stream.cuda_stream))
         self._host_data = (xp, xa, y, loss_out)
 

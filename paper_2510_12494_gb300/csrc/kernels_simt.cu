@@ -745,6 +745,51 @@ __device__ __forceinline__ void stage_block(const float* __restrict__ h, int d, 
     }
 }
 
+// The same for bf16 host rows into a bf16 slot: 16-byte copies of eight elements where rows allow.
+__device__ __forceinline__ void stage_block_b16(const uint16_t* __restrict__ h, int d, int rows, uint16_t* dst,
+                                                long long ld, int tid, int nthreads) {
+    const int n = rows * d;
+    if ((d & 7) == 0 && (reinterpret_cast<uintptr_t>(h) & 15) == 0 && (ld & 7) == 0) {
+        const int nq = n / 8;
+        constexpr int U = 4;
+        for (int q0 = tid; q0 < nq; q0 += nthreads * U) {
+            uint4 v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = q0 + u * nthreads;
+                if (q < nq) v[u] = __ldcs(reinterpret_cast<const uint4*>(h) + q);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = q0 + u * nthreads;
+                if (q >= nq) break;
+                const int f = 8 * q, r = f / d, c = f - r * d;
+                *reinterpret_cast<uint4*>(dst + (long long)r * ld + c) = v[u];
+            }
+        }
+    } else {
+        for (int i = tid; i < n; i += nthreads) {
+            const int r = i / d, c = i - r * d;
+            dst[(long long)r * ld + c] = h[i];
+        }
+    }
+    const int pad = (int)(ld - d);
+    for (int i = tid; i < rows * pad; i += nthreads) {
+        const int r = i / pad, c = d + (i - r * pad);
+        dst[(long long)r * ld + c] = 0;
+    }
+}
+
+__global__ void stage_rows_b16_kernel(const uint16_t* __restrict__ hxp, int dp, const uint16_t* __restrict__ hxa,
+                                      int da, const int* __restrict__ hy, int rows, uint16_t* xp, long long ld_p,
+                                      uint16_t* xa, long long ld_a, int* __restrict__ y) {
+    pdl_entry();
+    const int tid = blockIdx.x * blockDim.x + threadIdx.x, nt = gridDim.x * blockDim.x;
+    stage_block_b16(hxp, dp, rows, xp, ld_p, tid, nt);
+    stage_block_b16(hxa, da, rows, xa, ld_a, tid, nt);
+    for (int i = tid; i < rows; i += nt) y[i] = hy[i];
+}
+
 __global__ void stage_rows_kernel(const float* __restrict__ hxp, int dp, const float* __restrict__ hxa, int da,
                                   const int* __restrict__ hy, int rows, void* xp, long long ld_p, void* xa,
                                   long long ld_a, int* __restrict__ y, int bf16) {
@@ -909,6 +954,16 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
     return cudaGetLastError();
 }
 
+
+cudaError_t launch_stage_rows_b16(const uint16_t* hxp, int dp, const uint16_t* hxa, int da, const int* hy, int rows,
+                                  void* xp, long long ld_p, void* xa, long long ld_a, int* y, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    const long long n = (long long)rows * (ld_p + ld_a + 16) / 8;
+    SHARED_SPLIT(stage_rows_b16_kernel);
+    stage_rows_b16_kernel<<<grid_for(n, 256), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, static_cast<uint16_t*>(xp), ld_p,
+                                                          static_cast<uint16_t*>(xa), ld_a, y);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_to_f32(const void* src, long long ld, int rows, int cols, int bf16, float* dst, cudaStream_t s) {
     if (rows <= 0 || cols <= 0) return cudaSuccess;

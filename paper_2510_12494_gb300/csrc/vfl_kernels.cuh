@@ -174,6 +174,9 @@ cudaError_t launch_cast_rows(const float* src, int rows, int d, void* dst, long 
 // rows of ld_p / ld_a elements (bf16 or fp32, padding columns zero), and the labels.
 cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da, const int* hy, int rows, void* xp,
                               long long ld_p, void* xa, long long ld_a, int* y, int bf16, cudaStream_t s);
+// The same for bf16 host rows into a bf16 context (no rounding: a 16-byte copy of eight elements per thread).
+cudaError_t launch_stage_rows_b16(const uint16_t* hxp, int dp, const uint16_t* hxa, int da, const int* hy, int rows,
+                                  void* xp, long long ld_p, void* xa, long long ld_a, int* y, cudaStream_t s);
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);
 

@@ -172,9 +172,12 @@ struct vfl_ctx {
     // host-resident data (vfl_bind_host_data): each step reads its rows into slot k mod io_R of a
     // device staging ring on the caller's I/O stream; the loss kernels also write the host ring
     bool hio = false;
-    const float* h_xp = nullptr;
+    const float* h_xp = nullptr;                // device views of the bound arrays (fp32 features)
     const float* h_xa = nullptr;
+    const void* hv_xp = nullptr;                // the same views, any feature dtype
+    const void* hv_xa = nullptr;
     const int32_t* h_y = nullptr;
+    int h_esz = 4;                              // element bytes of the bound features (4 fp32, 2 bf16)
     float* h_loss = nullptr;
     long long h_loss_cap = 0;
     int io_R = 0;
@@ -1179,10 +1182,20 @@ vfl_status stage_step(vfl_ctx* ctx, long long k) {
         TRY(wait_ev(ctx, s, ctx->ev_pver[(prev + 1) % kEvPool]));
         TRY(wait_ev(ctx, s, ctx->ev_aver[(prev + 1) % kEvPool]));
     }
-    PLAUNCH(K_CAST, 0, (double)rows * (c.d_passive + c.d_active + 1) * 4 + (double)rows * (ctx->ldxp + ctx->ldxa) * ctx->esz,
-            s, launch_stage_rows(ctx->h_xp + r0 * c.d_passive, c.d_passive, ctx->h_xa + r0 * c.d_active, c.d_active,
-                                 ctx->h_y + r0, rows, ctx->io_xp[slot], ctx->ldxp, ctx->io_xa[slot], ctx->ldxa,
-                                 ctx->io_y[slot], ctx->bf16, s));
+    if (ctx->h_esz == 2) {
+        // bf16 rows into the bf16 slot: half the bytes over the host link
+        const uint16_t* hp = static_cast<const uint16_t*>(ctx->hv_xp);
+        const uint16_t* ha = static_cast<const uint16_t*>(ctx->hv_xa);
+        PLAUNCH(K_CAST, 0, (double)rows * (c.d_passive + c.d_active) * 2 * 2 + (double)rows * 8, s,
+                launch_stage_rows_b16(hp + r0 * c.d_passive, c.d_passive, ha + r0 * c.d_active, c.d_active,
+                                      ctx->h_y + r0, rows, ctx->io_xp[slot], ctx->ldxp, ctx->io_xa[slot], ctx->ldxa,
+                                      ctx->io_y[slot], s));
+    } else {
+        PLAUNCH(K_CAST, 0, (double)rows * (c.d_passive + c.d_active + 1) * 4 + (double)rows * (ctx->ldxp + ctx->ldxa) * ctx->esz,
+                s, launch_stage_rows(ctx->h_xp + r0 * c.d_passive, c.d_passive, ctx->h_xa + r0 * c.d_active, c.d_active,
+                                     ctx->h_y + r0, rows, ctx->io_xp[slot], ctx->ldxp, ctx->io_xa[slot], ctx->ldxa,
+                                     ctx->io_y[slot], ctx->bf16, s));
+    }
     CK(cudaEventRecord(ctx->ev_staged[k % kEvPool], s));
     return VFL_OK;
 }
@@ -1853,8 +1866,8 @@ const void* device_view(const void* p) {
 }
 }  // namespace
 
-vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* xp, const float* xa, const int32_t* y, float* loss_out,
-                              int64_t loss_cap, void* io_stream) {
+vfl_status bind_host_data(vfl_ctx* ctx, const void* xp, const void* xa, const int32_t* y, float* loss_out,
+                          int64_t loss_cap, void* io_stream, int esz) {
     if (!ctx) return VFL_E_INVAL;
     if (ctx->broken) return VFL_E_CUDA;
     if (ctx->n_fwd != ctx->n_bwd || ctx->n_act != ctx->n_bwd)
@@ -1864,6 +1877,7 @@ vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* xp, const float* xa, co
         ctx->hio = false;
         ctx->h_xp = ctx->h_xa = nullptr;
         ctx->h_y = nullptr;
+        ctx->hv_xp = ctx->hv_xa = nullptr;
         ctx->h_loss = nullptr;
         ctx->h_loss_cap = 0;
         ctx->io = nullptr;
@@ -1887,11 +1901,26 @@ vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* xp, const float* xa, co
     ctx->h_xp = static_cast<const float*>(dxp);
     ctx->h_xa = static_cast<const float*>(dxa);
     ctx->h_y = static_cast<const int32_t*>(dy);
+    ctx->hv_xp = dxp;
+    ctx->hv_xa = dxa;
+    ctx->h_esz = esz;
     ctx->h_loss = static_cast<float*>(const_cast<void*>(dl));
     ctx->h_loss_cap = loss_out ? loss_cap : 0;
     ctx->io = static_cast<cudaStream_t>(io_stream);
     ctx->hio = true;
     return VFL_OK;
+}
+
+vfl_status vfl_bind_host_data(vfl_ctx* ctx, const float* xp, const float* xa, const int32_t* y, float* loss_out,
+                              int64_t loss_cap, void* io_stream) {
+    return bind_host_data(ctx, xp, xa, y, loss_out, loss_cap, io_stream, 4);
+}
+
+vfl_status vfl_bind_host_data_bf16(vfl_ctx* ctx, const uint16_t* xp, const uint16_t* xa, const int32_t* y,
+                                   float* loss_out, int64_t loss_cap, void* io_stream) {
+    if (!ctx) return VFL_E_INVAL;
+    if (xp && !ctx->bf16) return ctx->fail(VFL_E_INVAL, "bf16 host data needs a bf16 context");
+    return bind_host_data(ctx, xp, xa, y, loss_out, loss_cap, io_stream, 2);
 }
 
 vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const float* W, const float* b) {

@@ -23,12 +23,16 @@ def vfl():
     return v
 
 
-def host_context(vfl, q, xp, xa, y, params, cap):
-    """A context that never loads the dataset: its resident copy stays zero."""
+def host_context(vfl, q, xp, xa, y, params, cap, bf16_host=False):
+    """A context that never loads the dataset: its resident copy stays zero.  With
+    bf16_host the features are bound as bf16 (vfl_bind_host_data_bf16)."""
     import torch
     ctx = vfl.Context(q, q.n_rows)
     ctx.set_params(params)
     pins = [torch.from_numpy(a).pin_memory() for a in (xp, xa, y)]
+    if bf16_host:
+        pins[0] = pins[0].to(torch.bfloat16).pin_memory()
+        pins[1] = pins[1].to(torch.bfloat16).pin_memory()
     loss = torch.full((cap,), float("nan"), dtype=torch.float32).pin_memory()
     ctx.bind_host_data(*pins, loss_out=loss)
     return ctx, loss
@@ -140,3 +144,38 @@ def test_host_data_uniform_order_graph_updates(vfl):
     ctx.synchronize()
     np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
     assert_same_state(ctx, ref)
+
+
+@pytest.mark.parametrize("cid,workers", [(3, 0), (3, 3), (4, 0)])
+def test_bf16_host_data_equals_resident(vfl, cid, workers):
+    """bf16 host arrays (round to nearest even of the fp32 features, as the
+    resident load rounds them) reach the staging ring by the copy engines;
+    training on them is bit-identical to training on the resident dataset,
+    directly enqueued and replayed from graphs."""
+    p = synth.preset(cid)
+    if workers:
+        p = p.with_(workers=workers)
+    rows = {3: 2 * 4096 + 288, 4: 2 * 8192 + 520}[cid]
+    q, xp, xa, y, params = setup(p, rows)
+    nb = q.steps_per_epoch
+    n = 2 * nb + 1
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx, loss = host_context(vfl, q, xp, xa, y, params, cap=n, bf16_host=True)
+    ctx.train_steps(0, nb, tp, ta)
+    ctx.launch_graph(ctx.capture(nb, n - nb, tp, ta))
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
+    assert_same_state(ctx, ref)
+
+
+def test_bf16_host_data_needs_bf16_context(vfl):
+    import torch
+    q, xp, xa, y, params = setup(synth.preset(1), 1024)
+    ctx = vfl.Context(q, q.n_rows)
+    pins = [torch.from_numpy(a).pin_memory() for a in (xp, xa, y)]
+    with pytest.raises(vfl.VflError):
+        ctx.bind_host_data(pins[0].to(torch.bfloat16).pin_memory(), pins[1].to(torch.bfloat16).pin_memory(), pins[2])
+    ctx.close()
