@@ -809,6 +809,10 @@ __global__ void to_f32_kernel(const void* src, long long ld, int rows, int cols,
     }
 }
 
+// Blocks of a host-staging kernel: four per SM already pull the host link's full rate, and the step's compute
+// kernels keep the rest of the SMs' warp slots.
+constexpr int kStageBlocks = 152 * 4;
+
 inline int grid_for(long long n, int nt) {
     long long b = (n + nt - 1) / nt;
     if (b < 1) b = 1;
@@ -950,7 +954,8 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
     if (rows <= 0) return cudaSuccess;
     const long long n = (long long)rows * (ld_p + ld_a + 1);
     SHARED_SPLIT(stage_rows_kernel);
-    stage_rows_kernel<<<grid_for(n, 256), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, xp, ld_p, xa, ld_a, y, bf16);
+    stage_rows_kernel<<<std::min(grid_for(n, 256), kStageBlocks), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, xp, ld_p, xa,
+                                                                              ld_a, y, bf16);
     return cudaGetLastError();
 }
 
@@ -960,7 +965,7 @@ cudaError_t launch_stage_rows_b16(const uint16_t* hxp, int dp, const uint16_t* h
     if (rows <= 0) return cudaSuccess;
     const long long n = (long long)rows * (ld_p + ld_a + 16) / 8;
     SHARED_SPLIT(stage_rows_b16_kernel);
-    stage_rows_b16_kernel<<<grid_for(n, 256), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, static_cast<uint16_t*>(xp), ld_p,
+    stage_rows_b16_kernel<<<std::min(grid_for(n, 256), kStageBlocks), 256, 0, s>>>(hxp, dp, hxa, da, hy, rows, static_cast<uint16_t*>(xp), ld_p,
                                                           static_cast<uint16_t*>(xa), ld_a, y);
     return cudaGetLastError();
 }
