@@ -173,6 +173,12 @@ __device__ __forceinline__ bool mbar_wait_idle(uint32_t bar, uint32_t parity, vo
     return false;
 }
 
+// Bring a tensor map (a __grid_constant__ kernel parameter) into the TMA unit's descriptor cache ahead of
+// its first copy.
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -512,6 +518,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int ntiles = p.tiles_m * p.tiles_n;
     const int nk = (p.K + BK - 1) / BK;
 
+    if (threadIdx.x == 32) {
+        prefetch_map(&ta);
+        prefetch_map(&ta2);
+        prefetch_map(&tb);
+    }
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
@@ -784,6 +795,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int nk = kend > kbeg ? (kend - kbeg + C::KS - 1) / C::KS : 0;
     const bool bias = p.Pb != nullptr && blockIdx.y == 0;   // one column of tiles takes db
 
+    if (threadIdx.x == 32) {
+        prefetch_map(&ta);
+        prefetch_map(&tb);
+        prefetch_map(&tb2);
+    }
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
