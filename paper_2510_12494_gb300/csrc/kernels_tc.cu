@@ -949,6 +949,230 @@ __global__ void __launch_bounds__(THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Layer chain: a bottom model's forward (every layer <= 256 wide) for one 128-row tile in one CTA.
+// The tile's activations stay in shared memory between layers as the next layer's A operand (K-major,
+// 128-byte swizzle: the epilogue writes them in the layout TMA would), only the weights stream through
+// the ring, and every layer's output also goes to global memory (the backward reads it).
+// ---------------------------------------------------------------------------
+constexpr int CH_MAX_LAYERS = 4;
+constexpr int CH_STAGES = 4;
+constexpr uint32_t CH_KB_BYTES = BM * BK * 2;          // one 128 x 64 k-block of the activation tile
+constexpr uint32_t CH_ACT_BYTES = 4 * CH_KB_BYTES;     // inputs up to 256 wide
+constexpr uint32_t CH_B_BYTES = 256 * BK * 2;          // one weight k-block of the widest layer
+constexpr uint32_t CH_RING_OFF = CH_ACT_BYTES;
+constexpr uint32_t CH_CTRL_OFF = CH_RING_OFF + CH_STAGES * CH_B_BYTES;
+constexpr uint32_t CH_STAGE_OFF = CH_CTRL_OFF + 256;
+constexpr size_t CH_SMEM = 1024 + CH_STAGE_OFF + GEMM_EPI_WARPS * 2048;
+
+struct ChainParams {
+    int L, M, K0;
+    int out[CH_MAX_LAYERS];
+    const float* bias[CH_MAX_LAYERS];
+    void* Y[CH_MAX_LAYERS];
+    long long ldy[CH_MAX_LAYERS];
+    int* err;
+    HeaderOps hdr;
+};
+struct ChainMaps {
+    CUtensorMap x;
+    CUtensorMap w[CH_MAX_LAYERS];
+};
+
+__device__ __forceinline__ uint32_t idesc_n(int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    tc_chain_kernel(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainParams p) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* act = base;
+    uint8_t* ring = base + CH_RING_OFF;
+    uint64_t* full = reinterpret_cast<uint64_t*>(base + CH_CTRL_OFF);
+    uint64_t* empty = full + CH_STAGES;
+    uint64_t* act_full = empty + CH_STAGES;    // the first layer's input tile landed (TMA)
+    uint64_t* acc_full = act_full + 1;         // a layer's MMAs are complete
+    uint64_t* act_ready = acc_full + 1;        // a layer's output is in `act` and TMEM is drained
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(act_ready + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * BM;
+    const int L = p.L;
+
+    if (threadIdx.x == 32) {
+        prefetch_map(&maps.x);
+        for (int l = 0; l < L; ++l) prefetch_map(&maps.w[l]);
+    }
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < CH_STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(act_full), 1);
+        mbar_init(smem_u32(acc_full), 1);
+        mbar_init(smem_u32(act_ready), GEMM_EPI_WARPS);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    // the activation tile starts at zero (columns no layer writes are read against zero weight columns);
+    // the generic-proxy writes are ordered before the tensor core's and the TMA's accesses
+    for (int i = threadIdx.x; i < (int)(CH_ACT_BYTES / 16); i += GEMM_THREADS)
+        sts128(smem_u32(act) + 16u * i, make_uint4(0u, 0u, 0u, 0u));
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(256)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_slot;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    header_check(p.hdr);
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer: the input tile, then every layer's weight k-blocks ----------------
+        const int nk0 = (p.K0 + BK - 1) / BK;
+        mbar_expect_tx(smem_u32(act_full), (uint32_t)nk0 * CH_KB_BYTES);
+        for (int kb = 0; kb < nk0; ++kb)
+            tma_load_2d(smem_u32(act + kb * CH_KB_BYTES), &maps.x, kb * BK, m0, smem_u32(act_full));
+        uint32_t it = 0;
+        bool ok = true;
+        for (int l = 0; l < L && ok; ++l) {
+            const int in = l == 0 ? p.K0 : p.out[l - 1];
+            const int nk = (in + BK - 1) / BK;
+            for (int kb = 0; kb < nk; ++kb, ++it) {
+                const int s = it % CH_STAGES;
+                if (!mbar_wait(smem_u32(&empty[s]), ((it / CH_STAGES) & 1) ^ 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t bar = smem_u32(&full[s]);
+                mbar_expect_tx(bar, (uint32_t)p.out[l] * BK * 2);
+                tma_load_2d(smem_u32(ring + s * CH_B_BYTES), &maps.w[l], kb * BK, 0, bar);
+            }
+        }
+        if (*abort_flag) {
+            // bounded drain of the loads in flight before the CTA may exit
+            const uint32_t first = it > (uint32_t)CH_STAGES ? it - CH_STAGES : 0;
+            for (uint32_t i = first; i < it; ++i)
+                for (long long t = 0; t < WAIT_LIMIT && !mbar_try(smem_u32(&full[i % CH_STAGES]), (i / CH_STAGES) & 1); ++t) {
+                }
+            for (long long t = 0; t < WAIT_LIMIT && !mbar_try(smem_u32(act_full), 0); ++t) {
+            }
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        uint32_t it = 0;
+        int commits = 0;
+        for (int l = 0; l < L; ++l) {
+            const bool ok = l == 0 ? mbar_wait(smem_u32(act_full), 0, abort_flag)
+                                   : mbar_wait(smem_u32(act_ready), (l - 1) & 1, abort_flag);
+            if (!ok) {
+                mma_commit(smem_u32(acc_full));
+                ++commits;
+                break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int in = l == 0 ? p.K0 : p.out[l - 1];
+            const int nk = (in + BK - 1) / BK;
+            const uint32_t idesc = idesc_n(p.out[l]);
+            bool good = true;
+            for (int kb = 0; kb < nk; ++kb, ++it) {
+                const int s = it % CH_STAGES;
+                if (!mbar_wait(smem_u32(&full[s]), (it / CH_STAGES) & 1, abort_flag)) {
+                    good = false;
+                    break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t aB = smem_u32(act + kb * CH_KB_BYTES), bB = smem_u32(ring + s * CH_B_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    mma_bf16(tmem, smem_desc(aB + kk * 32, 16, 1024), smem_desc(bB + kk * 32, 16, 1024), idesc,
+                             (kb > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(smem_u32(&empty[s]));
+            }
+            mma_commit(smem_u32(acc_full));
+            ++commits;
+            if (!good) break;
+        }
+        // the last commit tracks every MMA issued: wait (bounded) for it before TMEM can be freed
+        if (commits > 0)
+            for (long long t = 0; t < WAIT_LIMIT && !mbar_try(smem_u32(acc_full), (commits - 1) & 1); ++t) {
+            }
+    } else if (warp >= 2) {
+        // ---------------- epilogue: 16 warps, four per TMEM lane quarter, a quarter of the columns each ----
+        const int quarter = warp & 3;
+        const int group = (warp - 2) >> 2;
+        const int row = quarter * 32 + lane;            // this lane's row of the tile
+        const int r0 = m0 + quarter * 32;
+        const uint32_t stage = smem_u32(base + CH_STAGE_OFF + (warp - 2) * 2048);
+        const uint4 nomask[4] = {};
+        for (int l = 0; l < L; ++l) {
+            const int N = p.out[l];
+            const int cw = N / 4;                       // 32 or 64 columns: one or two passes
+            float bias[2];
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int c = group * cw + 32 * q + lane;
+                bias[q] = 32 * q < cw ? __ldg(p.bias[l] + c) : 0.f;
+            }
+            if (!mbar_wait_idle(smem_u32(acc_full), l & 1, abort_flag)) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+            __nv_bfloat16* Y = static_cast<__nv_bfloat16*>(p.Y[l]);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                if (32 * q >= cw) break;
+                const int c0 = group * cw + 32 * q;
+                float v[32];
+                tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
+                uint32_t u[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const float x0 = fmaxf(v[2 * j] + __shfl_sync(0xffffffffu, bias[q], 2 * j), 0.f);
+                    const float x1 = fmaxf(v[2 * j + 1] + __shfl_sync(0xffffffffu, bias[q], 2 * j + 1), 0.f);
+                    u[j] = pack_bf16(x0, x1);
+                }
+                // this row's 32 columns to global memory, through the staging buffer
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    sts128(stage_unit(stage, lane, c), make_uint4(u[4 * c], u[4 * c + 1], u[4 * c + 2], u[4 * c + 3]));
+                __syncwarp();
+                store_bf16_block(stage, lane, Y, p.ldy[l], nullptr, nomask, r0, p.M, c0, 32);
+                __syncwarp();
+                // and into the activation tile as the next layer's A operand: k-block c0 / 64, 16-byte chunks
+                // (c0 mod 64) / 8 + j of this row's 128 bytes, swizzled by row mod 8
+                if (l + 1 < L) {
+                    const uint32_t rowb = smem_u32(act + (c0 / BK) * CH_KB_BYTES) + (uint32_t)row * 128u;
+                    const int ch0 = (c0 % BK) / 8;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        sts128(rowb + (uint32_t)((((ch0 + j) ^ (row & 7)) & 7) << 4),
+                               make_uint4(u[4 * j], u[4 * j + 1], u[4 * j + 2], u[4 * j + 3]));
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(act_ready));
+        }
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) atomicOr(p.err, ST_KERNEL_TIMEOUT);
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256) : "memory");
+    }
+    header_publish(p.hdr);
+}
+
+// ---------------------------------------------------------------------------
 // host side: tensor maps through the driver entry point
 // ---------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -1018,12 +1242,49 @@ cudaError_t kernel_attrs() {
         cudaError_t e = set_smem(tc_gemm_kernel<128>, GemmCfg<128>::SMEM, false);
         if (e == cudaSuccess) e = set_smem(tc_gemm_kernel<256>, GemmCfg<256>::SMEM, false);
         if (e == cudaSuccess) e = set_smem(tc_dw_kernel, DwCfg::SMEM, true);
+        if (e == cudaSuccess) e = set_smem(tc_chain_kernel, CH_SMEM, false);
         return e;
     }();
     return attr;
 }
 
 }  // namespace
+
+bool tc_chain_supported(int L, int K0, const int* out) {
+    if (L < 2 || L > CH_MAX_LAYERS || K0 < 1 || K0 > 4 * BK) return false;
+    for (int l = 0; l < L; ++l)
+        if (out[l] != 128 && out[l] != 256) return false;
+    return tc_available();
+}
+
+cudaError_t launch_tc_chain(const TcChain& c, cudaStream_t s) {
+    int outs[CH_MAX_LAYERS];
+    for (int l = 0; l < c.L && l < CH_MAX_LAYERS; ++l) outs[l] = c.out[l];
+    if (!tc_chain_supported(c.L, c.K0, outs) || c.M < 1) return cudaErrorInvalidValue;
+    const cudaError_t attr = kernel_attrs();
+    if (attr != cudaSuccess) return attr;
+    ChainMaps maps;
+    std::memset(&maps, 0, sizeof maps);
+    ChainParams p;
+    std::memset(&p, 0, sizeof p);
+    bool ok = make_map(&maps.x, c.X, c.ldx, c.M, c.ldx, BK, BM);
+    for (int l = 0; l < c.L; ++l) {
+        const int in = l == 0 ? c.K0 : c.out[l - 1];
+        ok &= c.ldw[l] >= in && make_map(&maps.w[l], c.W[l], c.ldw[l], c.out[l], c.ldw[l], BK, c.out[l]);
+        p.out[l] = c.out[l];
+        p.bias[l] = c.bias[l];
+        p.Y[l] = c.Y[l];
+        p.ldy[l] = c.ldy[l];
+    }
+    if (!ok) return cudaErrorInvalidValue;
+    p.L = c.L;
+    p.M = c.M;
+    p.K0 = c.K0;
+    p.err = c.err;
+    p.hdr = c.hdr;
+    tc_chain_kernel<<<(c.M + BM - 1) / BM, GEMM_THREADS, CH_SMEM, s>>>(maps, p);
+    return cudaGetLastError();
+}
 
 bool tc_available() { return encode_fn() != nullptr; }
 

@@ -161,6 +161,7 @@ struct vfl_ctx {
 
     // bf16 path: g's output layer and the loss in one launch (narrow output over a narrow hidden layer)
     bool head = false;
+    bool chain = false;                           // bf16 bottom models forward as one layer-chain launch
     int* h_counter = nullptr;                   // per worker: blocks finished
     float* h_blk_loss[kMaxWorkers] = {};        // per worker: per-block loss sums
 
@@ -1282,6 +1283,40 @@ vfl_status do_drop_active(vfl_ctx* ctx, long long k) {
     return VFL_OK;
 }
 
+// A bottom model's forward as one layer-chain launch when its shape allows (every layer 128 or 256 wide,
+// 2-4 layers, an input of at most 256 features); *done = false when it does not (the caller runs the layers).
+vfl_status chain_forward(vfl_ctx* ctx, const std::vector<Layer>& Ls, int vslot, const void* X, long long ldx,
+                         int rows, void* const* Y, const HeaderOps* hdr, cudaStream_t s, bool* done) {
+    *done = false;
+    if (!ctx->chain || Ls.size() < 2 || Ls.size() > 4) return VFL_OK;
+    int outs[4];
+    for (size_t l = 0; l < Ls.size(); ++l) outs[l] = Ls[l].out;
+    if (!tc_chain_supported((int)Ls.size(), Ls[0].in, outs)) return VFL_OK;
+    TcChain t = {};
+    t.L = (int)Ls.size();
+    t.M = rows;
+    t.K0 = Ls[0].in;
+    t.X = X;
+    t.ldx = ldx;
+    double flops = 0.0, bytes = (double)rows * ldx * ctx->esz;
+    for (int l = 0; l < t.L; ++l) {
+        const Layer& L = Ls[l];
+        t.W[l] = L.cW[vslot];
+        t.ldw[l] = L.in_ld;
+        t.out[l] = L.out;
+        t.bias[l] = L.cb[vslot];
+        t.Y[l] = Y[l];
+        t.ldy[l] = ld8(L.out);
+        flops += 2.0 * rows * L.out * L.in;
+        bytes += ((double)L.out * L.in + (double)rows * L.out) * ctx->esz + L.out * 4.0;
+    }
+    t.err = ctx->status;
+    if (hdr) t.hdr = *hdr;
+    PLAUNCH(K_TC_FWD, flops, bytes, s, launch_tc_chain(t, s));
+    *done = true;
+    return VFL_OK;
+}
+
 vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = false) {
     const vfl_config& c = ctx->cfg;
     if (k != ctx->n_fwd) return ctx->fail(VFL_E_STATE, "passive_forward(%lld): next publish is step %lld", k, ctx->n_fwd);
@@ -1329,13 +1364,19 @@ vfl_status do_passive_forward(vfl_ctx* ctx, long long k, int tau_p, bool drop = 
     pub.k = k;
     pub.batch = (int)ctx->batch_of(k);
     pub.version = (int)v;
-    for (size_t l = 0; l < ctx->P.size(); ++l) {
-        const Layer& L = ctx->P[l];
-        void* Y = ctx->act_p[slot][l];
-        const bool publish = l + 1 == ctx->P.size() && !emb_dp(ctx);
-        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, Y, ld8(L.out), true, false, s, publish ? &pub : nullptr));
-        X = Y;
-        ldx = ld8(L.out);
+    bool chained = false;
+    TRY(chain_forward(ctx, ctx->P, vslot, X, ldx, rows, ctx->act_p[slot].data(), emb_dp(ctx) ? nullptr : &pub, s,
+                      &chained));
+    if (!chained) {
+        for (size_t l = 0; l < ctx->P.size(); ++l) {
+            const Layer& L = ctx->P[l];
+            void* Y = ctx->act_p[slot][l];
+            const bool publish = l + 1 == ctx->P.size() && !emb_dp(ctx);
+            TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, Y, ld8(L.out), true, false, s,
+                           publish ? &pub : nullptr));
+            X = Y;
+            ldx = ld8(L.out);
+        }
     }
     if (emb_dp(ctx)) {   // App. C: the published embedding is clipped and noised; z stays for the backward
         const int ep = ctx->P.back().out;
@@ -1397,11 +1438,15 @@ vfl_status do_active_step(vfl_ctx* ctx, long long k, int tau_a) {
     // active bottom forward: z^a = f_a(x^a)
     const void* X = Xa0;
     long long ldx = ctx->ldxa;
-    for (int l = 0; l < La; ++l) {
-        const Layer& L = ctx->A[l];
-        TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, ctx->act_a[w][l], ld8(L.out), true, false, s));
-        X = ctx->act_a[w][l];
-        ldx = ld8(L.out);
+    bool chained = false;
+    TRY(chain_forward(ctx, ctx->A, vslot, X, ldx, rows, ctx->act_a[w].data(), nullptr, s, &chained));
+    if (!chained) {
+        for (int l = 0; l < La; ++l) {
+            const Layer& L = ctx->A[l];
+            TRY(linear_fwd(ctx, L, vslot, X, ldx, nullptr, 0, 0, rows, ctx->act_a[w][l], ld8(L.out), true, false, s));
+            X = ctx->act_a[w][l];
+            ldx = ld8(L.out);
+        }
     }
     // subscribe: wait for the embedding of step k; the first kernel that reads it checks its header
     TRY(wait_ev(ctx, s, ctx->ev_emb[k % kEvPool]));
@@ -1722,6 +1767,7 @@ vfl_status vfl_create(const vfl_config* cfg, int64_t n_rows, void* workspace, ui
     for (int i = 0; i < kInfoRing; ++i) ctx->step_id[i] = -1;
     ctx->fused = fused_eligible(*cfg) && !getenv("VFL_DISABLE_FUSED");
     ctx->head = head_eligible(*cfg) && !getenv("VFL_DISABLE_HEAD");
+    ctx->chain = cfg->dtype == VFL_BF16 && !ctx->fused && !getenv("VFL_DISABLE_CHAIN");
     ctx->direct_pdl = !getenv("VFL_DISABLE_DIRECT_PDL");
     build_layers(ctx);
     const unsigned long long need = carve_all(ctx, nullptr);

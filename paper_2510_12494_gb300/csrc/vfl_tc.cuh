@@ -59,4 +59,21 @@ bool tc_supported_dx(int in, int out, int n_split, bool c2_f32);
 bool tc_supported_dw(int out, int in, bool concat, int kb);
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s);
 
+// A bottom model's whole forward for every 128-row tile in one launch (each layer 128 or 256 wide, 2-4
+// layers, the first layer's input at most 256 wide): Y_l = relu(Y_{l-1} W_l^T + b_l), Y_{-1} = X [M, ldx];
+// W_l [out_l, ldw_l] and every Y_l [M, ldy_l] bf16, biases fp32.  The activations stay in shared memory
+// between layers; every Y_l is also written out.  The header ops are those of the last layer's output.
+struct TcChain {
+    int L, M, K0;
+    const void* X; long long ldx;
+    const void* W[4]; long long ldw[4];
+    int out[4];
+    const float* bias[4];
+    void* Y[4]; long long ldy[4];
+    int* err;
+    HeaderOps hdr;
+};
+bool tc_chain_supported(int L, int K0, const int* out);
+cudaError_t launch_tc_chain(const TcChain& c, cudaStream_t s);
+
 }  // namespace vfl
