@@ -290,7 +290,7 @@ def peaks():
 # event class -> the kernel function that runs it (the launch list and the ncu captures are per function)
 KERNEL_OF_CLASS = {
     "gemm_tc_fwd": "tc_gemm_kernel", "gemm_tc_dx": "tc_gemm_kernel", "gemm_tc_dw": "tc_dw_kernel",
-    "gemm_tc_dw_sgd": "tc_dw_kernel", "gemm_simt_fwd": "gemm_simt_kernel", "gemm_simt_dx": "gemm_simt_kernel",
+    "gemm_tc_dw_sgd": "tc_dw_kernel", "gemm_tc_chain": "tc_chain_kernel", "gemm_simt_fwd": "gemm_simt_kernel", "gemm_simt_dx": "gemm_simt_kernel",
     "gemm_simt_dw": "gemm_simt_kernel", "head_loss": "head_kernel", "loss": "loss_kernel",
     "dp_clip_noise": "dp_kernel", "relu_mask": "relu_mask_kernel", "sgd": "sgd_kernel",
     "channel_header": "write_header_kernel", "cast": "cast_rows_kernel",

@@ -503,7 +503,7 @@ vfl_status vfl_exchange_bytes(const vfl_ctx* ctx, int64_t* emb, int64_t* grad);
  * graph has run returns VFL_E_STATE.  Such a graph should not be replayed
  * after the fold (its events go back to the context's pool).
  */
-#define VFL_KERNEL_CLASSES 19
+#define VFL_KERNEL_CLASSES 20
 vfl_status vfl_profile(vfl_ctx* ctx, int32_t enable);
 vfl_status vfl_profile_get(const vfl_ctx* ctx, int32_t cls, int64_t* launches, double* ms, double* flops,
                            double* bytes);

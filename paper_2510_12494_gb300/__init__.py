@@ -29,7 +29,7 @@ def TAP_ACT(party: int, layer: int) -> int:
     """Tap code of the output of Linear+ReLU layer `layer` of `party` (0 passive, 1 active, 2 top hidden)."""
     return 16 + 16 * party + layer
 PASSIVE, ACTIVE, TOP = 0, 1, 2
-KERNEL_CLASSES = 19
+KERNEL_CLASSES = 20
 
 STATUS_NAMES = {0: "VFL_OK", 1: "VFL_E_INVAL", 2: "VFL_E_OOM", 3: "VFL_E_CUDA", 4: "VFL_E_STATE",
                 5: "VFL_E_VERSION", 6: "VFL_E_TIMEOUT"}

@@ -50,13 +50,13 @@ thread_local std::string g_global_err;
 enum KClass : int {
     K_SIMT_FWD, K_SIMT_DX, K_SIMT_DW, K_TC_FWD, K_TC_DX, K_TC_DW,
     K_LOSS, K_DP, K_MASK, K_SGD, K_HEADER, K_CAST,
-    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_FUSED_UPDATE, K_HEAD, K_PS_AVG, K_TC_DW_SGD, K_NCLASS
+    K_FUSED_PFWD, K_FUSED_ACTIVE, K_FUSED_PBWD, K_FUSED_UPDATE, K_HEAD, K_PS_AVG, K_TC_DW_SGD, K_TC_CHAIN, K_NCLASS
 };
 const char* const kClassNames[K_NCLASS] = {
     "gemm_simt_fwd", "gemm_simt_dx", "gemm_simt_dw", "gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw",
     "loss", "dp_clip_noise", "relu_mask", "sgd", "channel_header", "cast",
     "fused_passive_fwd", "fused_active_step", "fused_passive_bwd", "fused_update", "head_loss",
-    "ps_average", "gemm_tc_dw_sgd"};
+    "ps_average", "gemm_tc_dw_sgd", "gemm_tc_chain"};
 
 struct ProfRec {
     int cls;
@@ -1312,7 +1312,7 @@ vfl_status chain_forward(vfl_ctx* ctx, const std::vector<Layer>& Ls, int vslot, 
     }
     t.err = ctx->status;
     if (hdr) t.hdr = *hdr;
-    PLAUNCH(K_TC_FWD, flops, bytes, s, launch_tc_chain(t, s));
+    PLAUNCH(K_TC_CHAIN, flops, bytes, s, launch_tc_chain(t, s));
     *done = true;
     return VFL_OK;
 }
