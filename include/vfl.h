@@ -246,6 +246,20 @@ vfl_status vfl_bind_host_data_bf16(vfl_ctx* ctx, const uint16_t* x_passive, cons
                                    const int32_t* y, float* loss_out, int64_t loss_cap, void* io_stream);
 
 /*
+ * The same binding for binary features (every feature 0 or 1, as in a party's indicator columns of the
+ * partitioned dataset of Sec. 3; no counterpart in the paper), held bit-packed on the host:
+ * x_passive [n_rows, ceil(d_p / 32)] and x_active [n_rows, ceil(d_a / 32)] uint32 words, feature c of a
+ * row in bit (c mod 32) of the row's word c / 32 (bits past d in a row's last word are ignored);
+ * y [n_rows] int32.  Each step's staging kernel reads its rows' words and writes the values 1 / 0 into
+ * the staging slot in the context's dtype (bf16 or fp32): 1/16 of the host-link bytes of bf16 rows, and
+ * exact, so the steps are bit-identical to a binding of the same features as fp32 or bf16 rows.
+ * Everything else (page-locked arrays, io_stream, labels, loss_out, graphs) is as for
+ * vfl_bind_host_data; x_passive = null unbinds.
+ */
+vfl_status vfl_bind_host_data_bits(vfl_ctx* ctx, const uint32_t* x_passive, const uint32_t* x_active,
+                                   const int32_t* y, float* loss_out, int64_t loss_cap, void* io_stream);
+
+/*
  * The parameters theta_2 (f_p) and theta_1 (f_a and g) of Sec. 3 that Eq. 2 updates.
  * Set / read the fp32 master parameters of one layer: W [out, in], b [out]
  * (host pointers).  vfl_set_params resets every stored weight version of the

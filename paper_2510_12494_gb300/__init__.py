@@ -74,6 +74,8 @@ EXPORTS = {
                                             ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_bind_host_data_bf16": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                                  ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
+    "vfl_bind_host_data_bits": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                                 ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "vfl_set_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
                                         ctypes.c_void_p]),
     "vfl_get_params": (ctypes.c_int32, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
@@ -315,6 +317,19 @@ def weight_grad_noalloc(dpre, x, dW, db, dtype: int, stream=None):
                                          ctypes.c_void_p(db.data_ptr()), ctypes.c_void_p(s.cuda_stream)))
 
 
+def pack_bits(x: np.ndarray) -> np.ndarray:
+    """Binary features [n, d] (every value 0 or 1) as the [n, ceil(d / 32)] int32 words
+    vfl_bind_host_data_bits reads: feature c of a row in bit c mod 32 of word c // 32."""
+    x = np.asarray(x)
+    if not ((x == 0) | (x == 1)).all():
+        raise ValueError("pack_bits: features must be 0 or 1")
+    n, d = x.shape
+    w = (d + 31) // 32
+    b = np.zeros((n, 4 * w), np.uint8)
+    b[:, : (d + 7) // 8] = np.packbits(x.astype(np.uint8, copy=False), axis=1, bitorder="little")
+    return b.view("<u4").view(np.int32).reshape(n, w)
+
+
 def workspace_bytes(p, n_rows: int) -> int:
     cfg = make_config(p)
     out = ctypes.c_uint64()
@@ -394,6 +409,25 @@ class Context:
         self._call(fn, ctypes.c_void_p(xp.data_ptr()), ctypes.c_void_p(xa.data_ptr()),
                    ctypes.c_void_p(y.data_ptr()), lp, cap, ctypes.c_void_p(self._io_stream.cuda_stream))
         self._host_data = (xp, xa, y, loss_out)
+
+    def bind_host_bits(self, xp_bits, xa_bits, y, loss_out=None):
+        """bind_host_data for binary features held bit-packed (vfl_bind_host_data_bits): pinned int32
+        tensors [n_rows, ceil(d_p / 32)] / [n_rows, ceil(d_a / 32)] of 32-bit words (pack_bits), the
+        labels and the loss ring as in bind_host_data.  bind_host_data(None, None, None) unbinds."""
+        import torch
+        assert tuple(xp_bits.shape) == (self.n_rows, (self.p.d_passive + 31) // 32)
+        assert tuple(xa_bits.shape) == (self.n_rows, (self.p.d_active + 31) // 32)
+        assert tuple(y.shape) == (self.n_rows,)
+        assert xp_bits.dtype == xa_bits.dtype == torch.int32 and y.dtype == torch.int32
+        assert xp_bits.is_contiguous() and xa_bits.is_contiguous() and y.is_contiguous()
+        if not hasattr(self, "_io_stream"):
+            self._io_stream = torch.cuda.Stream()
+        lp = ctypes.c_void_p(loss_out.data_ptr()) if loss_out is not None else None
+        cap = len(loss_out) if loss_out is not None else 0
+        self._call(lib().vfl_bind_host_data_bits, ctypes.c_void_p(xp_bits.data_ptr()),
+                   ctypes.c_void_p(xa_bits.data_ptr()), ctypes.c_void_p(y.data_ptr()), lp, cap,
+                   ctypes.c_void_p(self._io_stream.cuda_stream))
+        self._host_data = (xp_bits, xa_bits, y, loss_out)
 
     def set_params(self, params: dict):
         for (party, l), (W, b) in params.items():

@@ -12,8 +12,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libvfl.so")
-SOURCES = ["vfl_runtime.cu", "kernels_simt.cu", "kernels_tc.cu", "kernels_fused.cu", "noalloc.cu", "planner.cu",
-           "peaks.cu"]
+SOURCES = ["vfl_runtime.cu", "kernels_simt.cu", "kernels_tc.cu", "kernels_fused.cu", "kernels_io.cu", "noalloc.cu",
+           "planner.cu", "peaks.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -177,6 +177,11 @@ cudaError_t launch_stage_rows(const float* hxp, int dp, const float* hxa, int da
 // The same for bf16 host rows into a bf16 context (no rounding: a 16-byte copy of eight elements per thread).
 cudaError_t launch_stage_rows_b16(const uint16_t* hxp, int dp, const uint16_t* hxa, int da, const int* hy, int rows,
                                   void* xp, long long ld_p, void* xa, long long ld_a, int* y, cudaStream_t s);
+// The same for bit-packed binary host rows (ceil(d / 32) words a row, feature c in bit c mod 32 of word c / 32)
+// into bf16 (bf16 != 0) or fp32 slot rows of 0 / 1 values.
+cudaError_t launch_stage_rows_bits(const uint32_t* hxp, int dp, const uint32_t* hxa, int da, const int* hy, int rows,
+                                   void* xp, long long ld_p, void* xa, long long ld_a, int* y, int bf16,
+                                   cudaStream_t s);
 // Sets the message vfl_last_error(NULL) returns on this thread.
 void set_global_error(const char* msg);
 

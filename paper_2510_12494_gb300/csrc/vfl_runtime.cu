@@ -178,7 +178,8 @@ struct vfl_ctx {
     const void* hv_xp = nullptr;                // the same views, any feature dtype
     const void* hv_xa = nullptr;
     const int32_t* h_y = nullptr;
-    int h_esz = 4;                              // element bytes of the bound features (4 fp32, 2 bf16)
+    int h_esz = 4;                              // element bytes of the bound features (4 fp32, 2 bf16,
+                                                // 0 bit-packed words)
     float* h_loss = nullptr;
     long long h_loss_cap = 0;
     int io_R = 0;
@@ -1183,7 +1184,16 @@ vfl_status stage_step(vfl_ctx* ctx, long long k) {
         TRY(wait_ev(ctx, s, ctx->ev_pver[(prev + 1) % kEvPool]));
         TRY(wait_ev(ctx, s, ctx->ev_aver[(prev + 1) % kEvPool]));
     }
-    if (ctx->h_esz == 2) {
+    if (ctx->h_esz == 0) {
+        // bit-packed binary rows: ceil(d / 32) words a row over the host link, expanded to 0 / 1 on the device
+        const uint32_t* hp = static_cast<const uint32_t*>(ctx->hv_xp);
+        const uint32_t* ha = static_cast<const uint32_t*>(ctx->hv_xa);
+        const long long wp = (c.d_passive + 31) / 32, wa = (c.d_active + 31) / 32;
+        PLAUNCH(K_CAST, 0, (double)rows * (wp + wa + 2) * 4 + (double)rows * (ctx->ldxp + ctx->ldxa) * ctx->esz, s,
+                launch_stage_rows_bits(hp + r0 * wp, c.d_passive, ha + r0 * wa, c.d_active, ctx->h_y + r0, rows,
+                                       ctx->io_xp[slot], ctx->ldxp, ctx->io_xa[slot], ctx->ldxa, ctx->io_y[slot],
+                                       ctx->bf16, s));
+    } else if (ctx->h_esz == 2) {
         // bf16 rows into the bf16 slot: half the bytes over the host link
         const uint16_t* hp = static_cast<const uint16_t*>(ctx->hv_xp);
         const uint16_t* ha = static_cast<const uint16_t*>(ctx->hv_xa);
@@ -1967,6 +1977,11 @@ vfl_status vfl_bind_host_data_bf16(vfl_ctx* ctx, const uint16_t* xp, const uint1
     if (!ctx) return VFL_E_INVAL;
     if (xp && !ctx->bf16) return ctx->fail(VFL_E_INVAL, "bf16 host data needs a bf16 context");
     return bind_host_data(ctx, xp, xa, y, loss_out, loss_cap, io_stream, 2);
+}
+
+vfl_status vfl_bind_host_data_bits(vfl_ctx* ctx, const uint32_t* xp_bits, const uint32_t* xa_bits, const int32_t* y,
+                                   float* loss_out, int64_t loss_cap, void* io_stream) {
+    return bind_host_data(ctx, xp_bits, xa_bits, y, loss_out, loss_cap, io_stream, 0);
 }
 
 vfl_status vfl_set_params(vfl_ctx* ctx, int32_t party, int32_t layer, const float* W, const float* b) {

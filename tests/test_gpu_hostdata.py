@@ -179,3 +179,42 @@ def test_bf16_host_data_needs_bf16_context(vfl):
     with pytest.raises(vfl.VflError):
         ctx.bind_host_data(pins[0].to(torch.bfloat16).pin_memory(), pins[1].to(torch.bfloat16).pin_memory(), pins[2])
     ctx.close()
+
+
+def bits_context(vfl, q, xp, xa, y, params, cap):
+    """A context bound to bit-packed copies of binary features (vfl_bind_host_data_bits)."""
+    import torch
+    ctx = vfl.Context(q, q.n_rows)
+    ctx.set_params(params)
+    pins = [torch.from_numpy(a).pin_memory() for a in (vfl.pack_bits(xp), vfl.pack_bits(xa), y)]
+    loss = torch.full((cap,), float("nan"), dtype=torch.float32).pin_memory()
+    ctx.bind_host_bits(*pins, loss_out=loss)
+    return ctx, loss
+
+
+@pytest.mark.parametrize("cid,workers,binarize", [(4, 0, False), (4, 3, False), (1, 0, True)])
+def test_bits_host_data_equals_resident(vfl, cid, workers, binarize):
+    """Binary features bit-packed on the host (wide-dp's own Bernoulli columns, d = 1000 = 31 words and a
+    partial one; and the credit-shaped fp32 context on 0 / 1 features, d = 12 / 11 in one partial word):
+    the staging kernel's 0 / 1 values are exact, so training is bit-identical to training on the resident
+    dataset, directly enqueued and replayed from graphs."""
+    p = synth.preset(cid)
+    if workers:
+        p = p.with_(workers=workers)
+    rows = {1: 4096 - 100, 4: 2 * 8192 + 520}[cid]
+    q, xp, xa, y, params = setup(p, rows)
+    if binarize:
+        xp = (xp > 0).astype(np.float32)
+        xa = (xa > 0).astype(np.float32)
+    nb = q.steps_per_epoch
+    n = 2 * nb + 1
+    tp, ta = schedule(q, n)
+    ref = new_context(vfl, q, xp, xa, y, params)
+    ref.train_steps(0, n, tp, ta)
+    ctx, loss = bits_context(vfl, q, xp, xa, y, params, cap=n)
+    ctx.train_steps(0, nb, tp, ta)
+    ctx.launch_graph(ctx.capture(nb, n - nb, tp, ta))
+    ctx.synchronize()
+    np.testing.assert_array_equal(ctx.read_losses(0, n), ref.read_losses(0, n))
+    np.testing.assert_array_equal(loss.numpy(), ref.read_losses(0, n))
+    assert_same_state(ctx, ref)
