@@ -216,8 +216,11 @@ vfl_status vfl_load_data(vfl_ctx* ctx, const float* x_passive, const float* x_ac
  * counterpart for the staging).  After this call every step k reads its own rows
  * [r0, r1) of x_passive [n_rows, d_p] fp32, x_active [n_rows, d_a] fp32 and
  * y [n_rows] int32 straight from host memory into a device staging ring of
- * S + workers + 2 slots (part of the workspace), with one kernel on io_stream,
- * and its phases read the rows there; the kernel that computes the step's mean
+ * S + workers + 2 slots (part of the workspace), with one kernel on io_stream
+ * (or, when the arrays are page-locked and already in the slots' layout -- the
+ * context's dtype, d_p and d_a multiples of 8 -- with three copies by the copy
+ * engines, which leave the SMs to the steps' kernels), and its phases read the
+ * rows there; the kernel that computes the step's mean
  * loss also writes it to loss_out[k mod loss_cap] (skipped when loss_out is
  * null).  A step's rows are read once the step that last used its slot has
  * finished both updates.  The arrays must be page-locked (cudaHostAlloc,

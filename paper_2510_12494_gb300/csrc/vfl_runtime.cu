@@ -180,6 +180,12 @@ struct vfl_ctx {
     const int32_t* h_y = nullptr;
     int h_esz = 4;                              // element bytes of the bound features (4 fp32, 2 bf16,
                                                 // 0 bit-packed words)
+    // page-locked host rows already in the slot layout (the compute dtype, no padding columns): staged by
+    // the copy engines from these host addresses instead of by a kernel
+    bool h_copy = false;
+    const char* hc_xp = nullptr;
+    const char* hc_xa = nullptr;
+    const int32_t* hc_y = nullptr;
     float* h_loss = nullptr;
     long long h_loss_cap = 0;
     int io_R = 0;
@@ -1184,7 +1190,14 @@ vfl_status stage_step(vfl_ctx* ctx, long long k) {
         TRY(wait_ev(ctx, s, ctx->ev_pver[(prev + 1) % kEvPool]));
         TRY(wait_ev(ctx, s, ctx->ev_aver[(prev + 1) % kEvPool]));
     }
-    if (ctx->h_esz == 0) {
+    if (ctx->h_copy) {
+        // rows already in the slot layout: three contiguous copies by the copy engines, which leave the
+        // SMs to the steps' kernels
+        const size_t bp = (size_t)c.d_passive * ctx->esz, ba = (size_t)c.d_active * ctx->esz;
+        CK(cudaMemcpyAsync(ctx->io_xp[slot], ctx->hc_xp + r0 * bp, rows * bp, cudaMemcpyHostToDevice, s));
+        CK(cudaMemcpyAsync(ctx->io_xa[slot], ctx->hc_xa + r0 * ba, rows * ba, cudaMemcpyHostToDevice, s));
+        CK(cudaMemcpyAsync(ctx->io_y[slot], ctx->hc_y + r0, rows * sizeof(int32_t), cudaMemcpyHostToDevice, s));
+    } else if (ctx->h_esz == 0) {
         // bit-packed binary rows: ceil(d / 32) words a row over the host link, expanded to 0 / 1 on the device
         const uint32_t* hp = static_cast<const uint32_t*>(ctx->hv_xp);
         const uint32_t* ha = static_cast<const uint32_t*>(ctx->hv_xa);
@@ -1931,6 +1944,9 @@ vfl_status bind_host_data(vfl_ctx* ctx, const void* xp, const void* xa, const in
     if (!xp) {
         TRY(sync_all(ctx));
         ctx->hio = false;
+        ctx->h_copy = false;
+        ctx->hc_xp = ctx->hc_xa = nullptr;
+        ctx->hc_y = nullptr;
         ctx->h_xp = ctx->h_xa = nullptr;
         ctx->h_y = nullptr;
         ctx->hv_xp = ctx->hv_xa = nullptr;
@@ -1960,6 +1976,19 @@ vfl_status bind_host_data(vfl_ctx* ctx, const void* xp, const void* xa, const in
     ctx->hv_xp = dxp;
     ctx->hv_xa = dxa;
     ctx->h_esz = esz;
+    // the copy engines stage the rows when the host holds them page-locked in the slots' own layout
+    auto pinned = [](const void* q) {
+        cudaPointerAttributes at;
+        const bool ok = cudaPointerGetAttributes(&at, q) == cudaSuccess && at.type == cudaMemoryTypeHost;
+        cudaGetLastError();
+        return ok;
+    };
+    const char* no_copy = std::getenv("VFL_DISABLE_COPY_STAGING");
+    ctx->h_copy = esz == ctx->esz && ctx->ldxp == ctx->cfg.d_passive && ctx->ldxa == ctx->cfg.d_active &&
+                  pinned(xp) && pinned(xa) && pinned(y) && !(no_copy && *no_copy && *no_copy != '0');
+    ctx->hc_xp = static_cast<const char*>(xp);
+    ctx->hc_xa = static_cast<const char*>(xa);
+    ctx->hc_y = y;
     ctx->h_loss = static_cast<float*>(const_cast<void*>(dl));
     ctx->h_loss_cap = loss_out ? loss_cap : 0;
     ctx->io = static_cast<cudaStream_t>(io_stream);
