@@ -312,6 +312,7 @@ vfl_status vfl_set_cursor(vfl_ctx* ctx, int64_t k);
 vfl_status vfl_set_version(vfl_ctx* ctx, int32_t party, int32_t layer, int64_t v, const float* W, const float* b);
 
 /*
+ * The per-worker replicas of the intra-party parameter server (Sec. 4.1, Eq. 5).
  * Parameter-server mode only (VFL_E_STATE otherwise): the fp32 master of one
  * layer of replica `worker` (0 <= worker < workers), host pointers W [out, in]
  * and b [out].  Both synchronize the context and need no step in flight;
@@ -376,7 +377,8 @@ vfl_status vfl_get_drops(vfl_ctx* ctx, int64_t* n_drops);
 vfl_status vfl_set_drops(vfl_ctx* ctx, int64_t n_drops);
 
 /*
- * Seeded drop draws (host only, pure): drop[k] = 1 when word 0 of
+ * Seeded drop draws for the waiting-deadline / buffer-overflow drops of Sec. 4.1
+ * (host only, pure): drop[k] = 1 when word 0 of
  * Philox4x32-10(key = (seed lo, seed hi), counter = (k lo, k hi, 2, 0x4452)) is
  * below floor(rate * 2^32) (every step when rate == 1).  VFL_E_INVAL unless
  * 0 <= rate <= 1.
