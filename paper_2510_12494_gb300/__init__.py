@@ -352,7 +352,10 @@ class Context:
         _check(L.vfl_create(ctypes.byref(self.cfg), n_rows, ctypes.c_void_p(self.workspace.data_ptr()),
                             nbytes, ctypes.byref(handle)))
         self.h = handle
-        self.streams = streams if streams is not None else [torch.cuda.Stream() for _ in range(2 * p.workers)]
+        # the parties' worker streams one priority level above the I/O stream of the host-data bindings, so
+        # that the SMs go to a step's kernels before the staging of steps further ahead
+        self.streams = streams if streams is not None else [torch.cuda.Stream(priority=-1)
+                                                            for _ in range(2 * p.workers)]
         arr = (ctypes.c_void_p * len(self.streams))(*[s.cuda_stream for s in self.streams])
         self._call(L.vfl_set_streams, len(self.streams), arr)
         self.nb = -(-n_rows // p.batch)
