@@ -558,7 +558,10 @@ def run_ours(args):
         # the host keeps the features compactly (untimed, once): bit-packed when every feature is 0 or 1
         # (vfl_bind_host_data_bits: 1/16 of bf16's bytes, exact), else in the compute dtype (bf16 presets:
         # rounded exactly as the resident load rounds them); each step's staging kernel reads its rows
-        binary = bool(((xp == 0) | (xp == 1)).all() and ((xa == 0) | (xa == 1)).all())
+        def all_binary(a, rows=65536):
+            return all(((c == 0) | (c == 1)).all() for c in (a[i:i + rows] for i in range(0, len(a), rows)))
+
+        binary = all_binary(xp) and all_binary(xa)
         host_bf16 = p.dtype == "bf16" and not binary
         pin_y = torch.from_numpy(y).pin_memory()
         loss_host = torch.full((n_e2e,), float("nan"), dtype=torch.float32).pin_memory()
