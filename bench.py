@@ -297,7 +297,8 @@ KERNEL_OF_CLASS = {
     "fused_passive_fwd": "fused_passive_fwd_kernel", "fused_active_step": "fused_active_kernel",
     "fused_passive_bwd": "fused_passive_bwd_kernel", "fused_update": "fused_update_kernel",
     "ps_average": "ps_average_kernel"}
-KERNEL_SOURCE = {"tc_": "kernels_tc.cu", "fused_": "kernels_fused.cu"}   # everything else: kernels_simt.cu
+KERNEL_SOURCE = {"tc_": "kernels_tc.cu", "fused_": "kernels_fused.cu",
+                 "stage_rows_bits": "kernels_io.cu"}   # everything else: kernels_simt.cu
 
 
 def file_digest(src):
